@@ -1,0 +1,298 @@
+/*
+ * fastcoder.h - C ABI of the GB300 retrieve-and-verify step of FastCoder
+ * (arXiv 2502.17139): suffix-array draft retrieval from one or two token
+ * datastores, weighted draft-tree construction, tree-masked verification
+ * attention and greedy acceptance, plus the cache append that closes a
+ * decoding step.
+ *
+ * Conventions for every call
+ *   - Every pointer named d_* is DEVICE memory owned by the caller; the
+ *     library never allocates, frees or retains it beyond the call.  Plain
+ *     (non d_) pointers are host memory read during the call only.
+ *   - Calls are asynchronous on the given stream (fc_stream = cudaStream_t;
+ *     NULL is the legacy default stream) unless stated otherwise.  FC_OK
+ *     means "arguments valid and work enqueued".  Errors that only the GPU
+ *     can see (a token id >= vocab, a cache overflow, a bounded wait that ran
+ *     out) are recorded in a device error word that fc_get_error() reads.
+ *   - A host-detected error returns before anything is enqueued and leaves
+ *     every output untouched.
+ *   - Token ids are uint32 < vocab.  FC_PAD_TOKEN pads draft slots.
+ *   - bf16 tensors are raw IEEE bfloat16 (2 bytes, little endian).
+ *   - Outputs do not depend on the launch configuration (bit-exact
+ *     determinism for integer outputs).
+ */
+#ifndef FASTCODER_H_
+#define FASTCODER_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  FC_OK = 0,
+  FC_ERR_INVALID_ARG = 1,  /* bad pointer, size, layout or value */
+  FC_ERR_UNSUPPORTED = 2,  /* valid in principle, outside what the kernels support */
+  FC_ERR_WORKSPACE = 3,    /* workspace pointer missing or smaller than required */
+  FC_ERR_CAPACITY = 4,     /* a cache, context or path would overflow its capacity */
+  FC_ERR_TIMEOUT = 5,      /* a bounded device-side wait ran out; the kernel returned */
+  FC_ERR_CUDA = 6,         /* a CUDA runtime/driver call failed */
+  FC_ERR_INTERNAL = 7      /* an internal consistency check failed */
+} fc_status;
+
+typedef void* fc_stream; /* cudaStream_t */
+
+#define FC_PAD_TOKEN 0xFFFFFFFFu
+#define FC_MAX_NMAX 32        /* longest suffix length tried */
+#define FC_MAX_TOPK 256       /* drafts kept per query and source */
+#define FC_MAX_DRAFT_LEN 16   /* tokens per draft */
+#define FC_MAX_OCC 4096       /* occurrences examined per query and source */
+#define FC_MAX_SOURCES 4      /* datastores searched in one call */
+#define FC_MAX_NODES 128      /* draft-tree nodes (root included) */
+
+/* Human-readable name of a status code (static storage). */
+const char* fc_status_string(fc_status s);
+
+/* Library version, e.g. "0.1.0". */
+const char* fc_version(void);
+
+/*
+ * Waits for the stream, then returns and clears the device error word
+ * (the most severe device-detected error since the last call, or FC_OK).
+ * Synchronous.
+ */
+fc_status fc_get_error(fc_stream s);
+
+/* ------------------------------------------------------------------------
+ * Datastore (Section IV-A, Eq. 1-2; Section III-A).  Every position of a
+ * token corpus splits it into a context (the tokens before) and a
+ * continuation (the tokens after); the suffix array over the corpus turns
+ * "which contexts end with this suffix" into one contiguous SA range.
+ * ------------------------------------------------------------------------ */
+typedef struct {
+  const uint32_t* tokens;  /* device, [n_tokens] token ids < vocab */
+  const uint32_t* sa;      /* device, [n_tokens] suffix array of tokens */
+  const uint32_t* bucket;  /* device, [vocab + 1]: bucket[v] = first SA index whose
+                              suffix starts with a token >= v; bucket[vocab] = n_tokens */
+  uint64_t n_tokens;       /* 1 <= n_tokens < 2^32 - 1 */
+  uint32_t vocab;          /* 1 <= vocab < 2^31 */
+} fc_datastore;
+
+/* Workspace bytes fc_datastore_build needs for n_tokens tokens. */
+size_t fc_datastore_build_workspace(uint64_t n_tokens, uint32_t vocab);
+
+/*
+ * Builds the suffix array and first-token bucket table of a token corpus
+ * (the datastore organisation of Section IV-A, after REST).
+ *   d_tokens [n_tokens] uint32 ids < vocab (checked; FC_ERR_INVALID_ARG if not)
+ *   d_sa     [n_tokens] uint32 out: sa[j] = start of the j-th smallest suffix;
+ *            a suffix that is a proper prefix of another sorts first
+ *   d_bucket [vocab + 1] uint32 out (see fc_datastore.bucket)
+ *   d_ws     workspace of at least fc_datastore_build_workspace() bytes
+ *   out      host struct filled with the datastore view (may be NULL)
+ * Synchronous: returns when the build is finished (it reads a group count
+ * back after every doubling round).
+ */
+fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t vocab,
+                             uint32_t* d_sa, uint32_t* d_bucket, void* d_ws, size_t ws_bytes,
+                             fc_stream s, fc_datastore* out);
+
+/* ------------------------------------------------------------------------
+ * Retrieval (Section III-A; Section IV-C, Algorithm 1 par_search; Section
+ * V-C: n_max = 16).
+ * ------------------------------------------------------------------------ */
+typedef struct {
+  int32_t n_max;       /* longest suffix length tried, 1..FC_MAX_NMAX */
+  int32_t n_min;       /* shortest suffix length tried, 1..n_max */
+  int32_t top_k;       /* drafts kept, 1..FC_MAX_TOPK */
+  int32_t draft_len;   /* tokens per draft, 1..FC_MAX_DRAFT_LEN */
+  uint32_t max_occ;    /* occurrences examined, 1..FC_MAX_OCC */
+} fc_retrieve_params;
+
+/*
+ * For every query b and every source s: the longest n in
+ * [n_min, min(n_max, ctx_len[b])] whose last-n-token context suffix occurs
+ * in the corpus immediately before a position p <= n_tokens - 1 (so a
+ * continuation exists); the first max_occ occurrences in suffix-array order
+ * (the lexicographically smallest windows); their continuations
+ * T[p .. min(p + draft_len, n_tokens)) grouped by equality (length
+ * included); and the top_k groups by count descending, then token ids
+ * ascending (a prefix before its extensions).
+ *
+ *   sources     host array [n_sources] of datastore views (1..FC_MAX_SOURCES)
+ *   d_ctx       [batch][ctx_stride] uint32 contexts; query b is
+ *               d_ctx[b][0 .. ctx_len[b]) (ctx_len[b] in [0, ctx_stride])
+ *   d_skip      optional [batch] int32: nonzero leaves query b's outputs
+ *               untouched (they were served by a retrieval cache); may be NULL
+ * Outputs (source-major, [n_sources][batch]...):
+ *   d_drafts    [S][batch][top_k][draft_len] uint32, FC_PAD_TOKEN past a
+ *               draft's end and in absent slots
+ *   d_draft_len [S][batch][top_k] int32 (0 in absent slots)
+ *   d_count     [S][batch][top_k] uint32 occurrence counts (0 in absent slots)
+ *   d_n_drafts  [S][batch] int32 number of drafts found (<= top_k)
+ *   d_match_len [S][batch] int32 the matched suffix length n (0: no match)
+ * A context token >= vocab makes that query match nothing and records
+ * FC_ERR_INVALID_ARG in the device error word.
+ */
+fc_status fc_retrieve(const fc_datastore* sources, int n_sources, const uint32_t* d_ctx,
+                      int ctx_stride, const int32_t* d_ctx_len, int batch, const int32_t* d_skip,
+                      fc_retrieve_params p, uint32_t* d_drafts, int32_t* d_draft_len,
+                      uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len, fc_stream s);
+
+/* ------------------------------------------------------------------------
+ * Context-keyed retrieval cache (workload support for the step loop;
+ * Section IV-B motivates caching retrieval results, this cache replays a
+ * query's earlier result when its last n_max context tokens repeat).
+ * The table lives in caller-owned device memory.
+ * ------------------------------------------------------------------------ */
+size_t fc_rcache_bytes(int capacity, int n_sources, fc_retrieve_params p);
+
+/* Clears a table of `capacity` entries (a power of two, 1..2^24). */
+fc_status fc_rcache_init(void* d_table, size_t bytes, int capacity, int n_sources,
+                         fc_retrieve_params p, fc_stream s);
+
+/*
+ * For each query b with d_want_hit[b] != 0 whose key (its last
+ * min(n_max, ctx_len[b]) tokens) is in the table, copies the stored
+ * retrieval outputs into the output arrays (same layout as fc_retrieve) and
+ * sets d_skip[b] = 1; otherwise sets d_skip[b] = 0.  d_want_hit may be NULL
+ * (every query may hit).
+ */
+fc_status fc_rcache_lookup(const void* d_table, int capacity, int n_sources, fc_retrieve_params p,
+                           const uint32_t* d_ctx, int ctx_stride, const int32_t* d_ctx_len,
+                           int batch, const int32_t* d_want_hit, int32_t* d_skip,
+                           uint32_t* d_drafts, int32_t* d_draft_len, uint32_t* d_count,
+                           int32_t* d_n_drafts, int32_t* d_match_len, fc_stream s);
+
+/*
+ * Stores the retrieval outputs of every query with d_skip[b] == 0 under its
+ * key (replacing an equal key).  A full table records FC_ERR_CAPACITY.
+ */
+fc_status fc_rcache_insert(void* d_table, int capacity, int n_sources, fc_retrieve_params p,
+                           const uint32_t* d_ctx, int ctx_stride, const int32_t* d_ctx_len,
+                           int batch, const int32_t* d_skip, const uint32_t* d_drafts,
+                           const int32_t* d_draft_len, const uint32_t* d_count,
+                           const int32_t* d_n_drafts, const int32_t* d_match_len, fc_stream s);
+
+/* ------------------------------------------------------------------------
+ * Draft tree (Section IV-D: Eq. 3 node weight alpha*t_r + beta*t_c, the
+ * top-weighted trie nodes as the draft; Eq. 4 tree mask; position ids by
+ * depth; Section V-C: alpha = beta = 1, at most 64 draft tokens).
+ * ------------------------------------------------------------------------ */
+/*
+ * Merges the drafts of n_sources sources (the fc_retrieve output layout)
+ * into one trie per query rooted at d_root_tok[b] (the last context token,
+ * whose K/V is not yet cached).  A draft u weighs
+ * w(u) = sum_s src_weight[s] * count_s(u); a node weighs the sum of w over
+ * the drafts through it.  The root and the node_budget - 1 heaviest other
+ * nodes (ties: shallower first, then smaller token path) are kept and
+ * emitted in depth-first preorder with children in ascending token order.
+ *   src_weight  host [n_sources] uint32 (alpha, beta), each <= 65535
+ *   node_budget 1..n_pad, n_pad in {64, 128}
+ * Outputs, [batch][n_pad] unless noted; rows >= n_nodes[b] are padding
+ * (tok = FC_PAD_TOKEN, parent = depth = pos = -1, mask = 0):
+ *   d_tok, d_parent (parent[0] = -1, parent[i] < i), d_depth (root 0),
+ *   d_pos (= kv_len[b] + depth), d_mask [batch][n_pad][n_pad/64] uint64 with
+ *   bit j of row i set iff node j is an ancestor of node i or i itself,
+ *   d_n_nodes [batch].
+ * Limits: n_sources * top_k <= 512, draft_len <= FC_MAX_DRAFT_LEN.
+ */
+fc_status fc_build_tree(int n_sources, const uint32_t* d_drafts, const int32_t* d_draft_len,
+                        const uint32_t* d_count, const int32_t* d_n_drafts,
+                        const uint32_t* src_weight, int top_k, int draft_len,
+                        const uint32_t* d_root_tok, const int32_t* d_kv_len, int batch,
+                        int node_budget, int n_pad, uint32_t* d_tok, int32_t* d_parent,
+                        int32_t* d_depth, int32_t* d_pos, uint64_t* d_mask, int32_t* d_n_nodes,
+                        fc_stream s);
+
+/*
+ * Eq. 4 mask, depths and position ids of trees given by parent pointers in
+ * the layout above (parent[0] = -1, 0 <= parent[i] < i for 0 < i < n_nodes).
+ * A malformed parent records FC_ERR_INVALID_ARG and zeroes that tree's mask.
+ */
+fc_status fc_tree_mask(const int32_t* d_parent, const int32_t* d_n_nodes, const int32_t* d_kv_len,
+                       int batch, int n_pad, int32_t* d_depth, int32_t* d_pos, uint64_t* d_mask,
+                       fc_stream s);
+
+/* ------------------------------------------------------------------------
+ * Verification attention (Section IV-D, Eq. 4): every tree node attends to
+ * the whole KV cache and to its tree ancestors (and itself), one forward for
+ * all drafts.
+ * ------------------------------------------------------------------------ */
+/*
+ * out[b][i][h] = sum_j softmax_j(scale * q[b][i][h] . k_j) v_j over the keys
+ * j = every cached key of kv head g = h / (H / Hkv) at positions
+ * [0, kv_len[b]) and every tree key j with bit j of mask[b][i] set.
+ * Rows i >= n_nodes[b] are written as zeros.  Q and K arrive already
+ * position-encoded (the caller applies the depth-based position ids).
+ *   d_q       bf16 [batch][n_pad][H][D]
+ *   d_k_cache, d_v_cache  bf16 [batch][Hkv][kv_cap][D]
+ *   d_kv_len  [batch] int32, 0 <= kv_len <= kv_cap (checked on the device)
+ *   d_k_tree, d_v_tree    bf16 [batch][Hkv][n_pad][D] (the tree tokens' K/V)
+ *   d_mask    [batch][n_pad][n_pad/64] uint64 (fc_build_tree layout)
+ *   d_n_nodes [batch] int32 in [1, n_pad]
+ *   d_out     bf16 [batch][n_pad][H][D]
+ * Supported: D = 128, n_pad in {64, 128}, H % Hkv == 0, H / Hkv <= 16,
+ * all device pointers 16-byte aligned.  Arithmetic: bf16 tensor-core
+ * products with fp32 accumulation and an fp32 online softmax.
+ */
+fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const void* d_v_cache, int kv_cap,
+                       const int32_t* d_kv_len, const void* d_k_tree, const void* d_v_tree,
+                       const uint64_t* d_mask, const int32_t* d_n_nodes, int batch, int n_pad,
+                       int H, int Hkv, int D, float scale, void* d_out, fc_stream s);
+
+/* ------------------------------------------------------------------------
+ * Acceptance (Section IV-D: every correct token from the start is accepted,
+ * everything after the first error rejected; Eq. 7 counts tokens per step).
+ * ------------------------------------------------------------------------ */
+/*
+ * Walks each tree from the root: at node cur, if some child carries the
+ * target model's prediction d_argmax[b][cur], move to it; otherwise stop.
+ *   d_acc_len [batch] int32 draft tokens accepted
+ *   d_path    [batch][path_cap] int32 node ids path[0] = 0 .. path[acc_len],
+ *             -1 after
+ *   d_bonus   [batch] uint32 the prediction at the last accepted node
+ * A path longer than path_cap records FC_ERR_CAPACITY (it is cut there).
+ */
+fc_status fc_accept(const uint32_t* d_tok, const int32_t* d_parent, const int32_t* d_n_nodes,
+                    const uint32_t* d_argmax, int batch, int n_pad, int32_t* d_acc_len,
+                    int32_t* d_path, int path_cap, uint32_t* d_bonus, fc_stream s);
+
+/*
+ * Closes a decoding step: copies the K/V rows of the accepted path (root
+ * included) to cache rows kv_len_in[b] .. kv_len_in[b] + acc_len[b],
+ * writes kv_len_out = kv_len_in + acc_len + 1, appends the accepted draft
+ * tokens and the bonus token to the context (ctx_len_out likewise) and
+ * writes the bonus token to d_root_out (the next step's root).
+ * In and out length arrays must not alias.  An overflow of kv_cap or
+ * ctx_stride records FC_ERR_CAPACITY and leaves that sequence unchanged
+ * (its out lengths equal its in lengths).
+ */
+fc_status fc_kv_append(const int32_t* d_path, const int32_t* d_acc_len, const uint32_t* d_bonus,
+                       const uint32_t* d_tok, const void* d_k_tree, const void* d_v_tree,
+                       int batch, int n_pad, int Hkv, int D, int path_cap, void* d_k_cache,
+                       void* d_v_cache, int kv_cap, const int32_t* d_kv_len_in,
+                       int32_t* d_kv_len_out, uint32_t* d_ctx, int ctx_stride,
+                       const int32_t* d_ctx_len_in, int32_t* d_ctx_len_out,
+                       uint32_t* d_root_out, fc_stream s);
+
+/* ------------------------------------------------------------------------
+ * Synthetic target model (workload scaffolding, not part of the method;
+ * the paper's target model is an LLM whose greedy predictions drive
+ * acceptance).  Along the tree's first branch the model agrees with the
+ * tree for d_plen[b] steps; every other prediction is d_rtok[b][i] moved up
+ * by one (mod vocab) while it equals the token of a child of node i, at most
+ * n_pad times (if the children cover the whole vocabulary the last candidate
+ * stands).
+ * ------------------------------------------------------------------------ */
+fc_status fc_synth_argmax(const uint32_t* d_tok, const int32_t* d_parent, const int32_t* d_n_nodes,
+                          int batch, int n_pad, const int32_t* d_plen, const uint32_t* d_rtok,
+                          uint32_t vocab, uint32_t* d_argmax, fc_stream s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FASTCODER_H_ */

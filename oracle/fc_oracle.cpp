@@ -558,7 +558,9 @@ int orc_kv_append(const int32_t* path, const int32_t* acc_len, const uint32_t* b
 // Along the tree's first branch (root, its first child, that node's first
 // child, ...) the model agrees with the tree for the first plen[b] steps;
 // every other prediction is the node's random token rtok[b][i], moved up by
-// one (mod vocab) while it equals a token of one of the node's children.
+// one (mod vocab) while it equals a token of one of the node's children, at
+// most n_pad times (when the children cover the whole vocabulary the last
+// candidate stands).
 // ---------------------------------------------------------------------------
 int orc_synth_argmax(const uint32_t* tok, const int32_t* parent, const int32_t* n_nodes, int B,
                      int n_pad, const int32_t* plen, const uint32_t* rtok, uint32_t vocab,
@@ -583,7 +585,7 @@ int orc_synth_argmax(const uint32_t* tok, const int32_t* parent, const int32_t* 
         continue;
       }
       uint32_t x = rtok[base + i] % vocab;
-      for (;;) {
+      for (int tries = 0; tries < n_pad; ++tries) {
         bool clash = false;
         for (int j = 1; j < n; ++j)
           if (parent[base + j] == i && tok[base + j] == x) clash = true;

@@ -1,0 +1,387 @@
+// fc_build_tree / fc_tree_mask: draft-tree construction (Section IV-D: trie
+// over the retrieved drafts, node weight alpha*t_r + beta*t_c of Eq. 3, the
+// top-weighted nodes as the draft tree; the tree mask of Eq. 4; position ids
+// by depth; Section V-C: alpha = beta = 1, at most 64 draft tokens).
+//
+// One CTA per query, everything in shared memory, no pointer trie:
+//   1. gather the drafts of all sources with weight w = src_weight * count;
+//   2. sort them lexicographically (rank by counting) and merge duplicates
+//      across sources (weights add);
+//   3. with neighbour LCPs, every trie node is a pair (u, l): the prefix of
+//      length l of sorted unique draft u, new at u when l > lcp(u-1, u).
+//      Its weight is the weight sum of the contiguous run of drafts that
+//      share that prefix (prefix sums over the sorted drafts);
+//   4. a bitonic sort of (W, 31 - l, 8191 - u) keys selects the heaviest
+//      budget - 1 nodes (ties: shallower, then smaller path);
+//   5. sorting the kept nodes by (u, l) is depth-first preorder with
+//      children in ascending token order; parents come from the LCPs;
+//      masks are ancestor walks.
+#include <algorithm>
+
+#include "fc_common.cuh"
+
+FC_DEFINE_ERROR_WORD(tree)
+
+namespace {
+
+constexpr int BT_THREADS = 256;
+constexpr int BT_MAX_DRAFTS = 512;
+
+struct TreeIn {
+  const uint32_t* drafts;
+  const int32_t* draft_len;
+  const uint32_t* count;
+  const int32_t* n_drafts;
+  uint32_t w[FC_MAX_SOURCES];
+};
+struct TreeOut {
+  uint32_t* tok;
+  int32_t* parent;
+  int32_t* depth;
+  int32_t* pos;
+  uint64_t* mask;
+  int32_t* n_nodes;
+};
+
+__host__ __device__ inline uint32_t next_pow2(uint32_t x) {
+  uint32_t p = 1;
+  while (p < x) p <<= 1;
+  return p;
+}
+
+struct BtLayout {
+  size_t tok, len, w, order, uniq, wu, ps, lcp, coff, flag, ckey, total;
+};
+
+__host__ __device__ inline BtLayout bt_layout(int M, int d) {
+  BtLayout L;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = (off + bytes + 15) & ~(size_t)15;
+    return o;
+  };
+  L.tok = take((size_t)M * d * 4);
+  L.len = take((size_t)M * 4);
+  L.w = take((size_t)M * 8);
+  L.order = take((size_t)M * 4);
+  L.uniq = take((size_t)M * 4);
+  L.wu = take((size_t)M * 8);
+  L.ps = take((size_t)(M + 1) * 8);
+  L.lcp = take((size_t)(M + 1) * 4);
+  L.coff = take((size_t)(M + 1) * 4);
+  L.flag = take((size_t)(M + 1) * 4);
+  L.ckey = take((size_t)next_pow2((uint32_t)(M * d)) * 8);
+  L.total = off;
+  return L;
+}
+
+// Exclusive scan of a[0..n) in place (n <= 8192); returns the total.
+__device__ uint32_t block_scan_array(uint32_t* a, int n, uint32_t* wsum) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int chunk = (n + BT_THREADS - 1) / BT_THREADS;
+  const int lo = min(n, tid * chunk), hi = min(n, lo + chunk);
+  uint32_t s = 0;
+  for (int i = lo; i < hi; ++i) s += a[i];
+  uint32_t inc = s;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    uint32_t y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+    if (lane >= o) inc += y;
+  }
+  if (lane == 31) wsum[warp] = inc;
+  __syncthreads();
+  if (tid == 0) {
+    uint32_t run = 0;
+    for (int w = 0; w < BT_THREADS / 32; ++w) {
+      uint32_t c = wsum[w];
+      wsum[w] = run;
+      run += c;
+    }
+    wsum[BT_THREADS / 32] = run;
+  }
+  __syncthreads();
+  uint32_t pre = wsum[warp] + inc - s;
+  for (int i = lo; i < hi; ++i) {
+    uint32_t v = a[i];
+    a[i] = pre;
+    pre += v;
+  }
+  uint32_t total = wsum[BT_THREADS / 32];
+  __syncthreads();
+  return total;
+}
+
+// -1 / 0 / 1 lexicographic comparison of two drafts (a prefix sorts first).
+__device__ __forceinline__ int cmp_draft(const uint32_t* a, int la, const uint32_t* b, int lb) {
+  int l = min(la, lb);
+  for (int i = 0; i < l; ++i)
+    if (a[i] != b[i]) return a[i] < b[i] ? -1 : 1;
+  return la < lb ? -1 : (la > lb ? 1 : 0);
+}
+
+__global__ void __launch_bounds__(BT_THREADS) k_build_tree(TreeIn in, int S, int B, int k, int d,
+                                                           const uint32_t* __restrict__ root_tok,
+                                                           const int32_t* __restrict__ kv_len, int budget, int n_pad,
+                                                           TreeOut out) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ uint32_t wsum[BT_THREADS / 32 + 1];
+  __shared__ int32_t sel_u[FC_MAX_NODES], sel_l[FC_MAX_NODES], par_s[FC_MAX_NODES];
+  const int M0 = S * k;
+  const BtLayout L = bt_layout(M0, d);
+  uint32_t* tok = reinterpret_cast<uint32_t*>(smem_raw + L.tok);
+  int32_t* len = reinterpret_cast<int32_t*>(smem_raw + L.len);
+  uint64_t* w = reinterpret_cast<uint64_t*>(smem_raw + L.w);
+  uint32_t* order = reinterpret_cast<uint32_t*>(smem_raw + L.order);
+  uint32_t* uniq = reinterpret_cast<uint32_t*>(smem_raw + L.uniq);
+  uint64_t* wu = reinterpret_cast<uint64_t*>(smem_raw + L.wu);
+  uint64_t* ps = reinterpret_cast<uint64_t*>(smem_raw + L.ps);
+  uint32_t* lcp = reinterpret_cast<uint32_t*>(smem_raw + L.lcp);
+  uint32_t* coff = reinterpret_cast<uint32_t*>(smem_raw + L.coff);
+  uint32_t* flag = reinterpret_cast<uint32_t*>(smem_raw + L.flag);
+  uint64_t* ckey = reinterpret_cast<uint64_t*>(smem_raw + L.ckey);
+  const int b = blockIdx.x, tid = threadIdx.x;
+
+  // 1. valid drafts, compacted in (source, slot) order
+  for (int i = tid; i < M0; i += BT_THREADS) {
+    int s = i / k, t = i - s * k;
+    size_t sb = (size_t)s * B + b;
+    int nd = min(max((int)in.n_drafts[sb], 0), k);
+    int l = (t < nd) ? in.draft_len[sb * k + t] : 0;
+    flag[i] = (l > 0 && l <= d) ? 1u : 0u;
+  }
+  __syncthreads();
+  // keep the flags: scan a copy in coff
+  for (int i = tid; i < M0; i += BT_THREADS) coff[i] = flag[i];
+  __syncthreads();
+  uint32_t M = block_scan_array(coff, M0, wsum);
+  for (int i = tid; i < M0; i += BT_THREADS) {
+    if (!flag[i]) continue;
+    int s = i / k, t = i - s * k;
+    size_t sb = (size_t)s * B + b;
+    uint32_t j = coff[i];
+    int l = in.draft_len[sb * k + t];
+    len[j] = l;
+    uint32_t cnt = in.count[sb * k + t];
+    if (cnt > (1u << 20)) {  // weights are packed into 46-bit sort keys
+      fc_flag(&g_fc_err, FC_EBIT_INVALID);
+      cnt = 1u << 20;
+    }
+    w[j] = (uint64_t)in.w[s] * cnt;
+    for (int x = 0; x < d; ++x) tok[j * d + x] = (x < l) ? in.drafts[(sb * k + t) * d + x] : 0u;
+  }
+  __syncthreads();
+
+  // 2. sort by counting rank; equal drafts keep (source, slot) order
+  for (uint32_t i = tid; i < M; i += BT_THREADS) {
+    uint32_t r = 0;
+    const uint32_t* a = tok + i * d;
+    for (uint32_t j = 0; j < M; ++j) {
+      int c = cmp_draft(tok + j * d, len[j], a, len[i]);
+      r += (c < 0 || (c == 0 && j < i)) ? 1u : 0u;
+    }
+    order[r] = i;
+  }
+  __syncthreads();
+  for (uint32_t r = tid; r < M; r += BT_THREADS) {
+    uint32_t i = order[r];
+    flag[r] = (r == 0 || cmp_draft(tok + order[r - 1] * d, len[order[r - 1]], tok + i * d, len[i]) != 0) ? 1u : 0u;
+    coff[r] = flag[r];
+  }
+  __syncthreads();
+  uint32_t U = block_scan_array(coff, (int)M, wsum);  // coff[r] = unique index of run start
+  for (uint32_t u = tid; u < U; u += BT_THREADS) wu[u] = 0;
+  __syncthreads();
+  for (uint32_t r = tid; r < M; r += BT_THREADS) {
+    uint32_t u = coff[r] + flag[r] - 1u;  // unique index of the run containing r
+    if (flag[r]) uniq[u] = order[r];
+    atomicAdd(reinterpret_cast<unsigned long long*>(&wu[u]), (unsigned long long)w[order[r]]);
+  }
+  __syncthreads();
+
+  // 3. neighbour LCPs, prefix sums of weights, candidate counts
+  for (uint32_t u = tid; u < U; u += BT_THREADS) {
+    uint32_t l = 0;
+    if (u > 0) {
+      const uint32_t* a = tok + uniq[u - 1] * d;
+      const uint32_t* c = tok + uniq[u] * d;
+      int lim = min(len[uniq[u - 1]], len[uniq[u]]);
+      while ((int)l < lim && a[l] == c[l]) ++l;
+    }
+    lcp[u] = l;
+    coff[u] = (uint32_t)len[uniq[u]] - l;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    uint64_t run = 0;
+    for (uint32_t u = 0; u < U; ++u) {
+      ps[u] = run;
+      run += wu[u];
+    }
+    ps[U] = run;
+  }
+  uint32_t C = block_scan_array(coff, (int)U, wsum);
+  const uint32_t P2 = next_pow2(max(C, 1u));
+  for (uint32_t u = tid; u < U; u += BT_THREADS) {
+    const int lu = len[uniq[u]];
+    for (int l = (int)lcp[u] + 1; l <= lu; ++l) {
+      uint32_t e = u + 1;
+      while (e < U && (int)lcp[e] >= l) ++e;
+      uint64_t W = ps[e] - ps[u];
+      ckey[coff[u] + (l - lcp[u] - 1)] = (W << 18) | ((uint64_t)(31 - l) << 13) | (uint64_t)(8191u - u);
+    }
+  }
+  for (uint32_t c = C + tid; c < P2; c += BT_THREADS) ckey[c] = 0;
+  __syncthreads();
+
+  // 4. bitonic sort, descending
+  for (uint32_t size = 2; size <= P2; size <<= 1) {
+    for (uint32_t st = size >> 1; st > 0; st >>= 1) {
+      for (uint32_t i = tid; i < P2; i += BT_THREADS) {
+        uint32_t j = i ^ st;
+        if (j > i) {
+          uint64_t a = ckey[i], c = ckey[j];
+          bool desc = (i & size) == 0;
+          if (desc ? (a < c) : (a > c)) {
+            ckey[i] = c;
+            ckey[j] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+
+  // 5. kept nodes in preorder = ascending (u, l)
+  const int nsel = (int)umin((uint32_t)(budget - 1), C);
+  for (int i = tid; i < nsel; i += BT_THREADS) {
+    uint64_t key = ckey[i];
+    int u = 8191 - (int)(key & 8191u), l = 31 - (int)((key >> 13) & 31u);
+    int r = 0;
+    for (int j = 0; j < nsel; ++j) {
+      uint64_t kj = ckey[j];
+      int uj = 8191 - (int)(kj & 8191u), lj = 31 - (int)((kj >> 13) & 31u);
+      r += (uj < u || (uj == u && lj < l)) ? 1 : 0;
+    }
+    sel_u[1 + r] = u;
+    sel_l[1 + r] = l;
+  }
+  __syncthreads();
+  const int n = 1 + nsel;
+  for (int i = 1 + tid; i < n; i += BT_THREADS) {
+    int u = sel_u[i], l = sel_l[i];
+    int pidx = 0;
+    if (l > 1) {
+      int up = u;
+      while (up > 0 && (int)lcp[up] >= l - 1) --up;
+      for (int j = 1; j < i; ++j)
+        if (sel_u[j] == up && sel_l[j] == l - 1) pidx = j;
+    }
+    par_s[i] = pidx;
+  }
+  if (tid == 0) par_s[0] = -1;
+  __syncthreads();
+  const int nw = n_pad / 64;
+  const size_t base = (size_t)b * n_pad;
+  const int kvl = kv_len[b];
+  for (int i = tid; i < n_pad; i += BT_THREADS) {
+    uint32_t tk = FC_PAD_TOKEN;
+    int pa = -1, de = -1, po = -1;
+    uint64_t m0 = 0, m1 = 0;
+    if (i < n) {
+      tk = (i == 0) ? root_tok[b] : tok[uniq[sel_u[i]] * d + sel_l[i] - 1];
+      de = (i == 0) ? 0 : sel_l[i];
+      pa = par_s[i];
+      po = kvl + de;
+      for (int a = i; a >= 0; a = par_s[a]) {
+        if (a < 64) m0 |= 1ull << a;
+        else m1 |= 1ull << (a - 64);
+      }
+    }
+    out.tok[base + i] = tk;
+    out.parent[base + i] = pa;
+    out.depth[base + i] = de;
+    out.pos[base + i] = po;
+    out.mask[(base + i) * nw] = m0;
+    if (nw > 1) out.mask[(base + i) * nw + 1] = m1;
+  }
+  if (tid == 0) out.n_nodes[b] = n;
+}
+
+// Mask, depth, position ids from parent pointers: one warp per tree.
+__global__ void k_tree_mask(const int32_t* __restrict__ parent, const int32_t* __restrict__ n_nodes,
+                            const int32_t* __restrict__ kv_len, int B, int n_pad, int32_t* __restrict__ depth,
+                            int32_t* __restrict__ pos, uint64_t* __restrict__ mask) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (warp >= B) return;
+  const int b = warp, nw = n_pad / 64;
+  const size_t base = (size_t)b * n_pad;
+  const int n = n_nodes[b];
+  bool bad = (n < 1 || n > n_pad);
+  for (int i = lane; i < n_pad && !bad; i += 32)
+    if (i < n && i > 0 && (parent[base + i] < 0 || parent[base + i] >= i)) bad = true;
+  bad = __any_sync(0xFFFFFFFFu, bad);
+  if (bad && lane == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+  for (int i = lane; i < n_pad; i += 32) {
+    uint64_t m0 = 0, m1 = 0;
+    int de = -1, po = -1;
+    if (!bad && i < n) {
+      de = 0;
+      for (int a = i; a >= 0; a = (a == 0) ? -1 : parent[base + a]) {
+        if (a < 64) m0 |= 1ull << a;
+        else m1 |= 1ull << (a - 64);
+        if (a != i) ++de;
+      }
+      po = kv_len[b] + de;
+    }
+    depth[base + i] = de;
+    pos[base + i] = po;
+    mask[(base + i) * nw] = m0;
+    if (nw > 1) mask[(base + i) * nw + 1] = m1;
+  }
+}
+
+}  // namespace
+
+extern "C" fc_status fc_build_tree(int n_sources, const uint32_t* d_drafts, const int32_t* d_draft_len,
+                                   const uint32_t* d_count, const int32_t* d_n_drafts, const uint32_t* src_weight,
+                                   int top_k, int draft_len, const uint32_t* d_root_tok, const int32_t* d_kv_len,
+                                   int batch, int node_budget, int n_pad, uint32_t* d_tok, int32_t* d_parent,
+                                   int32_t* d_depth, int32_t* d_pos, uint64_t* d_mask, int32_t* d_n_nodes,
+                                   fc_stream stream) {
+  if (n_sources < 1 || n_sources > FC_MAX_SOURCES || top_k < 1 || draft_len < 1 || batch < 0 || !src_weight)
+    return FC_ERR_INVALID_ARG;
+  if (n_pad != 64 && n_pad != 128) return FC_ERR_UNSUPPORTED;
+  if (node_budget < 1 || node_budget > n_pad) return FC_ERR_INVALID_ARG;
+  if (n_sources * top_k > BT_MAX_DRAFTS || draft_len > FC_MAX_DRAFT_LEN || top_k > FC_MAX_TOPK)
+    return FC_ERR_UNSUPPORTED;
+  for (int s = 0; s < n_sources; ++s)
+    if (src_weight[s] > 65535u) return FC_ERR_UNSUPPORTED;
+  if (batch == 0) return FC_OK;
+  if (!d_drafts || !d_draft_len || !d_count || !d_n_drafts || !d_root_tok || !d_kv_len || !d_tok || !d_parent ||
+      !d_depth || !d_pos || !d_mask || !d_n_nodes)
+    return FC_ERR_INVALID_ARG;
+  TreeIn in{d_drafts, d_draft_len, d_count, d_n_drafts, {0, 0, 0, 0}};
+  for (int s = 0; s < n_sources; ++s) in.w[s] = src_weight[s];
+  TreeOut out{d_tok, d_parent, d_depth, d_pos, d_mask, d_n_nodes};
+  const size_t smem = bt_layout(n_sources * top_k, draft_len).total;
+  if (cudaFuncSetAttribute(k_build_tree, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+    return FC_ERR_CUDA;
+  k_build_tree<<<batch, BT_THREADS, smem, static_cast<cudaStream_t>(stream)>>>(
+      in, n_sources, batch, top_k, draft_len, d_root_tok, d_kv_len, node_budget, n_pad, out);
+  return FC_CHECK_LAUNCH();
+}
+
+extern "C" fc_status fc_tree_mask(const int32_t* d_parent, const int32_t* d_n_nodes, const int32_t* d_kv_len,
+                                  int batch, int n_pad, int32_t* d_depth, int32_t* d_pos, uint64_t* d_mask,
+                                  fc_stream stream) {
+  if (batch < 0) return FC_ERR_INVALID_ARG;
+  if (n_pad != 64 && n_pad != 128) return FC_ERR_UNSUPPORTED;
+  if (batch == 0) return FC_OK;
+  if (!d_parent || !d_n_nodes || !d_kv_len || !d_depth || !d_pos || !d_mask) return FC_ERR_INVALID_ARG;
+  const int threads = 128;
+  const unsigned blocks = (unsigned)((batch * 32 + threads - 1) / threads);
+  k_tree_mask<<<blocks, threads, 0, static_cast<cudaStream_t>(stream)>>>(d_parent, d_n_nodes, d_kv_len, batch, n_pad,
+                                                                         d_depth, d_pos, d_mask);
+  return FC_CHECK_LAUNCH();
+}

@@ -1,0 +1,505 @@
+// fc_retrieve: batched suffix-match draft retrieval (Section III-A; Section
+// IV-C, Algorithm 1 par_search over D_r and D_c; Section V-C n_max = 16),
+// and the context-keyed replay cache used by the step loop.
+//
+// One CTA per (query, source).  Design:
+//   * search: every (suffix length n, lower/upper bound) pair gets its own
+//     thread, so all lengths n_max..n_min are binary-searched at once and
+//     the longest non-empty range is picked afterwards (a match of length n
+//     implies matches of every shorter length, so the longest non-empty
+//     range is the answer).  The first-token bucket table narrows each search
+//     to the suffixes that start with the pattern's first token.
+//   * the suffix that is exactly the pattern at the corpus end (no
+//     continuation) is the smallest suffix of its range when present; it is
+//     dropped.
+//   * counting: in SA order the occurrences' continuations are sorted, so
+//     equal continuations are adjacent; runs are found with one compare per
+//     neighbour pair and a block scan (no hash table needed).
+//   * top-k: a bitonic sort in shared memory of (count << 12 | 4095 - run)
+//     keys gives count descending, then run order (= token order) ascending.
+#include <algorithm>
+
+#include "fc_common.cuh"
+
+FC_DEFINE_ERROR_WORD(ret)
+
+namespace {
+
+constexpr int RT_THREADS = 256;
+constexpr int RT_ITEMS = FC_MAX_OCC / RT_THREADS;  // 16
+
+struct DsView {
+  const uint32_t* T;
+  const uint32_t* sa;
+  const uint32_t* bucket;
+  uint64_t n;
+  uint32_t vocab;
+};
+struct DsArgs {
+  DsView ds[FC_MAX_SOURCES];
+};
+
+struct RetOut {
+  uint32_t* drafts;
+  int32_t* draft_len;
+  uint32_t* count;
+  int32_t* n_drafts;
+  int32_t* match_len;
+};
+
+// Compare the first n tokens of suffix T[i..N) with pat[0..n), knowing the
+// first tokens are equal.  -1: suffix smaller (or ends first), 0: equal, 1: larger.
+__device__ __forceinline__ int cmp_suffix(const uint32_t* __restrict__ T, uint64_t N, uint64_t i,
+                                          const uint32_t* pat, int n) {
+  for (int k = 1; k < n; ++k) {
+    if (i + k >= N) return -1;
+    uint32_t a = __ldg(T + i + k), b = pat[k];
+    if (a != b) return a < b ? -1 : 1;
+  }
+  return 0;
+}
+
+__device__ __forceinline__ bool cont_equal(const uint32_t* __restrict__ T, uint64_t N, uint32_t p1, uint32_t p2,
+                                           int d) {
+  uint64_t l1 = min((uint64_t)d, N - p1), l2 = min((uint64_t)d, N - p2);
+  if (l1 != l2) return false;
+  for (uint64_t k = 0; k < l1; ++k)
+    if (__ldg(T + p1 + k) != __ldg(T + p2 + k)) return false;
+  return true;
+}
+
+__device__ __forceinline__ uint32_t block_scan_256(uint32_t x, uint32_t* total, uint32_t* wsum) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t inc = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    uint32_t y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+    if (lane >= o) inc += y;
+  }
+  if (lane == 31) wsum[warp] = inc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t run = 0;
+    for (int w = 0; w < RT_THREADS / 32; ++w) {
+      uint32_t c = wsum[w];
+      wsum[w] = run;
+      run += c;
+    }
+    *total = run;
+  }
+  __syncthreads();
+  uint32_t r = wsum[warp] + inc - x;
+  __syncthreads();
+  return r;
+}
+
+struct RetSmem {
+  uint32_t pos[FC_MAX_OCC];
+  uint32_t runs[FC_MAX_OCC + 1];
+  uint32_t keys[FC_MAX_OCC];
+  uint32_t ctx[FC_MAX_NMAX];
+  uint32_t lo[FC_MAX_NMAX + 1];
+  uint32_t hi[FC_MAX_NMAX + 1];
+  uint32_t wsum[RT_THREADS / 32];
+  uint32_t n_star, first, cnt, n_runs, bad;
+};
+
+__global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint32_t* __restrict__ ctx, int stride,
+                                                         const int32_t* __restrict__ ctx_len, int B,
+                                                         const int32_t* __restrict__ skip, fc_retrieve_params p,
+                                                         RetOut o) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  RetSmem& sm = *reinterpret_cast<RetSmem*>(smem_raw);
+  const int b = blockIdx.x, s = blockIdx.y, tid = threadIdx.x;
+  if (skip && skip[b]) return;
+  const DsView ds = args.ds[s];
+  const uint32_t* __restrict__ T = ds.T;
+  const uint64_t N = ds.n;
+  const int k = p.top_k, d = p.draft_len;
+  const size_t sb = (size_t)s * B + b;
+
+  int m = ctx_len[b];
+  m = max(0, min(m, stride));
+  const int cap = min(p.n_max, m);
+  if (tid == 0) sm.bad = 0;
+  __syncthreads();
+  if (tid < cap) {
+    uint32_t t = ctx[(size_t)b * stride + (m - cap) + tid];
+    sm.ctx[tid] = t;
+    if (t >= ds.vocab) sm.bad = 1;
+  }
+  __syncthreads();
+  if (sm.bad && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+
+  // ---- search: one thread per (n, bound) -------------------------------
+  const int npairs = (cap >= p.n_min && !sm.bad) ? 2 * (cap - p.n_min + 1) : 0;
+  if (tid < npairs) {
+    const int n = cap - (tid >> 1);
+    const bool upper = tid & 1;
+    const uint32_t* pat = sm.ctx + (cap - n);
+    const uint32_t t0 = pat[0];
+    uint32_t lo = __ldg(ds.bucket + t0), hi = __ldg(ds.bucket + t0 + 1);
+    while (lo < hi) {
+      uint32_t mid = lo + ((hi - lo) >> 1);
+      int c = cmp_suffix(T, N, __ldg(ds.sa + mid), pat, n);
+      if (upper ? (c <= 0) : (c < 0)) lo = mid + 1;
+      else hi = mid;
+    }
+    if (upper) sm.hi[n] = lo;
+    else sm.lo[n] = lo;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    uint32_t ns = 0, first = 0, cnt = 0;
+    if (npairs) {
+      for (int n = cap; n >= p.n_min; --n) {
+        uint32_t l = sm.lo[n], h = sm.hi[n];
+        if (l < h && (uint64_t)__ldg(ds.sa + l) + n == N) ++l;  // exact pattern at the corpus end
+        if (l < h) {
+          ns = n;
+          first = l;
+          cnt = h - l;
+          break;
+        }
+      }
+    }
+    sm.n_star = ns;
+    sm.first = first;
+    sm.cnt = min(cnt, p.max_occ);
+  }
+  __syncthreads();
+  const int ns = (int)sm.n_star;
+  uint32_t* dr = o.drafts + sb * k * d;
+  int32_t* dl = o.draft_len + sb * k;
+  uint32_t* ct = o.count + sb * k;
+  if (ns == 0) {
+    for (int e = tid; e < k * d; e += RT_THREADS) dr[e] = FC_PAD_TOKEN;
+    for (int e = tid; e < k; e += RT_THREADS) {
+      dl[e] = 0;
+      ct[e] = 0;
+    }
+    if (tid == 0) {
+      o.n_drafts[sb] = 0;
+      o.match_len[sb] = 0;
+    }
+    return;
+  }
+  const uint32_t nocc = sm.cnt, first = sm.first;
+
+  // ---- occurrences -> continuation starts ------------------------------
+  for (uint32_t e = tid; e < nocc; e += RT_THREADS) sm.pos[e] = __ldg(ds.sa + first + e) + (uint32_t)ns;
+  __syncthreads();
+  // run heads: continuation differs from its SA predecessor
+  uint32_t head[RT_ITEMS];
+  uint32_t local = 0;
+#pragma unroll
+  for (int it = 0; it < RT_ITEMS; ++it) {
+    uint32_t e = tid * RT_ITEMS + it;
+    uint32_t h = 0;
+    if (e < nocc) h = (e == 0) || !cont_equal(T, N, sm.pos[e - 1], sm.pos[e], d);
+    head[it] = h;
+    local += h;
+  }
+  uint32_t total;
+  uint32_t run_id = block_scan_256(local, &total, sm.wsum);
+#pragma unroll
+  for (int it = 0; it < RT_ITEMS; ++it) {
+    uint32_t e = tid * RT_ITEMS + it;
+    if (head[it]) sm.runs[run_id] = e;
+    run_id += head[it];
+  }
+  if (tid == 0) {
+    sm.runs[total] = nocc;
+    sm.n_runs = total;
+  }
+  __syncthreads();
+  const uint32_t R = sm.n_runs;
+  uint32_t P2 = 1;
+  while (P2 < R) P2 <<= 1;
+  for (uint32_t r = tid; r < P2; r += RT_THREADS)
+    sm.keys[r] = (r < R) ? (((sm.runs[r + 1] - sm.runs[r]) << 12) | (4095u - r)) : 0u;
+  __syncthreads();
+  for (uint32_t size = 2; size <= P2; size <<= 1) {
+    for (uint32_t stride2 = size >> 1; stride2 > 0; stride2 >>= 1) {
+      for (uint32_t i = tid; i < P2; i += RT_THREADS) {
+        uint32_t j = i ^ stride2;
+        if (j > i) {
+          uint32_t a = sm.keys[i], c = sm.keys[j];
+          bool desc = (i & size) == 0;
+          if (desc ? (a < c) : (a > c)) {
+            sm.keys[i] = c;
+            sm.keys[j] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  // ---- outputs ---------------------------------------------------------
+  const int nd = (int)umin((uint32_t)k, R);
+  for (int e = tid; e < k * d; e += RT_THREADS) {
+    int t = e / d, x = e - t * d;
+    uint32_t v = FC_PAD_TOKEN;
+    if (t < nd) {
+      uint32_t r = 4095u - (sm.keys[t] & 4095u);
+      uint32_t pp = sm.pos[sm.runs[r]];
+      uint64_t len = min((uint64_t)d, N - pp);
+      if ((uint64_t)x < len) v = __ldg(T + pp + x);
+    }
+    dr[e] = v;
+  }
+  for (int t = tid; t < k; t += RT_THREADS) {
+    if (t < nd) {
+      uint32_t r = 4095u - (sm.keys[t] & 4095u);
+      uint32_t pp = sm.pos[sm.runs[r]];
+      dl[t] = (int32_t)min((uint64_t)d, N - pp);
+      ct[t] = sm.keys[t] >> 12;
+    } else {
+      dl[t] = 0;
+      ct[t] = 0;
+    }
+  }
+  if (tid == 0) {
+    o.n_drafts[sb] = nd;
+    o.match_len[sb] = ns;
+  }
+}
+
+bool params_ok(const fc_retrieve_params& p) {
+  return p.n_max >= 1 && p.n_max <= FC_MAX_NMAX && p.n_min >= 1 && p.n_min <= p.n_max && p.top_k >= 1 &&
+         p.top_k <= FC_MAX_TOPK && p.draft_len >= 1 && p.draft_len <= FC_MAX_DRAFT_LEN && p.max_occ >= 1 &&
+         p.max_occ <= FC_MAX_OCC;
+}
+
+// ---------------------------------------------------------------------------
+// Replay cache.  Entry layout (32-bit words): [0] key length or EMPTY /
+// CLAIMED, [1 .. 1+n_max) key tokens, then per source: drafts[k*d],
+// draft_len[k], count[k], n_drafts, match_len.
+// ---------------------------------------------------------------------------
+constexpr uint32_t RC_EMPTY = 0xFFFFFFFFu;
+constexpr uint32_t RC_CLAIMED = 0xFFFFFFFEu;
+
+__host__ __device__ inline size_t rc_src_words(const fc_retrieve_params& p) {
+  return (size_t)p.top_k * p.draft_len + 2 * (size_t)p.top_k + 2;
+}
+__host__ __device__ inline size_t rc_entry_words(int S, const fc_retrieve_params& p) {
+  size_t w = 1 + (size_t)p.n_max + (size_t)S * rc_src_words(p);
+  return (w + 3) & ~(size_t)3;
+}
+
+__device__ uint64_t rc_hash(const uint32_t* key, int len) {
+  uint64_t h = 1469598103934665603ull ^ (uint64_t)len;
+  for (int i = 0; i < len; ++i) {
+    h ^= key[i];
+    h *= 1099511628211ull;
+  }
+  h ^= h >> 29;
+  return h;
+}
+
+__global__ void k_rc_init(uint32_t* table, int capacity, size_t entry_words) {
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < (size_t)capacity;
+       e += (size_t)gridDim.x * blockDim.x)
+    table[e * entry_words] = RC_EMPTY;
+}
+
+struct RcSmem {
+  uint32_t key[FC_MAX_NMAX];
+  int klen;
+  int slot;
+};
+
+__device__ void rc_load_key(RcSmem& sm, const uint32_t* ctx, int stride, const int32_t* ctx_len, int b, int n_max) {
+  int m = max(0, min((int)ctx_len[b], stride));
+  int kl = min(n_max, m);
+  if (threadIdx.x < kl) sm.key[threadIdx.x] = ctx[(size_t)b * stride + (m - kl) + threadIdx.x];
+  if (threadIdx.x == 0) sm.klen = kl;
+  __syncthreads();
+}
+
+__device__ bool rc_key_equal(const uint32_t* entry, const RcSmem& sm) {
+  if (entry[0] != (uint32_t)sm.klen) return false;
+  for (int i = 0; i < sm.klen; ++i)
+    if (entry[1 + i] != sm.key[i]) return false;
+  return true;
+}
+
+__global__ void k_rc_lookup(const uint32_t* __restrict__ table, int capacity, int S, fc_retrieve_params p,
+                            const uint32_t* __restrict__ ctx, int stride, const int32_t* __restrict__ ctx_len,
+                            int B, const int32_t* __restrict__ want, int32_t* __restrict__ skip, RetOut o) {
+  __shared__ RcSmem sm;
+  const int b = blockIdx.x;
+  rc_load_key(sm, ctx, stride, ctx_len, b, p.n_max);
+  const size_t ew = rc_entry_words(S, p);
+  if (threadIdx.x == 0) {
+    int slot = -1;
+    if (!want || want[b]) {
+      uint64_t h = rc_hash(sm.key, sm.klen);
+      for (int probe = 0; probe < capacity; ++probe) {
+        size_t e = (h + probe) & (uint64_t)(capacity - 1);
+        const uint32_t* ent = table + e * ew;
+        uint32_t st = ent[0];
+        if (st == RC_EMPTY) break;
+        if (st != RC_CLAIMED && rc_key_equal(ent, sm)) {
+          slot = (int)e;
+          break;
+        }
+      }
+    }
+    sm.slot = slot;
+    skip[b] = slot >= 0 ? 1 : 0;
+  }
+  __syncthreads();
+  if (sm.slot < 0) return;
+  const uint32_t* src = table + (size_t)sm.slot * ew + 1 + p.n_max;
+  const int k = p.top_k, d = p.draft_len;
+  for (int s = 0; s < S; ++s) {
+    const uint32_t* e = src + s * rc_src_words(p);
+    size_t sb = (size_t)s * B + b;
+    for (int i = threadIdx.x; i < k * d; i += blockDim.x) o.drafts[sb * k * d + i] = e[i];
+    for (int i = threadIdx.x; i < k; i += blockDim.x) {
+      o.draft_len[sb * k + i] = (int32_t)e[k * d + i];
+      o.count[sb * k + i] = e[k * d + k + i];
+    }
+    if (threadIdx.x == 0) {
+      o.n_drafts[sb] = (int32_t)e[k * d + 2 * k];
+      o.match_len[sb] = (int32_t)e[k * d + 2 * k + 1];
+    }
+  }
+}
+
+__global__ void k_rc_insert(uint32_t* table, int capacity, int S, fc_retrieve_params p,
+                            const uint32_t* __restrict__ ctx, int stride, const int32_t* __restrict__ ctx_len, int B,
+                            const int32_t* __restrict__ skip, RetOut o) {
+  __shared__ RcSmem sm;
+  const int b = blockIdx.x;
+  if (skip && skip[b]) return;
+  rc_load_key(sm, ctx, stride, ctx_len, b, p.n_max);
+  const size_t ew = rc_entry_words(S, p);
+  if (threadIdx.x == 0) {
+    int slot = -1;
+    bool present = false;
+    uint64_t h = rc_hash(sm.key, sm.klen);
+    for (int probe = 0; probe < capacity && slot < 0 && !present; ++probe) {
+      size_t e = (h + probe) & (uint64_t)(capacity - 1);
+      uint32_t* ent = table + e * ew;
+      uint32_t st = atomicCAS(ent, RC_EMPTY, RC_CLAIMED);
+      if (st == RC_EMPTY) {
+        slot = (int)e;
+      } else if (st != RC_CLAIMED && rc_key_equal(ent, sm)) {
+        present = true;  // an equal key holds the same (deterministic) result
+      }
+    }
+    if (slot < 0 && !present) fc_flag(&g_fc_err, FC_EBIT_CAPACITY);
+    sm.slot = slot;
+  }
+  __syncthreads();
+  if (sm.slot < 0) return;
+  uint32_t* ent = table + (size_t)sm.slot * ew;
+  for (int i = threadIdx.x; i < sm.klen; i += blockDim.x) ent[1 + i] = sm.key[i];
+  uint32_t* dst = ent + 1 + p.n_max;
+  const int k = p.top_k, d = p.draft_len;
+  for (int s = 0; s < S; ++s) {
+    uint32_t* e = dst + s * rc_src_words(p);
+    size_t sb = (size_t)s * B + b;
+    for (int i = threadIdx.x; i < k * d; i += blockDim.x) e[i] = o.drafts[sb * k * d + i];
+    for (int i = threadIdx.x; i < k; i += blockDim.x) {
+      e[k * d + i] = (uint32_t)o.draft_len[sb * k + i];
+      e[k * d + k + i] = o.count[sb * k + i];
+    }
+    if (threadIdx.x == 0) {
+      e[k * d + 2 * k] = (uint32_t)o.n_drafts[sb];
+      e[k * d + 2 * k + 1] = (uint32_t)o.match_len[sb];
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) atomicExch(ent, (uint32_t)sm.klen);
+}
+
+}  // namespace
+
+extern "C" fc_status fc_retrieve(const fc_datastore* sources, int n_sources, const uint32_t* d_ctx, int ctx_stride,
+                                 const int32_t* d_ctx_len, int batch, const int32_t* d_skip, fc_retrieve_params p,
+                                 uint32_t* d_drafts, int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
+                                 int32_t* d_match_len, fc_stream stream) {
+  if (!sources || n_sources < 1 || n_sources > FC_MAX_SOURCES || batch < 0 || ctx_stride < 1 ||
+      batch > 65535 * 16)
+    return FC_ERR_INVALID_ARG;
+  if (!params_ok(p)) return (p.n_max > 0 && p.top_k > 0 && p.draft_len > 0) ? FC_ERR_UNSUPPORTED : FC_ERR_INVALID_ARG;
+  if (batch == 0) return FC_OK;
+  if (!d_ctx || !d_ctx_len || !d_drafts || !d_draft_len || !d_count || !d_n_drafts || !d_match_len)
+    return FC_ERR_INVALID_ARG;
+  DsArgs a{};
+  for (int s = 0; s < n_sources; ++s) {
+    const fc_datastore& ds = sources[s];
+    if (!ds.tokens || !ds.sa || !ds.bucket || ds.n_tokens == 0 || ds.n_tokens >= 0xFFFFFFFFull || ds.vocab == 0)
+      return FC_ERR_INVALID_ARG;
+    a.ds[s] = DsView{ds.tokens, ds.sa, ds.bucket, ds.n_tokens, ds.vocab};
+  }
+  static bool attr_done = false;
+  if (!attr_done) {
+    if (cudaFuncSetAttribute(k_retrieve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(RetSmem)) !=
+        cudaSuccess)
+      return FC_ERR_CUDA;
+    attr_done = true;
+  }
+  RetOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len};
+  dim3 grid((unsigned)batch, (unsigned)n_sources);
+  k_retrieve<<<grid, RT_THREADS, sizeof(RetSmem), static_cast<cudaStream_t>(stream)>>>(
+      a, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, o);
+  return FC_CHECK_LAUNCH();
+}
+
+extern "C" size_t fc_rcache_bytes(int capacity, int n_sources, fc_retrieve_params p) {
+  if (capacity < 1 || n_sources < 1 || n_sources > FC_MAX_SOURCES || !params_ok(p)) return 0;
+  return (size_t)capacity * rc_entry_words(n_sources, p) * 4;
+}
+
+static bool rc_args_ok(int capacity, int n_sources, const fc_retrieve_params& p) {
+  return capacity >= 1 && capacity <= (1 << 24) && (capacity & (capacity - 1)) == 0 && n_sources >= 1 &&
+         n_sources <= FC_MAX_SOURCES && params_ok(p);
+}
+
+extern "C" fc_status fc_rcache_init(void* d_table, size_t bytes, int capacity, int n_sources, fc_retrieve_params p,
+                                    fc_stream stream) {
+  if (!d_table || !rc_args_ok(capacity, n_sources, p)) return FC_ERR_INVALID_ARG;
+  if (bytes < fc_rcache_bytes(capacity, n_sources, p)) return FC_ERR_WORKSPACE;
+  unsigned g = (unsigned)std::min<size_t>((capacity + 255) / 256, 4096);
+  k_rc_init<<<g, 256, 0, static_cast<cudaStream_t>(stream)>>>(static_cast<uint32_t*>(d_table), capacity,
+                                                              rc_entry_words(n_sources, p));
+  return FC_CHECK_LAUNCH();
+}
+
+extern "C" fc_status fc_rcache_lookup(const void* d_table, int capacity, int n_sources, fc_retrieve_params p,
+                                      const uint32_t* d_ctx, int ctx_stride, const int32_t* d_ctx_len, int batch,
+                                      const int32_t* d_want_hit, int32_t* d_skip, uint32_t* d_drafts,
+                                      int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
+                                      int32_t* d_match_len, fc_stream stream) {
+  if (!d_table || !rc_args_ok(capacity, n_sources, p) || batch < 0 || ctx_stride < 1) return FC_ERR_INVALID_ARG;
+  if (batch == 0) return FC_OK;
+  if (!d_ctx || !d_ctx_len || !d_skip || !d_drafts || !d_draft_len || !d_count || !d_n_drafts || !d_match_len)
+    return FC_ERR_INVALID_ARG;
+  RetOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len};
+  k_rc_lookup<<<batch, 128, 0, static_cast<cudaStream_t>(stream)>>>(static_cast<const uint32_t*>(d_table), capacity,
+                                                                     n_sources, p, d_ctx, ctx_stride, d_ctx_len, batch,
+                                                                     d_want_hit, d_skip, o);
+  return FC_CHECK_LAUNCH();
+}
+
+extern "C" fc_status fc_rcache_insert(void* d_table, int capacity, int n_sources, fc_retrieve_params p,
+                                      const uint32_t* d_ctx, int ctx_stride, const int32_t* d_ctx_len, int batch,
+                                      const int32_t* d_skip, const uint32_t* d_drafts, const int32_t* d_draft_len,
+                                      const uint32_t* d_count, const int32_t* d_n_drafts, const int32_t* d_match_len,
+                                      fc_stream stream) {
+  if (!d_table || !rc_args_ok(capacity, n_sources, p) || batch < 0 || ctx_stride < 1) return FC_ERR_INVALID_ARG;
+  if (batch == 0) return FC_OK;
+  if (!d_ctx || !d_ctx_len || !d_drafts || !d_draft_len || !d_count || !d_n_drafts || !d_match_len)
+    return FC_ERR_INVALID_ARG;
+  RetOut o{const_cast<uint32_t*>(d_drafts), const_cast<int32_t*>(d_draft_len), const_cast<uint32_t*>(d_count),
+           const_cast<int32_t*>(d_n_drafts), const_cast<int32_t*>(d_match_len)};
+  k_rc_insert<<<batch, 128, 0, static_cast<cudaStream_t>(stream)>>>(static_cast<uint32_t*>(d_table), capacity,
+                                                                     n_sources, p, d_ctx, ctx_stride, d_ctx_len, batch,
+                                                                     d_skip, o);
+  return FC_CHECK_LAUNCH();
+}

@@ -1,0 +1,372 @@
+// fc_datastore_build: suffix array + first-token bucket table of a uint32
+// token corpus (the datastore organisation of Section IV-A, Eq. 1-2, which
+// follows REST's suffix-array index).
+//
+// Method (GPU prefix doubling): after round r every position i carries the
+// dense rank of its first 2^r tokens.  A round sorts the positions by the
+// pair (rank[i], rank[i + h] + 1) (0 when i + h runs past the end, so a
+// shorter suffix sorts first), with a stable LSD radix sort written here
+// (8-bit digits, per-block histograms, a global exclusive scan and a stable
+// scatter that ranks equal digits inside a warp with __match_any_sync), then
+// re-ranks by scanning "key differs from its predecessor" flags.  The loop
+// stops when every rank is distinct.  All passes stream the arrays once
+// (HBM-bound); only the rank gather rank[i + h] is random.
+#include "fc_common.cuh"
+
+FC_DEFINE_ERROR_WORD(sa)
+
+namespace {
+
+constexpr int RS_THREADS = 256;
+constexpr int RS_ITEMS = 16;
+constexpr int RS_TILE = RS_THREADS * RS_ITEMS;  // 4096 keys per block
+constexpr int RS_WARPS = RS_THREADS / 32;
+constexpr int RS_WARP_CHUNK = 32 * RS_ITEMS;    // 512 consecutive keys per warp
+
+constexpr int SCAN_THREADS = 1024;
+constexpr int SCAN_ITEMS = 4;
+constexpr int SCAN_TILE = SCAN_THREADS * SCAN_ITEMS;
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+inline size_t cdiv(size_t a, size_t b) { return (a + b - 1) / b; }
+
+struct Layout {
+  size_t key_a, key_b, val_b, rank, head, hist, scan_tmp, ctl, total;
+  size_t nb;          // radix blocks
+  size_t scan_len;    // longest array the scan sees
+};
+
+size_t scan_tmp_elems(size_t len) {
+  size_t t = 0;
+  while (len > (size_t)SCAN_TILE) {
+    len = cdiv(len, SCAN_TILE);
+    t += len;
+  }
+  return t + 16;
+}
+
+Layout layout_for(uint64_t n) {
+  Layout L;
+  L.nb = cdiv(n, RS_TILE);
+  L.scan_len = n > 256 * L.nb ? n : 256 * L.nb;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  L.key_a = take(n * 8);
+  L.key_b = take(n * 8);
+  L.val_b = take(n * 4);
+  L.rank = take(n * 4);
+  L.head = take(n * 4);
+  L.hist = take(256 * L.nb * 4);
+  L.scan_tmp = take(scan_tmp_elems(L.scan_len) * 4);
+  L.ctl = take(64);
+  L.total = off;
+  return L;
+}
+
+__global__ void k_check_tokens(const uint32_t* __restrict__ T, uint64_t n, uint32_t vocab, uint32_t* ctl) {
+  for (uint64_t i = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; i < n; i += (uint64_t)gridDim.x * blockDim.x)
+    if (T[i] >= vocab) {
+      atomicOr(ctl, 1u);
+      return;
+    }
+}
+
+// First round: key = (T[i], T[i+1] + 1 or 0), val = i.
+__global__ void k_keys_first(const uint32_t* __restrict__ T, uint64_t n, uint64_t* __restrict__ key,
+                             uint32_t* __restrict__ val) {
+  for (uint64_t i = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; i < n; i += (uint64_t)gridDim.x * blockDim.x) {
+    uint64_t lo = (i + 1 < n) ? (uint64_t)T[i + 1] + 1 : 0;
+    key[i] = ((uint64_t)T[i] << 32) | lo;
+    val[i] = (uint32_t)i;
+  }
+}
+
+// Later rounds: positions in current SA order; key = (rank[i], rank[i+h] + 1 or 0).
+// val may alias sa (each element rewrites its own value).
+__global__ void k_keys_round(const uint32_t* sa, const uint32_t* __restrict__ rank, uint64_t n, uint64_t h,
+                             uint64_t* __restrict__ key, uint32_t* val) {
+  for (uint64_t j = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; j < n; j += (uint64_t)gridDim.x * blockDim.x) {
+    uint32_t i = sa[j];
+    uint64_t lo = ((uint64_t)i + h < n) ? (uint64_t)rank[i + h] + 1 : 0;
+    key[j] = ((uint64_t)rank[i] << 32) | lo;
+    val[j] = i;
+  }
+}
+
+__global__ void __launch_bounds__(RS_THREADS) k_radix_hist(const uint64_t* __restrict__ key, uint64_t n, int shift,
+                                                           uint32_t* __restrict__ hist, uint64_t nb) {
+  __shared__ uint32_t h[256];
+  h[threadIdx.x] = 0;
+  __syncthreads();
+  uint64_t base = blockIdx.x * (uint64_t)RS_TILE;
+#pragma unroll 4
+  for (int k = 0; k < RS_ITEMS; ++k) {
+    uint64_t idx = base + (uint64_t)k * RS_THREADS + threadIdx.x;
+    if (idx < n) atomicAdd(&h[(uint32_t)(key[idx] >> shift) & 255u], 1u);
+  }
+  __syncthreads();
+  hist[(uint64_t)threadIdx.x * nb + blockIdx.x] = h[threadIdx.x];
+}
+
+// Stable scatter of one 8-bit digit.  offs[d * nb + block] is the exclusive
+// scan of the digit-major histogram: where this block's digit-d keys start.
+__global__ void __launch_bounds__(RS_THREADS) k_radix_scatter(const uint64_t* __restrict__ kin,
+                                                              const uint32_t* __restrict__ vin,
+                                                              uint64_t* __restrict__ kout,
+                                                              uint32_t* __restrict__ vout, uint64_t n, int shift,
+                                                              const uint32_t* __restrict__ offs, uint64_t nb) {
+  __shared__ uint32_t wbin[RS_WARPS][256];
+  __shared__ uint32_t base_s[256];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  for (int d = tid; d < RS_WARPS * 256; d += RS_THREADS) (&wbin[0][0])[d] = 0;
+  base_s[tid] = offs[(uint64_t)tid * nb + blockIdx.x];
+  __syncthreads();
+  const uint64_t w0 = blockIdx.x * (uint64_t)RS_TILE + (uint64_t)warp * RS_WARP_CHUNK;
+  const uint32_t lt = (1u << lane) - 1u;
+  uint64_t key[RS_ITEMS];
+  uint32_t val[RS_ITEMS];
+  uint32_t lr[RS_ITEMS];
+#pragma unroll
+  for (int it = 0; it < RS_ITEMS; ++it) {
+    uint64_t idx = w0 + (uint64_t)it * 32 + lane;
+    bool ok = idx < n;
+    key[it] = ok ? kin[idx] : 0ull;
+    val[it] = ok ? vin[idx] : 0u;
+    uint32_t d = ok ? ((uint32_t)(key[it] >> shift) & 255u) : 256u;
+    uint32_t peers = __match_any_sync(0xFFFFFFFFu, d);
+    uint32_t cnt = (d < 256u) ? wbin[warp][d] : 0u;
+    lr[it] = cnt + __popc(peers & lt);
+    __syncwarp();
+    if (d < 256u && lane == __ffs(peers) - 1) wbin[warp][d] = cnt + __popc(peers);
+    __syncwarp();
+  }
+  __syncthreads();
+  {
+    uint32_t run = 0;
+#pragma unroll
+    for (int w = 0; w < RS_WARPS; ++w) {
+      uint32_t c = wbin[w][tid];
+      wbin[w][tid] = run;
+      run += c;
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int it = 0; it < RS_ITEMS; ++it) {
+    uint64_t idx = w0 + (uint64_t)it * 32 + lane;
+    if (idx < n) {
+      uint32_t d = (uint32_t)(key[it] >> shift) & 255u;
+      uint64_t pos = (uint64_t)base_s[d] + wbin[warp][d] + lr[it];
+      kout[pos] = key[it];
+      vout[pos] = val[it];
+    }
+  }
+}
+
+// ---- exclusive sum scan of uint32 (three-phase, recursive on the host) ----
+__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t x, uint32_t* total) {
+  __shared__ uint32_t warp_sums[SCAN_THREADS / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t inc = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    uint32_t y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+    if (lane >= o) inc += y;
+  }
+  if (lane == 31) warp_sums[warp] = inc;
+  __syncthreads();
+  if (warp == 0) {
+    uint32_t v = (lane < (int)(blockDim.x >> 5)) ? warp_sums[lane] : 0u;
+    uint32_t vi = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      uint32_t y = __shfl_up_sync(0xFFFFFFFFu, vi, o);
+      if (lane >= o) vi += y;
+    }
+    warp_sums[lane] = vi - v;
+    if (lane == 31) *total = vi;
+  }
+  __syncthreads();
+  uint32_t r = warp_sums[warp] + inc - x;
+  __syncthreads();
+  return r;
+}
+
+__global__ void __launch_bounds__(SCAN_THREADS) k_scan_reduce(const uint32_t* __restrict__ in, uint64_t n,
+                                                              uint32_t* __restrict__ partial) {
+  __shared__ uint32_t tot;
+  uint64_t base = blockIdx.x * (uint64_t)SCAN_TILE + (uint64_t)threadIdx.x * SCAN_ITEMS;
+  uint32_t s = 0;
+#pragma unroll
+  for (int k = 0; k < SCAN_ITEMS; ++k)
+    if (base + k < n) s += in[base + k];
+  block_exclusive_scan(s, &tot);
+  if (threadIdx.x == 0) partial[blockIdx.x] = tot;
+}
+
+__global__ void __launch_bounds__(SCAN_THREADS) k_scan_apply(uint32_t* __restrict__ data, uint64_t n,
+                                                             const uint32_t* __restrict__ partial) {
+  __shared__ uint32_t tot;
+  uint64_t base = blockIdx.x * (uint64_t)SCAN_TILE + (uint64_t)threadIdx.x * SCAN_ITEMS;
+  uint32_t v[SCAN_ITEMS];
+  uint32_t s = 0;
+#pragma unroll
+  for (int k = 0; k < SCAN_ITEMS; ++k) {
+    v[k] = (base + k < n) ? data[base + k] : 0u;
+    s += v[k];
+  }
+  uint32_t pre = block_exclusive_scan(s, &tot) + (partial ? partial[blockIdx.x] : 0u);
+#pragma unroll
+  for (int k = 0; k < SCAN_ITEMS; ++k) {
+    if (base + k < n) data[base + k] = pre;
+    pre += v[k];
+  }
+}
+
+cudaError_t exclusive_scan(uint32_t* data, uint64_t n, uint32_t* tmp, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  uint64_t nt = cdiv(n, SCAN_TILE);
+  if (nt == 1) {
+    k_scan_apply<<<1, SCAN_THREADS, 0, s>>>(data, n, nullptr);
+    return cudaGetLastError();
+  }
+  k_scan_reduce<<<(unsigned)nt, SCAN_THREADS, 0, s>>>(data, n, tmp);
+  cudaError_t e = exclusive_scan(tmp, nt, tmp + nt, s);
+  if (e != cudaSuccess) return e;
+  k_scan_apply<<<(unsigned)nt, SCAN_THREADS, 0, s>>>(data, n, tmp);
+  return cudaGetLastError();
+}
+
+// rank[val[j]] = number of distinct keys before position j (dense rank);
+// sa[j] = val[j]; ctl[1] = number of distinct keys.
+__global__ void k_ranks(const uint64_t* __restrict__ key, const uint32_t* val, const uint32_t* __restrict__ excl,
+                        uint64_t n, uint32_t* __restrict__ rank, uint32_t* sa, uint32_t* ctl) {
+  for (uint64_t j = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; j < n; j += (uint64_t)gridDim.x * blockDim.x) {
+    uint32_t h = (j == 0 || key[j] != key[j - 1]) ? 1u : 0u;
+    uint32_t v = val[j];
+    rank[v] = excl[j] + h - 1u;
+    sa[j] = v;
+    if (j == n - 1) ctl[1] = excl[j] + h;
+  }
+}
+
+__global__ void k_heads(const uint64_t* __restrict__ key, uint64_t n, uint32_t* __restrict__ head) {
+  for (uint64_t j = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; j < n; j += (uint64_t)gridDim.x * blockDim.x)
+    head[j] = (j == 0 || key[j] != key[j - 1]) ? 1u : 0u;
+}
+
+// bucket[v] = first j with T[sa[j]] >= v (binary search), bucket[vocab] = n.
+__global__ void k_bucket(const uint32_t* __restrict__ T, const uint32_t* __restrict__ sa, uint64_t n,
+                         uint32_t vocab, uint32_t* __restrict__ bucket) {
+  for (uint64_t v = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; v <= vocab; v += (uint64_t)gridDim.x * blockDim.x) {
+    uint64_t lo = 0, hi = n;
+    while (lo < hi) {
+      uint64_t mid = (lo + hi) >> 1;
+      if (T[sa[mid]] < v) lo = mid + 1;
+      else hi = mid;
+    }
+    bucket[v] = (uint32_t)lo;
+  }
+}
+
+inline int bits_for(uint64_t x) {
+  int b = 0;
+  while (x) {
+    ++b;
+    x >>= 1;
+  }
+  return b;
+}
+
+inline unsigned grid_for(uint64_t n, int threads) {
+  uint64_t g = cdiv(n, threads);
+  if (g > 152ull * 64) g = 152ull * 64;
+  return (unsigned)(g ? g : 1);
+}
+
+}  // namespace
+
+extern "C" size_t fc_datastore_build_workspace(uint64_t n_tokens, uint32_t vocab) {
+  (void)vocab;
+  if (n_tokens == 0) return 0;
+  return layout_for(n_tokens).total;
+}
+
+extern "C" fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n, uint32_t vocab, uint32_t* d_sa,
+                                        uint32_t* d_bucket, void* d_ws, size_t ws_bytes, fc_stream stream,
+                                        fc_datastore* out) {
+  if (!d_tokens || !d_sa || !d_bucket || n == 0 || n >= 0xFFFFFFFFull || vocab == 0 || vocab >= 0x80000000u)
+    return FC_ERR_INVALID_ARG;
+  Layout L = layout_for(n);
+  if (!d_ws || ws_bytes < L.total) return FC_ERR_WORKSPACE;
+  if (reinterpret_cast<uintptr_t>(d_ws) % 256) return FC_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(d_ws);
+  uint64_t* key_a = reinterpret_cast<uint64_t*>(ws + L.key_a);
+  uint64_t* key_b = reinterpret_cast<uint64_t*>(ws + L.key_b);
+  uint32_t* val_b = reinterpret_cast<uint32_t*>(ws + L.val_b);
+  uint32_t* rank = reinterpret_cast<uint32_t*>(ws + L.rank);
+  uint32_t* head = reinterpret_cast<uint32_t*>(ws + L.head);
+  uint32_t* hist = reinterpret_cast<uint32_t*>(ws + L.hist);
+  uint32_t* stmp = reinterpret_cast<uint32_t*>(ws + L.scan_tmp);
+  uint32_t* ctl = reinterpret_cast<uint32_t*>(ws + L.ctl);
+  const unsigned g = grid_for(n, 256);
+  uint32_t hctl[2] = {0, 0};
+
+  if (cudaMemsetAsync(ctl, 0, 64, s) != cudaSuccess) return FC_ERR_CUDA;
+  k_check_tokens<<<g, 256, 0, s>>>(d_tokens, n, vocab, ctl);
+  if (cudaMemcpyAsync(hctl, ctl, 8, cudaMemcpyDeviceToHost, s) != cudaSuccess) return FC_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return FC_ERR_CUDA;
+  if (hctl[0]) return FC_ERR_INVALID_ARG;
+
+  k_keys_first<<<g, 256, 0, s>>>(d_tokens, n, key_a, d_sa);
+  uint64_t max_hi = vocab - 1, max_lo = vocab;
+  uint64_t h = 1;
+  for (int round = 0;; ++round) {
+    if (round > 40) return FC_ERR_INTERNAL;
+    // LSD passes over the populated bits of the low then the high word.
+    uint64_t* kin = key_a;
+    uint32_t* vin = d_sa;
+    uint64_t* kout = key_b;
+    uint32_t* vout = val_b;
+    int shifts[16];
+    int np = 0;
+    for (int b = 0; b < bits_for(max_lo); b += 8) shifts[np++] = b;
+    for (int b = 0; b < bits_for(max_hi); b += 8) shifts[np++] = 32 + b;
+    for (int p = 0; p < np; ++p) {
+      k_radix_hist<<<(unsigned)L.nb, RS_THREADS, 0, s>>>(kin, n, shifts[p], hist, L.nb);
+      if (exclusive_scan(hist, 256 * L.nb, stmp, s) != cudaSuccess) return FC_ERR_CUDA;
+      k_radix_scatter<<<(unsigned)L.nb, RS_THREADS, 0, s>>>(kin, vin, kout, vout, n, shifts[p], hist, L.nb);
+      std::swap(kin, kout);
+      std::swap(vin, vout);
+    }
+    // kin/vin now hold the sorted keys and positions.
+    k_heads<<<g, 256, 0, s>>>(kin, n, head);
+    if (exclusive_scan(head, n, stmp, s) != cudaSuccess) return FC_ERR_CUDA;
+    k_ranks<<<g, 256, 0, s>>>(kin, vin, head, n, rank, d_sa, ctl);
+    if (cudaMemcpyAsync(hctl, ctl, 8, cudaMemcpyDeviceToHost, s) != cudaSuccess) return FC_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return FC_ERR_CUDA;
+    uint64_t groups = hctl[1];
+    if (groups == n) break;
+    if (groups == 0 || groups > n) return FC_ERR_INTERNAL;
+    h = (round == 0) ? 2 : h * 2;
+    if (h >= 2 * n + 2) return FC_ERR_INTERNAL;
+    k_keys_round<<<g, 256, 0, s>>>(d_sa, rank, n, h, key_a, d_sa);
+    max_hi = groups - 1;
+    max_lo = groups;
+  }
+  k_bucket<<<grid_for((uint64_t)vocab + 1, 256), 256, 0, s>>>(d_tokens, d_sa, n, vocab, d_bucket);
+  if (cudaGetLastError() != cudaSuccess) return FC_ERR_CUDA;
+  if (out) {
+    out->tokens = d_tokens;
+    out->sa = d_sa;
+    out->bucket = d_bucket;
+    out->n_tokens = n;
+    out->vocab = vocab;
+  }
+  return FC_OK;
+}

@@ -1,0 +1,316 @@
+"""Python binding of libfastcoder.so: argument marshalling only.
+
+Every function here checks tensor dtypes, devices and shapes, passes raw
+device pointers and the current CUDA stream to the C ABI of the same name
+(include/fastcoder.h), and raises FastCoderError on a non-OK status.  All
+computation happens in the CUDA kernels behind that ABI; if the library
+cannot be loaded, importing this module raises (there is no fallback).
+
+Tensor conventions: uint32 token ids travel in int32 tensors (same bits),
+uint64 mask words in int64 tensors, bf16 tensors as torch.bfloat16.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import torch
+
+from . import build as _build
+
+PAD = 0xFFFFFFFF
+PAD_I32 = -1  # FC_PAD_TOKEN seen through an int32 tensor
+MAX_OCC = 4096
+MAX_NODES = 128
+
+STATUS = {0: "FC_OK", 1: "FC_ERR_INVALID_ARG", 2: "FC_ERR_UNSUPPORTED", 3: "FC_ERR_WORKSPACE",
+          4: "FC_ERR_CAPACITY", 5: "FC_ERR_TIMEOUT", 6: "FC_ERR_CUDA", 7: "FC_ERR_INTERNAL"}
+
+
+class FastCoderError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        super().__init__(f"{fn} returned {STATUS.get(code, code)}")
+        self.code = code
+        self.status = STATUS.get(code, str(code))
+
+
+class fc_datastore(C.Structure):
+    _fields_ = [("tokens", C.c_void_p), ("sa", C.c_void_p), ("bucket", C.c_void_p),
+                ("n_tokens", C.c_uint64), ("vocab", C.c_uint32)]
+
+
+class fc_retrieve_params(C.Structure):
+    _fields_ = [("n_max", C.c_int32), ("n_min", C.c_int32), ("top_k", C.c_int32),
+                ("draft_len", C.c_int32), ("max_occ", C.c_uint32)]
+
+
+EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
+           "fc_retrieve", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
+           "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_accept", "fc_kv_append", "fc_synth_argmax"]
+
+
+def _load():
+    path = _build.LIB
+    if not os.path.exists(path):
+        raise ImportError(f"libfastcoder.so is not built ({path}); run __graft_entry__.build()")
+    lib = C.CDLL(path)
+    vp, i32, u32, u64, sz = C.c_void_p, C.c_int, C.c_uint32, C.c_uint64, C.c_size_t
+    sig = {
+        "fc_status_string": (C.c_char_p, [C.c_int]),
+        "fc_version": (C.c_char_p, []),
+        "fc_get_error": (C.c_int, [vp]),
+        "fc_datastore_build_workspace": (sz, [u64, u32]),
+        "fc_datastore_build": (C.c_int, [vp, u64, u32, vp, vp, vp, sz, vp, C.POINTER(fc_datastore)]),
+        "fc_retrieve": (C.c_int, [C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp, fc_retrieve_params,
+                                  vp, vp, vp, vp, vp, vp]),
+        "fc_rcache_bytes": (sz, [i32, i32, fc_retrieve_params]),
+        "fc_rcache_init": (C.c_int, [vp, sz, i32, i32, fc_retrieve_params, vp]),
+        "fc_rcache_lookup": (C.c_int, [vp, i32, i32, fc_retrieve_params, vp, i32, vp, i32, vp, vp,
+                                       vp, vp, vp, vp, vp, vp]),
+        "fc_rcache_insert": (C.c_int, [vp, i32, i32, fc_retrieve_params, vp, i32, vp, i32, vp,
+                                       vp, vp, vp, vp, vp, vp]),
+        "fc_build_tree": (C.c_int, [i32, vp, vp, vp, vp, C.POINTER(C.c_uint32), i32, i32, vp, vp, i32, i32, i32,
+                                    vp, vp, vp, vp, vp, vp, vp]),
+        "fc_tree_mask": (C.c_int, [vp, vp, vp, i32, i32, vp, vp, vp, vp]),
+        "fc_tree_attn": (C.c_int, [vp, vp, vp, i32, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, C.c_float, vp, vp]),
+        "fc_accept": (C.c_int, [vp, vp, vp, vp, i32, i32, vp, vp, i32, vp, vp]),
+        "fc_kv_append": (C.c_int, [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, i32,
+                                   vp, vp, vp, vp]),
+        "fc_synth_argmax": (C.c_int, [vp, vp, vp, i32, i32, vp, vp, u32, vp, vp]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    return lib
+
+
+LIB = _load()
+
+
+def _stream():
+    return C.c_void_p(torch.cuda.current_stream().cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _check(fn, code):
+    if code != 0:
+        raise FastCoderError(fn, code)
+
+
+def _need(t, dtype, name, shape=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be on a CUDA device")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    return t
+
+
+def version() -> str:
+    return LIB.fc_version().decode()
+
+
+def fc_get_error(stream=None) -> str:
+    s = C.c_void_p(stream.cuda_stream) if stream is not None else _stream()
+    return STATUS.get(LIB.fc_get_error(s), "?")
+
+
+# --------------------------------------------------------------- datastore
+class Datastore:
+    """A built datastore: the token corpus, its suffix array and bucket table
+    (device tensors owned here), plus the C view struct."""
+
+    def __init__(self, tokens, sa, bucket, vocab):
+        self.tokens, self.sa, self.bucket, self.vocab = tokens, sa, bucket, int(vocab)
+        self.view = fc_datastore(tokens.data_ptr(), sa.data_ptr(), bucket.data_ptr(), tokens.numel(), int(vocab))
+
+    @property
+    def n_tokens(self):
+        return self.tokens.numel()
+
+
+def fc_datastore_build_workspace(n_tokens: int, vocab: int) -> int:
+    return int(LIB.fc_datastore_build_workspace(n_tokens, vocab))
+
+
+def fc_datastore_build(tokens: torch.Tensor, vocab: int, workspace: torch.Tensor | None = None) -> Datastore:
+    """tokens: int32 [N] on the GPU (uint32 ids < vocab).  Synchronous."""
+    _need(tokens, torch.int32, "tokens")
+    n = tokens.numel()
+    sa = torch.empty(n, dtype=torch.int32, device=tokens.device)
+    bucket = torch.empty(vocab + 1, dtype=torch.int32, device=tokens.device)
+    need = fc_datastore_build_workspace(n, vocab)
+    ws = workspace if workspace is not None else torch.empty(need, dtype=torch.uint8, device=tokens.device)
+    if ws.numel() < need:
+        raise ValueError("workspace too small")
+    _check("fc_datastore_build", LIB.fc_datastore_build(_ptr(tokens), n, vocab, _ptr(sa), _ptr(bucket), _ptr(ws),
+                                                        ws.numel(), _stream(), None))
+    return Datastore(tokens, sa, bucket, vocab)
+
+
+def datastore_from_parts(tokens, sa, bucket, vocab) -> Datastore:
+    for t, nm in ((tokens, "tokens"), (sa, "sa"), (bucket, "bucket")):
+        _need(t, torch.int32, nm)
+    return Datastore(tokens, sa, bucket, vocab)
+
+
+# --------------------------------------------------------------- retrieval
+def params(n_max, n_min, top_k, draft_len, max_occ=MAX_OCC) -> fc_retrieve_params:
+    return fc_retrieve_params(n_max, n_min, top_k, draft_len, max_occ)
+
+
+def retrieve_outputs(n_sources, batch, p: fc_retrieve_params, device="cuda"):
+    S, B, k, d = n_sources, batch, p.top_k, p.draft_len
+    return dict(drafts=torch.empty((S, B, k, d), dtype=torch.int32, device=device),
+                draft_len=torch.empty((S, B, k), dtype=torch.int32, device=device),
+                count=torch.empty((S, B, k), dtype=torch.int32, device=device),
+                n_drafts=torch.empty((S, B), dtype=torch.int32, device=device),
+                match_len=torch.empty((S, B), dtype=torch.int32, device=device))
+
+
+def fc_retrieve(sources, ctx, ctx_len, p: fc_retrieve_params, skip=None, out=None):
+    """ctx: int32 [B, stride]; ctx_len: int32 [B]; returns dict of outputs
+    shaped [S, B, ...] (see include/fastcoder.h)."""
+    S = len(sources)
+    _need(ctx, torch.int32, "ctx")
+    B, stride = ctx.shape
+    _need(ctx_len, torch.int32, "ctx_len", (B,))
+    if skip is not None:
+        _need(skip, torch.int32, "skip", (B,))
+    o = out if out is not None else retrieve_outputs(S, B, p, ctx.device)
+    views = (fc_datastore * S)(*[s.view for s in sources])
+    _check("fc_retrieve", LIB.fc_retrieve(views, S, _ptr(ctx), stride, _ptr(ctx_len), B, _ptr(skip), p,
+                                          _ptr(o["drafts"]), _ptr(o["draft_len"]), _ptr(o["count"]),
+                                          _ptr(o["n_drafts"]), _ptr(o["match_len"]), _stream()))
+    return o
+
+
+class RetrievalCache:
+    """Context-keyed replay cache in caller-owned device memory."""
+
+    def __init__(self, capacity, n_sources, p: fc_retrieve_params, device="cuda"):
+        self.capacity, self.n_sources, self.p = capacity, n_sources, p
+        nbytes = int(LIB.fc_rcache_bytes(capacity, n_sources, p))
+        if nbytes == 0:
+            raise ValueError("bad cache parameters")
+        self.table = torch.empty(nbytes, dtype=torch.uint8, device=device)
+        _check("fc_rcache_init", LIB.fc_rcache_init(_ptr(self.table), nbytes, capacity, n_sources, p, _stream()))
+
+
+def fc_rcache_lookup(cache: RetrievalCache, ctx, ctx_len, want_hit, skip, out):
+    B, stride = ctx.shape
+    _check("fc_rcache_lookup", LIB.fc_rcache_lookup(
+        _ptr(cache.table), cache.capacity, cache.n_sources, cache.p, _ptr(ctx), stride, _ptr(ctx_len), B,
+        _ptr(want_hit), _ptr(skip), _ptr(out["drafts"]), _ptr(out["draft_len"]), _ptr(out["count"]),
+        _ptr(out["n_drafts"]), _ptr(out["match_len"]), _stream()))
+
+
+def fc_rcache_insert(cache: RetrievalCache, ctx, ctx_len, skip, res):
+    B, stride = ctx.shape
+    _check("fc_rcache_insert", LIB.fc_rcache_insert(
+        _ptr(cache.table), cache.capacity, cache.n_sources, cache.p, _ptr(ctx), stride, _ptr(ctx_len), B,
+        _ptr(skip), _ptr(res["drafts"]), _ptr(res["draft_len"]), _ptr(res["count"]), _ptr(res["n_drafts"]),
+        _ptr(res["match_len"]), _stream()))
+
+
+# -------------------------------------------------------------------- tree
+def tree_outputs(batch, n_pad, device="cuda"):
+    return dict(tok=torch.empty((batch, n_pad), dtype=torch.int32, device=device),
+                parent=torch.empty((batch, n_pad), dtype=torch.int32, device=device),
+                depth=torch.empty((batch, n_pad), dtype=torch.int32, device=device),
+                pos=torch.empty((batch, n_pad), dtype=torch.int32, device=device),
+                mask=torch.empty((batch, n_pad, n_pad // 64), dtype=torch.int64, device=device),
+                n_nodes=torch.empty(batch, dtype=torch.int32, device=device))
+
+
+def fc_build_tree(res, src_weight, root_tok, kv_len, node_budget, n_pad, out=None):
+    """res: fc_retrieve outputs ([S, B, ...]); src_weight: S ints."""
+    S, B, k, d = res["drafts"].shape
+    _need(root_tok, torch.int32, "root_tok", (B,))
+    _need(kv_len, torch.int32, "kv_len", (B,))
+    w = (C.c_uint32 * S)(*[int(x) for x in src_weight])
+    o = out if out is not None else tree_outputs(B, n_pad, root_tok.device)
+    _check("fc_build_tree", LIB.fc_build_tree(S, _ptr(res["drafts"]), _ptr(res["draft_len"]), _ptr(res["count"]),
+                                              _ptr(res["n_drafts"]), w, k, d, _ptr(root_tok), _ptr(kv_len), B,
+                                              node_budget, n_pad, _ptr(o["tok"]), _ptr(o["parent"]),
+                                              _ptr(o["depth"]), _ptr(o["pos"]), _ptr(o["mask"]), _ptr(o["n_nodes"]),
+                                              _stream()))
+    return o
+
+
+def fc_tree_mask(parent, n_nodes, kv_len):
+    _need(parent, torch.int32, "parent")
+    B, n_pad = parent.shape
+    _need(n_nodes, torch.int32, "n_nodes", (B,))
+    _need(kv_len, torch.int32, "kv_len", (B,))
+    dev = parent.device
+    o = dict(depth=torch.empty((B, n_pad), dtype=torch.int32, device=dev),
+             pos=torch.empty((B, n_pad), dtype=torch.int32, device=dev),
+             mask=torch.empty((B, n_pad, n_pad // 64), dtype=torch.int64, device=dev))
+    _check("fc_tree_mask", LIB.fc_tree_mask(_ptr(parent), _ptr(n_nodes), _ptr(kv_len), B, n_pad, _ptr(o["depth"]),
+                                            _ptr(o["pos"]), _ptr(o["mask"]), _stream()))
+    return o
+
+
+# --------------------------------------------------------------- attention
+def fc_tree_attn(q, k_cache, v_cache, kv_len, k_tree, v_tree, mask, n_nodes, scale=None, out=None):
+    """q [B, Np, H, D]; caches [B, Hkv, cap, D]; tree K/V [B, Hkv, Np, D] (bf16)."""
+    _need(q, torch.bfloat16, "q")
+    B, Np, H, D = q.shape
+    _need(k_cache, torch.bfloat16, "k_cache")
+    Hkv, cap = k_cache.shape[1], k_cache.shape[2]
+    _need(v_cache, torch.bfloat16, "v_cache", k_cache.shape)
+    _need(k_tree, torch.bfloat16, "k_tree", (B, Hkv, Np, D))
+    _need(v_tree, torch.bfloat16, "v_tree", (B, Hkv, Np, D))
+    _need(mask, torch.int64, "mask", (B, Np, Np // 64))
+    _need(kv_len, torch.int32, "kv_len", (B,))
+    _need(n_nodes, torch.int32, "n_nodes", (B,))
+    o = out if out is not None else torch.empty_like(q)
+    sc = float(scale) if scale is not None else D ** -0.5
+    _check("fc_tree_attn", LIB.fc_tree_attn(_ptr(q), _ptr(k_cache), _ptr(v_cache), cap, _ptr(kv_len), _ptr(k_tree),
+                                            _ptr(v_tree), _ptr(mask), _ptr(n_nodes), B, Np, H, Hkv, D, sc, _ptr(o),
+                                            _stream()))
+    return o
+
+
+# ---------------------------------------------------------- accept / append
+def fc_accept(tok, parent, n_nodes, argmax, path_cap, out=None):
+    B, Np = tok.shape
+    for t, nm in ((tok, "tok"), (parent, "parent"), (argmax, "argmax")):
+        _need(t, torch.int32, nm, (B, Np))
+    _need(n_nodes, torch.int32, "n_nodes", (B,))
+    dev = tok.device
+    o = out if out is not None else dict(acc_len=torch.empty(B, dtype=torch.int32, device=dev),
+                                         path=torch.empty((B, path_cap), dtype=torch.int32, device=dev),
+                                         bonus=torch.empty(B, dtype=torch.int32, device=dev))
+    _check("fc_accept", LIB.fc_accept(_ptr(tok), _ptr(parent), _ptr(n_nodes), _ptr(argmax), B, Np, _ptr(o["acc_len"]),
+                                      _ptr(o["path"]), path_cap, _ptr(o["bonus"]), _stream()))
+    return o
+
+
+def fc_kv_append(acc, tok, k_tree, v_tree, k_cache, v_cache, kv_len_in, kv_len_out, ctx, ctx_len_in, ctx_len_out,
+                 root_out):
+    B, Hkv, Np, D = k_tree.shape
+    cap = k_cache.shape[2]
+    _need(ctx, torch.int32, "ctx")
+    _check("fc_kv_append", LIB.fc_kv_append(
+        _ptr(acc["path"]), _ptr(acc["acc_len"]), _ptr(acc["bonus"]), _ptr(tok), _ptr(k_tree), _ptr(v_tree), B, Np, Hkv,
+        D, acc["path"].shape[1], _ptr(k_cache), _ptr(v_cache), cap, _ptr(kv_len_in), _ptr(kv_len_out), _ptr(ctx),
+        ctx.shape[1], _ptr(ctx_len_in), _ptr(ctx_len_out), _ptr(root_out), _stream()))
+
+
+def fc_synth_argmax(tok, parent, n_nodes, plen, rtok, vocab, out=None):
+    B, Np = tok.shape
+    o = out if out is not None else torch.empty((B, Np), dtype=torch.int32, device=tok.device)
+    _check("fc_synth_argmax", LIB.fc_synth_argmax(_ptr(tok), _ptr(parent), _ptr(n_nodes), B, Np, _ptr(plen),
+                                                  _ptr(rtok), vocab, _ptr(o), _stream()))
+    return o

@@ -1,0 +1,82 @@
+"""One retrieve-and-verify decoding step, composed from the C-ABI calls.
+
+A step (Section IV-C Algorithm 1 and Section IV-D) for a batch of sequences:
+  cache lookup -> fc_retrieve on every source (queries the cache served are
+  skipped) -> cache insert -> fc_build_tree -> fc_tree_attn ->
+  target-model predictions (the synthetic stand-in) -> fc_accept ->
+  fc_kv_append (cache rows, context, lengths and next root).
+
+Every call is asynchronous on the current stream and allocates nothing, so a
+step can be captured once into a CUDA graph and replayed (lengths ping-pong
+between two buffers, so a graph holds two consecutive steps).
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import fastcoder as fc
+
+
+class StepLoop:
+    def __init__(self, sources, ctx, ctx_len, p, node_budget, n_pad, src_weight, H, Hkv, D, kv_cap, kv_len0, vocab,
+                 cache_capacity=1 << 14, device="cuda", k_cache=None, v_cache=None):
+        self.sources, self.p, self.node_budget, self.n_pad = sources, p, node_budget, n_pad
+        self.src_weight = list(src_weight)
+        self.H, self.Hkv, self.D, self.kv_cap, self.vocab = H, Hkv, D, kv_cap, vocab
+        ctx = torch.as_tensor(np.ascontiguousarray(ctx).view(np.int32)) if isinstance(ctx, np.ndarray) else ctx
+        ctx_len = torch.as_tensor(np.asarray(ctx_len, np.int32)) if isinstance(ctx_len, np.ndarray) else ctx_len
+        self.B = ctx.shape[0]
+        B = self.B
+        self.ctx = ctx.to(device=device, dtype=torch.int32).contiguous()
+        self.ctx_len = [ctx_len.to(device=device, dtype=torch.int32).clone(), torch.empty(B, dtype=torch.int32, device=device)]
+        kv0 = torch.as_tensor(np.broadcast_to(np.asarray(kv_len0, np.int32), (B,)).copy())
+        self.kv_len = [kv0.to(device), torch.empty(B, dtype=torch.int32, device=device)]
+        cl = self.ctx_len[0].long()
+        self.root = self.ctx.gather(1, (cl - 1).clamp(min=0).view(B, 1)).view(B).contiguous()
+        self.cur = 0
+        S = len(sources)
+        self.res = fc.retrieve_outputs(S, B, p, device)
+        self.skip = torch.zeros(B, dtype=torch.int32, device=device)
+        self.tree = fc.tree_outputs(B, n_pad, device)
+        self.argmax = torch.empty((B, n_pad), dtype=torch.int32, device=device)
+        self.path_cap = p.draft_len + 2
+        self.acc = dict(acc_len=torch.empty(B, dtype=torch.int32, device=device),
+                        path=torch.empty((B, self.path_cap), dtype=torch.int32, device=device),
+                        bonus=torch.empty(B, dtype=torch.int32, device=device))
+        shape = (B, Hkv, kv_cap, D)
+        self.k_cache = k_cache if k_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
+        self.v_cache = v_cache if v_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
+        self.attn_out = torch.empty((B, n_pad, H, D), dtype=torch.bfloat16, device=device)
+        self.cache = fc.RetrievalCache(cache_capacity, S, p, device) if cache_capacity else None
+
+    def step(self, q, k_tree, v_tree, want_hit, plen, rtok, attention=True):
+        """Enqueue one step.  q [B, Np, H, D], k_tree/v_tree [B, Hkv, Np, D]
+        (bf16); want_hit [B], plen [B], rtok [B, Np] (int32)."""
+        c, n = self.cur, 1 - self.cur
+        if self.cache is not None:
+            fc.fc_rcache_lookup(self.cache, self.ctx, self.ctx_len[c], want_hit, self.skip, self.res)
+            fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, skip=self.skip, out=self.res)
+            fc.fc_rcache_insert(self.cache, self.ctx, self.ctx_len[c], self.skip, self.res)
+        else:
+            fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, out=self.res)
+        fc.fc_build_tree(self.res, self.src_weight, self.root, self.kv_len[c], self.node_budget, self.n_pad,
+                         out=self.tree)
+        if attention:
+            fc.fc_tree_attn(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree, self.tree["mask"],
+                            self.tree["n_nodes"], out=self.attn_out)
+        fc.fc_synth_argmax(self.tree["tok"], self.tree["parent"], self.tree["n_nodes"], plen, rtok, self.vocab,
+                           out=self.argmax)
+        fc.fc_accept(self.tree["tok"], self.tree["parent"], self.tree["n_nodes"], self.argmax, self.path_cap,
+                     out=self.acc)
+        fc.fc_kv_append(self.acc, self.tree["tok"], k_tree, v_tree, self.k_cache, self.v_cache, self.kv_len[c],
+                        self.kv_len[n], self.ctx, self.ctx_len[c], self.ctx_len[n], self.root)
+        self.cur = n
+
+    @property
+    def kv_len_now(self):
+        return self.kv_len[self.cur]
+
+    @property
+    def ctx_len_now(self):
+        return self.ctx_len[self.cur]

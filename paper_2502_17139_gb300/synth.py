@@ -188,7 +188,8 @@ def random_tree(rng: np.random.Generator, n_nodes: int, depth_max: int = 10,
     tok = [int(rng.integers(0, vocab)) if root_tok is None else int(root_tok)]
     kids = [set()]
     while len(par) < n_nodes:
-        open_nodes = [i for i in range(len(par)) if dep[i] < depth_max and len(kids[i]) < branch_max]
+        open_nodes = [i for i in range(len(par))
+                      if dep[i] < depth_max and len(kids[i]) < min(branch_max, vocab)]
         v = open_nodes[int(rng.integers(0, len(open_nodes)))]
         while True:
             t = int(rng.integers(0, vocab))

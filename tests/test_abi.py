@@ -1,0 +1,79 @@
+"""The C-ABI library builds, loads and exports every entry point that
+include/fastcoder.h declares; host-side argument validation rejects bad calls
+before anything reaches a GPU (these calls launch nothing)."""
+import ctypes as C
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "fastcoder.h")
+
+
+def declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(fc_[a-z0-9_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2502_17139_gb300 import build
+    path = build.build()
+    return path
+
+
+def test_exports_match_header(lib):
+    names = declared()
+    assert "fc_tree_attn" in names and "fc_retrieve" in names and len(names) >= 15
+    out = subprocess.run(["nm", "-D", "--defined-only", lib], capture_output=True, text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (fc_[a-z0-9_]+)", out))
+    missing = [n for n in names if n not in exported]
+    assert not missing, missing
+
+
+def test_binding_names_match_header(lib):
+    import paper_2502_17139_gb300.fastcoder as fc
+    for n in declared():
+        assert hasattr(fc.LIB, n)
+    assert fc.version() == "0.1.0"
+    assert fc.LIB.fc_status_string(5) == b"FC_ERR_TIMEOUT"
+
+
+def test_host_validation_without_gpu(lib):
+    import paper_2502_17139_gb300.fastcoder as fc
+    L = fc.LIB
+    p = fc.params(16, 2, 16, 8)
+    nul = None
+    # no sources
+    assert L.fc_retrieve(nul, 0, nul, 64, nul, 4, nul, p, nul, nul, nul, nul, nul, nul) == 1
+    # parameters beyond what the kernels support
+    views = (fc.fc_datastore * 1)(fc.fc_datastore(1, 1, 1, 10, 5))
+    assert L.fc_retrieve(views, 1, 1, 64, 1, 4, nul, fc.params(40, 2, 16, 8), 1, 1, 1, 1, 1, nul) == 2
+    assert L.fc_retrieve(views, 1, 1, 64, 1, 4, nul, fc.params(16, 2, 16, 8, 0), 1, 1, 1, 1, 1, nul) == 2
+    # empty batch is a no-op
+    assert L.fc_retrieve(views, 1, nul, 64, nul, 0, nul, p, nul, nul, nul, nul, nul, nul) == 0
+    # attention: head dim / tree padding / GQA ratio outside the supported set
+    args = [1, 1, 1, 128, 1, 1, 1, 8, 1, 2]
+    assert L.fc_tree_attn(*args, 64, 32, 8, 64, C.c_float(0.1), 1, nul) == 2
+    assert L.fc_tree_attn(*args, 96, 32, 8, 128, C.c_float(0.1), 1, nul) == 2
+    assert L.fc_tree_attn(*args, 64, 30, 8, 128, C.c_float(0.1), 1, nul) == 2
+    assert L.fc_tree_attn(*args, 64, 32, 8, 128, C.c_float(-1.0), 1, nul) == 1
+    # misaligned pointer
+    assert L.fc_tree_attn(3, 16, 16, 128, 16, 16, 16, 8, 16, 2, 64, 32, 8, 128, C.c_float(0.1), 16, nul) == 1
+    # tree: budget larger than the padding, too many drafts
+    w = (C.c_uint32 * 2)(1, 1)
+    tree_ptrs = [1] * 6
+    assert L.fc_build_tree(2, 1, 1, 1, 1, w, 64, 10, 1, 1, 4, 65, 64, *tree_ptrs, nul) == 1
+    assert L.fc_build_tree(2, 1, 1, 1, 1, w, 300, 10, 1, 1, 4, 64, 64, *tree_ptrs, nul) == 2
+    # datastore: empty corpus, short workspace
+    assert L.fc_datastore_build(1, 0, 10, 1, 1, 1, 1 << 20, nul, nul) == 1
+    need = L.fc_datastore_build_workspace(1000, 10)
+    assert need > 1000 * 28
+    assert L.fc_datastore_build(1, 1000, 10, 1, 1, 256, need - 1, nul, nul) == 3
+    # kv append: aliasing in/out lengths
+    assert L.fc_kv_append(1, 1, 1, 1, 16, 16, 2, 64, 8, 128, 12, 16, 16, 100, 8, 8, 1, 64, 4, 12, 1, nul) == 1
+    # cache: capacity must be a power of two
+    assert L.fc_rcache_init(1, 1 << 30, 1000, 2, p, nul) == 1

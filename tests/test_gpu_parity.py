@@ -1,0 +1,428 @@
+"""GPU parity: every kernel behind the C ABI against the CPU oracle, element
+by element on the same seeded inputs.
+
+Integer outputs (suffix arrays, buckets, retrieval results, trees, masks,
+acceptance, cache append) must be bit-exact.  Tree attention (bf16 inputs,
+fp32 accumulation and softmax on the GPU) must be within max-abs 2e-2 of the
+fp64 oracle.
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2502_17139_gb300.synth as synth
+
+pytestmark = pytest.mark.gpu
+ATOL = 2e-2
+PAD = 0xFFFFFFFF
+
+
+@pytest.fixture(scope="module")
+def fc():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2502_17139_gb300 import build
+    build.build()
+    import paper_2502_17139_gb300.fastcoder as fcm
+    return fcm
+
+
+def dev(a):
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint32:
+        a = a.view(np.int32)
+    elif a.dtype == np.uint64:
+        a = a.view(np.int64)
+    return torch.from_numpy(a.copy()).cuda()
+
+
+def host_u32(t):
+    return t.cpu().numpy().view(np.uint32)
+
+
+def bits_bf16(t):
+    return t.cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def check_no_error(fc):
+    assert fc.fc_get_error() == "FC_OK"
+
+
+# ------------------------------------------------------------ suffix array
+@pytest.mark.parametrize("n,vocab,seed", [(1, 5, 0), (2, 2, 1), (3, 2, 2), (57, 2, 3), (4096, 3, 4),
+                                          (4097, 8, 5), (8192 + 17, 4, 6), (50000, 2, 7), (70001, 300, 8)])
+def test_sa_small_sweep(fc, orc, n, vocab, seed):
+    rng = np.random.default_rng(seed)
+    T = rng.integers(0, vocab, n).astype(np.uint32)
+    if n > 100:
+        T[n // 3:n // 3 + 60] = T[:60]  # a long repeat
+    ds = fc.fc_datastore_build(dev(T), vocab)
+    torch.cuda.synchronize()
+    assert np.array_equal(host_u32(ds.sa), orc.suffix_array(T))
+    assert np.array_equal(host_u32(ds.bucket), orc.bucket(T, orc.suffix_array(T), vocab))
+
+
+def test_sa_constant_corpus(fc, orc):
+    T = np.full(10000, 7, np.uint32)
+    ds = fc.fc_datastore_build(dev(T), 8)
+    assert host_u32(ds.sa).tolist() == list(range(9999, -1, -1))
+
+
+def test_sa_rejects_bad_token(fc):
+    T = np.array([1, 2, 9, 3], np.uint32)
+    with pytest.raises(fc.FastCoderError) as e:
+        fc.fc_datastore_build(dev(T), 5)
+    assert e.value.status == "FC_ERR_INVALID_ARG"
+
+
+@pytest.fixture(scope="module")
+def c1(fc, orc):
+    cfg = synth.CONFIGS[1]
+    rng = synth.rng_for(1)
+    T, _ = synth.build_corpus(rng, cfg["corpus"][0])
+    ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], [T], [1.0], 1.1)
+    ds = fc.fc_datastore_build(dev(T), synth.VOCAB)
+    return dict(cfg=cfg, T=T, ctx=ctx, cl=cl, ds=ds)
+
+
+def test_sa_c1_corpus(fc, orc, c1):
+    sa = orc.suffix_array(c1["T"])
+    assert np.array_equal(host_u32(c1["ds"].sa), sa)
+    assert np.array_equal(host_u32(c1["ds"].bucket), orc.bucket(c1["T"], sa, synth.VOCAB))
+
+
+# --------------------------------------------------------------- retrieval
+def compare_retrieval(gpu, ref, s=0):
+    for name in ("drafts", "draft_len", "count", "n_drafts", "match_len"):
+        g = gpu[name][s].cpu().numpy()
+        r = ref[name]
+        if r.dtype == np.uint32:
+            g = g.view(np.uint32)
+        assert np.array_equal(g, r), name
+
+
+def test_retrieve_c1(fc, orc, c1):
+    cfg = c1["cfg"]
+    p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
+    g = fc.fc_retrieve([c1["ds"]], dev(c1["ctx"]), dev(c1["cl"]), p)
+    r = orc.retrieve(c1["T"], c1["ctx"], c1["cl"], cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
+    compare_retrieval(g, r)
+    assert (r["match_len"] >= 8).mean() > 0.5  # most contexts end with a copied corpus span
+    check_no_error(fc)
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_retrieve_tiny_sweep(fc, orc, seed):
+    rng = np.random.default_rng(500 + seed)
+    N = int(rng.integers(2, 3000))
+    vocab = int(rng.integers(2, 7))
+    T = rng.integers(0, vocab, N).astype(np.uint32)
+    B, stride = 40, 24
+    ctx = rng.integers(0, vocab, (B, stride)).astype(np.uint32)
+    cl = rng.integers(0, stride + 1, B).astype(np.int32)
+    for b in range(0, B, 2):
+        L = int(min(cl[b], N))
+        if L:
+            p0 = int(rng.integers(0, N - L + 1))
+            ctx[b, cl[b] - L:cl[b]] = T[p0:p0 + L]
+    n_max = int(rng.integers(1, 33))
+    n_min = int(rng.integers(1, n_max + 1)) if seed % 2 else min(2, n_max)
+    k, d = int(rng.integers(1, 257)), int(rng.integers(1, 17))
+    max_occ = [1, 3, 4096, 17][seed % 4]
+    ds = fc.fc_datastore_build(dev(T), vocab)
+    g = fc.fc_retrieve([ds], dev(ctx), dev(cl), fc.params(n_max, n_min, k, d, max_occ))
+    r = orc.retrieve(T, ctx, cl, n_max, n_min, k, d, max_occ)
+    compare_retrieval(g, r)
+    check_no_error(fc)
+
+
+def test_retrieve_two_sources_and_skip(fc, orc):
+    rng = synth.rng_for(40)
+    Tr, _ = synth.make_corpus(rng, 60000, 1.3, 500, n_grams=300, len_range=(8, 40))
+    Tc, _ = synth.make_corpus(rng, 150000, 1.1, 500)
+    ctx, cl, _ = synth.make_contexts(rng, 64, 40, 16, [Tr, Tc, None], [0.5, 0.25, 0.25], 1.1, 500)
+    dsr, dsc = fc.fc_datastore_build(dev(Tr), 500), fc.fc_datastore_build(dev(Tc), 500)
+    p = fc.params(16, 2, 64, 10, 4096)
+    skip = np.zeros(64, np.int32)
+    skip[::5] = 1
+    out = fc.retrieve_outputs(2, 64, p)
+    for v in out.values():
+        v.fill_(-7)
+    g = fc.fc_retrieve([dsr, dsc], dev(ctx), dev(cl), p, skip=dev(skip), out=out)
+    for s, T in enumerate((Tr, Tc)):
+        r = orc.retrieve(T, ctx, cl, 16, 2, 64, 10, 4096)
+        keep = skip == 0
+        for name in r:
+            gg = g[name][s].cpu().numpy()
+            if r[name].dtype == np.uint32:
+                gg = gg.view(np.uint32)
+            assert np.array_equal(gg[keep], r[name][keep]), name
+            assert (g[name][s].cpu().numpy()[~keep] == -7).all()
+
+
+def test_retrieve_bad_context_token(fc):
+    T = np.arange(100, dtype=np.uint32) % 10
+    ds = fc.fc_datastore_build(dev(T), 10)
+    ctx = np.array([[1, 2, 3, 4], [1, 2, 99, 4]], np.uint32)
+    g = fc.fc_retrieve([ds], dev(ctx), dev(np.array([4, 4], np.int32)), fc.params(4, 1, 4, 4, 64))
+    assert fc.fc_get_error() == "FC_ERR_INVALID_ARG"
+    assert int(g["match_len"][0, 0]) == 4 and int(g["match_len"][0, 1]) == 0
+
+
+# -------------------------------------------------------------------- tree
+def compare_tree(g, r):
+    for name in ("tok", "parent", "depth", "pos", "n_nodes"):
+        gg = g[name].cpu().numpy()
+        if r[name].dtype == np.uint32:
+            gg = gg.view(np.uint32)
+        assert np.array_equal(gg, r[name]), name
+    assert np.array_equal(g["mask"].cpu().numpy().view(np.uint64), r["mask"])
+
+
+def test_tree_from_c1_retrieval(fc, orc, c1):
+    cfg = c1["cfg"]
+    p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
+    g = fc.fc_retrieve([c1["ds"]], dev(c1["ctx"]), dev(c1["cl"]), p)
+    r = orc.retrieve(c1["T"], c1["ctx"], c1["cl"], cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
+    root = c1["ctx"][np.arange(32), c1["cl"] - 1]
+    kvl = np.full(32, 512, np.int32)
+    for budget in (1, 17, 64):
+        gt = fc.fc_build_tree(g, [1], dev(root), dev(kvl), budget, 64)
+        rt = orc.build_tree([r], [1], root, kvl, budget, 64)
+        compare_tree(gt, rt)
+    check_no_error(fc)
+
+
+def _random_sources(rng, S, B, k, d, vocab):
+    res = []
+    for s in range(S):
+        o = dict(drafts=np.full((B, k, d), PAD, np.uint32), draft_len=np.zeros((B, k), np.int32),
+                 count=np.zeros((B, k), np.uint32), n_drafts=np.zeros(B, np.int32), match_len=np.ones(B, np.int32))
+        for b in range(B):
+            nd = int(rng.integers(0, k + 1))
+            seen, t = set(), 0
+            while t < nd:
+                L = int(rng.integers(1, d + 1))
+                u = tuple(int(x) for x in rng.integers(0, vocab, L))
+                if u in seen:
+                    continue
+                seen.add(u)
+                o["drafts"][b, t, :L] = u
+                o["draft_len"][b, t] = L
+                o["count"][b, t] = int(rng.integers(1, 4097))
+                t += 1
+            o["n_drafts"][b] = nd
+        res.append(o)
+    return res
+
+
+@pytest.mark.parametrize("S,k,d,vocab,n_pad", [(1, 16, 8, 3, 64), (2, 64, 10, 4, 128), (2, 64, 10, 32256, 64),
+                                               (2, 256, 16, 2, 128), (4, 128, 12, 5, 128)])
+def test_tree_random_drafts(fc, orc, S, k, d, vocab, n_pad):
+    rng = np.random.default_rng(S * 1000 + k + d + vocab)
+    B = 24
+    res = _random_sources(rng, S, B, k, d, vocab)
+    w = rng.integers(1, 5, S).astype(np.uint32)
+    root = rng.integers(0, vocab, B).astype(np.uint32)
+    kvl = rng.integers(0, 5000, B).astype(np.int32)
+    g_res = {name: dev(np.stack([r[name] for r in res])) for name in res[0]}
+    for budget in (1, 2, n_pad // 2 + 1, n_pad):
+        gt = fc.fc_build_tree(g_res, w, dev(root), dev(kvl), budget, n_pad)
+        rt = orc.build_tree(res, w, root, kvl, budget, n_pad)
+        compare_tree(gt, rt)
+    check_no_error(fc)
+
+
+def _random_trees(rng, B, n_pad, vocab=32256, full=False):
+    tok = np.full((B, n_pad), PAD, np.uint32)
+    par = np.full((B, n_pad), -1, np.int32)
+    nn = np.full(B, n_pad, np.int32) if full else rng.integers(1, n_pad + 1, B).astype(np.int32)
+    for b in range(B):
+        t, p = synth.random_tree(rng, int(nn[b]), 10, 4, vocab)
+        tok[b, :nn[b]], par[b, :nn[b]] = t, p
+    return tok, par, nn
+
+
+def test_tree_mask_from_parents(fc, orc):
+    rng = synth.rng_for(41)
+    for n_pad in (64, 128):
+        tok, par, nn = _random_trees(rng, 20, n_pad)
+        kvl = rng.integers(0, 100, 20).astype(np.int32)
+        g = fc.fc_tree_mask(dev(par), dev(nn), dev(kvl))
+        r = orc.tree_mask(par, nn, kvl, n_pad)
+        assert np.array_equal(g["mask"].cpu().numpy().view(np.uint64), r["mask"])
+        assert np.array_equal(g["depth"].cpu().numpy(), r["depth"])
+        assert np.array_equal(g["pos"].cpu().numpy(), r["pos"])
+
+
+# --------------------------------------------------------------- attention
+def _attn_case(fc, orc, seed, B, n_pad, H, Hkv, kv_len, cap, nn=None, full_rows=True, sample=None):
+    rng = synth.rng_for(50, seed)
+    tok, par, nn_r = _random_trees(rng, B, n_pad)
+    if nn is not None:
+        nn_r = np.asarray(nn, np.int32)
+        for b in range(B):
+            t, p = synth.random_tree(rng, int(nn_r[b]), 10, 4, 1000)
+            par[b] = -1
+            par[b, :nn_r[b]] = p
+    kvl = np.asarray(kv_len, np.int32)
+    D = 128
+    q = synth.randn_bf16((B, n_pad, H, D), 1000 + seed, "cuda")
+    kc = synth.randn_bf16((B, Hkv, cap, D), 2000 + seed, "cuda")
+    vc = synth.randn_bf16((B, Hkv, cap, D), 3000 + seed, "cuda")
+    kt = synth.randn_bf16((B, Hkv, n_pad, D), 4000 + seed, "cuda")
+    vt = synth.randn_bf16((B, Hkv, n_pad, D), 5000 + seed, "cuda")
+    gm = fc.fc_tree_mask(dev(par), dev(nn_r), dev(kvl))
+    out = torch.full_like(q, float("nan"))
+    fc.fc_tree_attn(q, kc, vc, dev(kvl), kt, vt, gm["mask"], dev(nn_r), out=out)
+    torch.cuda.synchronize()
+    check_no_error(fc)
+    rm = orc.tree_mask(par, nn_r, kvl, n_pad)["mask"]
+    args = [bits_bf16(x) for x in (q, kc, vc)] + [kvl] + [bits_bf16(x) for x in (kt, vt)] + [rm, nn_r]
+    got = out.float().cpu().numpy()
+    if full_rows:
+        ref = orc.tree_attn(args[0], args[1], args[2], args[3], args[4], args[5], args[6], args[7])
+        err = np.abs(got - ref).max()
+        assert np.isfinite(got).all()
+    else:
+        rows = []
+        for b in range(B):
+            for i in sorted({0, int(nn_r[b]) - 1, int(rng.integers(0, nn_r[b])), min(n_pad - 1, int(nn_r[b]))}):
+                for h in sorted({0, H - 1, int(rng.integers(0, H))}):
+                    rows.append((b, i, h))
+        if sample:
+            rows = [rows[i] for i in rng.choice(len(rows), min(sample, len(rows)), replace=False)]
+        rows = np.array(rows, np.int32)
+        ref = orc.tree_attn(args[0], args[1], args[2], args[3], args[4], args[5], args[6], args[7], rows=rows)
+        g = got[rows[:, 0], rows[:, 1], rows[:, 2]]
+        err = np.abs(g - ref).max()
+        assert np.isfinite(g).all()
+    assert err <= ATOL, err
+    return err
+
+
+def test_attn_c1_shape_full(fc, orc):
+    # c1: B=32, H=Hkv=32, D=128, KV 512, trees <= 64 nodes
+    _attn_case(fc, orc, 1, 32, 64, 32, 32, [512] * 32, 512)
+
+
+def test_attn_ragged_edges(fc, orc):
+    B = 8
+    kvl = [0, 1, 127, 128, 129, 300, 511, 512]
+    _attn_case(fc, orc, 2, B, 64, 8, 8, kvl, 512, nn=[1, 2, 63, 64, 64, 5, 1, 33])
+
+
+def test_attn_gqa_n128(fc, orc):
+    B = 6
+    kvl = [0, 5, 128, 1000, 2047, 2048]
+    _attn_case(fc, orc, 3, B, 128, 32, 8, kvl, 2048, nn=[1, 20, 32, 33, 127, 128])
+
+
+def test_attn_gqa_n64_group2(fc, orc):
+    _attn_case(fc, orc, 4, 5, 64, 16, 8, [300, 0, 64, 700, 129], 777, nn=[64, 1, 40, 64, 2])
+
+
+def test_attn_c3_shape_sampled(fc, orc):
+    # c3: B=16, H=Hkv=32, KV 4096, 64-node trees
+    _attn_case(fc, orc, 5, 16, 64, 32, 32, [4096] * 16, 4096, nn=[64] * 16, full_rows=False)
+
+
+def test_attn_c5_shape_sampled(fc, orc):
+    # c5: B=32, H=32, Hkv=8, KV 16384, trees <= 128 nodes
+    _attn_case(fc, orc, 6, 32, 128, 32, 8, [16384] * 32, 16384 + 256, full_rows=False, sample=160)
+
+
+# ------------------------------------------------------- accept / append
+def test_accept_and_synth_argmax(fc, orc):
+    rng = synth.rng_for(60)
+    for n_pad, vocab in ((64, 32256), (128, 4), (64, 3)):
+        B = 64
+        tok, par, nn = _random_trees(rng, B, n_pad, vocab=vocab)
+        plen, rtok = synth.argmax_draws(rng, B, n_pad, vocab)
+        g_am = fc.fc_synth_argmax(dev(tok), dev(par), dev(nn), dev(plen), dev(rtok), vocab)
+        r_am = orc.synth_argmax(tok, par, nn, plen, rtok, vocab)
+        assert np.array_equal(host_u32(g_am), r_am)
+        # random predictions that often follow some child
+        am = rng.integers(0, vocab, (B, n_pad)).astype(np.uint32)
+        for b in range(B):
+            for i in range(nn[b]):
+                ch = [j for j in range(1, nn[b]) if par[b, j] == i]
+                if ch and rng.random() < 0.85:
+                    am[b, i] = tok[b, ch[int(rng.integers(0, len(ch)))]]
+        for argmax in (r_am, am):
+            g = fc.fc_accept(dev(tok), dev(par), dev(nn), dev(argmax), 12)
+            r = orc.accept(tok, par, nn, argmax, 12)
+            assert np.array_equal(g["acc_len"].cpu().numpy(), r["acc_len"])
+            assert np.array_equal(g["path"].cpu().numpy(), r["path"])
+            assert np.array_equal(host_u32(g["bonus"]), r["bonus"])
+    check_no_error(fc)
+
+
+def test_kv_append_copy(fc, orc):
+    rng = synth.rng_for(61)
+    B, n_pad, Hkv, D, cap, stride = 16, 64, 8, 128, 300, 200
+    tok, par, nn = _random_trees(rng, B, n_pad)
+    plen, rtok = synth.argmax_draws(rng, B, n_pad, 32256)
+    am = orc.synth_argmax(tok, par, nn, plen, rtok, 32256)
+    acc = orc.accept(tok, par, nn, am, 12)
+    kt = synth.randn_bf16((B, Hkv, n_pad, D), 7, "cuda")
+    vt = synth.randn_bf16((B, Hkv, n_pad, D), 8, "cuda")
+    kc = synth.randn_bf16((B, Hkv, cap, D), 9, "cuda")
+    vc = synth.randn_bf16((B, Hkv, cap, D), 10, "cuda")
+    kvl = rng.integers(0, 280, B).astype(np.int32)
+    kvl[0] = cap - 1  # overflows unless nothing is accepted
+    ctx = rng.integers(0, 32256, (B, stride)).astype(np.uint32)
+    cl = rng.integers(1, 180, B).astype(np.int32)
+    kc_h, vc_h, ctx_h = bits_bf16(kc).copy(), bits_bf16(vc).copy(), ctx.copy()
+    gacc = dict(acc_len=dev(acc["acc_len"]), path=dev(acc["path"]), bonus=dev(acc["bonus"]))
+    kvo, clo, root = (torch.empty(B, dtype=torch.int32, device="cuda") for _ in range(3))
+    g_ctx = dev(ctx)
+    fc.fc_kv_append(gacc, dev(tok), kt, vt, kc, vc, dev(kvl), kvo, g_ctx, dev(cl), clo, root)
+    status = fc.fc_get_error()
+    ok = kvl + acc["acc_len"] + 1 <= cap
+    assert status == ("FC_OK" if ok.all() else "FC_ERR_CAPACITY")
+    sel = np.nonzero(ok)[0]
+    kc_s, vc_s, ctx_s = kc_h[sel].copy(), vc_h[sel].copy(), ctx_h[sel].copy()
+    r_kvo, r_clo, r_root = orc.kv_append(acc["path"][sel], acc["acc_len"][sel], acc["bonus"][sel], tok[sel],
+                                         bits_bf16(kt)[sel], bits_bf16(vt)[sel], kc_s, vc_s, kvl[sel], ctx_s, cl[sel])
+    assert np.array_equal(bits_bf16(kc)[sel], kc_s) and np.array_equal(bits_bf16(vc)[sel], vc_s)
+    assert np.array_equal(host_u32(g_ctx)[sel], ctx_s)
+    assert np.array_equal(kvo.cpu().numpy()[sel], r_kvo) and np.array_equal(clo.cpu().numpy()[sel], r_clo)
+    assert np.array_equal(host_u32(root)[sel], r_root)
+    bad = np.nonzero(~ok)[0]
+    assert np.array_equal(kvo.cpu().numpy()[bad], kvl[bad])
+
+
+# ------------------------------------------------------------- step loop
+def test_step_loop_matches_oracle(fc, orc):
+    """c5-shaped loop on small corpora: two sources, replay cache with a
+    seeded 50% hit pattern, 128-node trees, 24 steps."""
+    from paper_2502_17139_gb300.step import StepLoop
+    rng = synth.rng_for(70)
+    Tr, _ = synth.make_corpus(rng, 200_000, 1.3, synth.VOCAB, n_grams=2000, len_range=(8, 64))
+    Tc, _ = synth.make_corpus(rng, 1_000_000, 1.1, synth.VOCAB)
+    B, steps, n_pad, H, Hkv, D = 8, 24, 128, 8, 2, 128
+    stride = 128 + steps * 12
+    ctx, cl, _ = synth.make_contexts(rng, B, 128, 16, [Tr, Tc, None], [0.5, 0.25, 0.25], 1.1, ctx_stride=stride)
+    hits = synth.cache_hit_pattern(rng, steps, B)
+    plen = np.stack([synth.argmax_draws(rng, B, n_pad)[0] for _ in range(steps)])
+    rtok = np.stack([synth.argmax_draws(rng, B, n_pad)[1] for _ in range(steps)])
+    p = dict(n_max=16, n_min=2, top_k=64, draft_len=10, max_occ=4096, node_budget=128, n_pad=n_pad)
+    hist, r_ctx, r_cl, r_kvl = orc.step_loop([Tr, Tc], ctx, cl, steps, p, hits, plen, rtok, [1, 1], synth.VOCAB,
+                                             kv_len0=np.full(B, 100, np.int32))
+    srcs = [fc.fc_datastore_build(dev(Tr), synth.VOCAB), fc.fc_datastore_build(dev(Tc), synth.VOCAB)]
+    loop = StepLoop(srcs, ctx, cl, fc.params(16, 2, 64, 10, 4096), 128, n_pad, [1, 1], H, Hkv, D,
+                    kv_cap=100 + steps * 12, kv_len0=100, vocab=synth.VOCAB)
+    q = synth.randn_bf16((B, n_pad, H, D), 1, "cuda")
+    kt = synth.randn_bf16((B, Hkv, n_pad, D), 2, "cuda")
+    vt = synth.randn_bf16((B, Hkv, n_pad, D), 3, "cuda")
+    for st in range(steps):
+        loop.step(q, kt, vt, dev(hits[st]), dev(plen[st]), dev(rtok[st]))
+        assert np.array_equal(loop.acc["acc_len"].cpu().numpy(), hist["acc_len"][st]), st
+        assert np.array_equal(host_u32(loop.acc["bonus"]), hist["bonus"][st]), st
+        assert np.array_equal(loop.tree["n_nodes"].cpu().numpy(), hist["n_nodes"][st]), st
+    check_no_error(fc)
+    assert np.array_equal(host_u32(loop.ctx), r_ctx)
+    assert np.array_equal(loop.ctx_len_now.cpu().numpy(), r_cl)
+    assert np.array_equal(loop.kv_len_now.cpu().numpy(), r_kvl)
+    assert sum(h.sum() for h in hist["hit"]) > 0  # the replay cache served some queries
