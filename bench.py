@@ -1,0 +1,596 @@
+#!/usr/bin/env python
+"""Benchmark of the retrieve-and-verify step (FastCoder, arXiv 2502.17139).
+
+Workload (the full step loop): a general datastore of 100M tokens (Zipf 1.1)
+and a project datastore of 5M tokens (Zipf 1.3 + 20,000 planted 8-64-token
+repeats), vocab 32256; 32 sequences whose 128-token contexts end with spans
+copied from the project store (50%), the general store (25%) or pure Zipf
+draws (25%); retrieval n 16 -> 2, top-64 drafts of 10 tokens per source,
+alpha = beta = 1; draft trees of at most 128 nodes; tree attention with 32
+query / 8 KV heads, head dim 128, KV cache 16384 tokens (bf16); greedy
+acceptance against the synthetic target model; cache append; a context-keyed
+replay cache with a seeded 50% hit pattern.  One step = one pass of all of
+that over the batch.  The datastores are built once (offline, Section IV-A)
+before timing; their build time is reported separately.
+
+Arms:
+  default           the CUDA path (libfastcoder.so through its C ABI)
+  --impl reference  the CPU oracle, timed on the host cores on a bounded
+                    sample of the same workload per step, scaled to a step
+
+Under torchrun every rank runs an independent batch of 32 sequences on its
+own GPU against replicated datastores (no data-path collective); the timed
+region is bracketed by barriers and the slowest rank's time is used.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "retrieve+verify steps/s"
+UNIT = "steps/s"
+WORKLOAD = ("full step loop: two-source datastore 100M (Zipf 1.1) + 5M (Zipf 1.3, 20k planted repeats) tokens, "
+            "vocab 32256, batch 32, ctx 128, n 16->2, top-64 x 10 tokens per source, tree <=128 nodes, "
+            "GQA 32/8 heads, head_dim 128, KV 16384 bf16, 50% replay-cache hits")
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=256)
+    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--scale", type=float, default=1.0,
+                    help="shrink the datastores and KV length (tests only; 1.0 is the benchmark workload)")
+    ap.add_argument("--batch", type=int, default=32)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--mode", choices=["step", "attn"], default="step",
+                    help="step: the full step loop (the benchmark); attn: tree attention alone on the step loop's "
+                         "attention shape with seeded trees (a small profiling / sweep target)")
+    ap.add_argument("--nodes", type=int, default=128, help="attn mode: tree nodes per sequence")
+    ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
+    ap.add_argument("--traffic-bytes", type=float, default=None,
+                    help="ncu dram read+write bytes of one tree-attention launch of this workload")
+    return ap.parse_args(argv)
+
+
+# ---------------------------------------------------------------- helpers
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm=float(p["hbm_gbs"]), tc_burst=float(p["bf16_tflops"]),
+                    tc_sustained=float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), source="measured")
+    return dict(hbm=6800.0, tc_burst=1900.0, tc_sustained=1700.0, source="fallback")
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples during the timed region."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={gpu_index}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.file,
+                                         stderr=subprocess.DEVNULL)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.file.flush()
+        with open(self.file.name) as f:
+            rows = [r.strip().split(", ") for r in f if r.strip()]
+        os.unlink(self.file.name)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+            except (ValueError, IndexError):
+                continue
+            for k, nm in enumerate(names):
+                if len(r) > 5 + k and r[5 + k].strip().lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup(gpus: int):
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return rank, ws, local
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, ws: int) -> float:
+    if ws == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# --------------------------------------------------------------- workload
+def workload_spec(scale: float, batch: int):
+    import paper_2502_17139_gb300.synth as synth
+    cfg = dict(synth.CONFIGS[5])
+    c2 = synth.CONFIGS[2]
+    corpora = [synth.scaled_corpus_spec(s, scale) for s in c2["corpus"]]
+    kv = max(256, int(cfg["kv_len"] * scale))
+    return cfg, corpora, kv, batch
+
+
+def make_inputs(scale: float, batch: int, rank: int, steps_total: int):
+    """Host-side seeded inputs; rank r gets its own batch of sequences."""
+    import paper_2502_17139_gb300.synth as synth
+    cfg, corp_specs, kv0, B = workload_spec(scale, batch)
+    rng = synth.rng_for(2)                      # datastores: identical on every rank
+    corpora = []
+    for spec in corp_specs:
+        T, _ = synth.build_corpus(rng, spec)
+        corpora.append(T)
+    Tr, Tc = corpora                            # project store first (alpha), general second (beta)
+    rr = synth.rng_for(5, 1 + rank)             # per-rank sequences
+    n_pad, d = cfg["n_pad"], cfg["draft_len"]
+    stride = cfg["ctx_len"] + (steps_total + 1) * (d + 1)
+    ctx, cl, _ = synth.make_contexts(rr, B, cfg["ctx_len"], cfg["n_copy"], [Tr, Tc, None], cfg["probs"], 1.1,
+                                     ctx_stride=stride)
+    hits = synth.cache_hit_pattern(rr, steps_total, B, cfg["hit_p"])
+    plen = np.empty((steps_total, B), np.int32)
+    rtok = np.empty((steps_total, B, n_pad), np.uint32)
+    for s in range(steps_total):
+        plen[s], rtok[s] = synth.argmax_draws(rr, B, n_pad)
+    return dict(cfg=cfg, corpora=corpora, kv0=kv0, B=B, ctx=ctx, cl=cl, hits=hits, plen=plen, rtok=rtok,
+                stride=stride, seed=1000 * (rank + 1))
+
+
+# ---------------------------------------------------------------- our arm
+def run_ours(args, rank, ws, local):
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    import paper_2502_17139_gb300.synth as synth
+    from paper_2502_17139_gb300.step import StepLoop
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    K, W = args.steps, args.warmup
+    total = K + W + 1
+    inp = make_inputs(args.scale, args.batch, rank, total)
+    cfg, B = inp["cfg"], inp["B"]
+    H, Hkv, D, n_pad, d = cfg["H"], cfg["Hkv"], cfg["D"], cfg["n_pad"], cfg["draft_len"]
+    kv0 = inp["kv0"]
+    cap = kv0 + total * (d + 1) + 8
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).to(dev)
+
+    t0 = time.perf_counter()
+    sources = [fc.fc_datastore_build(to_dev(T), synth.VOCAB) for T in inp["corpora"]]
+    torch.cuda.synchronize()
+    build_s = time.perf_counter() - t0
+    build_tokens = sum(len(T) for T in inp["corpora"])
+
+    p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], d, 4096)
+    kc = torch.empty((B, Hkv, cap, D), dtype=torch.bfloat16, device=dev)
+    vc = torch.empty_like(kc)
+    g = torch.Generator(device=dev)
+    g.manual_seed(inp["seed"])
+    kc[:, :, :kv0].normal_(generator=g)
+    vc[:, :, :kv0].normal_(generator=g)
+    kc[:, :, kv0:].zero_()
+    vc[:, :, kv0:].zero_()
+
+    def new_loop():
+        return StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, [1, 1], H, Hkv, D, cap, kv0,
+                        synth.VOCAB, cache_capacity=1 << 14, device=dev, k_cache=kc, v_cache=vc)
+
+    # device-resident per-step inputs (a pool of distinct activations, cycled)
+    P = min(16, K + W)
+    q_pool = torch.randn((P, B, n_pad, H, D), generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    kt_pool = torch.randn((P, B, Hkv, n_pad, D), generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    vt_pool = torch.randn((P, B, Hkv, n_pad, D), generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    hits_d, plen_d, rtok_d = to_dev(inp["hits"]), to_dev(inp["plen"]), to_dev(inp["rtok"])
+
+    loop = new_loop()
+    no_hit = torch.zeros(B, dtype=torch.int32, device=dev)
+    for s in range(W + K):  # recording pass: fills the replay cache along the trajectory
+        loop.step(q_pool[s % P], kt_pool[s % P], vt_pool[s % P], no_hit, plen_d[s], rtok_d[s])
+    loop.reset()
+    stream = torch.cuda.current_stream()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    ev_ret = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+
+    def do_step(s, timed_idx=None):
+        j = s % P
+        if timed_idx is not None:
+            loop.step(q_pool[j], kt_pool[j], vt_pool[j], hits_d[s], plen_d[s], rtok_d[s],
+                      events=dict(attn=ev[timed_idx], retrieve=ev_ret[timed_idx]))
+        else:
+            loop.step(q_pool[j], kt_pool[j], vt_pool[j], hits_d[s], plen_d[s], rtok_d[s])
+
+    for s in range(W):
+        do_step(s)
+    assert fc.fc_get_error() == "FC_OK"
+    barrier(ws)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(K):
+        do_step(W + i, i)
+    end.record(stream)
+    torch.cuda.synchronize()
+    clock_rec = clocks.stop()
+    barrier(ws)
+    t_ms = start.elapsed_time(end)
+    status = fc.fc_get_error()
+    assert status == "FC_OK", status
+    t_max = max_over_ranks(t_ms, ws)
+    attn_ms = [a.elapsed_time(b) for a, b in ev]
+    ret_ms = [a.elapsed_time(b) for a, b in ev_ret]
+
+    # replay the same (deterministic) trajectory untimed to count the
+    # attention work of every timed launch
+    flops, bytes_, nodes_hist, acc_hist, hits_used = replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K)
+
+    peaks = load_peaks()
+    per_launch = []
+    for i in range(K):
+        t = attn_ms[i] * 1e-3
+        per_launch.append((flops[i], bytes_[i], t))
+    tot_f = sum(f for f, _, _ in per_launch)
+    tot_b = sum(b for _, b, _ in per_launch)
+    tot_t = sum(t for _, _, t in per_launch)
+    t_tc = tot_f / (peaks["tc_sustained"] * 1e12)
+    t_hbm = tot_b / (peaks["hbm"] * 1e9)
+    if t_tc >= t_hbm:
+        roof = dict(bound="tensor", achieved=tot_f / tot_t / 1e12, peak=peaks["tc_sustained"], unit="TFLOP/s")
+    else:
+        roof = dict(bound="hbm", achieved=tot_b / tot_t / 1e9, peak=peaks["hbm"], unit="GB/s")
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = args.traffic_bytes
+    roof["peak_source"] = peaks["source"] + (" sustained bf16" if roof["bound"] == "tensor" else " hbm copy")
+    roof["kernel"] = "k_tree_attn"
+    roof["mean_launch_us"] = 1e6 * tot_t / K
+    roof["algorithmic_flops_per_launch"] = tot_f / K
+    roof["algorithmic_bytes_per_launch"] = tot_b / K
+    roof["other_bound_frac"] = (t_hbm if roof["bound"] == "tensor" else t_tc) / tot_t
+
+    out = {
+        "metric": METRIC, "value": ws * K / (t_max * 1e-3), "unit": UNIT, "n_gpus": ws, "steps": K, "warmup": W,
+        "ms_per_step": t_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16 attention (fp32 accumulate) + u32 retrieval", "data": "synthetic",
+        "config": {"workload": WORKLOAD if args.scale == 1.0 else WORKLOAD + f" (scaled x{args.scale})",
+                   "batch_per_gpu": B, "global_batch": B * ws, "kv_len0": kv0, "n_pad": n_pad,
+                   "l2": "inputs larger than L2 (KV cache %.1f GB per GPU)" % (2 * kc.numel() * 2 / 1e9),
+                   "parallelism": f"replicas x{ws}"},
+        "roofline": roof,
+        "gpu_launches": 8 * K,
+        "clocks": clock_rec,
+        "stages_ms_per_step": {"tree_attn": statistics.mean(attn_ms), "retrieve": statistics.mean(ret_ms),
+                               "all": t_ms / K},
+        "queries_per_s": ws * B * K / (t_max * 1e-3),
+        "retrievals_per_s": ws * (2 * (B * K - hits_used)) / (t_max * 1e-3),
+        "tree_attn_tflops": tot_f / tot_t / 1e12,
+        "avg_acceptance_length": float(np.mean([a.mean() + 1 for a in acc_hist])),
+        "avg_tree_nodes": float(np.mean([n.mean() for n in nodes_hist])),
+        "datastore_build": {"tokens": build_tokens, "seconds": build_s, "tokens_per_s": build_tokens / build_s},
+    }
+    if not args.no_e2e:
+        loop.reset()
+        out["e2e"] = run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws)
+    if not args.no_cpu_baseline and rank == 0 and ws == 1:
+        out["cpu_baseline"] = cpu_baseline(inp, cfg, kv0, out["avg_tree_nodes"], B)
+    return out
+
+
+def replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K):
+    """Re-run the loop (untimed, fresh state) and count per-launch attention
+    work: FLOPs over unmasked (q, k) pairs and algorithmic HBM bytes."""
+    import torch
+
+    import paper_2502_17139_gb300.synth as synth
+    from paper_2502_17139_gb300.step import StepLoop
+    B, H, Hkv, D, n_pad = inp["B"], cfg["H"], cfg["Hkv"], cfg["D"], cfg["n_pad"]
+    kc = torch.zeros((B, Hkv, cap, D), dtype=torch.bfloat16, device=dev)
+    loop = StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, [1, 1], H, Hkv, D, cap, kv0,
+                    synth.VOCAB, cache_capacity=1 << 14, device=dev, k_cache=kc, v_cache=kc)
+    q = torch.zeros((B, n_pad, H, D), dtype=torch.bfloat16, device=dev)
+    kt = torch.zeros((B, Hkv, n_pad, D), dtype=torch.bfloat16, device=dev)
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).to(dev)
+    flops, bytes_, nodes_hist, acc_hist = [], [], [], []
+    hits_used = 0
+    zero = to_dev(np.zeros(B, np.int32))
+    for s in range(W + K):  # recording pass, as in the timed run
+        loop.step(q, kt, kt, zero, to_dev(inp["plen"][s]), to_dev(inp["rtok"][s]), attention=False)
+    loop.reset()
+    for s in range(W + K):
+        kvl = loop.kv_len_now.cpu().numpy().astype(np.int64)
+        loop.step(q, kt, kt, to_dev(inp["hits"][s]), to_dev(inp["plen"][s]), to_dev(inp["rtok"][s]), attention=False)
+        if s < W:
+            continue
+        nn = loop.tree["n_nodes"].cpu().numpy().astype(np.int64)
+        dep = loop.tree["depth"].cpu().numpy().astype(np.int64)
+        pairs = sum(H * (nn[b] * kvl[b] + int((dep[b, :nn[b]] + 1).sum())) for b in range(B))
+        flops.append(4.0 * D * pairs)
+        by = 0
+        for b in range(B):
+            by += 2 * Hkv * kvl[b] * D * 2          # K and V cache rows
+            by += 2 * Hkv * nn[b] * D * 2           # tree K and V
+            by += 2 * nn[b] * H * D * 2             # Q in, O out
+            by += nn[b] * (n_pad // 64) * 8         # mask rows
+        bytes_.append(float(by))
+        nodes_hist.append(nn)
+        acc_hist.append(loop.acc["acc_len"].cpu().numpy())
+        hits_used += int(loop.skip.sum().item())
+    return flops, bytes_, nodes_hist, acc_hist, hits_used
+
+
+def run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws):
+    """Same metric through the public API with host buffers: each step copies
+    its inputs host->device from pinned memory and reads its result
+    (accepted lengths and bonus tokens) back to the host."""
+    import torch
+    R = min(4, P)
+    hq = [q_pool[j].cpu().pin_memory() for j in range(R)]
+    hk = [kt_pool[j].cpu().pin_memory() for j in range(R)]
+    hv = [vt_pool[j].cpu().pin_memory() for j in range(R)]
+    B = inp["B"]
+    hh = torch.from_numpy(inp["hits"].view(np.int32)).pin_memory()
+    hp = torch.from_numpy(inp["plen"].view(np.int32)).pin_memory()
+    hr = torch.from_numpy(np.ascontiguousarray(inp["rtok"]).view(np.int32)).pin_memory()
+    dq, dk, dv = torch.empty_like(q_pool[0]), torch.empty_like(kt_pool[0]), torch.empty_like(vt_pool[0])
+    dh = torch.empty(B, dtype=torch.int32, device=dev)
+    dp = torch.empty(B, dtype=torch.int32, device=dev)
+    dr = torch.empty(inp["rtok"].shape[1:], dtype=torch.int32, device=dev)
+    res = torch.empty((2, B), dtype=torch.int32).pin_memory()
+    stream = torch.cuda.current_stream()
+
+    def one(s):
+        j = s % R
+        dq.copy_(hq[j], non_blocking=True)
+        dk.copy_(hk[j], non_blocking=True)
+        dv.copy_(hv[j], non_blocking=True)
+        dh.copy_(hh[s], non_blocking=True)
+        dp.copy_(hp[s], non_blocking=True)
+        dr.copy_(hr[s], non_blocking=True)
+        loop.step(dq, dk, dv, dh, dp, dr)
+        res[0].copy_(loop.acc["acc_len"], non_blocking=True)
+        res[1].copy_(loop.acc["bonus"], non_blocking=True)
+
+    for i in range(W):
+        one(i)
+    torch.cuda.synchronize()
+    barrier(ws)
+    t0 = time.perf_counter()
+    for i in range(K):
+        one(W + i)
+    torch.cuda.synchronize()
+    t = max_over_ranks(time.perf_counter() - t0, ws)
+    h2d = dq.numel() * 2 + dk.numel() * 2 + dv.numel() * 2 + 4 * (2 * B + dr.numel())
+    return {"value": ws * K / t, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(res.numel() * 4)}
+
+
+# ------------------------------------------------------------ CPU oracle
+def cpu_baseline(inp, cfg, kv0, avg_nodes, B, budget_s=20.0):
+    """The oracle (as it stands) on a bounded sample of one step, scaled to a
+    full step: retrieval for a few queries on both sources, a tree and an
+    acceptance walk for them, and attention for one (sequence, kv head)
+    group; each stage's time per unit times the units of one full step."""
+    import paper_2502_17139_gb300.synth as synth
+    from oracle import oracle as orc
+    rng = synth.rng_for(5, 777)
+    nq = 2
+    qs = np.arange(nq)
+    t0 = time.perf_counter()
+    res = [orc.retrieve(T, inp["ctx"][qs], inp["cl"][qs], cfg["n_max"], cfg["n_min"], cfg["top_k"],
+                        cfg["draft_len"], 4096) for T in inp["corpora"]]
+    t_ret = (time.perf_counter() - t0) / (nq * len(inp["corpora"]))
+    root = inp["ctx"][qs, inp["cl"][qs] - 1]
+    t0 = time.perf_counter()
+    tr = orc.build_tree(res, [1, 1], root, np.full(nq, kv0, np.int32), cfg["node_budget"], cfg["n_pad"])
+    am = orc.synth_argmax(tr["tok"], tr["parent"], tr["n_nodes"], inp["plen"][0][qs], inp["rtok"][0][qs], synth.VOCAB)
+    orc.accept(tr["tok"], tr["parent"], tr["n_nodes"], am, cfg["draft_len"] + 2)
+    t_tree = (time.perf_counter() - t0) / nq
+    # attention for one (sequence, kv group): G query heads x its nodes
+    H, Hkv, D, n_pad = cfg["H"], cfg["Hkv"], cfg["D"], cfg["n_pad"]
+    G = H // Hkv
+    n = max(1, int(round(avg_nodes)))
+    bits = lambda a: (a.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    q = bits(rng.standard_normal((1, n_pad, H, D), dtype=np.float32))
+    kc = bits(rng.standard_normal((1, Hkv, kv0, D), dtype=np.float32))
+    kt = bits(rng.standard_normal((1, Hkv, n_pad, D), dtype=np.float32))
+    par = np.full((1, n_pad), -1, np.int32)
+    _, pp = synth.random_tree(rng, n, 10, 4, 1000)
+    par[0, :n] = pp
+    mask = orc.tree_mask(par, np.array([n], np.int32), np.array([kv0], np.int32), n_pad)["mask"]
+    rows = np.array([(0, i, h) for i in range(n) for h in range(G)], np.int32)
+    t0 = time.perf_counter()
+    orc.tree_attn(q, kc, kc, np.array([kv0], np.int32), kt, kt, mask, np.array([n], np.int32), rows=rows)
+    t_attn_group = time.perf_counter() - t0
+    hit_rate = float(inp["hits"].mean())  # the replay cache holds every key of the trajectory
+    step_s = (t_ret * B * len(inp["corpora"]) * (1 - hit_rate) + t_tree * B + t_attn_group * B * Hkv)
+    cores = orc.hardware_threads()
+    return {"value": 1.0 / step_s, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": (f"{nq} queries x {len(inp['corpora'])} sources retrieval (linear corpus scans), their trees "
+                       f"and acceptance, attention for 1 (sequence, kv-head) group ({G} heads x {n} nodes x "
+                       f"{kv0} keys, fp64); per-unit times scaled to one step of {B} sequences"),
+            "stage_seconds_per_unit": {"retrieve": t_ret, "tree_accept": t_tree, "attn_group": t_attn_group}}
+
+
+def run_reference(args, rank, ws):
+    """CPU oracle arm: each step runs one sequence of the batch through the
+    whole oracle pipeline (its retrievals, tree, acceptance, append and the
+    attention of one kv-head group) and is scaled to a full step."""
+    if rank != 0:
+        return None
+    import paper_2502_17139_gb300.synth as synth
+    from oracle import oracle as orc
+    K, W = args.steps, args.warmup
+    inp = make_inputs(args.scale, args.batch, 0, K + W + 1)
+    cfg, B, kv0 = inp["cfg"], inp["B"], inp["kv0"]
+    H, Hkv, D, n_pad, d = cfg["H"], cfg["Hkv"], cfg["D"], cfg["n_pad"], cfg["draft_len"]
+    G = H // Hkv
+    rng = synth.rng_for(5, 999)
+    bits = lambda a: (a.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    kc = bits(rng.standard_normal((1, 1, kv0 + (K + W + 1) * (d + 1), D), dtype=np.float32))
+    kt = bits(rng.standard_normal((1, 1, n_pad, D), dtype=np.float32))
+    q = bits(rng.standard_normal((1, n_pad, G, D), dtype=np.float32))
+    ctx = inp["ctx"].copy()
+    cl = inp["cl"].copy()
+    times, attn_times = [], []
+    for s in range(K + W):
+        b = s % B
+        # the GPU arm replays a recorded trajectory, so every step that asks
+        # for a cache hit gets one: such a step's retrieval is not counted
+        tr0 = time.perf_counter()
+        res = [orc.retrieve(T, ctx[b:b + 1], cl[b:b + 1], cfg["n_max"], cfg["n_min"], cfg["top_k"], d, 4096)
+               for T in inp["corpora"]]
+        t_ret = 0.0 if inp["hits"][s, b] else time.perf_counter() - tr0
+        t0 = time.perf_counter()
+        root = ctx[b:b + 1, cl[b] - 1]
+        tr = orc.build_tree(res, [1, 1], root, np.array([kv0], np.int32), cfg["node_budget"], n_pad)
+        n = int(tr["n_nodes"][0])
+        rows = np.array([(0, i, h) for i in range(n) for h in range(G)], np.int32)
+        ta = time.perf_counter()
+        orc.tree_attn(q, kc, kc, np.array([kv0], np.int32), kt, kt, tr["mask"], tr["n_nodes"], rows=rows)
+        ta = time.perf_counter() - ta
+        am = orc.synth_argmax(tr["tok"], tr["parent"], tr["n_nodes"], inp["plen"][s][b:b + 1], inp["rtok"][s][b:b + 1],
+                              synth.VOCAB)
+        ac = orc.accept(tr["tok"], tr["parent"], tr["n_nodes"], am, d + 2)
+        a = int(ac["acc_len"][0])
+        for t in range(a):
+            ctx[b, cl[b] + t] = tr["tok"][0, ac["path"][0, t + 1]]
+        ctx[b, cl[b] + a] = ac["bonus"][0]
+        cl[b] += a + 1
+        dt = time.perf_counter() - t0
+        if s >= W:
+            times.append(dt - ta + t_ret)
+            attn_times.append(ta)
+    # one sampled step = one sequence with one of its Hkv attention groups;
+    # a full step is B sequences with all Hkv groups each
+    step_s = B * (statistics.mean(times) + Hkv * statistics.mean(attn_times))
+    cores = orc.hardware_threads()
+    value = 1.0 / step_s
+    return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": K, "warmup": W,
+            "ms_per_step": 1e3 * step_s, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64 attention + u32 retrieval", "data": "synthetic", "impl": "reference",
+            "config": {"workload": WORKLOAD, "batch_per_gpu": B, "kv_len0": kv0, "parallelism": "cpu oracle"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": (f"each step: 1 of {B} sequences through the oracle pipeline (retrieval on "
+                                        f"both sources, not counted when the replayed cache serves it, tree, 1 of {Hkv} kv-head "
+                                        f"attention groups, acceptance, append); attention scaled x{Hkv}, the "
+                                        f"sequence scaled x{B}")},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def run_attn(args, rank, ws, local):
+    """Tree attention alone: B sequences x 8 KV heads x 32 query heads,
+    head dim 128, KV length --kv, seeded random trees of --nodes nodes."""
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    import paper_2502_17139_gb300.synth as synth
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    B, H, Hkv, D, n_pad, L = args.batch, 32, 8, 128, 128, args.kv
+    rng = synth.rng_for(5, 500 + rank)
+    par = np.full((B, n_pad), -1, np.int32)
+    for b in range(B):
+        _, pp = synth.random_tree(rng, args.nodes, 10, 4, synth.VOCAB)
+        par[b, :args.nodes] = pp
+    nn = np.full(B, args.nodes, np.int32)
+    kvl = np.full(B, L, np.int32)
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    m = fc.fc_tree_mask(to_dev(par), to_dev(nn), to_dev(kvl))
+    g = torch.Generator(device=dev)
+    g.manual_seed(7 + rank)
+    rnd = lambda *shape: torch.randn(*shape, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    q, kc, vc = rnd(B, n_pad, H, D), rnd(B, Hkv, L, D), rnd(B, Hkv, L, D)
+    kt, vt = rnd(B, Hkv, n_pad, D), rnd(B, Hkv, n_pad, D)
+    out = torch.empty_like(q)
+    args_d = (q, kc, vc, to_dev(kvl), kt, vt, m["mask"], to_dev(nn))
+    for _ in range(args.warmup):
+        fc.fc_tree_attn(*args_d, out=out)
+    assert fc.fc_get_error() == "FC_OK"
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    barrier(ws)
+    torch.cuda.synchronize()
+    for e0, e1 in evs:
+        e0.record()
+        fc.fc_tree_attn(*args_d, out=out)
+        e1.record()
+    torch.cuda.synchronize()
+    ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in evs)
+    dep = m["depth"].cpu().numpy()
+    pairs = sum(H * (args.nodes * L + int((dep[b, :args.nodes] + 1).sum())) for b in range(B))
+    flops = 4.0 * D * pairs
+    bytes_ = B * (2 * Hkv * L * D * 2 + 2 * Hkv * args.nodes * D * 2 + 2 * args.nodes * H * D * 2)
+    peaks = load_peaks()
+    return {"metric": "tree-attn TFLOP/s", "value": flops / (ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+            "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "config": {"workload": f"tree attention B={B} H=32 Hkv=8 D=128 KV={L} nodes={args.nodes}"},
+            "frac_tensor_sustained": flops / (ms * 1e-3) / 1e12 / peaks["tc_sustained"],
+            "frac_hbm": bytes_ / (ms * 1e-3) / 1e9 / peaks["hbm"], "flops": flops, "bytes": bytes_}
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    rank, ws, local = dist_setup(args.gpus)
+    if args.impl == "reference":
+        out = run_reference(args, rank, ws)
+    elif args.mode == "attn":
+        out = run_attn(args, rank, ws, local)
+    else:
+        out = run_ours(args, rank, ws, local)
+    if rank == 0 and out is not None:
+        print(json.dumps(out))
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

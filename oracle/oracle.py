@@ -240,7 +240,7 @@ def cache_key(ctx_row: np.ndarray, ctx_len: int, n_max: int) -> bytes:
 
 
 def step_loop(corpora, ctx, ctx_len, steps, p, hits, plen, rtok, src_weight, vocab, kv_len0=None,
-              nthreads: int = 0, on_step=None):
+              nthreads: int = 0, on_step=None, cache=None):
     """Integer trajectory of the step loop (retrieve -> tree -> accept ->
     append) with the context-keyed replay cache.  Attention does not steer the
     trajectory (acceptance reads the target model's predictions only), so it
@@ -248,13 +248,15 @@ def step_loop(corpora, ctx, ctx_len, steps, p, hits, plen, rtok, src_weight, voc
 
     p: dict with n_max, n_min, top_k, draft_len, max_occ, node_budget, n_pad.
     hits[step, b]: want-hit flags; plen[step, b], rtok[step, b, n_pad]: the
-    synthetic target model's draws.  Returns per-step lists of acc_len and
-    bonus plus the final context."""
+    synthetic target model's draws.  ``cache`` (a dict) persists the replay
+    cache across calls: a first pass records retrieval results, a second pass
+    over the same trajectory replays them where hits[step, b] asks for it.
+    Returns per-step lists of acc_len and bonus plus the final context."""
     ctx = np.array(ctx, dtype=np.uint32, copy=True)
     ctx_len = np.array(ctx_len, dtype=np.int32, copy=True)
     B = ctx.shape[0]
     kv_len = np.zeros(B, np.int32) if kv_len0 is None else np.array(kv_len0, np.int32)
-    cache = {}
+    cache = {} if cache is None else cache
     hist = dict(acc_len=[], bonus=[], n_nodes=[], hit=[])
     S = len(corpora)
     for st in range(steps):

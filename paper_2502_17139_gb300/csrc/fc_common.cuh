@@ -81,18 +81,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 }
 
 // Bounded wait: returns false (and raises *abort) when the barrier phase has
-// not completed within limit_ns, or when another thread of the CTA already
-// gave up.
+// not completed within limit_cycles SM clock cycles, or when another thread
+// of the CTA already gave up.  The clock and the abort flag are only looked
+// at every 64 polls: the fast path is a single try_wait.
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort,
-                                                  uint64_t limit_ns) {
+                                                  uint64_t limit_cycles) {
   if (mbar_try_wait(bar, parity)) return true;
-  uint64_t t0 = globaltimer_ns();
-  for (;;) {
+  const long long t0 = clock64();
+  for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (*abort) return false;
-    if (globaltimer_ns() - t0 > limit_ns) {
-      *abort = 1;
-      return false;
+    if ((it & 63u) == 0) {
+      if (*abort) return false;
+      if ((uint64_t)(clock64() - t0) > limit_cycles) {
+        *abort = 1;
+        return false;
+      }
     }
   }
 }

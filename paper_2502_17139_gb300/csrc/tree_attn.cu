@@ -42,8 +42,12 @@ constexpr uint32_t OFF_P = OFF_V + 2 * TILE_BYTES;
 constexpr uint32_t OFF_BAR = OFF_P + TILE_BYTES;
 constexpr uint32_t SMEM_BYTES = OFF_BAR + 256 + 1024;  // + alignment slack
 constexpr uint32_t TMEM_COLS = 512;
-constexpr uint64_t WAIT_NS = 2000000000ull;   // 2 s
-constexpr uint64_t DRAIN_NS = 200000000ull;   // 0.2 s
+constexpr uint64_t WAIT_NS = 4000000000ull;   // ~2 s of SM clock cycles
+constexpr uint64_t DRAIN_NS = 400000000ull;   // ~0.2 s
+// Lazy rescaling: O and l are rescaled only when a row's running maximum
+// (base-2 logits) grows by more than this; until then probabilities may reach
+// 2^RESCALE_THRESHOLD, harmless in bf16/fp32.
+constexpr float RESCALE_THRESHOLD = 8.f;
 
 // barrier slots (8 bytes each) after OFF_BAR
 enum { B_KFULL = 0, B_VFULL = 2, B_EMPTY = 4, B_SFULL = 6, B_PFULL = 8, B_ODONE = 9, N_BARS = 10 };
@@ -252,24 +256,35 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
       tc_wait_ld();
       const bool tree = (j == nblk - 1);
       const int nv = tree ? BN : min(BN, kvl - j * BN);
-      float mx = -INFINITY;
+      if (tree || nv < BN) {  // block-uniform: only the ragged tail and the tree block are masked
 #pragma unroll
-      for (int c = 0; c < BN; ++c) {
-        const bool keep = tree ? (((c < 64 ? m0 >> c : m1 >> (c - 64)) & 1ull) != 0) : (c < nv);
-        const float x = keep ? __uint_as_float(sreg[c]) * a.scale_log2 : -INFINITY;
-        sreg[c] = __float_as_uint(x);
-        mx = fmaxf(mx, x);
+        for (int c = 0; c < BN; ++c) {
+          const bool keep = tree ? (((c < 64 ? m0 >> c : m1 >> (c - 64)) & 1ull) != 0) : (c < nv);
+          if (!keep) sreg[c] = __float_as_uint(-INFINITY);
+        }
       }
-      const float m_new = fmaxf(m_run, mx);
+      // raw row maximum with independent partial maxima (scale > 0 commutes with max)
+      float pm[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < BN; ++c) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sreg[c]));
+      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * a.scale_log2;
+      // lazy rescale: keep the old reference unless the maximum grew a lot
+      const float m_new = (mx > m_run + RESCALE_THRESHOLD) ? mx : m_run;
       const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
       const float alpha = fast_exp2(m_run - m_use);
-      float sum = 0.f;
+      float ps[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) ps[u] = 0.f;
 #pragma unroll
       for (int c = 0; c < BN; ++c) {
-        const float p = fast_exp2(__uint_as_float(sreg[c]) - m_use);
+        const float p = fast_exp2(fmaf(__uint_as_float(sreg[c]), a.scale_log2, -m_use));
         sreg[c] = __float_as_uint(p);
-        sum += p;
+        ps[c & 7] += p;
       }
+      const float sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
       l_run = l_run * alpha + sum;
       m_run = m_new;
       if (j >= 1) {  // PV(j-1) must be done before O is rescaled and P overwritten

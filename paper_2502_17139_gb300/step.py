@@ -35,6 +35,7 @@ class StepLoop:
         cl = self.ctx_len[0].long()
         self.root = self.ctx.gather(1, (cl - 1).clamp(min=0).view(B, 1)).view(B).contiguous()
         self.cur = 0
+        self._init = (self.ctx.clone(), self.ctx_len[0].clone(), self.kv_len[0].clone(), self.root.clone())
         S = len(sources)
         self.res = fc.retrieve_outputs(S, B, p, device)
         self.skip = torch.zeros(B, dtype=torch.int32, device=device)
@@ -50,21 +51,32 @@ class StepLoop:
         self.attn_out = torch.empty((B, n_pad, H, D), dtype=torch.bfloat16, device=device)
         self.cache = fc.RetrievalCache(cache_capacity, S, p, device) if cache_capacity else None
 
-    def step(self, q, k_tree, v_tree, want_hit, plen, rtok, attention=True):
+    def step(self, q, k_tree, v_tree, want_hit, plen, rtok, attention=True, events=None):
         """Enqueue one step.  q [B, Np, H, D], k_tree/v_tree [B, Hkv, Np, D]
-        (bf16); want_hit [B], plen [B], rtok [B, Np] (int32)."""
+        (bf16); want_hit [B], plen [B], rtok [B, Np] (int32).  ``events``
+        optionally maps "retrieve" / "attn" to (start, end) CUDA events
+        recorded around those stages on the current stream."""
         c, n = self.cur, 1 - self.cur
+        ev = events or {}
+        if "retrieve" in ev:
+            ev["retrieve"][0].record()
         if self.cache is not None:
             fc.fc_rcache_lookup(self.cache, self.ctx, self.ctx_len[c], want_hit, self.skip, self.res)
             fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, skip=self.skip, out=self.res)
             fc.fc_rcache_insert(self.cache, self.ctx, self.ctx_len[c], self.skip, self.res)
         else:
             fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, out=self.res)
+        if "retrieve" in ev:
+            ev["retrieve"][1].record()
         fc.fc_build_tree(self.res, self.src_weight, self.root, self.kv_len[c], self.node_budget, self.n_pad,
                          out=self.tree)
         if attention:
+            if "attn" in ev:
+                ev["attn"][0].record()
             fc.fc_tree_attn(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree, self.tree["mask"],
                             self.tree["n_nodes"], out=self.attn_out)
+            if "attn" in ev:
+                ev["attn"][1].record()
         fc.fc_synth_argmax(self.tree["tok"], self.tree["parent"], self.tree["n_nodes"], plen, rtok, self.vocab,
                            out=self.argmax)
         fc.fc_accept(self.tree["tok"], self.tree["parent"], self.tree["n_nodes"], self.argmax, self.path_cap,
@@ -72,6 +84,16 @@ class StepLoop:
         fc.fc_kv_append(self.acc, self.tree["tok"], k_tree, v_tree, self.k_cache, self.v_cache, self.kv_len[c],
                         self.kv_len[n], self.ctx, self.ctx_len[c], self.ctx_len[n], self.root)
         self.cur = n
+
+    def reset(self):
+        """Back to the initial contexts and cache lengths; the retrieval cache
+        keeps its entries (a replay of the same trajectory then hits it)."""
+        ctx0, cl0, kv0, root0 = self._init
+        self.ctx.copy_(ctx0)
+        self.ctx_len[0].copy_(cl0)
+        self.kv_len[0].copy_(kv0)
+        self.root.copy_(root0)
+        self.cur = 0
 
     @property
     def kv_len_now(self):

@@ -220,13 +220,15 @@ def random_tree(rng: np.random.Generator, n_nodes: int, depth_max: int = 10,
 # random numbers consumed by the synthetic target model
 # --------------------------------------------------------------------------
 def argmax_draws(rng: np.random.Generator, batch: int, n_pad: int, vocab: int = VOCAB,
-                 plen_max: int = 8):
+                 plen_max: int = 8, s: float = 1.1):
     """Per sequence: an agreeing-prefix length ~ U{0..plen_max} and one random
-    token per tree slot.  The synthetic target model follows the tree's first
+    token per tree slot, drawn from the corpus' Zipf(s) law (the target model
+    emits code-like tokens, so the next context suffix can match the
+    datastore again).  The synthetic target model follows the tree's first
     branch for that many steps and otherwise predicts the slot's random token
     (moved past any child token of the node)."""
     plen = rng.integers(0, plen_max + 1, size=batch).astype(np.int32)
-    rtok = rng.integers(0, vocab, size=(batch, n_pad)).astype(np.uint32)
+    rtok = zipf_tokens(rng, batch * n_pad, s, vocab).reshape(batch, n_pad)
     return plen, rtok
 
 
