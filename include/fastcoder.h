@@ -99,6 +99,28 @@ fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n_tokens, uint32
                              uint32_t* d_sa, uint32_t* d_bucket, void* d_ws, size_t ws_bytes,
                              fc_stream s, fc_datastore* out);
 
+/*
+ * The same build for callers that cannot allocate device memory.  The paper
+ * has no counterpart: this is a deployment variant of fc_datastore_build.
+ * Some callers cannot call cudaMalloc, e.g. a serving process whose memory
+ * manager reserves all free device memory for its KV cache up front, or a
+ * plugin inside an application that owns every device allocation.  This
+ * entry point allocates nothing: its scratch space is a fixed 30 MiB array
+ * compiled into the library, which every GPU that loads the library holds
+ * until the process exits.  The caller still passes the corpus, d_sa and
+ * d_bucket.
+ *   n_tokens must be <= FC_NOALLOC_MAX_TOKENS; larger corpora return
+ *   FC_ERR_CAPACITY (use fc_datastore_build with a workspace instead).
+ * The first call on a device looks up the array's device address on that
+ * device; make it before any stream capture.  All calls share the array:
+ * calls whose work overlaps on the GPU (other streams, other host threads)
+ * race on it and must not be made.  Synchronous, like fc_datastore_build.
+ */
+#define FC_NOALLOC_MAX_TOKENS 1048576ull
+fc_status fc_datastore_build_noalloc(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t vocab,
+                                     uint32_t* d_sa, uint32_t* d_bucket, fc_stream s,
+                                     fc_datastore* out);
+
 /* ------------------------------------------------------------------------
  * Retrieval (Section III-A; Section IV-C, Algorithm 1 par_search; Section
  * V-C: n_max = 16).

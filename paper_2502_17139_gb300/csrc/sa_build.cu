@@ -11,6 +11,8 @@
 // re-ranks by scanning "key differs from its predecessor" flags.  The loop
 // stops when every rank is distinct.  All passes stream the arrays once
 // (HBM-bound); only the rank gather rank[i + h] is random.
+#include <mutex>
+
 #include "fc_common.cuh"
 
 FC_DEFINE_ERROR_WORD(sa)
@@ -369,4 +371,57 @@ extern "C" fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n, ui
     out->vocab = vocab;
   }
   return FC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Datastore build without any allocation: the scratch space lives in a
+// fixed array compiled into this library instead of caller memory.
+//
+// Some callers cannot call cudaMalloc: a serving process whose memory manager
+// reserves all free device memory for its KV cache up front (a later
+// cudaMalloc fails, or fragments that reservation), or a plugin inside a host
+// application that owns every device allocation.  They can still build a
+// small datastore (a repository's own project store) here.
+//
+// The array is a file-scope __device__ variable, so every GPU that loads the
+// library holds it until the process exits.  Host code cannot pass the
+// variable's name to a kernel (on the host it is only a stand-in, not a device
+// address): the device address is looked up once per device, with that
+// device current, by cudaGetSymbolAddress on the first call made on it.  That
+// first call should come before any stream capture starts.  Every call shares
+// the one array and leaves its contents behind; the build clears what must
+// start at zero itself.  Calls whose work overlaps on the GPU (two streams,
+// two host threads) race on the array and must not be made.
+// ---------------------------------------------------------------------------
+namespace {
+constexpr size_t kNoAllocScratchBytes = (size_t)30 << 20;  // 30 MiB
+static __device__ __align__(256) unsigned char g_sa_scratch[kNoAllocScratchBytes];
+
+constexpr int kMaxDevices = 64;
+void* g_scratch_ptr[kMaxDevices] = {nullptr};
+std::mutex g_scratch_mu;
+
+fc_status scratch_for_current_device(void** out) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FC_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_sa_scratch) != cudaSuccess || !p) return FC_ERR_CUDA;
+    g_scratch_ptr[dev] = p;
+  }
+  *out = g_scratch_ptr[dev];
+  return FC_OK;
+}
+}  // namespace
+
+extern "C" fc_status fc_datastore_build_noalloc(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t vocab,
+                                                uint32_t* d_sa, uint32_t* d_bucket, fc_stream stream,
+                                                fc_datastore* out) {
+  if (n_tokens > FC_NOALLOC_MAX_TOKENS) return FC_ERR_CAPACITY;
+  if (n_tokens > 0 && fc_datastore_build_workspace(n_tokens, vocab) > kNoAllocScratchBytes) return FC_ERR_CAPACITY;
+  void* ws = nullptr;
+  fc_status st = scratch_for_current_device(&ws);
+  if (st != FC_OK) return st;
+  return fc_datastore_build(d_tokens, n_tokens, vocab, d_sa, d_bucket, ws, kNoAllocScratchBytes, stream, out);
 }

@@ -45,6 +45,7 @@ class fc_retrieve_params(C.Structure):
 
 
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
+           "fc_datastore_build_noalloc",
            "fc_retrieve", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_accept", "fc_kv_append", "fc_synth_argmax"]
 
@@ -61,6 +62,7 @@ def _load():
         "fc_get_error": (C.c_int, [vp]),
         "fc_datastore_build_workspace": (sz, [u64, u32]),
         "fc_datastore_build": (C.c_int, [vp, u64, u32, vp, vp, vp, sz, vp, C.POINTER(fc_datastore)]),
+        "fc_datastore_build_noalloc": (C.c_int, [vp, u64, u32, vp, vp, vp, C.POINTER(fc_datastore)]),
         "fc_retrieve": (C.c_int, [C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp, fc_retrieve_params,
                                   vp, vp, vp, vp, vp, vp]),
         "fc_rcache_bytes": (sz, [i32, i32, fc_retrieve_params]),
@@ -154,6 +156,24 @@ def fc_datastore_build(tokens: torch.Tensor, vocab: int, workspace: torch.Tensor
         raise ValueError("workspace too small")
     _check("fc_datastore_build", LIB.fc_datastore_build(_ptr(tokens), n, vocab, _ptr(sa), _ptr(bucket), _ptr(ws),
                                                         ws.numel(), _stream(), None))
+    return Datastore(tokens, sa, bucket, vocab)
+
+
+NOALLOC_MAX_TOKENS = 1 << 20
+
+
+def fc_datastore_build_noalloc(tokens: torch.Tensor, vocab: int, sa: torch.Tensor,
+                               bucket: torch.Tensor) -> Datastore:
+    """The datastore build for callers that cannot allocate device memory:
+    scratch comes from a fixed array inside the library, and the outputs go
+    to the caller's sa [N] and bucket [vocab + 1] (int32).  N is at most
+    NOALLOC_MAX_TOKENS.  This wrapper allocates nothing either."""
+    _need(tokens, torch.int32, "tokens")
+    n = tokens.numel()
+    _need(sa, torch.int32, "sa", (n,))
+    _need(bucket, torch.int32, "bucket", (vocab + 1,))
+    _check("fc_datastore_build_noalloc", LIB.fc_datastore_build_noalloc(_ptr(tokens), n, vocab, _ptr(sa),
+                                                                        _ptr(bucket), _stream(), None))
     return Datastore(tokens, sa, bucket, vocab)
 
 
