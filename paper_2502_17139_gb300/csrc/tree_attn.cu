@@ -2,21 +2,26 @@
 // Every draft-tree node attends to the whole KV cache of its sequence and to
 // its tree ancestors (and itself), so one forward verifies every draft.
 //
-// GB300 design (one CTA = 128 query rows of one (sequence, kv head) group):
-//   * GQA packing: the rows of a CTA are (query head in group, tree node)
-//     pairs over the group's H/Hkv heads and the sequence's n_nodes nodes,
-//     packed densely, so small trees do not waste tensor-core rows and every
-//     K/V tile loaded serves all heads that share it.
-//   * K/V tiles of 128 keys x 128 dims stream from HBM with TMA (128-byte
-//     swizzle, two stages); the tree's own K/V form one last tile.
-//   * S = Q K^T and O += P V run on the 5th-generation tensor cores
-//     (tcgen05.mma, bf16 in, fp32 accumulate) with S (double-buffered) and O
-//     in tensor memory; one thread issues the MMAs.
-//   * a 128-thread softmax warpgroup owns one row per thread: it reads S
-//     from tensor memory, applies the tree mask bits (and the ragged cache
-//     tail) in registers, runs the online softmax in base 2, rescales O in
-//     tensor memory, and writes P (bf16) to shared memory for the PV MMA.
-//   * QK of block j+1 and PV of block j-1 overlap the softmax of block j.
+// GB300 design.  One CTA serves one (sequence, kv head) group and up to 256
+// query rows of it, as two 128-row tiles A and B:
+//   * GQA packing: rows are (query head in group, tree node) pairs over the
+//     group's H/Hkv heads and the sequence's n_nodes nodes, packed densely, so
+//     small trees waste no tensor-core rows and each K/V tile loaded from HBM
+//     serves every query head that shares it (and both tiles).
+//   * K/V tiles of 128 keys x 128 dims stream in with TMA (128-byte swizzle,
+//     two K stages and two V stages, released separately: a K stage as soon
+//     as both tiles' QK MMAs are done, a V stage after both PV MMAs).  The
+//     tree's own K/V form one last tile.
+//   * tcgen05.mma (bf16 in, fp32 accumulate): S_X = Q_X K^T into tensor
+//     memory; the softmax writes P_X (bf16) over the first half of S_X in
+//     tensor memory, and O_X += P_X V takes P_X straight from tensor memory
+//     (A operand) with V as an MN-major shared-memory operand.  One thread
+//     issues every MMA, in the order PV_X(j-1) -> QK_X(j) per tile, so S_X is
+//     never overwritten before PV_X has read P_X from it.
+//   * two softmax warpgroups, one per tile, one row per thread: tile A's
+//     softmax runs while the tensor cores do tile B's PV and QK, and the
+//     other way round.  The tree mask and the ragged cache tail are applied in
+//     registers; the online softmax is in base 2 with lazy rescaling of O.
 //   * every mbarrier wait is bounded; a wait that runs out raises
 //     FC_ERR_TIMEOUT, the CTA drains its in-flight copies and MMAs (bounded
 //     again), frees its tensor memory and returns.
@@ -29,28 +34,38 @@ FC_DEFINE_ERROR_WORD(attn)
 
 namespace {
 
-constexpr int TA_THREADS = 256;
-constexpr int BM = 128;  // query rows per CTA
-constexpr int BN = 128;  // keys per block
-constexpr int HD = 128;  // head dim
+constexpr int TA_THREADS = 384;  // warp 0 TMA, warp 1 MMA, warps 4-7 softmax A, warps 8-11 softmax B
+constexpr int BM = 128;          // query rows per tile
+constexpr int TILES = 2;         // tiles per CTA
+constexpr int BN = 128;          // keys per block
+constexpr int HD = 128;          // head dim
 constexpr uint32_t HALF_BYTES = BN * 64 * 2;  // one 64-dim half of a 128-row tile
 constexpr uint32_t TILE_BYTES = 2 * HALF_BYTES;
-constexpr uint32_t OFF_Q = 0;
-constexpr uint32_t OFF_K = OFF_Q + TILE_BYTES;
-constexpr uint32_t OFF_V = OFF_K + 2 * TILE_BYTES;
-constexpr uint32_t OFF_P = OFF_V + 2 * TILE_BYTES;
-constexpr uint32_t OFF_BAR = OFF_P + TILE_BYTES;
-constexpr uint32_t SMEM_BYTES = OFF_BAR + 256 + 1024;  // + alignment slack
-constexpr uint32_t TMEM_COLS = 512;
-constexpr uint64_t WAIT_NS = 4000000000ull;   // ~2 s of SM clock cycles
-constexpr uint64_t DRAIN_NS = 400000000ull;   // ~0.2 s
+constexpr uint32_t OFF_Q = 0;                              // Q_A, Q_B
+constexpr uint32_t OFF_K = OFF_Q + TILES * TILE_BYTES;     // 2 stages
+constexpr uint32_t OFF_V = OFF_K + 2 * TILE_BYTES;         // 2 stages
+constexpr uint32_t OFF_BAR = OFF_V + 2 * TILE_BYTES;
+constexpr uint32_t SMEM_BYTES = OFF_BAR + 256 + 1024;      // + alignment slack
+constexpr uint32_t TMEM_COLS = 512;                        // S_A, S_B, O_A, O_B (128 columns each)
+constexpr uint64_t WAIT_CYCLES = 4000000000ull;            // ~2 s
+constexpr uint64_t DRAIN_CYCLES = 400000000ull;            // ~0.2 s
 // Lazy rescaling: O and l are rescaled only when a row's running maximum
 // (base-2 logits) grows by more than this; until then probabilities may reach
 // 2^RESCALE_THRESHOLD, harmless in bf16/fp32.
 constexpr float RESCALE_THRESHOLD = 8.f;
 
-// barrier slots (8 bytes each) after OFF_BAR
-enum { B_KFULL = 0, B_VFULL = 2, B_EMPTY = 4, B_SFULL = 6, B_PFULL = 8, B_ODONE = 9, N_BARS = 10 };
+// barrier slots (8 bytes each)
+enum {
+  B_KFULL = 0,   // [2] K tile landed
+  B_VFULL = 2,   // [2] V tile landed
+  B_KEMPTY = 4,  // [2] K tile consumed by both QK MMAs
+  B_VEMPTY = 6,  // [2] V tile consumed by both PV MMAs
+  B_SFULL = 8,   // [2 tiles] S_X ready
+  B_PFULL = 10,  // [2 tiles] P_X written (128 arrivals)
+  B_ODONE = 12,  // [2 tiles] last PV_X done
+  B_DRAIN = 14,  // MMA drain on abort
+  N_BARS = 15
+};
 
 struct AttnArgs {
   const __nv_bfloat16* q;
@@ -58,7 +73,7 @@ struct AttnArgs {
   const uint64_t* mask;
   const int32_t* n_nodes;
   __nv_bfloat16* out;
-  int B, n_pad, H, Hkv, G, kv_cap, tiles;
+  int B, n_pad, H, Hkv, G, kv_cap, ctas;  // ctas = CTAs per group
   float scale_log2;
 };
 
@@ -68,6 +83,11 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+// All 32 lanes wait; the result is warp-uniform.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
+  return __all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar, parity, abort, WAIT_CYCLES));
+}
+
 __global__ void __launch_bounds__(TA_THREADS, 1)
     k_tree_attn(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                 const __grid_constant__ CUtensorMap tm_kt, const __grid_constant__ CUtensorMap tm_vt, AttnArgs a) {
@@ -75,30 +95,32 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int bg = blockIdx.x / a.tiles, t = blockIdx.x - bg * a.tiles;
+  const int bg = blockIdx.x / a.ctas, c = blockIdx.x - bg * a.ctas;
   const int b = bg / a.Hkv, g = bg - b * a.Hkv;
   const int nn_raw = a.n_nodes[b], kvl = a.kv_len[b];
   const bool bad = nn_raw < 1 || nn_raw > a.n_pad || kvl < 0 || kvl > a.kv_cap;
   const int nn = bad ? 0 : nn_raw;
-  if (bad && t == 0 && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+  if (bad && c == 0 && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
 
-  // Zero the padding rows (nodes >= n_nodes) of this group; tiles share the work.
+  // Zero the padding rows (nodes >= n_nodes) of this group; the group's CTAs share the work.
   {
-    const int pad_rows = a.G * (a.n_pad - nn);
-    for (int e = t * TA_THREADS + tid; e < pad_rows * (HD / 8); e += a.tiles * TA_THREADS) {
+    const int pad = a.n_pad - nn;
+    for (int e = c * TA_THREADS + tid; e < a.G * pad * (HD / 8); e += a.ctas * TA_THREADS) {
       int r = e / (HD / 8), ch = e - r * (HD / 8);
-      int hh = r / (a.n_pad - nn), i = nn + (r - hh * (a.n_pad - nn));
-      uint4* dst = reinterpret_cast<uint4*>(a.out + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD) + ch;
-      *dst = make_uint4(0, 0, 0, 0);
+      int hh = r / pad, i = nn + (r - hh * pad);
+      reinterpret_cast<uint4*>(a.out + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD)[ch] =
+          make_uint4(0, 0, 0, 0);
     }
   }
   const int rows_total = a.G * nn;
-  const int row0 = t * BM;
+  const int row0 = c * (TILES * BM);
   if (row0 >= rows_total) return;
+  const bool has_b = row0 + BM < rows_total;
 
-  unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  unsigned char* smem =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const uint32_t sbase = smem_u32(smem);
-  const uint32_t sQ = sbase + OFF_Q, sK = sbase + OFF_K, sV = sbase + OFF_V, sP = sbase + OFF_P;
+  const uint32_t sQ = sbase + OFF_Q, sK = sbase + OFF_K, sV = sbase + OFF_V;
   const uint32_t bar0 = sbase + OFF_BAR;
   auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
 
@@ -107,7 +129,7 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
 
   if (tid == 0) {
     s_abort = 0;
-    for (int i = 0; i < N_BARS; ++i) mbar_init(bar(i), i == B_PFULL ? 128u : 1u);
+    for (int i = 0; i < N_BARS; ++i) mbar_init(bar(i), (i == B_PFULL || i == B_PFULL + 1) ? 128u : 1u);
     fence_mbar_init();
     prefetch_tmap(&tm_kc);
     prefetch_tmap(&tm_vc);
@@ -118,23 +140,24 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     tmem_alloc(smem_u32(&s_tmem), TMEM_COLS);
     tmem_relinquish();
   }
-  // Q tile: rows (head in group, node) packed densely, 128-byte swizzled, K-major.
-  for (int c = tid; c < BM * 16; c += TA_THREADS) {
-    const int r = c >> 4, ch = c & 15, half = ch >> 3, gran = ch & 7;
+  // Q tiles: rows (head in group, node) packed densely, 128-byte swizzled, K-major.
+  for (int e = tid; e < TILES * BM * 16; e += TA_THREADS) {
+    const int r = e >> 4, ch = e & 15, half = ch >> 3, gran = ch & 7;
+    const int tile = r / BM, rt = r - tile * BM;
     const int rg = row0 + r;
     uint4 v = make_uint4(0, 0, 0, 0);
     if (rg < rows_total) {
       const int hh = rg / nn, i = rg - hh * nn;
-      v = *(reinterpret_cast<const uint4*>(a.q + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD) + ch);
+      v = reinterpret_cast<const uint4*>(a.q + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD)[ch];
     }
-    *reinterpret_cast<uint4*>(smem + OFF_Q + half * HALF_BYTES + r * 128 + ((gran ^ (r & 7)) << 4)) = v;
+    *reinterpret_cast<uint4*>(smem + OFF_Q + tile * TILE_BYTES + half * HALF_BYTES + rt * 128 +
+                              ((gran ^ (rt & 7)) << 4)) = v;
   }
   fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = s_tmem;
-  const uint32_t tS0 = tmem, tO = tmem + 256;
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
@@ -142,31 +165,30 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
       int issued = 0;
       for (int j = 0; j < nblk; ++j) {
         const int st = j & 1;
-        if (j >= 2 && !mbar_wait_bounded(bar(B_EMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_NS)) break;
+        const bool tree = j >= nblk_c;
+        const uint32_t bytes = tree ? (uint32_t)a.n_pad * 64 * 2 * 2 : TILE_BYTES;
+        const CUtensorMap* mk = tree ? &tm_kt : &tm_kc;
+        const CUtensorMap* mv = tree ? &tm_vt : &tm_vc;
+        const int y = tree ? 0 : j * BN;
+        if (j >= 2 && !mbar_wait_bounded(bar(B_KEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) break;
         const uint32_t dK = sK + st * TILE_BYTES, dV = sV + st * TILE_BYTES;
-        if (j < nblk_c) {
-          mbar_expect_tx(bar(B_KFULL + st), TILE_BYTES);
-          tma_load_3d(dK, &tm_kc, 0, j * BN, bg, bar(B_KFULL + st));
-          tma_load_3d(dK + HALF_BYTES, &tm_kc, 64, j * BN, bg, bar(B_KFULL + st));
-          mbar_expect_tx(bar(B_VFULL + st), TILE_BYTES);
-          tma_load_3d(dV, &tm_vc, 0, j * BN, bg, bar(B_VFULL + st));
-          tma_load_3d(dV + HALF_BYTES, &tm_vc, 64, j * BN, bg, bar(B_VFULL + st));
-        } else {
-          const uint32_t bytes = (uint32_t)a.n_pad * 64 * 2 * 2;
-          mbar_expect_tx(bar(B_KFULL + st), bytes);
-          tma_load_3d(dK, &tm_kt, 0, 0, bg, bar(B_KFULL + st));
-          tma_load_3d(dK + HALF_BYTES, &tm_kt, 64, 0, bg, bar(B_KFULL + st));
-          mbar_expect_tx(bar(B_VFULL + st), bytes);
-          tma_load_3d(dV, &tm_vt, 0, 0, bg, bar(B_VFULL + st));
-          tma_load_3d(dV + HALF_BYTES, &tm_vt, 64, 0, bg, bar(B_VFULL + st));
+        mbar_expect_tx(bar(B_KFULL + st), bytes);
+        tma_load_3d(dK, mk, 0, y, bg, bar(B_KFULL + st));
+        tma_load_3d(dK + HALF_BYTES, mk, 64, y, bg, bar(B_KFULL + st));
+        if (j >= 2 && !mbar_wait_bounded(bar(B_VEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) {
+          issued = j + 1;  // the K copy of this block is in flight
+          break;
         }
+        mbar_expect_tx(bar(B_VFULL + st), bytes);
+        tma_load_3d(dV, mv, 0, y, bg, bar(B_VFULL + st));
+        tma_load_3d(dV + HALF_BYTES, mv, 64, y, bg, bar(B_VFULL + st));
         issued = j + 1;
       }
       if (s_abort) {  // let the copies already issued land before the CTA exits
         volatile int dummy = 0;
         for (int j = max(0, issued - 2); j < issued; ++j) {
-          mbar_wait_bounded(bar(B_KFULL + (j & 1)), (j >> 1) & 1, &dummy, DRAIN_NS);
-          mbar_wait_bounded(bar(B_VFULL + (j & 1)), (j >> 1) & 1, &dummy, DRAIN_NS);
+          mbar_wait_bounded(bar(B_KFULL + (j & 1)), (j >> 1) & 1, &dummy, DRAIN_CYCLES);
+          mbar_wait_bounded(bar(B_VFULL + (j & 1)), (j >> 1) & 1, &dummy, DRAIN_CYCLES);
         }
       }
     }
@@ -175,170 +197,201 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     // ---------------- MMA issuer (+ ragged V rows zeroed by the warp) -------
     constexpr uint32_t IDESC_QK = idesc_bf16_f32(BM, BN, 0);
     constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, HD, 1);
-    int last_qk = -1, last_pv = -1;
-    for (int j = 0; j <= nblk; ++j) {
-      if (j < nblk) {
-        const int st = j & 1;
-        if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar(B_KFULL + st), (j >> 1) & 1, &s_abort, WAIT_NS))) break;
-        if (lane == 0) {
-          tc_fence_after();
-          const uint32_t kb = sK + st * TILE_BYTES;
+    const int ntiles = has_b ? 2 : 1;
+    auto issue_qk = [&](int j, int x) {
+      const uint32_t kb = sK + (j & 1) * TILE_BYTES, qb = sQ + x * TILE_BYTES;
 #pragma unroll
-          for (int kk = 0; kk < HD / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * HALF_BYTES + (kk & 3) * 32;
-            tc_mma_f16(tS0 + st * 128, smem_desc_sw128(sQ + off, 16, 1024), smem_desc_sw128(kb + off, 16, 1024),
-                       IDESC_QK, kk > 0);
-          }
-          tc_commit(bar(B_SFULL + st));
-        }
-        last_qk = j;
-        __syncwarp();
+      for (int kk = 0; kk < HD / 16; ++kk) {
+        const uint32_t off = (kk >> 2) * HALF_BYTES + (kk & 3) * 32;
+        tc_mma_f16(tmem + x * 128, smem_desc_sw128(qb + off, 16, 1024), smem_desc_sw128(kb + off, 16, 1024),
+                   IDESC_QK, kk > 0);
       }
-      if (j >= 1) {
-        const int jj = j - 1, st = jj & 1;
-        if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar(B_PFULL), jj & 1, &s_abort, WAIT_NS))) break;
-        if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar(B_VFULL + st), (jj >> 1) & 1, &s_abort, WAIT_NS))) break;
-        const int nv = (jj < nblk_c) ? min(BN, kvl - jj * BN) : nn;
+      tc_commit(bar(B_SFULL + x));
+    };
+    auto issue_pv = [&](int jj, int x) {
+      const uint32_t vb = sV + (jj & 1) * TILE_BYTES;
+#pragma unroll
+      for (int kk = 0; kk < BN / 16; ++kk)  // P_X: 8 packed columns per 16 keys
+        tc_mma_f16_tmem_a(tmem + 256 + x * 128, tmem + x * 128 + kk * 8,
+                          smem_desc_sw128(vb + kk * 2048, HALF_BYTES, 1024), IDESC_PV, (jj > 0 || kk > 0));
+    };
+    bool ok = warp_wait(bar(B_KFULL), 0, &s_abort);
+    if (ok) {
+      if (lane == 0) {
+        tc_fence_after();
+        for (int x = 0; x < ntiles; ++x) issue_qk(0, x);
+        tc_commit(bar(B_KEMPTY));
+      }
+      __syncwarp();
+    }
+    for (int j = 1; ok && j <= nblk; ++j) {
+      const int jj = j - 1, st = jj & 1;
+      if (!(ok = warp_wait(bar(B_VFULL + st), (jj >> 1) & 1, &s_abort))) break;
+      const int nv = (jj < nblk_c) ? min(BN, kvl - jj * BN) : nn;
+      if (nv < BN) {  // never let garbage (possibly NaN) rows meet a zero probability
         unsigned char* vt = smem + OFF_V + st * TILE_BYTES;
-        if (nv < BN) {  // never let garbage (possibly NaN) rows meet a zero probability
-          for (int e = lane; e < (BN - nv) * 16; e += 32) {
-            const int r = nv + (e >> 4), ch = e & 15;
-            *reinterpret_cast<uint4*>(vt + (ch >> 3) * HALF_BYTES + r * 128 + (ch & 7) * 16) = make_uint4(0, 0, 0, 0);
-          }
-          fence_proxy_async_smem();
+        for (int e = lane; e < (BN - nv) * 16; e += 32) {
+          const int r = nv + (e >> 4), ch = e & 15;
+          *reinterpret_cast<uint4*>(vt + (ch >> 3) * HALF_BYTES + r * 128 + (ch & 7) * 16) = make_uint4(0, 0, 0, 0);
         }
-        __syncwarp();
+        fence_proxy_async_smem();
+      }
+      __syncwarp();
+      for (int x = 0; ok && x < ntiles; ++x) {
+        if (!(ok = warp_wait(bar(B_PFULL + x), jj & 1, &s_abort))) break;
         if (lane == 0) {
           tc_fence_after();
-          const uint32_t vb = sV + st * TILE_BYTES;
-#pragma unroll
-          for (int kk = 0; kk < BN / 16; ++kk) {
-            const uint32_t aoff = (kk >> 2) * HALF_BYTES + (kk & 3) * 32;
-            tc_mma_f16(tO, smem_desc_sw128(sP + aoff, 16, 1024), smem_desc_sw128(vb + kk * 2048, HALF_BYTES, 1024),
-                       IDESC_PV, (jj > 0 || kk > 0));
-          }
-          tc_commit(bar(B_ODONE));
-          tc_commit(bar(B_EMPTY + st));
+          issue_pv(jj, x);
         }
-        last_pv = jj;
         __syncwarp();
+        if (j < nblk) {
+          if (x == 0 && !(ok = warp_wait(bar(B_KFULL + (j & 1)), (j >> 1) & 1, &s_abort))) break;
+          if (lane == 0) issue_qk(j, x);
+          __syncwarp();
+        }
       }
+      if (!ok) break;
+      if (lane == 0) {
+        if (j < nblk) tc_commit(bar(B_KEMPTY + (j & 1)));
+        tc_commit(bar(B_VEMPTY + st));
+        if (j == nblk)
+          for (int x = 0; x < ntiles; ++x) tc_commit(bar(B_ODONE + x));
+      }
+      __syncwarp();
     }
     if (s_abort) {  // let issued MMAs retire before the tensor memory is freed
+      if (lane == 0) tc_commit(bar(B_DRAIN));
+      __syncwarp();
       volatile int dummy = 0;
-      if (last_qk >= 0) mbar_wait_bounded(bar(B_SFULL + (last_qk & 1)), (last_qk >> 1) & 1, &dummy, DRAIN_NS);
-      if (last_pv >= 0) mbar_wait_bounded(bar(B_ODONE), last_pv & 1, &dummy, DRAIN_NS);
+      mbar_wait_bounded(bar(B_DRAIN), 0, &dummy, DRAIN_CYCLES);
     }
   } else if (warp >= 4) {
-    // ---------------- softmax warpgroup: thread = row ----------------
-    const int q4 = warp - 4;
-    const int r = q4 * 32 + lane;
-    const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
-    const int rg = row0 + r;
-    const bool row_ok = rg < rows_total;
-    const int hh = row_ok ? rg / nn : 0, i = row_ok ? rg - hh * nn : 0;
-    const int nw = a.n_pad / 64;
-    const uint64_t* mrow = a.mask + ((size_t)b * a.n_pad + i) * nw;
-    const uint64_t m0 = mrow[0], m1 = (nw > 1) ? mrow[1] : 0ull;
-    float m_run = -INFINITY, l_run = 0.f;
-    bool ok = true;
-    uint32_t sreg[BN];
-    for (int j = 0; j < nblk && ok; ++j) {
-      const int st = j & 1;
-      if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar(B_SFULL + st), (j >> 1) & 1, &s_abort, WAIT_NS))) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-#pragma unroll
-      for (int c = 0; c < BN / 32; ++c)
-        tmem_ld32(tS0 + st * 128 + c * 32 + lane_off, *reinterpret_cast<uint32_t(*)[32]>(&sreg[c * 32]));
-      tc_wait_ld();
-      const bool tree = (j == nblk - 1);
-      const int nv = tree ? BN : min(BN, kvl - j * BN);
-      if (tree || nv < BN) {  // block-uniform: only the ragged tail and the tree block are masked
-#pragma unroll
-        for (int c = 0; c < BN; ++c) {
-          const bool keep = tree ? (((c < 64 ? m0 >> c : m1 >> (c - 64)) & 1ull) != 0) : (c < nv);
-          if (!keep) sreg[c] = __float_as_uint(-INFINITY);
-        }
-      }
-      // raw row maximum with independent partial maxima (scale > 0 commutes with max)
-      float pm[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
-#pragma unroll
-      for (int c = 0; c < BN; ++c) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sreg[c]));
-      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * a.scale_log2;
-      // lazy rescale: keep the old reference unless the maximum grew a lot
-      const float m_new = (mx > m_run + RESCALE_THRESHOLD) ? mx : m_run;
-      const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
-      const float alpha = fast_exp2(m_run - m_use);
-      float ps[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) ps[u] = 0.f;
-#pragma unroll
-      for (int c = 0; c < BN; ++c) {
-        const float p = fast_exp2(fmaf(__uint_as_float(sreg[c]), a.scale_log2, -m_use));
-        sreg[c] = __float_as_uint(p);
-        ps[c & 7] += p;
-      }
-      const float sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
-      l_run = l_run * alpha + sum;
-      m_run = m_new;
-      if (j >= 1) {  // PV(j-1) must be done before O is rescaled and P overwritten
-        if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar(B_ODONE), (j - 1) & 1, &s_abort, WAIT_NS))) {
-          ok = false;
-          break;
-        }
+    // ---------------- softmax warpgroups: tile x, thread = row ----------------
+    const int x = (warp - 4) >> 2;  // 0: warps 4-7, 1: warps 8-11
+    const int q4 = warp & 3;        // TMEM lane quarter of this warp
+    if (x == 0 || has_b) {
+      const int r = q4 * 32 + lane;
+      const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+      const uint32_t tS = tmem + x * 128 + lane_off, tO = tmem + 256 + x * 128 + lane_off;
+      const int rg = row0 + x * BM + r;
+      const bool row_ok = rg < rows_total;
+      const int hh = row_ok ? rg / nn : 0, i = row_ok ? rg - hh * nn : 0;
+      const int nw = a.n_pad / 64;
+      const uint64_t* mrow = a.mask + ((size_t)b * a.n_pad + i) * nw;
+      const uint64_t m0 = mrow[0], m1 = (nw > 1) ? mrow[1] : 0ull;
+      float m_run = -INFINITY, l_run = 0.f;
+      bool ok = true;
+      for (int j = 0; j < nblk; ++j) {
+        if (!(ok = warp_wait(bar(B_SFULL + x), j & 1, &s_abort))) break;
         tc_fence_after();
-        // tcgen05.ld/st are warp-collective: the branch must be warp-uniform.
-        if (__any_sync(0xFFFFFFFFu, alpha != 1.f)) {
+        const bool tree = (j == nblk - 1);
+        const int nv = tree ? BN : min(BN, kvl - j * BN);
+        const bool masked = tree || nv < BN;  // block-uniform
+        // keep-bits of 32-column chunk q: the tree mask row, or the ragged cache tail
+        auto keep_bits = [&](int q) -> uint32_t {
+          if (tree) return (uint32_t)((q < 2 ? m0 : m1) >> (32 * (q & 1)));
+          const int lo = nv - 32 * q;
+          return lo >= 32 ? 0xFFFFFFFFu : (lo <= 0 ? 0u : ((1u << lo) - 1u));
+        };
+        // masked scores become -inf (exp2 turns them into exact zeros)
+        auto apply_mask = [&](int h2, uint32_t (&s0)[32], uint32_t (&s1)[32]) {
+          const uint32_t k0 = keep_bits(2 * h2), k1 = keep_bits(2 * h2 + 1);
 #pragma unroll
-          for (int c = 0; c < HD / 32; ++c) {
+          for (int cc = 0; cc < 32; ++cc) {
+            if (!(k0 & (1u << cc))) s0[cc] = __float_as_uint(-INFINITY);
+            if (!(k1 & (1u << cc))) s1[cc] = __float_as_uint(-INFINITY);
+          }
+        };
+        // pass 1: raw row maximum over the block (scale > 0 commutes with max)
+        float pm[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          uint32_t s0[32], s1[32];
+          tmem_ld32(tS + h2 * 64, s0);
+          tmem_ld32(tS + h2 * 64 + 32, s1);
+          tc_wait_ld();
+          if (masked) apply_mask(h2, s0, s1);
+#pragma unroll
+          for (int cc = 0; cc < 32; ++cc) {
+            pm[cc & 7] = fmaxf(pm[cc & 7], __uint_as_float(s0[cc]));
+            pm[(cc + 4) & 7] = fmaxf(pm[(cc + 4) & 7], __uint_as_float(s1[cc]));
+          }
+        }
+        const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * a.scale_log2;
+        // lazy rescale: keep the old reference unless the maximum grew a lot
+        const float m_new = (mx > m_run + RESCALE_THRESHOLD) ? mx : m_run;
+        const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
+        const float alpha = fast_exp2(m_run - m_use);
+        // O_X is stable here: PV_X(j-1) was issued before QK_X(j) and MMAs retire in order.
+        if (j > 0 && __any_sync(0xFFFFFFFFu, alpha != 1.f)) {  // warp-uniform: tcgen05.ld/st are collective
+#pragma unroll
+          for (int cc = 0; cc < HD / 32; ++cc) {
             uint32_t o[32];
-            tmem_ld32(tO + c * 32 + lane_off, o);
+            tmem_ld32(tO + cc * 32, o);
             tc_wait_ld();
 #pragma unroll
-            for (int x = 0; x < 32; ++x) o[x] = __float_as_uint(__uint_as_float(o[x]) * alpha);
-            tmem_st32(tO + c * 32 + lane_off, o);
+            for (int u = 0; u < 32; ++u) o[u] = __float_as_uint(__uint_as_float(o[u]) * alpha);
+            tmem_st32(tO + cc * 32, o);
           }
-          tc_wait_st();
         }
+        // pass 2: P = exp2(s * scale - m), bf16 pairs written over S's first 64 columns
+        float ps[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) ps[u] = 0.f;
+        const float neg_m = -m_use;
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          uint32_t s0[32], s1[32];
+          tmem_ld32(tS + h2 * 64, s0);
+          tmem_ld32(tS + h2 * 64 + 32, s1);
+          tc_wait_ld();
+          if (masked) apply_mask(h2, s0, s1);
+          uint32_t pk[32];
+#pragma unroll
+          for (int cc = 0; cc < 32; cc += 2) {
+            const float p0 = fast_exp2(fmaf(__uint_as_float(s0[cc]), a.scale_log2, neg_m));
+            const float p1 = fast_exp2(fmaf(__uint_as_float(s0[cc + 1]), a.scale_log2, neg_m));
+            const float p2 = fast_exp2(fmaf(__uint_as_float(s1[cc]), a.scale_log2, neg_m));
+            const float p3 = fast_exp2(fmaf(__uint_as_float(s1[cc + 1]), a.scale_log2, neg_m));
+            ps[cc & 7] += p0;
+            ps[(cc + 1) & 7] += p1;
+            ps[(cc + 4) & 7] += p2;
+            ps[(cc + 5) & 7] += p3;
+            pk[cc >> 1] = pack_bf16x2(p0, p1);
+            pk[16 + (cc >> 1)] = pack_bf16x2(p2, p3);
+          }
+          tmem_st16(tS + h2 * 32, *reinterpret_cast<uint32_t(*)[16]>(&pk[0]));
+          tmem_st16(tS + h2 * 32 + 16, *reinterpret_cast<uint32_t(*)[16]>(&pk[16]));
+        }
+        tc_wait_st();
+        const float sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+        l_run = l_run * alpha + sum;
+        m_run = m_new;
+        tc_fence_before();
+        mbar_arrive(bar(B_PFULL + x));
       }
-      // P row -> shared memory (bf16, 128-byte swizzle, K-major A operand)
+      if (ok && warp_wait(bar(B_ODONE + x), 0, &s_abort)) {
+        tc_fence_after();
+        const float inv = 1.f / l_run;
+        __nv_bfloat16* dst = a.out + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD;
 #pragma unroll
-      for (int ch = 0; ch < 16; ++ch) {
-        uint4 v;
-        v.x = pack_bf16x2(__uint_as_float(sreg[ch * 8 + 0]), __uint_as_float(sreg[ch * 8 + 1]));
-        v.y = pack_bf16x2(__uint_as_float(sreg[ch * 8 + 2]), __uint_as_float(sreg[ch * 8 + 3]));
-        v.z = pack_bf16x2(__uint_as_float(sreg[ch * 8 + 4]), __uint_as_float(sreg[ch * 8 + 5]));
-        v.w = pack_bf16x2(__uint_as_float(sreg[ch * 8 + 6]), __uint_as_float(sreg[ch * 8 + 7]));
-        *reinterpret_cast<uint4*>(smem + OFF_P + (ch >> 3) * HALF_BYTES + r * 128 + (((ch & 7) ^ (r & 7)) << 4)) = v;
-      }
-      fence_proxy_async_smem();
-      tc_fence_before();
-      mbar_arrive(bar(B_PFULL));
-    }
-    if (ok && __all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar(B_ODONE), (nblk - 1) & 1, &s_abort, WAIT_NS))) {
-      tc_fence_after();
-      const float inv = 1.f / l_run;
-      __nv_bfloat16* dst = a.out + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD;
+        for (int cc = 0; cc < HD / 32; ++cc) {
+          uint32_t o[32];
+          tmem_ld32(tO + cc * 32, o);
+          tc_wait_ld();
+          if (row_ok) {
 #pragma unroll
-      for (int c = 0; c < HD / 32; ++c) {
-        uint32_t o[32];
-        tmem_ld32(tO + c * 32 + lane_off, o);
-        tc_wait_ld();
-        if (row_ok) {
-#pragma unroll
-          for (int x = 0; x < 32; x += 8) {
-            uint4 v;
-            v.x = pack_bf16x2(__uint_as_float(o[x + 0]) * inv, __uint_as_float(o[x + 1]) * inv);
-            v.y = pack_bf16x2(__uint_as_float(o[x + 2]) * inv, __uint_as_float(o[x + 3]) * inv);
-            v.z = pack_bf16x2(__uint_as_float(o[x + 4]) * inv, __uint_as_float(o[x + 5]) * inv);
-            v.w = pack_bf16x2(__uint_as_float(o[x + 6]) * inv, __uint_as_float(o[x + 7]) * inv);
-            *reinterpret_cast<uint4*>(dst + c * 32 + x) = v;
+            for (int u = 0; u < 32; u += 8) {
+              uint4 v;
+              v.x = pack_bf16x2(__uint_as_float(o[u + 0]) * inv, __uint_as_float(o[u + 1]) * inv);
+              v.y = pack_bf16x2(__uint_as_float(o[u + 2]) * inv, __uint_as_float(o[u + 3]) * inv);
+              v.z = pack_bf16x2(__uint_as_float(o[u + 4]) * inv, __uint_as_float(o[u + 5]) * inv);
+              v.w = pack_bf16x2(__uint_as_float(o[u + 6]) * inv, __uint_as_float(o[u + 7]) * inv);
+              *reinterpret_cast<uint4*>(dst + cc * 32 + u) = v;
+            }
           }
         }
       }
@@ -398,8 +451,8 @@ extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const 
   if (al % 16 || reinterpret_cast<uintptr_t>(d_mask) % 8) return FC_ERR_INVALID_ARG;
   const uint64_t groups = (uint64_t)batch * Hkv;
   const int G = H / Hkv;
-  const int tiles = (G * n_pad + BM - 1) / BM;
-  if (groups * tiles > 0x7FFFFFFFull) return FC_ERR_UNSUPPORTED;
+  const int ctas = (G * n_pad + TILES * BM - 1) / (TILES * BM);
+  if (groups * ctas > 0x7FFFFFFFull) return FC_ERR_UNSUPPORTED;
   CUtensorMap mkc, mvc, mkt, mvt;
   if (!make_map(&mkc, d_k_cache, (uint64_t)kv_cap, groups, BN) || !make_map(&mvc, d_v_cache, (uint64_t)kv_cap, groups, BN) ||
       !make_map(&mkt, d_k_tree, (uint64_t)n_pad, groups, (uint32_t)n_pad) ||
@@ -419,9 +472,9 @@ extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const 
   a.Hkv = Hkv;
   a.G = G;
   a.kv_cap = kv_cap;
-  a.tiles = tiles;
+  a.ctas = ctas;
   a.scale_log2 = scale * 1.4426950408889634f;
-  k_tree_attn<<<(unsigned)(groups * tiles), TA_THREADS, SMEM_BYTES, static_cast<cudaStream_t>(stream)>>>(mkc, mvc, mkt,
+  k_tree_attn<<<(unsigned)(groups * ctas), TA_THREADS, SMEM_BYTES, static_cast<cudaStream_t>(stream)>>>(mkc, mvc, mkt,
                                                                                                         mvt, a);
   return FC_CHECK_LAUNCH();
 }
