@@ -558,11 +558,13 @@ def run_attn(args, rank, ws, local):
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     barrier(ws)
     torch.cuda.synchronize()
+    clocks = ClockSampler(local)
     for e0, e1 in evs:
         e0.record()
         fc.fc_tree_attn(*args_d, out=out)
         e1.record()
     torch.cuda.synchronize()
+    clock_rec = clocks.stop()
     ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in evs)
     dep = m["depth"].cpu().numpy()
     pairs = sum(H * (args.nodes * L + int((dep[b, :args.nodes] + 1).sum())) for b in range(B))
@@ -573,7 +575,8 @@ def run_attn(args, rank, ws, local):
             "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "config": {"workload": f"tree attention B={B} H=32 Hkv=8 D=128 KV={L} nodes={args.nodes}"},
             "frac_tensor_sustained": flops / (ms * 1e-3) / 1e12 / peaks["tc_sustained"],
-            "frac_hbm": bytes_ / (ms * 1e-3) / 1e9 / peaks["hbm"], "flops": flops, "bytes": bytes_}
+            "frac_hbm": bytes_ / (ms * 1e-3) / 1e9 / peaks["hbm"], "flops": flops, "bytes": bytes_,
+            "clocks": clock_rec}
 
 
 def main(argv=None):

@@ -62,9 +62,10 @@ enum {
   B_VEMPTY = 6,  // [2] V tile consumed by both PV MMAs
   B_SFULL = 8,   // [2 tiles] S_X ready
   B_PFULL = 10,  // [2 tiles] P_X written (128 arrivals)
-  B_ODONE = 12,  // [2 tiles] last PV_X done
+  B_ODONE = 12,  // [2 tiles] a PV into O_X done (one completion per block)
   B_DRAIN = 14,  // MMA drain on abort
-  N_BARS = 15
+  B_OFIN = 15,   // [2 tiles] the last PV into O_X done
+  N_BARS = 17
 };
 
 struct AttnArgs {
@@ -197,39 +198,29 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     // ---------------- MMA issuer (+ ragged V rows zeroed by the warp) -------
     constexpr uint32_t IDESC_QK = idesc_bf16_f32(BM, BN, 0);
     constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, HD, 1);
-    const int ntiles = has_b ? 2 : 1;
-    auto issue_qk = [&](int j, int x) {
+    // S buffer sb (TMEM columns sb*128..) <- Q tile x . K(j)^T; arrives on S_FULL[sb]
+    auto issue_qk = [&](int j, int x, int sb) {
       const uint32_t kb = sK + (j & 1) * TILE_BYTES, qb = sQ + x * TILE_BYTES;
 #pragma unroll
       for (int kk = 0; kk < HD / 16; ++kk) {
         const uint32_t off = (kk >> 2) * HALF_BYTES + (kk & 3) * 32;
-        tc_mma_f16(tmem + x * 128, smem_desc_sw128(qb + off, 16, 1024), smem_desc_sw128(kb + off, 16, 1024),
+        tc_mma_f16(tmem + sb * 128, smem_desc_sw128(qb + off, 16, 1024), smem_desc_sw128(kb + off, 16, 1024),
                    IDESC_QK, kk > 0);
       }
-      tc_commit(bar(B_SFULL + x));
+      tc_commit(bar(B_SFULL + sb));
     };
-    auto issue_pv = [&](int jj, int x) {
+    // O tile x += P (bf16 pairs in the first 64 columns of S buffer sb) . V(jj)
+    auto issue_pv = [&](int jj, int x, int sb, int) {
       const uint32_t vb = sV + (jj & 1) * TILE_BYTES;
 #pragma unroll
-      for (int kk = 0; kk < BN / 16; ++kk)  // P_X: 8 packed columns per 16 keys
-        tc_mma_f16_tmem_a(tmem + 256 + x * 128, tmem + x * 128 + kk * 8,
+      for (int kk = 0; kk < BN / 16; ++kk)  // 8 packed columns per 16 keys
+        tc_mma_f16_tmem_a(tmem + 256 + x * 128, tmem + sb * 128 + kk * 8,
                           smem_desc_sw128(vb + kk * 2048, HALF_BYTES, 1024), IDESC_PV, (jj > 0 || kk > 0));
     };
-    bool ok = warp_wait(bar(B_KFULL), 0, &s_abort);
-    if (ok) {
-      if (lane == 0) {
-        tc_fence_after();
-        for (int x = 0; x < ntiles; ++x) issue_qk(0, x);
-        tc_commit(bar(B_KEMPTY));
-      }
-      __syncwarp();
-    }
-    for (int j = 1; ok && j <= nblk; ++j) {
-      const int jj = j - 1, st = jj & 1;
-      if (!(ok = warp_wait(bar(B_VFULL + st), (jj >> 1) & 1, &s_abort))) break;
+    auto zero_ragged_v = [&](int jj) {  // never let garbage (possibly NaN) rows meet a zero probability
       const int nv = (jj < nblk_c) ? min(BN, kvl - jj * BN) : nn;
-      if (nv < BN) {  // never let garbage (possibly NaN) rows meet a zero probability
-        unsigned char* vt = smem + OFF_V + st * TILE_BYTES;
+      if (nv < BN) {
+        unsigned char* vt = smem + OFF_V + (jj & 1) * TILE_BYTES;
         for (int e = lane; e < (BN - nv) * 16; e += 32) {
           const int r = nv + (e >> 4), ch = e & 15;
           *reinterpret_cast<uint4*>(vt + (ch >> 3) * HALF_BYTES + r * 128 + (ch & 7) * 16) = make_uint4(0, 0, 0, 0);
@@ -237,27 +228,82 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         fence_proxy_async_smem();
       }
       __syncwarp();
-      for (int x = 0; ok && x < ntiles; ++x) {
-        if (!(ok = warp_wait(bar(B_PFULL + x), jj & 1, &s_abort))) break;
+    };
+    bool ok = true;
+    if (has_b) {
+      // Two tiles, one S buffer each: per tile PV_X(j-1) -> QK_X(j); the
+      // other tile's softmax runs meanwhile.
+      ok = warp_wait(bar(B_KFULL), 0, &s_abort);
+      if (ok) {
         if (lane == 0) {
           tc_fence_after();
-          issue_pv(jj, x);
+          for (int x = 0; x < 2; ++x) issue_qk(0, x, x);
+          tc_commit(bar(B_KEMPTY));
         }
         __syncwarp();
-        if (j < nblk) {
-          if (x == 0 && !(ok = warp_wait(bar(B_KFULL + (j & 1)), (j >> 1) & 1, &s_abort))) break;
-          if (lane == 0) issue_qk(j, x);
+      }
+      for (int j = 1; ok && j <= nblk; ++j) {
+        const int jj = j - 1, st = jj & 1;
+        if (!(ok = warp_wait(bar(B_VFULL + st), (jj >> 1) & 1, &s_abort))) break;
+        zero_ragged_v(jj);
+        for (int x = 0; ok && x < 2; ++x) {
+          if (!(ok = warp_wait(bar(B_PFULL + x), jj & 1, &s_abort))) break;
+          if (lane == 0) {
+            tc_fence_after();
+            issue_pv(jj, x, x, x);
+            tc_commit(bar(B_ODONE + x));
+          }
+          __syncwarp();
+          if (j < nblk) {
+            if (x == 0 && !(ok = warp_wait(bar(B_KFULL + (j & 1)), (j >> 1) & 1, &s_abort))) break;
+            if (lane == 0) issue_qk(j, x, x);
+            __syncwarp();
+          } else if (lane == 0) {
+            tc_commit(bar(B_OFIN + x));
+          }
+        }
+        if (!ok) break;
+        if (lane == 0) {
+          if (j < nblk) tc_commit(bar(B_KEMPTY + (j & 1)));
+          tc_commit(bar(B_VEMPTY + st));
+        }
+        __syncwarp();
+      }
+    } else {
+      // One tile, S double-buffered in both S regions: QK(j+1) runs during
+      // softmax(j); PV(j) reads P from S(j&1) before QK(j+2) overwrites it.
+      for (int j = 0; ok && j < min(2, nblk); ++j) {
+        if (!(ok = warp_wait(bar(B_KFULL + j), 0, &s_abort))) break;
+        if (lane == 0) {
+          tc_fence_after();
+          issue_qk(j, 0, j);
+          tc_commit(bar(B_KEMPTY + j));
+        }
+        __syncwarp();
+      }
+      for (int jj = 0; ok && jj < nblk; ++jj) {
+        const int v = jj & 1;
+        if (!(ok = warp_wait(bar(B_VFULL + v), (jj >> 1) & 1, &s_abort))) break;
+        zero_ragged_v(jj);
+        if (!(ok = warp_wait(bar(B_PFULL + v), (jj >> 1) & 1, &s_abort))) break;
+        if (lane == 0) {
+          tc_fence_after();
+          issue_pv(jj, 0, v, 0);
+          tc_commit(bar(B_ODONE));
+          tc_commit(bar(B_VEMPTY + v));
+          if (jj == nblk - 1) tc_commit(bar(B_OFIN));
+        }
+        __syncwarp();
+        if (jj + 2 < nblk) {
+          if (!(ok = warp_wait(bar(B_KFULL + v), ((jj + 2) >> 1) & 1, &s_abort))) break;
+          if (lane == 0) {
+            tc_fence_after();
+            issue_qk(jj + 2, 0, v);
+            tc_commit(bar(B_KEMPTY + v));
+          }
           __syncwarp();
         }
       }
-      if (!ok) break;
-      if (lane == 0) {
-        if (j < nblk) tc_commit(bar(B_KEMPTY + (j & 1)));
-        tc_commit(bar(B_VEMPTY + st));
-        if (j == nblk)
-          for (int x = 0; x < ntiles; ++x) tc_commit(bar(B_ODONE + x));
-      }
-      __syncwarp();
     }
     if (s_abort) {  // let issued MMAs retire before the tensor memory is freed
       if (lane == 0) tc_commit(bar(B_DRAIN));
@@ -272,7 +318,7 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     if (x == 0 || has_b) {
       const int r = q4 * 32 + lane;
       const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
-      const uint32_t tS = tmem + x * 128 + lane_off, tO = tmem + 256 + x * 128 + lane_off;
+      const uint32_t tO = tmem + 256 + x * 128 + lane_off;
       const int rg = row0 + x * BM + r;
       const bool row_ok = rg < rows_total;
       const int hh = row_ok ? rg / nn : 0, i = row_ok ? rg - hh * nn : 0;
@@ -282,7 +328,11 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
       float m_run = -INFINITY, l_run = 0.f;
       bool ok = true;
       for (int j = 0; j < nblk; ++j) {
-        if (!(ok = warp_wait(bar(B_SFULL + x), j & 1, &s_abort))) break;
+        // two tiles: S buffer x, one phase per block; one tile: S buffers alternate
+        const int sb = has_b ? x : (j & 1);
+        const uint32_t par = has_b ? (j & 1) : ((j >> 1) & 1);
+        const uint32_t tS = tmem + sb * 128 + lane_off;
+        if (!(ok = warp_wait(bar(B_SFULL + sb), par, &s_abort))) break;
         tc_fence_after();
         const bool tree = (j == nblk - 1);
         const int nv = tree ? BN : min(BN, kvl - j * BN);
@@ -325,8 +375,11 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         const float m_new = (mx > m_run + RESCALE_THRESHOLD) ? mx : m_run;
         const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
         const float alpha = fast_exp2(m_run - m_use);
-        // O_X is stable here: PV_X(j-1) was issued before QK_X(j) and MMAs retire in order.
+        // Two tiles: O_X is stable here (PV_X(j-1) was issued before QK_X(j) and
+        // MMAs retire in order).  One tile: PV(j-1) may still run; wait for it.
         if (j > 0 && __any_sync(0xFFFFFFFFu, alpha != 1.f)) {  // warp-uniform: tcgen05.ld/st are collective
+          if (!has_b && !(ok = warp_wait(bar(B_ODONE), (j - 1) & 1, &s_abort))) break;
+          tc_fence_after();
 #pragma unroll
           for (int cc = 0; cc < HD / 32; ++cc) {
             uint32_t o[32];
@@ -371,9 +424,9 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         l_run = l_run * alpha + sum;
         m_run = m_new;
         tc_fence_before();
-        mbar_arrive(bar(B_PFULL + x));
+        mbar_arrive(bar(B_PFULL + sb));
       }
-      if (ok && warp_wait(bar(B_ODONE + x), 0, &s_abort)) {
+      if (ok && warp_wait(bar(B_OFIN + x), 0, &s_abort)) {
         tc_fence_after();
         const float inv = 1.f / l_run;
         __nv_bfloat16* dst = a.out + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD;
