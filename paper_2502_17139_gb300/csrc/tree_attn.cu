@@ -84,6 +84,60 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+// ---- packed fp32 pairs (sm_100 family f32x2 arithmetic) ----
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// 2^x for a pair on the FMA pipe (offloads the MUFU unit).  Round-to-nearest
+// range reduction x = n + f, f in [-1/2, 1/2] (adding 1.5 * 2^23 leaves n in
+// the low mantissa bits), p(f) = 1 + c1 f + c2 f^2 + c3 f^3 (least-squares fit
+// of 2^f, relative error <= 1.8e-4, see exp2_poly_fit.py), then n is added to
+// the exponent field.  Inputs are clamped to >= -125 so the result stays a
+// normal number (2^-125 is nil next to the row maximum's 1).
+__device__ __forceinline__ void exp2_poly_pair(uint64_t x2, float& p0, float& p1) {
+  constexpr float kRound = 12582912.f;  // 1.5 * 2^23
+  float x0, x1;
+  f2_unpack(x2, x0, x1);
+  x2 = f2_pack(fmaxf(x0, -125.f), fmaxf(x1, -125.f));
+  const uint64_t t2 = f2_add(x2, f2_pack(kRound, kRound));
+  const uint64_t r2 = f2_add(t2, f2_pack(-kRound, -kRound));
+  const uint64_t fr = f2_fma(r2, f2_pack(-1.f, -1.f), x2);
+  uint64_t p2 = f2_fma(f2_pack(0.054602622985839844f, 0.054602622985839844f), fr,
+                       f2_pack(0.24192412197589874f, 0.24192412197589874f));
+  p2 = f2_fma(p2, fr, f2_pack(0.6933164596557617f, 0.6933164596557617f));
+  p2 = f2_fma(p2, fr, f2_pack(1.f, 1.f));
+  float t0, t1, q0, q1;
+  f2_unpack(t2, t0, t1);
+  f2_unpack(p2, q0, q1);
+  p0 = __int_as_float(__float_as_int(q0) + (__float_as_int(t0) << 23));
+  p1 = __int_as_float(__float_as_int(q1) + (__float_as_int(t1) << 23));
+}
+
+// Which score pairs of a 32-column chunk take the polynomial exp2 (1 in 4):
+// the MUFU unit handles the rest, and the two pipes finish together.
+__device__ __forceinline__ constexpr bool poly_pair(int q) { return (q & 3) == 3; }
+
 // All 32 lanes wait; the result is warp-uniform.
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
   return __all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar, parity, abort, WAIT_CYCLES));
@@ -364,9 +418,10 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
           tc_wait_ld();
           if (masked) apply_mask(h2, s0, s1);
 #pragma unroll
-          for (int cc = 0; cc < 32; ++cc) {
-            pm[cc & 7] = fmaxf(pm[cc & 7], __uint_as_float(s0[cc]));
-            pm[(cc + 4) & 7] = fmaxf(pm[(cc + 4) & 7], __uint_as_float(s1[cc]));
+          for (int cc = 0; cc < 32; cc += 2) {
+            pm[(cc >> 1) & 7] = fmax3(pm[(cc >> 1) & 7], __uint_as_float(s0[cc]), __uint_as_float(s0[cc + 1]));
+            pm[((cc >> 1) + 4) & 7] =
+                fmax3(pm[((cc >> 1) + 4) & 7], __uint_as_float(s1[cc]), __uint_as_float(s1[cc + 1]));
           }
         }
         const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
@@ -391,35 +446,55 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
           }
         }
         // pass 2: P = exp2(s * scale - m), bf16 pairs written over S's first 64 columns
-        float ps[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) ps[u] = 0.f;
-        const float neg_m = -m_use;
+        uint64_t ps2[4] = {0ull, 0ull, 0ull, 0ull};  // packed partial row sums
+        const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2), nm2 = f2_pack(-m_use, -m_use);
 #pragma unroll
         for (int h2 = 0; h2 < 2; ++h2) {
           uint32_t s0[32], s1[32];
           tmem_ld32(tS + h2 * 64, s0);
           tmem_ld32(tS + h2 * 64 + 32, s1);
           tc_wait_ld();
-          if (masked) apply_mask(h2, s0, s1);
           uint32_t pk[32];
+          if (masked) {  // masked keys are -inf: MUFU exp2 makes them exact zeros
+            apply_mask(h2, s0, s1);
 #pragma unroll
-          for (int cc = 0; cc < 32; cc += 2) {
-            const float p0 = fast_exp2(fmaf(__uint_as_float(s0[cc]), a.scale_log2, neg_m));
-            const float p1 = fast_exp2(fmaf(__uint_as_float(s0[cc + 1]), a.scale_log2, neg_m));
-            const float p2 = fast_exp2(fmaf(__uint_as_float(s1[cc]), a.scale_log2, neg_m));
-            const float p3 = fast_exp2(fmaf(__uint_as_float(s1[cc + 1]), a.scale_log2, neg_m));
-            ps[cc & 7] += p0;
-            ps[(cc + 1) & 7] += p1;
-            ps[(cc + 4) & 7] += p2;
-            ps[(cc + 5) & 7] += p3;
-            pk[cc >> 1] = pack_bf16x2(p0, p1);
-            pk[16 + (cc >> 1)] = pack_bf16x2(p2, p3);
+            for (int q = 0; q < 32; ++q) {
+              const uint32_t* src = q < 16 ? s0 : s1;
+              const int cc = 2 * (q & 15);
+              float x0, x1;
+              f2_unpack(f2_fma(f2_pack(__uint_as_float(src[cc]), __uint_as_float(src[cc + 1])), sc2, nm2), x0, x1);
+              const float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
+              ps2[q & 3] = f2_add(ps2[q & 3], f2_pack(p0, p1));
+              pk[q] = pack_bf16x2(p0, p1);
+            }
+          } else {
+#pragma unroll
+            for (int q = 0; q < 32; ++q) {
+              const uint32_t* src = q < 16 ? s0 : s1;
+              const int cc = 2 * (q & 15);
+              const uint64_t x2 = f2_fma(f2_pack(__uint_as_float(src[cc]), __uint_as_float(src[cc + 1])), sc2, nm2);
+              float p0, p1;
+              if (poly_pair(q)) {
+                exp2_poly_pair(x2, p0, p1);
+              } else {
+                float x0, x1;
+                f2_unpack(x2, x0, x1);
+                p0 = fast_exp2(x0);
+                p1 = fast_exp2(x1);
+              }
+              ps2[q & 3] = f2_add(ps2[q & 3], f2_pack(p0, p1));
+              pk[q] = pack_bf16x2(p0, p1);
+            }
           }
           tmem_st16(tS + h2 * 32, *reinterpret_cast<uint32_t(*)[16]>(&pk[0]));
           tmem_st16(tS + h2 * 32 + 16, *reinterpret_cast<uint32_t(*)[16]>(&pk[16]));
         }
         tc_wait_st();
+        float ps[8];
+        f2_unpack(ps2[0], ps[0], ps[1]);
+        f2_unpack(ps2[1], ps[2], ps[3]);
+        f2_unpack(ps2[2], ps[4], ps[5]);
+        f2_unpack(ps2[3], ps[6], ps[7]);
         const float sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
         l_run = l_run * alpha + sum;
         m_run = m_new;
