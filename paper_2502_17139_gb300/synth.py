@@ -53,10 +53,27 @@ def zipf_cdf(s: float, vocab: int = VOCAB) -> np.ndarray:
 
 
 def zipf_tokens(rng: np.random.Generator, n: int, s: float, vocab: int = VOCAB,
-                chunk: int = 1 << 24) -> np.ndarray:
-    """``n`` i.i.d. token ids, id = rank - 1 with rank ~ Zipf(s) (inverse CDF)."""
+                chunk: int = 1 << 24, device=None) -> np.ndarray:
+    """``n`` i.i.d. token ids, id = rank - 1 with rank ~ Zipf(s) (inverse CDF).
+
+    With ``device`` (a CUDA device) and a large ``n`` the uniform draws and the
+    inverse-CDF lookup run there with a torch generator seeded from ``rng``
+    (the same numbers on every run, not the numpy stream); the result still
+    comes back as a host array."""
     cdf = zipf_cdf(s, vocab)
     out = np.empty(n, dtype=np.uint32)
+    if device is not None and n >= (1 << 26):
+        import torch
+        g = torch.Generator(device=device)
+        g.manual_seed(int(rng.integers(0, 1 << 62)))
+        cdf_d = torch.from_numpy(cdf).to(device)
+        step = 1 << 27
+        for lo in range(0, n, step):
+            hi = min(n, lo + step)
+            u = torch.rand(hi - lo, generator=g, device=device, dtype=torch.float64)
+            r = torch.searchsorted(cdf_d, u, right=True).clamp_(max=vocab - 1)
+            out[lo:hi] = r.to(torch.int32).cpu().numpy().view(np.uint32)
+        return out
     for lo in range(0, n, chunk):
         hi = min(n, lo + chunk)
         u = rng.random(hi - lo)
@@ -125,9 +142,9 @@ def grams_for_fraction(n: int, frac: float, len_range: tuple, copies_range: tupl
 
 
 def make_corpus(rng: np.random.Generator, n: int, s: float, vocab: int = VOCAB,
-                n_grams: int = 0, len_range=(8, 32), copies_range=(2, 8)):
+                n_grams: int = 0, len_range=(8, 32), copies_range=(2, 8), device=None):
     """Zipf(s) background with planted repeats; returns (uint32 tokens, Planted)."""
-    t = zipf_tokens(rng, n, s, vocab)
+    t = zipf_tokens(rng, n, s, vocab, device=device)
     p = plant_repeats(rng, t, n_grams, len_range, copies_range, s, vocab)
     return t, p
 
@@ -276,12 +293,12 @@ def scaled_corpus_spec(spec: dict, scale: float) -> dict:
     return out
 
 
-def build_corpus(rng: np.random.Generator, spec: dict, vocab: int = VOCAB):
-    """Corpus from a spec dict (see CONFIGS)."""
+def build_corpus(rng: np.random.Generator, spec: dict, vocab: int = VOCAB, device=None):
+    """Corpus from a spec dict (see CONFIGS); ``device`` as for zipf_tokens."""
     n = spec["n"]
     lr = spec.get("len_range", (8, 32))
     cr = spec.get("copies_range", (2, 8))
     grams = spec.get("n_grams", 0)
     if spec.get("frac"):
         grams = grams_for_fraction(n, spec["frac"], lr, cr)
-    return make_corpus(rng, n, spec["s"], vocab, grams, lr, cr)
+    return make_corpus(rng, n, spec["s"], vocab, grams, lr, cr, device=device)
