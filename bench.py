@@ -169,8 +169,10 @@ def make_inputs(scale: float, batch: int, rank: int, steps_total: int):
     cfg, corp_specs, kv0, B = workload_spec(scale, batch)
     rng = synth.rng_for(2)                      # datastores: identical on every rank
     corpora = []
+    import torch
+    gen_dev = "cuda" if torch.cuda.is_available() else None
     for spec in corp_specs:
-        T, _ = synth.build_corpus(rng, spec)
+        T, _ = synth.build_corpus(rng, spec, device=gen_dev)
         corpora.append(T)
     Tr, Tc = corpora                            # project store first (alpha), general second (beta)
     rr = synth.rng_for(5, 1 + rank)             # per-rank sequences

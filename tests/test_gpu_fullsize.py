@@ -60,7 +60,7 @@ def test_two_source_100m_5m(fc, orc):
     store 100M (Zipf 1.1), 256 contexts of 128 tokens, top-64 x 10, 64-node trees."""
     cfg = synth.CONFIGS[2]
     rng = synth.rng_for(2)
-    corpora = [synth.build_corpus(rng, spec)[0] for spec in cfg["corpus"]]
+    corpora = [synth.build_corpus(rng, spec, device="cuda")[0] for spec in cfg["corpus"]]
     Tr, Tc = corpora
     ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], [Tr, Tc, None], cfg["probs"],
                                      1.1)
