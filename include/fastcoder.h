@@ -51,6 +51,7 @@ typedef void* fc_stream; /* cudaStream_t */
 #define FC_MAX_OCC 4096       /* occurrences examined per query and source */
 #define FC_MAX_SOURCES 4      /* datastores searched in one call */
 #define FC_MAX_NODES 128      /* draft-tree nodes (root included) */
+#define FC_LCP_CAP 255        /* longest-common-prefix values are stored capped here */
 
 /* Human-readable name of a status code (static storage). */
 const char* fc_status_string(fc_status s);
@@ -76,6 +77,9 @@ typedef struct {
   const uint32_t* sa;      /* device, [n_tokens] suffix array of tokens */
   const uint32_t* bucket;  /* device, [vocab + 1]: bucket[v] = first SA index whose
                               suffix starts with a token >= v; bucket[vocab] = n_tokens */
+  const uint8_t* lcp;      /* device, [n_tokens]: lcp[j] = length of the longest common
+                              prefix of the suffixes at sa[j-1] and sa[j], capped at
+                              FC_LCP_CAP; lcp[0] = 0 */
   uint64_t n_tokens;       /* 1 <= n_tokens < 2^32 - 1 */
   uint32_t vocab;          /* 1 <= vocab < 2^31 */
 } fc_datastore;
@@ -90,14 +94,17 @@ size_t fc_datastore_build_workspace(uint64_t n_tokens, uint32_t vocab);
  *   d_sa     [n_tokens] uint32 out: sa[j] = start of the j-th smallest suffix;
  *            a suffix that is a proper prefix of another sorts first
  *   d_bucket [vocab + 1] uint32 out (see fc_datastore.bucket)
+ *   d_lcp    [n_tokens] uint8 out (see fc_datastore.lcp): adjacent suffixes'
+ *            common prefix lengths, which let retrieval group equal
+ *            continuations without reading them
  *   d_ws     workspace of at least fc_datastore_build_workspace() bytes
  *   out      host struct filled with the datastore view (may be NULL)
  * Synchronous: returns when the build is finished (it reads a group count
  * back after every doubling round).
  */
 fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t vocab,
-                             uint32_t* d_sa, uint32_t* d_bucket, void* d_ws, size_t ws_bytes,
-                             fc_stream s, fc_datastore* out);
+                             uint32_t* d_sa, uint32_t* d_bucket, uint8_t* d_lcp, void* d_ws,
+                             size_t ws_bytes, fc_stream s, fc_datastore* out);
 
 /*
  * The same build for callers that cannot allocate device memory.  The paper
@@ -107,8 +114,8 @@ fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n_tokens, uint32
  * plugin inside an application that owns every device allocation.  This
  * entry point allocates nothing: its scratch space is a fixed 30 MiB array
  * compiled into the library, which every GPU that loads the library holds
- * until the process exits.  The caller still passes the corpus, d_sa and
- * d_bucket.
+ * until the process exits.  The caller still passes the corpus, d_sa,
+ * d_bucket and d_lcp.
  *   n_tokens must be <= FC_NOALLOC_MAX_TOKENS; larger corpora return
  *   FC_ERR_CAPACITY (use fc_datastore_build with a workspace instead).
  * The first call on a device looks up the array's device address on that
@@ -118,8 +125,8 @@ fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n_tokens, uint32
  */
 #define FC_NOALLOC_MAX_TOKENS 1048576ull
 fc_status fc_datastore_build_noalloc(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t vocab,
-                                     uint32_t* d_sa, uint32_t* d_bucket, fc_stream s,
-                                     fc_datastore* out);
+                                     uint32_t* d_sa, uint32_t* d_bucket, uint8_t* d_lcp,
+                                     fc_stream s, fc_datastore* out);
 
 /* ------------------------------------------------------------------------
  * Retrieval (Section III-A; Section IV-C, Algorithm 1 par_search; Section

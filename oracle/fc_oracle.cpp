@@ -131,6 +131,21 @@ int orc_bucket(const uint32_t* T, uint64_t N, const uint32_t* sa, uint32_t vocab
   return 0;
 }
 
+// Longest common prefix of each suffix with its predecessor in SA order,
+// capped: lcp[j] = LCP(T[sa[j-1]..N), T[sa[j]..N)) limited to cap, lcp[0] = 0.
+// (An index over the SA that lets equal continuations be grouped without
+// reading them; its values follow from the definition directly.)
+int orc_lcp(const uint32_t* T, uint64_t N, const uint32_t* sa, uint32_t cap, uint8_t* lcp) {
+  if (N == 0) return 0;
+  lcp[0] = 0;
+  for (uint64_t j = 1; j < N; ++j) {
+    uint64_t a = sa[j - 1], b = sa[j], l = 0;
+    while (l < cap && a + l < N && b + l < N && T[a + l] == T[b + l]) ++l;
+    lcp[j] = (uint8_t)l;
+  }
+  return 0;
+}
+
 // Certificate that sa is the suffix array of T, usable at any size:
 // sa is a permutation of [0, N) and suffix(sa[j]) < suffix(sa[j+1]) for all j.
 // Returns -1 when valid; otherwise the first offending SA index (or N when

@@ -79,6 +79,15 @@ def bucket(T: np.ndarray, sa: np.ndarray, vocab: int) -> np.ndarray:
     return out
 
 
+def lcp(T: np.ndarray, sa: np.ndarray, cap: int = 255) -> np.ndarray:
+    """lcp[j] = common prefix length of the suffixes at sa[j-1], sa[j] (capped)."""
+    T = _c(T, np.uint32)
+    sa = _c(sa, np.uint32)
+    out = np.empty(len(T), dtype=np.uint8)
+    lib().orc_lcp(_p(T), C.c_uint64(len(T)), _p(sa), C.c_uint32(cap), _p(out))
+    return out
+
+
 def sa_certificate(T: np.ndarray, sa: np.ndarray, nthreads: int = 0) -> int:
     """-1 when sa is the suffix array of T, else the first failing index."""
     T = _c(T, np.uint32)

@@ -13,10 +13,14 @@
 //     continuation) is the smallest suffix of its range when present; it is
 //     dropped.
 //   * counting: in SA order the occurrences' continuations are sorted, so
-//     equal continuations are adjacent; runs are found with one compare per
-//     neighbour pair and a block scan (no hash table needed).
-//   * top-k: a bitonic sort in shared memory of (count << 12 | 4095 - run)
-//     keys gives count descending, then run order (= token order) ascending.
+//     equal continuations are adjacent, and two neighbours carry the same
+//     continuation exactly when their common prefix (the datastore's LCP
+//     array) covers the match plus the draft length.  Runs come from one
+//     coalesced byte read per occurrence and a block scan (no hash table and
+//     no token reads).
+//   * top-k: a histogram of run counts finds the k-th largest count; the runs
+//     above it and the first runs equal to it (in token order) are kept and
+//     ranked by (count descending, token order ascending).
 #include <algorithm>
 
 #include "fc_common.cuh"
@@ -32,6 +36,7 @@ struct DsView {
   const uint32_t* T;
   const uint32_t* sa;
   const uint32_t* bucket;
+  const uint8_t* lcp;
   uint64_t n;
   uint32_t vocab;
 };
@@ -57,15 +62,6 @@ __device__ __forceinline__ int cmp_suffix(const uint32_t* __restrict__ T, uint64
     if (a != b) return a < b ? -1 : 1;
   }
   return 0;
-}
-
-__device__ __forceinline__ bool cont_equal(const uint32_t* __restrict__ T, uint64_t N, uint32_t p1, uint32_t p2,
-                                           int d) {
-  uint64_t l1 = min((uint64_t)d, N - p1), l2 = min((uint64_t)d, N - p2);
-  if (l1 != l2) return false;
-  for (uint64_t k = 0; k < l1; ++k)
-    if (__ldg(T + p1 + k) != __ldg(T + p2 + k)) return false;
-  return true;
 }
 
 __device__ __forceinline__ uint32_t block_scan_256(uint32_t x, uint32_t* total, uint32_t* wsum) {
@@ -94,14 +90,16 @@ __device__ __forceinline__ uint32_t block_scan_256(uint32_t x, uint32_t* total, 
 }
 
 struct RetSmem {
-  uint32_t pos[FC_MAX_OCC];
-  uint32_t runs[FC_MAX_OCC + 1];
-  uint32_t keys[FC_MAX_OCC];
+  uint32_t runs[FC_MAX_OCC + 1];   // run starts (occurrence index), runs[R] = nocc
+  uint32_t work[FC_MAX_OCC];       // head flags, then the count histogram
+  uint32_t sel[FC_MAX_TOPK];       // kept runs
+  uint32_t order[FC_MAX_TOPK];     // kept runs by (count desc, run asc)
   uint32_t ctx[FC_MAX_NMAX];
   uint32_t lo[FC_MAX_NMAX + 1];
   uint32_t hi[FC_MAX_NMAX + 1];
+  uint32_t endhit[FC_MAX_NMAX + 1];
   uint32_t wsum[RT_THREADS / 32];
-  uint32_t n_star, first, cnt, n_runs, bad;
+  uint32_t n_star, first, cnt, n_runs, bad, cstar, n_greater, n_sel;
 };
 
 __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint32_t* __restrict__ ctx, int stride,
@@ -145,8 +143,13 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint
       if (upper ? (c <= 0) : (c < 0)) lo = mid + 1;
       else hi = mid;
     }
-    if (upper) sm.hi[n] = lo;
-    else sm.lo[n] = lo;
+    if (upper) {
+      sm.hi[n] = lo;
+    } else {
+      sm.lo[n] = lo;
+      // the suffix that is exactly the pattern at the corpus end sorts first in its range
+      sm.endhit[n] = (lo < N && (uint64_t)__ldg(ds.sa + lo) + n == N) ? 1u : 0u;
+    }
   }
   __syncthreads();
   if (tid == 0) {
@@ -154,7 +157,7 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint
     if (npairs) {
       for (int n = cap; n >= p.n_min; --n) {
         uint32_t l = sm.lo[n], h = sm.hi[n];
-        if (l < h && (uint64_t)__ldg(ds.sa + l) + n == N) ++l;  // exact pattern at the corpus end
+        if (l < h && sm.endhit[n]) ++l;
         if (l < h) {
           ns = n;
           first = l;
@@ -186,19 +189,19 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint
   }
   const uint32_t nocc = sm.cnt, first = sm.first;
 
-  // ---- occurrences -> continuation starts ------------------------------
-  for (uint32_t e = tid; e < nocc; e += RT_THREADS) sm.pos[e] = __ldg(ds.sa + first + e) + (uint32_t)ns;
+  // ---- runs of equal continuations -------------------------------------
+  // neighbours j-1, j share their continuation iff lcp[j] >= n* + d
+  const uint32_t need = (uint32_t)ns + (uint32_t)d;
+  for (uint32_t e = tid; e < nocc; e += RT_THREADS)
+    sm.work[e] = (e == 0 || (uint32_t)__ldg(ds.lcp + first + e) < need) ? 1u : 0u;
   __syncthreads();
-  // run heads: continuation differs from its SA predecessor
   uint32_t head[RT_ITEMS];
   uint32_t local = 0;
 #pragma unroll
   for (int it = 0; it < RT_ITEMS; ++it) {
     uint32_t e = tid * RT_ITEMS + it;
-    uint32_t h = 0;
-    if (e < nocc) h = (e == 0) || !cont_equal(T, N, sm.pos[e - 1], sm.pos[e], d);
-    head[it] = h;
-    local += h;
+    head[it] = (e < nocc) ? sm.work[e] : 0u;
+    local += head[it];
   }
   uint32_t total;
   uint32_t run_id = block_scan_256(local, &total, sm.wsum);
@@ -214,35 +217,85 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint
   }
   __syncthreads();
   const uint32_t R = sm.n_runs;
-  uint32_t P2 = 1;
-  while (P2 < R) P2 <<= 1;
-  for (uint32_t r = tid; r < P2; r += RT_THREADS)
-    sm.keys[r] = (r < R) ? (((sm.runs[r + 1] - sm.runs[r]) << 12) | (4095u - r)) : 0u;
-  __syncthreads();
-  for (uint32_t size = 2; size <= P2; size <<= 1) {
-    for (uint32_t stride2 = size >> 1; stride2 > 0; stride2 >>= 1) {
-      for (uint32_t i = tid; i < P2; i += RT_THREADS) {
-        uint32_t j = i ^ stride2;
-        if (j > i) {
-          uint32_t a = sm.keys[i], c = sm.keys[j];
-          bool desc = (i & size) == 0;
-          if (desc ? (a < c) : (a > c)) {
-            sm.keys[i] = c;
-            sm.keys[j] = a;
-          }
-        }
-      }
-      __syncthreads();
+  auto run_count = [&](uint32_t r) { return sm.runs[r + 1] - sm.runs[r]; };
+
+  // ---- top-k runs --------------------------------------------------------
+  if (R <= (uint32_t)k) {
+    for (uint32_t r = tid; r < R; r += RT_THREADS) sm.sel[r] = r;
+    if (tid == 0) sm.n_sel = R;
+  } else {
+    // histogram of counts (1..FC_MAX_OCC), bin q = FC_MAX_OCC - count so that
+    // a prefix over q counts the runs with a larger count
+    for (uint32_t q = tid; q < FC_MAX_OCC; q += RT_THREADS) sm.work[q] = 0;
+    __syncthreads();
+    for (uint32_t r = tid; r < R; r += RT_THREADS) atomicAdd(&sm.work[FC_MAX_OCC - run_count(r)], 1u);
+    __syncthreads();
+    uint32_t hq[RT_ITEMS];
+    uint32_t hsum = 0;
+#pragma unroll
+    for (int it = 0; it < RT_ITEMS; ++it) {
+      hq[it] = sm.work[tid * RT_ITEMS + it];
+      hsum += hq[it];
     }
+    uint32_t tot2;
+    uint32_t above = block_scan_256(hsum, &tot2, sm.wsum);  // runs with a larger count than this chunk's bins
+#pragma unroll
+    for (int it = 0; it < RT_ITEMS; ++it) {
+      if (above < (uint32_t)k && above + hq[it] >= (uint32_t)k) {  // the k-th largest count lives here
+        sm.cstar = FC_MAX_OCC - (tid * RT_ITEMS + it);
+        sm.n_greater = above;
+      }
+      above += hq[it];
+    }
+    __syncthreads();
+    const uint32_t cstar = sm.cstar, room = (uint32_t)k - sm.n_greater;
+    // keep: count > c*, or count == c* among the first `room` such runs in token order
+    uint32_t fl[RT_ITEMS], eq_local = 0;
+#pragma unroll
+    for (int it = 0; it < RT_ITEMS; ++it) {
+      uint32_t r = tid * RT_ITEMS + it;
+      fl[it] = (r < R) ? (run_count(r) > cstar ? 2u : (run_count(r) == cstar ? 1u : 0u)) : 0u;
+      eq_local += (fl[it] == 1u);
+    }
+    uint32_t tot3;
+    uint32_t eq_before = block_scan_256(eq_local, &tot3, sm.wsum);
+    uint32_t keep_local = 0;
+#pragma unroll
+    for (int it = 0; it < RT_ITEMS; ++it) {
+      if (fl[it] == 1u) {
+        fl[it] = (eq_before < room) ? 2u : 0u;
+        ++eq_before;
+      }
+      keep_local += (fl[it] == 2u);
+    }
+    uint32_t tot4;
+    uint32_t kept_before = block_scan_256(keep_local, &tot4, sm.wsum);
+#pragma unroll
+    for (int it = 0; it < RT_ITEMS; ++it) {
+      if (fl[it] == 2u) sm.sel[kept_before++] = tid * RT_ITEMS + it;
+    }
+    if (tid == 0) sm.n_sel = tot4;
   }
+  __syncthreads();
+  const uint32_t ks = sm.n_sel;  // == min(k, R)
+  // rank the kept runs by (count descending, run ascending)
+  for (uint32_t t = tid; t < ks; t += RT_THREADS) {
+    const uint32_t r = sm.sel[t], c = run_count(r);
+    uint32_t rank = 0;
+    for (uint32_t u = 0; u < ks; ++u) {
+      const uint32_t ru = sm.sel[u], cu = run_count(ru);
+      rank += (cu > c || (cu == c && ru < r)) ? 1u : 0u;
+    }
+    sm.order[rank] = r;
+  }
+  __syncthreads();
   // ---- outputs ---------------------------------------------------------
-  const int nd = (int)umin((uint32_t)k, R);
+  const int nd = (int)ks;
   for (int e = tid; e < k * d; e += RT_THREADS) {
     int t = e / d, x = e - t * d;
     uint32_t v = FC_PAD_TOKEN;
     if (t < nd) {
-      uint32_t r = 4095u - (sm.keys[t] & 4095u);
-      uint32_t pp = sm.pos[sm.runs[r]];
+      const uint32_t pp = __ldg(ds.sa + first + sm.runs[sm.order[t]]) + (uint32_t)ns;
       uint64_t len = min((uint64_t)d, N - pp);
       if ((uint64_t)x < len) v = __ldg(T + pp + x);
     }
@@ -250,10 +303,10 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint
   }
   for (int t = tid; t < k; t += RT_THREADS) {
     if (t < nd) {
-      uint32_t r = 4095u - (sm.keys[t] & 4095u);
-      uint32_t pp = sm.pos[sm.runs[r]];
+      const uint32_t r = sm.order[t];
+      const uint32_t pp = __ldg(ds.sa + first + sm.runs[r]) + (uint32_t)ns;
       dl[t] = (int32_t)min((uint64_t)d, N - pp);
-      ct[t] = sm.keys[t] >> 12;
+      ct[t] = run_count(r);
     } else {
       dl[t] = 0;
       ct[t] = 0;
@@ -433,9 +486,10 @@ extern "C" fc_status fc_retrieve(const fc_datastore* sources, int n_sources, con
   DsArgs a{};
   for (int s = 0; s < n_sources; ++s) {
     const fc_datastore& ds = sources[s];
-    if (!ds.tokens || !ds.sa || !ds.bucket || ds.n_tokens == 0 || ds.n_tokens >= 0xFFFFFFFFull || ds.vocab == 0)
+    if (!ds.tokens || !ds.sa || !ds.bucket || !ds.lcp || ds.n_tokens == 0 || ds.n_tokens >= 0xFFFFFFFFull ||
+        ds.vocab == 0)
       return FC_ERR_INVALID_ARG;
-    a.ds[s] = DsView{ds.tokens, ds.sa, ds.bucket, ds.n_tokens, ds.vocab};
+    a.ds[s] = DsView{ds.tokens, ds.sa, ds.bucket, ds.lcp, ds.n_tokens, ds.vocab};
   }
   static bool attr_done = false;
   if (!attr_done) {

@@ -275,6 +275,22 @@ __global__ void k_bucket(const uint32_t* __restrict__ T, const uint32_t* __restr
   }
 }
 
+// lcp[j] = common prefix length of the suffixes at sa[j-1] and sa[j], capped.
+// rank is the inverse suffix array; each thread takes one text position i
+// (so each suffix is compared with its predecessor in SA order once).
+__global__ void k_lcp(const uint32_t* __restrict__ T, const uint32_t* __restrict__ sa,
+                      const uint32_t* __restrict__ rank, uint64_t n, uint8_t* __restrict__ lcp) {
+  for (uint64_t i = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; i < n; i += (uint64_t)gridDim.x * blockDim.x) {
+    const uint32_t j = rank[i];
+    uint32_t l = 0;
+    if (j > 0) {
+      const uint64_t pr = sa[j - 1];
+      while (l < FC_LCP_CAP && i + l < n && pr + l < n && T[i + l] == T[pr + l]) ++l;
+    }
+    lcp[j] = (uint8_t)l;
+  }
+}
+
 inline int bits_for(uint64_t x) {
   int b = 0;
   while (x) {
@@ -299,9 +315,10 @@ extern "C" size_t fc_datastore_build_workspace(uint64_t n_tokens, uint32_t vocab
 }
 
 extern "C" fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n, uint32_t vocab, uint32_t* d_sa,
-                                        uint32_t* d_bucket, void* d_ws, size_t ws_bytes, fc_stream stream,
-                                        fc_datastore* out) {
-  if (!d_tokens || !d_sa || !d_bucket || n == 0 || n >= 0xFFFFFFFFull || vocab == 0 || vocab >= 0x80000000u)
+                                        uint32_t* d_bucket, uint8_t* d_lcp, void* d_ws, size_t ws_bytes,
+                                        fc_stream stream, fc_datastore* out) {
+  if (!d_tokens || !d_sa || !d_bucket || !d_lcp || n == 0 || n >= 0xFFFFFFFFull || vocab == 0 ||
+      vocab >= 0x80000000u)
     return FC_ERR_INVALID_ARG;
   Layout L = layout_for(n);
   if (!d_ws || ws_bytes < L.total) return FC_ERR_WORKSPACE;
@@ -362,11 +379,15 @@ extern "C" fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n, ui
     max_lo = groups;
   }
   k_bucket<<<grid_for((uint64_t)vocab + 1, 256), 256, 0, s>>>(d_tokens, d_sa, n, vocab, d_bucket);
+  // every group is a single suffix now, so rank is the inverse suffix array
+  k_lcp<<<g, 256, 0, s>>>(d_tokens, d_sa, rank, n, d_lcp);
   if (cudaGetLastError() != cudaSuccess) return FC_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return FC_ERR_CUDA;
   if (out) {
     out->tokens = d_tokens;
     out->sa = d_sa;
     out->bucket = d_bucket;
+    out->lcp = d_lcp;
     out->n_tokens = n;
     out->vocab = vocab;
   }
@@ -416,12 +437,12 @@ fc_status scratch_for_current_device(void** out) {
 }  // namespace
 
 extern "C" fc_status fc_datastore_build_noalloc(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t vocab,
-                                                uint32_t* d_sa, uint32_t* d_bucket, fc_stream stream,
-                                                fc_datastore* out) {
+                                                uint32_t* d_sa, uint32_t* d_bucket, uint8_t* d_lcp,
+                                                fc_stream stream, fc_datastore* out) {
   if (n_tokens > FC_NOALLOC_MAX_TOKENS) return FC_ERR_CAPACITY;
   if (n_tokens > 0 && fc_datastore_build_workspace(n_tokens, vocab) > kNoAllocScratchBytes) return FC_ERR_CAPACITY;
   void* ws = nullptr;
   fc_status st = scratch_for_current_device(&ws);
   if (st != FC_OK) return st;
-  return fc_datastore_build(d_tokens, n_tokens, vocab, d_sa, d_bucket, ws, kNoAllocScratchBytes, stream, out);
+  return fc_datastore_build(d_tokens, n_tokens, vocab, d_sa, d_bucket, d_lcp, ws, kNoAllocScratchBytes, stream, out);
 }

@@ -35,7 +35,7 @@ class FastCoderError(RuntimeError):
 
 
 class fc_datastore(C.Structure):
-    _fields_ = [("tokens", C.c_void_p), ("sa", C.c_void_p), ("bucket", C.c_void_p),
+    _fields_ = [("tokens", C.c_void_p), ("sa", C.c_void_p), ("bucket", C.c_void_p), ("lcp", C.c_void_p),
                 ("n_tokens", C.c_uint64), ("vocab", C.c_uint32)]
 
 
@@ -61,8 +61,8 @@ def _load():
         "fc_version": (C.c_char_p, []),
         "fc_get_error": (C.c_int, [vp]),
         "fc_datastore_build_workspace": (sz, [u64, u32]),
-        "fc_datastore_build": (C.c_int, [vp, u64, u32, vp, vp, vp, sz, vp, C.POINTER(fc_datastore)]),
-        "fc_datastore_build_noalloc": (C.c_int, [vp, u64, u32, vp, vp, vp, C.POINTER(fc_datastore)]),
+        "fc_datastore_build": (C.c_int, [vp, u64, u32, vp, vp, vp, vp, sz, vp, C.POINTER(fc_datastore)]),
+        "fc_datastore_build_noalloc": (C.c_int, [vp, u64, u32, vp, vp, vp, vp, C.POINTER(fc_datastore)]),
         "fc_retrieve": (C.c_int, [C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp, fc_retrieve_params,
                                   vp, vp, vp, vp, vp, vp]),
         "fc_rcache_bytes": (sz, [i32, i32, fc_retrieve_params]),
@@ -128,12 +128,13 @@ def fc_get_error(stream=None) -> str:
 
 # --------------------------------------------------------------- datastore
 class Datastore:
-    """A built datastore: the token corpus, its suffix array and bucket table
-    (device tensors owned here), plus the C view struct."""
+    """A built datastore: the token corpus, its suffix array, bucket table and
+    LCP array (device tensors owned here), plus the C view struct."""
 
-    def __init__(self, tokens, sa, bucket, vocab):
-        self.tokens, self.sa, self.bucket, self.vocab = tokens, sa, bucket, int(vocab)
-        self.view = fc_datastore(tokens.data_ptr(), sa.data_ptr(), bucket.data_ptr(), tokens.numel(), int(vocab))
+    def __init__(self, tokens, sa, bucket, lcp, vocab):
+        self.tokens, self.sa, self.bucket, self.lcp, self.vocab = tokens, sa, bucket, lcp, int(vocab)
+        self.view = fc_datastore(tokens.data_ptr(), sa.data_ptr(), bucket.data_ptr(), lcp.data_ptr(),
+                                 tokens.numel(), int(vocab))
 
     @property
     def n_tokens(self):
@@ -150,37 +151,41 @@ def fc_datastore_build(tokens: torch.Tensor, vocab: int, workspace: torch.Tensor
     n = tokens.numel()
     sa = torch.empty(n, dtype=torch.int32, device=tokens.device)
     bucket = torch.empty(vocab + 1, dtype=torch.int32, device=tokens.device)
+    lcp = torch.empty(n, dtype=torch.uint8, device=tokens.device)
     need = fc_datastore_build_workspace(n, vocab)
     ws = workspace if workspace is not None else torch.empty(need, dtype=torch.uint8, device=tokens.device)
     if ws.numel() < need:
         raise ValueError("workspace too small")
-    _check("fc_datastore_build", LIB.fc_datastore_build(_ptr(tokens), n, vocab, _ptr(sa), _ptr(bucket), _ptr(ws),
-                                                        ws.numel(), _stream(), None))
-    return Datastore(tokens, sa, bucket, vocab)
+    _check("fc_datastore_build", LIB.fc_datastore_build(_ptr(tokens), n, vocab, _ptr(sa), _ptr(bucket), _ptr(lcp),
+                                                        _ptr(ws), ws.numel(), _stream(), None))
+    return Datastore(tokens, sa, bucket, lcp, vocab)
 
 
 NOALLOC_MAX_TOKENS = 1 << 20
 
 
-def fc_datastore_build_noalloc(tokens: torch.Tensor, vocab: int, sa: torch.Tensor,
-                               bucket: torch.Tensor) -> Datastore:
+def fc_datastore_build_noalloc(tokens: torch.Tensor, vocab: int, sa: torch.Tensor, bucket: torch.Tensor,
+                               lcp: torch.Tensor) -> Datastore:
     """The datastore build for callers that cannot allocate device memory:
     scratch comes from a fixed array inside the library, and the outputs go
-    to the caller's sa [N] and bucket [vocab + 1] (int32).  N is at most
-    NOALLOC_MAX_TOKENS.  This wrapper allocates nothing either."""
+    to the caller's sa [N] (int32), bucket [vocab + 1] (int32) and lcp [N]
+    (uint8).  N is at most NOALLOC_MAX_TOKENS.  This wrapper allocates
+    nothing either."""
     _need(tokens, torch.int32, "tokens")
     n = tokens.numel()
     _need(sa, torch.int32, "sa", (n,))
     _need(bucket, torch.int32, "bucket", (vocab + 1,))
+    _need(lcp, torch.uint8, "lcp", (n,))
     _check("fc_datastore_build_noalloc", LIB.fc_datastore_build_noalloc(_ptr(tokens), n, vocab, _ptr(sa),
-                                                                        _ptr(bucket), _stream(), None))
-    return Datastore(tokens, sa, bucket, vocab)
+                                                                        _ptr(bucket), _ptr(lcp), _stream(), None))
+    return Datastore(tokens, sa, bucket, lcp, vocab)
 
 
-def datastore_from_parts(tokens, sa, bucket, vocab) -> Datastore:
+def datastore_from_parts(tokens, sa, bucket, lcp, vocab) -> Datastore:
     for t, nm in ((tokens, "tokens"), (sa, "sa"), (bucket, "bucket")):
         _need(t, torch.int32, nm)
-    return Datastore(tokens, sa, bucket, vocab)
+    _need(lcp, torch.uint8, "lcp")
+    return Datastore(tokens, sa, bucket, lcp, vocab)
 
 
 # --------------------------------------------------------------- retrieval

@@ -50,7 +50,7 @@ def test_host_validation_without_gpu(lib):
     # no sources
     assert L.fc_retrieve(nul, 0, nul, 64, nul, 4, nul, p, nul, nul, nul, nul, nul, nul) == 1
     # parameters beyond what the kernels support
-    views = (fc.fc_datastore * 1)(fc.fc_datastore(1, 1, 1, 10, 5))
+    views = (fc.fc_datastore * 1)(fc.fc_datastore(1, 1, 1, 1, 10, 5))
     assert L.fc_retrieve(views, 1, 1, 64, 1, 4, nul, fc.params(40, 2, 16, 8), 1, 1, 1, 1, 1, nul) == 2
     assert L.fc_retrieve(views, 1, 1, 64, 1, 4, nul, fc.params(16, 2, 16, 8, 0), 1, 1, 1, 1, 1, nul) == 2
     # empty batch is a no-op
@@ -69,10 +69,10 @@ def test_host_validation_without_gpu(lib):
     assert L.fc_build_tree(2, 1, 1, 1, 1, w, 64, 10, 1, 1, 4, 65, 64, *tree_ptrs, nul) == 1
     assert L.fc_build_tree(2, 1, 1, 1, 1, w, 300, 10, 1, 1, 4, 64, 64, *tree_ptrs, nul) == 2
     # datastore: empty corpus, short workspace
-    assert L.fc_datastore_build(1, 0, 10, 1, 1, 1, 1 << 20, nul, nul) == 1
+    assert L.fc_datastore_build(1, 0, 10, 1, 1, 1, 1, 1 << 20, nul, nul) == 1
     need = L.fc_datastore_build_workspace(1000, 10)
     assert need > 1000 * 28
-    assert L.fc_datastore_build(1, 1000, 10, 1, 1, 256, need - 1, nul, nul) == 3
+    assert L.fc_datastore_build(1, 1000, 10, 1, 1, 1, 256, need - 1, nul, nul) == 3
     # kv append: aliasing in/out lengths
     assert L.fc_kv_append(1, 1, 1, 1, 16, 16, 2, 64, 8, 128, 12, 16, 16, 100, 8, 8, 1, 64, 4, 12, 1, nul) == 1
     # cache: capacity must be a power of two

@@ -43,6 +43,16 @@ def check_datastore(orc, ds, T, vocab):
     counts = np.bincount(T, minlength=vocab).astype(np.int64)
     closed = np.concatenate([[0], np.cumsum(counts)])
     assert np.array_equal(host_u32(ds.bucket).astype(np.int64), closed)
+    # LCP of adjacent suffixes, from the definition, at sampled SA positions
+    lcp = ds.lcp.cpu().numpy()
+    assert lcp[0] == 0
+    n = len(T)
+    for j in synth.rng_for(99).integers(1, n, 2000):
+        a, b = int(sa[j - 1]), int(sa[j])
+        l = 0
+        while l < 255 and a + l < n and b + l < n and T[a + l] == T[b + l]:
+            l += 1
+        assert lcp[j] == l, j
 
 
 def compare_rows(g, r, rows):

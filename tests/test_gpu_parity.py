@@ -58,8 +58,10 @@ def test_sa_small_sweep(fc, orc, n, vocab, seed):
         T[n // 3:n // 3 + 60] = T[:60]  # a long repeat
     ds = fc.fc_datastore_build(dev(T), vocab)
     torch.cuda.synchronize()
-    assert np.array_equal(host_u32(ds.sa), orc.suffix_array(T))
-    assert np.array_equal(host_u32(ds.bucket), orc.bucket(T, orc.suffix_array(T), vocab))
+    sa = orc.suffix_array(T)
+    assert np.array_equal(host_u32(ds.sa), sa)
+    assert np.array_equal(host_u32(ds.bucket), orc.bucket(T, sa, vocab))
+    assert np.array_equal(ds.lcp.cpu().numpy(), orc.lcp(T, sa))
 
 
 def test_sa_constant_corpus(fc, orc):
@@ -89,6 +91,7 @@ def test_sa_c1_corpus(fc, orc, c1):
     sa = orc.suffix_array(c1["T"])
     assert np.array_equal(host_u32(c1["ds"].sa), sa)
     assert np.array_equal(host_u32(c1["ds"].bucket), orc.bucket(c1["T"], sa, synth.VOCAB))
+    assert np.array_equal(c1["ds"].lcp.cpu().numpy(), orc.lcp(c1["T"], sa))
 
 
 # --------------------------------------------------------------- retrieval

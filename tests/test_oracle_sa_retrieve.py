@@ -53,6 +53,24 @@ def test_sa_parallel_merge_path(orc):
     assert orc.sa_certificate(T, sa8) == -1
 
 
+@pytest.mark.parametrize("seed", range(6))
+def test_lcp_brute_force(orc, seed):
+    rng = np.random.default_rng(40 + seed)
+    n = int(rng.integers(1, 800))
+    T = rng.integers(0, 1 + seed % 3, n).astype(np.uint32)  # tiny vocabularies: long common prefixes
+    sa = orc.suffix_array(T)
+    cap = [255, 5, 255, 1, 40, 255][seed]
+    got = orc.lcp(T, sa, cap)
+    Tl = T.tolist()
+    assert got[0] == 0
+    for j in range(1, n):
+        a, b = Tl[sa[j - 1]:], Tl[sa[j]:]
+        l = 0
+        while l < min(len(a), len(b)) and a[l] == b[l]:
+            l += 1
+        assert got[j] == min(l, cap)
+
+
 def test_sa_certificate_rejects(orc):
     rng = np.random.default_rng(1)
     T = rng.integers(0, 4, 500).astype(np.uint32)

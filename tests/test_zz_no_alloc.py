@@ -40,23 +40,25 @@ def _noalloc_call(fc, tokens, vocab):
     n = tokens.numel()
     sa = torch.full((n,), -5, dtype=torch.int32, device="cuda")
     bucket = torch.full((vocab + 1,), -5, dtype=torch.int32, device="cuda")
+    lcp = torch.full((n,), 7, dtype=torch.uint8, device="cuda")
     view = fc.fc_datastore()
     rc = fc.LIB.fc_datastore_build_noalloc(C.c_void_p(tokens.data_ptr()), n, vocab, C.c_void_p(sa.data_ptr()),
-                                           C.c_void_p(bucket.data_ptr()),
+                                           C.c_void_p(bucket.data_ptr()), C.c_void_p(lcp.data_ptr()),
                                            C.c_void_p(torch.cuda.current_stream().cuda_stream), C.byref(view))
     assert rc == 0, fc.STATUS.get(rc, rc)
-    assert view.n_tokens == n and view.vocab == vocab and view.sa == sa.data_ptr()
-    return sa, bucket
+    assert view.n_tokens == n and view.vocab == vocab and view.sa == sa.data_ptr() and view.lcp == lcp.data_ptr()
+    return sa, bucket, lcp
 
 
 def test_noalloc_build_matches_regular_build(fc):
     for seed, n, vocab in ((1, 1 << 20, 32256), (2, 300_001, 7)):
         tokens = _corpus(seed, n, vocab)
-        sa, bucket = _noalloc_call(fc, tokens, vocab)
+        sa, bucket, lcp = _noalloc_call(fc, tokens, vocab)
         ref = fc.fc_datastore_build(tokens, vocab)
         torch.cuda.synchronize()
         assert torch.equal(sa, ref.sa), (seed, n)
         assert torch.equal(bucket, ref.bucket), (seed, n)
+        assert torch.equal(lcp, ref.lcp), (seed, n)
     assert fc.fc_get_error() == "FC_OK"
 
 
@@ -64,5 +66,5 @@ def test_noalloc_rejects_oversized_corpus(fc):
     n = fc.NOALLOC_MAX_TOKENS + 1
     tokens = torch.zeros(n, dtype=torch.int32, device="cuda")
     rc = fc.LIB.fc_datastore_build_noalloc(C.c_void_p(tokens.data_ptr()), n, 4, C.c_void_p(tokens.data_ptr()),
-                                           C.c_void_p(tokens.data_ptr()), None, None)
+                                           C.c_void_p(tokens.data_ptr()), C.c_void_p(tokens.data_ptr()), None, None)
     assert fc.STATUS[rc] == "FC_ERR_CAPACITY"
