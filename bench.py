@@ -243,12 +243,15 @@ def run_ours(args, rank, ws, local):
     stream = torch.cuda.current_stream()
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     ev_ret = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    ev_tree = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    ev_tail = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
 
     def do_step(s, timed_idx=None):
         j = s % P
         if timed_idx is not None:
             loop.step(q_pool[j], kt_pool[j], vt_pool[j], hits_d[s], plen_d[s], rtok_d[s],
-                      events=dict(attn=ev[timed_idx], retrieve=ev_ret[timed_idx]))
+                      events=dict(attn=ev[timed_idx], retrieve=ev_ret[timed_idx], tree=ev_tree[timed_idx],
+                                  tail=ev_tail[timed_idx]))
         else:
             loop.step(q_pool[j], kt_pool[j], vt_pool[j], hits_d[s], plen_d[s], rtok_d[s])
 
@@ -272,6 +275,8 @@ def run_ours(args, rank, ws, local):
     t_max = max_over_ranks(t_ms, ws)
     attn_ms = [a.elapsed_time(b) for a, b in ev]
     ret_ms = [a.elapsed_time(b) for a, b in ev_ret]
+    tree_ms = [a.elapsed_time(b) for a, b in ev_tree]
+    tail_ms = [a.elapsed_time(b) for a, b in ev_tail]
 
     # replay the same (deterministic) trajectory untimed to count the
     # attention work of every timed launch
@@ -312,7 +317,8 @@ def run_ours(args, rank, ws, local):
         "gpu_launches": 8 * K,
         "clocks": clock_rec,
         "stages_ms_per_step": {"tree_attn": statistics.mean(attn_ms), "retrieve": statistics.mean(ret_ms),
-                               "all": t_ms / K},
+                               "build_tree": statistics.mean(tree_ms),
+                               "argmax_accept_append": statistics.mean(tail_ms), "all": t_ms / K},
         "queries_per_s": ws * B * K / (t_max * 1e-3),
         "retrievals_per_s": ws * (2 * (B * K - hits_used)) / (t_max * 1e-3),
         "tree_attn_tflops": tot_f / tot_t / 1e12,

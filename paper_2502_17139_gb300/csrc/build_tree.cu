@@ -5,8 +5,8 @@
 //
 // One CTA per query, everything in shared memory, no pointer trie:
 //   1. gather the drafts of all sources with weight w = src_weight * count;
-//   2. sort them lexicographically (rank by counting) and merge duplicates
-//      across sources (weights add);
+//   2. sort them lexicographically (bitonic sort of indices) and merge
+//      duplicates across sources (weights add);
 //   3. with neighbour LCPs, every trie node is a pair (u, l): the prefix of
 //      length l of sorted unique draft u, new at u when l > lcp(u-1, u).
 //      Its weight is the weight sum of the contiguous run of drafts that
@@ -64,7 +64,7 @@ __host__ __device__ inline BtLayout bt_layout(int M, int d) {
   L.tok = take((size_t)M * d * 4);
   L.len = take((size_t)M * 4);
   L.w = take((size_t)M * 8);
-  L.order = take((size_t)M * 4);
+  L.order = take((size_t)next_pow2((uint32_t)(M > 0 ? M : 1)) * 4);
   L.uniq = take((size_t)M * 4);
   L.wu = take((size_t)M * 8);
   L.ps = take((size_t)(M + 1) * 8);
@@ -172,17 +172,33 @@ __global__ void __launch_bounds__(BT_THREADS) k_build_tree(TreeIn in, int S, int
   }
   __syncthreads();
 
-  // 2. sort by counting rank; equal drafts keep (source, slot) order
-  for (uint32_t i = tid; i < M; i += BT_THREADS) {
-    uint32_t r = 0;
-    const uint32_t* a = tok + i * d;
-    for (uint32_t j = 0; j < M; ++j) {
-      int c = cmp_draft(tok + j * d, len[j], a, len[i]);
-      r += (c < 0 || (c == 0 && j < i)) ? 1u : 0u;
-    }
-    order[r] = i;
-  }
+  // 2. bitonic sort of draft indices by token sequence; equal drafts keep
+  //    (source, slot) order through the index tie-break
+  const uint32_t PM = next_pow2(M > 0 ? M : 1);
+  for (uint32_t i = tid; i < PM; i += BT_THREADS) order[i] = (i < M) ? i : 0xFFFFFFFFu;
   __syncthreads();
+  auto draft_less = [&](uint32_t x, uint32_t y) -> bool {  // sentinels sort last
+    if (x == 0xFFFFFFFFu) return false;
+    if (y == 0xFFFFFFFFu) return true;
+    const int c = cmp_draft(tok + x * d, len[x], tok + y * d, len[y]);
+    return c < 0 || (c == 0 && x < y);
+  };
+  for (uint32_t size = 2; size <= PM; size <<= 1) {
+    for (uint32_t st = size >> 1; st > 0; st >>= 1) {
+      for (uint32_t i = tid; i < PM; i += BT_THREADS) {
+        const uint32_t j = i ^ st;
+        if (j > i) {
+          const uint32_t x = order[i], y = order[j];
+          const bool asc = (i & size) == 0;
+          if (asc ? draft_less(y, x) : draft_less(x, y)) {
+            order[i] = y;
+            order[j] = x;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
   for (uint32_t r = tid; r < M; r += BT_THREADS) {
     uint32_t i = order[r];
     flag[r] = (r == 0 || cmp_draft(tok + order[r - 1] * d, len[order[r - 1]], tok + i * d, len[i]) != 0) ? 1u : 0u;

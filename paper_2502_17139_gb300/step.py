@@ -54,8 +54,8 @@ class StepLoop:
     def step(self, q, k_tree, v_tree, want_hit, plen, rtok, attention=True, events=None):
         """Enqueue one step.  q [B, Np, H, D], k_tree/v_tree [B, Hkv, Np, D]
         (bf16); want_hit [B], plen [B], rtok [B, Np] (int32).  ``events``
-        optionally maps "retrieve" / "attn" to (start, end) CUDA events
-        recorded around those stages on the current stream."""
+        optionally maps "retrieve" / "tree" / "attn" / "tail" to (start, end)
+        CUDA events recorded around those stages on the current stream."""
         c, n = self.cur, 1 - self.cur
         ev = events or {}
         if "retrieve" in ev:
@@ -68,8 +68,12 @@ class StepLoop:
             fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, out=self.res)
         if "retrieve" in ev:
             ev["retrieve"][1].record()
+        if "tree" in ev:
+            ev["tree"][0].record()
         fc.fc_build_tree(self.res, self.src_weight, self.root, self.kv_len[c], self.node_budget, self.n_pad,
                          out=self.tree)
+        if "tree" in ev:
+            ev["tree"][1].record()
         if attention:
             if "attn" in ev:
                 ev["attn"][0].record()
@@ -77,12 +81,16 @@ class StepLoop:
                             self.tree["n_nodes"], out=self.attn_out)
             if "attn" in ev:
                 ev["attn"][1].record()
+        if "tail" in ev:
+            ev["tail"][0].record()
         fc.fc_synth_argmax(self.tree["tok"], self.tree["parent"], self.tree["n_nodes"], plen, rtok, self.vocab,
                            out=self.argmax)
         fc.fc_accept(self.tree["tok"], self.tree["parent"], self.tree["n_nodes"], self.argmax, self.path_cap,
                      out=self.acc)
         fc.fc_kv_append(self.acc, self.tree["tok"], k_tree, v_tree, self.k_cache, self.v_cache, self.kv_len[c],
                         self.kv_len[n], self.ctx, self.ctx_len[c], self.ctx_len[n], self.root)
+        if "tail" in ev:
+            ev["tail"][1].record()
         self.cur = n
 
     def reset(self):
