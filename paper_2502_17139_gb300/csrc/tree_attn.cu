@@ -78,9 +78,12 @@ struct AttnArgs {
   float scale_log2;
 };
 
+// 2^x on the MUFU unit.  The flush-to-zero form is a single instruction; the
+// results it flushes (below 2^-126) are probabilities that cannot move an
+// fp32 row sum whose largest term is >= 1.
 __device__ __forceinline__ float fast_exp2(float x) {
   float y;
-  asm("ex2.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
 
