@@ -53,6 +53,13 @@ constexpr uint64_t DRAIN_CYCLES = 400000000ull;            // ~0.2 s
 // (base-2 logits) grows by more than this; until then probabilities may reach
 // 2^RESCALE_THRESHOLD, harmless in bf16/fp32.
 constexpr float RESCALE_THRESHOLD = 8.f;
+// Register split (setmaxnreg): the kernel launches with REGS_LAUNCH per
+// thread; the TMA/MMA warpgroup drops to REGS_PRODUCER and the two softmax
+// warpgroups rise to REGS_SOFTMAX, enough to hold a row's 128 scores.  The
+// shares must add up to the launch's allocation or the increase never returns;
+// the host checks the compiled register count before launching.
+constexpr int REGS_LAUNCH = 168, REGS_PRODUCER = 40, REGS_SOFTMAX = 232;
+static_assert(128 * REGS_PRODUCER + 256 * REGS_SOFTMAX <= TA_THREADS * REGS_LAUNCH, "register split");
 
 // barrier slots (8 bytes each)
 enum {
@@ -112,34 +119,14 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   return d;
 }
 
-// 2^x for a pair on the FMA pipe (offloads the MUFU unit).  Round-to-nearest
-// range reduction x = n + f, f in [-1/2, 1/2] (adding 1.5 * 2^23 leaves n in
-// the low mantissa bits), p(f) = 1 + c1 f + c2 f^2 + c3 f^3 (least-squares fit
-// of 2^f, relative error <= 1.8e-4, see exp2_poly_fit.py), then n is added to
-// the exponent field.  Inputs are clamped to >= -125 so the result stays a
-// normal number (2^-125 is nil next to the row maximum's 1).
-__device__ __forceinline__ void exp2_poly_pair(uint64_t x2, float& p0, float& p1) {
-  constexpr float kRound = 12582912.f;  // 1.5 * 2^23
-  float x0, x1;
-  f2_unpack(x2, x0, x1);
-  x2 = f2_pack(fmaxf(x0, -125.f), fmaxf(x1, -125.f));
-  const uint64_t t2 = f2_add(x2, f2_pack(kRound, kRound));
-  const uint64_t r2 = f2_add(t2, f2_pack(-kRound, -kRound));
-  const uint64_t fr = f2_fma(r2, f2_pack(-1.f, -1.f), x2);
-  uint64_t p2 = f2_fma(f2_pack(0.054602622985839844f, 0.054602622985839844f), fr,
-                       f2_pack(0.24192412197589874f, 0.24192412197589874f));
-  p2 = f2_fma(p2, fr, f2_pack(0.6933164596557617f, 0.6933164596557617f));
-  p2 = f2_fma(p2, fr, f2_pack(1.f, 1.f));
-  float t0, t1, q0, q1;
-  f2_unpack(t2, t0, t1);
-  f2_unpack(p2, q0, q1);
-  p0 = __int_as_float(__float_as_int(q0) + (__float_as_int(t0) << 23));
-  p1 = __int_as_float(__float_as_int(q1) + (__float_as_int(t1) << 23));
+template <int N>
+__device__ __forceinline__ void regs_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
 }
-
-// Which score pairs of a 32-column chunk take the polynomial exp2 (1 in 4):
-// the MUFU unit handles the rest, and the two pipes finish together.
-__device__ __forceinline__ constexpr bool poly_pair(int q) { return (q & 3) == 3; }
+template <int N>
+__device__ __forceinline__ void regs_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
 
 // All 32 lanes wait; the result is warp-uniform.
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
@@ -216,159 +203,162 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = s_tmem;
-
-  if (warp == 0) {
-    // ---------------- TMA producer ----------------
-    if (lane == 0) {
-      int issued = 0;
-      for (int j = 0; j < nblk; ++j) {
-        const int st = j & 1;
-        const bool tree = j >= nblk_c;
-        const uint32_t bytes = tree ? (uint32_t)a.n_pad * 64 * 2 * 2 : TILE_BYTES;
-        const CUtensorMap* mk = tree ? &tm_kt : &tm_kc;
-        const CUtensorMap* mv = tree ? &tm_vt : &tm_vc;
-        const int y = tree ? 0 : j * BN;
-        if (j >= 2 && !mbar_wait_bounded(bar(B_KEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) break;
-        const uint32_t dK = sK + st * TILE_BYTES, dV = sV + st * TILE_BYTES;
-        mbar_expect_tx(bar(B_KFULL + st), bytes);
-        tma_load_3d(dK, mk, 0, y, bg, bar(B_KFULL + st));
-        tma_load_3d(dK + HALF_BYTES, mk, 64, y, bg, bar(B_KFULL + st));
-        if (j >= 2 && !mbar_wait_bounded(bar(B_VEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) {
-          issued = j + 1;  // the K copy of this block is in flight
-          break;
+  if (warp < 4) {
+    regs_dec<REGS_PRODUCER>();  // the whole warpgroup (warps 2 and 3 only wait)
+    if (warp == 0) {
+      // ---------------- TMA producer ----------------
+      if (lane == 0) {
+        int issued = 0;
+        for (int j = 0; j < nblk; ++j) {
+          const int st = j & 1;
+          const bool tree = j >= nblk_c;
+          const uint32_t bytes = tree ? (uint32_t)a.n_pad * 64 * 2 * 2 : TILE_BYTES;
+          const CUtensorMap* mk = tree ? &tm_kt : &tm_kc;
+          const CUtensorMap* mv = tree ? &tm_vt : &tm_vc;
+          const int y = tree ? 0 : j * BN;
+          if (j >= 2 && !mbar_wait_bounded(bar(B_KEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) break;
+          const uint32_t dK = sK + st * TILE_BYTES, dV = sV + st * TILE_BYTES;
+          mbar_expect_tx(bar(B_KFULL + st), bytes);
+          tma_load_3d(dK, mk, 0, y, bg, bar(B_KFULL + st));
+          tma_load_3d(dK + HALF_BYTES, mk, 64, y, bg, bar(B_KFULL + st));
+          if (j >= 2 && !mbar_wait_bounded(bar(B_VEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) {
+            issued = j + 1;  // the K copy of this block is in flight
+            break;
+          }
+          mbar_expect_tx(bar(B_VFULL + st), bytes);
+          tma_load_3d(dV, mv, 0, y, bg, bar(B_VFULL + st));
+          tma_load_3d(dV + HALF_BYTES, mv, 64, y, bg, bar(B_VFULL + st));
+          issued = j + 1;
         }
-        mbar_expect_tx(bar(B_VFULL + st), bytes);
-        tma_load_3d(dV, mv, 0, y, bg, bar(B_VFULL + st));
-        tma_load_3d(dV + HALF_BYTES, mv, 64, y, bg, bar(B_VFULL + st));
-        issued = j + 1;
-      }
-      if (s_abort) {  // let the copies already issued land before the CTA exits
-        volatile int dummy = 0;
-        for (int j = max(0, issued - 2); j < issued; ++j) {
-          mbar_wait_bounded(bar(B_KFULL + (j & 1)), (j >> 1) & 1, &dummy, DRAIN_CYCLES);
-          mbar_wait_bounded(bar(B_VFULL + (j & 1)), (j >> 1) & 1, &dummy, DRAIN_CYCLES);
+        if (s_abort) {  // let the copies already issued land before the CTA exits
+          volatile int dummy = 0;
+          for (int j = max(0, issued - 2); j < issued; ++j) {
+            mbar_wait_bounded(bar(B_KFULL + (j & 1)), (j >> 1) & 1, &dummy, DRAIN_CYCLES);
+            mbar_wait_bounded(bar(B_VFULL + (j & 1)), (j >> 1) & 1, &dummy, DRAIN_CYCLES);
+          }
         }
-      }
-    }
-    __syncwarp();
-  } else if (warp == 1) {
-    // ---------------- MMA issuer (+ ragged V rows zeroed by the warp) -------
-    constexpr uint32_t IDESC_QK = idesc_bf16_f32(BM, BN, 0);
-    constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, HD, 1);
-    // S buffer sb (TMEM columns sb*128..) <- Q tile x . K(j)^T; arrives on S_FULL[sb]
-    auto issue_qk = [&](int j, int x, int sb) {
-      const uint32_t kb = sK + (j & 1) * TILE_BYTES, qb = sQ + x * TILE_BYTES;
-#pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) {
-        const uint32_t off = (kk >> 2) * HALF_BYTES + (kk & 3) * 32;
-        tc_mma_f16(tmem + sb * 128, smem_desc_sw128(qb + off, 16, 1024), smem_desc_sw128(kb + off, 16, 1024),
-                   IDESC_QK, kk > 0);
-      }
-      tc_commit(bar(B_SFULL + sb));
-    };
-    // O tile x += P (bf16 pairs in the first 64 columns of S buffer sb) . V(jj)
-    auto issue_pv = [&](int jj, int x, int sb, int) {
-      const uint32_t vb = sV + (jj & 1) * TILE_BYTES;
-#pragma unroll
-      for (int kk = 0; kk < BN / 16; ++kk)  // 8 packed columns per 16 keys
-        tc_mma_f16_tmem_a(tmem + 256 + x * 128, tmem + sb * 128 + kk * 8,
-                          smem_desc_sw128(vb + kk * 2048, HALF_BYTES, 1024), IDESC_PV, (jj > 0 || kk > 0));
-    };
-    auto zero_ragged_v = [&](int jj) {  // never let garbage (possibly NaN) rows meet a zero probability
-      const int nv = (jj < nblk_c) ? min(BN, kvl - jj * BN) : nn;
-      if (nv < BN) {
-        unsigned char* vt = smem + OFF_V + (jj & 1) * TILE_BYTES;
-        for (int e = lane; e < (BN - nv) * 16; e += 32) {
-          const int r = nv + (e >> 4), ch = e & 15;
-          *reinterpret_cast<uint4*>(vt + (ch >> 3) * HALF_BYTES + r * 128 + (ch & 7) * 16) = make_uint4(0, 0, 0, 0);
-        }
-        fence_proxy_async_smem();
       }
       __syncwarp();
-    };
-    bool ok = true;
-    if (has_b) {
-      // Two tiles, one S buffer each: per tile PV_X(j-1) -> QK_X(j); the
-      // other tile's softmax runs meanwhile.
-      ok = warp_wait(bar(B_KFULL), 0, &s_abort);
-      if (ok) {
-        if (lane == 0) {
-          tc_fence_after();
-          for (int x = 0; x < 2; ++x) issue_qk(0, x, x);
-          tc_commit(bar(B_KEMPTY));
+    } else if (warp == 1) {
+      // ---------------- MMA issuer (+ ragged V rows zeroed by the warp) -------
+      constexpr uint32_t IDESC_QK = idesc_bf16_f32(BM, BN, 0);
+      constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, HD, 1);
+      // S buffer sb (TMEM columns sb*128..) <- Q tile x . K(j)^T; arrives on S_FULL[sb]
+      auto issue_qk = [&](int j, int x, int sb) {
+        const uint32_t kb = sK + (j & 1) * TILE_BYTES, qb = sQ + x * TILE_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * HALF_BYTES + (kk & 3) * 32;
+          tc_mma_f16(tmem + sb * 128, smem_desc_sw128(qb + off, 16, 1024), smem_desc_sw128(kb + off, 16, 1024),
+                     IDESC_QK, kk > 0);
+        }
+        tc_commit(bar(B_SFULL + sb));
+      };
+      // O tile x += P (bf16 pairs in the first 64 columns of S buffer sb) . V(jj)
+      auto issue_pv = [&](int jj, int x, int sb, int) {
+        const uint32_t vb = sV + (jj & 1) * TILE_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk)  // 8 packed columns per 16 keys
+          tc_mma_f16_tmem_a(tmem + 256 + x * 128, tmem + sb * 128 + kk * 8,
+                            smem_desc_sw128(vb + kk * 2048, HALF_BYTES, 1024), IDESC_PV, (jj > 0 || kk > 0));
+      };
+      auto zero_ragged_v = [&](int jj) {  // never let garbage (possibly NaN) rows meet a zero probability
+        const int nv = (jj < nblk_c) ? min(BN, kvl - jj * BN) : nn;
+        if (nv < BN) {
+          unsigned char* vt = smem + OFF_V + (jj & 1) * TILE_BYTES;
+          for (int e = lane; e < (BN - nv) * 16; e += 32) {
+            const int r = nv + (e >> 4), ch = e & 15;
+            *reinterpret_cast<uint4*>(vt + (ch >> 3) * HALF_BYTES + r * 128 + (ch & 7) * 16) = make_uint4(0, 0, 0, 0);
+          }
+          fence_proxy_async_smem();
         }
         __syncwarp();
-      }
-      for (int j = 1; ok && j <= nblk; ++j) {
-        const int jj = j - 1, st = jj & 1;
-        if (!(ok = warp_wait(bar(B_VFULL + st), (jj >> 1) & 1, &s_abort))) break;
-        zero_ragged_v(jj);
-        for (int x = 0; ok && x < 2; ++x) {
-          if (!(ok = warp_wait(bar(B_PFULL + x), jj & 1, &s_abort))) break;
+      };
+      bool ok = true;
+      if (has_b) {
+        // Two tiles, one S buffer each: per tile PV_X(j-1) -> QK_X(j); the
+        // other tile's softmax runs meanwhile.
+        ok = warp_wait(bar(B_KFULL), 0, &s_abort);
+        if (ok) {
           if (lane == 0) {
             tc_fence_after();
-            issue_pv(jj, x, x, x);
-            tc_commit(bar(B_ODONE + x));
+            for (int x = 0; x < 2; ++x) issue_qk(0, x, x);
+            tc_commit(bar(B_KEMPTY));
           }
           __syncwarp();
-          if (j < nblk) {
-            if (x == 0 && !(ok = warp_wait(bar(B_KFULL + (j & 1)), (j >> 1) & 1, &s_abort))) break;
-            if (lane == 0) issue_qk(j, x, x);
+        }
+        for (int j = 1; ok && j <= nblk; ++j) {
+          const int jj = j - 1, st = jj & 1;
+          if (!(ok = warp_wait(bar(B_VFULL + st), (jj >> 1) & 1, &s_abort))) break;
+          zero_ragged_v(jj);
+          for (int x = 0; ok && x < 2; ++x) {
+            if (!(ok = warp_wait(bar(B_PFULL + x), jj & 1, &s_abort))) break;
+            if (lane == 0) {
+              tc_fence_after();
+              issue_pv(jj, x, x, x);
+              tc_commit(bar(B_ODONE + x));
+            }
             __syncwarp();
-          } else if (lane == 0) {
-            tc_commit(bar(B_OFIN + x));
+            if (j < nblk) {
+              if (x == 0 && !(ok = warp_wait(bar(B_KFULL + (j & 1)), (j >> 1) & 1, &s_abort))) break;
+              if (lane == 0) issue_qk(j, x, x);
+              __syncwarp();
+            } else if (lane == 0) {
+              tc_commit(bar(B_OFIN + x));
+            }
           }
-        }
-        if (!ok) break;
-        if (lane == 0) {
-          if (j < nblk) tc_commit(bar(B_KEMPTY + (j & 1)));
-          tc_commit(bar(B_VEMPTY + st));
-        }
-        __syncwarp();
-      }
-    } else {
-      // One tile, S double-buffered in both S regions: QK(j+1) runs during
-      // softmax(j); PV(j) reads P from S(j&1) before QK(j+2) overwrites it.
-      for (int j = 0; ok && j < min(2, nblk); ++j) {
-        if (!(ok = warp_wait(bar(B_KFULL + j), 0, &s_abort))) break;
-        if (lane == 0) {
-          tc_fence_after();
-          issue_qk(j, 0, j);
-          tc_commit(bar(B_KEMPTY + j));
-        }
-        __syncwarp();
-      }
-      for (int jj = 0; ok && jj < nblk; ++jj) {
-        const int v = jj & 1;
-        if (!(ok = warp_wait(bar(B_VFULL + v), (jj >> 1) & 1, &s_abort))) break;
-        zero_ragged_v(jj);
-        if (!(ok = warp_wait(bar(B_PFULL + v), (jj >> 1) & 1, &s_abort))) break;
-        if (lane == 0) {
-          tc_fence_after();
-          issue_pv(jj, 0, v, 0);
-          tc_commit(bar(B_ODONE));
-          tc_commit(bar(B_VEMPTY + v));
-          if (jj == nblk - 1) tc_commit(bar(B_OFIN));
-        }
-        __syncwarp();
-        if (jj + 2 < nblk) {
-          if (!(ok = warp_wait(bar(B_KFULL + v), ((jj + 2) >> 1) & 1, &s_abort))) break;
+          if (!ok) break;
           if (lane == 0) {
-            tc_fence_after();
-            issue_qk(jj + 2, 0, v);
-            tc_commit(bar(B_KEMPTY + v));
+            if (j < nblk) tc_commit(bar(B_KEMPTY + (j & 1)));
+            tc_commit(bar(B_VEMPTY + st));
           }
           __syncwarp();
         }
+      } else {
+        // One tile, S double-buffered in both S regions: QK(j+1) runs during
+        // softmax(j); PV(j) reads P from S(j&1) before QK(j+2) overwrites it.
+        for (int j = 0; ok && j < min(2, nblk); ++j) {
+          if (!(ok = warp_wait(bar(B_KFULL + j), 0, &s_abort))) break;
+          if (lane == 0) {
+            tc_fence_after();
+            issue_qk(j, 0, j);
+            tc_commit(bar(B_KEMPTY + j));
+          }
+          __syncwarp();
+        }
+        for (int jj = 0; ok && jj < nblk; ++jj) {
+          const int v = jj & 1;
+          if (!(ok = warp_wait(bar(B_VFULL + v), (jj >> 1) & 1, &s_abort))) break;
+          zero_ragged_v(jj);
+          if (!(ok = warp_wait(bar(B_PFULL + v), (jj >> 1) & 1, &s_abort))) break;
+          if (lane == 0) {
+            tc_fence_after();
+            issue_pv(jj, 0, v, 0);
+            tc_commit(bar(B_ODONE));
+            tc_commit(bar(B_VEMPTY + v));
+            if (jj == nblk - 1) tc_commit(bar(B_OFIN));
+          }
+          __syncwarp();
+          if (jj + 2 < nblk) {
+            if (!(ok = warp_wait(bar(B_KFULL + v), ((jj + 2) >> 1) & 1, &s_abort))) break;
+            if (lane == 0) {
+              tc_fence_after();
+              issue_qk(jj + 2, 0, v);
+              tc_commit(bar(B_KEMPTY + v));
+            }
+            __syncwarp();
+          }
+        }
+      }
+      if (s_abort) {  // let issued MMAs retire before the tensor memory is freed
+        if (lane == 0) tc_commit(bar(B_DRAIN));
+        __syncwarp();
+        volatile int dummy = 0;
+        mbar_wait_bounded(bar(B_DRAIN), 0, &dummy, DRAIN_CYCLES);
       }
     }
-    if (s_abort) {  // let issued MMAs retire before the tensor memory is freed
-      if (lane == 0) tc_commit(bar(B_DRAIN));
-      __syncwarp();
-      volatile int dummy = 0;
-      mbar_wait_bounded(bar(B_DRAIN), 0, &dummy, DRAIN_CYCLES);
-    }
-  } else if (warp >= 4) {
+  } else {
+    regs_inc<REGS_SOFTMAX>();
     // ---------------- softmax warpgroups: tile x, thread = row ----------------
     const int x = (warp - 4) >> 2;  // 0: warps 4-7, 1: warps 8-11
     const int q4 = warp & 3;        // TMEM lane quarter of this warp
@@ -400,33 +390,27 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
           const int lo = nv - 32 * q;
           return lo >= 32 ? 0xFFFFFFFFu : (lo <= 0 ? 0u : ((1u << lo) - 1u));
         };
-        // masked scores become -inf (exp2 turns them into exact zeros)
-        auto apply_mask = [&](int h2, uint32_t (&s0)[32], uint32_t (&s1)[32]) {
-          const uint32_t k0 = keep_bits(2 * h2), k1 = keep_bits(2 * h2 + 1);
+        // The block's 128 scores of this row stay in registers from here on.
+        uint32_t sv[128];
 #pragma unroll
-          for (int cc = 0; cc < 32; ++cc) {
-            if (!(k0 & (1u << cc))) s0[cc] = __float_as_uint(-INFINITY);
-            if (!(k1 & (1u << cc))) s1[cc] = __float_as_uint(-INFINITY);
+        for (int c4 = 0; c4 < 4; ++c4) tmem_ld32(tS + c4 * 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[c4 * 32]));
+        tc_wait_ld();
+        if (masked) {  // masked scores become -inf (exp2 turns them into exact zeros)
+#pragma unroll
+          for (int c4 = 0; c4 < 4; ++c4) {
+            const uint32_t kb = keep_bits(c4);
+#pragma unroll
+            for (int cc = 0; cc < 32; ++cc)
+              if (!(kb & (1u << cc))) sv[c4 * 32 + cc] = __float_as_uint(-INFINITY);
           }
-        };
-        // pass 1: raw row maximum over the block (scale > 0 commutes with max)
+        }
+        // raw row maximum over the block (scale > 0 commutes with max)
         float pm[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
 #pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
-          uint32_t s0[32], s1[32];
-          tmem_ld32(tS + h2 * 64, s0);
-          tmem_ld32(tS + h2 * 64 + 32, s1);
-          tc_wait_ld();
-          if (masked) apply_mask(h2, s0, s1);
-#pragma unroll
-          for (int cc = 0; cc < 32; cc += 2) {
-            pm[(cc >> 1) & 7] = fmax3(pm[(cc >> 1) & 7], __uint_as_float(s0[cc]), __uint_as_float(s0[cc + 1]));
-            pm[((cc >> 1) + 4) & 7] =
-                fmax3(pm[((cc >> 1) + 4) & 7], __uint_as_float(s1[cc]), __uint_as_float(s1[cc + 1]));
-          }
-        }
+        for (int cc = 0; cc < 128; cc += 2)
+          pm[(cc >> 1) & 7] = fmax3(pm[(cc >> 1) & 7], __uint_as_float(sv[cc]), __uint_as_float(sv[cc + 1]));
         const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
                                fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * a.scale_log2;
         // lazy rescale: keep the old reference unless the maximum grew a lot
@@ -448,49 +432,22 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
             tmem_st32(tO + cc * 32, o);
           }
         }
-        // pass 2: P = exp2(s * scale - m), bf16 pairs written over S's first 64 columns
+        // P = exp2(s * scale - m), bf16 pairs written over S's first 64 columns
         uint64_t ps2[4] = {0ull, 0ull, 0ull, 0ull};  // packed partial row sums
         const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2), nm2 = f2_pack(-m_use, -m_use);
 #pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
-          uint32_t s0[32], s1[32];
-          tmem_ld32(tS + h2 * 64, s0);
-          tmem_ld32(tS + h2 * 64 + 32, s1);
-          tc_wait_ld();
-          uint32_t pk[32];
-          if (masked) {  // masked keys are -inf: MUFU exp2 makes them exact zeros
-            apply_mask(h2, s0, s1);
+        for (int c4 = 0; c4 < 4; ++c4) {
+          uint32_t pk[16];
 #pragma unroll
-            for (int q = 0; q < 32; ++q) {
-              const uint32_t* src = q < 16 ? s0 : s1;
-              const int cc = 2 * (q & 15);
-              float x0, x1;
-              f2_unpack(f2_fma(f2_pack(__uint_as_float(src[cc]), __uint_as_float(src[cc + 1])), sc2, nm2), x0, x1);
-              const float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
-              ps2[q & 3] = f2_add(ps2[q & 3], f2_pack(p0, p1));
-              pk[q] = pack_bf16x2(p0, p1);
-            }
-          } else {
-#pragma unroll
-            for (int q = 0; q < 32; ++q) {
-              const uint32_t* src = q < 16 ? s0 : s1;
-              const int cc = 2 * (q & 15);
-              const uint64_t x2 = f2_fma(f2_pack(__uint_as_float(src[cc]), __uint_as_float(src[cc + 1])), sc2, nm2);
-              float p0, p1;
-              if (poly_pair(q)) {
-                exp2_poly_pair(x2, p0, p1);
-              } else {
-                float x0, x1;
-                f2_unpack(x2, x0, x1);
-                p0 = fast_exp2(x0);
-                p1 = fast_exp2(x1);
-              }
-              ps2[q & 3] = f2_add(ps2[q & 3], f2_pack(p0, p1));
-              pk[q] = pack_bf16x2(p0, p1);
-            }
+          for (int q = 0; q < 16; ++q) {
+            const int cc = c4 * 32 + 2 * q;
+            float x0, x1;
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sv[cc]), __uint_as_float(sv[cc + 1])), sc2, nm2), x0, x1);
+            const float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
+            ps2[q & 3] = f2_add(ps2[q & 3], f2_pack(p0, p1));
+            pk[q] = pack_bf16x2(p0, p1);
           }
-          tmem_st16(tS + h2 * 32, *reinterpret_cast<uint32_t(*)[16]>(&pk[0]));
-          tmem_st16(tS + h2 * 32 + 16, *reinterpret_cast<uint32_t(*)[16]>(&pk[16]));
+          tmem_st16(tS + c4 * 16, pk);
         }
         tc_wait_st();
         float ps[8];
@@ -591,6 +548,11 @@ extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const 
     return FC_ERR_CUDA;
   if (cudaFuncSetAttribute(k_tree_attn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES) != cudaSuccess)
     return FC_ERR_CUDA;
+  {  // the register split needs the whole launch allocation (see REGS_LAUNCH)
+    cudaFuncAttributes fa;
+    if (cudaFuncGetAttributes(&fa, k_tree_attn) != cudaSuccess) return FC_ERR_CUDA;
+    if (fa.numRegs < REGS_LAUNCH) return FC_ERR_INTERNAL;
+  }
   AttnArgs a;
   a.q = static_cast<const __nv_bfloat16*>(d_q);
   a.kv_len = d_kv_len;
