@@ -15,8 +15,9 @@
 //   * tcgen05.mma (bf16 in, fp32 accumulate): S_X = Q_X K^T into tensor
 //     memory; the softmax writes P_X (bf16) over the first half of S_X in
 //     tensor memory, and O_X += P_X V takes P_X straight from tensor memory
-//     (A operand) with V as an MN-major shared-memory operand.  One thread
-//     issues every MMA, in the order PV_X(j-1) -> QK_X(j) per tile, so S_X is
+//     (A operand) with V as an MN-major shared-memory operand.  One warp
+//     issues every MMA (warp-uniform, one lane elected inside each
+//     instruction), in the order PV_X(j-1) -> QK_X(j) per tile, so S_X is
 //     never overwritten before PV_X has read P_X from it.
 //   * two softmax warpgroups, one per tile, one row per thread: tile A's
 //     softmax runs while the tensor cores do tile B's PV and QK, and the
@@ -69,7 +70,7 @@ enum {
   B_VEMPTY = 6,  // [2] V tile consumed by both PV MMAs
   B_SFULL = 8,   // [2 tiles] S_X ready
   B_PFULL = 10,  // [2 tiles] P_X written (128 arrivals)
-  B_ODONE = 12,  // [2 tiles] a PV into O_X done (one completion per block)
+  B_ODONE = 12,  // one-tile CTAs: a PV into O done (one completion per block)
   B_DRAIN = 14,  // MMA drain on abort
   B_OFIN = 15,   // [2 tiles] the last PV into O_X done
   N_BARS = 17
@@ -280,12 +281,9 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         // other tile's softmax runs meanwhile.
         ok = warp_wait(bar(B_KFULL), 0, &s_abort);
         if (ok) {
-          if (lane == 0) {
-            tc_fence_after();
-            for (int x = 0; x < 2; ++x) issue_qk(0, x, x);
-            tc_commit(bar(B_KEMPTY));
-          }
-          __syncwarp();
+          tc_fence_after();
+          for (int x = 0; x < 2; ++x) issue_qk(0, x, x);
+          tc_commit(bar(B_KEMPTY));
         }
         for (int j = 1; ok && j <= nblk; ++j) {
           const int jj = j - 1, st = jj & 1;
@@ -293,66 +291,48 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
           zero_ragged_v(jj);
           for (int x = 0; ok && x < 2; ++x) {
             if (!(ok = warp_wait(bar(B_PFULL + x), jj & 1, &s_abort))) break;
-            if (lane == 0) {
-              tc_fence_after();
-              issue_pv(jj, x, x, x);
-              tc_commit(bar(B_ODONE + x));
-            }
-            __syncwarp();
+            tc_fence_after();
+            issue_pv(jj, x, x, x);
             if (j < nblk) {
               if (x == 0 && !(ok = warp_wait(bar(B_KFULL + (j & 1)), (j >> 1) & 1, &s_abort))) break;
-              if (lane == 0) issue_qk(j, x, x);
-              __syncwarp();
-            } else if (lane == 0) {
+              issue_qk(j, x, x);
+            } else {
               tc_commit(bar(B_OFIN + x));
             }
           }
           if (!ok) break;
-          if (lane == 0) {
-            if (j < nblk) tc_commit(bar(B_KEMPTY + (j & 1)));
-            tc_commit(bar(B_VEMPTY + st));
-          }
-          __syncwarp();
+          if (j < nblk) tc_commit(bar(B_KEMPTY + (j & 1)));
+          tc_commit(bar(B_VEMPTY + st));
         }
       } else {
         // One tile, S double-buffered in both S regions: QK(j+1) runs during
         // softmax(j); PV(j) reads P from S(j&1) before QK(j+2) overwrites it.
         for (int j = 0; ok && j < min(2, nblk); ++j) {
           if (!(ok = warp_wait(bar(B_KFULL + j), 0, &s_abort))) break;
-          if (lane == 0) {
-            tc_fence_after();
-            issue_qk(j, 0, j);
-            tc_commit(bar(B_KEMPTY + j));
-          }
-          __syncwarp();
+          tc_fence_after();
+          issue_qk(j, 0, j);
+          tc_commit(bar(B_KEMPTY + j));
         }
         for (int jj = 0; ok && jj < nblk; ++jj) {
           const int v = jj & 1;
           if (!(ok = warp_wait(bar(B_VFULL + v), (jj >> 1) & 1, &s_abort))) break;
           zero_ragged_v(jj);
           if (!(ok = warp_wait(bar(B_PFULL + v), (jj >> 1) & 1, &s_abort))) break;
-          if (lane == 0) {
-            tc_fence_after();
-            issue_pv(jj, 0, v, 0);
-            tc_commit(bar(B_ODONE));
-            tc_commit(bar(B_VEMPTY + v));
-            if (jj == nblk - 1) tc_commit(bar(B_OFIN));
-          }
-          __syncwarp();
+          tc_fence_after();
+          issue_pv(jj, 0, v, 0);
+          tc_commit(bar(B_ODONE));
+          tc_commit(bar(B_VEMPTY + v));
+          if (jj == nblk - 1) tc_commit(bar(B_OFIN));
           if (jj + 2 < nblk) {
             if (!(ok = warp_wait(bar(B_KFULL + v), ((jj + 2) >> 1) & 1, &s_abort))) break;
-            if (lane == 0) {
-              tc_fence_after();
-              issue_qk(jj + 2, 0, v);
-              tc_commit(bar(B_KEMPTY + v));
-            }
-            __syncwarp();
+            tc_fence_after();
+            issue_qk(jj + 2, 0, v);
+            tc_commit(bar(B_KEMPTY + v));
           }
         }
       }
-      if (s_abort) {  // let issued MMAs retire before the tensor memory is freed
-        if (lane == 0) tc_commit(bar(B_DRAIN));
-        __syncwarp();
+      if (__any_sync(0xFFFFFFFFu, s_abort)) {  // let issued MMAs retire before the tensor memory is freed
+        tc_commit(bar(B_DRAIN));
         volatile int dummy = 0;
         mbar_wait_bounded(bar(B_DRAIN), 0, &dummy, DRAIN_CYCLES);
       }
