@@ -263,14 +263,33 @@ fc_status fc_tree_mask(const int32_t* d_parent, const int32_t* d_n_nodes, const 
  *   d_mask    [batch][n_pad][n_pad/64] uint64 (fc_build_tree layout)
  *   d_n_nodes [batch] int32 in [1, n_pad]
  *   d_out     bf16 [batch][n_pad][H][D]
+ *   d_ws, ws_bytes  optional device workspace (may be NULL / 0).  With
+ *             fc_tree_attn_workspace() bytes the call may split each row
+ *             chunk's keys over up to 4 CTAs (so that the grid fills the GPU
+ *             in whole waves) and merge their partial softmax sums; with less
+ *             it uses fewer parts.  Owned by the caller, no initial contents
+ *             needed (the call clears its counters on the stream first).
+ *             Concurrent calls on different streams need separate workspaces.
  * Supported: D = 128, n_pad in {64, 128}, H % Hkv == 0, H / Hkv <= 16,
  * all device pointers 16-byte aligned.  Arithmetic: bf16 tensor-core
- * products with fp32 accumulation and an fp32 online softmax.
+ * products with fp32 accumulation and an fp32 online softmax; the split
+ * merge is fp32.  Results agree to rounding for every workspace size.
  */
 fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const void* d_v_cache, int kv_cap,
                        const int32_t* d_kv_len, const void* d_k_tree, const void* d_v_tree,
                        const uint64_t* d_mask, const int32_t* d_n_nodes, int batch, int n_pad,
-                       int H, int Hkv, int D, float scale, void* d_out, fc_stream s);
+                       int H, int Hkv, int D, float scale, void* d_out, void* d_ws,
+                       size_t ws_bytes, fc_stream s);
+
+/* Workspace bytes that let fc_tree_attn use its largest key split for this
+ * shape (0 for an unsupported shape).  Not part of the paper's method: a
+ * scheduling aid for filling the GPU. */
+size_t fc_tree_attn_workspace(int batch, int n_pad, int H, int Hkv);
+
+/* How many parts fc_tree_attn splits each row chunk's keys into for this
+ * shape and workspace size on the current device (1 = no split; 0 for an
+ * unsupported shape).  Host-only, launches nothing. */
+int fc_tree_attn_parts(int batch, int n_pad, int H, int Hkv, int kv_cap, size_t ws_bytes);
 
 /* ------------------------------------------------------------------------
  * Acceptance (Section IV-D: every correct token from the start is accepted,

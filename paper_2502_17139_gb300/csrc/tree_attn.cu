@@ -27,6 +27,7 @@
 //     FC_ERR_TIMEOUT, the CTA drains its in-flight copies and MMAs (bounded
 //     again), frees its tensor memory and returns.
 #include <algorithm>
+#include <cmath>
 #include <mutex>
 
 #include "fc_common.cuh"
@@ -40,6 +41,7 @@ constexpr int BM = 128;          // query rows per tile
 constexpr int TILES = 2;         // tiles per CTA
 constexpr int BN = 128;          // keys per block
 constexpr int HD = 128;          // head dim
+constexpr int MAX_PARTS = 4;     // most CTAs one unit's KV blocks are split over
 constexpr uint32_t HALF_BYTES = BN * 64 * 2;  // one 64-dim half of a 128-row tile
 constexpr uint32_t TILE_BYTES = 2 * HALF_BYTES;
 constexpr uint32_t OFF_Q = 0;                              // Q_A, Q_B
@@ -59,7 +61,7 @@ constexpr float RESCALE_THRESHOLD = 8.f;
 // warpgroups rise to REGS_SOFTMAX, enough to hold a row's 128 scores.  The
 // shares must add up to the launch's allocation or the increase never returns;
 // the host checks the compiled register count before launching.
-constexpr int REGS_LAUNCH = 168, REGS_PRODUCER = 40, REGS_SOFTMAX = 232;
+constexpr int REGS_LAUNCH = 168, REGS_PRODUCER = 48, REGS_SOFTMAX = 224;
 static_assert(128 * REGS_PRODUCER + 256 * REGS_SOFTMAX <= TA_THREADS * REGS_LAUNCH, "register split");
 
 // barrier slots (8 bytes each)
@@ -82,7 +84,12 @@ struct AttnArgs {
   const uint64_t* mask;
   const int32_t* n_nodes;
   __nv_bfloat16* out;
-  int B, n_pad, H, Hkv, G, kv_cap, ctas;  // ctas = CTAs per group
+  int B, n_pad, H, Hkv, G, kv_cap, ctas;  // ctas = row chunks (units) per group
+  int u_split;     // units [0, u_split) run whole, one CTA each; the rest ...
+  int parts;       // ... have their KV blocks split over this many CTAs (1..MAX_PARTS)
+  int* ws_cnt;     // [split units][2]: arrival tickets, finished partials (zeroed before the launch)
+  float2* ws_ml;   // [split units][parts - 1][256 rows]: (m, l) of a partial
+  float* ws_o;     // [split units][parts - 1][256 rows][128]: unnormalised O of a partial
   float scale_log2;
 };
 
@@ -129,6 +136,11 @@ __device__ __forceinline__ void regs_inc() {
   asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
 }
 
+// Named barrier among `count` threads (the softmax warpgroups use id 1).
+__device__ __forceinline__ void named_sync(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // All 32 lanes wait; the result is warp-uniform.
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
   return __all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar, parity, abort, WAIT_CYCLES));
@@ -140,16 +152,33 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
+  __shared__ int s_ticket, s_ready;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int bg = blockIdx.x / a.ctas, c = blockIdx.x - bg * a.ctas;
+  // Units (group, row chunk) in launch order, so the row chunks of a group,
+  // which stream the same K/V blocks, run together and share them through
+  // L2.  The units of the last, partial wave are split over `parts` CTAs each
+  // (launched last: whole units first, the short split CTAs fill the tail).
+  int unit, part, nparts;
+  if ((int)blockIdx.x < a.u_split) {
+    unit = blockIdx.x;
+    part = 0;
+    nparts = 1;
+  } else {
+    const int k = blockIdx.x - a.u_split;
+    unit = a.u_split + k / a.parts;
+    part = k - (unit - a.u_split) * a.parts;
+    nparts = a.parts;
+  }
+  const int su = unit - a.u_split;  // index among the split units
+  const int bg = unit / a.ctas, c = unit - bg * a.ctas;
   const int b = bg / a.Hkv, g = bg - b * a.Hkv;
   const int nn_raw = a.n_nodes[b], kvl = a.kv_len[b];
   const bool bad = nn_raw < 1 || nn_raw > a.n_pad || kvl < 0 || kvl > a.kv_cap;
   const int nn = bad ? 0 : nn_raw;
-  if (bad && c == 0 && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+  if (bad && c == 0 && part == 0 && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
 
-  // Zero the padding rows (nodes >= n_nodes) of this group; the group's CTAs share the work.
-  {
+  // Zero the padding rows (nodes >= n_nodes) of this group; the group's part-0 CTAs share the work.
+  if (part == 0) {
     const int pad = a.n_pad - nn;
     for (int e = c * TA_THREADS + tid; e < a.G * pad * (HD / 8); e += a.ctas * TA_THREADS) {
       int r = e / (HD / 8), ch = e - r * (HD / 8);
@@ -171,7 +200,14 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
 
   const int nblk_c = (kvl + BN - 1) / BN;
-  const int nblk = nblk_c + 1;  // + the tree block
+  const int nblk_all = nblk_c + 1;  // + the tree block (always the unit's last block)
+  // This CTA's share of the unit's blocks: [kb, kb + nblk).  Parts may be
+  // empty when a unit has fewer blocks than parts.
+  const int kb = part * nblk_all / nparts;
+  const int nblk = (part + 1) * nblk_all / nparts - kb;
+  int n_contrib = 0;
+  for (int h = 0; h < nparts; ++h) n_contrib += ((h + 1) * nblk_all / nparts > h * nblk_all / nparts);
+  if (nblk == 0) return;
 
   if (tid == 0) {
     s_abort = 0;
@@ -212,11 +248,11 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         int issued = 0;
         for (int j = 0; j < nblk; ++j) {
           const int st = j & 1;
-          const bool tree = j >= nblk_c;
+          const bool tree = kb + j >= nblk_c;
           const uint32_t bytes = tree ? (uint32_t)a.n_pad * 64 * 2 * 2 : TILE_BYTES;
           const CUtensorMap* mk = tree ? &tm_kt : &tm_kc;
           const CUtensorMap* mv = tree ? &tm_vt : &tm_vc;
-          const int y = tree ? 0 : j * BN;
+          const int y = tree ? 0 : (kb + j) * BN;
           if (j >= 2 && !mbar_wait_bounded(bar(B_KEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) break;
           const uint32_t dK = sK + st * TILE_BYTES, dV = sV + st * TILE_BYTES;
           mbar_expect_tx(bar(B_KFULL + st), bytes);
@@ -264,7 +300,8 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
                             smem_desc_sw128(vb + kk * 2048, HALF_BYTES, 1024), IDESC_PV, (jj > 0 || kk > 0));
       };
       auto zero_ragged_v = [&](int jj) {  // never let garbage (possibly NaN) rows meet a zero probability
-        const int nv = (jj < nblk_c) ? min(BN, kvl - jj * BN) : nn;
+        const int gj = kb + jj;
+        const int nv = (gj < nblk_c) ? min(BN, kvl - gj * BN) : nn;
         if (nv < BN) {
           unsigned char* vt = smem + OFF_V + (jj & 1) * TILE_BYTES;
           for (int e = lane; e < (BN - nv) * 16; e += 32) {
@@ -342,17 +379,20 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     // ---------------- softmax warpgroups: tile x, thread = row ----------------
     const int x = (warp - 4) >> 2;  // 0: warps 4-7, 1: warps 8-11
     const int q4 = warp & 3;        // TMEM lane quarter of this warp
-    if (x == 0 || has_b) {
-      const int r = q4 * 32 + lane;
-      const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
-      const uint32_t tO = tmem + 256 + x * 128 + lane_off;
-      const int rg = row0 + x * BM + r;
-      const bool row_ok = rg < rows_total;
-      const int hh = row_ok ? rg / nn : 0, i = row_ok ? rg - hh * nn : 0;
+    const bool active = (x == 0 || has_b);
+    const int r = q4 * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+    const uint32_t tO = tmem + 256 + x * 128 + lane_off;
+    const int rg = row0 + x * BM + r;
+    const bool row_ok = active && rg < rows_total;
+    const int hh = row_ok ? rg / nn : 0, i = row_ok ? rg - hh * nn : 0;
+    __nv_bfloat16* dst = a.out + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool fin = false;  // warp-uniform: the row's O is complete in tensor memory
+    if (active) {
       const int nw = a.n_pad / 64;
       const uint64_t* mrow = a.mask + ((size_t)b * a.n_pad + i) * nw;
       const uint64_t m0 = mrow[0], m1 = (nw > 1) ? mrow[1] : 0ull;
-      float m_run = -INFINITY, l_run = 0.f;
       bool ok = true;
       for (int j = 0; j < nblk; ++j) {
         // two tiles: S buffer x, one phase per block; one tile: S buffers alternate
@@ -361,8 +401,8 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         const uint32_t tS = tmem + sb * 128 + lane_off;
         if (!(ok = warp_wait(bar(B_SFULL + sb), par, &s_abort))) break;
         tc_fence_after();
-        const bool tree = (j == nblk - 1);
-        const int nv = tree ? BN : min(BN, kvl - j * BN);
+        const bool tree = (kb + j == nblk_all - 1);
+        const int nv = tree ? BN : min(BN, kvl - (kb + j) * BN);
         const bool masked = tree || nv < BN;  // block-uniform
         // keep-bits of 32-column chunk q: the tree mask row, or the ragged cache tail
         auto keep_bits = [&](int q) -> uint32_t {
@@ -441,10 +481,12 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         tc_fence_before();
         mbar_arrive(bar(B_PFULL + sb));
       }
-      if (ok && warp_wait(bar(B_OFIN + x), 0, &s_abort)) {
-        tc_fence_after();
+      fin = ok && warp_wait(bar(B_OFIN + x), 0, &s_abort);
+      if (fin) tc_fence_after();
+    }
+    if (n_contrib == 1) {
+      if (fin) {
         const float inv = 1.f / l_run;
-        __nv_bfloat16* dst = a.out + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD;
 #pragma unroll
         for (int cc = 0; cc < HD / 32; ++cc) {
           uint32_t o[32];
@@ -459,6 +501,105 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
               v.z = pack_bf16x2(__uint_as_float(o[u + 4]) * inv, __uint_as_float(o[u + 5]) * inv);
               v.w = pack_bf16x2(__uint_as_float(o[u + 6]) * inv, __uint_as_float(o[u + 7]) * inv);
               *reinterpret_cast<uint4*>(dst + cc * 32 + u) = v;
+            }
+          }
+        }
+      }
+    } else {
+      // The unit's KV blocks are split over n_contrib CTAs.  Softmax
+      // attention over a key set is a ratio of two sums over its keys, so the
+      // parts' (m, l, O) over disjoint key ranges merge exactly:
+      //   m* = max m_t,  l* = sum l_t 2^(m_t - m*),  O = sum O_t 2^(m_t - m*) / l*.
+      // Each CTA takes a ticket when done; all but the last store their rows,
+      // the last waits (bounded) until they have, then merges and writes out.
+      // The CTAs it waits for are resident: they took their tickets before it.
+      named_sync(1, 256);
+      if (tid == 128) s_ticket = atomicAdd(a.ws_cnt + 2 * su, 1);
+      named_sync(1, 256);
+      const int t = s_ticket;
+      const size_t slot0 = (size_t)su * (a.parts - 1) * (TILES * BM);  // the unit's first slot row
+      const int lr = x * BM + r;                                          // row within the unit
+      if (t < n_contrib - 1) {
+        if (fin) {
+          float* od = a.ws_o + (slot0 + (size_t)t * (TILES * BM) + lr) * HD;
+#pragma unroll
+          for (int cc = 0; cc < HD / 32; ++cc) {
+            uint32_t o[32];
+            tmem_ld32(tO + cc * 32, o);
+            tc_wait_ld();
+            if (row_ok) {
+#pragma unroll
+              for (int u = 0; u < 32; u += 4)
+                __stcg(reinterpret_cast<float4*>(od + cc * 32 + u),
+                       make_float4(__uint_as_float(o[u]), __uint_as_float(o[u + 1]), __uint_as_float(o[u + 2]),
+                                   __uint_as_float(o[u + 3])));
+            }
+          }
+          if (row_ok) __stcg(a.ws_ml + slot0 + (size_t)t * (TILES * BM) + lr, make_float2(m_run, l_run));
+        }
+        named_sync(1, 256);
+        if (tid == 128) {
+          __threadfence();
+          atomicAdd(a.ws_cnt + 2 * su + 1, 1);
+        }
+      } else {
+        if (tid == 128) {
+          const volatile int* done = a.ws_cnt + 2 * su + 1;
+          const long long t0 = clock64();
+          int ready;
+          while (!(ready = (*done >= n_contrib - 1)) && !s_abort && (uint64_t)(clock64() - t0) < WAIT_CYCLES)
+            __nanosleep(128);
+          if (!ready) s_abort = 1;
+          __threadfence();
+          s_ready = ready;
+        }
+        named_sync(1, 256);
+        if (fin && s_ready) {
+          float mt[MAX_PARTS - 1], wt[MAX_PARTS - 1];
+          float mstar = m_run;
+          for (int u = 0; u < n_contrib - 1; ++u) {
+            const float2 ml = row_ok ? __ldcg(a.ws_ml + slot0 + (size_t)u * (TILES * BM) + lr) : make_float2(m_run, 0.f);
+            mt[u] = ml.x;
+            wt[u] = ml.y;  // l for now
+            mstar = fmaxf(mstar, ml.x);
+          }
+          const float w_own = exp2f(m_run - mstar);
+          float lstar = l_run * w_own;
+          for (int u = 0; u < n_contrib - 1; ++u) {
+            const float w = exp2f(mt[u] - mstar);
+            lstar += wt[u] * w;
+            wt[u] = w;
+          }
+          const float inv = 1.f / lstar;
+#pragma unroll
+          for (int cc = 0; cc < HD / 32; ++cc) {
+            uint32_t o[32];
+            tmem_ld32(tO + cc * 32, o);
+            tc_wait_ld();
+            if (row_ok) {
+              float acc[32];
+#pragma unroll
+              for (int u = 0; u < 32; ++u) acc[u] = __uint_as_float(o[u]) * w_own;
+              for (int t2 = 0; t2 < n_contrib - 1; ++t2) {
+                const float* os = a.ws_o + (slot0 + (size_t)t2 * (TILES * BM) + lr) * HD + cc * 32;
+#pragma unroll
+                for (int u = 0; u < 32; u += 4) {
+                  const float4 v = __ldcg(reinterpret_cast<const float4*>(os + u));
+                  acc[u] += v.x * wt[t2];
+                  acc[u + 1] += v.y * wt[t2];
+                  acc[u + 2] += v.z * wt[t2];
+                  acc[u + 3] += v.w * wt[t2];
+                }
+              }
+#pragma unroll
+              for (int u = 0; u < 32; u += 8) {
+                uint4 v;
+                v.x = pack_bf16x2(acc[u + 0] * inv, acc[u + 1] * inv);
+                v.y = pack_bf16x2(acc[u + 2] * inv, acc[u + 3] * inv);
+                v.z = pack_bf16x2(acc[u + 4] * inv, acc[u + 5] * inv);
+                v.w = pack_bf16x2(acc[u + 6] * inv, acc[u + 7] * inv);
+                *reinterpret_cast<uint4*>(dst + cc * 32 + u) = v;
+              }
             }
           }
         }
@@ -501,12 +642,75 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t outer, u
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Workspace layout for `parts` KV parts per unit (units = batch * Hkv * row chunks).
+struct WsLayout {
+  size_t cnt, ml, o, total;
+};
+WsLayout ws_layout(uint64_t units, int parts) {
+  WsLayout w;
+  const uint64_t slots = units * (uint64_t)(parts - 1) * (TILES * BM);
+  w.cnt = 0;
+  w.ml = (units * 2 * sizeof(int) + 255) / 256 * 256;
+  w.o = w.ml + (slots * sizeof(float2) + 255) / 256 * 256;
+  w.total = w.o + slots * HD * sizeof(float);
+  return w;
+}
+
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 0;
+  return n;
+}
+
+// Tail split: with U units on P SMs, the first U - R units (R = U mod P)
+// fill whole waves and run unsplit; the R units of the last, partial wave are
+// split into the most parts that still fit one wave (R * parts <= P), as long
+// as each part keeps at least MIN_PART_BLOCKS blocks (the block count is
+// bounded by kv_cap; the actual lengths live on the device) and the
+// workspace holds their partial sums.
+constexpr int MIN_PART_BLOCKS = 8;
+struct SplitPlan {
+  uint64_t u_split;
+  int parts;
+};
+SplitPlan choose_split(uint64_t units, int kv_cap, size_t ws_bytes) {
+  SplitPlan sp{units, 1};
+  const int sms = sm_count();
+  if (sms <= 0 || units <= (uint64_t)sms) return sp;
+  const uint64_t rem = units % (uint64_t)sms;
+  if (rem == 0) return sp;
+  const int nb = (kv_cap + BN - 1) / BN + 1;
+  int parts = (int)std::min<uint64_t>((uint64_t)MAX_PARTS, (uint64_t)sms / rem);
+  parts = std::min(parts, nb / MIN_PART_BLOCKS);
+  while (parts > 1 && ws_bytes < ws_layout(rem, parts).total) --parts;
+  if (parts > 1) sp = SplitPlan{units - rem, parts};
+  return sp;
+}
+
+uint64_t attn_units(int batch, int n_pad, int H, int Hkv) {
+  return (uint64_t)batch * Hkv * (((uint64_t)(H / Hkv) * n_pad + TILES * BM - 1) / (TILES * BM));
+}
+
 }  // namespace
+
+extern "C" size_t fc_tree_attn_workspace(int batch, int n_pad, int H, int Hkv) {
+  if (batch < 1 || H < 1 || Hkv < 1 || H % Hkv != 0 || (n_pad != 64 && n_pad != 128)) return 0;
+  // only the units of the last partial wave are ever split (fewer than the SM count)
+  const uint64_t units = attn_units(batch, n_pad, H, Hkv);
+  const int sms = sm_count();
+  return ws_layout(std::min<uint64_t>(units, (uint64_t)std::max(sms, 1)), MAX_PARTS).total;
+}
+
+extern "C" int fc_tree_attn_parts(int batch, int n_pad, int H, int Hkv, int kv_cap, size_t ws_bytes) {
+  if (batch < 1 || H < 1 || Hkv < 1 || kv_cap < 1 || H % Hkv != 0 || (n_pad != 64 && n_pad != 128)) return 0;
+  return choose_split(attn_units(batch, n_pad, H, Hkv), kv_cap, ws_bytes).parts;
+}
 
 extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const void* d_v_cache, int kv_cap,
                                   const int32_t* d_kv_len, const void* d_k_tree, const void* d_v_tree,
                                   const uint64_t* d_mask, const int32_t* d_n_nodes, int batch, int n_pad, int H, int Hkv,
-                                  int D, float scale, void* d_out, fc_stream stream) {
+                                  int D, float scale, void* d_out, void* d_ws, size_t ws_bytes, fc_stream stream) {
   if (batch < 0 || H < 1 || Hkv < 1 || kv_cap < 1) return FC_ERR_INVALID_ARG;
   if (D != HD || (n_pad != 64 && n_pad != 128) || H % Hkv != 0 || H / Hkv > 16) return FC_ERR_UNSUPPORTED;
   if (!(scale > 0.f)) return FC_ERR_INVALID_ARG;
@@ -515,12 +719,17 @@ extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const 
     return FC_ERR_INVALID_ARG;
   const uintptr_t al = reinterpret_cast<uintptr_t>(d_q) | reinterpret_cast<uintptr_t>(d_k_cache) |
                        reinterpret_cast<uintptr_t>(d_v_cache) | reinterpret_cast<uintptr_t>(d_k_tree) |
-                       reinterpret_cast<uintptr_t>(d_v_tree) | reinterpret_cast<uintptr_t>(d_out);
+                       reinterpret_cast<uintptr_t>(d_v_tree) | reinterpret_cast<uintptr_t>(d_out) |
+                       reinterpret_cast<uintptr_t>(d_ws);
   if (al % 16 || reinterpret_cast<uintptr_t>(d_mask) % 8) return FC_ERR_INVALID_ARG;
   const uint64_t groups = (uint64_t)batch * Hkv;
   const int G = H / Hkv;
   const int ctas = (G * n_pad + TILES * BM - 1) / (TILES * BM);
-  if (groups * ctas > 0x7FFFFFFFull) return FC_ERR_UNSUPPORTED;
+  const uint64_t units = attn_units(batch, n_pad, H, Hkv);
+  const SplitPlan sp = choose_split(units, kv_cap, d_ws ? ws_bytes : 0);
+  const uint64_t n_split = units - sp.u_split;
+  const uint64_t grid = sp.u_split + n_split * sp.parts;
+  if (grid > 0x7FFFFFFFull) return FC_ERR_UNSUPPORTED;
   CUtensorMap mkc, mvc, mkt, mvt;
   if (!make_map(&mkc, d_k_cache, (uint64_t)kv_cap, groups, BN) || !make_map(&mvc, d_v_cache, (uint64_t)kv_cap, groups, BN) ||
       !make_map(&mkt, d_k_tree, (uint64_t)n_pad, groups, (uint32_t)n_pad) ||
@@ -546,8 +755,22 @@ extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const 
   a.G = G;
   a.kv_cap = kv_cap;
   a.ctas = ctas;
+  a.u_split = (int)sp.u_split;
+  a.parts = sp.parts;
   a.scale_log2 = scale * 1.4426950408889634f;
-  k_tree_attn<<<(unsigned)(groups * ctas), TA_THREADS, SMEM_BYTES, static_cast<cudaStream_t>(stream)>>>(mkc, mvc, mkt,
+  a.ws_cnt = nullptr;
+  a.ws_ml = nullptr;
+  a.ws_o = nullptr;
+  if (sp.parts > 1) {
+    const WsLayout w = ws_layout(n_split, sp.parts);
+    unsigned char* base = static_cast<unsigned char*>(d_ws);
+    a.ws_cnt = reinterpret_cast<int*>(base + w.cnt);
+    a.ws_ml = reinterpret_cast<float2*>(base + w.ml);
+    a.ws_o = reinterpret_cast<float*>(base + w.o);
+    if (cudaMemsetAsync(a.ws_cnt, 0, n_split * 2 * sizeof(int), static_cast<cudaStream_t>(stream)) != cudaSuccess)
+      return FC_ERR_CUDA;
+  }
+  k_tree_attn<<<(unsigned)grid, TA_THREADS, SMEM_BYTES, static_cast<cudaStream_t>(stream)>>>(mkc, mvc, mkt,
                                                                                                         mvt, a);
   return FC_CHECK_LAUNCH();
 }

@@ -47,7 +47,7 @@ class fc_retrieve_params(C.Structure):
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
            "fc_datastore_build_noalloc",
            "fc_retrieve", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
-           "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_accept", "fc_kv_append", "fc_synth_argmax"]
+           "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_accept", "fc_kv_append", "fc_synth_argmax"]
 
 
 def _load():
@@ -74,7 +74,10 @@ def _load():
         "fc_build_tree": (C.c_int, [i32, vp, vp, vp, vp, C.POINTER(C.c_uint32), i32, i32, vp, vp, i32, i32, i32,
                                     vp, vp, vp, vp, vp, vp, vp]),
         "fc_tree_mask": (C.c_int, [vp, vp, vp, i32, i32, vp, vp, vp, vp]),
-        "fc_tree_attn": (C.c_int, [vp, vp, vp, i32, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, C.c_float, vp, vp]),
+        "fc_tree_attn": (C.c_int, [vp, vp, vp, i32, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, C.c_float, vp, vp, sz,
+                                   vp]),
+        "fc_tree_attn_workspace": (sz, [i32, i32, i32, i32]),
+        "fc_tree_attn_parts": (C.c_int, [i32, i32, i32, i32, i32, sz]),
         "fc_accept": (C.c_int, [vp, vp, vp, vp, i32, i32, vp, vp, i32, vp, vp]),
         "fc_kv_append": (C.c_int, [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, i32,
                                    vp, vp, vp, vp]),
@@ -287,8 +290,23 @@ def fc_tree_mask(parent, n_nodes, kv_len):
 
 
 # --------------------------------------------------------------- attention
-def fc_tree_attn(q, k_cache, v_cache, kv_len, k_tree, v_tree, mask, n_nodes, scale=None, out=None):
-    """q [B, Np, H, D]; caches [B, Hkv, cap, D]; tree K/V [B, Hkv, Np, D] (bf16)."""
+_ATTN_WS = {}
+
+
+def attn_workspace(B, Np, H, Hkv, device):
+    """A cached device workspace of fc_tree_attn_workspace() bytes for this shape."""
+    n = int(LIB.fc_tree_attn_workspace(B, Np, H, Hkv))
+    key = (str(device), n)
+    if key not in _ATTN_WS:
+        _ATTN_WS[key] = torch.empty(max(n, 16), dtype=torch.uint8, device=device)
+    return _ATTN_WS[key]
+
+
+def fc_tree_attn(q, k_cache, v_cache, kv_len, k_tree, v_tree, mask, n_nodes, scale=None, out=None, workspace="auto"):
+    """q [B, Np, H, D]; caches [B, Hkv, cap, D]; tree K/V [B, Hkv, Np, D] (bf16).
+
+    ``workspace``: "auto" (a cached one of the full size), None (no key
+    split) or a uint8 device tensor."""
     _need(q, torch.bfloat16, "q")
     B, Np, H, D = q.shape
     _need(k_cache, torch.bfloat16, "k_cache")
@@ -301,9 +319,12 @@ def fc_tree_attn(q, k_cache, v_cache, kv_len, k_tree, v_tree, mask, n_nodes, sca
     _need(n_nodes, torch.int32, "n_nodes", (B,))
     o = out if out is not None else torch.empty_like(q)
     sc = float(scale) if scale is not None else D ** -0.5
+    if isinstance(workspace, str):
+        workspace = attn_workspace(B, Np, H, Hkv, q.device)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check("fc_tree_attn", LIB.fc_tree_attn(_ptr(q), _ptr(k_cache), _ptr(v_cache), cap, _ptr(kv_len), _ptr(k_tree),
                                             _ptr(v_tree), _ptr(mask), _ptr(n_nodes), B, Np, H, Hkv, D, sc, _ptr(o),
-                                            _stream()))
+                                            _ptr(workspace), ws_bytes, _stream()))
     return o
 
 

@@ -7,6 +7,7 @@ import re
 import subprocess
 
 import pytest
+import torch
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 HEADER = os.path.join(ROOT, "include", "fastcoder.h")
@@ -57,12 +58,20 @@ def test_host_validation_without_gpu(lib):
     assert L.fc_retrieve(views, 1, nul, 64, nul, 0, nul, p, nul, nul, nul, nul, nul, nul) == 0
     # attention: head dim / tree padding / GQA ratio outside the supported set
     args = [1, 1, 1, 128, 1, 1, 1, 8, 1, 2]
-    assert L.fc_tree_attn(*args, 64, 32, 8, 64, C.c_float(0.1), 1, nul) == 2
-    assert L.fc_tree_attn(*args, 96, 32, 8, 128, C.c_float(0.1), 1, nul) == 2
-    assert L.fc_tree_attn(*args, 64, 30, 8, 128, C.c_float(0.1), 1, nul) == 2
-    assert L.fc_tree_attn(*args, 64, 32, 8, 128, C.c_float(-1.0), 1, nul) == 1
-    # misaligned pointer
-    assert L.fc_tree_attn(3, 16, 16, 128, 16, 16, 16, 8, 16, 2, 64, 32, 8, 128, C.c_float(0.1), 16, nul) == 1
+    assert L.fc_tree_attn(*args, 64, 32, 8, 64, C.c_float(0.1), 1, nul, 0, nul) == 2
+    assert L.fc_tree_attn(*args, 96, 32, 8, 128, C.c_float(0.1), 1, nul, 0, nul) == 2
+    assert L.fc_tree_attn(*args, 64, 30, 8, 128, C.c_float(0.1), 1, nul, 0, nul) == 2
+    assert L.fc_tree_attn(*args, 64, 32, 8, 128, C.c_float(-1.0), 1, nul, 0, nul) == 1
+    # misaligned pointers (an operand, or the workspace)
+    assert L.fc_tree_attn(3, 16, 16, 128, 16, 16, 16, 8, 16, 2, 64, 32, 8, 128, C.c_float(0.1), 16, nul, 0, nul) == 1
+    assert L.fc_tree_attn(16, 16, 16, 128, 16, 16, 16, 8, 16, 2, 64, 32, 8, 128, C.c_float(0.1), 16, 8, 1 << 20,
+                          nul) == 1
+    # workspace query: positive, never shrinking with the batch (it is capped at
+    # one wave of split units), 0 for an unsupported shape; no device, no split
+    w1, w2 = L.fc_tree_attn_workspace(1, 128, 32, 8), L.fc_tree_attn_workspace(2, 128, 32, 8)
+    assert 0 < w1 <= w2 and L.fc_tree_attn_workspace(1, 100, 32, 8) == 0
+    if not torch.cuda.is_available():
+        assert L.fc_tree_attn_parts(64, 128, 32, 8, 16384, 1 << 40) == 1
     # tree: budget larger than the padding, too many drafts
     w = (C.c_uint32 * 2)(1, 1)
     tree_ptrs = [1] * 6

@@ -259,7 +259,8 @@ def test_tree_mask_from_parents(fc, orc):
 
 
 # --------------------------------------------------------------- attention
-def _attn_case(fc, orc, seed, B, n_pad, H, Hkv, kv_len, cap, nn=None, full_rows=True, sample=None):
+def _attn_case(fc, orc, seed, B, n_pad, H, Hkv, kv_len, cap, nn=None, full_rows=True, sample=None,
+               workspace="auto", want_parts=None):
     rng = synth.rng_for(50, seed)
     tok, par, nn_r = _random_trees(rng, B, n_pad)
     if nn is not None:
@@ -277,9 +278,20 @@ def _attn_case(fc, orc, seed, B, n_pad, H, Hkv, kv_len, cap, nn=None, full_rows=
     vt = synth.randn_bf16((B, Hkv, n_pad, D), 5000 + seed, "cuda")
     gm = fc.fc_tree_mask(dev(par), dev(nn_r), dev(kvl))
     out = torch.full_like(q, float("nan"))
-    fc.fc_tree_attn(q, kc, vc, dev(kvl), kt, vt, gm["mask"], dev(nn_r), out=out)
+    fc.fc_tree_attn(q, kc, vc, dev(kvl), kt, vt, gm["mask"], dev(nn_r), out=out, workspace=workspace)
     torch.cuda.synchronize()
     check_no_error(fc)
+    if want_parts is not None:  # the same call without a workspace: one CTA per row chunk
+        ws = fc.attn_workspace(B, n_pad, H, Hkv, "cuda") if workspace == "auto" else workspace
+        nbytes = 0 if ws is None else ws.numel()
+        parts = fc.LIB.fc_tree_attn_parts(B, n_pad, H, Hkv, cap, nbytes)
+        assert parts >= want_parts, parts
+        single = torch.full_like(q, float("nan"))
+        fc.fc_tree_attn(q, kc, vc, dev(kvl), kt, vt, gm["mask"], dev(nn_r), out=single, workspace=None)
+        torch.cuda.synchronize()
+        check_no_error(fc)
+        assert torch.isfinite(out.float()).all()
+        assert (out.float() - single.float()).abs().max().item() <= ATOL
     rm = orc.tree_mask(par, nn_r, kvl, n_pad)["mask"]
     args = [bits_bf16(x) for x in (q, kc, vc)] + [kvl] + [bits_bf16(x) for x in (kt, vt)] + [rm, nn_r]
     got = out.float().cpu().numpy()
@@ -323,6 +335,32 @@ def test_attn_gqa_n128(fc, orc):
 
 def test_attn_gqa_n64_group2(fc, orc):
     _attn_case(fc, orc, 4, 5, 64, 16, 8, [300, 0, 64, 700, 129], 777, nn=[64, 1, 40, 64, 2])
+
+
+def _units_over_sms(per_seq_units):
+    """A batch whose row-chunk count is a little over one wave of CTAs: the
+    chunks of the last sequence form a short second wave and have their keys
+    split over several CTAs (the sampled rows always include that sequence)."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    return -(-(sms + 8) // per_seq_units)
+
+
+def test_attn_kv_split_one_tile(fc, orc):
+    # G = 1, 64-node trees: one 128-row tile per (sequence, kv head); ragged
+    # caches (empty, one key, block edges) mixed with full ones
+    B = _units_over_sms(8)
+    rng = synth.rng_for(51)
+    kvl = [[0, 1, 127, 128, 129, 2047, 2048][b % 7] if b < 14 else int(rng.integers(0, 2049)) for b in range(B)]
+    _attn_case(fc, orc, 6, B, 64, 8, 8, kvl, 2048, full_rows=False, want_parts=2)
+
+
+def test_attn_kv_split_two_tiles(fc, orc):
+    # G = 4, 128-node trees: two row chunks per group, the first with two tiles
+    B = _units_over_sms(16)
+    rng = synth.rng_for(52)
+    kvl = [int(rng.integers(0, 2049)) for _ in range(B)]
+    nn = [int(rng.integers(1, 129)) if b % 3 else 128 for b in range(B)]
+    _attn_case(fc, orc, 7, B, 128, 32, 8, kvl, 2048, nn=nn, full_rows=False, want_parts=2)
 
 
 def test_attn_c3_shape_sampled(fc, orc):
