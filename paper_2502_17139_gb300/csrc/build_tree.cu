@@ -5,16 +5,19 @@
 //
 // One CTA per query, everything in shared memory, no pointer trie:
 //   1. gather the drafts of all sources with weight w = src_weight * count;
-//   2. sort them lexicographically (bitonic sort of indices) and merge
+//   2. sort them lexicographically (every thread ranks its drafts against
+//      all others, a packed prefix key settling most comparisons) and merge
 //      duplicates across sources (weights add);
 //   3. with neighbour LCPs, every trie node is a pair (u, l): the prefix of
 //      length l of sorted unique draft u, new at u when l > lcp(u-1, u).
 //      Its weight is the weight sum of the contiguous run of drafts that
 //      share that prefix (prefix sums over the sorted drafts);
-//   4. a bitonic sort of (W, 31 - l, 8191 - u) keys selects the heaviest
-//      budget - 1 nodes (ties: shallower, then smaller path);
-//   5. sorting the kept nodes by (u, l) is depth-first preorder with
-//      children in ascending token order; parents come from the LCPs;
+//   4. a radix select on the distinct (W, 31 - l, 8191 - u) keys finds the
+//      heaviest budget - 1 nodes (ties: shallower, then smaller path); a
+//      parent's key always exceeds its child's, so the kept set is a tree;
+//   5. (u, l) order is depth-first preorder with children in ascending
+//      token order: a scan over a kept-flag table [u][l] numbers the nodes
+//      and maps a parent (the run start of prefix l - 1) to its index;
 //      masks are ancestor walks.
 #include <algorithm>
 
@@ -43,14 +46,8 @@ struct TreeOut {
   int32_t* n_nodes;
 };
 
-__host__ __device__ inline uint32_t next_pow2(uint32_t x) {
-  uint32_t p = 1;
-  while (p < x) p <<= 1;
-  return p;
-}
-
 struct BtLayout {
-  size_t tok, len, w, order, uniq, wu, ps, lcp, coff, flag, ckey, total;
+  size_t tok, len, w, order, uniq, wu, ps, lcp, coff, flag, ckey, pk, tab, total;
 };
 
 __host__ __device__ inline BtLayout bt_layout(int M, int d) {
@@ -64,14 +61,16 @@ __host__ __device__ inline BtLayout bt_layout(int M, int d) {
   L.tok = take((size_t)M * d * 4);
   L.len = take((size_t)M * 4);
   L.w = take((size_t)M * 8);
-  L.order = take((size_t)next_pow2((uint32_t)(M > 0 ? M : 1)) * 4);
+  L.order = take((size_t)M * 4);
   L.uniq = take((size_t)M * 4);
   L.wu = take((size_t)M * 8);
   L.ps = take((size_t)(M + 1) * 8);
   L.lcp = take((size_t)(M + 1) * 4);
   L.coff = take((size_t)(M + 1) * 4);
   L.flag = take((size_t)(M + 1) * 4);
-  L.ckey = take((size_t)next_pow2((uint32_t)(M * d)) * 8);
+  L.ckey = take((size_t)M * d * 8);
+  L.pk = take((size_t)M * 16);      // packed first four tokens of each draft
+  L.tab = take((size_t)M * d * 4);  // kept flags [u][l - 1], then their preorder ranks
   L.total = off;
   return L;
 }
@@ -112,6 +111,81 @@ __device__ uint32_t block_scan_array(uint32_t* a, int n, uint32_t* wsum) {
   return total;
 }
 
+// Warp 0 (all 32 lanes): out[i] = sum of a[0..i) for i <= n (64-bit).  The
+// caller synchronises the block before reading out.
+__device__ void warp_scan_u64(const uint64_t* a, uint64_t* out, uint32_t n) {
+  const uint32_t lane = threadIdx.x & 31;
+  const uint32_t chunk = (n + 31) / 32;
+  const uint32_t lo = min(n, lane * chunk), hi = min(n, lo + chunk);
+  uint64_t s = 0;
+  for (uint32_t i = lo; i < hi; ++i) s += a[i];
+  uint64_t inc = s;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint64_t y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+    if ((int)lane >= o) inc += y;
+  }
+  uint64_t pre = inc - s;
+  for (uint32_t i = lo; i < hi; ++i) {
+    out[i] = pre;
+    pre += a[i];
+  }
+  if (lane == 31) out[n] = inc;
+}
+
+// The k-th largest (1 <= k <= n) of n distinct 64-bit keys, by radix select
+// over bytes from the most significant: each pass histograms the byte of
+// the keys that match the bytes fixed so far and fixes the byte whose bin
+// holds the k-th largest.  Called by the whole block.
+__device__ uint64_t radix_select_desc(const uint64_t* key, uint32_t n, uint32_t k, uint32_t* hist) {
+  __shared__ uint64_t s_pre;
+  __shared__ uint32_t s_k;
+  const int tid = threadIdx.x;
+  uint64_t pre = 0, pmask = 0;
+  for (int shift = 56; shift >= 0; shift -= 8) {
+    for (int i = tid; i < 256; i += BT_THREADS) hist[i] = 0;
+    if (tid == 0) {
+      s_pre = pre;
+      s_k = k;
+    }
+    __syncthreads();
+    for (uint32_t i = tid; i < n; i += BT_THREADS) {
+      const uint64_t x = key[i];
+      if ((x & pmask) == pre) atomicAdd(&hist[(x >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (tid < 32) {  // lane L owns bins [8L, 8L + 8); suffix sums from the top bin
+      uint32_t c[8], tot = 0;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) tot += (c[q] = hist[8 * tid + q]);
+      uint32_t suf = tot;  // inclusive suffix over lanes >= tid
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_down_sync(0xFFFFFFFFu, suf, o);
+        if (tid + o < 32) suf += y;
+      }
+      const uint32_t above = suf - tot;  // keys in higher lanes' bins
+      if (above < k && suf >= k) {       // the k-th largest lies in this lane's bins
+        uint32_t acc = above;
+        for (int q = 7; q >= 0; --q) {
+          if (acc + c[q] >= k) {
+            s_pre = pre | ((uint64_t)(8 * tid + q) << shift);
+            s_k = k - acc;
+            break;
+          }
+          acc += c[q];
+        }
+      }
+    }
+    __syncthreads();
+    pre = s_pre;
+    k = s_k;
+    pmask |= (uint64_t)0xFF << shift;
+    __syncthreads();
+  }
+  return pre;
+}
+
 // -1 / 0 / 1 lexicographic comparison of two drafts (a prefix sorts first).
 __device__ __forceinline__ int cmp_draft(const uint32_t* a, int la, const uint32_t* b, int lb) {
   int l = min(la, lb);
@@ -140,6 +214,9 @@ __global__ void __launch_bounds__(BT_THREADS) k_build_tree(TreeIn in, int S, int
   uint32_t* coff = reinterpret_cast<uint32_t*>(smem_raw + L.coff);
   uint32_t* flag = reinterpret_cast<uint32_t*>(smem_raw + L.flag);
   uint64_t* ckey = reinterpret_cast<uint64_t*>(smem_raw + L.ckey);
+  uint64_t* pk = reinterpret_cast<uint64_t*>(smem_raw + L.pk);
+  uint32_t* tab = reinterpret_cast<uint32_t*>(smem_raw + L.tab);
+  __shared__ uint32_t hist[256];
   const int b = blockIdx.x, tid = threadIdx.x;
 
   // 1. valid drafts, compacted in (source, slot) order
@@ -172,33 +249,36 @@ __global__ void __launch_bounds__(BT_THREADS) k_build_tree(TreeIn in, int S, int
   }
   __syncthreads();
 
-  // 2. bitonic sort of draft indices by token sequence; equal drafts keep
-  //    (source, slot) order through the index tie-break
-  const uint32_t PM = next_pow2(M > 0 ? M : 1);
-  for (uint32_t i = tid; i < PM; i += BT_THREADS) order[i] = (i < M) ? i : 0xFFFFFFFFu;
-  __syncthreads();
-  auto draft_less = [&](uint32_t x, uint32_t y) -> bool {  // sentinels sort last
-    if (x == 0xFFFFFFFFu) return false;
-    if (y == 0xFFFFFFFFu) return true;
-    const int c = cmp_draft(tok + x * d, len[x], tok + y * d, len[y]);
-    return c < 0 || (c == 0 && x < y);
-  };
-  for (uint32_t size = 2; size <= PM; size <<= 1) {
-    for (uint32_t st = size >> 1; st > 0; st >>= 1) {
-      for (uint32_t i = tid; i < PM; i += BT_THREADS) {
-        const uint32_t j = i ^ st;
-        if (j > i) {
-          const uint32_t x = order[i], y = order[j];
-          const bool asc = (i & size) == 0;
-          if (asc ? draft_less(y, x) : draft_less(x, y)) {
-            order[i] = y;
-            order[j] = x;
-          }
-        }
-      }
-      __syncthreads();
-    }
+  // 2. rank sort of the drafts by token sequence; equal drafts keep
+  //    (source, slot) order through the index tie-break.  Comparing the
+  //    zero-padded packed prefixes is exact whenever they differ (a zero
+  //    pad only ever ties with a real token); ties fall back to the tokens.
+  for (uint32_t i = tid; i < M; i += BT_THREADS) {
+    const uint32_t* t = tok + i * d;
+    const int l = len[i];
+    pk[2 * i] = ((uint64_t)t[0] << 32) | (l > 1 ? t[1] : 0u);
+    pk[2 * i + 1] = ((uint64_t)(l > 2 ? t[2] : 0u) << 32) | (l > 3 ? t[3] : 0u);
   }
+  __syncthreads();
+  for (uint32_t i = tid; i < M; i += BT_THREADS) {
+    const uint64_t a0 = pk[2 * i], a1 = pk[2 * i + 1];
+    uint32_t rank = 0;
+    for (uint32_t j = 0; j < M; ++j) {
+      const uint64_t b0 = pk[2 * j], b1 = pk[2 * j + 1];
+      bool less;
+      if (b0 != a0) {
+        less = b0 < a0;
+      } else if (b1 != a1) {
+        less = b1 < a1;
+      } else {
+        const int c = cmp_draft(tok + j * d, len[j], tok + i * d, len[i]);
+        less = c < 0 || (c == 0 && j < i);
+      }
+      rank += less ? 1u : 0u;
+    }
+    order[rank] = i;
+  }
+  __syncthreads();
   for (uint32_t r = tid; r < M; r += BT_THREADS) {
     uint32_t i = order[r];
     flag[r] = (r == 0 || cmp_draft(tok + order[r - 1] * d, len[order[r - 1]], tok + i * d, len[i]) != 0) ? 1u : 0u;
@@ -228,16 +308,8 @@ __global__ void __launch_bounds__(BT_THREADS) k_build_tree(TreeIn in, int S, int
     coff[u] = (uint32_t)len[uniq[u]] - l;
   }
   __syncthreads();
-  if (tid == 0) {
-    uint64_t run = 0;
-    for (uint32_t u = 0; u < U; ++u) {
-      ps[u] = run;
-      run += wu[u];
-    }
-    ps[U] = run;
-  }
+  if (tid < 32) warp_scan_u64(wu, ps, U);  // ps[u] = sum of wu[0..u), ps[U] = total
   uint32_t C = block_scan_array(coff, (int)U, wsum);
-  const uint32_t P2 = next_pow2(max(C, 1u));
   for (uint32_t u = tid; u < U; u += BT_THREADS) {
     const int lu = len[uniq[u]];
     for (int l = (int)lcp[u] + 1; l <= lu; ++l) {
@@ -247,51 +319,45 @@ __global__ void __launch_bounds__(BT_THREADS) k_build_tree(TreeIn in, int S, int
       ckey[coff[u] + (l - lcp[u] - 1)] = (W << 18) | ((uint64_t)(31 - l) << 13) | (uint64_t)(8191u - u);
     }
   }
-  for (uint32_t c = C + tid; c < P2; c += BT_THREADS) ckey[c] = 0;
+  for (uint32_t x = tid; x < U * (uint32_t)d; x += BT_THREADS) tab[x] = 0;
   __syncthreads();
 
-  // 4. bitonic sort, descending
-  for (uint32_t size = 2; size <= P2; size <<= 1) {
-    for (uint32_t st = size >> 1; st > 0; st >>= 1) {
-      for (uint32_t i = tid; i < P2; i += BT_THREADS) {
-        uint32_t j = i ^ st;
-        if (j > i) {
-          uint64_t a = ckey[i], c = ckey[j];
-          bool desc = (i & size) == 0;
-          if (desc ? (a < c) : (a > c)) {
-            ckey[i] = c;
-            ckey[j] = a;
-          }
-        }
-      }
-      __syncthreads();
-    }
-  }
-
-  // 5. kept nodes in preorder = ascending (u, l)
+  // 4. the nsel largest keys (all distinct): radix select of the threshold,
+  //    8 bits at a time from the top
   const int nsel = (int)umin((uint32_t)(budget - 1), C);
-  for (int i = tid; i < nsel; i += BT_THREADS) {
-    uint64_t key = ckey[i];
-    int u = 8191 - (int)(key & 8191u), l = 31 - (int)((key >> 13) & 31u);
-    int r = 0;
-    for (int j = 0; j < nsel; ++j) {
-      uint64_t kj = ckey[j];
-      int uj = 8191 - (int)(kj & 8191u), lj = 31 - (int)((kj >> 13) & 31u);
-      r += (uj < u || (uj == u && lj < l)) ? 1 : 0;
+  uint64_t thr = 0;
+  if (nsel > 0 && (uint32_t)nsel < C) thr = radix_select_desc(ckey, C, (uint32_t)nsel, hist);
+  // 5. kept flags in the (u, l) table, scanned into preorder ranks
+  for (uint32_t c = tid; c < C; c += BT_THREADS) {
+    const uint64_t key = ckey[c];
+    if (nsel > 0 && key >= thr) {
+      const int u = 8191 - (int)(key & 8191u), l = 31 - (int)((key >> 13) & 31u);
+      tab[u * d + l - 1] = 1u;
     }
-    sel_u[1 + r] = u;
-    sel_l[1 + r] = l;
   }
   __syncthreads();
-  const int n = 1 + nsel;
+  const uint32_t nkept = block_scan_array(tab, (int)(U * (uint32_t)d), wsum);
+  if (nkept != (uint32_t)nsel && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INTERNAL);
+  for (uint32_t c = tid; c < C; c += BT_THREADS) {
+    const uint64_t key = ckey[c];
+    if (nsel > 0 && key >= thr) {
+      const int u = 8191 - (int)(key & 8191u), l = 31 - (int)((key >> 13) & 31u);
+      const int idx = 1 + (int)tab[u * d + l - 1];
+      if (idx < FC_MAX_NODES) {
+        sel_u[idx] = u;
+        sel_l[idx] = l;
+      }
+    }
+  }
+  __syncthreads();
+  const int n = 1 + min(nsel, FC_MAX_NODES - 1);
   for (int i = 1 + tid; i < n; i += BT_THREADS) {
-    int u = sel_u[i], l = sel_l[i];
+    const int u = sel_u[i], l = sel_l[i];
     int pidx = 0;
-    if (l > 1) {
+    if (l > 1) {  // the parent is the prefix l - 1, first seen at the start of its run
       int up = u;
       while (up > 0 && (int)lcp[up] >= l - 1) --up;
-      for (int j = 1; j < i; ++j)
-        if (sel_u[j] == up && sel_l[j] == l - 1) pidx = j;
+      pidx = 1 + (int)tab[up * d + l - 2];
     }
     par_s[i] = pidx;
   }
