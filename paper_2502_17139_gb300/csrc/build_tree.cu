@@ -5,9 +5,9 @@
 //
 // One CTA per query, everything in shared memory, no pointer trie:
 //   1. gather the drafts of all sources with weight w = src_weight * count;
-//   2. sort them lexicographically (every thread ranks its drafts against
-//      all others, a packed prefix key settling most comparisons) and merge
-//      duplicates across sources (weights add);
+//   2. sort them lexicographically (threads rank drafts against all others,
+//      comparing zero-padded pairs of tokens packed in 64-bit words, then
+//      lengths) and merge duplicates across sources (weights add);
 //   3. with neighbour LCPs, every trie node is a pair (u, l): the prefix of
 //      length l of sorted unique draft u, new at u when l > lcp(u-1, u).
 //      Its weight is the weight sum of the contiguous run of drafts that
@@ -27,8 +27,9 @@ FC_DEFINE_ERROR_WORD(tree)
 
 namespace {
 
-constexpr int BT_THREADS = 256;
+constexpr int BT_THREADS = 512;
 constexpr int BT_MAX_DRAFTS = 512;
+constexpr int PK_WORDS = FC_MAX_DRAFT_LEN / 2;  // 64-bit words per packed draft
 
 struct TreeIn {
   const uint32_t* drafts;
@@ -69,7 +70,7 @@ __host__ __device__ inline BtLayout bt_layout(int M, int d) {
   L.coff = take((size_t)(M + 1) * 4);
   L.flag = take((size_t)(M + 1) * 4);
   L.ckey = take((size_t)M * d * 8);
-  L.pk = take((size_t)M * 16);      // packed first four tokens of each draft
+  L.pk = take((size_t)M * PK_WORDS * 8);  // each draft as zero-padded token pairs
   L.tab = take((size_t)M * d * 4);  // kept flags [u][l - 1], then their preorder ranks
   L.total = off;
   return L;
@@ -138,11 +139,38 @@ __device__ void warp_scan_u64(const uint64_t* a, uint64_t* out, uint32_t n) {
 // the keys that match the bytes fixed so far and fixes the byte whose bin
 // holds the k-th largest.  Called by the whole block.
 __device__ uint64_t radix_select_desc(const uint64_t* key, uint32_t n, uint32_t k, uint32_t* hist) {
-  __shared__ uint64_t s_pre;
+  __shared__ uint64_t s_pre, s_or, s_and;
   __shared__ uint32_t s_k;
   const int tid = threadIdx.x;
-  uint64_t pre = 0, pmask = 0;
-  for (int shift = 56; shift >= 0; shift -= 8) {
+  // bytes on which all keys agree need no pass: start below them
+  if (tid == 0) {
+    s_or = 0;
+    s_and = ~0ull;
+  }
+  __syncthreads();
+  {
+    uint64_t o = 0, a = ~0ull;
+    for (uint32_t i = tid; i < n; i += BT_THREADS) {
+      o |= key[i];
+      a &= key[i];
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      o |= __shfl_xor_sync(0xFFFFFFFFu, o, off);
+      a &= __shfl_xor_sync(0xFFFFFFFFu, a, off);
+    }
+    if ((tid & 31) == 0) {
+      atomicOr(reinterpret_cast<unsigned long long*>(&s_or), o);
+      atomicAnd(reinterpret_cast<unsigned long long*>(&s_and), a);
+    }
+  }
+  __syncthreads();
+  const uint64_t diff = s_or ^ s_and;  // bits that vary among the keys
+  if (diff == 0) return s_or;          // n == 1
+  const int top = 63 - __clzll((long long)diff);
+  uint64_t pmask = (top >= 63) ? 0ull : ~((2ull << top) - 1ull);  // agreed bits above `top`
+  uint64_t pre = s_or & pmask;
+  for (int shift = top & ~7; shift >= 0; shift -= 8) {
     for (int i = tid; i < 256; i += BT_THREADS) hist[i] = 0;
     if (tid == 0) {
       s_pre = pre;
@@ -166,15 +194,21 @@ __device__ uint64_t radix_select_desc(const uint64_t* key, uint32_t n, uint32_t 
       }
       const uint32_t above = suf - tot;  // keys in higher lanes' bins
       if (above < k && suf >= k) {       // the k-th largest lies in this lane's bins
-        uint32_t acc = above;
+        uint32_t acc = above, k_rem = 0;
+        int chosen = -1;
+#pragma unroll
         for (int q = 7; q >= 0; --q) {
-          if (acc + c[q] >= k) {
-            s_pre = pre | ((uint64_t)(8 * tid + q) << shift);
-            s_k = k - acc;
-            break;
+          if (chosen < 0) {
+            if (acc + c[q] >= k) {
+              chosen = q;
+              k_rem = k - acc;
+            } else {
+              acc += c[q];
+            }
           }
-          acc += c[q];
         }
+        s_pre = pre | ((uint64_t)(8 * tid + chosen) << shift);
+        s_k = k_rem;
       }
     }
     __syncthreads();
@@ -250,34 +284,54 @@ __global__ void __launch_bounds__(BT_THREADS) k_build_tree(TreeIn in, int S, int
   __syncthreads();
 
   // 2. rank sort of the drafts by token sequence; equal drafts keep
-  //    (source, slot) order through the index tie-break.  Comparing the
-  //    zero-padded packed prefixes is exact whenever they differ (a zero
-  //    pad only ever ties with a real token); ties fall back to the tokens.
-  for (uint32_t i = tid; i < M; i += BT_THREADS) {
-    const uint32_t* t = tok + i * d;
+  //    (source, slot) order through the index tie-break.  Drafts compare as
+  //    their token pairs packed in 64-bit words, zero-padded, then by
+  //    length: a difference in the padded words always has the lexicographic
+  //    sign (a zero pad only ever ties with a real token), and padded words
+  //    that agree mean one draft is a prefix of the other.
+  for (uint32_t x = tid; x < M * (uint32_t)PK_WORDS; x += BT_THREADS) {
+    const uint32_t i = x / PK_WORDS, q = x - i * PK_WORDS;
     const int l = len[i];
-    pk[2 * i] = ((uint64_t)t[0] << 32) | (l > 1 ? t[1] : 0u);
-    pk[2 * i + 1] = ((uint64_t)(l > 2 ? t[2] : 0u) << 32) | (l > 3 ? t[3] : 0u);
+    const uint32_t t0 = (2 * (int)q < l) ? tok[i * d + 2 * q] : 0u;
+    const uint32_t t1 = (2 * (int)q + 1 < l) ? tok[i * d + 2 * q + 1] : 0u;
+    pk[x] = ((uint64_t)t0 << 32) | t1;
+  }
+  for (uint32_t i = tid; i < M; i += BT_THREADS) order[i] = 0;
+  __syncthreads();
+  {
+    // several threads per draft when they fit (slices of the j range)
+    const uint32_t split = M > 0 ? umax(1u, umin(8u, (uint32_t)BT_THREADS / M)) : 1u;
+    for (uint32_t x = tid; x < M * split; x += BT_THREADS) {
+      const uint32_t i = x / split, h = x - i * split;
+      const ulonglong2* pv = reinterpret_cast<const ulonglong2*>(pk);
+      uint64_t a[PK_WORDS];
+#pragma unroll
+      for (int q = 0; q < PK_WORDS / 2; ++q) {
+        const ulonglong2 v = pv[i * (PK_WORDS / 2) + q];
+        a[2 * q] = v.x;
+        a[2 * q + 1] = v.y;
+      }
+      const int la = len[i];
+      const uint32_t j0 = h * M / split, j1 = (h + 1) * M / split;
+      uint32_t rank = 0;
+      for (uint32_t j = j0; j < j1; ++j) {
+        int res = 0;  // sign of draft j vs draft i
+#pragma unroll
+        for (int q = 0; q < PK_WORDS / 2; ++q) {
+          const ulonglong2 v = pv[j * (PK_WORDS / 2) + q];
+          if (res == 0 && v.x != a[2 * q]) res = (v.x < a[2 * q]) ? -1 : 1;
+          if (res == 0 && v.y != a[2 * q + 1]) res = (v.y < a[2 * q + 1]) ? -1 : 1;
+        }
+        if (res == 0) res = (len[j] < la) ? -1 : (len[j] > la ? 1 : 0);
+        rank += (res < 0 || (res == 0 && j < i)) ? 1u : 0u;
+      }
+      atomicAdd(&order[i], rank);  // order[] holds ranks here
+    }
   }
   __syncthreads();
-  for (uint32_t i = tid; i < M; i += BT_THREADS) {
-    const uint64_t a0 = pk[2 * i], a1 = pk[2 * i + 1];
-    uint32_t rank = 0;
-    for (uint32_t j = 0; j < M; ++j) {
-      const uint64_t b0 = pk[2 * j], b1 = pk[2 * j + 1];
-      bool less;
-      if (b0 != a0) {
-        less = b0 < a0;
-      } else if (b1 != a1) {
-        less = b1 < a1;
-      } else {
-        const int c = cmp_draft(tok + j * d, len[j], tok + i * d, len[i]);
-        less = c < 0 || (c == 0 && j < i);
-      }
-      rank += less ? 1u : 0u;
-    }
-    order[rank] = i;
-  }
+  for (uint32_t i = tid; i < M; i += BT_THREADS) flag[i] = order[i];  // rank of draft i
+  __syncthreads();
+  for (uint32_t i = tid; i < M; i += BT_THREADS) order[flag[i]] = i;
   __syncthreads();
   for (uint32_t r = tid; r < M; r += BT_THREADS) {
     uint32_t i = order[r];
