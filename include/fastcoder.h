@@ -73,7 +73,8 @@ fc_status fc_get_error(fc_stream s);
  * "which contexts end with this suffix" into one contiguous SA range.
  * ------------------------------------------------------------------------ */
 typedef struct {
-  const uint32_t* tokens;  /* device, [n_tokens] token ids < vocab */
+  const uint32_t* tokens;  /* device, [n_tokens] token ids < vocab, 16-byte aligned
+                              (fc_retrieve reads it as 16-byte vectors) */
   const uint32_t* sa;      /* device, [n_tokens] suffix array of tokens */
   const uint32_t* bucket;  /* device, [vocab + 1]: bucket[v] = first SA index whose
                               suffix starts with a token >= v; bucket[vocab] = n_tokens */
