@@ -106,15 +106,27 @@ class ClockSampler:
              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
              "clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, interval_ms: int = 20):
         self.proc = None
         self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
         try:
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={gpu_index}", f"--query-gpu={self.QUERY}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.file,
-                                         stderr=subprocess.DEVNULL)
+                                          "--format=csv,noheader,nounits", "-lms", str(interval_ms)],
+                                         stdout=self.file, stderr=subprocess.DEVNULL)
         except (FileNotFoundError, OSError):
             self.proc = None
+
+    def wait_first(self, timeout_s: float = 3.0):
+        """Block until the sampler has written its first sample (nvidia-smi takes a
+        moment to start), so that the samples cover the region that follows."""
+        self.skip = 0
+        t0 = time.perf_counter()
+        while self.proc is not None and time.perf_counter() - t0 < timeout_s:
+            if os.path.getsize(self.file.name) > 0:
+                with open(self.file.name) as f:  # samples taken so far precede the region
+                    self.skip = sum(1 for r in f if r.strip())
+                return
+            time.sleep(0.01)
 
     def stop(self):
         if self.proc is None:
@@ -128,6 +140,7 @@ class ClockSampler:
         with open(self.file.name) as f:
             rows = [r.strip().split(", ") for r in f if r.strip()]
         os.unlink(self.file.name)
+        rows = rows[getattr(self, "skip", 0):] or rows[-1:]
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for r in rows:
@@ -290,6 +303,7 @@ def run_ours(args, rank, ws, local):
     barrier(ws)
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
+    clocks.wait_first()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     start.record(stream)
     for i in range(K):
@@ -596,6 +610,7 @@ def run_attn(args, rank, ws, local):
     barrier(ws)
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
+    clocks.wait_first()
     for e0, e1 in evs:
         e0.record()
         fc.fc_tree_attn(*args_d, out=out)

@@ -109,17 +109,23 @@ __global__ void k_synth_argmax(const uint32_t* __restrict__ tok, const int32_t* 
                                const int32_t* __restrict__ n_nodes, int n_pad, const int32_t* __restrict__ plen,
                                const uint32_t* __restrict__ rtok, uint32_t vocab, uint32_t* __restrict__ argmax) {
   __shared__ int agree[FC_MAX_NODES];
+  __shared__ int par_s[FC_MAX_NODES];
+  __shared__ uint32_t tok_s[FC_MAX_NODES];
   const int b = blockIdx.x;
   const size_t base = (size_t)b * n_pad;
   const int n = min(max((int)n_nodes[b], 1), n_pad);
-  for (int i = threadIdx.x; i < n_pad; i += blockDim.x) agree[i] = -1;
+  for (int i = threadIdx.x; i < n_pad; i += blockDim.x) {  // the tree, staged once (coalesced)
+    agree[i] = -1;
+    par_s[i] = parent[base + i];
+    tok_s[i] = tok[base + i];
+  }
   __syncthreads();
   if (threadIdx.x == 0) {
     int cur = 0;
     for (int t = 0; t < plen[b]; ++t) {
       int first = -1;
       for (int j = cur + 1; j < n && first < 0; ++j)
-        if (parent[base + j] == cur) first = j;
+        if (par_s[j] == cur) first = j;
       if (first < 0) break;
       agree[cur] = first;
       cur = first;
@@ -130,13 +136,13 @@ __global__ void k_synth_argmax(const uint32_t* __restrict__ tok, const int32_t* 
     uint32_t x = 0;
     if (i < n) {
       if (agree[i] >= 0) {
-        x = tok[base + agree[i]];
+        x = tok_s[agree[i]];
       } else {
         x = rtok[base + i] % vocab;
         for (int tries = 0; tries < n_pad; ++tries) {  // bounded: children may cover a tiny vocabulary
           bool clash = false;
           for (int j = i + 1; j < n; ++j)
-            if (parent[base + j] == i && tok[base + j] == x) clash = true;
+            if (par_s[j] == i && tok_s[j] == x) clash = true;
           if (!clash) break;
           x = (x + 1u) % vocab;
         }
