@@ -337,6 +337,18 @@ def test_attn_gqa_n64_group2(fc, orc):
     _attn_case(fc, orc, 4, 5, 64, 16, 8, [300, 0, 64, 700, 129], 777, nn=[64, 1, 40, 64, 2])
 
 
+def test_attn_gqa_group8_n64(fc, orc):
+    # G = 8 with 64-node trees: 512 rows per group, two row chunks of two tiles
+    kvl = [0, 1, 300, 1000, 2048, 129]
+    _attn_case(fc, orc, 8, 6, 64, 64, 8, kvl, 2048, nn=[64, 1, 33, 64, 17, 48], full_rows=False)
+
+
+def test_attn_gqa_group16_n128(fc, orc):
+    # G = 16 (the largest supported): up to 2048 rows per group, eight row chunks
+    kvl = [700, 0, 2048, 1]
+    _attn_case(fc, orc, 9, 4, 128, 32, 2, kvl, 2048, nn=[128, 3, 100, 65], full_rows=False)
+
+
 def _units_over_sms(per_seq_units):
     """A batch whose row-chunk count is a little over one wave of CTAs: the
     chunks of the last sequence form a short second wave and have their keys
