@@ -531,6 +531,40 @@ int orc_accept(const uint32_t* tok, const int32_t* parent, const int32_t* n_node
 }
 
 // ---------------------------------------------------------------------------
+// O10. The target model's greedy prediction at every tree node (Section IV-D:
+// verification compares each draft token with the model's most likely next
+// token): argmax over the vocabulary of the node's logits row.  bf16 values
+// are compared exactly as real numbers (-0 equals +0); the first index of the
+// maximum wins; a NaN counts as larger than every number and the first NaN
+// wins (the convention of torch.argmax and numpy.argmax).  Rows >= n_nodes[b]
+// get 0.
+int orc_argmax_rows(const uint16_t* logits, int B, int n_pad, int vocab, const int32_t* n_nodes,
+                    uint32_t* argmax) {
+  for (int b = 0; b < B; ++b) {
+    for (int i = 0; i < n_pad; ++i) {
+      uint32_t best = 0;
+      if (i < n_nodes[b]) {
+        const uint16_t* row = logits + ((size_t)b * n_pad + i) * (size_t)vocab;
+        double bv = bf16_to_double(row[0]);
+        bool bnan = std::isnan(bv);
+        for (int v = 1; v < vocab && !bnan; ++v) {
+          const double x = bf16_to_double(row[v]);
+          if (std::isnan(x)) {
+            best = (uint32_t)v;
+            bnan = true;
+          } else if (x > bv) {
+            best = (uint32_t)v;
+            bv = x;
+          }
+        }
+      }
+      argmax[(size_t)b * n_pad + i] = best;
+    }
+  }
+  return 0;
+}
+
+// ---------------------------------------------------------------------------
 // O8. Cache update after acceptance (implied by the decoding loop of
 // Section II and Section IV-D): the K/V rows of the accepted path (root
 // included) move into the cache at kv_len..kv_len+acc_len, kv_len grows by

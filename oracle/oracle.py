@@ -198,6 +198,18 @@ def accept(tok, parent, n_nodes, argmax, path_cap):
     return out
 
 
+# ------------------------------------------------------------------- O10
+def argmax_rows(logits, n_nodes):
+    """logits: bf16 bit patterns uint16 [B, Np, V] -> uint32 [B, Np] (rows >= n_nodes are 0)."""
+    logits = _c(logits, np.uint16)
+    n_nodes = _c(n_nodes, np.int32)
+    B, Np, V = logits.shape
+    out = np.empty((B, Np), np.uint32)
+    rc = lib().orc_argmax_rows(_p(logits), C.c_int(B), C.c_int(Np), C.c_int(V), _p(n_nodes), _p(out))
+    assert rc == 0, rc
+    return out
+
+
 # -------------------------------------------------------------------- O8
 def kv_append(path, acc_len, bonus, tok, k_tree, v_tree, k_cache, v_cache, kv_len, ctx, ctx_len):
     """In place on k_cache, v_cache, ctx; returns (kv_len_out, ctx_len_out, root_out)."""
