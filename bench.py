@@ -67,9 +67,10 @@ def parse_args(argv=None):
     ap.add_argument("--batch", type=int, default=32)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--mode", choices=["step", "attn"], default="step",
+    ap.add_argument("--mode", choices=["step", "attn", "argmax"], default="step",
                     help="step: the full step loop (the benchmark); attn: tree attention alone on the step loop's "
-                         "attention shape with seeded trees (a small profiling / sweep target)")
+                         "attention shape with seeded trees (a small profiling / sweep target); argmax: greedy "
+                         "verification from bf16 logits (fc_argmax_accept) on the step loop's tree shape")
     ap.add_argument("--nodes", type=int, default=128, help="attn mode: tree nodes per sequence")
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
     ap.add_argument("--traffic-bytes", type=float, default=None,
@@ -631,6 +632,64 @@ def run_attn(args, rank, ws, local):
             "clocks": clock_rec}
 
 
+def run_argmax(args, rank, ws, local):
+    """fc_argmax_accept alone: B sequences of seeded random trees (node counts
+    uniform in [40, 128], mean ~84 like the step loop's), bf16 N(0,1) logits over
+    the 32256-token vocabulary whose argmax follows the first branch for a
+    seeded 0-8 prefix.  HBM-bound: every valid row is read once."""
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    import paper_2502_17139_gb300.synth as synth
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    B, n_pad, V = args.batch, 128, synth.VOCAB
+    rng = synth.rng_for(6, 600 + rank)
+    tok = np.full((B, n_pad), 0xFFFFFFFF, np.uint32)
+    par = np.full((B, n_pad), -1, np.int32)
+    nn = rng.integers(40, n_pad + 1, B).astype(np.int32)
+    for b in range(B):
+        t, pp = synth.random_tree(rng, int(nn[b]), 10, 4, V)
+        tok[b, :nn[b]], par[b, :nn[b]] = t, pp
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32) if a.dtype == np.uint32
+                                        else np.ascontiguousarray(a)).to(dev)
+    plen, rtok = synth.argmax_draws(rng, B, n_pad, V)
+    pred = fc.fc_synth_argmax(to_dev(tok), to_dev(par), to_dev(nn), to_dev(plen), to_dev(rtok), V)
+    g = torch.Generator(device=dev)
+    g.manual_seed(11 + rank)
+    logits = torch.randn((B, n_pad, V), generator=g, device=dev, dtype=torch.float32)
+    logits.scatter_(2, pred.long().unsqueeze(2), 8.0)  # the planted predictions win
+    logits = logits.to(torch.bfloat16)
+    args_d = (logits, to_dev(tok), to_dev(par), to_dev(nn), 12)
+    out = fc.fc_argmax_accept(*args_d)
+    assert torch.equal(out["argmax"], pred), "planted predictions were not the argmax"
+    for _ in range(args.warmup):
+        fc.fc_argmax_accept(*args_d, out=out)
+    assert fc.fc_get_error() == "FC_OK"
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    barrier(ws)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.wait_first()
+    for e0, e1 in evs:
+        e0.record()
+        fc.fc_argmax_accept(*args_d, out=out)
+        e1.record()
+    torch.cuda.synchronize()
+    clock_rec = clocks.stop()
+    ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in evs)
+    rows = int(nn.sum())
+    bytes_ = rows * V * 2 + B * n_pad * 4 + B * n_pad * 8  # logits rows read, predictions written, tree read
+    peaks = load_peaks()
+    gbs = bytes_ / (ms * 1e-3) / 1e9
+    return {"metric": "argmax+accept GB/s", "value": gbs, "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "config": {"workload": f"greedy verification from logits B={B} n_pad={n_pad} vocab={V} "
+                                   f"rows={rows} (logits {B * n_pad * V * 2 / 1e6:.0f} MB)"},
+            "frac_hbm": gbs / peaks["hbm"], "bytes": bytes_,
+            "mean_acc_len": float(out["acc_len"].float().mean().item()), "clocks": clock_rec}
+
+
 def main(argv=None):
     args = parse_args(argv)
     rank, ws, local = dist_setup(args.gpus)
@@ -638,6 +697,8 @@ def main(argv=None):
         out = run_reference(args, rank, ws)
     elif args.mode == "attn":
         out = run_attn(args, rank, ws, local)
+    elif args.mode == "argmax":
+        out = run_argmax(args, rank, ws, local)
     else:
         out = run_ours(args, rank, ws, local)
     if rank == 0 and out is not None:

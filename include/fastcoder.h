@@ -310,6 +310,24 @@ fc_status fc_accept(const uint32_t* d_tok, const int32_t* d_parent, const int32_
                     int32_t* d_path, int path_cap, uint32_t* d_bonus, fc_stream s);
 
 /*
+ * Greedy verification straight from the target model's logits (Section IV-D:
+ * each draft token is checked against the model's most likely next token):
+ * the argmax of every tree node's logits row, then the walk of fc_accept.
+ *   d_logits  bf16 [batch][n_pad][vocab]; rows i >= n_nodes[b] are not read;
+ *             2-byte aligned (rows need not be 16-byte aligned)
+ *   d_argmax  [batch][n_pad] uint32 out: the prediction at every node (0 for
+ *             rows >= n_nodes)
+ *   the other arguments and outputs as fc_accept
+ * Ties go to the smallest index; a NaN counts as larger than every number and
+ * the first NaN wins (the convention of torch.argmax).  Each valid row is read
+ * once with 16-byte loads (HBM-bound).  Two kernels on `s`.
+ */
+fc_status fc_argmax_accept(const void* d_logits, int vocab, const uint32_t* d_tok,
+                           const int32_t* d_parent, const int32_t* d_n_nodes, int batch,
+                           int n_pad, uint32_t* d_argmax, int32_t* d_acc_len, int32_t* d_path,
+                           int path_cap, uint32_t* d_bonus, fc_stream s);
+
+/*
  * Closes a decoding step: copies the K/V rows of the accepted path (root
  * included) to cache rows kv_len_in[b] .. kv_len_in[b] + acc_len[b],
  * writes kv_len_out = kv_len_in + acc_len + 1, appends the accepted draft

@@ -1,4 +1,5 @@
-// fc_accept, fc_kv_append and fc_synth_argmax: the end of a decoding step.
+// fc_accept, fc_argmax_accept, fc_kv_append and fc_synth_argmax: the end of a
+// decoding step.
 //
 // Acceptance follows Section IV-D (every correct token from the start is
 // accepted, everything after the first error rejected); the cache append
@@ -11,28 +12,43 @@ FC_DEFINE_ERROR_WORD(step)
 
 namespace {
 
-// One warp per sequence.  Children of `cur` sit after it in preorder, so the
-// warp scans node ids cur+1 .. n-1 in chunks of 32 with one ballot each.
-__global__ void k_accept(const uint32_t* __restrict__ tok, const int32_t* __restrict__ parent,
-                         const int32_t* __restrict__ n_nodes, const uint32_t* __restrict__ argmax, int B, int n_pad,
-                         int32_t* __restrict__ acc_len, int32_t* __restrict__ path, int path_cap,
-                         uint32_t* __restrict__ bonus) {
-  const int b = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+// One warp per sequence.  The tree (parents, tokens, predictions) is staged in
+// shared memory with one coalesced read; children of `cur` sit after it in
+// preorder, so the warp scans node ids cur+1 .. n-1 in chunks of 32 with one
+// ballot each.
+constexpr int ACC_WARPS = 4;  // sequences per CTA
+__global__ void __launch_bounds__(ACC_WARPS * 32) k_accept(const uint32_t* __restrict__ tok,
+                                                           const int32_t* __restrict__ parent,
+                                                           const int32_t* __restrict__ n_nodes,
+                                                           const uint32_t* __restrict__ argmax, int B, int n_pad,
+                                                           int32_t* __restrict__ acc_len, int32_t* __restrict__ path,
+                                                           int path_cap, uint32_t* __restrict__ bonus) {
+  extern __shared__ uint32_t acc_smem[];  // [ACC_WARPS][3][n_pad]
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * ACC_WARPS + w;
   if (b >= B) return;
+  uint32_t* s_tok = acc_smem + (size_t)w * 3 * n_pad;
+  int32_t* s_par = reinterpret_cast<int32_t*>(s_tok + n_pad);
+  uint32_t* s_am = s_tok + 2 * n_pad;
   const size_t base = (size_t)b * n_pad;
   const int n = min(max((int)n_nodes[b], 1), n_pad);
+  for (int j = lane; j < n; j += 32) {
+    s_tok[j] = tok[base + j];
+    s_par[j] = parent[base + j];
+    s_am[j] = argmax[base + j];
+  }
   int32_t* pth = path + (size_t)b * path_cap;
   for (int t = lane; t < path_cap; t += 32) pth[t] = -1;
   __syncwarp();
   int cur = 0, len = 0;
   bool overflow = false;
   for (;;) {
-    const uint32_t want = argmax[base + cur];
+    const uint32_t want = s_am[cur];
     int next = -1;
     for (int j0 = cur + 1; j0 < n && next < 0; j0 += 32) {
-      int j = j0 + lane;
-      bool hit = j < n && parent[base + j] == cur && tok[base + j] == want;
-      uint32_t m = __ballot_sync(0xFFFFFFFFu, hit);
+      const int j = j0 + lane;
+      const bool hit = j < n && s_par[j] == cur && s_tok[j] == want;
+      const uint32_t m = __ballot_sync(0xFFFFFFFFu, hit);
       if (m) next = j0 + __ffs(m) - 1;
     }
     if (next < 0) break;
@@ -47,7 +63,7 @@ __global__ void k_accept(const uint32_t* __restrict__ tok, const int32_t* __rest
   if (lane == 0) {
     pth[0] = 0;
     acc_len[b] = len;
-    bonus[b] = argmax[base + cur];
+    bonus[b] = s_am[cur];
     if (overflow) fc_flag(&g_fc_err, FC_EBIT_CAPACITY);
   }
 }
@@ -102,6 +118,114 @@ __global__ void k_kv_append(const int32_t* __restrict__ path, const int32_t* __r
     ctx_len_out[b] = cl + a + 1;
     root_out[b] = bonus[b];
   }
+}
+
+// ---- greedy predictions from logits: one warp per tree node's row ----
+// Ordering of (value, index) candidates: a NaN beats every number (the first
+// NaN wins), otherwise the larger value, ties to the smaller index (-0 == +0).
+__device__ __forceinline__ bool am_better(float a, int ia, float b, int ib) {
+  const bool na = a != a, nb = b != b;
+  if (na || nb) return na && (!nb || ia < ib);
+  return a > b || (a == b && ia < ib);
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+constexpr int AM_WARPS = 8;  // rows per CTA
+
+// NaN-propagating maximum of two bf16 pairs.
+__device__ __forceinline__ uint32_t max_nan_bf16x2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.NaN.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+
+// Rows (b, i) with i < n_nodes[b]: argmax over the vocabulary.  The row is read
+// once: a scalar head up to a 16-byte boundary, then 16-byte chunks (8 bf16)
+// with eight loads in flight per lane, then a scalar tail.  Per chunk a lane
+// only takes the NaN-propagating maximum (three max.bf16x2) and keeps the
+// first chunk holding its best value (or its first NaN); afterwards it rereads
+// that one chunk for the first element equal to it.  The warp reduction then
+// orders candidates by (value, index).
+__global__ void __launch_bounds__(AM_WARPS * 32) k_argmax_rows(const uint16_t* __restrict__ logits, int vocab,
+                                                                const int32_t* __restrict__ n_nodes, int n_pad,
+                                                                uint32_t* __restrict__ argmax) {
+  const int b = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int i = blockIdx.x * AM_WARPS + warp;
+  if (i >= n_pad) return;
+  const int n = min(max((int)n_nodes[b], 0), n_pad);
+  const size_t row = (size_t)b * n_pad + i;
+  if (i >= n) {
+    if (lane == 0) argmax[row] = 0u;
+    return;
+  }
+  const uint16_t* p = logits + row * (size_t)vocab;
+  float bv = -INFINITY;
+  int bi = 0x7FFFFFFF;
+  // head: elements before the first 16-byte boundary
+  const int head = min(vocab, (int)(((16u - (uint32_t)(reinterpret_cast<uintptr_t>(p) & 15u)) & 15u) >> 1));
+  if (lane < head) {
+    bv = __uint_as_float((uint32_t)__ldg(p + lane) << 16);
+    bi = lane;
+  }
+  const int nvec = (vocab - head) >> 3;  // whole 8-element chunks
+  const uint4* pv = reinterpret_cast<const uint4*>(p + head);
+  float cv = -INFINITY;  // this lane's best chunk maximum
+  int cc = -1;           // and its chunk
+  auto take = [&](uint4 v, int c) {
+    const uint32_t m = max_nan_bf16x2(max_nan_bf16x2(v.x, v.y), max_nan_bf16x2(v.z, v.w));
+    const float lo = bf16_lo(m), hi = bf16_hi(m);
+    const float mc = (lo != lo || hi != hi) ? __int_as_float(0x7FC00000) : fmaxf(lo, hi);
+    if (cv == cv && (mc != mc || mc > cv || cc < 0)) {  // a NaN sticks; otherwise a strictly larger one
+      cv = mc;
+      cc = c;
+    }
+  };
+  int c = lane;
+  for (; c + 7 * 32 < nvec; c += 8 * 32) {  // eight 16-byte loads in flight per lane
+    uint4 v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) v[u] = __ldg(pv + c + 32 * u);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) take(v[u], c + 32 * u);
+  }
+  for (; c < nvec; c += 32) take(__ldg(pv + c), c);
+  if (cc >= 0) {  // the first element of the best chunk that attains its maximum
+    const uint4 v = __ldg(pv + cc);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    int e = 7;
+#pragma unroll
+    for (int q = 3; q >= 0; --q) {
+      const float hi = bf16_hi(w[q]), lo = bf16_lo(w[q]);
+      if (hi == cv || (cv != cv && hi != hi)) e = 2 * q + 1;
+      if (lo == cv || (cv != cv && lo != lo)) e = 2 * q;
+    }
+    const int idx = head + 8 * cc + e;
+    if (am_better(cv, idx, bv, bi)) {
+      bv = cv;
+      bi = idx;
+    }
+  }
+  // tail: the last (vocab - head) % 8 elements
+  const int t0 = head + 8 * nvec;
+  if (t0 + lane < vocab) {
+    const float x = __uint_as_float((uint32_t)__ldg(p + t0 + lane) << 16);
+    if (am_better(x, t0 + lane, bv, bi)) {
+      bv = x;
+      bi = t0 + lane;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xFFFFFFFFu, bv, o);
+    const int oi = __shfl_xor_sync(0xFFFFFFFFu, bi, o);
+    if (am_better(ov, oi, bv, bi)) {
+      bv = ov;
+      bi = oi;
+    }
+  }
+  if (lane == 0) argmax[row] = (uint32_t)bi;
 }
 
 // One CTA per sequence, one thread per node.
@@ -160,11 +284,30 @@ extern "C" fc_status fc_accept(const uint32_t* d_tok, const int32_t* d_parent, c
   if (batch < 0 || n_pad < 1 || n_pad > 1024 || path_cap < 1) return FC_ERR_INVALID_ARG;
   if (batch == 0) return FC_OK;
   if (!d_tok || !d_parent || !d_n_nodes || !d_argmax || !d_acc_len || !d_path || !d_bonus) return FC_ERR_INVALID_ARG;
-  const int threads = 128;
-  const unsigned blocks = (unsigned)((batch * 32 + threads - 1) / threads);
-  k_accept<<<blocks, threads, 0, static_cast<cudaStream_t>(stream)>>>(d_tok, d_parent, d_n_nodes, d_argmax, batch,
-                                                                      n_pad, d_acc_len, d_path, path_cap, d_bonus);
+  const unsigned blocks = (unsigned)((batch + ACC_WARPS - 1) / ACC_WARPS);
+  const size_t smem = (size_t)ACC_WARPS * 3 * n_pad * sizeof(uint32_t);  // <= 48 KB for n_pad <= 1024
+  k_accept<<<blocks, ACC_WARPS * 32, smem, static_cast<cudaStream_t>(stream)>>>(
+      d_tok, d_parent, d_n_nodes, d_argmax, batch, n_pad, d_acc_len, d_path, path_cap, d_bonus);
   return FC_CHECK_LAUNCH();
+}
+
+extern "C" fc_status fc_argmax_accept(const void* d_logits, int vocab, const uint32_t* d_tok,
+                                      const int32_t* d_parent, const int32_t* d_n_nodes, int batch, int n_pad,
+                                      uint32_t* d_argmax, int32_t* d_acc_len, int32_t* d_path, int path_cap,
+                                      uint32_t* d_bonus, fc_stream stream) {
+  if (batch < 0 || n_pad < 1 || n_pad > 1024 || path_cap < 1 || vocab < 1) return FC_ERR_INVALID_ARG;
+  if (batch > 65535) return FC_ERR_UNSUPPORTED;
+  if (batch == 0) return FC_OK;
+  if (!d_logits || !d_tok || !d_parent || !d_n_nodes || !d_argmax || !d_acc_len || !d_path || !d_bonus)
+    return FC_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(d_logits) % 2) return FC_ERR_INVALID_ARG;
+  const dim3 grid((unsigned)((n_pad + AM_WARPS - 1) / AM_WARPS), (unsigned)batch);
+  k_argmax_rows<<<grid, AM_WARPS * 32, 0, static_cast<cudaStream_t>(stream)>>>(
+      static_cast<const uint16_t*>(d_logits), vocab, d_n_nodes, n_pad, d_argmax);
+  const fc_status st = FC_CHECK_LAUNCH();
+  if (st != FC_OK) return st;
+  return fc_accept(d_tok, d_parent, d_n_nodes, d_argmax, batch, n_pad, d_acc_len, d_path, path_cap, d_bonus,
+                   stream);
 }
 
 extern "C" fc_status fc_kv_append(const int32_t* d_path, const int32_t* d_acc_len, const uint32_t* d_bonus,

@@ -47,7 +47,7 @@ class fc_retrieve_params(C.Structure):
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
            "fc_datastore_build_noalloc",
            "fc_retrieve", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
-           "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_accept", "fc_kv_append", "fc_synth_argmax"]
+           "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
 
 
 def _load():
@@ -79,6 +79,7 @@ def _load():
         "fc_tree_attn_workspace": (sz, [i32, i32, i32, i32]),
         "fc_tree_attn_parts": (C.c_int, [i32, i32, i32, i32, i32, sz]),
         "fc_accept": (C.c_int, [vp, vp, vp, vp, i32, i32, vp, vp, i32, vp, vp]),
+        "fc_argmax_accept": (C.c_int, [vp, i32, vp, vp, vp, i32, i32, vp, vp, vp, i32, vp, vp]),
         "fc_kv_append": (C.c_int, [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, i32,
                                    vp, vp, vp, vp]),
         "fc_synth_argmax": (C.c_int, [vp, vp, vp, i32, i32, vp, vp, u32, vp, vp]),
@@ -340,6 +341,24 @@ def fc_accept(tok, parent, n_nodes, argmax, path_cap, out=None):
                                          bonus=torch.empty(B, dtype=torch.int32, device=dev))
     _check("fc_accept", LIB.fc_accept(_ptr(tok), _ptr(parent), _ptr(n_nodes), _ptr(argmax), B, Np, _ptr(o["acc_len"]),
                                       _ptr(o["path"]), path_cap, _ptr(o["bonus"]), _stream()))
+    return o
+
+
+def fc_argmax_accept(logits, tok, parent, n_nodes, path_cap, out=None):
+    """logits bf16 [B, Np, V]; returns dict(argmax [B, Np], acc_len, path, bonus) (int32)."""
+    _need(logits, torch.bfloat16, "logits")
+    B, Np, V = logits.shape
+    for t, nm in ((tok, "tok"), (parent, "parent")):
+        _need(t, torch.int32, nm, (B, Np))
+    _need(n_nodes, torch.int32, "n_nodes", (B,))
+    dev = tok.device
+    o = out if out is not None else dict(argmax=torch.empty((B, Np), dtype=torch.int32, device=dev),
+                                         acc_len=torch.empty(B, dtype=torch.int32, device=dev),
+                                         path=torch.empty((B, path_cap), dtype=torch.int32, device=dev),
+                                         bonus=torch.empty(B, dtype=torch.int32, device=dev))
+    _check("fc_argmax_accept", LIB.fc_argmax_accept(_ptr(logits), V, _ptr(tok), _ptr(parent), _ptr(n_nodes), B, Np,
+                                                    _ptr(o["argmax"]), _ptr(o["acc_len"]), _ptr(o["path"]), path_cap,
+                                                    _ptr(o["bonus"]), _stream()))
     return o
 
 

@@ -84,5 +84,8 @@ def test_host_validation_without_gpu(lib):
     assert L.fc_datastore_build(1, 1000, 10, 1, 1, 1, 256, need - 1, nul, nul) == 3
     # kv append: aliasing in/out lengths
     assert L.fc_kv_append(1, 1, 1, 1, 16, 16, 2, 64, 8, 128, 12, 16, 16, 100, 8, 8, 1, 64, 4, 12, 1, nul) == 1
+    # argmax + accept: an empty vocabulary, an odd logits address
+    assert L.fc_argmax_accept(16, 0, 16, 16, 16, 2, 64, 16, 16, 16, 12, 16, nul) == 1
+    assert L.fc_argmax_accept(17, 100, 16, 16, 16, 2, 64, 16, 16, 16, 12, 16, nul) == 1
     # cache: capacity must be a power of two
     assert L.fc_rcache_init(1, 1 << 30, 1000, 2, p, nul) == 1

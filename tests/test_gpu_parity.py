@@ -411,6 +411,48 @@ def test_accept_and_synth_argmax(fc, orc):
     check_no_error(fc)
 
 
+def _logits_with_predictions(rng, pred, V, n_nodes, extras=True):
+    """bf16 logits [B, Np, V] whose row argmax is `pred` (planted maxima; ties
+    and NaNs placed so that the first index / first NaN rule decides)."""
+    B, Np = pred.shape
+    x = rng.standard_normal((B, Np, V)).astype(np.float32)
+    for b in range(B):
+        for i in range(Np):
+            p = int(pred[b, i])
+            x[b, i, p] = 8.0 + rng.random()  # clear winner
+            if extras and V > 3 and rng.random() < 0.2:
+                x[b, i, p:] = np.minimum(x[b, i, p:], x[b, i, p])  # later ties lose
+                q = int(rng.integers(p, V))
+                x[b, i, q] = x[b, i, p]
+            if extras and rng.random() < 0.05:
+                x[b, i, p] = np.nan                               # the first NaN wins
+    h = (x.view(np.uint32) >> 16).astype(np.uint16)  # truncation: exact bf16 values
+    return h
+
+
+def test_argmax_accept_from_logits(fc, orc):
+    rng = synth.rng_for(62)
+    for n_pad, V, B in ((64, 32256, 8), (128, 1001, 6), (64, 7, 10)):
+        tok, par, nn = _random_trees(rng, B, n_pad, vocab=V)
+        plen, rtok = synth.argmax_draws(rng, B, n_pad, V)
+        pred = orc.synth_argmax(tok, par, nn, plen, rtok, V)
+        h = _logits_with_predictions(rng, pred, V, nn)
+        # odd element offset: rows start off any 16-byte boundary
+        flat = torch.zeros(h.size + 1, dtype=torch.int16, device="cuda")
+        flat[1:] = torch.from_numpy(h.reshape(-1).view(np.int16)).cuda()
+        logits = flat[1:].view(torch.bfloat16).view(B, n_pad, V)
+        g = fc.fc_argmax_accept(logits, dev(tok), dev(par), dev(nn), 12)
+        r_am = orc.argmax_rows(h, nn)
+        assert np.array_equal(host_u32(g["argmax"]), r_am)
+        r = orc.accept(tok, par, nn, r_am, 12)
+        assert np.array_equal(g["acc_len"].cpu().numpy(), r["acc_len"])
+        assert np.array_equal(g["path"].cpu().numpy(), r["path"])
+        assert np.array_equal(host_u32(g["bonus"]), r["bonus"])
+        if V == 32256:  # the planted predictions are the argmax where no NaN was planted
+            assert (r["acc_len"] > 0).any()
+    check_no_error(fc)
+
+
 def test_kv_append_copy(fc, orc):
     rng = synth.rng_for(61)
     B, n_pad, Hkv, D, cap, stride = 16, 64, 8, 128, 300, 200
