@@ -24,6 +24,9 @@ __global__ void __launch_bounds__(ACC_WARPS * 32) k_accept(const uint32_t* __res
                                                            int32_t* __restrict__ acc_len, int32_t* __restrict__ path,
                                                            int path_cap, uint32_t* __restrict__ bonus) {
   extern __shared__ uint32_t acc_smem[];  // [ACC_WARPS][3][n_pad]
+  // Launched as a programmatic dependent of the row argmax (fc_argmax_accept):
+  // wait here until that grid's results are visible.  A no-op otherwise.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.x * ACC_WARPS + w;
   if (b >= B) return;
@@ -151,6 +154,8 @@ __device__ __forceinline__ uint32_t max_nan_bf16x2(uint32_t a, uint32_t b) {
 __global__ void __launch_bounds__(AM_WARPS * 32) k_argmax_rows(const uint16_t* __restrict__ logits, int vocab,
                                                                 const int32_t* __restrict__ n_nodes, int n_pad,
                                                                 uint32_t* __restrict__ argmax) {
+  // the acceptance walk may be scheduled now; it waits for this grid's results
+  asm volatile("griddepcontrol.launch_dependents;");
   const int b = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * AM_WARPS + warp;
   if (i >= n_pad) return;
@@ -306,8 +311,22 @@ extern "C" fc_status fc_argmax_accept(const void* d_logits, int vocab, const uin
       static_cast<const uint16_t*>(d_logits), vocab, d_n_nodes, n_pad, d_argmax);
   const fc_status st = FC_CHECK_LAUNCH();
   if (st != FC_OK) return st;
-  return fc_accept(d_tok, d_parent, d_n_nodes, d_argmax, batch, n_pad, d_acc_len, d_path, path_cap, d_bonus,
-                   stream);
+  // the walk as a programmatic dependent launch: it is scheduled while the
+  // argmax grid runs and waits (griddepcontrol.wait) for its completion
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)((batch + ACC_WARPS - 1) / ACC_WARPS));
+  cfg.blockDim = dim3(ACC_WARPS * 32);
+  cfg.dynamicSmemBytes = (size_t)ACC_WARPS * 3 * n_pad * sizeof(uint32_t);
+  cfg.stream = static_cast<cudaStream_t>(stream);
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, k_accept, d_tok, d_parent, d_n_nodes, (const uint32_t*)d_argmax, batch, n_pad,
+                         d_acc_len, d_path, path_cap, d_bonus) != cudaSuccess)
+    return FC_ERR_CUDA;
+  return FC_CHECK_LAUNCH();
 }
 
 extern "C" fc_status fc_kv_append(const int32_t* d_path, const int32_t* d_acc_len, const uint32_t* d_bonus,
