@@ -67,12 +67,15 @@ def parse_args(argv=None):
     ap.add_argument("--batch", type=int, default=32)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--mode", choices=["step", "attn", "argmax"], default="step",
+    ap.add_argument("--mode", choices=["step", "attn", "argmax", "configs", "retrieve"], default="step",
                     help="step: the full step loop (the benchmark); attn: tree attention alone on the step loop's "
                          "attention shape with seeded trees (a small profiling / sweep target); argmax: greedy "
-                         "verification from bf16 logits (fc_argmax_accept) on the step loop's tree shape")
+                         "verification from bf16 logits (fc_argmax_accept) on the step loop's tree shape; configs: "
+                         "every stage of the five benchmark configurations timed once each (a report, not the "
+                         "benchmark line); retrieve: two-source retrieval alone for --batch queries (batch sweeps)")
     ap.add_argument("--nodes", type=int, default=128, help="attn mode: tree nodes per sequence")
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
+    ap.add_argument("--skip-1b", action="store_true", help="configs mode: leave out the 1B-token configuration")
     ap.add_argument("--traffic-bytes", type=float, default=None,
                     help="ncu dram read+write bytes of one tree-attention launch of this workload")
     return ap.parse_args(argv)
@@ -690,6 +693,178 @@ def run_argmax(args, rank, ws, local):
             "mean_acc_len": float(out["acc_len"].float().mean().item()), "clocks": clock_rec}
 
 
+def _cuda_ms(fn, reps=10, warm=3):
+    """Mean CUDA-event time of fn() on the current stream, after warm-up."""
+    import torch
+    for _ in range(warm):
+        fn()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    for e0, e1 in ev:
+        e0.record()
+        fn()
+        e1.record()
+    torch.cuda.synchronize()
+    return statistics.mean(a.elapsed_time(b) for a, b in ev)
+
+
+def _attn_work(fc, tree, kvl, H, Hkv, D):
+    """Unmasked (q, k) pair FLOPs and algorithmic bytes of one tree-attention call."""
+    nn = tree["n_nodes"].cpu().numpy().astype(np.int64)
+    dep = tree["depth"].cpu().numpy().astype(np.int64)
+    B = len(nn)
+    pairs = sum(H * (nn[b] * kvl[b] + int((dep[b, :nn[b]] + 1).sum())) for b in range(B))
+    by = sum(2 * Hkv * kvl[b] * D * 2 + 2 * Hkv * nn[b] * D * 2 + 2 * nn[b] * H * D * 2 for b in range(B))
+    return 4.0 * D * pairs, float(by)
+
+
+def run_configs(args, rank, ws, local):
+    """Every stage of the five configurations on this GPU (CUDA events, mean of
+    10 after 3 warm-up calls): a report of where each configuration stands
+    against its roofline; the benchmark line is the step loop (--mode step)."""
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    import paper_2502_17139_gb300.synth as synth
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    peaks = load_peaks()
+    tc, bw = peaks["tc_sustained"] * 1e12, peaks["hbm"] * 1e9
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32) if a.dtype == np.uint32
+                                        else np.ascontiguousarray(a)).to(dev)
+    out = {"metric": "per-configuration stage times", "unit": "ms", "configs": {}}
+
+    def attn_entry(tree, kvl, H, Hkv, D, L_cap, seed):
+        B, n_pad = tree["tok"].shape
+        g = torch.Generator(device=dev)
+        g.manual_seed(seed)
+        rnd = lambda *sh: torch.randn(*sh, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+        q, kc, vc = rnd(B, n_pad, H, D), rnd(B, Hkv, L_cap, D), rnd(B, Hkv, L_cap, D)
+        kt, vt = rnd(B, Hkv, n_pad, D), rnd(B, Hkv, n_pad, D)
+        o = torch.empty_like(q)
+        kv_d = to_dev(np.asarray(kvl, np.int32))
+        ms = _cuda_ms(lambda: fc.fc_tree_attn(q, kc, vc, kv_d, kt, vt, tree["mask"], tree["n_nodes"], out=o))
+        F, By = _attn_work(fc, tree, kvl, H, Hkv, D)
+        t_roof = max(F / tc, By / bw)
+        return {"ms": ms, "tflops": F / (ms * 1e-3) / 1e12, "gbs": By / (ms * 1e-3) / 1e9,
+                "bound": "tensor" if F / tc >= By / bw else "hbm", "frac_of_roofline": t_roof / (ms * 1e-3)}
+
+    def accept_entry(tree, V, seed, plen_max=8):
+        B, n_pad = tree["tok"].shape
+        rng = synth.rng_for(7, seed)
+        plen, rtok = synth.argmax_draws(rng, B, n_pad, V, plen_max)
+        am = fc.fc_synth_argmax(tree["tok"], tree["parent"], tree["n_nodes"], to_dev(plen), to_dev(rtok), V)
+        acc = fc.fc_accept(tree["tok"], tree["parent"], tree["n_nodes"], am, 12)
+        ms = _cuda_ms(lambda: fc.fc_accept(tree["tok"], tree["parent"], tree["n_nodes"], am, 12, out=acc))
+        nn = tree["n_nodes"].cpu().numpy()
+        by = float(sum(12 * int(n) + 4 * (12 + 2) for n in nn))
+        return {"ms": ms, "gbs": by / (ms * 1e-3) / 1e9, "frac_hbm": by / (ms * 1e-3) / bw,
+                "mean_acc_len": float(acc["acc_len"].float().mean().item())}
+
+    def retrieval_entry(sources, ctx, cl, cfg, budget, n_pad, kv0):
+        p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
+        ctx_d, cl_d = to_dev(ctx), to_dev(cl)
+        res = fc.fc_retrieve(sources, ctx_d, cl_d, p)
+        ms_r = _cuda_ms(lambda: fc.fc_retrieve(sources, ctx_d, cl_d, p, out=res))
+        B = ctx.shape[0]
+        root = to_dev(ctx[np.arange(B), cl - 1].astype(np.uint32))
+        kvl = to_dev(np.full(B, kv0, np.int32))
+        tree = fc.fc_build_tree(res, [1] * len(sources), root, kvl, budget, n_pad)
+        ms_t = _cuda_ms(lambda: fc.fc_build_tree(res, [1] * len(sources), root, kvl, budget, n_pad, out=tree))
+        ml = res["match_len"].cpu().numpy()
+        return tree, {"retrieve_ms": ms_r, "queries_per_s": B / (ms_r * 1e-3),
+                      "us_per_query_source": ms_r * 1e3 / (B * len(sources)),
+                      "matched_share": float((ml > 0).mean()), "build_tree_ms": ms_t,
+                      "mean_tree_nodes": float(tree["n_nodes"].float().mean().item())}
+
+    def build_entry(T):
+        t0 = time.perf_counter()
+        ds = fc.fc_datastore_build(to_dev(T), synth.VOCAB)
+        torch.cuda.synchronize()
+        sec = time.perf_counter() - t0
+        return ds, {"tokens": int(len(T)), "seconds": sec, "tokens_per_s": len(T) / sec}
+
+    # c1: single source 1M, B=32, attention H = Hkv = 32, KV 512
+    cfg = synth.CONFIGS[1]
+    rng = synth.rng_for(1)
+    T, _ = synth.build_corpus(rng, cfg["corpus"][0], device="cuda")
+    ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], [T], [1.0], 1.1)
+    ds, e_build = build_entry(T)
+    tree, e_ret = retrieval_entry([ds], ctx, cl, cfg, cfg["node_budget"], cfg["n_pad"], cfg["kv_len"])
+    kvl = [cfg["kv_len"]] * cfg["batch"]
+    out["configs"]["c1"] = dict(datastore_build=e_build, retrieval_and_tree=e_ret,
+                                tree_attn=attn_entry(tree, kvl, cfg["H"], cfg["Hkv"], cfg["D"], cfg["kv_len"], 1),
+                                accept=accept_entry(tree, synth.VOCAB, 1))
+    del ds, T
+    # c2: two sources 5M + 100M, B=256, 64-node trees
+    cfg = synth.CONFIGS[2]
+    rng = synth.rng_for(2)
+    corpora = [synth.build_corpus(rng, spec, device="cuda")[0] for spec in cfg["corpus"]]
+    ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], corpora + [None], cfg["probs"],
+                                     1.1)
+    built = [build_entry(T) for T in corpora]
+    tree, e_ret = retrieval_entry([b[0] for b in built], ctx, cl, cfg, cfg["node_budget"], cfg["n_pad"], 4096)
+    out["configs"]["c2"] = dict(datastore_build=[b[1] for b in built], retrieval_and_tree=e_ret)
+    del built, corpora
+    # c3: attention at the 7B shape, B=16, H = Hkv = 32, KV 4096, 64-node random trees; acceptance
+    cfg = synth.CONFIGS[3]
+    rng = synth.rng_for(3)
+    B, n_pad, nnod = cfg["batch"], cfg["n_pad"], cfg["n_nodes"]
+    tok = np.full((B, n_pad), 0xFFFFFFFF, np.uint32)
+    par = np.full((B, n_pad), -1, np.int32)
+    for b in range(B):
+        t, pp = synth.random_tree(rng, nnod, cfg["depth_max"], cfg["branch_max"], synth.VOCAB)
+        tok[b, :nnod], par[b, :nnod] = t, pp
+    nn = np.full(B, nnod, np.int32)
+    kvl = [cfg["kv_len"]] * B
+    m = fc.fc_tree_mask(to_dev(par), to_dev(nn), to_dev(np.asarray(kvl, np.int32)))
+    tree3 = dict(tok=to_dev(tok), parent=to_dev(par), n_nodes=to_dev(nn), mask=m["mask"], depth=m["depth"])
+    out["configs"]["c3"] = dict(tree_attn=attn_entry(tree3, kvl, cfg["H"], cfg["Hkv"], cfg["D"], cfg["kv_len"], 3),
+                                accept=accept_entry(tree3, synth.VOCAB, 3))
+    # c4: 1B tokens, B=1024, n 24 -> 2, top-64 x 12, 128-node trees
+    if not args.skip_1b:
+        cfg = synth.CONFIGS[4]
+        rng = synth.rng_for(4)
+        T, planted = synth.build_corpus(rng, cfg["corpus"][0], device="cuda")
+        ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], [T], [1.0], 1.1,
+                                         planted=[planted], planted_share=cfg["planted_share"])
+        ds, e_build = build_entry(T)
+        tree, e_ret = retrieval_entry([ds], ctx, cl, cfg, cfg["node_budget"], cfg["n_pad"], 0)
+        out["configs"]["c4"] = dict(datastore_build=e_build, retrieval_and_tree=e_ret)
+        del ds, T
+    out["configs"]["c5"] = "the step loop: python bench.py (the benchmark line)"
+    return out
+
+
+def run_retrieve(args, rank, ws, local):
+    """Two-source retrieval alone on the step loop's datastores (5M + 100M) for
+    --batch contexts of the step loop's query mix: a batch sweep shows where the
+    dependent-probe chain stops hiding behind parallelism."""
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    import paper_2502_17139_gb300.synth as synth
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    cfg = synth.CONFIGS[2]
+    rng = synth.rng_for(2)
+    corpora = [synth.build_corpus(rng, spec, device="cuda")[0] for spec in cfg["corpus"]]
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32) if a.dtype == np.uint32
+                                        else np.ascontiguousarray(a)).to(dev)
+    sources = [fc.fc_datastore_build(to_dev(T), synth.VOCAB) for T in corpora]
+    ctx, cl, _ = synth.make_contexts(rng, args.batch, cfg["ctx_len"], cfg["n_copy"], corpora + [None], cfg["probs"],
+                                     1.1)
+    p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
+    ctx_d, cl_d = to_dev(ctx), to_dev(cl)
+    res = fc.fc_retrieve(sources, ctx_d, cl_d, p)
+    ms = _cuda_ms(lambda: fc.fc_retrieve(sources, ctx_d, cl_d, p, out=res), reps=args.steps, warm=args.warmup)
+    return {"metric": "retrievals/s", "value": 2 * args.batch / (ms * 1e-3), "unit": "query-sources/s",
+            "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "config": {"workload": f"two-source retrieval (5M + 100M tokens), {args.batch} contexts of 128, "
+                                   f"n 16->2, top-64 x 10"},
+            "us_per_query_source": ms * 1e3 / (2 * args.batch)}
+
+
 def main(argv=None):
     args = parse_args(argv)
     rank, ws, local = dist_setup(args.gpus)
@@ -699,6 +874,10 @@ def main(argv=None):
         out = run_attn(args, rank, ws, local)
     elif args.mode == "argmax":
         out = run_argmax(args, rank, ws, local)
+    elif args.mode == "configs":
+        out = run_configs(args, rank, ws, local)
+    elif args.mode == "retrieve":
+        out = run_retrieve(args, rank, ws, local)
     else:
         out = run_ours(args, rank, ws, local)
     if rank == 0 and out is not None:
