@@ -177,19 +177,26 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   const int nn = bad ? 0 : nn_raw;
   if (bad && c == 0 && part == 0 && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
 
-  // Zero the padding rows (nodes >= n_nodes) of this group; the group's part-0 CTAs share the work.
-  if (part == 0) {
+  // Zero the padding rows (nodes >= n_nodes) of this group: the group's part-0
+  // CTAs share them (row r of the G x pad padding rows goes to CTA r mod ctas),
+  // threads [t0, t0 + nthr) of this CTA take its rows.
+  auto zero_pad = [&](int t0, int nthr) {
+    if (part != 0 || tid < t0 || tid >= t0 + nthr) return;
     const int pad = a.n_pad - nn;
-    for (int e = c * TA_THREADS + tid; e < a.G * pad * (HD / 8); e += a.ctas * TA_THREADS) {
-      int r = e / (HD / 8), ch = e - r * (HD / 8);
-      int hh = r / pad, i = nn + (r - hh * pad);
+    const int my_rows = (a.G * pad - c + a.ctas - 1) / a.ctas;  // rows c, c + ctas, ...
+    for (int e = tid - t0; e < my_rows * (HD / 8); e += nthr) {
+      const int r = c + (e / (HD / 8)) * a.ctas, ch = e % (HD / 8);
+      const int hh = r / pad, i = nn + (r - hh * pad);
       reinterpret_cast<uint4*>(a.out + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD)[ch] =
           make_uint4(0, 0, 0, 0);
     }
-  }
+  };
   const int rows_total = a.G * nn;
   const int row0 = c * (TILES * BM);
-  if (row0 >= rows_total) return;
+  if (row0 >= rows_total) {
+    zero_pad(0, TA_THREADS);
+    return;
+  }
   const bool has_b = row0 + BM < rows_total;
 
   unsigned char* smem =
@@ -207,8 +214,24 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   const int nblk = (part + 1) * nblk_all / nparts - kb;
   int n_contrib = 0;
   for (int h = 0; h < nparts; ++h) n_contrib += ((h + 1) * nblk_all / nparts > h * nblk_all / nparts);
-  if (nblk == 0) return;
+  if (nblk == 0) {
+    zero_pad(0, TA_THREADS);
+    return;
+  }
 
+  // K and V of block j into stage j & 1 (the tree's own K/V form the last block)
+  auto load_kv = [&](int j, bool k_part) {
+    const int st = j & 1;
+    const bool tree = kb + j >= nblk_c;
+    const uint32_t bytes = tree ? (uint32_t)a.n_pad * 64 * 2 * 2 : TILE_BYTES;
+    const CUtensorMap* m = k_part ? (tree ? &tm_kt : &tm_kc) : (tree ? &tm_vt : &tm_vc);
+    const int y = tree ? 0 : (kb + j) * BN;
+    const uint32_t dst = (k_part ? sK : sV) + st * TILE_BYTES, fb = bar((k_part ? B_KFULL : B_VFULL) + st);
+    mbar_expect_tx(fb, bytes);
+    tma_load_3d(dst, m, 0, y, bg, fb);
+    tma_load_3d(dst + HALF_BYTES, m, 64, y, bg, fb);
+  };
+  const int n_early = min(2, nblk);  // blocks whose loads start before Q is staged
   if (tid == 0) {
     s_abort = 0;
     for (int i = 0; i < N_BARS; ++i) mbar_init(bar(i), (i == B_PFULL || i == B_PFULL + 1) ? 128u : 1u);
@@ -217,6 +240,10 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     prefetch_tmap(&tm_vc);
     prefetch_tmap(&tm_kt);
     prefetch_tmap(&tm_vt);
+    for (int j = 0; j < n_early; ++j) {  // the stages are free: start the first copies now
+      load_kv(j, true);
+      load_kv(j, false);
+    }
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(&s_tmem), TMEM_COLS);
@@ -245,26 +272,16 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     if (warp == 0) {
       // ---------------- TMA producer ----------------
       if (lane == 0) {
-        int issued = 0;
-        for (int j = 0; j < nblk; ++j) {
+        int issued = n_early;  // blocks 0 and 1 were issued at setup
+        for (int j = n_early; j < nblk; ++j) {
           const int st = j & 1;
-          const bool tree = kb + j >= nblk_c;
-          const uint32_t bytes = tree ? (uint32_t)a.n_pad * 64 * 2 * 2 : TILE_BYTES;
-          const CUtensorMap* mk = tree ? &tm_kt : &tm_kc;
-          const CUtensorMap* mv = tree ? &tm_vt : &tm_vc;
-          const int y = tree ? 0 : (kb + j) * BN;
-          if (j >= 2 && !mbar_wait_bounded(bar(B_KEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) break;
-          const uint32_t dK = sK + st * TILE_BYTES, dV = sV + st * TILE_BYTES;
-          mbar_expect_tx(bar(B_KFULL + st), bytes);
-          tma_load_3d(dK, mk, 0, y, bg, bar(B_KFULL + st));
-          tma_load_3d(dK + HALF_BYTES, mk, 64, y, bg, bar(B_KFULL + st));
-          if (j >= 2 && !mbar_wait_bounded(bar(B_VEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) {
+          if (!mbar_wait_bounded(bar(B_KEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) break;
+          load_kv(j, true);
+          if (!mbar_wait_bounded(bar(B_VEMPTY + st), ((j >> 1) - 1) & 1, &s_abort, WAIT_CYCLES)) {
             issued = j + 1;  // the K copy of this block is in flight
             break;
           }
-          mbar_expect_tx(bar(B_VFULL + st), bytes);
-          tma_load_3d(dV, mv, 0, y, bg, bar(B_VFULL + st));
-          tma_load_3d(dV + HALF_BYTES, mv, 64, y, bg, bar(B_VFULL + st));
+          load_kv(j, false);
           issued = j + 1;
         }
         if (s_abort) {  // let the copies already issued land before the CTA exits
@@ -276,6 +293,8 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         }
       }
       __syncwarp();
+    } else if (warp >= 2) {
+      zero_pad(64, 64);  // warps 2-3: the padding output rows, while the pipeline runs
     } else if (warp == 1) {
       // ---------------- MMA issuer (+ ragged V rows zeroed by the warp) -------
       constexpr uint32_t IDESC_QK = idesc_bf16_f32(BM, BN, 0);
