@@ -647,6 +647,98 @@ int orc_synth_argmax(const uint32_t* tok, const int32_t* parent, const int32_t* 
   return 0;
 }
 
+// ---------------------------------------------------------------------------
+// O11. CACHE search (Section IV-B: the CACHE stores token sequences, each a
+// verified retrieval "context + accepted draft" or a piece of the model's
+// output; Section IV-C, Algorithm 1: search(CACHE) retrieves from it the same
+// way the datastore is searched).
+//
+// Query b owns the entries e in [qent[b], qent[b+1]); entry e is the token
+// sequence tok[eoff[e] .. eoff[e+1]).  The search is O2-O4 with the entries
+// as the corpus, under the reading that a stored sequence is a unit of its
+// own: a match lies inside one entry, and a continuation stops at the end of
+// its entry.  So for a context c of length m and cap = min(n_max, m):
+//   * n* is the largest n in [n_min, cap] for which some entry E of length L
+//     has E[p-n .. p) = c[m-n .. m) with n <= p <= L-1 (one continuation
+//     token or more);
+//   * the occurrences are all such (e, p) for n*; with more than max_occ of
+//     them, the max_occ whose windows E[p-n* .. min(p+d, L)) are
+//     lexicographically smallest are kept (max_occ = 0 keeps all);
+//   * continuations u = E[p .. min(p+d, L)) are counted as distinct
+//     sequences and ranked by count descending, then token ids ascending.
+// Method: for every entry and position, the common suffix length by direct
+// comparison; then the occurrences of n*; then std::map counting.  Outputs as
+// orc_retrieve.
+// ---------------------------------------------------------------------------
+int orc_cache_search(const uint32_t* tok, const int64_t* eoff, const int64_t* qent, const uint32_t* ctx,
+                     int ctx_stride, const int32_t* ctx_len, int B, int n_max, int n_min, int top_k, int d,
+                     uint32_t max_occ, uint32_t* drafts, int32_t* draft_len, uint32_t* count,
+                     int32_t* n_drafts, int32_t* match_len, int nthreads) {
+  if (n_min < 1 || n_max < n_min || top_k < 1 || d < 1) return 1;
+  parallel_for(B, nthreads, [&](int64_t b) {
+    const uint32_t* c = ctx + (size_t)b * ctx_stride;
+    const int m = ctx_len[b];
+    uint32_t* dr = drafts + (size_t)b * top_k * d;
+    int32_t* dl = draft_len + (size_t)b * top_k;
+    uint32_t* ct = count + (size_t)b * top_k;
+    for (int i = 0; i < top_k * d; ++i) dr[i] = kPad;
+    for (int i = 0; i < top_k; ++i) { dl[i] = 0; ct[i] = 0; }
+    n_drafts[b] = 0;
+    match_len[b] = 0;
+    const int cap = std::min(n_max, m);
+    if (cap < n_min) return;
+    // common suffix length of E[0..p) and c, at most cap
+    auto common = [&](const uint32_t* E, int64_t p) {
+      int k = 0;
+      while (k < cap && k < p && E[p - 1 - k] == c[m - 1 - k]) ++k;
+      return k;
+    };
+    int best = 0;
+    for (int64_t e = qent[b]; e < qent[b + 1]; ++e) {
+      const uint32_t* E = tok + eoff[e];
+      const int64_t L = eoff[e + 1] - eoff[e];
+      for (int64_t p = 1; p <= L - 1; ++p) best = std::max(best, common(E, p));
+    }
+    if (best < n_min) return;
+    const int ns = best;
+    struct Occ {
+      std::vector<uint32_t> window, cont;
+    };
+    std::vector<Occ> occ;
+    for (int64_t e = qent[b]; e < qent[b + 1]; ++e) {
+      const uint32_t* E = tok + eoff[e];
+      const int64_t L = eoff[e + 1] - eoff[e];
+      for (int64_t p = ns; p <= L - 1; ++p) {
+        if (common(E, p) < ns) continue;
+        const int64_t end = std::min<int64_t>(p + d, L);
+        occ.push_back({std::vector<uint32_t>(E + p - ns, E + end), std::vector<uint32_t>(E + p, E + end)});
+      }
+    }
+    if (max_occ > 0 && occ.size() > max_occ) {
+      std::stable_sort(occ.begin(), occ.end(), [](const Occ& x, const Occ& y) { return x.window < y.window; });
+      occ.resize(max_occ);
+    }
+    std::map<std::vector<uint32_t>, uint32_t> freq;
+    for (const Occ& o : occ) freq[o.cont] += 1;
+    std::vector<std::pair<uint32_t, std::vector<uint32_t>>> ranked;
+    for (auto& kv : freq) ranked.push_back({kv.second, kv.first});
+    std::stable_sort(ranked.begin(), ranked.end(), [](const auto& x, const auto& y) {
+      if (x.first != y.first) return x.first > y.first;
+      return x.second < y.second;
+    });
+    const int nd = (int)std::min<size_t>(ranked.size(), (size_t)top_k);
+    for (int t = 0; t < nd; ++t) {
+      const auto& seq = ranked[t].second;
+      for (size_t i = 0; i < seq.size(); ++i) dr[(size_t)t * d + i] = seq[i];
+      dl[t] = (int32_t)seq.size();
+      ct[t] = ranked[t].first;
+    }
+    n_drafts[b] = nd;
+    match_len[b] = ns;
+  });
+  return 0;
+}
+
 int orc_hardware_threads(void) { return resolve_threads(0); }
 
 }  // extern "C"
