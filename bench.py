@@ -47,9 +47,9 @@ UNIT = "steps/s"
 #       python bench.py --steps 4 --warmup 3 --no-e2e --no-cpu-baseline
 # It is valid only for the kernel sources it was taken on (their SHA-256 below); once
 # those change, the bench reports traffic as null until it is measured again.
-ATTN_TRAFFIC = {"bytes_per_launch": 2.3702e9,
+ATTN_TRAFFIC = {"bytes_per_launch": 2.3679e9,
                 "sources": ["paper_2502_17139_gb300/csrc/tree_attn.cu", "paper_2502_17139_gb300/csrc/fc_common.cuh"],
-                "sha256": "e942b6e254896908ad1724b6de7a19bdbf1940173cfc767144ac2f6d595349fd"}
+                "sha256": "16c816b6bfa050af822e61dc01a220cdae361212071af71bc053544e664f68bb"}
 
 WORKLOAD = ("full step loop: two-source datastore 100M (Zipf 1.1) + 5M (Zipf 1.3, 20k planted repeats) tokens, "
             "vocab 32256, batch 32, ctx 128, n 16->2, top-64 x 10 tokens per source, tree <=128 nodes, "

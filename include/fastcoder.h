@@ -207,6 +207,106 @@ fc_status fc_rcache_insert(void* d_table, int capacity, int n_sources, fc_retrie
                            const int32_t* d_n_drafts, const int32_t* d_match_len, fc_stream s);
 
 /* ------------------------------------------------------------------------
+ * CACHE and missing table (Section IV-B; Section IV-C, Algorithm 1;
+ * Section V-C: l = 50, the model's output stored in pieces of 20 tokens).
+ *
+ * Every sequence b of a batch owns a CACHE: a store of token sequences, each
+ * either a verified retrieval (the last ctx_keep context tokens before a step
+ * followed by the draft tokens that step accepted) or a complete piece of
+ * `chunk` tokens of the model's output (the tokens appended to the context
+ * after the prompt).  Once it holds min_size sequences or more, a CACHE is
+ * searched before the datastore, with fc_retrieve's definition applied to
+ * the stored sequences: a match lies inside one stored sequence and a
+ * continuation stops at the end of its sequence.
+ *
+ * The missing table M (one per batch) holds the n_min-token context
+ * suffixes for which every datastore source returned nothing.  A match of
+ * length n implies matches of all shorter lengths at the same position, so
+ * for a static datastore this key decides exactly whether retrieval can
+ * return anything.  A context that ends with a key in M skips the datastore.
+ *
+ * Per step: fc_cache_search -> fc_retrieve (d_skip = the state array) ->
+ * fc_missing_insert -> tree, verification, acceptance, fc_kv_append ->
+ * fc_cache_update.
+ *
+ * CACHE layout (caller-owned device memory):
+ *   d_words [batch][capacity] uint32: the stored sequences back to back,
+ *           each followed by FC_SEP_TOKEN (a sequence of L tokens costs L+1
+ *           words; one that does not fit is dropped and counted);
+ *   d_meta  [batch][4] int32: words used, sequences stored, output mark (the
+ *           context length where the next output piece starts), sequences
+ *           dropped for lack of room.
+ * M layout: uint32 words [0] keys stored, [1] keys dropped, [2..3] zero, then
+ * `capacity` slots of 1 + key_len words (a nonzero tag, then the key).  M
+ * holds at most capacity / 2 keys.
+ * ------------------------------------------------------------------------ */
+#define FC_SEP_TOKEN 0xFFFFFFFEu
+#define FC_CACHE_MAX_WORDS 16384
+#define FC_SERVE_DATASTORE 0 /* search the datastore sources */
+#define FC_SERVE_CACHE 1     /* the CACHE returned drafts */
+#define FC_SKIP_MISSING 2    /* the context's key is in M: no retrieval */
+
+typedef struct {
+  uint32_t* d_words;  /* [batch][capacity] */
+  int32_t* d_meta;    /* [batch][4] */
+  int32_t capacity;   /* words per sequence: a multiple of 4 in 16..FC_CACHE_MAX_WORDS */
+  int32_t min_size;   /* l: stored sequences needed before a search, >= 0 */
+  int32_t chunk;      /* output piece length, >= 1 */
+  int32_t ctx_keep;   /* context tokens stored before a verified draft, 0..FC_MAX_NMAX */
+} fc_cache;
+
+/* Empties every CACHE; the output mark starts at d_prompt_len[b]. */
+fc_status fc_cache_init(const fc_cache* cache, int batch, const int32_t* d_prompt_len, fc_stream s);
+
+/* Bytes of a missing table with `capacity` slots (a power of two, 2..2^24)
+ * and keys of key_len tokens (1..FC_MAX_NMAX); 0 for bad arguments. */
+size_t fc_missing_bytes(int capacity, int key_len);
+
+/* Empties a missing table. */
+fc_status fc_missing_init(void* d_table, size_t bytes, int capacity, int key_len, fc_stream s);
+
+/*
+ * Algorithm 1 up to the datastore search.  The result arrays have the
+ * fc_retrieve layout with n_sources + 1 slots ([n_sources + 1][batch]...):
+ * slot n_sources receives the CACHE's result (empty while the CACHE holds
+ * fewer than min_size sequences), and for every query not sent to the
+ * datastore, slots 0..n_sources-1 are cleared.  d_state[b] gets
+ * FC_SERVE_CACHE when the CACHE returned drafts, else FC_SKIP_MISSING when
+ * the context's last p.n_min tokens are in M, else FC_SERVE_DATASTORE; pass
+ * it to fc_retrieve as d_skip.  d_missing may be NULL (no table); its keys
+ * are p.n_min tokens long.  Limits as fc_retrieve.
+ */
+fc_status fc_cache_search(const fc_cache* cache, const void* d_missing, int missing_capacity,
+                          const uint32_t* d_ctx, int ctx_stride, const int32_t* d_ctx_len, int batch,
+                          fc_retrieve_params p, int n_sources, uint32_t* d_drafts, int32_t* d_draft_len,
+                          uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len, int32_t* d_state,
+                          fc_stream s);
+
+/*
+ * Adds to M the key (last key_len context tokens) of every query with
+ * d_state[b] == FC_SERVE_DATASTORE, ctx_len[b] >= key_len and no draft in
+ * any of the n_sources datastore slots of d_n_drafts ([>= n_sources][batch],
+ * fc_retrieve's output).  Keys new to M are admitted in query order while M
+ * holds fewer than capacity / 2 keys; the others are counted as dropped.
+ */
+fc_status fc_missing_insert(void* d_missing, int missing_capacity, int key_len, const uint32_t* d_ctx,
+                            int ctx_stride, const int32_t* d_ctx_len, int batch, const int32_t* d_state,
+                            const int32_t* d_n_drafts, int n_sources, fc_stream s);
+
+/*
+ * The CACHE update after verification.  For a query whose context grew by
+ * acc_len + 1 tokens this step (d_ctx_len_new = d_ctx_len_old + acc_len + 1)
+ * and acc_len >= 1, stores ctx[old - min(ctx_keep, old) .. old + acc_len)
+ * (the verified retrieval: context suffix, then the accepted draft tokens).
+ * Then, while d_ctx_len_new - mark >= chunk, stores ctx[mark .. mark + chunk)
+ * and advances the mark.  A token >= FC_SEP_TOKEN in a sequence to store
+ * records FC_ERR_INVALID_ARG and that sequence is skipped.
+ */
+fc_status fc_cache_update(const fc_cache* cache, const uint32_t* d_ctx, int ctx_stride,
+                          const int32_t* d_ctx_len_old, const int32_t* d_ctx_len_new, const int32_t* d_acc_len,
+                          int batch, fc_stream s);
+
+/* ------------------------------------------------------------------------
  * Draft tree (Section IV-D: Eq. 3 node weight alpha*t_r + beta*t_c, the
  * top-weighted trie nodes as the draft; Eq. 4 tree mask; position ids by
  * depth; Section V-C: alpha = beta = 1, at most 64 draft tokens).

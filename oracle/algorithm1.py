@@ -164,20 +164,26 @@ def retrieve_step(state: State, corpora, ctx, ctx_len, p, nthreads: int = 0):
             r = O.retrieve(T, ctx[todo], ctx_len[todo], p["n_max"], p["n_min"], k, d, p["max_occ"], nthreads)
             for name in RESULT_FIELDS:
                 res[s][name][todo] = r[name]
-    # step 3: M grows by the keys whose datastore search found nothing
+    missing_update(state, ctx, ctx_len, code, np.stack([r["n_drafts"] for r in res]) if res else np.zeros((0, B)))
+    return res + [rc], code
+
+
+def missing_update(state: State, ctx, ctx_len, code, n_drafts):
+    """Step 3: M grows by the keys of the queries whose datastore search
+    (code SERVE_DATASTORE) found nothing in any source (n_drafts [S, B]),
+    in query order (reading R1), while M has room (R7)."""
     seen = set()
-    for b in todo:
-        if keys[b] is None or any(res[s]["n_drafts"][b] > 0 for s in range(len(corpora))):
+    for b in range(len(code)):
+        if code[b] != SERVE_DATASTORE or any(n_drafts[s][b] > 0 for s in range(len(n_drafts))):
             continue
-        key = keys[b]
-        if key in state.missing or key in seen:
+        key = state.key(ctx[b], int(ctx_len[b]))
+        if key is None or key in state.missing or key in seen:
             continue
         seen.add(key)
         if len(state.missing) < state.missing_max:
             state.missing.add(key)
         else:
             state.missing_dropped += 1
-    return res + [rc], code
 
 
 def cache_update(state: State, ctx, old_len, new_len, acc_len):

@@ -38,6 +38,13 @@ static inline fc_status fc_cuda_status(cudaError_t e) { return e == cudaSuccess 
 
 #define FC_CHECK_LAUNCH() fc_cuda_status(cudaGetLastError())
 
+// Host: the limits every retrieval-shaped call accepts.
+static inline bool fc_retrieve_params_ok(const fc_retrieve_params& p) {
+  return p.n_max >= 1 && p.n_max <= FC_MAX_NMAX && p.n_min >= 1 && p.n_min <= p.n_max && p.top_k >= 1 &&
+         p.top_k <= FC_MAX_TOPK && p.draft_len >= 1 && p.draft_len <= FC_MAX_DRAFT_LEN && p.max_occ >= 1 &&
+         p.max_occ <= FC_MAX_OCC;
+}
+
 // ---------------------------------------------------------------------------
 // Small PTX wrappers (sm_100 family).  Shared-memory addresses are 32-bit
 // CTA-window addresses.

@@ -28,13 +28,13 @@
 #include <algorithm>
 
 #include "fc_common.cuh"
+#include "fc_topk.cuh"
 
 FC_DEFINE_ERROR_WORD(ret)
 
 namespace {
 
 constexpr int RT_THREADS = 512;
-constexpr int RT_ITEMS = FC_MAX_OCC / RT_THREADS;  // 8
 constexpr int CMP_GROUPS = FC_MAX_NMAX / 4 + 1;    // 16-byte groups covering a pattern at any alignment
 
 struct DsView {
@@ -99,31 +99,6 @@ __device__ __forceinline__ int cmp_suffix_vec(const uint32_t* __restrict__ T, ui
   return res;
 }
 
-__device__ __forceinline__ uint32_t block_scan_256(uint32_t x, uint32_t* total, uint32_t* wsum) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t inc = x;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    uint32_t y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
-    if (lane >= o) inc += y;
-  }
-  if (lane == 31) wsum[warp] = inc;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    uint32_t run = 0;
-    for (int w = 0; w < RT_THREADS / 32; ++w) {
-      uint32_t c = wsum[w];
-      wsum[w] = run;
-      run += c;
-    }
-    *total = run;
-  }
-  __syncthreads();
-  uint32_t r = wsum[warp] + inc - x;
-  __syncthreads();
-  return r;
-}
-
 struct RetSmem {
   uint32_t runs[FC_MAX_OCC + 1];   // run starts (occurrence index), runs[R] = nocc
   uint32_t work[FC_MAX_OCC];       // head flags, then the count histogram
@@ -134,7 +109,8 @@ struct RetSmem {
   uint32_t hi[FC_MAX_NMAX + 1];
   uint32_t endhit[FC_MAX_NMAX + 1];
   uint32_t wsum[RT_THREADS / 32];
-  uint32_t n_star, first, cnt, n_runs, bad, cstar, n_greater, n_sel;
+  RunsScratch rs;
+  uint32_t n_star, first, cnt, bad;
 };
 
 __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint32_t* __restrict__ ctx, int stride,
@@ -251,102 +227,10 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint
   for (uint32_t e = tid; e < nocc; e += RT_THREADS)
     sm.work[e] = (e == 0 || (uint32_t)__ldg(ds.lcp + first + e) < need) ? 1u : 0u;
   __syncthreads();
-  uint32_t head[RT_ITEMS];
-  uint32_t local = 0;
-#pragma unroll
-  for (int it = 0; it < RT_ITEMS; ++it) {
-    uint32_t e = tid * RT_ITEMS + it;
-    head[it] = (e < nocc) ? sm.work[e] : 0u;
-    local += head[it];
-  }
-  uint32_t total;
-  uint32_t run_id = block_scan_256(local, &total, sm.wsum);
-#pragma unroll
-  for (int it = 0; it < RT_ITEMS; ++it) {
-    uint32_t e = tid * RT_ITEMS + it;
-    if (head[it]) sm.runs[run_id] = e;
-    run_id += head[it];
-  }
-  if (tid == 0) {
-    sm.runs[total] = nocc;
-    sm.n_runs = total;
-  }
-  __syncthreads();
-  const uint32_t R = sm.n_runs;
+  const uint32_t nd_sel = rank_runs<RT_THREADS>(nocc, k, sm.runs, sm.work, sm.sel, sm.order, sm.wsum, sm.rs);
   auto run_count = [&](uint32_t r) { return sm.runs[r + 1] - sm.runs[r]; };
-
-  // ---- top-k runs --------------------------------------------------------
-  if (R <= (uint32_t)k) {
-    for (uint32_t r = tid; r < R; r += RT_THREADS) sm.sel[r] = r;
-    if (tid == 0) sm.n_sel = R;
-  } else {
-    // histogram of counts (1..FC_MAX_OCC), bin q = FC_MAX_OCC - count so that
-    // a prefix over q counts the runs with a larger count
-    for (uint32_t q = tid; q < FC_MAX_OCC; q += RT_THREADS) sm.work[q] = 0;
-    __syncthreads();
-    for (uint32_t r = tid; r < R; r += RT_THREADS) atomicAdd(&sm.work[FC_MAX_OCC - run_count(r)], 1u);
-    __syncthreads();
-    uint32_t hq[RT_ITEMS];
-    uint32_t hsum = 0;
-#pragma unroll
-    for (int it = 0; it < RT_ITEMS; ++it) {
-      hq[it] = sm.work[tid * RT_ITEMS + it];
-      hsum += hq[it];
-    }
-    uint32_t tot2;
-    uint32_t above = block_scan_256(hsum, &tot2, sm.wsum);  // runs with a larger count than this chunk's bins
-#pragma unroll
-    for (int it = 0; it < RT_ITEMS; ++it) {
-      if (above < (uint32_t)k && above + hq[it] >= (uint32_t)k) {  // the k-th largest count lives here
-        sm.cstar = FC_MAX_OCC - (tid * RT_ITEMS + it);
-        sm.n_greater = above;
-      }
-      above += hq[it];
-    }
-    __syncthreads();
-    const uint32_t cstar = sm.cstar, room = (uint32_t)k - sm.n_greater;
-    // keep: count > c*, or count == c* among the first `room` such runs in token order
-    uint32_t fl[RT_ITEMS], eq_local = 0;
-#pragma unroll
-    for (int it = 0; it < RT_ITEMS; ++it) {
-      uint32_t r = tid * RT_ITEMS + it;
-      fl[it] = (r < R) ? (run_count(r) > cstar ? 2u : (run_count(r) == cstar ? 1u : 0u)) : 0u;
-      eq_local += (fl[it] == 1u);
-    }
-    uint32_t tot3;
-    uint32_t eq_before = block_scan_256(eq_local, &tot3, sm.wsum);
-    uint32_t keep_local = 0;
-#pragma unroll
-    for (int it = 0; it < RT_ITEMS; ++it) {
-      if (fl[it] == 1u) {
-        fl[it] = (eq_before < room) ? 2u : 0u;
-        ++eq_before;
-      }
-      keep_local += (fl[it] == 2u);
-    }
-    uint32_t tot4;
-    uint32_t kept_before = block_scan_256(keep_local, &tot4, sm.wsum);
-#pragma unroll
-    for (int it = 0; it < RT_ITEMS; ++it) {
-      if (fl[it] == 2u) sm.sel[kept_before++] = tid * RT_ITEMS + it;
-    }
-    if (tid == 0) sm.n_sel = tot4;
-  }
-  __syncthreads();
-  const uint32_t ks = sm.n_sel;  // == min(k, R)
-  // rank the kept runs by (count descending, run ascending)
-  for (uint32_t t = tid; t < ks; t += RT_THREADS) {
-    const uint32_t r = sm.sel[t], c = run_count(r);
-    uint32_t rank = 0;
-    for (uint32_t u = 0; u < ks; ++u) {
-      const uint32_t ru = sm.sel[u], cu = run_count(ru);
-      rank += (cu > c || (cu == c && ru < r)) ? 1u : 0u;
-    }
-    sm.order[rank] = r;
-  }
-  __syncthreads();
   // ---- outputs ---------------------------------------------------------
-  const int nd = (int)ks;
+  const int nd = (int)nd_sel;
   for (int e = tid; e < k * d; e += RT_THREADS) {
     int t = e / d, x = e - t * d;
     uint32_t v = FC_PAD_TOKEN;
@@ -374,11 +258,7 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint
   }
 }
 
-bool params_ok(const fc_retrieve_params& p) {
-  return p.n_max >= 1 && p.n_max <= FC_MAX_NMAX && p.n_min >= 1 && p.n_min <= p.n_max && p.top_k >= 1 &&
-         p.top_k <= FC_MAX_TOPK && p.draft_len >= 1 && p.draft_len <= FC_MAX_DRAFT_LEN && p.max_occ >= 1 &&
-         p.max_occ <= FC_MAX_OCC;
-}
+bool params_ok(const fc_retrieve_params& p) { return fc_retrieve_params_ok(p); }
 
 // ---------------------------------------------------------------------------
 // Replay cache.  Entry layout (32-bit words): [0] key length or EMPTY /

@@ -44,10 +44,16 @@ class fc_retrieve_params(C.Structure):
                 ("draft_len", C.c_int32), ("max_occ", C.c_uint32)]
 
 
+class fc_cache(C.Structure):
+    _fields_ = [("d_words", C.c_void_p), ("d_meta", C.c_void_p), ("capacity", C.c_int32), ("min_size", C.c_int32),
+                ("chunk", C.c_int32), ("ctx_keep", C.c_int32)]
+
+
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
            "fc_datastore_build_noalloc",
            "fc_retrieve", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
-           "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
+           "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
+           "fc_missing_insert", "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
 
 
 def _load():
@@ -71,6 +77,13 @@ def _load():
                                        vp, vp, vp, vp, vp, vp]),
         "fc_rcache_insert": (C.c_int, [vp, i32, i32, fc_retrieve_params, vp, i32, vp, i32, vp,
                                        vp, vp, vp, vp, vp, vp]),
+        "fc_cache_init": (C.c_int, [C.POINTER(fc_cache), i32, vp, vp]),
+        "fc_cache_search": (C.c_int, [C.POINTER(fc_cache), vp, i32, vp, i32, vp, i32, fc_retrieve_params, i32,
+                                      vp, vp, vp, vp, vp, vp, vp]),
+        "fc_cache_update": (C.c_int, [C.POINTER(fc_cache), vp, i32, vp, vp, vp, i32, vp]),
+        "fc_missing_bytes": (sz, [i32, i32]),
+        "fc_missing_init": (C.c_int, [vp, sz, i32, i32, vp]),
+        "fc_missing_insert": (C.c_int, [vp, i32, i32, vp, i32, vp, i32, vp, vp, i32, vp]),
         "fc_build_tree": (C.c_int, [i32, vp, vp, vp, vp, C.POINTER(C.c_uint32), i32, i32, vp, vp, i32, i32, i32,
                                     vp, vp, vp, vp, vp, vp, vp]),
         "fc_tree_mask": (C.c_int, [vp, vp, vp, i32, i32, vp, vp, vp, vp]),
@@ -249,6 +262,77 @@ def fc_rcache_insert(cache: RetrievalCache, ctx, ctx_len, skip, res):
         _ptr(cache.table), cache.capacity, cache.n_sources, cache.p, _ptr(ctx), stride, _ptr(ctx_len), B,
         _ptr(skip), _ptr(res["drafts"]), _ptr(res["draft_len"]), _ptr(res["count"]), _ptr(res["n_drafts"]),
         _ptr(res["match_len"]), _stream()))
+
+
+# ------------------------------------------------- CACHE and missing table
+SERVE_DATASTORE, SERVE_CACHE, SKIP_MISSING = 0, 1, 2
+SEP_I32 = -2  # FC_SEP_TOKEN seen through an int32 tensor
+
+
+class SequenceCache:
+    """The CACHE of Section IV-B for a batch: per sequence, a store of
+    verified retrievals and output pieces (words [B, capacity] int32, meta
+    [B, 4] int32: words used, sequences stored, output mark, dropped)."""
+
+    def __init__(self, batch, capacity=8192, min_size=50, chunk=20, ctx_keep=16, device="cuda"):
+        self.batch = batch
+        self.words = torch.zeros((batch, capacity), dtype=torch.int32, device=device)
+        self.meta = torch.zeros((batch, 4), dtype=torch.int32, device=device)
+        self.view = fc_cache(self.words.data_ptr(), self.meta.data_ptr(), capacity, min_size, chunk, ctx_keep)
+
+    def init(self, prompt_len):
+        _need(prompt_len, torch.int32, "prompt_len", (self.batch,))
+        _check("fc_cache_init", LIB.fc_cache_init(C.byref(self.view), self.batch, _ptr(prompt_len), _stream()))
+
+
+class MissingTable:
+    """The missing table M of Algorithm 1 (keys of key_len tokens)."""
+
+    def __init__(self, capacity, key_len, device="cuda"):
+        self.capacity, self.key_len = capacity, key_len
+        nbytes = int(LIB.fc_missing_bytes(capacity, key_len))
+        if nbytes == 0:
+            raise ValueError("bad missing-table parameters")
+        self.table = torch.empty(nbytes // 4, dtype=torch.int32, device=device)
+        self.clear()
+
+    def clear(self):
+        _check("fc_missing_init", LIB.fc_missing_init(_ptr(self.table), self.table.numel() * 4, self.capacity,
+                                                      self.key_len, _stream()))
+
+
+def fc_cache_search(cache: SequenceCache, missing, ctx, ctx_len, p: fc_retrieve_params, n_sources, out, state):
+    """out: retrieve_outputs(n_sources + 1, B, p); slot n_sources gets the
+    CACHE's result.  state: int32 [B]."""
+    _need(ctx, torch.int32, "ctx")
+    B, stride = ctx.shape
+    _need(ctx_len, torch.int32, "ctx_len", (B,))
+    _need(state, torch.int32, "state", (B,))
+    if out["n_drafts"].shape != (n_sources + 1, B):
+        raise ValueError("out must hold n_sources + 1 result slots")
+    tab = None if missing is None else missing.table
+    cap = 0 if missing is None else missing.capacity
+    _check("fc_cache_search", LIB.fc_cache_search(
+        C.byref(cache.view), _ptr(tab), cap, _ptr(ctx), stride, _ptr(ctx_len), B, p, n_sources,
+        _ptr(out["drafts"]), _ptr(out["draft_len"]), _ptr(out["count"]), _ptr(out["n_drafts"]),
+        _ptr(out["match_len"]), _ptr(state), _stream()))
+
+
+def fc_missing_insert(missing: MissingTable, ctx, ctx_len, state, n_drafts, n_sources):
+    """n_drafts: the [>= n_sources, B] retrieval counts (datastore slots first)."""
+    B, stride = ctx.shape
+    _need(n_drafts, torch.int32, "n_drafts")
+    _check("fc_missing_insert", LIB.fc_missing_insert(
+        _ptr(missing.table), missing.capacity, missing.key_len, _ptr(ctx), stride, _ptr(ctx_len), B, _ptr(state),
+        _ptr(n_drafts), n_sources, _stream()))
+
+
+def fc_cache_update(cache: SequenceCache, ctx, ctx_len_old, ctx_len_new, acc_len):
+    B, stride = ctx.shape
+    for t, nm in ((ctx_len_old, "ctx_len_old"), (ctx_len_new, "ctx_len_new"), (acc_len, "acc_len")):
+        _need(t, torch.int32, nm, (B,))
+    _check("fc_cache_update", LIB.fc_cache_update(C.byref(cache.view), _ptr(ctx), stride, _ptr(ctx_len_old),
+                                                  _ptr(ctx_len_new), _ptr(acc_len), B, _stream()))
 
 
 # -------------------------------------------------------------------- tree

@@ -1,10 +1,19 @@
 """One retrieve-and-verify decoding step, composed from the C-ABI calls.
 
 A step (Section IV-C Algorithm 1 and Section IV-D) for a batch of sequences:
-  cache lookup -> fc_retrieve on every source (queries the cache served are
-  skipped) -> cache insert -> fc_build_tree -> fc_tree_attn ->
-  target-model predictions (the synthetic stand-in) -> fc_accept ->
-  fc_kv_append (cache rows, context, lengths and next root).
+  retrieval -> fc_build_tree -> fc_tree_attn -> target-model predictions (the
+  synthetic stand-in) -> fc_accept -> fc_kv_append (cache rows, context,
+  lengths and next root).
+
+Retrieval takes one of two forms:
+  * with ``seq_cache`` (Algorithm 1 with the CACHE of Section IV-B and the
+    missing table): fc_cache_search -> fc_retrieve on the datastore sources
+    for the queries the CACHE did not serve and M did not skip ->
+    fc_missing_insert; after the append, fc_cache_update stores the verified
+    retrieval and the completed output pieces.  The tree merges S + 1 result
+    slots, the CACHE's last.
+  * otherwise the context-keyed replay cache: lookup -> fc_retrieve on the
+    queries it did not serve -> insert.
 
 Every call is asynchronous on the current stream and allocates nothing, so a
 step can be captured once into a CUDA graph and replayed (lengths ping-pong
@@ -20,7 +29,10 @@ from . import fastcoder as fc
 
 class StepLoop:
     def __init__(self, sources, ctx, ctx_len, p, node_budget, n_pad, src_weight, H, Hkv, D, kv_cap, kv_len0, vocab,
-                 cache_capacity=1 << 14, device="cuda", k_cache=None, v_cache=None):
+                 cache_capacity=1 << 14, device="cuda", k_cache=None, v_cache=None, seq_cache=None):
+        """seq_cache: None, or a dict with capacity, min_size, chunk, ctx_keep
+        (the CACHE), missing_capacity (M) and weight (the CACHE slot's tree
+        weight); it replaces the replay cache."""
         self.sources, self.p, self.node_budget, self.n_pad = sources, p, node_budget, n_pad
         self.src_weight = list(src_weight)
         self.H, self.Hkv, self.D, self.kv_cap, self.vocab = H, Hkv, D, kv_cap, vocab
@@ -37,7 +49,9 @@ class StepLoop:
         self.cur = 0
         self._init = (self.ctx.clone(), self.ctx_len[0].clone(), self.kv_len[0].clone(), self.root.clone())
         S = len(sources)
-        self.res = fc.retrieve_outputs(S, B, p, device)
+        self.seq = dict(seq_cache) if seq_cache else None
+        n_slots = S + 1 if self.seq else S
+        self.res = fc.retrieve_outputs(n_slots, B, p, device)
         self.skip = torch.zeros(B, dtype=torch.int32, device=device)
         self.tree = fc.tree_outputs(B, n_pad, device)
         self.argmax = torch.empty((B, n_pad), dtype=torch.int32, device=device)
@@ -49,7 +63,16 @@ class StepLoop:
         self.k_cache = k_cache if k_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         self.v_cache = v_cache if v_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         self.attn_out = torch.empty((B, n_pad, H, D), dtype=torch.bfloat16, device=device)
-        self.cache = fc.RetrievalCache(cache_capacity, S, p, device) if cache_capacity else None
+        self.cache = fc.RetrievalCache(cache_capacity, S, p, device) if cache_capacity and not self.seq else None
+        if self.seq:
+            q = self.seq
+            self.seq_cache = fc.SequenceCache(B, q.get("capacity", 8192), q.get("min_size", 50), q.get("chunk", 20),
+                                              q.get("ctx_keep", p.n_max), device)
+            self.missing = fc.MissingTable(q.get("missing_capacity", 1 << 16), p.n_min, device)
+            self.tree_weight = self.src_weight + [int(q.get("weight", 1))]
+            self.seq_cache.init(self.ctx_len[0])
+        else:
+            self.tree_weight = self.src_weight
 
     def step(self, q, k_tree, v_tree, want_hit, plen, rtok, attention=True, events=None):
         """Enqueue one step.  q [B, Np, H, D], k_tree/v_tree [B, Hkv, Np, D]
@@ -60,7 +83,12 @@ class StepLoop:
         ev = events or {}
         if "retrieve" in ev:
             ev["retrieve"][0].record()
-        if self.cache is not None:
+        S = len(self.sources)
+        if self.seq:
+            fc.fc_cache_search(self.seq_cache, self.missing, self.ctx, self.ctx_len[c], self.p, S, self.res, self.skip)
+            fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, skip=self.skip, out=self.res)
+            fc.fc_missing_insert(self.missing, self.ctx, self.ctx_len[c], self.skip, self.res["n_drafts"], S)
+        elif self.cache is not None:
             fc.fc_rcache_lookup(self.cache, self.ctx, self.ctx_len[c], want_hit, self.skip, self.res)
             fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, skip=self.skip, out=self.res)
             fc.fc_rcache_insert(self.cache, self.ctx, self.ctx_len[c], self.skip, self.res)
@@ -70,7 +98,7 @@ class StepLoop:
             ev["retrieve"][1].record()
         if "tree" in ev:
             ev["tree"][0].record()
-        fc.fc_build_tree(self.res, self.src_weight, self.root, self.kv_len[c], self.node_budget, self.n_pad,
+        fc.fc_build_tree(self.res, self.tree_weight, self.root, self.kv_len[c], self.node_budget, self.n_pad,
                          out=self.tree)
         if "tree" in ev:
             ev["tree"][1].record()
@@ -89,19 +117,26 @@ class StepLoop:
                      out=self.acc)
         fc.fc_kv_append(self.acc, self.tree["tok"], k_tree, v_tree, self.k_cache, self.v_cache, self.kv_len[c],
                         self.kv_len[n], self.ctx, self.ctx_len[c], self.ctx_len[n], self.root)
+        if self.seq:
+            fc.fc_cache_update(self.seq_cache, self.ctx, self.ctx_len[c], self.ctx_len[n], self.acc["acc_len"])
         if "tail" in ev:
             ev["tail"][1].record()
         self.cur = n
 
     def reset(self):
-        """Back to the initial contexts and cache lengths; the retrieval cache
-        keeps its entries (a replay of the same trajectory then hits it)."""
+        """Back to the initial contexts and cache lengths.  The replay cache
+        keeps its entries (a replay of the same trajectory then hits it); the
+        CACHE and the missing table start empty again, as for a new
+        generation."""
         ctx0, cl0, kv0, root0 = self._init
         self.ctx.copy_(ctx0)
         self.ctx_len[0].copy_(cl0)
         self.kv_len[0].copy_(kv0)
         self.root.copy_(root0)
         self.cur = 0
+        if self.seq:
+            self.seq_cache.init(self.ctx_len[0])
+            self.missing.clear()
 
     @property
     def kv_len_now(self):

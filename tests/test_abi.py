@@ -89,3 +89,35 @@ def test_host_validation_without_gpu(lib):
     assert L.fc_argmax_accept(17, 100, 16, 16, 16, 2, 64, 16, 16, 16, 12, 16, nul) == 1
     # cache: capacity must be a power of two
     assert L.fc_rcache_init(1, 1 << 30, 1000, 2, p, nul) == 1
+
+
+def test_cache_host_validation_without_gpu(lib):
+    import paper_2502_17139_gb300.fastcoder as fc
+    L = fc.LIB
+    p = fc.params(16, 2, 16, 8)
+    nul = None
+    good = fc.fc_cache(256, 256, 8192, 50, 20, 16)
+    bad_cap = fc.fc_cache(256, 256, 8190, 50, 20, 16)      # not a multiple of 4
+    big_cap = fc.fc_cache(256, 256, 32768, 50, 20, 16)     # beyond FC_CACHE_MAX_WORDS
+    odd_words = fc.fc_cache(260, 256, 8192, 50, 20, 16)    # words not 16-byte aligned
+    bad_keep = fc.fc_cache(256, 256, 8192, 50, 20, 40)     # ctx_keep > FC_MAX_NMAX
+    zero_chunk = fc.fc_cache(256, 256, 8192, 50, 0, 16)
+    outs = [16] * 5
+    for c in (bad_cap, big_cap, odd_words, bad_keep, zero_chunk):
+        assert L.fc_cache_search(C.byref(c), nul, 0, 16, 64, 16, 4, p, 2, *outs, 16, nul) == 1
+        assert L.fc_cache_update(C.byref(c), 16, 64, 16, 16, 16, 4, nul) == 1
+        assert L.fc_cache_init(C.byref(c), 4, 16, nul) == 1
+    # the CACHE slot must fit next to the datastore slots
+    assert L.fc_cache_search(C.byref(good), nul, 0, 16, 64, 16, 4, p, 4, *outs, 16, nul) == 1
+    # a missing table whose capacity is not a power of two
+    assert L.fc_cache_search(C.byref(good), 16, 1000, 16, 64, 16, 4, p, 2, *outs, 16, nul) == 1
+    # unsupported retrieval parameters, missing state array, empty batch
+    assert L.fc_cache_search(C.byref(good), nul, 0, 16, 64, 16, 4, fc.params(40, 2, 16, 8), 2, *outs, 16, nul) == 2
+    assert L.fc_cache_search(C.byref(good), nul, 0, 16, 64, 16, 4, p, 2, *outs, nul, nul) == 1
+    assert L.fc_cache_search(C.byref(good), nul, 0, nul, 64, nul, 0, p, 2, *([nul] * 5), nul, nul) == 0
+    # missing table sizes: header + capacity slots of 1 + key_len words
+    assert L.fc_missing_bytes(1024, 2) == 4 * (4 + 1024 * 3)
+    assert L.fc_missing_bytes(1000, 2) == 0 and L.fc_missing_bytes(1024, 0) == 0 and L.fc_missing_bytes(1024, 33) == 0
+    assert L.fc_missing_init(16, 4 * (4 + 1024 * 3) - 1, 1024, 2, nul) == 3
+    assert L.fc_missing_insert(16, 1024, 0, 16, 64, 16, 4, 16, 16, 2, nul) == 1
+    assert L.fc_missing_insert(nul, 1024, 2, 16, 64, 16, 4, 16, 16, 2, nul) == 1
