@@ -67,7 +67,8 @@ def parse_args(argv=None):
     ap.add_argument("--batch", type=int, default=32)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--mode", choices=["step", "attn", "argmax", "configs", "retrieve"], default="step",
+    ap.add_argument("--mode", choices=["step", "attn", "argmax", "configs", "retrieve", "algorithm1", "cache"],
+                    default="step",
                     help="step: the full step loop (the benchmark); attn: tree attention alone on the step loop's "
                          "attention shape with seeded trees (a small profiling / sweep target); argmax: greedy "
                          "verification from bf16 logits (fc_argmax_accept) on the step loop's tree shape; configs: "
@@ -75,6 +76,8 @@ def parse_args(argv=None):
                          "benchmark line); retrieve: two-source retrieval alone for --batch queries (batch sweeps)")
     ap.add_argument("--nodes", type=int, default=128, help="attn mode: tree nodes per sequence")
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
+    ap.add_argument("--fill", type=int, default=None,
+                    help="algorithm1 / cache modes: steps that fill the CACHE first (default 100 / 450)")
     ap.add_argument("--skip-1b", action="store_true", help="configs mode: leave out the 1B-token configuration")
     ap.add_argument("--traffic-bytes", type=float, default=None,
                     help="ncu dram read+write bytes of one tree-attention launch of this workload")
@@ -693,6 +696,25 @@ def run_argmax(args, rank, ws, local):
             "mean_acc_len": float(out["acc_len"].float().mean().item()), "clocks": clock_rec}
 
 
+def _gpu_ms(fn, reps=20, warm=3, spin_cycles=4_000_000):
+    """Mean device time of fn() over `reps` back-to-back calls, with the host
+    enqueueing ahead of the device (the stream first spins ~2 ms), so that a
+    kernel of a few microseconds is not timed together with the host's own
+    per-call overhead."""
+    import torch
+    for _ in range(warm):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda._sleep(spin_cycles)
+    e0.record()
+    for _ in range(reps):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps
+
+
 def _cuda_ms(fn, reps=10, warm=3):
     """Mean CUDA-event time of fn() on the current stream, after warm-up."""
     import torch
@@ -743,7 +765,7 @@ def run_configs(args, rank, ws, local):
         kt, vt = rnd(B, Hkv, n_pad, D), rnd(B, Hkv, n_pad, D)
         o = torch.empty_like(q)
         kv_d = to_dev(np.asarray(kvl, np.int32))
-        ms = _cuda_ms(lambda: fc.fc_tree_attn(q, kc, vc, kv_d, kt, vt, tree["mask"], tree["n_nodes"], out=o))
+        ms = _gpu_ms(lambda: fc.fc_tree_attn(q, kc, vc, kv_d, kt, vt, tree["mask"], tree["n_nodes"], out=o))
         F, By = _attn_work(fc, tree, kvl, H, Hkv, D)
         t_roof = max(F / tc, By / bw)
         return {"ms": ms, "tflops": F / (ms * 1e-3) / 1e12, "gbs": By / (ms * 1e-3) / 1e9,
@@ -755,7 +777,7 @@ def run_configs(args, rank, ws, local):
         plen, rtok = synth.argmax_draws(rng, B, n_pad, V, plen_max)
         am = fc.fc_synth_argmax(tree["tok"], tree["parent"], tree["n_nodes"], to_dev(plen), to_dev(rtok), V)
         acc = fc.fc_accept(tree["tok"], tree["parent"], tree["n_nodes"], am, 12)
-        ms = _cuda_ms(lambda: fc.fc_accept(tree["tok"], tree["parent"], tree["n_nodes"], am, 12, out=acc))
+        ms = _gpu_ms(lambda: fc.fc_accept(tree["tok"], tree["parent"], tree["n_nodes"], am, 12, out=acc))
         nn = tree["n_nodes"].cpu().numpy()
         by = float(sum(12 * int(n) + 4 * (12 + 2) for n in nn))
         return {"ms": ms, "gbs": by / (ms * 1e-3) / 1e9, "frac_hbm": by / (ms * 1e-3) / bw,
@@ -765,12 +787,12 @@ def run_configs(args, rank, ws, local):
         p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
         ctx_d, cl_d = to_dev(ctx), to_dev(cl)
         res = fc.fc_retrieve(sources, ctx_d, cl_d, p)
-        ms_r = _cuda_ms(lambda: fc.fc_retrieve(sources, ctx_d, cl_d, p, out=res))
+        ms_r = _gpu_ms(lambda: fc.fc_retrieve(sources, ctx_d, cl_d, p, out=res))
         B = ctx.shape[0]
         root = to_dev(ctx[np.arange(B), cl - 1].astype(np.uint32))
         kvl = to_dev(np.full(B, kv0, np.int32))
         tree = fc.fc_build_tree(res, [1] * len(sources), root, kvl, budget, n_pad)
-        ms_t = _cuda_ms(lambda: fc.fc_build_tree(res, [1] * len(sources), root, kvl, budget, n_pad, out=tree))
+        ms_t = _gpu_ms(lambda: fc.fc_build_tree(res, [1] * len(sources), root, kvl, budget, n_pad, out=tree))
         ml = res["match_len"].cpu().numpy()
         return tree, {"retrieve_ms": ms_r, "queries_per_s": B / (ms_r * 1e-3),
                       "us_per_query_source": ms_r * 1e3 / (B * len(sources)),
@@ -857,12 +879,187 @@ def run_retrieve(args, rank, ws, local):
     p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
     ctx_d, cl_d = to_dev(ctx), to_dev(cl)
     res = fc.fc_retrieve(sources, ctx_d, cl_d, p)
-    ms = _cuda_ms(lambda: fc.fc_retrieve(sources, ctx_d, cl_d, p, out=res), reps=args.steps, warm=args.warmup)
+    ms = _gpu_ms(lambda: fc.fc_retrieve(sources, ctx_d, cl_d, p, out=res), reps=args.steps, warm=args.warmup)
     return {"metric": "retrievals/s", "value": 2 * args.batch / (ms * 1e-3), "unit": "query-sources/s",
             "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "config": {"workload": f"two-source retrieval (5M + 100M tokens), {args.batch} contexts of 128, "
                                    f"n 16->2, top-64 x 10"},
             "us_per_query_source": ms * 1e3 / (2 * args.batch)}
+
+
+def run_algorithm1(args, rank, ws, local):
+    """The step loop of the default workload with Algorithm 1 in place of the
+    replay cache: per sequence a CACHE (l = 50, 20-token output pieces,
+    8192 words), one missing table for the batch.  --fill untimed steps fill
+    the CACHE first, so the timed steps search active stores; the stage
+    events time the CACHE search, the whole retrieval stage (CACHE search,
+    datastore fallback, missing-table insert) and the CACHE update."""
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    import paper_2502_17139_gb300.synth as synth
+    from paper_2502_17139_gb300.step import StepLoop
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    K, W, F = args.steps, args.warmup, (100 if args.fill is None else args.fill)
+    total = F + W + K + 1
+    inp = make_inputs(args.scale, args.batch, rank, total)
+    cfg, B = inp["cfg"], inp["B"]
+    H, Hkv, D, n_pad, d = cfg["H"], cfg["Hkv"], cfg["D"], cfg["n_pad"], cfg["draft_len"]
+    kv0 = inp["kv0"]
+    cap = kv0 + total * (d + 1) + 8
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).to(dev)
+    sources = [fc.fc_datastore_build(to_dev(T), synth.VOCAB) for T in inp["corpora"]]
+    p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], d, 4096)
+    kc = torch.empty((B, Hkv, cap, D), dtype=torch.bfloat16, device=dev)
+    vc = torch.empty_like(kc)
+    g = torch.Generator(device=dev)
+    g.manual_seed(inp["seed"])
+    kc[:, :, :kv0].normal_(generator=g)
+    vc[:, :, :kv0].normal_(generator=g)
+    seq = dict(capacity=8192, min_size=50, chunk=20, ctx_keep=cfg["n_max"], missing_capacity=1 << 16, weight=1)
+    P = min(16, K + W)
+    q_pool = torch.randn((P, B, n_pad, H, D), generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    kt_pool = torch.randn((P, B, Hkv, n_pad, D), generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    vt_pool = torch.randn((P, B, Hkv, n_pad, D), generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    plen_d, rtok_d = to_dev(inp["plen"]), to_dev(inp["rtok"])
+    zeros = torch.zeros(B, dtype=torch.int32, device=dev)
+
+    def make():
+        return StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, [1, 1], H, Hkv, D, cap, kv0,
+                        synth.VOCAB, device=dev, k_cache=kc, v_cache=vc, seq_cache=seq)
+
+    # untimed pass over the whole trajectory: what each step's retrieval did
+    loop = make()
+    codes, accs = [], []
+    for s in range(F + W + K):
+        j = s % P
+        loop.step(q_pool[j], kt_pool[j], vt_pool[j], zeros, plen_d[s], rtok_d[s], attention=False)
+        codes.append(loop.skip.clone())
+        accs.append(loop.acc["acc_len"].clone())
+    codes = torch.stack(codes).cpu().numpy()[F + W:]
+    accs = torch.stack(accs).cpu().numpy()[F + W:]
+    kc[:, :, kv0:].zero_()
+    vc[:, :, kv0:].zero_()
+
+    loop = make()
+    names = ("retrieve", "cache_search", "cache_update", "tree", "attn", "tail")
+    ev = {nm: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+          for nm in names}
+
+    def do_step(s, i=None):
+        j = s % P
+        loop.step(q_pool[j], kt_pool[j], vt_pool[j], zeros, plen_d[s], rtok_d[s],
+                  events=None if i is None else {nm: ev[nm][i] for nm in names})
+
+    for s in range(F + W):
+        do_step(s)
+    assert fc.fc_get_error() == "FC_OK"
+    barrier(ws)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.wait_first()
+    stream = torch.cuda.current_stream()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(K):
+        do_step(F + W + i, i)
+    end.record(stream)
+    torch.cuda.synchronize()
+    clock_rec = clocks.stop()
+    barrier(ws)
+    assert fc.fc_get_error() == "FC_OK"
+    t_max = max_over_ranks(start.elapsed_time(end), ws)
+    stage = {nm: statistics.mean(a.elapsed_time(b) for a, b in ev[nm]) for nm in names}
+    meta = loop.seq_cache.meta.cpu().numpy()
+    m_stored = int(loop.missing.table[0].item())
+    # the same contexts, retrieved from the datastore alone, and the CACHE
+    # search alone on the final stores (both repeatable: they write only
+    # their outputs)
+    res_all = fc.fc_retrieve(sources, loop.ctx, loop.ctx_len_now, p)
+    ds_ms = _gpu_ms(lambda: fc.fc_retrieve(sources, loop.ctx, loop.ctx_len_now, p, out=res_all), reps=20, warm=3)
+    st = torch.empty(B, dtype=torch.int32, device=dev)
+    res_c = fc.retrieve_outputs(len(sources) + 1, B, p, dev)
+    cs_ms = _gpu_ms(lambda: fc.fc_cache_search(loop.seq_cache, loop.missing, loop.ctx, loop.ctx_len_now, p,
+                                               len(sources), res_c, st), reps=20, warm=3)
+    n_q = codes.size
+    return {"metric": METRIC, "value": weak_value(K, ws, t_max), "unit": UNIT, "n_gpus": ws, "steps": K,
+            "warmup": W, "ms_per_step": t_max / K, "higher_is_better": True, "scaling": "weak",
+            "dtype": "bf16 attention (fp32 accumulate) + u32 retrieval", "data": "synthetic",
+            "config": {"workload": WORKLOAD.replace("50% replay-cache hits", "Algorithm 1: per-sequence CACHE "
+                                                    "(l=50, 20-token pieces, 8192 words) + missing table"),
+                       "fill_steps": F, "batch_per_gpu": B, "kv_len0": kv0,
+                       "l2": "inputs larger than L2 (KV cache 2.2 GB per GPU)"},
+            "stages_ms_per_step": stage,
+            "cache": {"served_frac": float((codes == 1).sum() / n_q), "skipped_frac": float((codes == 2).sum() / n_q),
+                      "datastore_frac": float((codes == 0).sum() / n_q),
+                      "acc_len_served": float(accs[codes == 1].mean()) if (codes == 1).any() else None,
+                      "acc_len_datastore": float(accs[codes == 0].mean()) if (codes == 0).any() else None,
+                      "mean_sequences": float(meta[:, 1].mean()), "mean_words": float(meta[:, 0].mean()),
+                      "missing_keys": m_stored, "cache_search_alone_us": cs_ms * 1e3,
+                      "datastore_retrieval_all_queries_us": ds_ms * 1e3},
+            "clocks": clock_rec}
+
+
+def run_cache(args, rank, ws, local):
+    """fc_cache_search alone on full stores: --batch sequences whose CACHE
+    (8192 words, l = 50) was filled through fc_cache_update along a synthetic
+    generation of --fill steps (each step the context suffix plus the accepted
+    draft tokens, and every 20-token output piece), as in the step loop.
+    Three contexts in four then end with a fresh token, as a context whose
+    last token is the model's bonus token usually does; the others end inside
+    the generation the store was built from."""
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    import paper_2502_17139_gb300.synth as synth
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    B, F, d, n0 = args.batch, (450 if args.fill is None else args.fill), 10, 128
+    rng = synth.rng_for(5, 700 + rank)
+    stride = n0 + F * (d + 1) + 1
+    G = synth.zipf_tokens(rng, B * stride, 1.1).reshape(B, stride)
+    acc = np.stack([np.minimum(synth.argmax_draws(rng, B, 1)[0], d) for _ in range(F)])
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).to(dev)
+    ctx_d = to_dev(G)
+    cache = fc.SequenceCache(B, capacity=8192, min_size=50, chunk=20, ctx_keep=16, device=dev)
+    cur = np.full(B, n0, np.int32)
+    cache.init(to_dev(cur))
+    for s in range(F):
+        new = cur + acc[s] + 1
+        fc.fc_cache_update(cache, ctx_d, to_dev(cur), to_dev(new), to_dev(acc[s].astype(np.int32)))
+        cur = new
+    fresh = rng.random(B) < 0.75
+    Gq = G.copy()
+    Gq[np.arange(B)[fresh], cur[fresh] - 1] = synth.zipf_tokens(rng, int(fresh.sum()), 1.1)
+    q_d, ql_d = to_dev(Gq), to_dev(cur)
+    missing = fc.MissingTable(1 << 16, 2, device=dev)
+    p = fc.params(16, 2, 64, d, 4096)
+    res = fc.retrieve_outputs(3, B, p, dev)
+    state = torch.empty(B, dtype=torch.int32, device=dev)
+    call = lambda: fc.fc_cache_search(cache, missing, q_d, ql_d, p, 2, res, state)
+    call()
+    assert fc.fc_get_error() == "FC_OK"
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.wait_first()
+    ms = _gpu_ms(call, reps=args.steps, warm=args.warmup)
+    clock_rec = clocks.stop()
+    meta = cache.meta.cpu().numpy()
+    words = float(meta[:, 0].sum())
+    peaks = load_peaks()
+    achieved = 4 * words / (ms * 1e-3) / 1e9
+    return {"metric": "CACHE searches/s", "value": B / (ms * 1e-3), "unit": "query-searches/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "config": {"workload": f"fc_cache_search on {B} full stores (8192 words, l=50) filled along {F} "
+                                   "generation steps; n 16->2, top-64 x 10"},
+            "us_per_call": ms * 1e3, "served_frac": float((state.cpu().numpy() == 1).mean()),
+            "mean_words": words / B, "mean_sequences": float(meta[:, 1].mean()),
+            "roofline": {"bound": "latency", "achieved": achieved, "peak": peaks["hbm"], "unit": "GB/s",
+                         "frac": achieved / peaks["hbm"], "traffic": None, "kernel": "k_cache_search",
+                         "note": "bytes = the store words read once; the kernel is bound by its phase latency"},
+            "clocks": clock_rec}
 
 
 def main(argv=None):
@@ -878,6 +1075,10 @@ def main(argv=None):
         out = run_configs(args, rank, ws, local)
     elif args.mode == "retrieve":
         out = run_retrieve(args, rank, ws, local)
+    elif args.mode == "algorithm1":
+        out = run_algorithm1(args, rank, ws, local)
+    elif args.mode == "cache":
+        out = run_cache(args, rank, ws, local)
     else:
         out = run_ours(args, rank, ws, local)
     if rank == 0 and out is not None:

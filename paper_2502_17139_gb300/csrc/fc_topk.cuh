@@ -45,11 +45,12 @@ struct RunsScratch {
   uint32_t n_runs, cstar, n_greater, n_sel, total;
 };
 
-// runs: FC_MAX_OCC + 1 words; work: FC_MAX_OCC words; sel, order: FC_MAX_TOPK
-// words; wsum: NT / 32 words.  Ends with the block synchronised.
+// Run starts from head flags: work[e] (e < nocc <= FC_MAX_OCC) is 1 where
+// occurrence e starts a run.  Writes runs[0..R] (runs[R] = nocc) and returns
+// R.  Ends with the block synchronised.
 template <int NT>
-__device__ uint32_t rank_runs(uint32_t nocc, int k, uint32_t* runs, uint32_t* work, uint32_t* sel, uint32_t* order,
-                              uint32_t* wsum, RunsScratch& sc) {
+__device__ uint32_t runs_from_heads(uint32_t nocc, uint32_t* runs, const uint32_t* work, uint32_t* wsum,
+                                    RunsScratch& sc) {
   constexpr int ITEMS = FC_MAX_OCC / NT;
   static_assert(ITEMS * NT == FC_MAX_OCC, "FC_MAX_OCC must be a multiple of the block size");
   const int tid = threadIdx.x;
@@ -73,7 +74,18 @@ __device__ uint32_t rank_runs(uint32_t nocc, int k, uint32_t* runs, uint32_t* wo
     sc.n_runs = sc.total;
   }
   __syncthreads();
-  const uint32_t R = sc.n_runs;
+  return sc.n_runs;
+}
+
+// Top-k of R runs given by their starts runs[0..R] (counts runs[r+1] -
+// runs[r], between 1 and FC_MAX_OCC), in token order.  Writes order[0..ks),
+// the kept runs ranked by (count descending, run ascending), and returns
+// ks = min(k, R).  work, sel: scratch.  Ends with the block synchronised.
+template <int NT>
+__device__ uint32_t topk_runs(uint32_t R, int k, const uint32_t* runs, uint32_t* work, uint32_t* sel,
+                              uint32_t* order, uint32_t* wsum, RunsScratch& sc) {
+  constexpr int ITEMS = FC_MAX_OCC / NT;
+  const int tid = threadIdx.x;
   auto run_count = [&](uint32_t r) { return runs[r + 1] - runs[r]; };
 
   if (R <= (uint32_t)k) {
@@ -143,4 +155,13 @@ __device__ uint32_t rank_runs(uint32_t nocc, int k, uint32_t* runs, uint32_t* wo
   }
   __syncthreads();
   return ks;
+}
+
+// Both steps: head flags in work -> runs -> top-k (runs: FC_MAX_OCC + 1
+// words; work: FC_MAX_OCC words; sel, order: FC_MAX_TOPK words; wsum: NT / 32).
+template <int NT>
+__device__ uint32_t rank_runs(uint32_t nocc, int k, uint32_t* runs, uint32_t* work, uint32_t* sel, uint32_t* order,
+                              uint32_t* wsum, RunsScratch& sc) {
+  const uint32_t R = runs_from_heads<NT>(nocc, runs, work, wsum, sc);
+  return topk_runs<NT>(R, k, runs, work, sel, order, wsum, sc);
 }

@@ -77,15 +77,20 @@ class StepLoop:
     def step(self, q, k_tree, v_tree, want_hit, plen, rtok, attention=True, events=None):
         """Enqueue one step.  q [B, Np, H, D], k_tree/v_tree [B, Hkv, Np, D]
         (bf16); want_hit [B], plen [B], rtok [B, Np] (int32).  ``events``
-        optionally maps "retrieve" / "tree" / "attn" / "tail" to (start, end)
-        CUDA events recorded around those stages on the current stream."""
+        optionally maps "retrieve" / "tree" / "attn" / "tail" (and, with the
+        CACHE, "cache_search" / "cache_update") to (start, end) CUDA events
+        recorded around those stages on the current stream."""
         c, n = self.cur, 1 - self.cur
         ev = events or {}
         if "retrieve" in ev:
             ev["retrieve"][0].record()
         S = len(self.sources)
         if self.seq:
+            if "cache_search" in ev:
+                ev["cache_search"][0].record()
             fc.fc_cache_search(self.seq_cache, self.missing, self.ctx, self.ctx_len[c], self.p, S, self.res, self.skip)
+            if "cache_search" in ev:
+                ev["cache_search"][1].record()
             fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, skip=self.skip, out=self.res)
             fc.fc_missing_insert(self.missing, self.ctx, self.ctx_len[c], self.skip, self.res["n_drafts"], S)
         elif self.cache is not None:
@@ -118,7 +123,11 @@ class StepLoop:
         fc.fc_kv_append(self.acc, self.tree["tok"], k_tree, v_tree, self.k_cache, self.v_cache, self.kv_len[c],
                         self.kv_len[n], self.ctx, self.ctx_len[c], self.ctx_len[n], self.root)
         if self.seq:
+            if "cache_update" in ev:
+                ev["cache_update"][0].record()
             fc.fc_cache_update(self.seq_cache, self.ctx, self.ctx_len[c], self.ctx_len[n], self.acc["acc_len"])
+            if "cache_update" in ev:
+                ev["cache_update"][1].record()
         if "tail" in ev:
             ev["tail"][1].record()
         self.cur = n

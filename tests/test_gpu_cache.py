@@ -162,20 +162,25 @@ def test_cache_search_parity(fc, a1, case):
     assert served.sum() > 0 or min_size > max_entries
 
 
-def test_cache_search_large_store(fc, a1):
-    """Full 16384-word stores in which one bigram recurs thousands of times:
-    the occurrence sort runs at its largest size and max_occ cuts it."""
-    rng = np.random.default_rng(5100)
+@pytest.mark.parametrize("capacity,plant", [(16384, 1.0), (8192, 0.8), (8192, 0.45), (16384, 0.25), (8192, 0.05)])
+def test_cache_search_large_store(fc, a1, capacity, plant):
+    """Full stores in which one bigram starts a share `plant` of the stored
+    sequences: from a few dozen to a few thousand occurrences, so the
+    occurrence sort runs by ranking, by bitonic stages over packed rows and,
+    past the rows that fit in shared memory, over the store itself; max_occ
+    cuts the largest."""
+    rng = np.random.default_rng(5100 + int(plant * 100) + capacity)
     B, stride = 6, 40
     entries = []
     for b in range(B):
         es, w = [], 0
         while True:
             L = int(rng.integers(3, 12))
-            if w + L + 1 > 16384:
+            if w + L + 1 > capacity:
                 break
             e = rng.integers(0, 6, L).astype(np.uint32)
-            e[:2] = (7, 8)
+            if rng.random() < plant:
+                e[:2] = (7, 8)
             es.append(e)
             w += L + 1
         entries.append(es)
@@ -184,7 +189,7 @@ def test_cache_search_large_store(fc, a1):
     ctx[1, -3:] = (3, 7, 8)
     cl = np.full(B, stride, np.int32)
     for max_occ, d in ((4096, 16), (100, 4), (1, 1)):
-        cache = fc.SequenceCache(B, capacity=16384, min_size=50, chunk=20, ctx_keep=16)
+        cache = fc.SequenceCache(B, capacity=capacity, min_size=50, chunk=20, ctx_keep=16)
         write_stores(cache, entries, cl)
         p = fc.params(16, 2, 64, d, max_occ)
         out = fc.retrieve_outputs(2, B, p)
