@@ -56,6 +56,13 @@ WORKLOAD = ("full step loop: two-source datastore 100M (Zipf 1.1) + 5M (Zipf 1.3
             "GQA 32/8 heads, head_dim 128, KV 16384 bf16, 50% replay-cache hits")
 
 
+def src_weights(args):
+    w = [int(x) for x in args.weights.split(",")]
+    if len(w) != 2 or min(w) < 0 or max(w) > 65535:
+        raise SystemExit("--weights takes two integers in 0..65535")
+    return w
+
+
 def parse_args(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -76,6 +83,8 @@ def parse_args(argv=None):
                          "benchmark line); retrieve: two-source retrieval alone for --batch queries (batch sweeps)")
     ap.add_argument("--nodes", type=int, default=128, help="attn mode: tree nodes per sequence")
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
+    ap.add_argument("--weights", type=str, default="1,1",
+                    help="Eq. 3 source weights alpha,beta (project store, general store) for the step loop")
     ap.add_argument("--fill", type=int, default=None,
                     help="algorithm1 / cache modes: steps that fill the CACHE first (default 100 / 450)")
     ap.add_argument("--skip-1b", action="store_true", help="configs mode: leave out the 1B-token configuration")
@@ -273,8 +282,10 @@ def run_ours(args, rank, ws, local):
     kc[:, :, kv0:].zero_()
     vc[:, :, kv0:].zero_()
 
+    weights = src_weights(args)
+
     def new_loop():
-        return StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, [1, 1], H, Hkv, D, cap, kv0,
+        return StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, weights, H, Hkv, D, cap, kv0,
                         synth.VOCAB, cache_capacity=1 << 14, device=dev, k_cache=kc, v_cache=vc)
 
     # device-resident per-step inputs (a pool of distinct activations, cycled)
@@ -330,7 +341,7 @@ def run_ours(args, rank, ws, local):
 
     # replay the same (deterministic) trajectory untimed to count the
     # attention work of every timed launch
-    flops, bytes_, nodes_hist, acc_hist, hits_used = replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K)
+    flops, bytes_, nodes_hist, acc_hist, hits_used = replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K, weights)
 
     peaks = load_peaks()
     per_launch = []
@@ -359,7 +370,8 @@ def run_ours(args, rank, ws, local):
         "metric": METRIC, "value": weak_value(K, ws, t_max), "unit": UNIT, "n_gpus": ws, "steps": K, "warmup": W,
         "ms_per_step": t_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16 attention (fp32 accumulate) + u32 retrieval", "data": "synthetic",
-        "config": {"workload": WORKLOAD if args.scale == 1.0 else WORKLOAD + f" (scaled x{args.scale})",
+        "config": {"workload": (WORKLOAD if args.scale == 1.0 else WORKLOAD + f" (scaled x{args.scale})")
+                   + ("" if weights == [1, 1] else f", source weights alpha={weights[0]} beta={weights[1]}"),
                    "batch_per_gpu": B, "global_batch": B * ws, "kv_len0": kv0, "n_pad": n_pad,
                    "l2": "inputs larger than L2 (KV cache %.1f GB per GPU)" % (2 * kc.numel() * 2 / 1e9),
                    "parallelism": f"replicas x{ws}"},
@@ -384,7 +396,7 @@ def run_ours(args, rank, ws, local):
     return out
 
 
-def replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K):
+def replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K, weights=(1, 1)):
     """Re-run the loop (untimed, fresh state) and count per-launch attention
     work: FLOPs over unmasked (q, k) pairs and algorithmic HBM bytes."""
     import torch
@@ -393,7 +405,7 @@ def replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K):
     from paper_2502_17139_gb300.step import StepLoop
     B, H, Hkv, D, n_pad = inp["B"], cfg["H"], cfg["Hkv"], cfg["D"], cfg["n_pad"]
     kc = torch.zeros((B, Hkv, cap, D), dtype=torch.bfloat16, device=dev)
-    loop = StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, [1, 1], H, Hkv, D, cap, kv0,
+    loop = StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, list(weights), H, Hkv, D, cap, kv0,
                     synth.VOCAB, cache_capacity=1 << 14, device=dev, k_cache=kc, v_cache=kc)
     q = torch.zeros((B, n_pad, H, D), dtype=torch.bfloat16, device=dev)
     kt = torch.zeros((B, Hkv, n_pad, D), dtype=torch.bfloat16, device=dev)
@@ -549,7 +561,7 @@ def run_reference(args, rank, ws):
         t_ret = 0.0 if inp["hits"][s, b] else time.perf_counter() - tr0
         t0 = time.perf_counter()
         root = ctx[b:b + 1, cl[b] - 1]
-        tr = orc.build_tree(res, [1, 1], root, np.array([kv0], np.int32), cfg["node_budget"], n_pad)
+        tr = orc.build_tree(res, src_weights(args), root, np.array([kv0], np.int32), cfg["node_budget"], n_pad)
         n = int(tr["n_nodes"][0])
         rows = np.array([(0, i, h) for i in range(n) for h in range(G)], np.int32)
         ta = time.perf_counter()

@@ -425,17 +425,40 @@ int orc_tree_mask(const int32_t* parent, const int32_t* n_nodes, const int32_t* 
 //   s     = scale * (q . k) in double precision from the exact bf16 values;
 //   out   = sum softmax(s) * v.
 // Rows i >= n_nodes[b] are zero.  Q and K are taken as already rotated by the
-// caller (position encoding is outside this operation).
+// caller (position encoding is outside this operation); orc_tree_attn_rope
+// below is the same attention with the rotation of O12 applied to the
+// queries and the tree keys.
 //
 // rows == nullptr: every (b, i, h) is computed into out[B][n_pad][H][D].
 // Otherwise rows holds n_rows triples (b, i, h) and out is [n_rows][D].
 // ---------------------------------------------------------------------------
-int orc_tree_attn(const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache, int kv_cap,
-                  const int32_t* kv_len, const uint16_t* k_tree, const uint16_t* v_tree,
-                  const uint64_t* mask, const int32_t* n_nodes, int B, int n_pad, int H, int Hkv,
-                  int D, double scale, const int32_t* rows, int64_t n_rows, double* out,
-                  int nthreads) {
-  if (Hkv < 1 || H % Hkv != 0) return 1;
+}  // extern "C"
+
+namespace {
+
+// O12. Rotary position embedding (Su et al., "RoFormer", 2021): dimension
+// pairs are rotated by pos * f_i with f_i = base^(-2i/D).  The pairing is the
+// rotate-half one of the LLaMA family that the paper's models (DeepSeek-Coder,
+// CodeLlama) belong to: dimension i pairs with i + D/2, for i < D/2.  The
+// position of a tree node is kv_len + depth (Section IV-D adjusts the
+// positional indices of the tree's tokens).
+void rope_row(double* x, int D, double pos, double base) {
+  const int h = D / 2;
+  for (int i = 0; i < h; ++i) {
+    const double a = pos * std::pow(base, -2.0 * i / D);
+    const double c = std::cos(a), sn = std::sin(a);
+    const double x0 = x[i], x1 = x[i + h];
+    x[i] = x0 * c - x1 * sn;
+    x[i + h] = x1 * c + x0 * sn;
+  }
+}
+
+int tree_attn_impl(const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache, int kv_cap,
+                   const int32_t* kv_len, const uint16_t* k_tree, const uint16_t* v_tree, const uint64_t* mask,
+                   const int32_t* n_nodes, int B, int n_pad, int H, int Hkv, int D, double scale,
+                   const int32_t* pos, double base, const int32_t* rows, int64_t n_rows, double* out,
+                   int nthreads) {
+  if (Hkv < 1 || H % Hkv != 0 || (pos && D % 2)) return 1;
   int G = H / Hkv;
   int nw = (n_pad + 63) / 64;
   int64_t total = rows ? n_rows : (int64_t)B * n_pad * H;
@@ -457,8 +480,9 @@ int orc_tree_attn(const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_
     if (i >= n_nodes[b]) return;
     int g = h / G;
     const uint16_t* qv = q + (((size_t)b * n_pad + i) * H + h) * D;
-    std::vector<double> qd(D);
+    std::vector<double> qd(D), kd(D);
     for (int x = 0; x < D; ++x) qd[x] = bf16_to_double(qv[x]);
+    if (pos) rope_row(qd.data(), D, pos[(size_t)b * n_pad + i], base);
     std::vector<double> s;
     std::vector<const uint16_t*> vrow;
     int L = kv_len[b];
@@ -473,8 +497,10 @@ int orc_tree_attn(const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_
     for (int j = 0; j < n_pad; ++j) {
       if (!((mrow[j / 64] >> (j % 64)) & 1)) continue;
       const uint16_t* kr = k_tree + (((size_t)b * Hkv + g) * n_pad + j) * D;
+      for (int x = 0; x < D; ++x) kd[x] = bf16_to_double(kr[x]);
+      if (pos) rope_row(kd.data(), D, pos[(size_t)b * n_pad + j], base);
       double acc = 0.0;
-      for (int x = 0; x < D; ++x) acc += qd[x] * bf16_to_double(kr[x]);
+      for (int x = 0; x < D; ++x) acc += qd[x] * kd[x];
       s.push_back(acc * scale);
       vrow.push_back(v_tree + (((size_t)b * Hkv + g) * n_pad + j) * D);
     }
@@ -491,6 +517,41 @@ int orc_tree_attn(const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_
       for (int x = 0; x < D; ++x) o[x] += pj * bf16_to_double(vrow[j][x]);
     }
   });
+  return 0;
+}
+
+}  // namespace
+
+extern "C" {
+
+int orc_tree_attn(const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache, int kv_cap,
+                  const int32_t* kv_len, const uint16_t* k_tree, const uint16_t* v_tree,
+                  const uint64_t* mask, const int32_t* n_nodes, int B, int n_pad, int H, int Hkv,
+                  int D, double scale, const int32_t* rows, int64_t n_rows, double* out,
+                  int nthreads) {
+  return tree_attn_impl(q, k_cache, v_cache, kv_cap, kv_len, k_tree, v_tree, mask, n_nodes, B, n_pad, H, Hkv, D,
+                        scale, nullptr, 0.0, rows, n_rows, out, nthreads);
+}
+
+// The same attention with the queries of node i and the tree keys of node j
+// rotated (O12) by pos[b][i] and pos[b][j]; the cached keys are taken as
+// rotated already (they were rotated at their own positions when appended).
+int orc_tree_attn_rope(const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache, int kv_cap,
+                       const int32_t* kv_len, const uint16_t* k_tree, const uint16_t* v_tree,
+                       const uint64_t* mask, const int32_t* n_nodes, int B, int n_pad, int H, int Hkv,
+                       int D, double scale, const int32_t* pos, double base, const int32_t* rows,
+                       int64_t n_rows, double* out, int nthreads) {
+  return tree_attn_impl(q, k_cache, v_cache, kv_cap, kv_len, k_tree, v_tree, mask, n_nodes, B, n_pad, H, Hkv, D,
+                        scale, pos, base, rows, n_rows, out, nthreads);
+}
+
+// O12 on its own: rows x[n][D] (double) rotated by pos[n].
+int orc_rope(const double* x, int64_t n, int D, const int32_t* pos, double base, double* out) {
+  if (D < 2 || D % 2) return 1;
+  for (int64_t r = 0; r < n; ++r) {
+    for (int c = 0; c < D; ++c) out[r * D + c] = x[r * D + c];
+    rope_row(out + r * D, D, pos[r], base);
+  }
   return 0;
 }
 

@@ -153,11 +153,24 @@ def tree_mask(parent, n_nodes, kv_len, n_pad):
 
 
 # -------------------------------------------------------------------- O6
+def rope(x, pos, base=10000.0):
+    """O12: rows x[..., D] (float64) rotated by pos[...] (int), rotate-half
+    pairing.  Returns float64 of x's shape."""
+    x = np.ascontiguousarray(x, np.float64)
+    D = x.shape[-1]
+    pos = _c(np.broadcast_to(np.asarray(pos, np.int32), x.shape[:-1]), np.int32)
+    out = np.empty_like(x)
+    rc = lib().orc_rope(_p(x), C.c_int64(x.size // D), C.c_int(D), _p(pos), C.c_double(base), _p(out))
+    assert rc == 0, rc
+    return out
+
+
 def tree_attn(q, k_cache, v_cache, kv_len, k_tree, v_tree, mask, n_nodes, scale=None, rows=None,
-              nthreads: int = 0):
+              nthreads: int = 0, pos=None, rope_base=10000.0):
     """bf16 arrays as uint16 bit patterns: q[B,Np,H,D], caches [B,Hkv,cap,D],
     tree K/V [B,Hkv,Np,D].  Returns fp64 out[B,Np,H,D], or [n_rows, D] for
-    ``rows`` = int32[n_rows, 3] of (b, i, h)."""
+    ``rows`` = int32[n_rows, 3] of (b, i, h).  With ``pos`` (int32 [B,Np]),
+    the queries and the tree keys are rotated by O12 at those positions."""
     q = _c(q, np.uint16)
     k_cache = _c(k_cache, np.uint16)
     v_cache = _c(v_cache, np.uint16)
@@ -177,9 +190,18 @@ def tree_attn(q, k_cache, v_cache, kv_len, k_tree, v_tree, mask, n_nodes, scale=
         rows = _c(rows, np.int32).reshape(-1, 3)
         out = np.empty((rows.shape[0], D), np.float64)
         rp, nr = _p(rows), rows.shape[0]
-    rc = lib().orc_tree_attn(_p(q), _p(k_cache), _p(v_cache), C.c_int(cap), _p(kv_len), _p(k_tree), _p(v_tree),
-                             _p(mask), _p(n_nodes), C.c_int(B), C.c_int(Np), C.c_int(H), C.c_int(Hkv), C.c_int(D),
-                             C.c_double(scale), rp, C.c_int64(nr), _p(out), C.c_int(nthreads))
+    if pos is None:
+        rc = lib().orc_tree_attn(_p(q), _p(k_cache), _p(v_cache), C.c_int(cap), _p(kv_len), _p(k_tree),
+                                 _p(v_tree), _p(mask), _p(n_nodes), C.c_int(B), C.c_int(Np), C.c_int(H),
+                                 C.c_int(Hkv), C.c_int(D), C.c_double(scale), rp, C.c_int64(nr), _p(out),
+                                 C.c_int(nthreads))
+    else:
+        pos = _c(pos, np.int32)
+        assert pos.shape == (B, Np)
+        rc = lib().orc_tree_attn_rope(_p(q), _p(k_cache), _p(v_cache), C.c_int(cap), _p(kv_len), _p(k_tree),
+                                      _p(v_tree), _p(mask), _p(n_nodes), C.c_int(B), C.c_int(Np), C.c_int(H),
+                                      C.c_int(Hkv), C.c_int(D), C.c_double(scale), _p(pos), C.c_double(rope_base),
+                                      rp, C.c_int64(nr), _p(out), C.c_int(nthreads))
     assert rc == 0, rc
     return out
 

@@ -236,6 +236,60 @@ def test_tree_random_drafts(fc, orc, S, k, d, vocab, n_pad):
     check_no_error(fc)
 
 
+WEIGHTS = [(0, 1), (1, 0), (65535, 1), (1, 65535), (3, 1), (1, 3), (0, 0)]
+
+
+@pytest.mark.parametrize("w", WEIGHTS, ids=[f"a{a}b{b}" for a, b in WEIGHTS])
+def test_tree_weight_sweep(fc, orc, w):
+    """Eq. 3 with alpha/beta away from 1, down to 0 and up to the largest
+    weight, on two sources sharing many drafts (small vocabularies) so that
+    merged weights decide which nodes are kept."""
+    rng = np.random.default_rng(4200 + w[0] + 7 * w[1])
+    B, k, d, n_pad = 24, 64, 10, 128
+    res = _random_sources(rng, 2, B, k, d, 3)
+    root = rng.integers(0, 3, B).astype(np.uint32)
+    kvl = rng.integers(0, 5000, B).astype(np.int32)
+    g_res = {name: dev(np.stack([r[name] for r in res])) for name in res[0]}
+    wv = np.array(w, np.uint32)
+    for budget in (2, 17, 64, 128):
+        gt = fc.fc_build_tree(g_res, wv, dev(root), dev(kvl), budget, n_pad)
+        rt = orc.build_tree(res, wv, root, kvl, budget, n_pad)
+        compare_tree(gt, rt)
+    check_no_error(fc)
+
+
+def test_tree_handmade_on_gpu(fc):
+    """The hand-worked trees of tests/golden/tree_handmade.json (weights
+    (1,1), (3,1), (0,1), (1,0), (65535,1)) built by the GPU."""
+    import json
+    import os
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "tree_handmade.json")))
+
+    def src(drafts, lens, counts):
+        k, d = 4, 3
+        o = dict(drafts=np.full((1, k, d), PAD, np.uint32), draft_len=np.zeros((1, k), np.int32),
+                 count=np.zeros((1, k), np.uint32), n_drafts=np.array([len(drafts)], np.int32),
+                 match_len=np.ones(1, np.int32))
+        for t, (u, L, c) in enumerate(zip(drafts, lens, counts)):
+            o["drafts"][0, t, :L] = u[:L]
+            o["draft_len"][0, t] = L
+            o["count"][0, t] = c
+        return o
+
+    r = src(g["src_r"]["drafts"], [3, 3], g["src_r"]["count"])
+    c = src(g["src_c"]["drafts"], g["src_c"]["len"], g["src_c"]["count"])
+    g_res = {name: dev(np.stack([r[name], c[name]])) for name in r}
+    for case in g["cases"]:
+        t = fc.fc_build_tree(g_res, np.array(case["weights"], np.uint32), dev(np.array([9], np.uint32)),
+                             dev(np.array([100], np.int32)), case["budget"], 64)
+        n = int(t["n_nodes"].cpu()[0])
+        assert n == len(case["tok"]), case["why"]
+        assert t["tok"].cpu().numpy()[0, :n].tolist() == case["tok"], case["why"]
+        assert t["parent"].cpu().numpy()[0, :n].tolist() == case["parent"], case["why"]
+        assert t["depth"].cpu().numpy()[0, :n].tolist() == case["depth"], case["why"]
+    check_no_error(fc)
+
+
 def _random_trees(rng, B, n_pad, vocab=32256, full=False):
     tok = np.full((B, n_pad), PAD, np.uint32)
     par = np.full((B, n_pad), -1, np.int32)
