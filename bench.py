@@ -47,9 +47,9 @@ UNIT = "steps/s"
 #       python bench.py --steps 4 --warmup 3 --no-e2e --no-cpu-baseline
 # It is valid only for the kernel sources it was taken on (their SHA-256 below); once
 # those change, the bench reports traffic as null until it is measured again.
-ATTN_TRAFFIC = {"bytes_per_launch": 2.3679e9,
+ATTN_TRAFFIC = {"bytes_per_launch": 2.3670e9,
                 "sources": ["paper_2502_17139_gb300/csrc/tree_attn.cu", "paper_2502_17139_gb300/csrc/fc_common.cuh"],
-                "sha256": "16c816b6bfa050af822e61dc01a220cdae361212071af71bc053544e664f68bb"}
+                "sha256": "ef8c93976042c50443c18522134a35334265e92729d5d394c2d7ce71f39a35b3"}
 
 WORKLOAD = ("full step loop: two-source datastore 100M (Zipf 1.1) + 5M (Zipf 1.3, 20k planted repeats) tokens, "
             "vocab 32256, batch 32, ctx 128, n 16->2, top-64 x 10 tokens per source, tree <=128 nodes, "
@@ -83,6 +83,8 @@ def parse_args(argv=None):
                          "benchmark line); retrieve: two-source retrieval alone for --batch queries (batch sweeps)")
     ap.add_argument("--nodes", type=int, default=128, help="attn mode: tree nodes per sequence")
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
+    ap.add_argument("--rope", action="store_true",
+                    help="attn mode: unrotated queries, rotated in the kernel by node position (fc_tree_attn_rope)")
     ap.add_argument("--weights", type=str, default="1,1",
                     help="Eq. 3 source weights alpha,beta (project store, general store) for the step loop")
     ap.add_argument("--fill", type=int, default=None,
@@ -622,8 +624,16 @@ def run_attn(args, rank, ws, local):
     kt, vt = rnd(B, Hkv, n_pad, D), rnd(B, Hkv, n_pad, D)
     out = torch.empty_like(q)
     args_d = (q, kc, vc, to_dev(kvl), kt, vt, m["mask"], to_dev(nn))
+    if args.rope:
+        pos = m["pos"]
+        kt_rot = fc.fc_rope(kt, pos, 10000.0, layout=1)
+        args_d = (q, kc, vc, to_dev(kvl), kt_rot, vt, m["mask"], to_dev(nn))
+        attn = lambda: fc.fc_tree_attn_rope(*args_d, pos, 10000.0, out=out)
+        rope_k_ms = _gpu_ms(lambda: fc.fc_rope(kt, pos, 10000.0, layout=1, out=kt_rot))
+    else:
+        attn = lambda: fc.fc_tree_attn(*args_d, out=out)
     for _ in range(args.warmup):
-        fc.fc_tree_attn(*args_d, out=out)
+        attn()
     assert fc.fc_get_error() == "FC_OK"
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     barrier(ws)
@@ -632,7 +642,7 @@ def run_attn(args, rank, ws, local):
     clocks.wait_first()
     for e0, e1 in evs:
         e0.record()
-        fc.fc_tree_attn(*args_d, out=out)
+        attn()
         e1.record()
     torch.cuda.synchronize()
     clock_rec = clocks.stop()
@@ -644,9 +654,12 @@ def run_attn(args, rank, ws, local):
     peaks = load_peaks()
     return {"metric": "tree-attn TFLOP/s", "value": flops / (ms * 1e-3) / 1e12, "unit": "TFLOP/s",
             "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-            "config": {"workload": f"tree attention B={B} H=32 Hkv=8 D=128 KV={L} nodes={args.nodes}"},
+            "config": {"workload": f"tree attention B={B} H=32 Hkv=8 D=128 KV={L} nodes={args.nodes}"
+                                   + (", RoPE by node position" if args.rope else "")},
             "frac_tensor_sustained": flops / (ms * 1e-3) / 1e12 / peaks["tc_sustained"],
             "frac_hbm": bytes_ / (ms * 1e-3) / 1e9 / peaks["hbm"], "flops": flops, "bytes": bytes_,
+            "rope": ({"queries": "rotated inside the attention kernel", "tree_key_rotation_ms": rope_k_ms}
+                     if args.rope else None),
             "clocks": clock_rec}
 
 

@@ -393,6 +393,37 @@ size_t fc_tree_attn_workspace(int batch, int n_pad, int H, int Hkv);
 int fc_tree_attn_parts(int batch, int n_pad, int H, int Hkv, int kv_cap, size_t ws_bytes);
 
 /* ------------------------------------------------------------------------
+ * Rotary position embedding by node position (Section IV-D: the tree's tokens
+ * take adjusted position indices, kv_len + depth, which fc_build_tree writes
+ * to d_pos).  RoPE (Su et al., RoFormer) with the rotate-half pairing of the
+ * LLaMA family: dimension i pairs with i + D/2 and turns by
+ * pos * base^(-2i/D).  Angles in fp32, reduced modulo 2 pi before the
+ * sine and cosine; results rounded to bf16.  A negative position (a padding
+ * row of a tree) leaves its row unchanged.
+ * ------------------------------------------------------------------------ */
+/*
+ * Rotates bf16 rows: layout 0 = node-major [batch][n_pad][heads][D] (queries),
+ * layout 1 = head-major [batch][heads][n_pad][D] (tree keys); row (b, i, h)
+ * turns by d_pos[b][i].  d_out may equal d_in.  D a multiple of 16 up to
+ * 1024; pointers 16-byte aligned; base > 0.
+ */
+fc_status fc_rope(const void* d_in, void* d_out, int batch, int n_pad, int heads, int D, int layout,
+                  const int32_t* d_pos, float base, fc_stream s);
+
+/*
+ * fc_tree_attn with unrotated queries: the query of node i is rotated by
+ * d_pos[b][i] inside the kernel, while its tile is staged.  d_k_tree must
+ * hold the tree keys already rotated (fc_rope, layout 1, the same d_pos and
+ * base); the cached keys are the rotated keys of earlier steps.  Limits and
+ * workspace as fc_tree_attn.
+ */
+fc_status fc_tree_attn_rope(const void* d_q, const void* d_k_cache, const void* d_v_cache, int kv_cap,
+                            const int32_t* d_kv_len, const void* d_k_tree, const void* d_v_tree,
+                            const uint64_t* d_mask, const int32_t* d_n_nodes, int batch, int n_pad,
+                            int H, int Hkv, int D, float scale, const int32_t* d_pos, float rope_base,
+                            void* d_out, void* d_ws, size_t ws_bytes, fc_stream s);
+
+/* ------------------------------------------------------------------------
  * Acceptance (Section IV-D: every correct token from the start is accepted,
  * everything after the first error rejected; Eq. 7 counts tokens per step).
  * ------------------------------------------------------------------------ */

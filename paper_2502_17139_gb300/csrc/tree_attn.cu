@@ -91,7 +91,86 @@ struct AttnArgs {
   float2* ws_ml;   // [split units][parts - 1][256 rows]: (m, l) of a partial
   float* ws_o;     // [split units][parts - 1][256 rows][128]: unnormalised O of a partial
   float scale_log2;
+  const int32_t* pos;  // [B][n_pad] node positions: rotate Q by them (RoPE), or nullptr
+  double rope_nl2f;    // -2 log2(base) / D: pair i turns by pos * 2^(i * rope_nl2f)
 };
+
+// ---- rotary position embedding (Su et al., RoFormer), rotate-half pairing:
+// dimension i pairs with i + D/2 and turns by pos * f_i, f_i = base^(-2i/D).
+// f_i is held as two floats (hi + lo, from fp64), so that pos * f_i comes out
+// as hi * pos, its exact rounding error (an fma) and lo * pos: the angle is
+// good to ~1e-7 rad at any position below 2^24, where a plain fp32 product
+// would be off by pos * f_i * 2^-24.  The angle is reduced modulo 2 pi with a
+// two-constant Cody-Waite split (2 pi rounded to fp32, then the rest) before
+// the MUFU sine and cosine, which are accurate on [-pi, pi].
+constexpr int ROPE_MAX_HALF = 512;  // D / 2 for D up to 1024
+
+// tab[i] = (hi, lo) of f_i for i < half, filled by the calling block's
+// threads; the caller synchronises before use.
+__device__ __forceinline__ void rope_table(float2* tab, int half, double nl2f) {
+  for (int i = threadIdx.x; i < half; i += blockDim.x) {
+    const double f = exp2((double)i * nl2f);
+    const float hi = (float)f;
+    tab[i] = make_float2(hi, (float)(f - (double)hi));
+  }
+}
+
+__device__ __forceinline__ void rope_sincos(float pos, float2 f, float& sn, float& cs) {
+  const float a_hi = pos * f.x;
+  const float a_lo = fmaf(pos, f.y, fmaf(pos, f.x, -a_hi));
+  const float k = rintf(a_hi * 0.15915493667125702f);  // a / (2 pi), rounded
+  float r = fmaf(-k, 6.2831854820251465f, a_hi);        // 2 pi rounded to fp32
+  r = fmaf(-k, -1.7484555314695172e-07f, r) + a_lo;     // 2 pi minus that
+  __sincosf(r, &sn, &cs);
+}
+
+// Rotates the two pairs held by one 32-bit word of each half: l holds
+// dimensions i, i + 1 and h the same dimensions + D/2.
+__device__ __forceinline__ void rope_word(uint32_t& l, uint32_t& h, float pos, const float2* tab, int i) {
+  __nv_bfloat162 lb = *reinterpret_cast<__nv_bfloat162*>(&l), hb = *reinterpret_cast<__nv_bfloat162*>(&h);
+  const float2 xl = __bfloat1622float2(lb), xh = __bfloat1622float2(hb);
+  float s0, c0, s1, c1;
+  rope_sincos(pos, tab[i], s0, c0);
+  rope_sincos(pos, tab[i + 1], s1, c1);
+  lb = __float22bfloat162_rn(make_float2(xl.x * c0 - xh.x * s0, xl.y * c1 - xh.y * s1));
+  hb = __float22bfloat162_rn(make_float2(xh.x * c0 + xl.x * s0, xh.y * c1 + xl.y * s1));
+  l = *reinterpret_cast<uint32_t*>(&lb);
+  h = *reinterpret_cast<uint32_t*>(&hb);
+}
+
+// Rotates the 8 pairs held by two 16-byte chunks: lo = dimensions
+// i0 .. i0 + 7, hi = the same dimensions + D/2.
+__device__ __forceinline__ void rope_chunks(uint4& lo, uint4& hi, float pos, const float2* tab, int i0) {
+  rope_word(lo.x, hi.x, pos, tab, i0);
+  rope_word(lo.y, hi.y, pos, tab, i0 + 2);
+  rope_word(lo.z, hi.z, pos, tab, i0 + 4);
+  rope_word(lo.w, hi.w, pos, tab, i0 + 6);
+}
+
+// The Q tiles of a CTA with RoPE fused into the staging: a 16-byte chunk of
+// the first 64 dimensions and its partner chunk of the second 64 are rotated
+// together and land at the same swizzled offset of the two halves.
+__device__ __forceinline__ void stage_q_rope(unsigned char* sq, const __nv_bfloat16* q, const int32_t* pos,
+                                             const float2* tab, int b, int g, int G, int H, int n_pad, int nn,
+                                             int row0, int rows_total, int tid) {
+  for (int e = tid; e < TILES * BM * 8; e += TA_THREADS) {
+    const int r = e >> 3, gran = e & 7;
+    const int tile = r / BM, rt = r - tile * BM;
+    const int rg = row0 + r;
+    uint4 lo = make_uint4(0, 0, 0, 0), hi = lo;
+    if (rg < rows_total) {
+      const int hh = rg / nn, i = rg - hh * nn;
+      const uint4* src = reinterpret_cast<const uint4*>(q + (((size_t)b * n_pad + i) * H + g * G + hh) * HD);
+      lo = src[gran];
+      hi = src[gran + 8];
+      const int p = pos[(size_t)b * n_pad + i];
+      if (p >= 0) rope_chunks(lo, hi, (float)p, tab, 8 * gran);
+    }
+    unsigned char* dst = sq + tile * TILE_BYTES + rt * 128 + ((gran ^ (rt & 7)) << 4);
+    *reinterpret_cast<uint4*>(dst) = lo;
+    *reinterpret_cast<uint4*>(dst + HALF_BYTES) = hi;
+  }
+}
 
 // 2^x on the MUFU unit.  The flush-to-zero form is a single instruction; the
 // results it flushes (below 2^-126) are probabilities that cannot move an
@@ -146,6 +225,9 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
   return __all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar, parity, abort, WAIT_CYCLES));
 }
 
+// ROPE: the queries arrive unrotated and are rotated by a.pos while staged
+// (a separate instance, so the plain kernel's code is unchanged).
+template <bool ROPE>
 __global__ void __launch_bounds__(TA_THREADS, 1)
     k_tree_attn(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                 const __grid_constant__ CUtensorMap tm_kt, const __grid_constant__ CUtensorMap tm_vt, AttnArgs a) {
@@ -250,6 +332,12 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     tmem_relinquish();
   }
   // Q tiles: rows (head in group, node) packed densely, 128-byte swizzled, K-major.
+  if constexpr (ROPE) {
+    __shared__ float2 s_rope[HD / 2];
+    rope_table(s_rope, HD / 2, a.rope_nl2f);
+    __syncthreads();
+    stage_q_rope(smem + OFF_Q, a.q, a.pos, s_rope, b, g, a.G, a.H, a.n_pad, nn, row0, rows_total, tid);
+  } else
   for (int e = tid; e < TILES * BM * 16; e += TA_THREADS) {
     const int r = e >> 4, ch = e & 15, half = ch >> 3, gran = ch & 7;
     const int tile = r / BM, rt = r - tile * BM;
@@ -711,6 +799,37 @@ uint64_t attn_units(int batch, int n_pad, int H, int Hkv) {
   return (uint64_t)batch * Hkv * (((uint64_t)(H / Hkv) * n_pad + TILES * BM - 1) / (TILES * BM));
 }
 
+// fc_rope: rows of bf16 vectors rotated by their node's position.  layout 0
+// is node-major [B][n_pad][heads][D] (queries), layout 1 head-major
+// [B][heads][n_pad][D] (tree keys).  One thread per pair of partner chunks.
+__global__ void k_rope(const uint4* __restrict__ in, uint4* __restrict__ out, int B, int n_pad, int heads, int D,
+                       int layout, const int32_t* __restrict__ pos, double nl2f) {
+  __shared__ float2 tab[ROPE_MAX_HALF];
+  rope_table(tab, D / 2, nl2f);
+  __syncthreads();
+  const int ch = D / 16;  // 16-byte chunks per half row
+  const size_t items = (size_t)B * n_pad * heads * ch;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < items; e += (size_t)gridDim.x * blockDim.x) {
+    const int gran = (int)(e % ch);
+    const size_t row = e / ch;
+    int bb, i;
+    if (layout == 0) {
+      const size_t bi = row / heads;
+      bb = (int)(bi / n_pad);
+      i = (int)(bi % n_pad);
+    } else {
+      i = (int)(row % n_pad);
+      bb = (int)(row / ((size_t)heads * n_pad));
+    }
+    const uint4* src = in + row * (D / 8);
+    uint4 lo = src[gran], hi = src[gran + ch];
+    const int p = pos[(size_t)bb * n_pad + i];
+    if (p >= 0) rope_chunks(lo, hi, (float)p, tab, 8 * gran);
+    out[row * (D / 8) + gran] = lo;
+    out[row * (D / 8) + gran + ch] = hi;
+  }
+}
+
 }  // namespace
 
 extern "C" size_t fc_tree_attn_workspace(int batch, int n_pad, int H, int Hkv) {
@@ -726,10 +845,11 @@ extern "C" int fc_tree_attn_parts(int batch, int n_pad, int H, int Hkv, int kv_c
   return choose_split(attn_units(batch, n_pad, H, Hkv), kv_cap, ws_bytes).parts;
 }
 
-extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const void* d_v_cache, int kv_cap,
+static fc_status launch_tree_attn(const void* d_q, const void* d_k_cache, const void* d_v_cache, int kv_cap,
                                   const int32_t* d_kv_len, const void* d_k_tree, const void* d_v_tree,
-                                  const uint64_t* d_mask, const int32_t* d_n_nodes, int batch, int n_pad, int H, int Hkv,
-                                  int D, float scale, void* d_out, void* d_ws, size_t ws_bytes, fc_stream stream) {
+                                  const uint64_t* d_mask, const int32_t* d_n_nodes, int batch, int n_pad, int H,
+                                  int Hkv, int D, float scale, void* d_out, void* d_ws, size_t ws_bytes,
+                                  const int32_t* d_pos, float rope_base, fc_stream stream) {
   if (batch < 0 || H < 1 || Hkv < 1 || kv_cap < 1) return FC_ERR_INVALID_ARG;
   if (D != HD || (n_pad != 64 && n_pad != 128) || H % Hkv != 0 || H / Hkv > 16) return FC_ERR_UNSUPPORTED;
   if (!(scale > 0.f)) return FC_ERR_INVALID_ARG;
@@ -754,11 +874,12 @@ extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const 
       !make_map(&mkt, d_k_tree, (uint64_t)n_pad, groups, (uint32_t)n_pad) ||
       !make_map(&mvt, d_v_tree, (uint64_t)n_pad, groups, (uint32_t)n_pad))
     return FC_ERR_CUDA;
-  if (cudaFuncSetAttribute(k_tree_attn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES) != cudaSuccess)
+  auto kern = d_pos ? k_tree_attn<true> : k_tree_attn<false>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES) != cudaSuccess)
     return FC_ERR_CUDA;
   {  // the register split needs the whole launch allocation (see REGS_LAUNCH)
     cudaFuncAttributes fa;
-    if (cudaFuncGetAttributes(&fa, k_tree_attn) != cudaSuccess) return FC_ERR_CUDA;
+    if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess) return FC_ERR_CUDA;
     if (fa.numRegs < REGS_LAUNCH) return FC_ERR_INTERNAL;
   }
   AttnArgs a;
@@ -780,6 +901,8 @@ extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const 
   a.ws_cnt = nullptr;
   a.ws_ml = nullptr;
   a.ws_o = nullptr;
+  a.pos = d_pos;
+  a.rope_nl2f = d_pos ? -2.0 * std::log2((double)rope_base) / HD : 0.0;
   if (sp.parts > 1) {
     const WsLayout w = ws_layout(n_split, sp.parts);
     unsigned char* base = static_cast<unsigned char*>(d_ws);
@@ -789,7 +912,41 @@ extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const 
     if (cudaMemsetAsync(a.ws_cnt, 0, n_split * 2 * sizeof(int), static_cast<cudaStream_t>(stream)) != cudaSuccess)
       return FC_ERR_CUDA;
   }
-  k_tree_attn<<<(unsigned)grid, TA_THREADS, SMEM_BYTES, static_cast<cudaStream_t>(stream)>>>(mkc, mvc, mkt,
-                                                                                                        mvt, a);
+  kern<<<(unsigned)grid, TA_THREADS, SMEM_BYTES, static_cast<cudaStream_t>(stream)>>>(mkc, mvc, mkt, mvt, a);
+  return FC_CHECK_LAUNCH();
+}
+
+extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const void* d_v_cache, int kv_cap,
+                                  const int32_t* d_kv_len, const void* d_k_tree, const void* d_v_tree,
+                                  const uint64_t* d_mask, const int32_t* d_n_nodes, int batch, int n_pad, int H, int Hkv,
+                                  int D, float scale, void* d_out, void* d_ws, size_t ws_bytes, fc_stream stream) {
+  return launch_tree_attn(d_q, d_k_cache, d_v_cache, kv_cap, d_kv_len, d_k_tree, d_v_tree, d_mask, d_n_nodes, batch,
+                          n_pad, H, Hkv, D, scale, d_out, d_ws, ws_bytes, nullptr, 0.f, stream);
+}
+
+extern "C" fc_status fc_tree_attn_rope(const void* d_q, const void* d_k_cache, const void* d_v_cache, int kv_cap,
+                                       const int32_t* d_kv_len, const void* d_k_tree, const void* d_v_tree,
+                                       const uint64_t* d_mask, const int32_t* d_n_nodes, int batch, int n_pad, int H,
+                                       int Hkv, int D, float scale, const int32_t* d_pos, float rope_base,
+                                       void* d_out, void* d_ws, size_t ws_bytes, fc_stream stream) {
+  if (!(rope_base > 0.f) || !std::isfinite(rope_base)) return FC_ERR_INVALID_ARG;
+  if (batch > 0 && !d_pos) return FC_ERR_INVALID_ARG;
+  return launch_tree_attn(d_q, d_k_cache, d_v_cache, kv_cap, d_kv_len, d_k_tree, d_v_tree, d_mask, d_n_nodes, batch,
+                          n_pad, H, Hkv, D, scale, d_out, d_ws, ws_bytes, d_pos, rope_base, stream);
+}
+
+extern "C" fc_status fc_rope(const void* d_in, void* d_out, int batch, int n_pad, int heads, int D, int layout,
+                             const int32_t* d_pos, float base, fc_stream stream) {
+  if (batch < 0 || n_pad < 1 || heads < 1 || D < 16 || D > 1024 || D % 16 || (layout != 0 && layout != 1))
+    return FC_ERR_INVALID_ARG;
+  if (!(base > 0.f) || !std::isfinite(base)) return FC_ERR_INVALID_ARG;
+  if (batch == 0) return FC_OK;
+  if (!d_in || !d_out || !d_pos) return FC_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(d_in) | reinterpret_cast<uintptr_t>(d_out)) % 16) return FC_ERR_INVALID_ARG;
+  const size_t items = (size_t)batch * n_pad * heads * (D / 16);
+  const unsigned blocks = (unsigned)std::min<size_t>((items + 255) / 256, 152 * 16);
+  k_rope<<<blocks, 256, 0, static_cast<cudaStream_t>(stream)>>>(static_cast<const uint4*>(d_in),
+                                                                static_cast<uint4*>(d_out), batch, n_pad, heads, D,
+                                                                layout, d_pos, -2.0 * std::log2((double)base) / D);
   return FC_CHECK_LAUNCH();
 }

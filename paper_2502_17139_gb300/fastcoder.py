@@ -53,7 +53,7 @@ EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build
            "fc_datastore_build_noalloc",
            "fc_retrieve", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
-           "fc_missing_insert", "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
+           "fc_missing_insert", "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
 
 
 def _load():
@@ -90,6 +90,9 @@ def _load():
         "fc_tree_attn": (C.c_int, [vp, vp, vp, i32, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, C.c_float, vp, vp, sz,
                                    vp]),
         "fc_tree_attn_workspace": (sz, [i32, i32, i32, i32]),
+        "fc_rope": (C.c_int, [vp, vp, i32, i32, i32, i32, i32, vp, C.c_float, vp]),
+        "fc_tree_attn_rope": (C.c_int, [vp, vp, vp, i32, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, C.c_float, vp,
+                                        C.c_float, vp, vp, sz, vp]),
         "fc_tree_attn_parts": (C.c_int, [i32, i32, i32, i32, i32, sz]),
         "fc_accept": (C.c_int, [vp, vp, vp, vp, i32, i32, vp, vp, i32, vp, vp]),
         "fc_argmax_accept": (C.c_int, [vp, i32, vp, vp, vp, i32, i32, vp, vp, vp, i32, vp, vp]),
@@ -410,6 +413,50 @@ def fc_tree_attn(q, k_cache, v_cache, kv_len, k_tree, v_tree, mask, n_nodes, sca
     _check("fc_tree_attn", LIB.fc_tree_attn(_ptr(q), _ptr(k_cache), _ptr(v_cache), cap, _ptr(kv_len), _ptr(k_tree),
                                             _ptr(v_tree), _ptr(mask), _ptr(n_nodes), B, Np, H, Hkv, D, sc, _ptr(o),
                                             _ptr(workspace), ws_bytes, _stream()))
+    return o
+
+
+def fc_rope(x, pos, base=10000.0, layout=None, out=None):
+    """bf16 x [B, Np, heads, D] (layout 0, queries) or [B, heads, Np, D]
+    (layout 1, tree keys; pass layout=1); pos int32 [B, Np].  Returns the
+    rotated rows (``out`` may be ``x``)."""
+    _need(x, torch.bfloat16, "x")
+    B = x.shape[0]
+    layout = 0 if layout is None else layout
+    if layout == 0:
+        _, Np, heads, D = x.shape
+    else:
+        _, heads, Np, D = x.shape
+    _need(pos, torch.int32, "pos", (B, Np))
+    o = out if out is not None else torch.empty_like(x)
+    _check("fc_rope", LIB.fc_rope(_ptr(x), _ptr(o), B, Np, heads, D, layout, _ptr(pos), C.c_float(base), _stream()))
+    return o
+
+
+def fc_tree_attn_rope(q, k_cache, v_cache, kv_len, k_tree_rot, v_tree, mask, n_nodes, pos, rope_base=10000.0,
+                      scale=None, out=None, workspace="auto"):
+    """fc_tree_attn with unrotated q (rotated in the kernel by pos [B, Np]);
+    k_tree_rot: the tree keys rotated by fc_rope(..., layout=1)."""
+    _need(q, torch.bfloat16, "q")
+    B, Np, H, D = q.shape
+    _need(k_cache, torch.bfloat16, "k_cache")
+    Hkv, cap = k_cache.shape[1], k_cache.shape[2]
+    _need(v_cache, torch.bfloat16, "v_cache", k_cache.shape)
+    _need(k_tree_rot, torch.bfloat16, "k_tree_rot", (B, Hkv, Np, D))
+    _need(v_tree, torch.bfloat16, "v_tree", (B, Hkv, Np, D))
+    _need(mask, torch.int64, "mask", (B, Np, Np // 64))
+    _need(kv_len, torch.int32, "kv_len", (B,))
+    _need(n_nodes, torch.int32, "n_nodes", (B,))
+    _need(pos, torch.int32, "pos", (B, Np))
+    o = out if out is not None else torch.empty_like(q)
+    sc = float(scale) if scale is not None else D ** -0.5
+    if isinstance(workspace, str):
+        workspace = attn_workspace(B, Np, H, Hkv, q.device)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check("fc_tree_attn_rope", LIB.fc_tree_attn_rope(
+        _ptr(q), _ptr(k_cache), _ptr(v_cache), cap, _ptr(kv_len), _ptr(k_tree_rot), _ptr(v_tree), _ptr(mask),
+        _ptr(n_nodes), B, Np, H, Hkv, D, sc, _ptr(pos), C.c_float(rope_base), _ptr(o), _ptr(workspace), ws_bytes,
+        _stream()))
     return o
 
 

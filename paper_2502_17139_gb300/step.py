@@ -29,10 +29,15 @@ from . import fastcoder as fc
 
 class StepLoop:
     def __init__(self, sources, ctx, ctx_len, p, node_budget, n_pad, src_weight, H, Hkv, D, kv_cap, kv_len0, vocab,
-                 cache_capacity=1 << 14, device="cuda", k_cache=None, v_cache=None, seq_cache=None):
+                 cache_capacity=1 << 14, device="cuda", k_cache=None, v_cache=None, seq_cache=None,
+                 rope_base=None):
         """seq_cache: None, or a dict with capacity, min_size, chunk, ctx_keep
         (the CACHE), missing_capacity (M) and weight (the CACHE slot's tree
-        weight); it replaces the replay cache."""
+        weight); it replaces the replay cache.  rope_base: None (q and the
+        tree keys arrive rotated), or the RoPE base: step() then takes them
+        unrotated, the tree keys are rotated once by their node positions
+        (fc_rope) for the attention and the cache append, and the queries are
+        rotated inside the attention kernel (fc_tree_attn_rope)."""
         self.sources, self.p, self.node_budget, self.n_pad = sources, p, node_budget, n_pad
         self.src_weight = list(src_weight)
         self.H, self.Hkv, self.D, self.kv_cap, self.vocab = H, Hkv, D, kv_cap, vocab
@@ -63,6 +68,9 @@ class StepLoop:
         self.k_cache = k_cache if k_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         self.v_cache = v_cache if v_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         self.attn_out = torch.empty((B, n_pad, H, D), dtype=torch.bfloat16, device=device)
+        self.rope_base = rope_base
+        self.k_tree_rot = (torch.empty((B, Hkv, n_pad, D), dtype=torch.bfloat16, device=device)
+                           if rope_base is not None else None)
         self.cache = fc.RetrievalCache(cache_capacity, S, p, device) if cache_capacity and not self.seq else None
         if self.seq:
             q = self.seq
@@ -107,11 +115,17 @@ class StepLoop:
                          out=self.tree)
         if "tree" in ev:
             ev["tree"][1].record()
+        if self.rope_base is not None:
+            k_tree = fc.fc_rope(k_tree, self.tree["pos"], self.rope_base, layout=1, out=self.k_tree_rot)
         if attention:
             if "attn" in ev:
                 ev["attn"][0].record()
-            fc.fc_tree_attn(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree, self.tree["mask"],
-                            self.tree["n_nodes"], out=self.attn_out)
+            if self.rope_base is not None:
+                fc.fc_tree_attn_rope(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree, self.tree["mask"],
+                                     self.tree["n_nodes"], self.tree["pos"], self.rope_base, out=self.attn_out)
+            else:
+                fc.fc_tree_attn(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree, self.tree["mask"],
+                                self.tree["n_nodes"], out=self.attn_out)
             if "attn" in ev:
                 ev["attn"][1].record()
         if "tail" in ev:

@@ -121,3 +121,22 @@ def test_cache_host_validation_without_gpu(lib):
     assert L.fc_missing_init(16, 4 * (4 + 1024 * 3) - 1, 1024, 2, nul) == 3
     assert L.fc_missing_insert(16, 1024, 0, 16, 64, 16, 4, 16, 16, 2, nul) == 1
     assert L.fc_missing_insert(nul, 1024, 2, 16, 64, 16, 4, 16, 16, 2, nul) == 1
+
+
+def test_rope_host_validation_without_gpu(lib):
+    import paper_2502_17139_gb300.fastcoder as fc
+    L = fc.LIB
+    nul = None
+    f = C.c_float
+    # head dims that are not a multiple of 16, a bad layout, a non-positive base, odd addresses
+    assert L.fc_rope(16, 16, 2, 64, 4, 100, 0, 16, f(10000.0), nul) == 1
+    assert L.fc_rope(16, 16, 2, 64, 4, 128, 2, 16, f(10000.0), nul) == 1
+    assert L.fc_rope(16, 16, 2, 64, 4, 128, 0, 16, f(0.0), nul) == 1
+    assert L.fc_rope(17, 16, 2, 64, 4, 128, 0, 16, f(10000.0), nul) == 1
+    assert L.fc_rope(nul, nul, 0, 64, 4, 128, 0, nul, f(10000.0), nul) == 0
+    # the rotated attention: missing positions, a non-positive base, then fc_tree_attn's own limits
+    args = [16, 16, 16, 128, 16, 16, 16, 8, 16, 2, 64, 32, 8, 128, f(0.1)]
+    assert L.fc_tree_attn_rope(*args, nul, f(10000.0), 16, nul, 0, nul) == 1
+    assert L.fc_tree_attn_rope(*args, 16, f(-1.0), 16, nul, 0, nul) == 1
+    bad_d = args[:13] + [96, f(0.1)]
+    assert L.fc_tree_attn_rope(*bad_d, 16, f(10000.0), 16, nul, 0, nul) == 2
