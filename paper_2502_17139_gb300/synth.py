@@ -302,3 +302,34 @@ def build_corpus(rng: np.random.Generator, spec: dict, vocab: int = VOCAB, devic
     if spec.get("frac"):
         grams = grams_for_fraction(n, spec["frac"], lr, cr)
     return make_corpus(rng, n, spec["s"], vocab, grams, lr, cr, device=device)
+
+
+def decoder_weights(hidden: int, layers: int, H: int, Hkv: int, D: int, inter: int, vocab: int, seed: int,
+                    device="cpu"):
+    """Seeded random-init weights of a LLaMA-family decoder (the paper's
+    target models are DeepSeek-Coder and CodeLlama; no trained weights are
+    available), as bf16 torch tensors on ``device``: every projection
+    N(0, 1/fan_in), the embedding N(0, 1), norm weights 1 + N(0, 0.1^2).
+    Layout: per layer attn_norm [hidden], wq [hidden][H*D], wkv
+    [hidden][2*Hkv*D] (K columns, then V), wo [H*D][hidden], mlp_norm
+    [hidden], wgu [hidden][2*inter] (gate, then up), wd [inter][hidden];
+    embed [vocab][hidden], final_norm [hidden], lm_head [hidden][vocab]."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed) & ((1 << 63) - 1))
+
+    def mat(k, n, scale=None):
+        s = (1.0 / math.sqrt(k)) if scale is None else scale
+        return (torch.randn((k, n), generator=g, device=device, dtype=torch.float32) * s).to(torch.bfloat16)
+
+    def norm(n):
+        return (1.0 + 0.1 * torch.randn((n,), generator=g, device=device, dtype=torch.float32)).to(torch.bfloat16)
+
+    W = {"embed": mat(vocab, hidden, 1.0), "layers": []}
+    for _ in range(layers):
+        W["layers"].append({"attn_norm": norm(hidden), "wq": mat(hidden, H * D), "wkv": mat(hidden, 2 * Hkv * D),
+                            "wo": mat(H * D, hidden), "mlp_norm": norm(hidden), "wgu": mat(hidden, 2 * inter),
+                            "wd": mat(inter, hidden)})
+    W["final_norm"] = norm(hidden)
+    W["lm_head"] = mat(hidden, vocab)
+    return W
