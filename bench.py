@@ -74,7 +74,8 @@ def parse_args(argv=None):
     ap.add_argument("--batch", type=int, default=32)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--mode", choices=["step", "attn", "argmax", "configs", "retrieve", "algorithm1", "cache"],
+    ap.add_argument("--mode", choices=["step", "attn", "argmax", "configs", "retrieve", "algorithm1", "cache",
+                                       "decoder"],
                     default="step",
                     help="step: the full step loop (the benchmark); attn: tree attention alone on the step loop's "
                          "attention shape with seeded trees (a small profiling / sweep target); argmax: greedy "
@@ -1087,6 +1088,102 @@ def run_cache(args, rank, ws, local):
             "clocks": clock_rec}
 
 
+def run_decoder(args, rank, ws, local):
+    """The step loop with the target model's forward as the verifier: a
+    randomly initialised decoder of DeepSeek-Coder 1.3B's shape (24 layers,
+    hidden 2048, 16 heads of 128, MLP 5504, vocab 32256) verifies 64-node
+    draft trees for --batch sequences over a 2048-token cache, greedy
+    acceptance from its logits; retrieval from the default two-source store
+    (replay cache off).  With random weights the acceptance carries no
+    meaning; the step's cost does."""
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    import paper_2502_17139_gb300.synth as synth
+    from paper_2502_17139_gb300.decoder import DEEPSEEK_CODER_1_3B, TreeDecoder
+    from paper_2502_17139_gb300.step import StepLoop
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    s = DEEPSEEK_CODER_1_3B
+    K, W = args.steps, args.warmup
+    total = K + W + 1
+    inp = make_inputs(args.scale, args.batch, rank, total)
+    cfg, B = inp["cfg"], inp["B"]
+    n_pad, d, kv0 = 64, cfg["draft_len"], 2048
+    cap = kv0 + total * (d + 1) + 8
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).to(dev)
+    sources = [fc.fc_datastore_build(to_dev(T), synth.VOCAB) for T in inp["corpora"]]
+    p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], d, 4096)
+    Wt = synth.decoder_weights(s.hidden, s.layers, s.H, s.Hkv, s.D, s.inter, s.vocab, inp["seed"], device=dev)
+    caches = []
+    for l in range(s.layers):
+        kc = torch.zeros((B, s.Hkv, cap, s.D), dtype=torch.bfloat16, device=dev)
+        vc = torch.zeros_like(kc)
+        kc[:, :, :kv0] = synth.randn_bf16((B, s.Hkv, kv0, s.D), inp["seed"] + 10 + l, dev)
+        vc[:, :, :kv0] = synth.randn_bf16((B, s.Hkv, kv0, s.D), inp["seed"] + 500 + l, dev)
+        caches.append((kc, vc))
+    td = TreeDecoder(s, Wt, B, n_pad, cap, device=dev, caches=caches)
+    loop = StepLoop(sources, inp["ctx"], inp["cl"], p, n_pad, n_pad, src_weights(args), s.H, s.Hkv, s.D, cap, kv0,
+                    synth.VOCAB, device=dev, k_cache=caches[0][0], v_cache=caches[0][1], decoder=td,
+                    cache_capacity=0)
+    zeros = torch.zeros(B, dtype=torch.int32, device=dev)
+    names = ("retrieve", "tree", "attn", "tail")
+    ev = {nm: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+          for nm in names}
+    for _ in range(W):
+        loop.step(None, None, None, zeros, zeros, None)
+    assert fc.fc_get_error() == "FC_OK"
+    barrier(ws)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.wait_first()
+    stream = torch.cuda.current_stream()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    accs = []
+    start.record(stream)
+    for i in range(K):
+        loop.step(None, None, None, zeros, zeros, None, events={nm: ev[nm][i] for nm in names})
+        accs.append(loop.acc["acc_len"].clone())
+    end.record(stream)
+    torch.cuda.synchronize()
+    clock_rec = clocks.stop()
+    barrier(ws)
+    assert fc.fc_get_error() == "FC_OK"
+    t_max = max_over_ranks(start.elapsed_time(end), ws)
+    stage = {nm: statistics.mean(a.elapsed_time(b) for a, b in ev[nm]) for nm in names}
+    acc = torch.stack(accs).cpu().numpy()
+    # the forward's GEMM work (every row of the padded tree) and its attention
+    # share, from one more untimed forward with per-layer events
+    T = B * n_pad
+    per_layer = s.hidden * (s.H * s.D + 2 * s.Hkv * s.D) + s.H * s.D * s.hidden + s.hidden * 3 * s.inter
+    gemm_flops = 2.0 * T * (s.layers * per_layer + s.hidden * s.vocab)
+    t = loop.tree
+    aev = {"attn": []}
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record()
+    td.forward(t["tok"], t["n_nodes"], t["mask"], t["pos"], loop.kv_len_now, events=aev)
+    f1.record()
+    torch.cuda.synchronize()
+    fwd_ms = f0.elapsed_time(f1)
+    attn_ms = sum(a.elapsed_time(b) for a, b in aev["attn"])
+    peaks = load_peaks()
+    gemm_tflops = gemm_flops / ((fwd_ms - attn_ms) * 1e-3) / 1e12
+    return {"metric": METRIC, "value": weak_value(K, ws, t_max), "unit": UNIT, "n_gpus": ws, "steps": K, "warmup": W,
+            "ms_per_step": t_max / K, "higher_is_better": True, "scaling": "weak",
+            "dtype": "bf16 (fp32 accumulate) + u32 retrieval", "data": "synthetic (random-init weights)",
+            "config": {"workload": f"step loop verified by a random-init DeepSeek-Coder-1.3B-shaped decoder "
+                                   f"(24 x hidden 2048, 16 heads x 128, MLP 5504, vocab 32256), {B} sequences, "
+                                   f"64-node trees, cache {kv0}, two-source store 100M + 5M",
+                       "batch_per_gpu": B, "n_pad": n_pad, "kv_len0": kv0},
+            "stages_ms_per_step": stage,
+            "tokens_per_s": float((acc + 1).sum() / (t_max * 1e-3) * ws),
+            "mean_accepted": float(acc.mean()),
+            "forward": {"ms": fwd_ms, "attention_ms": attn_ms, "gemm_and_rest_ms": fwd_ms - attn_ms,
+                        "gemm_tflops": gemm_tflops, "gemm_frac_of_sustained_bf16": gemm_tflops / peaks["tc_sustained"]},
+            "clocks": clock_rec}
+
+
 def main(argv=None):
     args = parse_args(argv)
     rank, ws, local = dist_setup(args.gpus)
@@ -1104,6 +1201,8 @@ def main(argv=None):
         out = run_algorithm1(args, rank, ws, local)
     elif args.mode == "cache":
         out = run_cache(args, rank, ws, local)
+    elif args.mode == "decoder":
+        out = run_decoder(args, rank, ws, local)
     else:
         out = run_ours(args, rank, ws, local)
     if rank == 0 and out is not None:

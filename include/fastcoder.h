@@ -424,6 +424,43 @@ fc_status fc_tree_attn_rope(const void* d_q, const void* d_k_cache, const void* 
                             void* d_out, void* d_ws, size_t ws_bytes, fc_stream s);
 
 /* ------------------------------------------------------------------------
+ * The decoder around the tree attention (Section IV-D: the target model
+ * verifies every draft in one forward).  Building blocks of a LLaMA-family
+ * decoder like the paper's models: embedding, residual add + RMSNorm, the
+ * SiLU-gated MLP activation, the head-major layout of the tree's keys
+ * (rotated) and values, and plain GEMMs.  bf16 tensors, row-major, 16-byte
+ * aligned; fp32 arithmetic inside.
+ * ------------------------------------------------------------------------ */
+/* Workspace bytes fc_gemm_bf16 can use (a caller-owned buffer; NULL works,
+ * possibly slower). */
+size_t fc_gemm_workspace(void);
+
+/* C[M][N] = A[M][K] B[K][N] (cuBLASLt, fp32 accumulate).  N and K multiples
+ * of 8.  Not part of the paper's method: plain library GEMMs. */
+fc_status fc_gemm_bf16(const void* d_a, const void* d_b, void* d_c, int M, int N, int K, void* d_ws,
+                       size_t ws_bytes, fc_stream s);
+
+/* out[t][:] = table[tok[t]][:]; an id >= vocab (tree padding) gives zeros.
+ * hidden a multiple of 8. */
+fc_status fc_embed(const uint32_t* d_tok, int n, const void* d_table, int vocab, int hidden, void* d_out,
+                   fc_stream s);
+
+/* Per row: if d_r, x += r (in place, rounded to bf16: the residual stream);
+ * then out = x / sqrt(mean(x^2) + eps) * w.  dim a multiple of 8. */
+fc_status fc_add_rmsnorm(void* d_x, const void* d_r, const void* d_w, void* d_out, int rows, int dim,
+                         float eps, fc_stream s);
+
+/* out[r][j] = silu(gu[r][j]) * gu[r][inter + j], silu(z) = z / (1 + e^-z):
+ * gu holds the gate columns, then the up columns. */
+fc_status fc_silu_mul(const void* d_gu, void* d_out, int rows, int inter, fc_stream s);
+
+/* Node-major projection rows in[(b * n_pad + i) * in_stride + h * D + d]
+ * (elements) to head-major out[b][h][i][d], rotated as fc_rope by
+ * d_pos[b][i] when base > 0, copied when base <= 0 (the values). */
+fc_status fc_rope_heads(const void* d_in, int in_stride, void* d_out, int batch, int n_pad, int heads, int D,
+                        const int32_t* d_pos, float base, fc_stream s);
+
+/* ------------------------------------------------------------------------
  * Acceptance (Section IV-D: every correct token from the start is accepted,
  * everything after the first error rejected; Eq. 7 counts tokens per step).
  * ------------------------------------------------------------------------ */

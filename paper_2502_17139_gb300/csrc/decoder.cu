@@ -1,0 +1,307 @@
+// The pieces of a decoder forward around the tree attention (Section IV-D:
+// the target model verifies every draft in one forward), for a LLaMA-family
+// model like the paper's: token embedding, residual add + RMSNorm, the
+// SiLU-gated MLP's activation, the head-major layout of the tree's keys
+// (rotated) and values, and plain GEMMs through cuBLASLt.
+//
+//   * fc_gemm_bf16: C[M][N] = A[M][K] B[K][N], row-major bf16, fp32
+//     accumulate.  Row-major C = A B is column-major C^T = B^T A^T, so B's
+//     memory is cuBLASLt's first operand.  The heuristic's algorithm is cached
+//     per shape.
+//   * k_embed: one row per warp; ids >= vocab (tree padding) embed as zeros.
+//   * k_add_rmsnorm: one row per warp; x += r is rounded to bf16 (the
+//     residual stream), then out = x / sqrt(mean(x^2) + eps) * w in fp32.
+//   * k_silu_mul: out = silu(gate) * up, fp32 math.
+//   * k_rope_heads: node-major projection rows -> head-major [B][heads][n][D],
+//     rotated by position (the rotation of tree_attn.cu) or copied.
+#include <cublasLt.h>
+
+#include <algorithm>
+#include <cmath>
+
+#include <map>
+#include <mutex>
+#include <tuple>
+
+#include "fc_common.cuh"
+
+FC_DEFINE_ERROR_WORD(dec)
+
+namespace {
+
+constexpr int ROWS_PER_BLOCK = 8;  // one warp per row
+
+__global__ void k_embed(const uint32_t* __restrict__ tok, int n, const uint4* __restrict__ table, int vocab,
+                        int hidden, uint4* __restrict__ out) {
+  const int row = blockIdx.x * ROWS_PER_BLOCK + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= n) return;
+  const uint32_t t = tok[row];
+  const int w = hidden / 8;
+  uint4* o = out + (size_t)row * w;
+  if (t >= (uint32_t)vocab) {
+    for (int c = lane; c < w; c += 32) o[c] = make_uint4(0, 0, 0, 0);
+    return;
+  }
+  const uint4* src = table + (size_t)t * w;
+  for (int c = lane; c < w; c += 32) o[c] = src[c];
+}
+
+__device__ __forceinline__ float2 bf2f(uint32_t v) {
+  return __bfloat1622float2(*reinterpret_cast<__nv_bfloat162*>(&v));
+}
+__device__ __forceinline__ uint32_t f2bf(float a, float b) {
+  __nv_bfloat162 r = __float22bfloat162_rn(make_float2(a, b));
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+
+__global__ void k_add_rmsnorm(uint4* __restrict__ x, const uint4* __restrict__ r, const uint4* __restrict__ w,
+                              uint4* __restrict__ out, int rows, int dim, float eps) {
+  const int row = blockIdx.x * ROWS_PER_BLOCK + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const int cw = dim / 8;
+  uint4* xr = x + (size_t)row * cw;
+  const uint4* rr = r ? r + (size_t)row * cw : nullptr;
+  float ss = 0.f;
+  for (int c = lane; c < cw; c += 32) {
+    uint4 v = xr[c];
+    if (rr) {  // the residual stream in bf16: x + r, rounded
+      const uint4 a = rr[c];
+      uint32_t* vv = &v.x;
+      const uint32_t* aa = &a.x;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 xv = bf2f(vv[q]), av = bf2f(aa[q]);
+        vv[q] = f2bf(xv.x + av.x, xv.y + av.y);
+      }
+      xr[c] = v;
+    }
+    const uint32_t* vv = &v.x;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float2 f = bf2f(vv[q]);
+      ss = fmaf(f.x, f.x, fmaf(f.y, f.y, ss));
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
+  const float inv = rsqrtf(ss / (float)dim + eps);
+  uint4* orow = out + (size_t)row * cw;
+  for (int c = lane; c < cw; c += 32) {
+    const uint4 v = xr[c], g = w[c];
+    const uint32_t* vv = &v.x;
+    const uint32_t* gg = &g.x;
+    uint4 res;
+    uint32_t* rv = &res.x;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float2 f = bf2f(vv[q]), gw = bf2f(gg[q]);
+      rv[q] = f2bf(f.x * inv * gw.x, f.y * inv * gw.y);
+    }
+    orow[c] = res;
+  }
+}
+
+__global__ void k_silu_mul(const uint4* __restrict__ gu, uint4* __restrict__ out, int rows, int inter) {
+  const int cw = inter / 8;
+  const size_t items = (size_t)rows * cw;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < items; e += (size_t)gridDim.x * blockDim.x) {
+    const size_t row = e / cw;
+    const int c = (int)(e - row * cw);
+    const uint4 g = gu[row * 2 * cw + c], u = gu[row * 2 * cw + cw + c];
+    const uint32_t* gg = &g.x;
+    const uint32_t* uu = &u.x;
+    uint4 res;
+    uint32_t* rv = &res.x;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float2 a = bf2f(gg[q]), b = bf2f(uu[q]);
+      rv[q] = f2bf(a.x / (1.f + __expf(-a.x)) * b.x, a.y / (1.f + __expf(-a.y)) * b.y);
+    }
+    out[e] = res;
+  }
+}
+
+// ---- the rotation of tree_attn.cu (rotate-half pairing, f_i as a float
+// pair from fp64, Cody-Waite reduction of the angle, MUFU sine/cosine)
+constexpr int ROPE_MAX_HALF = 512;
+
+__device__ __forceinline__ void rope_sincos(float pos, float2 f, float& sn, float& cs) {
+  const float a_hi = pos * f.x;
+  const float a_lo = fmaf(pos, f.y, fmaf(pos, f.x, -a_hi));
+  const float k = rintf(a_hi * 0.15915493667125702f);
+  float r = fmaf(-k, 6.2831854820251465f, a_hi);
+  r = fmaf(-k, -1.7484555314695172e-07f, r) + a_lo;
+  __sincosf(r, &sn, &cs);
+}
+
+// node-major rows in[(b * n_pad + i) * stride + h * D + d] -> head-major
+// out[((b * heads + h) * n_pad + i) * D + d], rotated by pos[b][i] when
+// rotate != 0 (a negative position is copied unrotated).  One thread per pair
+// of partner 16-byte chunks (dimensions 8c..8c+7 and D/2 + 8c..).
+__global__ void k_rope_heads(const __nv_bfloat16* __restrict__ in, int stride, __nv_bfloat16* __restrict__ out,
+                             int B, int n_pad, int heads, int D, const int32_t* __restrict__ pos, int rotate,
+                             double nl2f) {
+  __shared__ float2 tab[ROPE_MAX_HALF];
+  if (rotate) {
+    for (int i = threadIdx.x; i < D / 2; i += blockDim.x) {
+      const double f = exp2((double)i * nl2f);
+      const float hi = (float)f;
+      tab[i] = make_float2(hi, (float)(f - (double)hi));
+    }
+  }
+  __syncthreads();
+  const int ch = D / 16;
+  const size_t items = (size_t)B * n_pad * heads * ch;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < items; e += (size_t)gridDim.x * blockDim.x) {
+    const int c = (int)(e % ch);
+    size_t t = e / ch;
+    const int h = (int)(t % heads);
+    t /= heads;
+    const int i = (int)(t % n_pad);
+    const int b = (int)(t / n_pad);
+    const uint4* src = reinterpret_cast<const uint4*>(in + ((size_t)b * n_pad + i) * stride + (size_t)h * D);
+    uint4 lo = src[c], hi = src[c + ch];
+    const int p = rotate ? pos[(size_t)b * n_pad + i] : -1;
+    if (p >= 0) {
+      uint32_t* l = &lo.x;
+      uint32_t* hh = &hi.x;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 xl = bf2f(l[q]), xh = bf2f(hh[q]);
+        float s0, c0, s1, c1;
+        rope_sincos((float)p, tab[8 * c + 2 * q], s0, c0);
+        rope_sincos((float)p, tab[8 * c + 2 * q + 1], s1, c1);
+        l[q] = f2bf(xl.x * c0 - xh.x * s0, xl.y * c1 - xh.y * s1);
+        hh[q] = f2bf(xh.x * c0 + xl.x * s0, xh.y * c1 + xl.y * s1);
+      }
+    }
+    uint4* dst = reinterpret_cast<uint4*>(out + (((size_t)b * heads + h) * n_pad + i) * D);
+    dst[c] = lo;
+    dst[c + ch] = hi;
+  }
+}
+
+// ---- cuBLASLt
+struct Lt {
+  std::mutex mu;
+  cublasLtHandle_t h = nullptr;
+  std::map<std::tuple<int, int, int, size_t>, cublasLtMatmulAlgo_t> algos;
+};
+Lt& lt() {
+  static Lt s;
+  return s;
+}
+
+bool aligned16(const void* p) { return reinterpret_cast<uintptr_t>(p) % 16 == 0; }
+
+}  // namespace
+
+extern "C" size_t fc_gemm_workspace(void) { return (size_t)32 << 20; }
+
+extern "C" fc_status fc_gemm_bf16(const void* d_a, const void* d_b, void* d_c, int M, int N, int K, void* d_ws,
+                                  size_t ws_bytes, fc_stream stream) {
+  if (M < 0 || N < 1 || K < 1) return FC_ERR_INVALID_ARG;
+  if (M == 0) return FC_OK;
+  if (!d_a || !d_b || !d_c) return FC_ERR_INVALID_ARG;
+  if (!aligned16(d_a) || !aligned16(d_b) || !aligned16(d_c) || (d_ws && !aligned16(d_ws))) return FC_ERR_INVALID_ARG;
+  if (N % 8 || K % 8) return FC_ERR_UNSUPPORTED;
+  Lt& s = lt();
+  std::lock_guard<std::mutex> g(s.mu);
+  if (!s.h && cublasLtCreate(&s.h) != CUBLAS_STATUS_SUCCESS) return FC_ERR_CUDA;
+  const size_t ws = d_ws ? ws_bytes : 0;
+  cublasLtMatmulDesc_t op = nullptr;
+  cublasLtMatrixLayout_t lb = nullptr, la = nullptr, lc = nullptr;
+  fc_status st = FC_OK;
+  // column-major: C^T (N x M, ld N) = B^T (N x K, ld N) * A^T (K x M, ld K)
+  if (cublasLtMatmulDescCreate(&op, CUBLAS_COMPUTE_32F, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS ||
+      cublasLtMatrixLayoutCreate(&lb, CUDA_R_16BF, N, K, N) != CUBLAS_STATUS_SUCCESS ||
+      cublasLtMatrixLayoutCreate(&la, CUDA_R_16BF, K, M, K) != CUBLAS_STATUS_SUCCESS ||
+      cublasLtMatrixLayoutCreate(&lc, CUDA_R_16BF, N, M, N) != CUBLAS_STATUS_SUCCESS) {
+    st = FC_ERR_CUDA;
+  }
+  cublasLtMatmulAlgo_t algo;
+  if (st == FC_OK) {
+    auto key = std::make_tuple(M, N, K, ws);
+    auto it = s.algos.find(key);
+    if (it != s.algos.end()) {
+      algo = it->second;
+    } else {
+      cublasLtMatmulPreference_t pref = nullptr;
+      cublasLtMatmulHeuristicResult_t res;
+      int n_res = 0;
+      if (cublasLtMatmulPreferenceCreate(&pref) != CUBLAS_STATUS_SUCCESS ||
+          cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES, &ws, sizeof ws) !=
+              CUBLAS_STATUS_SUCCESS ||
+          cublasLtMatmulAlgoGetHeuristic(s.h, op, lb, la, lc, lc, pref, 1, &res, &n_res) != CUBLAS_STATUS_SUCCESS ||
+          n_res < 1) {
+        st = FC_ERR_UNSUPPORTED;
+      } else {
+        algo = res.algo;
+        s.algos[key] = algo;
+      }
+      if (pref) cublasLtMatmulPreferenceDestroy(pref);
+    }
+  }
+  if (st == FC_OK) {
+    const float one = 1.f, zero = 0.f;
+    if (cublasLtMatmul(s.h, op, &one, d_b, lb, d_a, la, &zero, d_c, lc, d_c, lc, &algo, d_ws, ws,
+                       static_cast<cudaStream_t>(stream)) != CUBLAS_STATUS_SUCCESS)
+      st = FC_ERR_CUDA;
+  }
+  if (lc) cublasLtMatrixLayoutDestroy(lc);
+  if (la) cublasLtMatrixLayoutDestroy(la);
+  if (lb) cublasLtMatrixLayoutDestroy(lb);
+  if (op) cublasLtMatmulDescDestroy(op);
+  return st;
+}
+
+extern "C" fc_status fc_embed(const uint32_t* d_tok, int n, const void* d_table, int vocab, int hidden, void* d_out,
+                              fc_stream stream) {
+  if (n < 0 || vocab < 1 || hidden < 8 || hidden % 8) return FC_ERR_INVALID_ARG;
+  if (n == 0) return FC_OK;
+  if (!d_tok || !d_table || !d_out || !aligned16(d_table) || !aligned16(d_out)) return FC_ERR_INVALID_ARG;
+  k_embed<<<(n + ROWS_PER_BLOCK - 1) / ROWS_PER_BLOCK, ROWS_PER_BLOCK * 32, 0, static_cast<cudaStream_t>(stream)>>>(
+      d_tok, n, static_cast<const uint4*>(d_table), vocab, hidden, static_cast<uint4*>(d_out));
+  return FC_CHECK_LAUNCH();
+}
+
+extern "C" fc_status fc_add_rmsnorm(void* d_x, const void* d_r, const void* d_w, void* d_out, int rows, int dim,
+                                    float eps, fc_stream stream) {
+  if (rows < 0 || dim < 8 || dim % 8 || !(eps >= 0.f)) return FC_ERR_INVALID_ARG;
+  if (rows == 0) return FC_OK;
+  if (!d_x || !d_w || !d_out || !aligned16(d_x) || !aligned16(d_w) || !aligned16(d_out) || (d_r && !aligned16(d_r)))
+    return FC_ERR_INVALID_ARG;
+  k_add_rmsnorm<<<(rows + ROWS_PER_BLOCK - 1) / ROWS_PER_BLOCK, ROWS_PER_BLOCK * 32, 0,
+                  static_cast<cudaStream_t>(stream)>>>(static_cast<uint4*>(d_x), static_cast<const uint4*>(d_r),
+                                                       static_cast<const uint4*>(d_w), static_cast<uint4*>(d_out),
+                                                       rows, dim, eps);
+  return FC_CHECK_LAUNCH();
+}
+
+extern "C" fc_status fc_silu_mul(const void* d_gu, void* d_out, int rows, int inter, fc_stream stream) {
+  if (rows < 0 || inter < 8 || inter % 8) return FC_ERR_INVALID_ARG;
+  if (rows == 0) return FC_OK;
+  if (!d_gu || !d_out || !aligned16(d_gu) || !aligned16(d_out)) return FC_ERR_INVALID_ARG;
+  const size_t items = (size_t)rows * (inter / 8);
+  const unsigned blocks = (unsigned)std::min<size_t>((items + 255) / 256, 152 * 32);
+  k_silu_mul<<<blocks, 256, 0, static_cast<cudaStream_t>(stream)>>>(static_cast<const uint4*>(d_gu),
+                                                                    static_cast<uint4*>(d_out), rows, inter);
+  return FC_CHECK_LAUNCH();
+}
+
+extern "C" fc_status fc_rope_heads(const void* d_in, int in_stride, void* d_out, int batch, int n_pad, int heads, int D,
+                                   const int32_t* d_pos, float base, fc_stream stream) {
+  if (batch < 0 || n_pad < 1 || heads < 1 || D < 16 || D > 1024 || D % 16 || in_stride < heads * D ||
+      in_stride % 8)
+    return FC_ERR_INVALID_ARG;
+  const bool rotate = base > 0.f;
+  if (rotate && !std::isfinite(base)) return FC_ERR_INVALID_ARG;
+  if (batch == 0) return FC_OK;
+  if (!d_in || !d_out || (rotate && !d_pos) || !aligned16(d_in) || !aligned16(d_out)) return FC_ERR_INVALID_ARG;
+  const size_t items = (size_t)batch * n_pad * heads * (D / 16);
+  const unsigned blocks = (unsigned)std::min<size_t>((items + 255) / 256, 152 * 16);
+  k_rope_heads<<<blocks, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+      static_cast<const __nv_bfloat16*>(d_in), in_stride, static_cast<__nv_bfloat16*>(d_out), batch, n_pad, heads, D,
+      d_pos, rotate ? 1 : 0, rotate ? -2.0 * std::log2((double)base) / D : 0.0);
+  return FC_CHECK_LAUNCH();
+}

@@ -7,6 +7,7 @@ extern "C" unsigned int fc_take_error_tree(cudaStream_t s);
 extern "C" unsigned int fc_take_error_step(cudaStream_t s);
 extern "C" unsigned int fc_take_error_attn(cudaStream_t s);
 extern "C" unsigned int fc_take_error_cache(cudaStream_t s);
+extern "C" unsigned int fc_take_error_dec(cudaStream_t s);
 
 extern "C" const char* fc_status_string(fc_status s) {
   switch (s) {
@@ -28,7 +29,8 @@ extern "C" fc_status fc_get_error(fc_stream stream) {
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (cudaStreamSynchronize(s) != cudaSuccess) return FC_ERR_CUDA;
   unsigned int e = fc_take_error_sa(s) | fc_take_error_ret(s) | fc_take_error_tree(s) | fc_take_error_step(s) |
-                   fc_take_error_attn(s) | fc_take_error_cache(s);
+                   fc_take_error_attn(s) | fc_take_error_cache(s) |
+                   fc_take_error_dec(s);
   if (e & FC_EBIT_INTERNAL) return FC_ERR_INTERNAL;
   if (e & FC_EBIT_TIMEOUT) return FC_ERR_TIMEOUT;
   if (e & FC_EBIT_CAPACITY) return FC_ERR_CAPACITY;

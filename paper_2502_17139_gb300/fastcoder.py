@@ -53,7 +53,8 @@ EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build
            "fc_datastore_build_noalloc",
            "fc_retrieve", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
-           "fc_missing_insert", "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
+           "fc_missing_insert", "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_embed",
+           "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
 
 
 def _load():
@@ -91,6 +92,12 @@ def _load():
                                    vp]),
         "fc_tree_attn_workspace": (sz, [i32, i32, i32, i32]),
         "fc_rope": (C.c_int, [vp, vp, i32, i32, i32, i32, i32, vp, C.c_float, vp]),
+        "fc_gemm_workspace": (sz, []),
+        "fc_gemm_bf16": (C.c_int, [vp, vp, vp, i32, i32, i32, vp, sz, vp]),
+        "fc_embed": (C.c_int, [vp, i32, vp, i32, i32, vp, vp]),
+        "fc_add_rmsnorm": (C.c_int, [vp, vp, vp, vp, i32, i32, C.c_float, vp]),
+        "fc_silu_mul": (C.c_int, [vp, vp, i32, i32, vp]),
+        "fc_rope_heads": (C.c_int, [vp, i32, vp, i32, i32, i32, i32, vp, C.c_float, vp]),
         "fc_tree_attn_rope": (C.c_int, [vp, vp, vp, i32, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, C.c_float, vp,
                                         C.c_float, vp, vp, sz, vp]),
         "fc_tree_attn_parts": (C.c_int, [i32, i32, i32, i32, i32, sz]),
@@ -458,6 +465,62 @@ def fc_tree_attn_rope(q, k_cache, v_cache, kv_len, k_tree_rot, v_tree, mask, n_n
         _ptr(n_nodes), B, Np, H, Hkv, D, sc, _ptr(pos), C.c_float(rope_base), _ptr(o), _ptr(workspace), ws_bytes,
         _stream()))
     return o
+
+
+# ------------------------------------------------------- decoder blocks
+_GEMM_WS = {}
+
+
+def gemm_workspace(device):
+    key = str(device)
+    if key not in _GEMM_WS:
+        _GEMM_WS[key] = torch.empty(int(LIB.fc_gemm_workspace()), dtype=torch.uint8, device=device)
+    return _GEMM_WS[key]
+
+
+def fc_gemm_bf16(a, b, out=None):
+    """a [M, K] @ b [K, N] (bf16, row-major) -> [M, N] bf16."""
+    _need(a, torch.bfloat16, "a")
+    _need(b, torch.bfloat16, "b")
+    M, K = a.shape
+    K2, N = b.shape
+    if K != K2:
+        raise ValueError("inner dimensions differ")
+    o = out if out is not None else torch.empty((M, N), dtype=torch.bfloat16, device=a.device)
+    ws = gemm_workspace(a.device)
+    _check("fc_gemm_bf16", LIB.fc_gemm_bf16(_ptr(a), _ptr(b), _ptr(o), M, N, K, _ptr(ws), ws.numel(), _stream()))
+    return o
+
+
+def fc_embed(tok, table, out):
+    _need(tok, torch.int32, "tok")
+    vocab, hidden = table.shape
+    _check("fc_embed", LIB.fc_embed(_ptr(tok), tok.numel(), _ptr(table), vocab, hidden, _ptr(out), _stream()))
+    return out
+
+
+def fc_add_rmsnorm(x, r, w, out, eps=1e-6):
+    """x += r (if r is not None), out = rmsnorm(x) * w; x, r, out [rows, dim]."""
+    rows, dim = x.shape
+    _check("fc_add_rmsnorm", LIB.fc_add_rmsnorm(_ptr(x), _ptr(r), _ptr(w), _ptr(out), rows, dim, C.c_float(eps),
+                                                _stream()))
+    return out
+
+
+def fc_silu_mul(gu, out):
+    rows, two_inter = gu.shape
+    _check("fc_silu_mul", LIB.fc_silu_mul(_ptr(gu), _ptr(out), rows, two_inter // 2, _stream()))
+    return out
+
+
+def fc_rope_heads(x, col0, stride, out, B, n_pad, heads, D, pos, base):
+    """Node-major rows of x (row stride ``stride`` elements, head h at column
+    col0 + h*D) -> head-major out [B, heads, n_pad, D], rotated by pos when
+    base > 0."""
+    ptr = C.c_void_p(x.data_ptr() + col0 * x.element_size())
+    _check("fc_rope_heads", LIB.fc_rope_heads(ptr, stride, _ptr(out), B, n_pad, heads, D, _ptr(pos), C.c_float(base),
+                                              _stream()))
+    return out
 
 
 # ---------------------------------------------------------- accept / append

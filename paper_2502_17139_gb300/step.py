@@ -30,14 +30,18 @@ from . import fastcoder as fc
 class StepLoop:
     def __init__(self, sources, ctx, ctx_len, p, node_budget, n_pad, src_weight, H, Hkv, D, kv_cap, kv_len0, vocab,
                  cache_capacity=1 << 14, device="cuda", k_cache=None, v_cache=None, seq_cache=None,
-                 rope_base=None):
+                 rope_base=None, decoder=None):
         """seq_cache: None, or a dict with capacity, min_size, chunk, ctx_keep
         (the CACHE), missing_capacity (M) and weight (the CACHE slot's tree
         weight); it replaces the replay cache.  rope_base: None (q and the
         tree keys arrive rotated), or the RoPE base: step() then takes them
         unrotated, the tree keys are rotated once by their node positions
         (fc_rope) for the attention and the cache append, and the queries are
-        rotated inside the attention kernel (fc_tree_attn_rope)."""
+        rotated inside the attention kernel (fc_tree_attn_rope).  decoder: None,
+        or a decoder.TreeDecoder: the verification is then its forward over the
+        tree (step()'s q, k_tree, v_tree, plen and rtok are unused), greedy
+        acceptance from its logits (fc_argmax_accept), and the accepted path
+        appended to every layer's cache."""
         self.sources, self.p, self.node_budget, self.n_pad = sources, p, node_budget, n_pad
         self.src_weight = list(src_weight)
         self.H, self.Hkv, self.D, self.kv_cap, self.vocab = H, Hkv, D, kv_cap, vocab
@@ -69,6 +73,7 @@ class StepLoop:
         self.v_cache = v_cache if v_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         self.attn_out = torch.empty((B, n_pad, H, D), dtype=torch.bfloat16, device=device)
         self.rope_base = rope_base
+        self.decoder = decoder
         self.k_tree_rot = (torch.empty((B, Hkv, n_pad, D), dtype=torch.bfloat16, device=device)
                            if rope_base is not None else None)
         self.cache = fc.RetrievalCache(cache_capacity, S, p, device) if cache_capacity and not self.seq else None
@@ -115,6 +120,10 @@ class StepLoop:
                          out=self.tree)
         if "tree" in ev:
             ev["tree"][1].record()
+        if self.decoder is not None:
+            self._verify_with_decoder(c, n, ev)
+            self.cur = n
+            return
         if self.rope_base is not None:
             k_tree = fc.fc_rope(k_tree, self.tree["pos"], self.rope_base, layout=1, out=self.k_tree_rot)
         if attention:
@@ -145,6 +154,24 @@ class StepLoop:
         if "tail" in ev:
             ev["tail"][1].record()
         self.cur = n
+
+    def _verify_with_decoder(self, c, n, ev):
+        t = self.tree
+        if "attn" in ev:
+            ev["attn"][0].record()
+        logits = self.decoder.forward(t["tok"], t["n_nodes"], t["mask"], t["pos"], self.kv_len[c])
+        if "attn" in ev:
+            ev["attn"][1].record()
+        if "tail" in ev:
+            ev["tail"][0].record()
+        fc.fc_argmax_accept(logits, t["tok"], t["parent"], t["n_nodes"], self.path_cap,
+                            out=dict(self.acc, argmax=self.argmax))
+        self.decoder.append(self.acc, t["tok"], self.kv_len[c], self.kv_len[n], self.ctx, self.ctx_len[c],
+                            self.ctx_len[n], self.root)
+        if self.seq:
+            fc.fc_cache_update(self.seq_cache, self.ctx, self.ctx_len[c], self.ctx_len[n], self.acc["acc_len"])
+        if "tail" in ev:
+            ev["tail"][1].record()
 
     def reset(self):
         """Back to the initial contexts and cache lengths.  The replay cache

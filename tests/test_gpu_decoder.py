@@ -1,0 +1,190 @@
+"""GPU parity for the decoder forward over a draft tree (paper_2502_17139_gb300/
+decoder.py) against the fp64 oracle (oracle/decoder.py), on seeded
+random-init weights of a small LLaMA-family shape.
+
+The GPU keeps bf16 between operations (fp32 inside each), so values are
+compared within tolerances that allow that rounding to accumulate over a few
+layers: the building blocks to one or two bf16 roundings, logits and the
+rotated keys and values to a max-abs of 0.06 at unit scale.  Greedy
+predictions must agree wherever the oracle's top-2 logit gap exceeds 0.25.
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2502_17139_gb300.synth as synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def fc():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2502_17139_gb300 import build
+    build.build()
+    import paper_2502_17139_gb300.fastcoder as fcm
+    return fcm
+
+
+@pytest.fixture(scope="module")
+def dec(orc):
+    from oracle import decoder
+    return decoder
+
+
+def dev(a):
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint32:
+        a = a.view(np.int32)
+    return torch.from_numpy(a.copy()).cuda()
+
+
+def f64(t):
+    return t.float().cpu().numpy().astype(np.float64)
+
+
+def test_blocks(fc, dec):
+    rng = np.random.default_rng(7000)
+    torch.manual_seed(7001)
+    # GEMM, rows not a multiple of any tile
+    a = torch.randn((777, 256)).to(torch.bfloat16).cuda()
+    b = (torch.randn((256, 392)) / 16).to(torch.bfloat16).cuda()
+    c = fc.fc_gemm_bf16(a, b)
+    ref = f64(a) @ f64(b)
+    assert np.abs(f64(c) - ref).max() <= 2.0 ** -7 * np.abs(ref).max()
+    # embedding with padding ids
+    table = torch.randn((300, 256)).to(torch.bfloat16).cuda()
+    ids = rng.integers(0, 300, 64).astype(np.uint32)
+    ids[[3, 9]] = 0xFFFFFFFF
+    out = torch.empty((64, 256), dtype=torch.bfloat16, device="cuda")
+    fc.fc_embed(dev(ids), table, out)
+    want = f64(table)[np.minimum(ids, 299).astype(np.int64)]
+    want[[3, 9]] = 0
+    assert np.array_equal(f64(out), want)
+    # residual add + RMSNorm
+    x = torch.randn((50, 264)).to(torch.bfloat16).cuda()
+    r = torch.randn((50, 264)).to(torch.bfloat16).cuda()
+    w = (1 + 0.1 * torch.randn(264)).to(torch.bfloat16).cuda()
+    x0 = f64(x)
+    o = torch.empty_like(x)
+    fc.fc_add_rmsnorm(x, r, w, o, 1e-6)
+    xs = x0 + f64(r)
+    assert np.abs(f64(x) - xs).max() <= 2.0 ** -8 * np.abs(xs).max()
+    ref = dec.rmsnorm(f64(x), f64(w), 1e-6)
+    assert np.abs(f64(o) - ref).max() <= 2.0 ** -7 * np.abs(ref).max()
+    # SiLU * up
+    gu = torch.randn((40, 2 * 96)).to(torch.bfloat16).cuda()
+    act = torch.empty((40, 96), dtype=torch.bfloat16, device="cuda")
+    fc.fc_silu_mul(gu, act)
+    g = f64(gu)
+    ref = dec.silu(g[:, :96]) * g[:, 96:]
+    assert np.abs(f64(act) - ref).max() <= 2.0 ** -7 * np.abs(ref).max() + 1e-3
+    assert fc.fc_get_error() == "FC_OK"
+
+
+def test_rope_heads(fc, orc):
+    rng = np.random.default_rng(7100)
+    B, n_pad, Hkv, D = 2, 64, 3, 128
+    kv = torch.randn((B * n_pad, 2 * Hkv * D)).to(torch.bfloat16).cuda()
+    pos = rng.integers(0, 50000, (B, n_pad)).astype(np.int32)
+    pos[0, -2:] = -1
+    k = torch.empty((B, Hkv, n_pad, D), dtype=torch.bfloat16, device="cuda")
+    v = torch.empty_like(k)
+    fc.fc_rope_heads(kv, 0, 2 * Hkv * D, k, B, n_pad, Hkv, D, dev(pos), 10000.0)
+    fc.fc_rope_heads(kv, Hkv * D, 2 * Hkv * D, v, B, n_pad, Hkv, D, dev(pos), 0.0)
+    x = f64(kv).reshape(B, n_pad, 2, Hkv, D)
+    want_v = x[:, :, 1].transpose(0, 2, 1, 3)
+    assert np.array_equal(f64(v), want_v)
+    kk = x[:, :, 0].transpose(0, 2, 1, 3)
+    p = np.broadcast_to(pos[:, None, :], (B, Hkv, n_pad))
+    want_k = orc.rope(kk, np.maximum(p, 0), 10000.0)
+    want_k[p < 0] = kk[p < 0]
+    assert (np.abs(f64(k) - want_k) <= 2.0 ** -8 * np.abs(want_k) + 1e-5).all()
+
+
+SHAPES = [dict(hidden=256, layers=2, H=4, Hkv=2, inter=384, vocab=304),
+          dict(hidden=512, layers=2, H=4, Hkv=4, inter=768, vocab=1000)]
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=["gqa", "mha"])
+def test_decoder_forward_parity(fc, dec, orc, shape):
+    from paper_2502_17139_gb300.decoder import DecoderShape, TreeDecoder
+    s = DecoderShape(**shape)
+    cfg = dec.DecoderConfig(**shape)
+    Wt = synth.decoder_weights(s.hidden, s.layers, s.H, s.Hkv, s.D, s.inter, s.vocab, 77)
+    Wd = {k: v.cuda() for k, v in Wt.items() if k != "layers"}
+    Wd["layers"] = [{k: v.cuda() for k, v in Lw.items()} for Lw in Wt["layers"]]
+    tobits = lambda t: t.view(torch.int16).numpy().view(np.uint16)
+    Wb = {k: tobits(v) for k, v in Wt.items() if k != "layers"}
+    Wb["layers"] = [{k: tobits(v) for k, v in Lw.items()} for Lw in Wt["layers"]]
+    W = dec.widen_weights(Wb)
+    B, n_pad, cap = 3, 64, 80
+    rng = synth.rng_for(92)
+    tok = np.full((B, n_pad), 0xFFFFFFFF, np.uint32)
+    par = np.full((B, n_pad), -1, np.int32)
+    nn = np.array([30, 64, 1], np.int32)
+    for b in range(B):
+        t, p = synth.random_tree(rng, int(nn[b]), 8, 4, s.vocab)
+        tok[b, :nn[b]], par[b, :nn[b]] = t, p
+    kvl = np.array([50, 3, 80], np.int32)
+    m = orc.tree_mask(par, nn, kvl, n_pad)
+    caches = [(synth.randn_bf16((B, s.Hkv, cap, s.D), 900 + l, "cuda"),
+               synth.randn_bf16((B, s.Hkv, cap, s.D), 950 + l, "cuda")) for l in range(s.layers)]
+    kc = [f64(c[0]) for c in caches]
+    vc = [f64(c[1]) for c in caches]
+    td = TreeDecoder(s, Wd, B, n_pad, cap, caches=caches)
+    logits = td.forward(dev(tok), dev(nn), dev(m["mask"].view(np.int64)), dev(m["pos"]), dev(kvl))
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_OK"
+    ref, k_new, v_new = dec.forward(cfg, W, tok, par, nn, kvl, kc, vc, m["pos"])
+    got = f64(logits)
+    for b in range(B):
+        n = int(nn[b])
+        err = np.abs(got[b, :n] - ref[b, :n]).max()
+        assert err <= 0.06, (b, err)
+        top2 = np.sort(ref[b, :n], axis=1)[:, -2:]
+        clear = top2[:, 1] - top2[:, 0] > 0.25
+        assert (np.argmax(got[b, :n], 1)[clear] == np.argmax(ref[b, :n], 1)[clear]).all()
+        for l in range(s.layers):
+            gk = f64(td.k_rot[l])[b, :, :n].transpose(1, 0, 2)
+            gv = f64(td.v_heads[l])[b, :, :n].transpose(1, 0, 2)
+            assert np.abs(gk - k_new[l, b, :n]).max() <= 0.06
+            assert np.abs(gv - v_new[l, b, :n]).max() <= 0.06
+
+
+def test_decoder_step_loop(fc):
+    """The step loop verifying with the decoder: acceptance from its logits,
+    every layer's cache grows by acc_len + 1 rows, and those rows are the
+    tree's rotated keys and values along the accepted path."""
+    from paper_2502_17139_gb300.decoder import DecoderShape, TreeDecoder
+    from paper_2502_17139_gb300.step import StepLoop
+    s = DecoderShape(hidden=256, layers=2, H=4, Hkv=2, inter=384, vocab=synth.VOCAB)
+    Wt = synth.decoder_weights(s.hidden, s.layers, s.H, s.Hkv, s.D, s.inter, s.vocab, 78, device="cuda")
+    rng = synth.rng_for(75)
+    Tr, _ = synth.make_corpus(rng, 200_000, 1.3, synth.VOCAB, n_grams=500, len_range=(8, 64))
+    B, n_pad, kv0, steps = 4, 64, 20, 5
+    ctx, cl, _ = synth.make_contexts(rng, B, 128, 16, [Tr, None], [0.75, 0.25], 1.1, ctx_stride=128 + 12 * steps)
+    cap = kv0 + 12 * steps + 8
+    td = TreeDecoder(s, Wt, B, n_pad, cap)
+    srcs = [fc.fc_datastore_build(dev(Tr), synth.VOCAB)]
+    loop = StepLoop(srcs, ctx, cl, fc.params(16, 2, 16, 10, 4096), n_pad, n_pad, [1], s.H, s.Hkv, s.D, cap, kv0,
+                    synth.VOCAB, k_cache=td.k_cache[0], v_cache=td.v_cache[0], decoder=td, cache_capacity=0)
+    zeros = torch.zeros(B, dtype=torch.int32, device="cuda")
+    for st in range(steps):
+        kv_before = loop.kv_len_now.cpu().numpy().copy()
+        loop.step(None, None, None, zeros, zeros, None)
+        torch.cuda.synchronize()
+        assert fc.fc_get_error() == "FC_OK"
+        acc = loop.acc["acc_len"].cpu().numpy()
+        path = loop.acc["path"].cpu().numpy()
+        assert np.array_equal(loop.kv_len_now.cpu().numpy(), kv_before + acc + 1)
+        for l in range(s.layers):
+            kc = td.k_cache[l].cpu()
+            kr = td.k_rot[l].cpu()
+            vc = td.v_cache[l].cpu()
+            vh = td.v_heads[l].cpu()
+            for b in range(B):
+                for t in range(int(acc[b]) + 1):
+                    assert torch.equal(kc[b, :, kv_before[b] + t], kr[b, :, path[b, t]])
+                    assert torch.equal(vc[b, :, kv_before[b] + t], vh[b, :, path[b, t]])
