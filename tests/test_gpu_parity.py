@@ -290,6 +290,37 @@ def test_tree_handmade_on_gpu(fc):
     check_no_error(fc)
 
 
+@pytest.mark.parametrize("w", [(1, 1), (3, 1)])
+def test_all_occurrence_trie_within_cap(fc, orc, w):
+    """The trie over every retrieved continuation (the "top-k prefixes"
+    reading of Section III-A and Eq. 3's occurrence counts over all of R_r and
+    R_c): with max_occ <= 256 a source has at most 256 distinct
+    continuations, so top_k = max_occ keeps all of them and the GPU tree
+    equals the oracle's tree over its untruncated retrieval."""
+    rng = synth.rng_for(42)
+    Tr, _ = synth.make_corpus(rng, 60000, 1.3, 300, n_grams=300, len_range=(8, 40))
+    Tc, _ = synth.make_corpus(rng, 150000, 1.05, 300)
+    B, n_pad = 48, 128
+    ctx, cl, _ = synth.make_contexts(rng, B, 40, 16, [Tr, Tc, None], [0.5, 0.25, 0.25], 1.1, 300)
+    dsr, dsc = fc.fc_datastore_build(dev(Tr), 300), fc.fc_datastore_build(dev(Tc), 300)
+    cap, d = 256, 10
+    p = fc.params(16, 2, cap, d, cap)
+    g = fc.fc_retrieve([dsr, dsc], dev(ctx), dev(cl), p)
+    root = ctx[np.arange(B), cl - 1]
+    kvl = np.full(B, 700, np.int32)
+    wv = np.array(w, np.uint32)
+    gt = fc.fc_build_tree(g, wv, dev(root), dev(kvl), n_pad, n_pad)
+    res = [orc.retrieve(T, ctx, cl, 16, 2, 4096, d, cap) for T in (Tr, Tc)]
+    assert max(int(r["n_drafts"].max()) for r in res) > 64  # more distinct continuations than a top-64 keeps
+    assert all(int(r["n_drafts"].max()) <= cap for r in res)
+    for r in res:  # the untruncated lists, cut to the slot count (every draft fits)
+        for name in ("drafts", "draft_len", "count"):
+            r[name] = np.ascontiguousarray(r[name][:, :cap])
+    rt = orc.build_tree(res, wv, root, kvl, n_pad, n_pad)
+    compare_tree(gt, rt)
+    check_no_error(fc)
+
+
 def _random_trees(rng, B, n_pad, vocab=32256, full=False):
     tok = np.full((B, n_pad), PAD, np.uint32)
     par = np.full((B, n_pad), -1, np.int32)
