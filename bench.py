@@ -84,6 +84,8 @@ def parse_args(argv=None):
                          "benchmark line); retrieve: two-source retrieval alone for --batch queries (batch sweeps)")
     ap.add_argument("--nodes", type=int, default=128, help="attn mode: tree nodes per sequence")
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="step mode: skip timing the same steps replayed from CUDA graphs (two steps per graph)")
     ap.add_argument("--rope", action="store_true",
                     help="attn mode: unrotated queries, rotated in the kernel by node position (fc_tree_attn_rope)")
     ap.add_argument("--weights", type=str, default="1,1",
@@ -337,6 +339,13 @@ def run_ours(args, rank, ws, local):
     status = fc.fc_get_error()
     assert status == "FC_OK", status
     t_max = max_over_ranks(t_ms, ws)
+    graph_rec = None
+    if not args.no_graph:
+        try:
+            graph_rec = run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W, K)
+            assert fc.fc_get_error() == "FC_OK"
+        except Exception as e:  # reported, not fatal: the eager line stands
+            graph_rec = {"error": f"{type(e).__name__}: {e}"[:200]}
     attn_ms = [a.elapsed_time(b) for a, b in ev]
     ret_ms = [a.elapsed_time(b) for a, b in ev_ret]
     tree_ms = [a.elapsed_time(b) for a, b in ev_tree]
@@ -373,6 +382,7 @@ def run_ours(args, rank, ws, local):
         "metric": METRIC, "value": weak_value(K, ws, t_max), "unit": UNIT, "n_gpus": ws, "steps": K, "warmup": W,
         "ms_per_step": t_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16 attention (fp32 accumulate) + u32 retrieval", "data": "synthetic",
+        **({"graph": graph_rec} if graph_rec else {}),
         "config": {"workload": (WORKLOAD if args.scale == 1.0 else WORKLOAD + f" (scaled x{args.scale})")
                    + ("" if weights == [1, 1] else f", source weights alpha={weights[0]} beta={weights[1]}"),
                    "batch_per_gpu": B, "global_batch": B * ws, "kv_len0": kv0, "n_pad": n_pad,
@@ -397,6 +407,46 @@ def run_ours(args, rank, ws, local):
     if not args.no_cpu_baseline and rank == 0 and ws == 1:
         out["cpu_baseline"] = cpu_baseline(inp, cfg, kv0, out["avg_tree_nodes"], B)
     return out
+
+
+def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W, K):
+    """The same trajectory again, from the start, with every pair of steps
+    replayed from a CUDA graph: one graph per pair of pooled activations
+    (they read the pool tensors directly); a step's small draws are copied
+    into the graph's input buffers before each replay."""
+    import torch
+    if P % 2 or W % 2 or K % 2:
+        return {"skipped": "needs an even pool size, warm-up and step count"}
+    loop.reset()
+    B = hits_d.shape[1]
+    small = [(torch.empty_like(hits_d[0]), torch.empty_like(plen_d[0]), torch.empty_like(rtok_d[0])) for _ in range(2)]
+    # one eager pair first (workspaces and kernel attributes), then the captures
+    for s in range(2):
+        loop.step(q_pool[s % P], kt_pool[s % P], vt_pool[s % P], hits_d[s], plen_d[s], rtok_d[s])
+    graphs = {}
+    for j in range(0, P, 2):
+        ins = [(q_pool[j + t], kt_pool[j + t], vt_pool[j + t]) + small[t] for t in range(2)]
+        graphs[j] = loop.capture(ins)
+
+    def pair(s):
+        for t in range(2):
+            small[t][0].copy_(hits_d[s + t])
+            small[t][1].copy_(plen_d[s + t])
+            small[t][2].copy_(rtok_d[s + t])
+        graphs[s % P].replay()
+
+    for s in range(2, W, 2):
+        pair(s)
+    torch.cuda.synchronize()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record()
+    for i in range(0, K, 2):
+        pair(W + i)
+    end.record()
+    torch.cuda.synchronize()
+    ms = start.elapsed_time(end) / K
+    return {"ms_per_step": ms, "steps_per_s": 1e3 / ms, "graphs": len(graphs),
+            "note": "two steps per graph replay; the step's small draws copied in before each replay"}
 
 
 def replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K, weights=(1, 1)):

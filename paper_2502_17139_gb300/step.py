@@ -173,6 +173,21 @@ class StepLoop:
         if "tail" in ev:
             ev["tail"][1].record()
 
+    def capture(self, inputs, attention=True):
+        """Capture two consecutive steps into a CUDA graph.  ``inputs`` holds
+        two tuples (q, k_tree, v_tree, want_hit, plen, rtok) of device tensors
+        that the graph reads at every replay (update them in place between
+        replays).  Call with the loop at an even step, after one eager pair of
+        steps so that lazily made workspaces and kernel attributes exist.
+        Each replay advances the loop by two steps."""
+        if self.cur != 0:
+            raise RuntimeError("capture at an even step")
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            self.step(*inputs[0], attention=attention)
+            self.step(*inputs[1], attention=attention)
+        return g
+
     def reset(self):
         """Back to the initial contexts and cache lengths.  The replay cache
         keeps its entries (a replay of the same trajectory then hits it); the
