@@ -6,6 +6,11 @@
 * Retrieval and draft trees for every query on the GPU, compared bit-exactly
   with the oracle on a seeded sample of queries (the oracle scans the whole
   corpus once per query and source).
+* The decoder forward at DeepSeek-Coder 1.3B's layer width against the fp64
+  oracle on every node of two sequences.
+* Algorithm 1 on the default two-source store through properties that hold
+  at any size (served drafts and their counts recounted in the stores, no
+  longer match, missing-table keys absent from both corpora).
 """
 import numpy as np
 import pytest
@@ -122,3 +127,135 @@ def test_one_billion_tokens(fc, orc):
     rt = orc.build_tree([r], [1], root[sample], kvl[sample], cfg["node_budget"], cfg["n_pad"])
     compare_rows(gt, rt, sample)
     assert (g["match_len"].cpu().numpy() == 24).mean() > 0.9
+
+
+def test_decoder_full_width(fc, orc):
+    """The decoder forward at DeepSeek-Coder 1.3B's layer width (hidden 2048,
+    16 heads x 128, MLP 5504, vocab 32256; two layers of it) over 64-node
+    trees and 2048-token caches, the shapes the decoder bench runs, against the
+    fp64 oracle on every node of two sequences."""
+    from oracle import decoder as dec
+    from paper_2502_17139_gb300.decoder import DecoderShape, TreeDecoder
+    shape = dict(hidden=2048, layers=2, H=16, Hkv=16, inter=5504, vocab=32256)
+    s = DecoderShape(**shape)
+    cfg = dec.DecoderConfig(**shape)
+    Wt = synth.decoder_weights(s.hidden, s.layers, s.H, s.Hkv, s.D, s.inter, s.vocab, 79)
+    Wd = {k: v.cuda() for k, v in Wt.items() if k != "layers"}
+    Wd["layers"] = [{k: v.cuda() for k, v in Lw.items()} for Lw in Wt["layers"]]
+    tobits = lambda t: t.view(torch.int16).numpy().view(np.uint16)
+    Wb = {k: tobits(v) for k, v in Wt.items() if k != "layers"}
+    Wb["layers"] = [{k: tobits(v) for k, v in Lw.items()} for Lw in Wt["layers"]]
+    W = dec.widen_weights(Wb)
+    B, n_pad, kv, cap = 2, 64, 2048, 2056
+    rng = synth.rng_for(93)
+    tok = np.full((B, n_pad), 0xFFFFFFFF, np.uint32)
+    par = np.full((B, n_pad), -1, np.int32)
+    nn = np.array([24, 9], np.int32)
+    for b in range(B):
+        t, p = synth.random_tree(rng, int(nn[b]), 10, 4, s.vocab)
+        tok[b, :nn[b]], par[b, :nn[b]] = t, p
+    kvl = np.array([kv, kv - 777], np.int32)
+    m = orc.tree_mask(par, nn, kvl, n_pad)
+    caches = [(synth.randn_bf16((B, s.Hkv, cap, s.D), 960 + l, "cuda"),
+               synth.randn_bf16((B, s.Hkv, cap, s.D), 980 + l, "cuda")) for l in range(s.layers)]
+    f64 = lambda t: t.float().cpu().numpy().astype(np.float64)
+    kc = [f64(c[0]) for c in caches]
+    vc = [f64(c[1]) for c in caches]
+    td = TreeDecoder(s, Wd, B, n_pad, cap, caches=caches)
+    logits = td.forward(dev(tok), dev(nn), dev(m["mask"].view(np.int64)), dev(m["pos"]), dev(kvl))
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_OK"
+    ref, k_new, v_new = dec.forward(cfg, W, tok, par, nn, kvl, kc, vc, m["pos"])
+    got = f64(logits)
+    for b in range(B):
+        n = int(nn[b])
+        assert np.abs(got[b, :n] - ref[b, :n]).max() <= 0.06
+        top2 = np.sort(ref[b, :n], axis=1)[:, -2:]
+        clear = top2[:, 1] - top2[:, 0] > 0.25
+        assert (np.argmax(got[b, :n], 1)[clear] == np.argmax(ref[b, :n], 1)[clear]).all()
+        for l in range(s.layers):
+            assert np.abs(f64(td.k_rot[l])[b, :, :n].transpose(1, 0, 2) - k_new[l, b, :n]).max() <= 0.06
+            assert np.abs(f64(td.v_heads[l])[b, :, :n].transpose(1, 0, 2) - v_new[l, b, :n]).max() <= 0.06
+
+
+def test_algorithm1_full_size_properties(fc):
+    """Algorithm 1 on the default step loop's two-source store (100M + 5M
+    tokens, 32 sequences, l = 50, 20-token pieces, 8192-word CACHEs) after 100
+    steps, checked through properties that hold at any size: a draft the CACHE
+    returns follows the matched context suffix inside one stored sequence, as
+    often as its count says; no stored sequence holds a longer match; every
+    sampled key of the missing table occurs in neither corpus followed by a
+    token."""
+    import bench
+    from paper_2502_17139_gb300.step import StepLoop
+    steps = 100
+    inp = bench.make_inputs(1.0, 32, 0, steps + 1)
+    cfg, B = inp["cfg"], inp["B"]
+    d = cfg["draft_len"]
+    sources = [fc.fc_datastore_build(dev(T), synth.VOCAB) for T in inp["corpora"]]
+    p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], d, 4096)
+    seq = dict(capacity=8192, min_size=50, chunk=20, ctx_keep=16, missing_capacity=1 << 16, weight=1)
+    kv0 = 64
+    loop = StepLoop(sources, inp["ctx"], inp["cl"], p, 128, 128, [1, 1], 32, 8, 128, kv0 + (steps + 1) * (d + 1) + 8,
+                    kv0, synth.VOCAB, seq_cache=seq)
+    q = torch.zeros((B, 128, 32, 128), dtype=torch.bfloat16, device="cuda")
+    kt = torch.zeros((B, 8, 128, 128), dtype=torch.bfloat16, device="cuda")
+    zeros = torch.zeros(B, dtype=torch.int32, device="cuda")
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).cuda()
+    for s in range(steps):
+        loop.step(q, kt, kt, zeros, to_dev(inp["plen"][s]), to_dev(inp["rtok"][s]), attention=False)
+    # one more search on the final state, read back
+    S = 2
+    res = fc.retrieve_outputs(S + 1, B, p)
+    state = torch.empty(B, dtype=torch.int32, device="cuda")
+    fc.fc_cache_search(loop.seq_cache, loop.missing, loop.ctx, loop.ctx_len_now, p, S, res, state)
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_OK"
+    words = host_u32(loop.seq_cache.words)
+    meta = loop.seq_cache.meta.cpu().numpy()
+    ctx = host_u32(loop.ctx)
+    cl = loop.ctx_len_now.cpu().numpy()
+    st = state.cpu().numpy()
+    nd = res["n_drafts"][S].cpu().numpy()
+    ml = res["match_len"][S].cpu().numpy()
+    drafts = host_u32(res["drafts"][S])
+    dl = res["draft_len"][S].cpu().numpy()
+    cnt = res["count"][S].cpu().numpy()
+    SEP = 0xFFFFFFFE
+    assert (meta[:, 1] >= 50).any()
+    served = np.nonzero(st == 1)[0]
+    assert len(served) > 0
+    for b in served:
+        entries = np.split(words[b, :meta[b, 0]], np.nonzero(words[b, :meta[b, 0]] == SEP)[0] + 1)[:-1]
+        entries = [e[:-1] for e in entries]  # drop the separators
+        assert len(entries) == meta[b, 1]
+        n = int(ml[b])
+        suf = ctx[b, cl[b] - n:cl[b]].tolist()
+        # every occurrence of the matched suffix followed by a token, and its continuation
+        conts = {}
+        longer = False
+        for e in entries:
+            el = e.tolist()
+            for p0 in range(n, len(el)):
+                if el[p0 - n:p0] == suf:
+                    key = tuple(el[p0:p0 + d])
+                    conts[key] = conts.get(key, 0) + 1
+                    if n < min(16, cl[b]) and p0 > n and el[p0 - n - 1] == ctx[b, cl[b] - n - 1]:
+                        longer = True
+        assert not longer
+        if sum(conts.values()) > 4096:  # past max_occ only the smallest windows count
+            continue
+        assert nd[b] == min(len(conts), cfg["top_k"])
+        for t in range(nd[b]):
+            key = tuple(drafts[b, t, :dl[b, t]].tolist())
+            assert conts.get(key) == cnt[b, t], (b, t)
+        assert list(cnt[b, :nd[b]]) == sorted(cnt[b, :nd[b]], reverse=True)
+    # sampled missing-table keys: no occurrence followed by a token in either corpus
+    tab = loop.missing.table.cpu().numpy().view(np.uint32)
+    slots = tab[4:].reshape(-1, 3)
+    keys = slots[slots[:, 0] != 0][:, 1:]
+    assert len(keys) > 0
+    for k0, k1 in keys[synth.rng_for(94).permutation(len(keys))[:4]]:
+        for T in inp["corpora"]:
+            hit = (T[:-2] == k0) & (T[1:-1] == k1)
+            assert not hit.any()
