@@ -53,6 +53,14 @@ typedef void* fc_stream; /* cudaStream_t */
 #define FC_MAX_NODES 128      /* draft-tree nodes (root included) */
 #define FC_LCP_CAP 255        /* longest-common-prefix values are stored capped here */
 
+/* Self-test of failure detection (no counterpart in the paper): one CTA
+ * waits on an mbarrier phase with the kernels' bounded wait.  arrive != 0
+ * completes the phase first (FC_OK from fc_get_error); arrive == 0 leaves it
+ * pending, so the wait gives up after limit_cycles (1..4e9 SM cycles; a poll
+ * may add ~0.5 ms) and fc_get_error reports FC_ERR_TIMEOUT.  Nothing faults or
+ * hangs and the context stays usable. */
+fc_status fc_selftest_wait(int arrive, unsigned long long limit_cycles, fc_stream s);
+
 /* Human-readable name of a status code (static storage). */
 const char* fc_status_string(fc_status s);
 

@@ -362,3 +362,35 @@ extern "C" fc_status fc_synth_argmax(const uint32_t* d_tok, const int32_t* d_par
                                                                        d_rtok, vocab, d_argmax);
   return FC_CHECK_LAUNCH();
 }
+
+// ---------------------------------------------------------------------------
+// Self-test of the bounded waits (no counterpart in the paper): one CTA waits
+// on an mbarrier phase with the kernels' own bounded wait.  With arrive != 0
+// the phase completes first and the wait succeeds; with arrive == 0 nothing
+// ever arrives, the wait gives up after limit_cycles and the kernel records
+// FC_ERR_TIMEOUT and returns: the path a stuck pipeline takes, exercised
+// without faulting or hanging anything.
+// ---------------------------------------------------------------------------
+namespace {
+__global__ void k_selftest_wait(int arrive, unsigned long long limit_cycles) {
+  __shared__ __align__(8) uint64_t bar_word;
+  __shared__ int abort_flag;
+  const uint32_t bar = smem_u32(&bar_word);
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    mbar_init(bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (arrive) mbar_arrive(bar);
+    if (!mbar_wait_bounded(bar, 0, &abort_flag, limit_cycles)) fc_flag(&g_fc_err, FC_EBIT_TIMEOUT);
+  }
+}
+}  // namespace
+
+extern "C" fc_status fc_selftest_wait(int arrive, unsigned long long limit_cycles, fc_stream stream) {
+  if (limit_cycles == 0 || limit_cycles > 4000000000ull) return FC_ERR_INVALID_ARG;
+  k_selftest_wait<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(arrive, limit_cycles);
+  return FC_CHECK_LAUNCH();
+}

@@ -54,7 +54,7 @@ EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build
            "fc_retrieve", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
            "fc_missing_insert", "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_embed",
-           "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
+           "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
 
 
 def _load():
@@ -93,6 +93,7 @@ def _load():
         "fc_tree_attn_workspace": (sz, [i32, i32, i32, i32]),
         "fc_rope": (C.c_int, [vp, vp, i32, i32, i32, i32, i32, vp, C.c_float, vp]),
         "fc_gemm_workspace": (sz, []),
+        "fc_selftest_wait": (C.c_int, [i32, C.c_ulonglong, vp]),
         "fc_gemm_bf16": (C.c_int, [vp, vp, vp, i32, i32, i32, vp, sz, vp]),
         "fc_embed": (C.c_int, [vp, i32, vp, i32, i32, vp, vp]),
         "fc_add_rmsnorm": (C.c_int, [vp, vp, vp, vp, i32, i32, C.c_float, vp]),
@@ -146,6 +147,12 @@ def _need(t, dtype, name, shape=None):
 
 def version() -> str:
     return LIB.fc_version().decode()
+
+
+def fc_selftest_wait(arrive: bool, limit_cycles: int = 2_000_000):
+    """Bounded-wait self-test: with arrive=False the wait runs out and
+    fc_get_error() then reports FC_ERR_TIMEOUT."""
+    _check("fc_selftest_wait", LIB.fc_selftest_wait(1 if arrive else 0, int(limit_cycles), _stream()))
 
 
 def fc_get_error(stream=None) -> str:

@@ -140,3 +140,11 @@ def test_rope_host_validation_without_gpu(lib):
     assert L.fc_tree_attn_rope(*args, 16, f(-1.0), 16, nul, 0, nul) == 1
     bad_d = args[:13] + [96, f(0.1)]
     assert L.fc_tree_attn_rope(*bad_d, 16, f(10000.0), 16, nul, 0, nul) == 2
+
+
+def test_selftest_validation_without_gpu(lib):
+    import paper_2502_17139_gb300.fastcoder as fc
+    L = fc.LIB
+    # a wait limit of zero or beyond ~4e9 cycles is refused before any launch
+    assert L.fc_selftest_wait(0, 0, None) == 1
+    assert L.fc_selftest_wait(0, 5_000_000_000, None) == 1
