@@ -86,6 +86,8 @@ def parse_args(argv=None):
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
     ap.add_argument("--no-graph", action="store_true",
                     help="step mode: skip timing the same steps replayed from CUDA graphs (two steps per graph)")
+    ap.add_argument("--rev", action="store_true",
+                    help="retrieve mode: also time the reversed-corpus variant (fc_retrieve_rev) on the same queries")
     ap.add_argument("--rope", action="store_true",
                     help="attn mode: unrotated queries, rotated in the kernel by node position (fc_tree_attn_rope)")
     ap.add_argument("--weights", type=str, default="1,1",
@@ -979,11 +981,28 @@ def run_retrieve(args, rank, ws, local):
     ctx_d, cl_d = to_dev(ctx), to_dev(cl)
     res = fc.fc_retrieve(sources, ctx_d, cl_d, p)
     ms = _gpu_ms(lambda: fc.fc_retrieve(sources, ctx_d, cl_d, p, out=res), reps=args.steps, warm=args.warmup)
-    return {"metric": "retrievals/s", "value": 2 * args.batch / (ms * 1e-3), "unit": "query-sources/s",
-            "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-            "config": {"workload": f"two-source retrieval (5M + 100M tokens), {args.batch} contexts of 128, "
-                                   f"n 16->2, top-64 x 10"},
-            "us_per_query_source": ms * 1e3 / (2 * args.batch)}
+    out = {"metric": "retrievals/s", "value": 2 * args.batch / (ms * 1e-3), "unit": "query-sources/s",
+           "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+           "config": {"workload": f"two-source retrieval (5M + 100M tokens), {args.batch} contexts of 128, "
+                                  f"n 16->2, top-64 x 10"},
+           "us_per_query_source": ms * 1e3 / (2 * args.batch)}
+    if args.rev:
+        # the reversed-corpus variant on the same queries: n* by one narrowing
+        # search in the reversed suffix arrays, then the forward search for n*
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        revs = [fc.fc_datastore_build_reversed(s.tokens, synth.VOCAB) for s in sources]
+        torch.cuda.synchronize()
+        build_s = time.perf_counter() - t0
+        rr = fc.fc_retrieve_rev(sources, revs, ctx_d, cl_d, p)
+        same = all(torch.equal(res[k], rr[k]) for k in res)
+        assert same and fc.fc_get_error() == "FC_OK"
+        ms_r = _gpu_ms(lambda: fc.fc_retrieve_rev(sources, revs, ctx_d, cl_d, p, out=rr), reps=args.steps,
+                       warm=args.warmup)
+        out["reversed"] = {"ms_per_step": ms_r, "query_sources_per_s": 2 * args.batch / (ms_r * 1e-3),
+                           "us_per_query_source": ms_r * 1e3 / (2 * args.batch), "same_outputs": same,
+                           "reversed_build_seconds": build_s}
+    return out
 
 
 def run_algorithm1(args, rank, ws, local):

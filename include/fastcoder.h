@@ -137,6 +137,13 @@ fc_status fc_datastore_build_noalloc(const uint32_t* d_tokens, uint64_t n_tokens
                                      uint32_t* d_sa, uint32_t* d_bucket, uint8_t* d_lcp,
                                      fc_stream s, fc_datastore* out);
 
+/*
+ * The reversed corpus out[i] = tokens[n_tokens - 1 - i] (device buffers of
+ * n_tokens uint32, not overlapping), from which fc_datastore_build makes the
+ * reversed-corpus datastore that fc_retrieve_rev takes.  Asynchronous.
+ */
+fc_status fc_reverse_tokens(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t* d_out, fc_stream s);
+
 /* ------------------------------------------------------------------------
  * Retrieval (Section III-A; Section IV-C, Algorithm 1 par_search; Section
  * V-C: n_max = 16).
@@ -178,6 +185,27 @@ fc_status fc_retrieve(const fc_datastore* sources, int n_sources, const uint32_t
                       int ctx_stride, const int32_t* d_ctx_len, int batch, const int32_t* d_skip,
                       fc_retrieve_params p, uint32_t* d_drafts, int32_t* d_draft_len,
                       uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len, fc_stream s);
+
+/*
+ * fc_retrieve with the longest match found through the reversed corpus
+ * (a retrieval variant of Section III-A): the context suffixes of lengths
+ * 1, 2, ... read backwards are prefixes of one another, so in the suffix
+ * array of the reversed corpus their ranges are nested and one narrowing
+ * search, one token longer per step, finds n*; the forward suffix array is
+ * then searched for n* alone.  The outputs are exactly fc_retrieve's.
+ *   rev_sources host array [n_sources]: rev_sources[s] is the datastore of
+ *               sources[s]'s corpus reversed (fc_reverse_tokens, then
+ *               fc_datastore_build); its lcp is not read and may be NULL.
+ *               n_tokens and vocab must equal sources[s]'s
+ *               (FC_ERR_INVALID_ARG otherwise); that the corpus really is
+ *               the reverse is the caller's contract.
+ * Every other argument, limit and output as fc_retrieve.
+ */
+fc_status fc_retrieve_rev(const fc_datastore* sources, const fc_datastore* rev_sources, int n_sources,
+                          const uint32_t* d_ctx, int ctx_stride, const int32_t* d_ctx_len, int batch,
+                          const int32_t* d_skip, fc_retrieve_params p, uint32_t* d_drafts,
+                          int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
+                          int32_t* d_match_len, fc_stream s);
 
 /* ------------------------------------------------------------------------
  * Context-keyed retrieval cache (workload support for the step loop;

@@ -25,6 +25,13 @@
 //   * top-k: a histogram of run counts finds the k-th largest count; the runs
 //     above it and the first runs equal to it (in token order) are kept and
 //     ranked by (count descending, token order ascending).
+//   * reversed-corpus variant (fc_retrieve_rev): with the suffix array of the
+//     reversed corpus, the context suffixes of lengths 1, 2, ... read
+//     backwards are prefixes of one another, so their ranges are nested and
+//     one narrowing search (a warp, one more token per step, 16 pivots a
+//     round, two loads a probe) finds n* without trying every length; the
+//     forward suffix array is then searched for n* alone, and everything
+//     after it is shared with fc_retrieve, so the outputs are the same.
 #include <algorithm>
 
 #include "fc_common.cuh"
@@ -110,11 +117,69 @@ struct RetSmem {
   uint32_t endhit[FC_MAX_NMAX + 1];
   uint32_t wsum[RT_THREADS / 32];
   RunsScratch rs;
-  uint32_t n_star, first, cnt, bad;
+  uint32_t n_star, first, cnt, bad, n_rev;
 };
 
-__global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint32_t* __restrict__ ctx, int stride,
-                                                         const int32_t* __restrict__ ctx_len, int B,
+// n* through the reversed corpus R (R[i] = T[N-1-i]), by one warp.  The
+// context read backwards, rp = ctx[m-1], ctx[m-2], ..., has range(n) = the
+// reversed-SA range of suffixes that start with rp[0..n); range(n+1) is the
+// part of range(n) whose token at depth n is rp[n] (a suffix of exactly n
+// tokens sorts before the rest).  An occurrence at R position r ends the
+// forward window just before T position N - r, so the one at r = 0 (the
+// corpus ends with the pattern) has no continuation and does not count.  The
+// counts only fall as n grows, so the narrowing stops at the first empty
+// one.  Returns the longest n in [n_min, cap] with a count, or 0.
+__device__ int rev_match_len(const DsView& rv, const uint32_t* __restrict__ T, uint64_t N, const uint32_t* ctx,
+                             int cap, int n_min) {
+  const int lane = threadIdx.x & 31, hl = lane & 15;
+  const bool upper = lane >= 16;
+  const unsigned half_mask = upper ? 0xFFFF0000u : 0x0000FFFFu;
+  const uint32_t* __restrict__ R = rv.T;
+  int best = 0;
+  uint32_t c = ctx[cap - 1];
+  uint32_t lo = __ldg(rv.bucket + c), hi = __ldg(rv.bucket + c + 1);
+  bool ends = __ldg(T + N - 1) == c;  // T[N-n .. N) equals the pattern (R suffix 0 in the range)
+  for (int n = 1;; ++n) {
+    if (hi - lo <= (ends ? 1u : 0u)) break;
+    if (n >= n_min) best = n;
+    if (n == cap) break;
+    c = ctx[cap - 1 - n];
+    // bound search in [lo, hi): lower half-warp the first suffix whose token at
+    // depth n is >= c, upper half-warp the first one > c
+    uint32_t blo = lo, bhi = hi;
+    while (__any_sync(0xFFFFFFFFu, blo < bhi)) {
+      const bool active = blo < bhi;
+      const uint32_t piv = blo + (uint32_t)(((uint64_t)(hl + 1) * (bhi - blo)) / 17u);
+      bool pred = true;  // the suffix at piv is past the bound
+      if (active) {
+        const uint64_t at = (uint64_t)__ldg(rv.sa + piv) + (uint64_t)n;
+        if (at >= N) {
+          pred = false;  // exactly n tokens: before every suffix that has a token at depth n
+        } else {
+          const uint32_t t = __ldg(R + at);
+          pred = upper ? (t > c) : (t >= c);
+        }
+      }
+      const unsigned bal = __ballot_sync(0xFFFFFFFFu, !pred) & half_mask;
+      const int t = __popc(bal);
+      const int base_lane = upper ? 16 : 0;
+      const uint32_t p_before = __shfl_sync(0xFFFFFFFFu, piv, base_lane + max(t - 1, 0));
+      const uint32_t p_at = __shfl_sync(0xFFFFFFFFu, piv, base_lane + min(t, 15));
+      if (active) {
+        if (t > 0) blo = p_before + 1;
+        if (t < 16) bhi = p_at;
+      }
+    }
+    lo = __shfl_sync(0xFFFFFFFFu, blo, 0);
+    hi = __shfl_sync(0xFFFFFFFFu, blo, 16);
+    ends = ends && (uint64_t)n < N && __ldg(T + N - 1 - n) == c;
+  }
+  return best;
+}
+
+template <bool REV>
+__global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev, const uint32_t* __restrict__ ctx,
+                                                         int stride, const int32_t* __restrict__ ctx_len, int B,
                                                          const int32_t* __restrict__ skip, fc_retrieve_params p,
                                                          RetOut o) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -141,14 +206,24 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint
   if (sm.bad && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
 
   // ---- search: one warp per n, one half-warp per bound, 16 pivots a round
-  const int n_count = (cap >= p.n_min && !sm.bad) ? cap - p.n_min + 1 : 0;
+  // (lengths n_top down to n_top - n_count + 1; with the reversed corpus only n*)
+  int n_top = cap, n_count = (cap >= p.n_min && !sm.bad) ? cap - p.n_min + 1 : 0;
+  if constexpr (REV) {
+    if (tid < 32) {
+      const int r = n_count ? rev_match_len(rev.ds[s], T, N, sm.ctx, cap, p.n_min) : 0;
+      if (tid == 0) sm.n_rev = (uint32_t)r;
+    }
+    __syncthreads();
+    n_top = (int)sm.n_rev;
+    n_count = n_top ? 1 : 0;
+  }
   const int npairs = 2 * n_count;
   {
     const int warp = tid >> 5, lane = tid & 31, hl = lane & 15;
     const bool upper = lane >= 16;
     const unsigned half_mask = upper ? 0xFFFF0000u : 0x0000FFFFu;
     for (int w = warp; w < n_count; w += RT_THREADS / 32) {
-      const int n = cap - w;
+      const int n = n_top - w;
       const uint32_t* pat = sm.ctx + (cap - n);
       const uint32_t t0 = pat[0];
       uint32_t lo = __ldg(ds.bucket + t0), hi = __ldg(ds.bucket + t0 + 1);
@@ -187,7 +262,7 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, const uint
   if (tid == 0) {
     uint32_t ns = 0, first = 0, cnt = 0;
     if (npairs) {
-      for (int n = cap; n >= p.n_min; --n) {
+      for (int n = n_top; n > n_top - n_count; --n) {
         uint32_t l = sm.lo[n], h = sm.hi[n];
         if (l < h && sm.endhit[n]) ++l;
         if (l < h) {
@@ -408,10 +483,11 @@ __global__ void k_rc_insert(uint32_t* table, int capacity, int S, fc_retrieve_pa
 
 }  // namespace
 
-extern "C" fc_status fc_retrieve(const fc_datastore* sources, int n_sources, const uint32_t* d_ctx, int ctx_stride,
-                                 const int32_t* d_ctx_len, int batch, const int32_t* d_skip, fc_retrieve_params p,
-                                 uint32_t* d_drafts, int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
-                                 int32_t* d_match_len, fc_stream stream) {
+static fc_status launch_retrieve(const fc_datastore* sources, const fc_datastore* rev_sources, int n_sources,
+                                 const uint32_t* d_ctx, int ctx_stride, const int32_t* d_ctx_len, int batch,
+                                 const int32_t* d_skip, fc_retrieve_params p, uint32_t* d_drafts,
+                                 int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len,
+                                 fc_stream stream) {
   if (!sources || n_sources < 1 || n_sources > FC_MAX_SOURCES || batch < 0 || ctx_stride < 1 ||
       batch > 65535 * 16)
     return FC_ERR_INVALID_ARG;
@@ -428,18 +504,45 @@ extern "C" fc_status fc_retrieve(const fc_datastore* sources, int n_sources, con
     if (reinterpret_cast<uintptr_t>(ds.tokens) % 16) return FC_ERR_INVALID_ARG;  // read as 16-byte vectors
     a.ds[s] = DsView{ds.tokens, ds.sa, ds.bucket, ds.lcp, ds.n_tokens, ds.vocab};
   }
-  static bool attr_done = false;
-  if (!attr_done) {
-    if (cudaFuncSetAttribute(k_retrieve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(RetSmem)) !=
-        cudaSuccess)
+  DsArgs r{};
+  if (rev_sources) {
+    for (int s = 0; s < n_sources; ++s) {
+      const fc_datastore& rv = rev_sources[s];
+      if (!rv.tokens || !rv.sa || !rv.bucket || rv.n_tokens != sources[s].n_tokens || rv.vocab != sources[s].vocab)
+        return FC_ERR_INVALID_ARG;
+      r.ds[s] = DsView{rv.tokens, rv.sa, rv.bucket, rv.lcp, rv.n_tokens, rv.vocab};
+    }
+  }
+  auto kern = rev_sources ? k_retrieve<true> : k_retrieve<false>;
+  static bool attr_done[2] = {false, false};
+  if (!attr_done[rev_sources ? 1 : 0]) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(RetSmem)) != cudaSuccess)
       return FC_ERR_CUDA;
-    attr_done = true;
+    attr_done[rev_sources ? 1 : 0] = true;
   }
   RetOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len};
   dim3 grid((unsigned)batch, (unsigned)n_sources);
-  k_retrieve<<<grid, RT_THREADS, sizeof(RetSmem), static_cast<cudaStream_t>(stream)>>>(
-      a, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, o);
+  kern<<<grid, RT_THREADS, sizeof(RetSmem), static_cast<cudaStream_t>(stream)>>>(a, r, d_ctx, ctx_stride, d_ctx_len,
+                                                                                 batch, d_skip, p, o);
   return FC_CHECK_LAUNCH();
+}
+
+extern "C" fc_status fc_retrieve(const fc_datastore* sources, int n_sources, const uint32_t* d_ctx, int ctx_stride,
+                                 const int32_t* d_ctx_len, int batch, const int32_t* d_skip, fc_retrieve_params p,
+                                 uint32_t* d_drafts, int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
+                                 int32_t* d_match_len, fc_stream stream) {
+  return launch_retrieve(sources, nullptr, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, d_drafts,
+                         d_draft_len, d_count, d_n_drafts, d_match_len, stream);
+}
+
+extern "C" fc_status fc_retrieve_rev(const fc_datastore* sources, const fc_datastore* rev_sources, int n_sources,
+                                     const uint32_t* d_ctx, int ctx_stride, const int32_t* d_ctx_len, int batch,
+                                     const int32_t* d_skip, fc_retrieve_params p, uint32_t* d_drafts,
+                                     int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
+                                     int32_t* d_match_len, fc_stream stream) {
+  if (!rev_sources) return FC_ERR_INVALID_ARG;
+  return launch_retrieve(sources, rev_sources, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, d_drafts,
+                         d_draft_len, d_count, d_n_drafts, d_match_len, stream);
 }
 
 extern "C" size_t fc_rcache_bytes(int capacity, int n_sources, fc_retrieve_params p) {

@@ -446,3 +446,38 @@ extern "C" fc_status fc_datastore_build_noalloc(const uint32_t* d_tokens, uint64
   if (st != FC_OK) return st;
   return fc_datastore_build(d_tokens, n_tokens, vocab, d_sa, d_bucket, d_lcp, ws, kNoAllocScratchBytes, stream, out);
 }
+
+// ---------------------------------------------------------------------------
+// The reversed corpus R[i] = T[n-1-i], whose suffix array serves
+// fc_retrieve_rev.  Aligned 16-byte groups where both sides allow it: output
+// group q (tokens 4q .. 4q+3) reads input tokens n-4-4q .. n-1-4q, which are
+// 16-byte aligned exactly when n is a multiple of 4.
+// ---------------------------------------------------------------------------
+namespace {
+__global__ void k_reverse(const uint32_t* __restrict__ in, uint64_t n, uint32_t* __restrict__ out) {
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  const uint64_t t0 = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x;
+  const bool vec = (n % 4 == 0) && (reinterpret_cast<uintptr_t>(in) % 16 == 0) &&
+                   (reinterpret_cast<uintptr_t>(out) % 16 == 0);
+  if (vec) {
+    const uint64_t groups = n / 4;
+    for (uint64_t q = t0; q < groups; q += stride) {
+      const uint4 v = __ldg(reinterpret_cast<const uint4*>(in) + (groups - 1 - q));
+      reinterpret_cast<uint4*>(out)[q] = make_uint4(v.w, v.z, v.y, v.x);
+    }
+  } else {
+    for (uint64_t i = t0; i < n; i += stride) out[i] = __ldg(in + (n - 1 - i));
+  }
+}
+}  // namespace
+
+extern "C" fc_status fc_reverse_tokens(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t* d_out,
+                                       fc_stream stream) {
+  if (n_tokens == 0) return FC_OK;
+  if (!d_tokens || !d_out || d_tokens == d_out || n_tokens >= 0xFFFFFFFFull) return FC_ERR_INVALID_ARG;
+  const uint64_t a = reinterpret_cast<uintptr_t>(d_tokens), b = reinterpret_cast<uintptr_t>(d_out);
+  if (a < b + 4 * n_tokens && b < a + 4 * n_tokens) return FC_ERR_INVALID_ARG;  // overlapping buffers
+  k_reverse<<<grid_for(cdiv(n_tokens, 4), 256), 256, 0, static_cast<cudaStream_t>(stream)>>>(d_tokens, n_tokens,
+                                                                                            d_out);
+  return FC_CHECK_LAUNCH();
+}

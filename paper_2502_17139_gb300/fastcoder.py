@@ -51,7 +51,7 @@ class fc_cache(C.Structure):
 
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
            "fc_datastore_build_noalloc",
-           "fc_retrieve", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
+           "fc_retrieve", "fc_retrieve_rev", "fc_reverse_tokens", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
            "fc_missing_insert", "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_embed",
            "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
@@ -72,6 +72,9 @@ def _load():
         "fc_datastore_build_noalloc": (C.c_int, [vp, u64, u32, vp, vp, vp, vp, C.POINTER(fc_datastore)]),
         "fc_retrieve": (C.c_int, [C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp, fc_retrieve_params,
                                   vp, vp, vp, vp, vp, vp]),
+        "fc_retrieve_rev": (C.c_int, [C.POINTER(fc_datastore), C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp,
+                                      fc_retrieve_params, vp, vp, vp, vp, vp, vp]),
+        "fc_reverse_tokens": (C.c_int, [vp, u64, vp, vp]),
         "fc_rcache_bytes": (sz, [i32, i32, fc_retrieve_params]),
         "fc_rcache_init": (C.c_int, [vp, sz, i32, i32, fc_retrieve_params, vp]),
         "fc_rcache_lookup": (C.c_int, [vp, i32, i32, fc_retrieve_params, vp, i32, vp, i32, vp, vp,
@@ -250,6 +253,39 @@ def fc_retrieve(sources, ctx, ctx_len, p: fc_retrieve_params, skip=None, out=Non
     _check("fc_retrieve", LIB.fc_retrieve(views, S, _ptr(ctx), stride, _ptr(ctx_len), B, _ptr(skip), p,
                                           _ptr(o["drafts"]), _ptr(o["draft_len"]), _ptr(o["count"]),
                                           _ptr(o["n_drafts"]), _ptr(o["match_len"]), _stream()))
+    return o
+
+
+def fc_reverse_tokens(tokens: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:
+    """The reversed corpus (int32 [N] on the GPU); asynchronous."""
+    _need(tokens, torch.int32, "tokens")
+    o = out if out is not None else torch.empty_like(tokens)
+    _need(o, torch.int32, "out", tuple(tokens.shape))
+    _check("fc_reverse_tokens", LIB.fc_reverse_tokens(_ptr(tokens), tokens.numel(), _ptr(o), _stream()))
+    return o
+
+
+def fc_datastore_build_reversed(tokens: torch.Tensor, vocab: int) -> Datastore:
+    """The datastore of the reversed corpus, for fc_retrieve_rev."""
+    return fc_datastore_build(fc_reverse_tokens(tokens), vocab)
+
+
+def fc_retrieve_rev(sources, rev_sources, ctx, ctx_len, p: fc_retrieve_params, skip=None, out=None):
+    """fc_retrieve with n* found in the reversed corpora (same outputs)."""
+    S = len(sources)
+    if len(rev_sources) != S:
+        raise ValueError("one reversed datastore per source")
+    _need(ctx, torch.int32, "ctx")
+    B, stride = ctx.shape
+    _need(ctx_len, torch.int32, "ctx_len", (B,))
+    if skip is not None:
+        _need(skip, torch.int32, "skip", (B,))
+    o = out if out is not None else retrieve_outputs(S, B, p, ctx.device)
+    views = (fc_datastore * S)(*[s.view for s in sources])
+    rviews = (fc_datastore * S)(*[s.view for s in rev_sources])
+    _check("fc_retrieve_rev", LIB.fc_retrieve_rev(views, rviews, S, _ptr(ctx), stride, _ptr(ctx_len), B, _ptr(skip),
+                                                  p, _ptr(o["drafts"]), _ptr(o["draft_len"]), _ptr(o["count"]),
+                                                  _ptr(o["n_drafts"]), _ptr(o["match_len"]), _stream()))
     return o
 
 

@@ -148,3 +148,21 @@ def test_selftest_validation_without_gpu(lib):
     # a wait limit of zero or beyond ~4e9 cycles is refused before any launch
     assert L.fc_selftest_wait(0, 0, None) == 1
     assert L.fc_selftest_wait(0, 5_000_000_000, None) == 1
+
+
+def test_reversed_retrieval_validation_without_gpu(lib):
+    import paper_2502_17139_gb300.fastcoder as fc
+    L = fc.LIB
+    nul = None
+    p = fc.params(16, 2, 16, 8)
+    views = (fc.fc_datastore * 1)(fc.fc_datastore(16, 16, 16, 16, 10, 5))
+    # no reversed stores; a reversed store of another length or vocabulary
+    assert L.fc_retrieve_rev(views, nul, 1, 16, 64, 16, 4, nul, p, 16, 16, 16, 16, 16, nul) == 1
+    rv = (fc.fc_datastore * 1)(fc.fc_datastore(16, 16, 16, nul, 9, 5))
+    assert L.fc_retrieve_rev(views, rv, 1, 16, 64, 16, 4, nul, p, 16, 16, 16, 16, 16, nul) == 1
+    rv = (fc.fc_datastore * 1)(fc.fc_datastore(16, 16, 16, nul, 10, 6))
+    assert L.fc_retrieve_rev(views, rv, 1, 16, 64, 16, 4, nul, p, 16, 16, 16, 16, 16, nul) == 1
+    # reversal: empty is a no-op; overlapping buffers and null pointers are refused
+    assert L.fc_reverse_tokens(nul, 0, nul, nul) == 0
+    assert L.fc_reverse_tokens(4096, 100, 4096 + 200, nul) == 1
+    assert L.fc_reverse_tokens(nul, 100, 4096, nul) == 1

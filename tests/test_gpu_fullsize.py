@@ -98,6 +98,16 @@ def test_two_source_100m_5m(fc, orc):
         res.append(r)
     rt = orc.build_tree(res, [1, 1], root[sample], kvl[sample], cfg["node_budget"], cfg["n_pad"])
     compare_rows(gt, rt, sample)
+    # the reversed-corpus variant: the oracle's rows on the sample, and the
+    # forward search's outputs for every query
+    revs = [fc.fc_datastore_build_reversed(dev(T), synth.VOCAB) for T in corpora]
+    gr = fc.fc_retrieve_rev(sources, revs, dev(ctx), dev(cl), p)
+    assert fc.fc_get_error() == "FC_OK"
+    for s, r in enumerate(res):
+        compare_rows({k: v[s] for k, v in gr.items()}, r, sample)
+    for name in g:
+        assert torch.equal(g[name], gr[name]), name
+    del revs
     # the sample exercises long project-store matches and short general ones
     ml = g["match_len"].cpu().numpy()
     assert (ml[0] == 16).mean() > 0.3 and (ml[1] > 0).mean() > 0.9
