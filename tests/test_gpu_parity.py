@@ -418,6 +418,15 @@ def test_attn_gqa_n128(fc, orc):
     _attn_case(fc, orc, 3, B, 128, 32, 8, kvl, 2048, nn=[1, 20, 32, 33, 127, 128])
 
 
+def test_attn_one_tile_chunks(fc, orc):
+    # G = 4, 128-node trees whose second row chunk holds one tile (65..96
+    # nodes): that CTA splits its KV blocks between its two softmax
+    # warpgroups (odd and even block counts, an empty cache, one block)
+    B = 8
+    kvl = [0, 1, 128, 129, 383, 384, 2047, 2048]
+    _attn_case(fc, orc, 10, B, 128, 32, 8, kvl, 2048, nn=[65, 70, 88, 96, 97, 30, 66, 96])
+
+
 def test_attn_gqa_n64_group2(fc, orc):
     _attn_case(fc, orc, 4, 5, 64, 16, 8, [300, 0, 64, 700, 129], 777, nn=[64, 1, 40, 64, 2])
 
