@@ -86,6 +86,8 @@ def parse_args(argv=None):
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
     ap.add_argument("--no-graph", action="store_true",
                     help="step mode: skip timing the same steps replayed from CUDA graphs (two steps per graph)")
+    ap.add_argument("--all-occ", action="store_true",
+                    help="retrieve mode: also time the all-occurrence trie (fc_retrieve_all + fc_build_tree_all)")
     ap.add_argument("--rev", action="store_true",
                     help="retrieve mode: also time the reversed-corpus variant (fc_retrieve_rev) on the same queries")
     ap.add_argument("--rope", action="store_true",
@@ -401,6 +403,9 @@ def run_ours(args, rank, ws, local):
         "tree_attn_tflops": tot_f / tot_t / 1e12,
         "avg_acceptance_length": float(np.mean([a.mean() + 1 for a in acc_hist])),
         "avg_tree_nodes": float(np.mean([n.mean() for n in nodes_hist])),
+        # trees by node count in 32-node bins (1-32, 33-64, 65-96, 97-128): with four
+        # query heads per kv head, the number of 128-row tiles a group needs
+        "tree_nodes_bins": np.bincount((np.concatenate(nodes_hist) - 1) // 32, minlength=n_pad // 32).tolist(),
         "datastore_build": {"tokens": build_tokens, "seconds": build_s, "tokens_per_s": build_tokens / build_s},
     }
     if not args.no_e2e:
@@ -1002,6 +1007,27 @@ def run_retrieve(args, rank, ws, local):
         out["reversed"] = {"ms_per_step": ms_r, "query_sources_per_s": 2 * args.batch / (ms_r * 1e-3),
                            "us_per_query_source": ms_r * 1e3 / (2 * args.batch), "same_outputs": same,
                            "reversed_build_seconds": build_s}
+    if args.all_occ:
+        # the all-occurrence trie: every distinct continuation of the first 4096
+        # occurrences per source, and the weighted trie over all of them
+        pa = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
+        ra = fc.fc_retrieve_all(sources, ctx_d, cl_d, pa)
+        root = to_dev(ctx[np.arange(args.batch), cl - 1])
+        kvl = to_dev(np.full(args.batch, 4096, np.int32))
+        ws_t = torch.empty(int(fc.LIB.fc_build_tree_all_workspace(2, 4096, cfg["draft_len"], args.batch)),
+                           dtype=torch.uint8, device=dev)
+        tr = fc.fc_build_tree_all(ra, [1, 1], root, kvl, cfg["node_budget"], cfg["n_pad"], workspace=ws_t)
+        assert fc.fc_get_error() == "FC_OK"
+        ms_a = _gpu_ms(lambda: fc.fc_retrieve_all(sources, ctx_d, cl_d, pa, out=ra), reps=args.steps,
+                       warm=args.warmup)
+        ms_t = _gpu_ms(lambda: fc.fc_build_tree_all(ra, [1, 1], root, kvl, cfg["node_budget"], cfg["n_pad"],
+                                                    workspace=ws_t, out=tr), reps=args.steps, warm=args.warmup)
+        nd = ra["n_drafts"].cpu().numpy()
+        out["all_occurrence"] = {"retrieve_all_ms": ms_a, "build_tree_all_ms": ms_t,
+                                 "mean_distinct_per_query_source": float(nd.mean()),
+                                 "max_distinct_per_query_source": int(nd.max()),
+                                 "mean_tree_nodes": float(tr["n_nodes"].float().mean().item()),
+                                 "workspace_bytes": int(ws_t.numel())}
     return out
 
 

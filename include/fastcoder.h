@@ -187,6 +187,20 @@ fc_status fc_retrieve(const fc_datastore* sources, int n_sources, const uint32_t
                       uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len, fc_stream s);
 
 /*
+ * fc_retrieve without the top-k (the input of the all-occurrence trie,
+ * fc_build_tree_all): every distinct continuation among the first max_occ
+ * occurrences, in ascending token order (a prefix before its extensions),
+ * with its count.  p.top_k is not used; the output arrays have p.max_occ
+ * slots per query and source: d_drafts [S][batch][max_occ][draft_len],
+ * d_draft_len and d_count [S][batch][max_occ], d_n_drafts and d_match_len
+ * [S][batch].  Everything else as fc_retrieve.
+ */
+fc_status fc_retrieve_all(const fc_datastore* sources, int n_sources, const uint32_t* d_ctx,
+                          int ctx_stride, const int32_t* d_ctx_len, int batch, const int32_t* d_skip,
+                          fc_retrieve_params p, uint32_t* d_drafts, int32_t* d_draft_len,
+                          uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len, fc_stream s);
+
+/*
  * fc_retrieve with the longest match found through the reversed corpus
  * (a retrieval variant of Section III-A): the context suffixes of lengths
  * 1, 2, ... read backwards are prefixes of one another, so in the suffix
@@ -372,6 +386,33 @@ fc_status fc_build_tree(int n_sources, const uint32_t* d_drafts, const int32_t* 
                         int node_budget, int n_pad, uint32_t* d_tok, int32_t* d_parent,
                         int32_t* d_depth, int32_t* d_pos, uint64_t* d_mask, int32_t* d_n_nodes,
                         fc_stream s);
+
+/*
+ * The all-occurrence trie (Section III-A, Eq. 3 over every retrieved
+ * continuation instead of the top-k): fc_build_tree's tree over the
+ * drafts that fc_retrieve_all writes, every distinct continuation of each
+ * source with its count.  Each source's valid drafts (the first
+ * n_drafts[s][b] slots with 1 <= draft_len <= draft_len) must be in strictly
+ * ascending token order (a prefix before its extensions), as
+ * fc_retrieve_all writes them; a query that breaks this records
+ * FC_ERR_INVALID_ARG and gets a root-only tree.
+ *   d_drafts    [n_sources][batch][slots][draft_len] (the fc_retrieve_all
+ *               layout, slots = its max_occ); d_draft_len, d_count
+ *               [n_sources][batch][slots]; d_n_drafts [n_sources][batch]
+ *   d_ws        device workspace, 256-byte aligned, of at least
+ *               fc_build_tree_all_workspace(n_sources, slots, draft_len, batch)
+ *               bytes (FC_ERR_WORKSPACE otherwise)
+ * Weights, budget, tie-breaks and outputs as fc_build_tree.  Counts above
+ * 2^17 are clamped (FC_ERR_INVALID_ARG recorded).
+ * Limits: n_sources * slots <= 8192, draft_len <= FC_MAX_DRAFT_LEN.
+ */
+size_t fc_build_tree_all_workspace(int n_sources, int slots, int draft_len, int batch);
+fc_status fc_build_tree_all(int n_sources, const uint32_t* d_drafts, const int32_t* d_draft_len,
+                            const uint32_t* d_count, const int32_t* d_n_drafts, const uint32_t* src_weight,
+                            int slots, int draft_len, const uint32_t* d_root_tok, const int32_t* d_kv_len,
+                            int batch, int node_budget, int n_pad, void* d_ws, size_t ws_bytes,
+                            uint32_t* d_tok, int32_t* d_parent, int32_t* d_depth, int32_t* d_pos,
+                            uint64_t* d_mask, int32_t* d_n_nodes, fc_stream s);
 
 /*
  * Eq. 4 mask, depths and position ids of trees given by parent pointers in

@@ -32,6 +32,9 @@
 //     round, two loads a probe) finds n* without trying every length; the
 //     forward suffix array is then searched for n* alone, and everything
 //     after it is shared with fc_retrieve, so the outputs are the same.
+//   * all-continuations variant (fc_retrieve_all): no top-k; every run is
+//     written, in SA order, which is ascending token order (the input of the
+//     all-occurrence trie).
 #include <algorithm>
 
 #include "fc_common.cuh"
@@ -177,7 +180,7 @@ __device__ int rev_match_len(const DsView& rv, const uint32_t* __restrict__ T, u
   return best;
 }
 
-template <bool REV>
+template <bool REV, bool ALL>
 __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev, const uint32_t* __restrict__ ctx,
                                                          int stride, const int32_t* __restrict__ ctx_len, int B,
                                                          const int32_t* __restrict__ skip, fc_retrieve_params p,
@@ -189,7 +192,7 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev
   const DsView ds = args.ds[s];
   const uint32_t* __restrict__ T = ds.T;
   const uint64_t N = ds.n;
-  const int k = p.top_k, d = p.draft_len;
+  const int k = ALL ? (int)p.max_occ : p.top_k, d = p.draft_len;  // output slots per query and source
   const size_t sb = (size_t)s * B + b;
 
   int m = ctx_len[b];
@@ -302,15 +305,20 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev
   for (uint32_t e = tid; e < nocc; e += RT_THREADS)
     sm.work[e] = (e == 0 || (uint32_t)__ldg(ds.lcp + first + e) < need) ? 1u : 0u;
   __syncthreads();
-  const uint32_t nd_sel = rank_runs<RT_THREADS>(nocc, k, sm.runs, sm.work, sm.sel, sm.order, sm.wsum, sm.rs);
+  uint32_t nd_sel;
+  if constexpr (ALL)
+    nd_sel = runs_from_heads<RT_THREADS>(nocc, sm.runs, sm.work, sm.wsum, sm.rs);
+  else
+    nd_sel = rank_runs<RT_THREADS>(nocc, k, sm.runs, sm.work, sm.sel, sm.order, sm.wsum, sm.rs);
   auto run_count = [&](uint32_t r) { return sm.runs[r + 1] - sm.runs[r]; };
+  auto run_at = [&](int t) -> uint32_t { return ALL ? (uint32_t)t : sm.order[t]; };  // the run in output slot t
   // ---- outputs ---------------------------------------------------------
   const int nd = (int)nd_sel;
   for (int e = tid; e < k * d; e += RT_THREADS) {
     int t = e / d, x = e - t * d;
     uint32_t v = FC_PAD_TOKEN;
     if (t < nd) {
-      const uint32_t pp = __ldg(ds.sa + first + sm.runs[sm.order[t]]) + (uint32_t)ns;
+      const uint32_t pp = __ldg(ds.sa + first + sm.runs[run_at(t)]) + (uint32_t)ns;
       uint64_t len = min((uint64_t)d, N - pp);
       if ((uint64_t)x < len) v = __ldg(T + pp + x);
     }
@@ -318,7 +326,7 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev
   }
   for (int t = tid; t < k; t += RT_THREADS) {
     if (t < nd) {
-      const uint32_t r = sm.order[t];
+      const uint32_t r = run_at(t);
       const uint32_t pp = __ldg(ds.sa + first + sm.runs[r]) + (uint32_t)ns;
       dl[t] = (int32_t)min((uint64_t)d, N - pp);
       ct[t] = run_count(r);
@@ -483,7 +491,7 @@ __global__ void k_rc_insert(uint32_t* table, int capacity, int S, fc_retrieve_pa
 
 }  // namespace
 
-static fc_status launch_retrieve(const fc_datastore* sources, const fc_datastore* rev_sources, int n_sources,
+static fc_status launch_retrieve(bool all, const fc_datastore* sources, const fc_datastore* rev_sources, int n_sources,
                                  const uint32_t* d_ctx, int ctx_stride, const int32_t* d_ctx_len, int batch,
                                  const int32_t* d_skip, fc_retrieve_params p, uint32_t* d_drafts,
                                  int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len,
@@ -513,12 +521,13 @@ static fc_status launch_retrieve(const fc_datastore* sources, const fc_datastore
       r.ds[s] = DsView{rv.tokens, rv.sa, rv.bucket, rv.lcp, rv.n_tokens, rv.vocab};
     }
   }
-  auto kern = rev_sources ? k_retrieve<true> : k_retrieve<false>;
-  static bool attr_done[2] = {false, false};
-  if (!attr_done[rev_sources ? 1 : 0]) {
+  const int variant = all ? 2 : (rev_sources ? 1 : 0);
+  auto kern = all ? k_retrieve<false, true> : (rev_sources ? k_retrieve<true, false> : k_retrieve<false, false>);
+  static bool attr_done[3] = {false, false, false};
+  if (!attr_done[variant]) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(RetSmem)) != cudaSuccess)
       return FC_ERR_CUDA;
-    attr_done[rev_sources ? 1 : 0] = true;
+    attr_done[variant] = true;
   }
   RetOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len};
   dim3 grid((unsigned)batch, (unsigned)n_sources);
@@ -531,7 +540,15 @@ extern "C" fc_status fc_retrieve(const fc_datastore* sources, int n_sources, con
                                  const int32_t* d_ctx_len, int batch, const int32_t* d_skip, fc_retrieve_params p,
                                  uint32_t* d_drafts, int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
                                  int32_t* d_match_len, fc_stream stream) {
-  return launch_retrieve(sources, nullptr, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, d_drafts,
+  return launch_retrieve(false, sources, nullptr, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, d_drafts,
+                         d_draft_len, d_count, d_n_drafts, d_match_len, stream);
+}
+
+extern "C" fc_status fc_retrieve_all(const fc_datastore* sources, int n_sources, const uint32_t* d_ctx,
+                                     int ctx_stride, const int32_t* d_ctx_len, int batch, const int32_t* d_skip,
+                                     fc_retrieve_params p, uint32_t* d_drafts, int32_t* d_draft_len,
+                                     uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len, fc_stream stream) {
+  return launch_retrieve(true, sources, nullptr, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, d_drafts,
                          d_draft_len, d_count, d_n_drafts, d_match_len, stream);
 }
 
@@ -541,7 +558,7 @@ extern "C" fc_status fc_retrieve_rev(const fc_datastore* sources, const fc_datas
                                      int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
                                      int32_t* d_match_len, fc_stream stream) {
   if (!rev_sources) return FC_ERR_INVALID_ARG;
-  return launch_retrieve(sources, rev_sources, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, d_drafts,
+  return launch_retrieve(false, sources, rev_sources, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, d_drafts,
                          d_draft_len, d_count, d_n_drafts, d_match_len, stream);
 }
 

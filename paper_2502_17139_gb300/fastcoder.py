@@ -51,9 +51,9 @@ class fc_cache(C.Structure):
 
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
            "fc_datastore_build_noalloc",
-           "fc_retrieve", "fc_retrieve_rev", "fc_reverse_tokens", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
+           "fc_retrieve", "fc_retrieve_all", "fc_retrieve_rev", "fc_reverse_tokens", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
-           "fc_missing_insert", "fc_build_tree", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_embed",
+           "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_embed",
            "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
 
 
@@ -72,6 +72,8 @@ def _load():
         "fc_datastore_build_noalloc": (C.c_int, [vp, u64, u32, vp, vp, vp, vp, C.POINTER(fc_datastore)]),
         "fc_retrieve": (C.c_int, [C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp, fc_retrieve_params,
                                   vp, vp, vp, vp, vp, vp]),
+        "fc_retrieve_all": (C.c_int, [C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp, fc_retrieve_params,
+                                      vp, vp, vp, vp, vp, vp]),
         "fc_retrieve_rev": (C.c_int, [C.POINTER(fc_datastore), C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp,
                                       fc_retrieve_params, vp, vp, vp, vp, vp, vp]),
         "fc_reverse_tokens": (C.c_int, [vp, u64, vp, vp]),
@@ -90,6 +92,9 @@ def _load():
         "fc_missing_insert": (C.c_int, [vp, i32, i32, vp, i32, vp, i32, vp, vp, i32, vp]),
         "fc_build_tree": (C.c_int, [i32, vp, vp, vp, vp, C.POINTER(C.c_uint32), i32, i32, vp, vp, i32, i32, i32,
                                     vp, vp, vp, vp, vp, vp, vp]),
+        "fc_build_tree_all_workspace": (sz, [i32, i32, i32, i32]),
+        "fc_build_tree_all": (C.c_int, [i32, vp, vp, vp, vp, C.POINTER(C.c_uint32), i32, i32, vp, vp, i32, i32, i32,
+                                        vp, sz, vp, vp, vp, vp, vp, vp, vp]),
         "fc_tree_mask": (C.c_int, [vp, vp, vp, i32, i32, vp, vp, vp, vp]),
         "fc_tree_attn": (C.c_int, [vp, vp, vp, i32, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, C.c_float, vp, vp, sz,
                                    vp]),
@@ -230,8 +235,8 @@ def params(n_max, n_min, top_k, draft_len, max_occ=MAX_OCC) -> fc_retrieve_param
     return fc_retrieve_params(n_max, n_min, top_k, draft_len, max_occ)
 
 
-def retrieve_outputs(n_sources, batch, p: fc_retrieve_params, device="cuda"):
-    S, B, k, d = n_sources, batch, p.top_k, p.draft_len
+def retrieve_outputs(n_sources, batch, p: fc_retrieve_params, device="cuda", slots=None):
+    S, B, k, d = n_sources, batch, (p.top_k if slots is None else slots), p.draft_len
     return dict(drafts=torch.empty((S, B, k, d), dtype=torch.int32, device=device),
                 draft_len=torch.empty((S, B, k), dtype=torch.int32, device=device),
                 count=torch.empty((S, B, k), dtype=torch.int32, device=device),
@@ -253,6 +258,23 @@ def fc_retrieve(sources, ctx, ctx_len, p: fc_retrieve_params, skip=None, out=Non
     _check("fc_retrieve", LIB.fc_retrieve(views, S, _ptr(ctx), stride, _ptr(ctx_len), B, _ptr(skip), p,
                                           _ptr(o["drafts"]), _ptr(o["draft_len"]), _ptr(o["count"]),
                                           _ptr(o["n_drafts"]), _ptr(o["match_len"]), _stream()))
+    return o
+
+
+def fc_retrieve_all(sources, ctx, ctx_len, p: fc_retrieve_params, skip=None, out=None):
+    """Every distinct continuation (no top-k), in ascending token order:
+    outputs shaped [S, B, p.max_occ, ...]."""
+    S = len(sources)
+    _need(ctx, torch.int32, "ctx")
+    B, stride = ctx.shape
+    _need(ctx_len, torch.int32, "ctx_len", (B,))
+    if skip is not None:
+        _need(skip, torch.int32, "skip", (B,))
+    o = out if out is not None else retrieve_outputs(S, B, p, ctx.device, slots=int(p.max_occ))
+    views = (fc_datastore * S)(*[s.view for s in sources])
+    _check("fc_retrieve_all", LIB.fc_retrieve_all(views, S, _ptr(ctx), stride, _ptr(ctx_len), B, _ptr(skip), p,
+                                                  _ptr(o["drafts"]), _ptr(o["draft_len"]), _ptr(o["count"]),
+                                                  _ptr(o["n_drafts"]), _ptr(o["match_len"]), _stream()))
     return o
 
 
@@ -410,6 +432,24 @@ def fc_build_tree(res, src_weight, root_tok, kv_len, node_budget, n_pad, out=Non
                                               node_budget, n_pad, _ptr(o["tok"]), _ptr(o["parent"]),
                                               _ptr(o["depth"]), _ptr(o["pos"]), _ptr(o["mask"]), _ptr(o["n_nodes"]),
                                               _stream()))
+    return o
+
+
+def fc_build_tree_all(res, src_weight, root_tok, kv_len, node_budget, n_pad, workspace=None, out=None):
+    """The all-occurrence trie over fc_retrieve_all's outputs ([S, B, slots, ...])."""
+    S, B, k, d = res["drafts"].shape
+    _need(root_tok, torch.int32, "root_tok", (B,))
+    _need(kv_len, torch.int32, "kv_len", (B,))
+    need = int(LIB.fc_build_tree_all_workspace(S, k, d, B))
+    if need == 0:
+        raise ValueError("unsupported shape for the all-occurrence trie")
+    ws = workspace if workspace is not None else torch.empty(need, dtype=torch.uint8, device=root_tok.device)
+    w = (C.c_uint32 * S)(*[int(x) for x in src_weight])
+    o = out if out is not None else tree_outputs(B, n_pad, root_tok.device)
+    _check("fc_build_tree_all", LIB.fc_build_tree_all(
+        S, _ptr(res["drafts"]), _ptr(res["draft_len"]), _ptr(res["count"]), _ptr(res["n_drafts"]), w, k, d,
+        _ptr(root_tok), _ptr(kv_len), B, node_budget, n_pad, _ptr(ws), ws.numel(), _ptr(o["tok"]), _ptr(o["parent"]),
+        _ptr(o["depth"]), _ptr(o["pos"]), _ptr(o["mask"]), _ptr(o["n_nodes"]), _stream()))
     return o
 
 

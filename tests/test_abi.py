@@ -166,3 +166,20 @@ def test_reversed_retrieval_validation_without_gpu(lib):
     assert L.fc_reverse_tokens(nul, 0, nul, nul) == 0
     assert L.fc_reverse_tokens(4096, 100, 4096 + 200, nul) == 1
     assert L.fc_reverse_tokens(nul, 100, 4096, nul) == 1
+
+
+def test_trie_all_validation_without_gpu(lib):
+    import paper_2502_17139_gb300.fastcoder as fc
+    L = fc.LIB
+    nul = None
+    w = (C.c_uint32 * 2)(1, 1)
+    # workspace size: zero for unsupported shapes (more than 8192 drafts, long drafts)
+    assert L.fc_build_tree_all_workspace(2, 4096, 10, 32) > 0
+    assert L.fc_build_tree_all_workspace(3, 4096, 10, 32) == 0
+    assert L.fc_build_tree_all_workspace(2, 64, 17, 32) == 0
+    args = [16, 16, 16, 16, w, 4096, 10, 16, 16, 32, 128, 128]
+    outs = [16, 16, 16, 16, 16, 16, nul]
+    assert L.fc_build_tree_all(2, *args, 256, 1000, *outs) == 3          # FC_ERR_WORKSPACE
+    assert L.fc_build_tree_all(3, *args, 256, 1 << 40, *outs) == 2       # too many drafts: FC_ERR_UNSUPPORTED
+    assert L.fc_build_tree_all(2, *args[:10], 128, 96, 256, 1 << 40, *outs) == 2  # n_pad 96
+    assert L.fc_build_tree_all(2, *args[:10], 0, 128, 256, 1 << 40, *outs) == 1   # budget 0

@@ -108,6 +108,16 @@ def test_two_source_100m_5m(fc, orc):
     for name in g:
         assert torch.equal(g[name], gr[name]), name
     del revs
+    # the all-occurrence trie (every distinct continuation, up to 4096 per
+    # source) on the sampled queries, against the oracle's untruncated lists
+    pa = fc.params(cfg["n_max"], cfg["n_min"], 8, cfg["draft_len"], 4096)
+    ga = fc.fc_retrieve_all(sources, dev(ctx[sample]), dev(cl[sample]), pa)
+    ra = [orc.retrieve(T, ctx[sample], cl[sample], cfg["n_max"], cfg["n_min"], 4096, cfg["draft_len"], 4096)
+          for T in corpora]
+    gta = fc.fc_build_tree_all(ga, [1, 1], dev(root[sample]), dev(kvl[sample]), cfg["node_budget"], cfg["n_pad"])
+    assert fc.fc_get_error() == "FC_OK"
+    rta = orc.build_tree(ra, [1, 1], root[sample], kvl[sample], cfg["node_budget"], cfg["n_pad"])
+    compare_rows(gta, rta, np.arange(len(sample)))
     # the sample exercises long project-store matches and short general ones
     ml = g["match_len"].cpu().numpy()
     assert (ml[0] == 16).mean() > 0.3 and (ml[1] > 0).mean() > 0.9
