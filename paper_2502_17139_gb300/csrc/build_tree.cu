@@ -365,11 +365,13 @@ __global__ void __launch_bounds__(BT_THREADS) k_build_tree(TreeIn in, int S, int
   if (tid < 32) warp_scan_u64(wu, ps, U);  // ps[u] = sum of wu[0..u), ps[U] = total
   uint32_t C = block_scan_array(coff, (int)U, wsum);
   for (uint32_t u = tid; u < U; u += BT_THREADS) {
+    // deepest first: the run of (u, l) ends at the first e > u with lcp[e] < l,
+    // which only moves right as l falls, so one scan serves every depth
     const int lu = len[uniq[u]];
-    for (int l = (int)lcp[u] + 1; l <= lu; ++l) {
-      uint32_t e = u + 1;
+    uint32_t e = u + 1;
+    for (int l = lu; l > (int)lcp[u]; --l) {
       while (e < U && (int)lcp[e] >= l) ++e;
-      uint64_t W = ps[e] - ps[u];
+      const uint64_t W = ps[e] - ps[u];
       ckey[coff[u] + (l - lcp[u] - 1)] = (W << 18) | ((uint64_t)(31 - l) << 13) | (uint64_t)(8191u - u);
     }
   }

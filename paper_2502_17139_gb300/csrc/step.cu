@@ -239,23 +239,28 @@ __global__ void k_synth_argmax(const uint32_t* __restrict__ tok, const int32_t* 
                                const uint32_t* __restrict__ rtok, uint32_t vocab, uint32_t* __restrict__ argmax) {
   __shared__ int agree[FC_MAX_NODES];
   __shared__ int par_s[FC_MAX_NODES];
+  __shared__ int first_child[FC_MAX_NODES];
   __shared__ uint32_t tok_s[FC_MAX_NODES];
   const int b = blockIdx.x;
   const size_t base = (size_t)b * n_pad;
   const int n = min(max((int)n_nodes[b], 1), n_pad);
   for (int i = threadIdx.x; i < n_pad; i += blockDim.x) {  // the tree, staged once (coalesced)
     agree[i] = -1;
+    first_child[i] = n_pad;
     par_s[i] = parent[base + i];
     tok_s[i] = tok[base + i];
+  }
+  __syncthreads();
+  for (int j = 1 + threadIdx.x; j < n; j += blockDim.x) {  // first child: the smallest later node below
+    const int p = par_s[j];
+    if (p >= 0 && p < j) atomicMin(&first_child[p], j);
   }
   __syncthreads();
   if (threadIdx.x == 0) {
     int cur = 0;
     for (int t = 0; t < plen[b]; ++t) {
-      int first = -1;
-      for (int j = cur + 1; j < n && first < 0; ++j)
-        if (par_s[j] == cur) first = j;
-      if (first < 0) break;
+      const int first = first_child[cur];
+      if (first >= n) break;
       agree[cur] = first;
       cur = first;
     }
