@@ -41,13 +41,17 @@ sys.path.insert(0, ROOT)
 METRIC = "retrieve+verify steps/s"
 UNIT = "steps/s"
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one tree-attention
-# launch of the step loop, from one ncu capture: the mean over 14 k_tree_attn launches of
-#   ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum
-#       --clock-control none -k regex:k_tree_attn -c 14 --csv
-#       python bench.py --steps 4 --warmup 3 --no-e2e --no-cpu-baseline
-# It is valid only for the kernel sources it was taken on (their SHA-256 below); once
-# those change, the bench reports traffic as null until it is measured again.
-ATTN_TRAFFIC = {"bytes_per_launch": 2.3670e9,
+# launch of the step loop with the sequences in 2 sub-batches (16 sequences a
+# launch, 256 CTAs), from one ncu capture: the mean over the 28 launches with a grid
+# of 256 of
+#   ncu --metrics gpu__time_duration.sum,dram__bytes_read.sum,dram__bytes_write.sum
+#       --clock-control none -k regex:k_tree_attn -c 60 --csv
+#       python bench.py --steps 4 --warmup 3 --no-e2e --no-cpu-baseline --no-graph
+# (the 568-CTA launches in the same capture are the single-stream pass over all 32
+# sequences: 2.367e9 bytes each).  It is valid only for the kernel sources it was
+# taken on (their SHA-256 below) and that split; otherwise the bench reports traffic
+# as null until it is measured again.
+ATTN_TRAFFIC = {"bytes_per_launch": 1.1714e9, "sub_batches": 2,
                 "sources": ["paper_2502_17139_gb300/csrc/tree_attn.cu", "paper_2502_17139_gb300/csrc/fc_common.cuh"],
                 "sha256": "ef8c93976042c50443c18522134a35334265e92729d5d394c2d7ce71f39a35b3"}
 
@@ -86,6 +90,8 @@ def parse_args(argv=None):
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
     ap.add_argument("--no-graph", action="store_true",
                     help="step mode: skip timing the same steps replayed from CUDA graphs (two steps per graph)")
+    ap.add_argument("--split", type=int, default=2,
+                    help="step mode: sub-batches of the sequences, each on its own CUDA stream (1: one stream)")
     ap.add_argument("--all-occ", action="store_true",
                     help="retrieve mode: also time the all-occurrence trie (fc_retrieve_all + fc_build_tree_all)")
     ap.add_argument("--rev", action="store_true",
@@ -103,10 +109,13 @@ def parse_args(argv=None):
 
 
 # ---------------------------------------------------------------- helpers
-def attn_traffic(args):
-    """Measured DRAM bytes per attention launch, or None when the kernel changed since."""
+def attn_traffic(args, nsub=1):
+    """Measured DRAM bytes per attention launch, or None when the kernel or the
+    launch's sub-batch split changed since."""
     if args.traffic_bytes is not None:
         return args.traffic_bytes
+    if nsub != ATTN_TRAFFIC["sub_batches"]:
+        return None
     import hashlib
     h = hashlib.sha256()
     for f in ATTN_TRAFFIC["sources"]:
@@ -262,7 +271,7 @@ def run_ours(args, rank, ws, local):
 
     import paper_2502_17139_gb300.fastcoder as fc
     import paper_2502_17139_gb300.synth as synth
-    from paper_2502_17139_gb300.step import StepLoop
+    from paper_2502_17139_gb300.step import PipelinedStepLoop, StepLoop
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
@@ -293,9 +302,19 @@ def run_ours(args, rank, ws, local):
 
     weights = src_weights(args)
 
+    nsub = max(1, min(args.split, B))
+
     def new_loop():
+        if nsub > 1:
+            return PipelinedStepLoop(nsub, sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, weights, H,
+                                     Hkv, D, cap, kv0, synth.VOCAB, cache_capacity=1 << 14, device=dev, k_cache=kc,
+                                     v_cache=vc)
         return StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, weights, H, Hkv, D, cap, kv0,
                         synth.VOCAB, cache_capacity=1 << 14, device=dev, k_cache=kc, v_cache=vc)
+
+    def join(lp):
+        if nsub > 1:
+            lp.join()
 
     # device-resident per-step inputs (a pool of distinct activations, cycled)
     P = min(16, K + W)
@@ -310,22 +329,18 @@ def run_ours(args, rank, ws, local):
         loop.step(q_pool[s % P], kt_pool[s % P], vt_pool[s % P], no_hit, plen_d[s], rtok_d[s])
     loop.reset()
     stream = torch.cuda.current_stream()
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    ev_ret = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    ev_tree = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    ev_tail = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    mk = lambda: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    # stage events per timed step and sub-batch (recorded on the sub-batch's stream)
+    stage_ev = [[dict(attn=mk(), retrieve=mk(), tree=mk(), tail=mk()) for _ in range(nsub)] for _ in range(K)]
 
     def do_step(s, timed_idx=None):
         j = s % P
-        if timed_idx is not None:
-            loop.step(q_pool[j], kt_pool[j], vt_pool[j], hits_d[s], plen_d[s], rtok_d[s],
-                      events=dict(attn=ev[timed_idx], retrieve=ev_ret[timed_idx], tree=ev_tree[timed_idx],
-                                  tail=ev_tail[timed_idx]))
-        else:
-            loop.step(q_pool[j], kt_pool[j], vt_pool[j], hits_d[s], plen_d[s], rtok_d[s])
+        evs = None if timed_idx is None else (stage_ev[timed_idx] if nsub > 1 else stage_ev[timed_idx][0])
+        loop.step(q_pool[j], kt_pool[j], vt_pool[j], hits_d[s], plen_d[s], rtok_d[s], events=evs)
 
     for s in range(W):
         do_step(s)
+    join(loop)
     assert fc.fc_get_error() == "FC_OK"
     barrier(ws)
     torch.cuda.synchronize()
@@ -335,6 +350,7 @@ def run_ours(args, rank, ws, local):
     start.record(stream)
     for i in range(K):
         do_step(W + i, i)
+    join(loop)
     end.record(stream)
     torch.cuda.synchronize()
     clock_rec = clocks.stop()
@@ -350,23 +366,26 @@ def run_ours(args, rank, ws, local):
             assert fc.fc_get_error() == "FC_OK"
         except Exception as e:  # reported, not fatal: the eager line stands
             graph_rec = {"error": f"{type(e).__name__}: {e}"[:200]}
-    attn_ms = [a.elapsed_time(b) for a, b in ev]
-    ret_ms = [a.elapsed_time(b) for a, b in ev_ret]
-    tree_ms = [a.elapsed_time(b) for a, b in ev_tree]
-    tail_ms = [a.elapsed_time(b) for a, b in ev_tail]
+    stage_ms = {k: [[a.elapsed_time(b) for a, b in (stage_ev[i][h][k] for h in range(nsub))] for i in range(K)]
+                for k in ("attn", "retrieve", "tree", "tail")}  # [K][nsub] per stage
+    attn_ms = stage_ms["attn"]
 
     # replay the same (deterministic) trajectory untimed to count the
     # attention work of every timed launch
-    flops, bytes_, nodes_hist, acc_hist, hits_used = replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K, weights)
+    flops_seq, bytes_seq, nodes_hist, acc_hist, hits_used = replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K,
+                                                                          weights, nsub)
+    sub = [slice(B * h // nsub, B * (h + 1) // nsub) for h in range(nsub)]
 
     peaks = load_peaks()
-    per_launch = []
+    per_launch = []  # one attention launch per timed step and sub-batch
     for i in range(K):
-        t = attn_ms[i] * 1e-3
-        per_launch.append((flops[i], bytes_[i], t))
+        for h in range(nsub):
+            per_launch.append((float(flops_seq[i][sub[h]].sum()), float(bytes_seq[i][sub[h]].sum()),
+                               attn_ms[i][h] * 1e-3))
     tot_f = sum(f for f, _, _ in per_launch)
     tot_b = sum(b for _, b, _ in per_launch)
     tot_t = sum(t for _, _, t in per_launch)
+    n_launch = len(per_launch)
     t_tc = tot_f / (peaks["tc_sustained"] * 1e12)
     t_hbm = tot_b / (peaks["hbm"] * 1e9)
     if t_tc >= t_hbm:
@@ -374,12 +393,13 @@ def run_ours(args, rank, ws, local):
     else:
         roof = dict(bound="hbm", achieved=tot_b / tot_t / 1e9, peak=peaks["hbm"], unit="GB/s")
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = attn_traffic(args) if args.scale == 1.0 else args.traffic_bytes
+    roof["traffic"] = attn_traffic(args, nsub) if args.scale == 1.0 else args.traffic_bytes
     roof["peak_source"] = peaks["source"] + (" sustained bf16" if roof["bound"] == "tensor" else " hbm copy")
     roof["kernel"] = "k_tree_attn"
-    roof["mean_launch_us"] = 1e6 * tot_t / K
-    roof["algorithmic_flops_per_launch"] = tot_f / K
-    roof["algorithmic_bytes_per_launch"] = tot_b / K
+    roof["mean_launch_us"] = 1e6 * tot_t / n_launch
+    roof["algorithmic_flops_per_launch"] = tot_f / n_launch
+    roof["algorithmic_bytes_per_launch"] = tot_b / n_launch
+    roof["launches_per_step"] = nsub
     roof["other_bound_frac"] = (t_hbm if roof["bound"] == "tensor" else t_tc) / tot_t
 
     out = {
@@ -391,13 +411,17 @@ def run_ours(args, rank, ws, local):
                    + ("" if weights == [1, 1] else f", source weights alpha={weights[0]} beta={weights[1]}"),
                    "batch_per_gpu": B, "global_batch": B * ws, "kv_len0": kv0, "n_pad": n_pad,
                    "l2": "inputs larger than L2 (KV cache %.1f GB per GPU)" % (2 * kc.numel() * 2 / 1e9),
-                   "parallelism": f"replicas x{ws}"},
+                   "parallelism": f"replicas x{ws}",
+                   "streams": f"{nsub} sub-batches of {B // nsub}-{-(-B // nsub)} sequences, one CUDA stream each"},
         "roofline": roof,
-        "gpu_launches": 8 * K,
+        "gpu_launches": 8 * K * nsub,
         "clocks": clock_rec,
-        "stages_ms_per_step": {"tree_attn": statistics.mean(attn_ms), "retrieve": statistics.mean(ret_ms),
-                               "build_tree": statistics.mean(tree_ms),
-                               "argmax_accept_append": statistics.mean(tail_ms), "all": t_ms / K},
+        # each stage's mean time per sub-batch launch; with sub-batches on separate
+        # streams the stages of different sub-batches overlap, so they do not add up to "all"
+        "sub_batches": nsub,
+        "stages_ms_per_step": {"tree_attn": mean2(attn_ms), "retrieve": mean2(stage_ms["retrieve"]),
+                               "build_tree": mean2(stage_ms["tree"]),
+                               "argmax_accept_append": mean2(stage_ms["tail"]), "all": t_ms / K},
         "queries_per_s": ws * B * K / (t_max * 1e-3),
         "retrievals_per_s": ws * (2 * (B * K - hits_used)) / (t_max * 1e-3),
         "tree_attn_tflops": tot_f / tot_t / 1e12,
@@ -408,6 +432,13 @@ def run_ours(args, rank, ws, local):
         "tree_nodes_bins": np.bincount((np.concatenate(nodes_hist) - 1) // 32, minlength=n_pad // 32).tolist(),
         "datastore_build": {"tokens": build_tokens, "seconds": build_s, "tokens_per_s": build_tokens / build_s},
     }
+    if nsub > 1:
+        # the attention kernel alone on the step loop's launches: the same
+        # trajectory on one stream (its launches share the GPU with nothing), for
+        # the kernel's own roofline beside the pipelined step's
+        out["attn_single_stream"] = single_stream_attn(
+            sources, inp, p, cfg, cap, kv0, dev, weights, kc, vc, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P,
+            W, min(K, 64), flops_seq, bytes_seq, peaks, roof["bound"])
     if not args.no_e2e:
         loop.reset()
         out["e2e"] = run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws)
@@ -456,17 +487,60 @@ def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W,
             "note": "two steps per graph replay; the step's small draws copied in before each replay"}
 
 
-def replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K, weights=(1, 1)):
-    """Re-run the loop (untimed, fresh state) and count per-launch attention
-    work: FLOPs over unmasked (q, k) pairs and algorithmic HBM bytes."""
+def single_stream_attn(sources, inp, p, cfg, cap, kv0, dev, weights, kc, vc, q_pool, kt_pool, vt_pool, hits_d, plen_d,
+                       rtok_d, P, W, K2, flops_seq, bytes_seq, peaks, bound):
+    """Per-launch attention roofline of the first K2 timed steps run on one
+    stream (the step loop over the whole batch), from the same starting state."""
     import torch
 
     import paper_2502_17139_gb300.synth as synth
     from paper_2502_17139_gb300.step import StepLoop
+    kc[:, :, kv0:].zero_()
+    vc[:, :, kv0:].zero_()
+    lp = StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], cfg["n_pad"], weights, cfg["H"], cfg["Hkv"],
+                  cfg["D"], cap, kv0, synth.VOCAB, cache_capacity=1 << 14, device=dev, k_cache=kc, v_cache=vc)
+    mk = lambda: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    no_hit = torch.zeros_like(hits_d[0])
+    for s in range(W + K2):  # recording pass, as in the timed run
+        lp.step(q_pool[s % P], kt_pool[s % P], vt_pool[s % P], no_hit, plen_d[s], rtok_d[s])
+    lp.reset()
+    evs = []
+    for s in range(W + K2):
+        e = dict(attn=mk()) if s >= W else None
+        lp.step(q_pool[s % P], kt_pool[s % P], vt_pool[s % P], hits_d[s], plen_d[s], rtok_d[s], events=e)
+        if e:
+            evs.append(e["attn"])
+    torch.cuda.synchronize()
+    t = sum(a.elapsed_time(b) for a, b in evs) * 1e-3
+    f = sum(float(flops_seq[i].sum()) for i in range(K2))
+    by = sum(float(bytes_seq[i].sum()) for i in range(K2))
+    if bound == "tensor":
+        ach, peak, unit = f / t / 1e12, peaks["tc_sustained"], "TFLOP/s"
+    else:
+        ach, peak, unit = by / t / 1e9, peaks["hbm"], "GB/s"
+    return {"steps": K2, "mean_launch_us": 1e6 * t / K2, "achieved": ach, "peak": peak, "unit": unit,
+            "frac": ach / peak}
+
+
+def mean2(rows):
+    return float(np.mean(np.asarray(rows, np.float64)))
+
+
+def replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K, weights=(1, 1), nsub=1):
+    """Re-run the loop (untimed, fresh state, the same sub-batches) and count
+    the attention work of every timed step per sequence: FLOPs over unmasked
+    (q, k) pairs and algorithmic HBM bytes ([K] arrays over the batch)."""
+    import torch
+
+    import paper_2502_17139_gb300.synth as synth
+    from paper_2502_17139_gb300.step import PipelinedStepLoop, StepLoop
     B, H, Hkv, D, n_pad = inp["B"], cfg["H"], cfg["Hkv"], cfg["D"], cfg["n_pad"]
     kc = torch.zeros((B, Hkv, cap, D), dtype=torch.bfloat16, device=dev)
-    loop = StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, list(weights), H, Hkv, D, cap, kv0,
-                    synth.VOCAB, cache_capacity=1 << 14, device=dev, k_cache=kc, v_cache=kc)
+    largs = (sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, list(weights), H, Hkv, D, cap, kv0,
+             synth.VOCAB)
+    lkw = dict(cache_capacity=1 << 14, device=dev, k_cache=kc, v_cache=kc)
+    loop = PipelinedStepLoop(nsub, *largs, **lkw) if nsub > 1 else StepLoop(*largs, **lkw)
+    join = loop.join if nsub > 1 else (lambda: None)
     q = torch.zeros((B, n_pad, H, D), dtype=torch.bfloat16, device=dev)
     kt = torch.zeros((B, Hkv, n_pad, D), dtype=torch.bfloat16, device=dev)
     to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).to(dev)
@@ -477,21 +551,21 @@ def replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K, weights=(1, 1)):
         loop.step(q, kt, kt, zero, to_dev(inp["plen"][s]), to_dev(inp["rtok"][s]), attention=False)
     loop.reset()
     for s in range(W + K):
+        join()
         kvl = loop.kv_len_now.cpu().numpy().astype(np.int64)
         loop.step(q, kt, kt, to_dev(inp["hits"][s]), to_dev(inp["plen"][s]), to_dev(inp["rtok"][s]), attention=False)
+        join()
         if s < W:
             continue
         nn = loop.tree["n_nodes"].cpu().numpy().astype(np.int64)
         dep = loop.tree["depth"].cpu().numpy().astype(np.int64)
-        pairs = sum(H * (nn[b] * kvl[b] + int((dep[b, :nn[b]] + 1).sum())) for b in range(B))
+        pairs = np.array([H * (nn[b] * kvl[b] + int((dep[b, :nn[b]] + 1).sum())) for b in range(B)], np.float64)
         flops.append(4.0 * D * pairs)
-        by = 0
-        for b in range(B):
-            by += 2 * Hkv * kvl[b] * D * 2          # K and V cache rows
-            by += 2 * Hkv * nn[b] * D * 2           # tree K and V
-            by += 2 * nn[b] * H * D * 2             # Q in, O out
-            by += nn[b] * (n_pad // 64) * 8         # mask rows
-        bytes_.append(float(by))
+        by = (2 * Hkv * kvl * D * 2          # K and V cache rows
+              + 2 * Hkv * nn * D * 2         # tree K and V
+              + 2 * nn * H * D * 2           # Q in, O out
+              + nn * (n_pad // 64) * 8)      # mask rows
+        bytes_.append(by.astype(np.float64))
         nodes_hist.append(nn)
         acc_hist.append(loop.acc["acc_len"].cpu().numpy())
         hits_used += int(loop.skip.sum().item())
@@ -520,16 +594,21 @@ def run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws):
     res = torch.empty((2, B), dtype=torch.int32).pin_memory()
     main = torch.cuda.current_stream()
     cs = torch.cuda.Stream()
+    # (loop, sequences, stream) per sub-batch: a pipelined loop's sub-batches
+    # read the inputs and write the results on their own streams
+    subs = list(zip(loop.loops, loop.slices, loop.streams)) if hasattr(loop, "loops") else [(loop, slice(0, B), main)]
     copied = [torch.cuda.Event() for _ in range(2)]
-    consumed = [torch.cuda.Event() for _ in range(2)]
-    for e in consumed:
-        e.record(main)
+    consumed = [[torch.cuda.Event() for _ in subs] for _ in range(2)]
+    for evs in consumed:
+        for e in evs:
+            e.record(main)
 
     def copy_in(s):
         slot, j = s % 2, s % R
         d = sets[slot]
         with torch.cuda.stream(cs):
-            cs.wait_event(consumed[slot])
+            for e in consumed[slot]:
+                cs.wait_event(e)
             d["q"].copy_(hq[j], non_blocking=True)
             d["k"].copy_(hk[j], non_blocking=True)
             d["v"].copy_(hv[j], non_blocking=True)
@@ -547,9 +626,11 @@ def run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws):
             d = sets[slot]
             main.wait_event(copied[slot])
             loop.step(d["q"], d["k"], d["v"], d["h"], d["p"], d["r"])
-            consumed[slot].record(main)
-            res[0].copy_(loop.acc["acc_len"], non_blocking=True)
-            res[1].copy_(loop.acc["bonus"], non_blocking=True)
+            for h, (lp, sl, st) in enumerate(subs):
+                with torch.cuda.stream(st):
+                    consumed[slot][h].record(st)
+                    res[0][sl].copy_(lp.acc["acc_len"], non_blocking=True)
+                    res[1][sl].copy_(lp.acc["bonus"], non_blocking=True)
 
     run(0, W)
     torch.cuda.synchronize()

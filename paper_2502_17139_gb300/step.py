@@ -210,3 +210,116 @@ class StepLoop:
     @property
     def ctx_len_now(self):
         return self.ctx_len[self.cur]
+
+
+class PipelinedStepLoop:
+    """The step loop over sub-batches of the sequences, each on its own CUDA
+    stream.
+
+    The sequences of a batch are independent, so sub-batch h can run step
+    s + 1 while sub-batch h' is still in step s. Then one sub-batch's small,
+    latency-bound kernels (retrieval, tree build, acceptance, append) run on
+    the SMs that the other's attention launch leaves idle in its last wave;
+    an SM that holds an attention CTA has no room for any other CTA.  Each
+    sub-batch is a StepLoop over a slice of the sequences.  They share the
+    datastores and slices of one pair of KV caches, and every per-sequence
+    result is the single loop's.  The replay cache is per sub-batch; it
+    replays deterministic retrieval results, so that changes no output.
+
+    step() makes every sub-batch stream wait for the work already enqueued
+    on the caller's stream, so inputs written there are visible.  It does not
+    make the caller's stream wait for the sub-batches, or they could not
+    overlap; join() does that, and must precede any read of the results on
+    the caller's stream.  Only the replay-cache configuration (with optional
+    RoPE) is pipelined; Algorithm 1's missing table is shared by the whole
+    batch, so it stays with StepLoop."""
+
+    def __init__(self, n_split, sources, ctx, ctx_len, p, node_budget, n_pad, src_weight, H, Hkv, D, kv_cap,
+                 kv_len0, vocab, cache_capacity=1 << 14, device="cuda", k_cache=None, v_cache=None, rope_base=None):
+        B = ctx.shape[0]
+        if not 1 <= n_split <= B:
+            raise ValueError("n_split must be between 1 and the batch size")
+        edges = [B * h // n_split for h in range(n_split + 1)]
+        self.slices = [slice(edges[h], edges[h + 1]) for h in range(n_split)]
+        self.B = B
+        shape = (B, Hkv, kv_cap, D)
+        self.k_cache = k_cache if k_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
+        self.v_cache = v_cache if v_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
+        kv0 = np.broadcast_to(np.asarray(kv_len0, np.int32), (B,))
+        self.loops = [StepLoop(sources, ctx[sl], ctx_len[sl], p, node_budget, n_pad, src_weight, H, Hkv, D, kv_cap,
+                               kv0[sl], vocab, cache_capacity=cache_capacity, device=device,
+                               k_cache=self.k_cache[sl], v_cache=self.v_cache[sl], rope_base=rope_base)
+                      for sl in self.slices]
+        self.streams = [torch.cuda.Stream(device=device) for _ in self.slices]
+        self._start = torch.cuda.Event()
+        self._done = [torch.cuda.Event() for _ in self.slices]
+
+    def step(self, q, k_tree, v_tree, want_hit, plen, rtok, attention=True, events=None):
+        """Enqueue one step of every sub-batch (arguments as StepLoop.step,
+        for the whole batch); ``events``: None or one StepLoop events dict per
+        sub-batch, recorded on its stream."""
+        self._start.record()
+        cut = lambda t, sl: None if t is None else t[sl]
+        for h, (lp, sl, st) in enumerate(zip(self.loops, self.slices, self.streams)):
+            st.wait_event(self._start)
+            with torch.cuda.stream(st):
+                lp.step(cut(q, sl), cut(k_tree, sl), cut(v_tree, sl), want_hit[sl], plen[sl], rtok[sl],
+                        attention=attention, events=None if events is None else events[h])
+
+    def join(self):
+        """The caller's current stream waits for everything enqueued so far."""
+        cur = torch.cuda.current_stream()
+        for ev, st in zip(self._done, self.streams):
+            ev.record(st)
+            cur.wait_event(ev)
+
+    def capture(self, inputs, attention=True):
+        """Two steps of every sub-batch in one CUDA graph (fork and join
+        inside it); as StepLoop.capture."""
+        if any(lp.cur != 0 for lp in self.loops):
+            raise RuntimeError("capture at an even step")
+        self.join()  # no eager work may still be pending on the streams the graph forks to
+        torch.cuda.current_stream().synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            self.step(*inputs[0], attention=attention)
+            self.step(*inputs[1], attention=attention)
+            self.join()
+        return g
+
+    def reset(self):
+        self.join()
+        for lp in self.loops:
+            lp.reset()
+
+    # gathered copies over the whole batch (they allocate; call after join())
+    def _cat(self, get):
+        return torch.cat([get(lp) for lp in self.loops])
+
+    @property
+    def kv_len_now(self):
+        return self._cat(lambda lp: lp.kv_len_now)
+
+    @property
+    def ctx_len_now(self):
+        return self._cat(lambda lp: lp.ctx_len_now)
+
+    @property
+    def ctx(self):
+        return self._cat(lambda lp: lp.ctx)
+
+    @property
+    def acc(self):
+        return {k: self._cat(lambda lp, k=k: lp.acc[k]) for k in self.loops[0].acc}
+
+    @property
+    def tree(self):
+        return {k: self._cat(lambda lp, k=k: lp.tree[k]) for k in self.loops[0].tree}
+
+    @property
+    def skip(self):
+        return self._cat(lambda lp: lp.skip)
+
+    @property
+    def attn_out(self):
+        return self._cat(lambda lp: lp.attn_out)

@@ -1,0 +1,118 @@
+"""The step loop over sub-batches on separate streams (PipelinedStepLoop):
+every per-sequence result equals the single loop's (contexts, lengths, trees,
+acceptance and cache rows bit-exact, attention within max-abs 2e-2), for two
+and three sub-batches of unequal size, and a CUDA graph of two pipelined steps
+(fork and join inside the graph) replays the eager pipelined trajectory."""
+import numpy as np
+import pytest
+import torch
+
+import paper_2502_17139_gb300.synth as synth
+
+pytestmark = pytest.mark.gpu
+ATOL = 2e-2
+
+
+@pytest.fixture(scope="module")
+def fc():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2502_17139_gb300 import build
+    build.build()
+    import paper_2502_17139_gb300.fastcoder as fcm
+    return fcm
+
+
+def dev(a):
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint32:
+        a = a.view(np.int32)
+    return torch.from_numpy(a.copy()).cuda()
+
+
+@pytest.fixture(scope="module")
+def setup(fc):
+    rng = synth.rng_for(77)
+    Tr, _ = synth.make_corpus(rng, 200_000, 1.3, synth.VOCAB, n_grams=500, len_range=(8, 64))
+    Tc, _ = synth.make_corpus(rng, 1_000_000, 1.1, synth.VOCAB)
+    B, steps, n_pad, H, Hkv, D, kv0 = 9, 10, 128, 8, 2, 128, 100
+    stride = 128 + steps * 12
+    ctx, cl, _ = synth.make_contexts(rng, B, 128, 16, [Tr, Tc, None], [0.5, 0.25, 0.25], 1.1, ctx_stride=stride)
+    hits = synth.cache_hit_pattern(rng, steps, B)
+    draws = [synth.argmax_draws(rng, B, n_pad) for _ in range(steps)]
+    srcs = [fc.fc_datastore_build(dev(Tr), synth.VOCAB), fc.fc_datastore_build(dev(Tc), synth.VOCAB)]
+    ins = [(synth.randn_bf16((B, n_pad, H, D), 10 + s, "cuda"), synth.randn_bf16((B, Hkv, n_pad, D), 40 + s, "cuda"),
+            synth.randn_bf16((B, Hkv, n_pad, D), 70 + s, "cuda"), dev(hits[s]), dev(draws[s][0]), dev(draws[s][1]))
+           for s in range(steps)]
+    args = (srcs, ctx, cl, fc.params(16, 2, 64, 10, 4096), n_pad, n_pad, [1, 1], H, Hkv, D)
+    kw = dict(kv_cap=kv0 + steps * 12, kv_len0=kv0, vocab=synth.VOCAB)
+    return dict(args=args, kw=kw, ins=ins, steps=steps)
+
+
+def state(loop):
+    s = dict(ctx=loop.ctx, cl=loop.ctx_len_now, kv=loop.kv_len_now, kc=loop.k_cache, vc=loop.v_cache)
+    s.update({"acc_" + k: v for k, v in loop.acc.items()})
+    s.update({"tree_" + k: v for k, v in loop.tree.items()})
+    out = {k: v.cpu().clone() for k, v in s.items()}
+    out["attn"] = loop.attn_out.float().cpu().clone()
+    return out
+
+
+def same(a, b):
+    for k in a:
+        if k == "attn":
+            assert (a[k] - b[k]).abs().max().item() <= ATOL, k
+        else:
+            assert torch.equal(a[k], b[k]), k
+
+
+@pytest.mark.parametrize("n_split", [2, 3])
+def test_pipelined_matches_single_loop(fc, setup, n_split):
+    from paper_2502_17139_gb300.step import PipelinedStepLoop, StepLoop
+    single = StepLoop(*setup["args"], **setup["kw"])
+    piped = PipelinedStepLoop(n_split, *setup["args"], **setup["kw"])
+    assert [sl.stop - sl.start for sl in piped.slices] == ([4, 5] if n_split == 2 else [3, 3, 3])
+    for s in range(setup["steps"]):
+        single.step(*setup["ins"][s])
+        piped.step(*setup["ins"][s])
+        piped.join()
+        same(state(single), state(piped))
+    assert fc.fc_get_error() == "FC_OK"
+    # reset replays the same trajectory
+    piped.reset()
+    for s in range(2):
+        piped.step(*setup["ins"][s])
+    piped.join()
+    single.reset()
+    for s in range(2):
+        single.step(*setup["ins"][s])
+    same(state(single), state(piped))
+
+
+def test_pipelined_graph_replay(fc, setup):
+    from paper_2502_17139_gb300.step import PipelinedStepLoop
+    ins, steps = setup["ins"], setup["steps"]
+    eager = PipelinedStepLoop(2, *setup["args"], **setup["kw"])
+    want = []
+    for s in range(steps):
+        eager.step(*ins[s])
+        if s % 2 == 1:
+            eager.join()
+            want.append(state(eager))
+    graphed = PipelinedStepLoop(2, *setup["args"], **setup["kw"])
+    graphed.step(*ins[0])
+    graphed.step(*ins[1])
+    graphed.join()
+    static = [tuple(t.clone() for t in ins[2]), tuple(t.clone() for t in ins[3])]
+    g = graphed.capture(static)
+    got = []
+    for s in range(2, steps, 2):
+        for j in range(2):
+            for dst, src in zip(static[j], ins[s + j]):
+                dst.copy_(src)
+        g.replay()
+        got.append(state(graphed))
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_OK"
+    for w, gt in zip(want[1:], got):
+        same(w, gt)
