@@ -591,12 +591,14 @@ def run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws):
     sets = [dict(q=torch.empty_like(q_pool[0]), k=torch.empty_like(kt_pool[0]), v=torch.empty_like(vt_pool[0]),
                  h=torch.empty(B, dtype=torch.int32, device=dev), p=torch.empty(B, dtype=torch.int32, device=dev),
                  r=torch.empty(inp["rtok"].shape[1:], dtype=torch.int32, device=dev)) for _ in range(2)]
-    res = torch.empty((2, B), dtype=torch.int32).pin_memory()
     main = torch.cuda.current_stream()
     cs = torch.cuda.Stream()
     # (loop, sequences, stream) per sub-batch: a pipelined loop's sub-batches
-    # read the inputs and write the results on their own streams
+    # read the inputs and write the results on their own streams, each into its
+    # own pinned buffer (a copy into a slice of one buffer at an odd offset is
+    # not asynchronous)
     subs = list(zip(loop.loops, loop.slices, loop.streams)) if hasattr(loop, "loops") else [(loop, slice(0, B), main)]
+    res = [torch.empty((2, sl.stop - sl.start), dtype=torch.int32).pin_memory() for _, sl, _ in subs]
     copied = [torch.cuda.Event() for _ in range(2)]
     consumed = [[torch.cuda.Event() for _ in subs] for _ in range(2)]
     for evs in consumed:
@@ -629,8 +631,8 @@ def run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws):
             for h, (lp, sl, st) in enumerate(subs):
                 with torch.cuda.stream(st):
                     consumed[slot][h].record(st)
-                    res[0][sl].copy_(lp.acc["acc_len"], non_blocking=True)
-                    res[1][sl].copy_(lp.acc["bonus"], non_blocking=True)
+                    res[h][0].copy_(lp.acc["acc_len"], non_blocking=True)
+                    res[h][1].copy_(lp.acc["bonus"], non_blocking=True)
 
     run(0, W)
     torch.cuda.synchronize()
@@ -642,7 +644,7 @@ def run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws):
     d = sets[0]
     h2d = d["q"].numel() * 2 + d["k"].numel() * 2 + d["v"].numel() * 2 + 4 * (2 * B + d["r"].numel())
     return {"value": weak_value(K, ws, t * 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(res.numel() * 4),
+            "d2h_bytes_per_step": int(sum(r.numel() for r in res) * 4),
             "note": "host->device copies on a second stream, double-buffered: step s + 1's inputs travel while "
                     "step s computes"}
 

@@ -479,6 +479,15 @@ def test_attn_c5_shape_sampled(fc, orc):
     _attn_case(fc, orc, 6, 32, 128, 32, 8, [16384] * 32, 16384 + 256, full_rows=False, sample=160)
 
 
+def test_attn_c5_subbatch_sampled(fc, orc):
+    # the launch the step bench times: one sub-batch of 16 sequences (256 CTAs,
+    # 1.7 waves, no KV split), KV lengths grown over the steps, trees of every size
+    rng = synth.rng_for(53)
+    kvl = [16384 + int(x) for x in rng.integers(0, 700, 16)]
+    nn = [int(x) for x in rng.choice([1, 20, 40, 70, 97, 128], 16)]
+    _attn_case(fc, orc, 11, 16, 128, 32, 8, kvl, 16384 + 768, nn=nn, full_rows=False, sample=160)
+
+
 # ------------------------------------------------------- accept / append
 def test_accept_and_synth_argmax(fc, orc):
     rng = synth.rng_for(60)
