@@ -174,18 +174,21 @@ class StepLoop:
             ev["tail"][1].record()
 
     def capture(self, inputs, attention=True):
-        """Capture two consecutive steps into a CUDA graph.  ``inputs`` holds
-        two tuples (q, k_tree, v_tree, want_hit, plen, rtok) of device tensors
-        that the graph reads at every replay (update them in place between
-        replays).  Call with the loop at an even step, after one eager pair of
-        steps so that lazily made workspaces and kernel attributes exist.
-        Each replay advances the loop by two steps."""
+        """Capture consecutive steps into a CUDA graph.  ``inputs`` holds an
+        even number of tuples (q, k_tree, v_tree, want_hit, plen, rtok) of
+        device tensors, one per step, that the graph reads at every replay
+        (update them in place between replays).  Call with the loop at an even
+        step, after one eager pair of steps so that lazily made workspaces and
+        kernel attributes exist.  Each replay advances the loop by
+        len(inputs) steps."""
         if self.cur != 0:
             raise RuntimeError("capture at an even step")
+        if len(inputs) < 2 or len(inputs) % 2:
+            raise ValueError("capture an even number of steps (the lengths alternate between two buffers)")
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, capture_error_mode="thread_local"):
-            self.step(*inputs[0], attention=attention)
-            self.step(*inputs[1], attention=attention)
+            for ins in inputs:
+                self.step(*ins, attention=attention)
         return g
 
     def reset(self):
@@ -274,16 +277,19 @@ class PipelinedStepLoop:
             cur.wait_event(ev)
 
     def capture(self, inputs, attention=True):
-        """Two steps of every sub-batch in one CUDA graph (fork and join
-        inside it); as StepLoop.capture."""
+        """An even number of steps of every sub-batch in one CUDA graph (fork
+        and join inside it); as StepLoop.capture.  The sub-batches rejoin only
+        at the end of the graph."""
         if any(lp.cur != 0 for lp in self.loops):
             raise RuntimeError("capture at an even step")
+        if len(inputs) < 2 or len(inputs) % 2:
+            raise ValueError("capture an even number of steps (the lengths alternate between two buffers)")
         self.join()  # no eager work may still be pending on the streams the graph forks to
         torch.cuda.current_stream().synchronize()
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, capture_error_mode="thread_local"):
-            self.step(*inputs[0], attention=attention)
-            self.step(*inputs[1], attention=attention)
+            for ins in inputs:
+                self.step(*ins, attention=attention)
             self.join()
         return g
 
