@@ -116,3 +116,22 @@ def test_pipelined_graph_replay(fc, setup):
     assert fc.fc_get_error() == "FC_OK"
     for w, gt in zip(want[1:], got):
         same(w, gt)
+
+
+def test_pipelined_one_sequence_per_sub_batch(fc, setup):
+    """As many sub-batches as sequences (nine streams of one sequence each), and
+    the bounds of n_split."""
+    from paper_2502_17139_gb300.step import PipelinedStepLoop, StepLoop
+    B = setup["args"][1].shape[0]
+    with pytest.raises(ValueError):
+        PipelinedStepLoop(0, *setup["args"], **setup["kw"])
+    with pytest.raises(ValueError):
+        PipelinedStepLoop(B + 1, *setup["args"], **setup["kw"])
+    single = StepLoop(*setup["args"], **setup["kw"])
+    piped = PipelinedStepLoop(B, *setup["args"], **setup["kw"])
+    for s in range(4):
+        single.step(*setup["ins"][s])
+        piped.step(*setup["ins"][s])
+    piped.join()
+    same(state(single), state(piped))
+    assert fc.fc_get_error() == "FC_OK"
