@@ -483,8 +483,9 @@ def attn_workspace(B, Np, H, Hkv, device):
 def fc_tree_attn(q, k_cache, v_cache, kv_len, k_tree, v_tree, mask, n_nodes, scale=None, out=None, workspace="auto"):
     """q [B, Np, H, D]; caches [B, Hkv, cap, D]; tree K/V [B, Hkv, Np, D] (bf16).
 
-    ``workspace``: "auto" (a cached one of the full size), None (no key
-    split) or a uint8 device tensor."""
+    ``workspace``: "auto" (a cached one of the full size, shared by every call
+    with that size: calls that may overlap on different streams must each pass
+    their own), None (no key split) or a uint8 device tensor."""
     _need(q, torch.bfloat16, "q")
     B, Np, H, D = q.shape
     _need(k_cache, torch.bfloat16, "k_cache")

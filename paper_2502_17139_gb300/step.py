@@ -72,6 +72,10 @@ class StepLoop:
         self.k_cache = k_cache if k_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         self.v_cache = v_cache if v_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         self.attn_out = torch.empty((B, n_pad, H, D), dtype=torch.bfloat16, device=device)
+        # the attention's own workspace (KV-split partials and counters): loops whose
+        # steps overlap on different streams must not share one
+        self.attn_ws = torch.empty(max(int(fc.LIB.fc_tree_attn_workspace(B, n_pad, H, Hkv)), 16), dtype=torch.uint8,
+                                   device=device)
         self.rope_base = rope_base
         self.decoder = decoder
         self.k_tree_rot = (torch.empty((B, Hkv, n_pad, D), dtype=torch.bfloat16, device=device)
@@ -131,10 +135,11 @@ class StepLoop:
                 ev["attn"][0].record()
             if self.rope_base is not None:
                 fc.fc_tree_attn_rope(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree, self.tree["mask"],
-                                     self.tree["n_nodes"], self.tree["pos"], self.rope_base, out=self.attn_out)
+                                     self.tree["n_nodes"], self.tree["pos"], self.rope_base, out=self.attn_out,
+                                     workspace=self.attn_ws)
             else:
                 fc.fc_tree_attn(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree, self.tree["mask"],
-                                self.tree["n_nodes"], out=self.attn_out)
+                                self.tree["n_nodes"], out=self.attn_out, workspace=self.attn_ws)
             if "attn" in ev:
                 ev["attn"][1].record()
         if "tail" in ev:

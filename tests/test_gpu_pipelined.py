@@ -135,3 +135,38 @@ def test_pipelined_one_sequence_per_sub_batch(fc, setup):
     piped.join()
     same(state(single), state(piped))
     assert fc.fc_get_error() == "FC_OK"
+
+
+def test_pipelined_kv_split_workspaces(fc):
+    """Two sub-batches whose attention launches both split their last wave's
+    KV blocks over several CTAs (10 sequences x 8 kv heads x 2 row chunks =
+    160 units on 152 SMs) while they overlap: each sub-batch has its own
+    workspace, so the results equal the single loop's."""
+    from paper_2502_17139_gb300.step import PipelinedStepLoop, StepLoop
+    rng = synth.rng_for(78)
+    Tr, _ = synth.make_corpus(rng, 200_000, 1.3, synth.VOCAB, n_grams=500, len_range=(8, 64))
+    Tc, _ = synth.make_corpus(rng, 1_000_000, 1.1, synth.VOCAB)
+    B, steps, n_pad, H, Hkv, D, kv0 = 20, 4, 128, 32, 8, 128, 4000
+    ctx, cl, _ = synth.make_contexts(rng, B, 128, 16, [Tr, Tc, None], [0.5, 0.25, 0.25], 1.1, ctx_stride=128 + 60)
+    hits = synth.cache_hit_pattern(rng, steps, B)
+    draws = [synth.argmax_draws(rng, B, n_pad) for _ in range(steps)]
+    srcs = [fc.fc_datastore_build(dev(Tr), synth.VOCAB), fc.fc_datastore_build(dev(Tc), synth.VOCAB)]
+    ins = [(synth.randn_bf16((B, n_pad, H, D), 110 + s, "cuda"), synth.randn_bf16((B, Hkv, n_pad, D), 140 + s, "cuda"),
+            synth.randn_bf16((B, Hkv, n_pad, D), 170 + s, "cuda"), dev(hits[s]), dev(draws[s][0]), dev(draws[s][1]))
+           for s in range(steps)]
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    cap = kv0 + steps * 12
+    assert fc.LIB.fc_tree_attn_parts(B // 2, n_pad, H, Hkv, cap, int(fc.LIB.fc_tree_attn_workspace(B // 2, n_pad, H, Hkv))) > 1 \
+        or (B // 2) * Hkv * 2 <= sms  # the split is active on a 152-SM part
+    args = (srcs, ctx, cl, fc.params(16, 2, 64, 10, 4096), n_pad, n_pad, [1, 1], H, Hkv, D)
+    kw = dict(kv_cap=cap, kv_len0=kv0, vocab=synth.VOCAB)
+    kc0 = synth.randn_bf16((B, Hkv, cap, D), 200, "cuda")
+    vc0 = synth.randn_bf16((B, Hkv, cap, D), 201, "cuda")
+    single = StepLoop(*args, **kw, k_cache=kc0.clone(), v_cache=vc0.clone())
+    piped = PipelinedStepLoop(2, *args, **kw, k_cache=kc0.clone(), v_cache=vc0.clone())
+    for s in range(steps):
+        single.step(*ins[s])
+        piped.step(*ins[s])
+        piped.join()
+        same(state(single), state(piped))
+    assert fc.fc_get_error() == "FC_OK"
