@@ -556,14 +556,17 @@ _GEMM_WS = {}
 
 
 def gemm_workspace(device):
+    """The cuBLASLt workspace fc_gemm_bf16 uses, one per device and shared by every
+    call: GEMMs that may overlap on different streams need their own."""
     key = str(device)
     if key not in _GEMM_WS:
         _GEMM_WS[key] = torch.empty(int(LIB.fc_gemm_workspace()), dtype=torch.uint8, device=device)
     return _GEMM_WS[key]
 
 
-def fc_gemm_bf16(a, b, out=None):
-    """a [M, K] @ b [K, N] (bf16, row-major) -> [M, N] bf16."""
+def fc_gemm_bf16(a, b, out=None, workspace=None):
+    """a [M, K] @ b [K, N] (bf16, row-major) -> [M, N] bf16.  ``workspace``:
+    None (the shared per-device one) or a uint8 device tensor."""
     _need(a, torch.bfloat16, "a")
     _need(b, torch.bfloat16, "b")
     M, K = a.shape
@@ -571,7 +574,7 @@ def fc_gemm_bf16(a, b, out=None):
     if K != K2:
         raise ValueError("inner dimensions differ")
     o = out if out is not None else torch.empty((M, N), dtype=torch.bfloat16, device=a.device)
-    ws = gemm_workspace(a.device)
+    ws = workspace if workspace is not None else gemm_workspace(a.device)
     _check("fc_gemm_bf16", LIB.fc_gemm_bf16(_ptr(a), _ptr(b), _ptr(o), M, N, K, _ptr(ws), ws.numel(), _stream()))
     return o
 
