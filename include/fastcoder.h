@@ -70,7 +70,10 @@ const char* fc_version(void);
 /*
  * Waits for the stream, then returns and clears the device error word
  * (the most severe device-detected error since the last call, or FC_OK).
- * Synchronous.
+ * Synchronous.  The word is shared by every stream of the process: with
+ * work on several streams, have s wait for them first (or synchronize the
+ * device), or an error recorded later on another stream is missed by this
+ * call and reported by the next.
  */
 fc_status fc_get_error(fc_stream s);
 
