@@ -72,6 +72,10 @@ class StepLoop:
         self.k_cache = k_cache if k_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         self.v_cache = v_cache if v_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         self.attn_out = torch.empty((B, n_pad, H, D), dtype=torch.bfloat16, device=device)
+        # optional: a stream of its own for the attention launch (the step's other
+        # work waits for it through an event)
+        self.attn_stream = None
+        self._ev_pre, self._ev_post = torch.cuda.Event(), torch.cuda.Event()
         # the attention's own workspace (KV-split partials and counters): loops whose
         # steps overlap on different streams must not share one
         self.attn_ws = torch.empty(max(int(fc.LIB.fc_tree_attn_workspace(B, n_pad, H, Hkv)), 16), dtype=torch.uint8,
@@ -131,6 +135,12 @@ class StepLoop:
         if self.rope_base is not None:
             k_tree = fc.fc_rope(k_tree, self.tree["pos"], self.rope_base, layout=1, out=self.k_tree_rot)
         if attention:
+            side = self.attn_stream
+            if side is not None:  # the attention on its own stream, ordered by events
+                self._ev_pre.record()
+                side.wait_event(self._ev_pre)
+                ctx_mgr = torch.cuda.stream(side)
+                ctx_mgr.__enter__()
             if "attn" in ev:
                 ev["attn"][0].record()
             if self.rope_base is not None:
@@ -142,6 +152,10 @@ class StepLoop:
                                 self.tree["n_nodes"], out=self.attn_out, workspace=self.attn_ws)
             if "attn" in ev:
                 ev["attn"][1].record()
+            if side is not None:
+                self._ev_post.record(side)
+                ctx_mgr.__exit__(None, None, None)
+                torch.cuda.current_stream().wait_event(self._ev_post)
         if "tail" in ev:
             ev["tail"][0].record()
         fc.fc_synth_argmax(self.tree["tok"], self.tree["parent"], self.tree["n_nodes"], plen, rtok, self.vocab,
@@ -258,7 +272,13 @@ class PipelinedStepLoop:
                                kv0[sl], vocab, cache_capacity=cache_capacity, device=device,
                                k_cache=self.k_cache[sl], v_cache=self.v_cache[sl], rope_base=rope_base)
                       for sl in self.slices]
-        self.streams = [torch.cuda.Stream(device=device) for _ in self.slices]
+        # Each sub-batch's small kernels run on a high-priority stream and its
+        # attention on a low-priority one: when SMs free up, the block scheduler
+        # then starts the other sub-batch's latency-bound chain (retrieval, tree,
+        # acceptance) ahead of this sub-batch's remaining attention CTAs.
+        self.streams = [torch.cuda.Stream(device=device, priority=-1) for _ in self.slices]
+        for lp in self.loops:
+            lp.attn_stream = torch.cuda.Stream(device=device, priority=0)
         self._start = torch.cuda.Event()
         self._done = [torch.cuda.Event() for _ in self.slices]
 
