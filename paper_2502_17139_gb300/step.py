@@ -15,11 +15,15 @@ Retrieval takes one of two forms:
   * otherwise the context-keyed replay cache: lookup -> fc_retrieve on the
     queries it did not serve -> insert.
 
-Every call is asynchronous on the current stream and allocates nothing, so a
-step can be captured once into a CUDA graph and replayed (lengths ping-pong
-between two buffers, so a graph holds two consecutive steps).
+Every call is asynchronous on the current stream and allocates nothing, so
+steps can be captured once into a CUDA graph and replayed (lengths ping-pong
+between two buffers, so a graph holds an even number of consecutive steps).
+PipelinedStepLoop runs the step over sub-batches of the sequences on streams
+of their own.
 """
 from __future__ import annotations
+
+import contextlib
 
 import numpy as np
 import torch
@@ -139,22 +143,21 @@ class StepLoop:
             if side is not None:  # the attention on its own stream, ordered by events
                 self._ev_pre.record()
                 side.wait_event(self._ev_pre)
-                ctx_mgr = torch.cuda.stream(side)
-                ctx_mgr.__enter__()
-            if "attn" in ev:
-                ev["attn"][0].record()
-            if self.rope_base is not None:
-                fc.fc_tree_attn_rope(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree, self.tree["mask"],
-                                     self.tree["n_nodes"], self.tree["pos"], self.rope_base, out=self.attn_out,
-                                     workspace=self.attn_ws)
-            else:
-                fc.fc_tree_attn(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree, self.tree["mask"],
-                                self.tree["n_nodes"], out=self.attn_out, workspace=self.attn_ws)
-            if "attn" in ev:
-                ev["attn"][1].record()
+            with torch.cuda.stream(side) if side is not None else contextlib.nullcontext():
+                if "attn" in ev:
+                    ev["attn"][0].record()
+                if self.rope_base is not None:
+                    fc.fc_tree_attn_rope(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree,
+                                         self.tree["mask"], self.tree["n_nodes"], self.tree["pos"], self.rope_base,
+                                         out=self.attn_out, workspace=self.attn_ws)
+                else:
+                    fc.fc_tree_attn(q, self.k_cache, self.v_cache, self.kv_len[c], k_tree, v_tree, self.tree["mask"],
+                                    self.tree["n_nodes"], out=self.attn_out, workspace=self.attn_ws)
+                if "attn" in ev:
+                    ev["attn"][1].record()
+                if side is not None:
+                    self._ev_post.record(side)
             if side is not None:
-                self._ev_post.record(side)
-                ctx_mgr.__exit__(None, None, None)
                 torch.cuda.current_stream().wait_event(self._ev_post)
         if "tail" in ev:
             ev["tail"][0].record()
