@@ -237,6 +237,16 @@ class StepLoop:
         return self.ctx_len[self.cur]
 
 
+def sub_batch_slices(B, n_split):
+    """The sub-batches of a batch of B sequences: n_split contiguous slices, the
+    h-th ending at floor(B (h + 1) / n_split), so their sizes differ by at most
+    one."""
+    if not 1 <= n_split <= B:
+        raise ValueError("n_split must be between 1 and the batch size")
+    edges = [B * h // n_split for h in range(n_split + 1)]
+    return [slice(edges[h], edges[h + 1]) for h in range(n_split)]
+
+
 class PipelinedStepLoop:
     """The step loop over sub-batches of the sequences, each on its own CUDA
     stream.
@@ -262,10 +272,7 @@ class PipelinedStepLoop:
     def __init__(self, n_split, sources, ctx, ctx_len, p, node_budget, n_pad, src_weight, H, Hkv, D, kv_cap,
                  kv_len0, vocab, cache_capacity=1 << 14, device="cuda", k_cache=None, v_cache=None, rope_base=None):
         B = ctx.shape[0]
-        if not 1 <= n_split <= B:
-            raise ValueError("n_split must be between 1 and the batch size")
-        edges = [B * h // n_split for h in range(n_split + 1)]
-        self.slices = [slice(edges[h], edges[h + 1]) for h in range(n_split)]
+        self.slices = sub_batch_slices(B, n_split)
         self.B = B
         shape = (B, Hkv, kv_cap, D)
         self.k_cache = k_cache if k_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
