@@ -232,8 +232,8 @@ def max_over_ranks(x: float, ws: int) -> float:
 # --------------------------------------------------------------- workload
 def workload_spec(scale: float, batch: int):
     import paper_2502_17139_gb300.synth as synth
-    cfg = dict(synth.CONFIGS[5])
-    c2 = synth.CONFIGS[2]
+    cfg = dict(synth.WORKLOADS[5])
+    c2 = synth.WORKLOADS[2]
     corpora = [synth.scaled_corpus_spec(s, scale) for s in c2["corpus"]]
     kv = max(256, int(cfg["kv_len"] * scale))
     return cfg, corpora, kv, batch
@@ -998,7 +998,7 @@ def run_configs(args, rank, ws, local):
         return ds, {"tokens": int(len(T)), "seconds": sec, "tokens_per_s": len(T) / sec}
 
     # c1: single source 1M, B=32, attention H = Hkv = 32, KV 512
-    cfg = synth.CONFIGS[1]
+    cfg = synth.WORKLOADS[1]
     rng = synth.rng_for(1)
     T, _ = synth.build_corpus(rng, cfg["corpus"][0], device="cuda")
     ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], [T], [1.0], 1.1)
@@ -1010,7 +1010,7 @@ def run_configs(args, rank, ws, local):
                                 accept=accept_entry(tree, synth.VOCAB, 1))
     del ds, T
     # c2: two sources 5M + 100M, B=256, 64-node trees
-    cfg = synth.CONFIGS[2]
+    cfg = synth.WORKLOADS[2]
     rng = synth.rng_for(2)
     corpora = [synth.build_corpus(rng, spec, device="cuda")[0] for spec in cfg["corpus"]]
     ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], corpora + [None], cfg["probs"],
@@ -1020,7 +1020,7 @@ def run_configs(args, rank, ws, local):
     out["configs"]["c2"] = dict(datastore_build=[b[1] for b in built], retrieval_and_tree=e_ret)
     del built, corpora
     # c3: attention at the 7B shape, B=16, H = Hkv = 32, KV 4096, 64-node random trees; acceptance
-    cfg = synth.CONFIGS[3]
+    cfg = synth.WORKLOADS[3]
     rng = synth.rng_for(3)
     B, n_pad, nnod = cfg["batch"], cfg["n_pad"], cfg["n_nodes"]
     tok = np.full((B, n_pad), 0xFFFFFFFF, np.uint32)
@@ -1036,7 +1036,7 @@ def run_configs(args, rank, ws, local):
                                 accept=accept_entry(tree3, synth.VOCAB, 3))
     # c4: 1B tokens, B=1024, n 24 -> 2, top-64 x 12, 128-node trees
     if not args.skip_1b:
-        cfg = synth.CONFIGS[4]
+        cfg = synth.WORKLOADS[4]
         rng = synth.rng_for(4)
         T, planted = synth.build_corpus(rng, cfg["corpus"][0], device="cuda")
         ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], [T], [1.0], 1.1,
@@ -1059,7 +1059,7 @@ def run_retrieve(args, rank, ws, local):
     import paper_2502_17139_gb300.synth as synth
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
-    cfg = synth.CONFIGS[2]
+    cfg = synth.WORKLOADS[2]
     rng = synth.rng_for(2)
     corpora = [synth.build_corpus(rng, spec, device="cuda")[0] for spec in cfg["corpus"]]
     to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32) if a.dtype == np.uint32

@@ -265,7 +265,7 @@ def randn_bf16(shape, seed: int, device="cpu"):
 # --------------------------------------------------------------------------
 # the five workloads (sizes follow the benchmark configurations)
 # --------------------------------------------------------------------------
-CONFIGS = {
+WORKLOADS = {
     1: dict(name="c1 single-source 1M", corpus=[dict(n=1_000_000, s=1.1, n_grams=2000, len_range=(8, 32), copies_range=(2, 8))],
             batch=32, ctx_len=64, n_copy=16, probs=[1.0], n_max=16, n_min=2, top_k=16, draft_len=8,
             node_budget=64, n_pad=64, H=32, Hkv=32, D=128, kv_len=512),
@@ -294,7 +294,7 @@ def scaled_corpus_spec(spec: dict, scale: float) -> dict:
 
 
 def build_corpus(rng: np.random.Generator, spec: dict, vocab: int = VOCAB, device=None):
-    """Corpus from a spec dict (see CONFIGS); ``device`` as for zipf_tokens."""
+    """Corpus from a spec dict (see WORKLOADS); ``device`` as for zipf_tokens."""
     n = spec["n"]
     lr = spec.get("len_range", (8, 32))
     cr = spec.get("copies_range", (2, 8))

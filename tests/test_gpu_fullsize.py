@@ -73,7 +73,7 @@ def compare_rows(g, r, rows):
 def test_two_source_100m_5m(fc, orc):
     """Two-source workload: project store 5M (Zipf 1.3, planted repeats), general
     store 100M (Zipf 1.1), 256 contexts of 128 tokens, top-64 x 10, 64-node trees."""
-    cfg = synth.CONFIGS[2]
+    cfg = synth.WORKLOADS[2]
     rng = synth.rng_for(2)
     corpora = [synth.build_corpus(rng, spec, device="cuda")[0] for spec in cfg["corpus"]]
     Tr, Tc = corpora
@@ -128,7 +128,7 @@ def test_one_billion_tokens(fc, orc):
     16-128-token repeats), 1024 contexts whose last 24 tokens are copied from
     the corpus (half from inside planted repeats), n 24 -> 2, top-64 x 12,
     128-node trees."""
-    cfg = synth.CONFIGS[4]
+    cfg = synth.WORKLOADS[4]
     rng = synth.rng_for(4)
     T, planted = synth.build_corpus(rng, cfg["corpus"][0], device="cuda")
     ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], [T], [1.0], 1.1,

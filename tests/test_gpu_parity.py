@@ -79,7 +79,7 @@ def test_sa_rejects_bad_token(fc):
 
 @pytest.fixture(scope="module")
 def c1(fc, orc):
-    cfg = synth.CONFIGS[1]
+    cfg = synth.WORKLOADS[1]
     rng = synth.rng_for(1)
     T, _ = synth.build_corpus(rng, cfg["corpus"][0])
     ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], [T], [1.0], 1.1)

@@ -99,7 +99,7 @@ def test_retrieve_rev_tiny_sweep(fc, orc, seed):
 def test_retrieve_rev_c1(fc, orc):
     """The 1M-token configuration: 32 contexts whose last 16 tokens are copied
     from the corpus, n 16 -> 2, top-16 x 8."""
-    cfg = synth.CONFIGS[1]
+    cfg = synth.WORKLOADS[1]
     rng = synth.rng_for(1)
     T, _ = synth.build_corpus(rng, cfg["corpus"][0])
     ctx, cl, _ = synth.make_contexts(rng, cfg["batch"], cfg["ctx_len"], cfg["n_copy"], [T], [1.0], 1.1)
