@@ -104,3 +104,46 @@ def test_rank_merge_is_a_stable_sort(seed):
     for i in range(1, len(merged)):
         if merged[i][0] == merged[i - 1][0]:
             assert merged[i][1] > merged[i - 1][1]
+
+
+def runs_by_depth(drafts, w):
+    """For sorted unique drafts with weights w: every trie node (u, l) (the
+    length-l prefix of draft u, new at u when l > lcp(u-1, u)) with its weight
+    and parent, found by numbering, for each depth l, the run starts (lcp < l)."""
+    U = len(drafts)
+    lcp = [0] * U
+    for u in range(1, U):
+        a, b = drafts[u - 1], drafts[u]
+        k = 0
+        while k < min(len(a), len(b)) and a[k] == b[k]:
+            k += 1
+        lcp[u] = k
+    ps = np.concatenate([[0], np.cumsum(w)])
+    nodes = {}
+    prev_rid = prev_rpos = None
+    for l in range(1, max(len(d) for d in drafts) + 1):
+        start = [u == 0 or lcp[u] < l for u in range(U)]
+        rid = list(np.cumsum(start) - 1)      # the run each draft belongs to
+        rpos = [u for u in range(U) if start[u]] + [U]
+        for u in range(U):
+            if lcp[u] < l <= len(drafts[u]):
+                W = ps[rpos[rid[u] + 1]] - ps[u]
+                parent = drafts[prev_rpos[prev_rid[u]]][:l - 1] if l > 1 else ()
+                nodes[drafts[u][:l]] = (int(W), parent)
+        prev_rid, prev_rpos = rid, rpos
+    return nodes
+
+
+@pytest.mark.parametrize("seed", range(5))
+def test_run_numbering_gives_trie_weights_and_parents(seed):
+    rng = np.random.default_rng(4300 + seed)
+    drafts = sorted({tuple(int(x) for x in rng.integers(0, 3, int(rng.integers(1, 7)))) for _ in range(60)})
+    w = [int(x) for x in rng.integers(1, 9, len(drafts))]
+    got = runs_by_depth(drafts, w)
+    # brute force: a prefix weighs the drafts that start with it; its parent drops one token
+    want = {}
+    for d in drafts:
+        for l in range(1, len(d) + 1):
+            p = d[:l]
+            want[p] = (sum(wi for di, wi in zip(drafts, w) if di[:l] == p), p[:-1])
+    assert got == want
