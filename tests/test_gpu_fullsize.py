@@ -1,11 +1,16 @@
-"""Parity at the full benchmark sizes, where the oracle cannot redo everything.
+"""Parity at the full benchmark sizes.
 
 * Suffix arrays of 100M- and 1B-token corpora: the oracle's certificate (a
   permutation whose adjacent suffixes are strictly increasing), and the bucket
   table against its closed form bucket[v] = #{i : T[i] < v}.
-* Retrieval and draft trees for every query on the GPU, compared bit-exactly
-  with the oracle on a seeded sample of queries (the oracle scans the whole
-  corpus once per query and source).
+* Retrieval and draft trees of every query of the two-source workload (256
+  contexts, both sources; forward, reversed-corpus and all-occurrence
+  variants) and of the 1B-token workload (1024 contexts), bit-exact against
+  the oracle's linear corpus scans, which run on all host cores.
+* The benchmarked step loop on the real 100M + 5M store (32 sequences in the
+  bench's two sub-batch streams, GQA 32/8, KV 16384, 128-node trees, 50%
+  replay hits) in lockstep with the oracle's step loop, and its tree
+  attention on every row of one step against the fp64 oracle.
 * The decoder forward at DeepSeek-Coder 1.3B's layer width against the fp64
   oracle on every node of two sequences.
 * Algorithm 1 on the default two-source store through properties that hold
@@ -90,35 +95,33 @@ def test_two_source_100m_5m(fc, orc):
     kvl = np.full(cfg["batch"], 4096, np.int32)
     gt = fc.fc_build_tree(g, [1, 1], dev(root), dev(kvl), cfg["node_budget"], cfg["n_pad"])
     assert fc.fc_get_error() == "FC_OK"
-    sample = np.sort(synth.rng_for(2, 9).choice(cfg["batch"], 16, replace=False))
+    every = np.arange(cfg["batch"])
     res = []
     for s, T in enumerate(corpora):
-        r = orc.retrieve(T, ctx[sample], cl[sample], cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
-        compare_rows({k: v[s] for k, v in g.items()}, r, sample)
+        r = orc.retrieve(T, ctx, cl, cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
+        compare_rows({k: v[s] for k, v in g.items()}, r, every)
         res.append(r)
-    rt = orc.build_tree(res, [1, 1], root[sample], kvl[sample], cfg["node_budget"], cfg["n_pad"])
-    compare_rows(gt, rt, sample)
-    # the reversed-corpus variant: the oracle's rows on the sample, and the
-    # forward search's outputs for every query
+    rt = orc.build_tree(res, [1, 1], root, kvl, cfg["node_budget"], cfg["n_pad"])
+    compare_rows(gt, rt, every)
+    # the reversed-corpus variant, every query
     revs = [fc.fc_datastore_build_reversed(dev(T), synth.VOCAB) for T in corpora]
     gr = fc.fc_retrieve_rev(sources, revs, dev(ctx), dev(cl), p)
     assert fc.fc_get_error() == "FC_OK"
     for s, r in enumerate(res):
-        compare_rows({k: v[s] for k, v in gr.items()}, r, sample)
-    for name in g:
-        assert torch.equal(g[name], gr[name]), name
-    del revs
+        compare_rows({k: v[s] for k, v in gr.items()}, r, every)
+    del revs, gr
     # the all-occurrence trie (every distinct continuation, up to 4096 per
-    # source) on the sampled queries, against the oracle's untruncated lists
+    # source) of every query, against the oracle's untruncated lists
     pa = fc.params(cfg["n_max"], cfg["n_min"], 8, cfg["draft_len"], 4096)
-    ga = fc.fc_retrieve_all(sources, dev(ctx[sample]), dev(cl[sample]), pa)
-    ra = [orc.retrieve(T, ctx[sample], cl[sample], cfg["n_max"], cfg["n_min"], 4096, cfg["draft_len"], 4096)
-          for T in corpora]
-    gta = fc.fc_build_tree_all(ga, [1, 1], dev(root[sample]), dev(kvl[sample]), cfg["node_budget"], cfg["n_pad"])
+    ga = fc.fc_retrieve_all(sources, dev(ctx), dev(cl), pa)
+    ra = [orc.retrieve(T, ctx, cl, cfg["n_max"], cfg["n_min"], 4096, cfg["draft_len"], 4096) for T in corpora]
+    gta = fc.fc_build_tree_all(ga, [1, 1], dev(root), dev(kvl), cfg["node_budget"], cfg["n_pad"])
     assert fc.fc_get_error() == "FC_OK"
-    rta = orc.build_tree(ra, [1, 1], root[sample], kvl[sample], cfg["node_budget"], cfg["n_pad"])
-    compare_rows(gta, rta, np.arange(len(sample)))
-    # the sample exercises long project-store matches and short general ones
+    rta = orc.build_tree(ra, [1, 1], root, kvl, cfg["node_budget"], cfg["n_pad"])
+    compare_rows(gta, rta, every)
+    del ga, gta
+    torch.cuda.empty_cache()
+    # the workload has long project-store matches and short general ones
     ml = g["match_len"].cpu().numpy()
     assert (ml[0] == 16).mean() > 0.3 and (ml[1] > 0).mean() > 0.9
 
@@ -141,12 +144,108 @@ def test_one_billion_tokens(fc, orc):
     kvl = np.zeros(cfg["batch"], np.int32)
     gt = fc.fc_build_tree(g, [1], dev(root), dev(kvl), cfg["node_budget"], cfg["n_pad"])
     assert fc.fc_get_error() == "FC_OK"
-    sample = np.sort(synth.rng_for(4, 9).choice(cfg["batch"], 8, replace=False))
-    r = orc.retrieve(T, ctx[sample], cl[sample], cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
-    compare_rows({k: v[0] for k, v in g.items()}, r, sample)
-    rt = orc.build_tree([r], [1], root[sample], kvl[sample], cfg["node_budget"], cfg["n_pad"])
-    compare_rows(gt, rt, sample)
+    every = np.arange(cfg["batch"])
+    r = orc.retrieve(T, ctx, cl, cfg["n_max"], cfg["n_min"], cfg["top_k"], cfg["draft_len"], 4096)
+    compare_rows({k: v[0] for k, v in g.items()}, r, every)
+    rt = orc.build_tree([r], [1], root, kvl, cfg["node_budget"], cfg["n_pad"])
+    compare_rows(gt, rt, every)
     assert (g["match_len"].cpu().numpy() == 24).mean() > 0.9
+
+
+def bits_bf16(t):
+    return t.cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def test_step_loop_full_store_lockstep(fc, orc):
+    """The benchmarked configuration at full size: the 100M + 5M two-source
+    store, 32 sequences with 128-token contexts, n 16 -> 2, top-64 x 10 per
+    source, 128-node trees, GQA 32/8, head dim 128, KV 16384, a seeded 50%
+    replay-cache hit pattern, and the bench's launch configuration (two
+    sub-batches of 16 sequences on streams of their own, each with its own
+    replay cache).  A recording pass fills the caches; the replayed pass is
+    compared with the oracle's step loop step by step: which queries the
+    cache served, tree sizes, accepted lengths, bonus tokens, and at the end
+    every context, context length and KV length.  The last step's tree
+    attention is compared on every row with the fp64 oracle."""
+    import bench
+    from paper_2502_17139_gb300.step import PipelinedStepLoop
+    steps = 24
+    inp = bench.make_inputs(1.0, 32, 0, steps + 1)
+    cfg, B = inp["cfg"], inp["B"]
+    H, Hkv, D, n_pad, d = cfg["H"], cfg["Hkv"], cfg["D"], cfg["n_pad"], cfg["draft_len"]
+    kv0 = inp["kv0"]
+    assert kv0 == 16384 and B == 32
+    cap = kv0 + (steps + 1) * (d + 1) + 8
+    sources = [fc.fc_datastore_build(dev(T), synth.VOCAB) for T in inp["corpora"]]
+    p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], d, 4096)
+    kc = synth.randn_bf16((B, Hkv, cap, D), 501, "cuda")
+    vc = synth.randn_bf16((B, Hkv, cap, D), 502, "cuda")
+    acts = [(synth.randn_bf16((B, n_pad, H, D), 510 + i, "cuda"), synth.randn_bf16((B, Hkv, n_pad, D), 520 + i, "cuda"),
+             synth.randn_bf16((B, Hkv, n_pad, D), 530 + i, "cuda")) for i in range(2)]
+    loop = PipelinedStepLoop(2, sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, [1, 1], H, Hkv, D, cap,
+                             kv0, synth.VOCAB, cache_capacity=1 << 14, k_cache=kc, v_cache=vc)
+    # the per-step inputs stay resident: the sub-batch streams read them after
+    # step() returns, so they must not be temporaries
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).cuda()
+    hits = inp["hits"][:steps]
+    no_hits = np.zeros_like(hits)
+    hits_d, no_hits_d = to_dev(hits), to_dev(no_hits)
+    plen_d, rtok_d = to_dev(inp["plen"][:steps]), to_dev(inp["rtok"][:steps])
+    for s in range(steps):  # recording pass
+        loop.step(*acts[s % 2], no_hits_d[s], plen_d[s], rtok_d[s])
+    loop.reset()
+    got = dict(hit=[], acc_len=[], bonus=[], n_nodes=[])
+    for s in range(steps):
+        last = s == steps - 1
+        if last:
+            loop.join()
+            kvl_before = loop.kv_len_now.cpu().numpy()
+        loop.step(*acts[s % 2], hits_d[s], plen_d[s], rtok_d[s])
+        loop.join()
+        got["hit"].append(loop.skip.cpu().numpy())
+        got["acc_len"].append(loop.acc["acc_len"].cpu().numpy())
+        got["bonus"].append(host_u32(loop.acc["bonus"]))
+        got["n_nodes"].append(loop.tree["n_nodes"].cpu().numpy())
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_OK"
+    # the oracle, one sub-batch at a time with a replay cache of its own
+    po = dict(n_max=cfg["n_max"], n_min=cfg["n_min"], top_k=cfg["top_k"], draft_len=d, max_occ=4096,
+              node_budget=cfg["node_budget"], n_pad=n_pad)
+    ref = dict(hit=[], acc_len=[], bonus=[], n_nodes=[])
+    r_ctx, r_cl, r_kvl = [], [], []
+    for sl in loop.slices:
+        cache = {}
+        args = (inp["corpora"], inp["ctx"][sl], inp["cl"][sl], steps, po)
+        draws = (inp["plen"][:steps, sl], inp["rtok"][:steps, sl], [1, 1], synth.VOCAB)
+        orc.step_loop(*args, no_hits[:, sl], *draws, kv_len0=np.full(sl.stop - sl.start, kv0, np.int32), cache=cache)
+        hist, c_, l_, k_ = orc.step_loop(*args, hits[:, sl], *draws, kv_len0=np.full(sl.stop - sl.start, kv0, np.int32),
+                                         cache=cache)
+        for name in ref:
+            ref[name].append(hist[name])
+        r_ctx.append(c_)
+        r_cl.append(l_)
+        r_kvl.append(k_)
+    for s in range(steps):
+        for name in ("acc_len", "bonus", "n_nodes", "hit"):
+            assert np.array_equal(got[name][s], np.concatenate([h[s] for h in ref[name]])), (name, s)
+    assert np.array_equal(host_u32(loop.ctx), np.concatenate(r_ctx))
+    assert np.array_equal(loop.ctx_len_now.cpu().numpy(), np.concatenate(r_cl))
+    assert np.array_equal(loop.kv_len_now.cpu().numpy(), np.concatenate(r_kvl))
+    served = sum(int(h.sum()) for h in got["hit"])
+    assert 0.3 * hits.sum() < served <= hits.sum()
+    nn_all = np.concatenate(got["n_nodes"])
+    assert nn_all.mean() > 40 and (nn_all == 128).any() and (nn_all < 64).any()
+    # the last step's attention, every row, against the fp64 oracle (the cache
+    # rows it read, [0, kv_len), were not touched by that step's append)
+    q, kt, vt = acts[(steps - 1) % 2]
+    tree = loop.tree
+    nn = tree["n_nodes"].cpu().numpy()
+    mask = tree["mask"].cpu().numpy().view(np.uint64)
+    out = loop.attn_out.float().cpu().numpy()
+    ref_out = orc.tree_attn(bits_bf16(q), bits_bf16(kc), bits_bf16(vc), kvl_before, bits_bf16(kt), bits_bf16(vt),
+                            mask, nn)
+    assert np.isfinite(out).all()
+    assert np.abs(out - ref_out).max() <= 2e-2
 
 
 def test_decoder_full_width(fc, orc):

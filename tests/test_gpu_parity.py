@@ -469,23 +469,24 @@ def test_attn_kv_split_two_tiles(fc, orc):
     _attn_case(fc, orc, 7, B, 128, 32, 8, kvl, 2048, nn=nn, full_rows=False, want_parts=2)
 
 
-def test_attn_c3_shape_sampled(fc, orc):
-    # c3: B=16, H=Hkv=32, KV 4096, 64-node trees
-    _attn_case(fc, orc, 5, 16, 64, 32, 32, [4096] * 16, 4096, nn=[64] * 16, full_rows=False)
+def test_attn_c3_shape_full(fc, orc):
+    # c3: B=16, H=Hkv=32, KV 4096, 64-node trees; every row against the fp64 oracle
+    _attn_case(fc, orc, 5, 16, 64, 32, 32, [4096] * 16, 4096, nn=[64] * 16)
 
 
-def test_attn_c5_shape_sampled(fc, orc):
-    # c5: B=32, H=32, Hkv=8, KV 16384, trees <= 128 nodes
-    _attn_case(fc, orc, 6, 32, 128, 32, 8, [16384] * 32, 16384 + 256, full_rows=False, sample=160)
+def test_attn_c5_shape_full(fc, orc):
+    # c5: B=32, H=32, Hkv=8, KV 16384, trees <= 128 nodes; every row
+    _attn_case(fc, orc, 6, 32, 128, 32, 8, [16384] * 32, 16384 + 256)
 
 
-def test_attn_c5_subbatch_sampled(fc, orc):
+def test_attn_c5_subbatch_full(fc, orc):
     # the launch the step bench times: one sub-batch of 16 sequences (256 CTAs,
-    # 1.7 waves, no KV split), KV lengths grown over the steps, trees of every size
+    # 1.7 waves, no KV split), KV lengths grown over the steps, trees of every
+    # size; every row
     rng = synth.rng_for(53)
     kvl = [16384 + int(x) for x in rng.integers(0, 700, 16)]
     nn = [int(x) for x in rng.choice([1, 20, 40, 70, 97, 128], 16)]
-    _attn_case(fc, orc, 11, 16, 128, 32, 8, kvl, 16384 + 768, nn=nn, full_rows=False, sample=160)
+    _attn_case(fc, orc, 11, 16, 128, 32, 8, kvl, 16384 + 768, nn=nn)
 
 
 # ------------------------------------------------------- accept / append
