@@ -39,19 +39,22 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "retrieve+verify steps/s"
+PAD_TOKEN = 0xFFFFFFFF
 UNIT = "steps/s"
-# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one tree-attention
-# launch of the step loop with the sequences in 2 sub-batches (16 sequences a
-# launch, 256 CTAs), from one ncu capture: the mean over the 28 launches with a grid
-# of 256 of
-#   ncu --metrics gpu__time_duration.sum,dram__bytes_read.sum,dram__bytes_write.sum
-#       --clock-control none -k regex:k_tree_attn -c 60 --csv
-#       python bench.py --steps 4 --warmup 3 --no-e2e --no-cpu-baseline --no-graph
-# (the 568-CTA launches in the same capture are the single-stream pass over all 32
-# sequences: 2.367e9 bytes each).  It is valid only for the kernel sources it was
-# taken on (their SHA-256 below) and that split; otherwise the bench reports traffic
-# as null until it is measured again.
-ATTN_TRAFFIC = {"bytes_per_launch": 1.1714e9, "sub_batches": 2,
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of the tree-attention
+# launch the roofline times (all 32 sequences on one stream), as a ratio to the
+# launch's algorithmic bytes, from one ncu capture of three launches:
+#   ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum
+#       --clock-control none -k regex:k_tree_attn -s 10 -c 3 --csv
+#       python bench.py --steps 4 --warmup 3 --split 1 --no-e2e --no-cpu-baseline --no-graph
+# (one pass per launch; the recording pass's 7 launches and the 3 warm-up launches are
+# skipped, so the captured launches are timed steps 3-5 of the trajectory, the first
+# three launches of the bench's single-stream pass, whose algorithmic bytes that run
+# prints as roofline.algorithmic_bytes_first_launches).  The bench reports traffic =
+# ratio x the algorithmic bytes per launch of its own launches.  The ratio is valid
+# only for the kernel sources it was taken on (their SHA-256 below); otherwise the
+# bench reports traffic as null until it is measured again.
+ATTN_TRAFFIC = {"ratio": 1.0622,
                 "sources": ["paper_2502_17139_gb300/csrc/tree_attn.cu", "paper_2502_17139_gb300/csrc/fc_common.cuh"],
                 "sha256": "ef8c93976042c50443c18522134a35334265e92729d5d394c2d7ce71f39a35b3"}
 
@@ -78,7 +81,7 @@ def parse_args(argv=None):
     ap.add_argument("--batch", type=int, default=32)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--mode", choices=["step", "attn", "argmax", "configs", "retrieve", "algorithm1", "cache",
+    ap.add_argument("--mode", choices=["step", "attn", "argmax", "configs", "retrieve", "algorithm1", "cache", "gemm",
                                        "decoder"],
                     default="step",
                     help="step: the full step loop (the benchmark); attn: tree attention alone on the step loop's "
@@ -104,24 +107,27 @@ def parse_args(argv=None):
                     help="algorithm1 / cache modes: steps that fill the CACHE first (default 100 / 450)")
     ap.add_argument("--skip-1b", action="store_true", help="configs mode: leave out the 1B-token configuration")
     ap.add_argument("--traffic-bytes", type=float, default=None,
-                    help="ncu dram read+write bytes of one tree-attention launch of this workload")
+                    help="ncu dram read+write bytes of one single-stream tree-attention launch of this workload")
     return ap.parse_args(argv)
 
 
 # ---------------------------------------------------------------- helpers
-def attn_traffic(args, nsub=1):
-    """Measured DRAM bytes per attention launch, or None when the kernel or the
-    launch's sub-batch split changed since."""
+def attn_traffic(args, algorithmic_bytes_per_launch):
+    """DRAM bytes per attention launch: the measured ratio to the algorithmic
+    bytes times this run's algorithmic bytes per launch, or None when the
+    kernel changed since the ratio was measured."""
     if args.traffic_bytes is not None:
         return args.traffic_bytes
-    if nsub != ATTN_TRAFFIC["sub_batches"]:
+    if ATTN_TRAFFIC["ratio"] is None or ATTN_TRAFFIC["sha256"] is None:
         return None
     import hashlib
     h = hashlib.sha256()
     for f in ATTN_TRAFFIC["sources"]:
         with open(os.path.join(ROOT, f), "rb") as fh:
             h.update(fh.read())
-    return ATTN_TRAFFIC["bytes_per_launch"] if h.hexdigest() == ATTN_TRAFFIC["sha256"] else None
+    if h.hexdigest() != ATTN_TRAFFIC["sha256"]:
+        return None
+    return ATTN_TRAFFIC["ratio"] * algorithmic_bytes_per_launch
 
 
 def load_peaks():
@@ -374,33 +380,27 @@ def run_ours(args, rank, ws, local):
     # attention work of every timed launch
     flops_seq, bytes_seq, nodes_hist, acc_hist, hits_used = replay_counts(inp, sources, p, cfg, cap, kv0, dev, W, K,
                                                                           weights, nsub)
-    sub = [slice(B * h // nsub, B * (h + 1) // nsub) for h in range(nsub)]
-
     peaks = load_peaks()
-    per_launch = []  # one attention launch per timed step and sub-batch
-    for i in range(K):
-        for h in range(nsub):
-            per_launch.append((float(flops_seq[i][sub[h]].sum()), float(bytes_seq[i][sub[h]].sum()),
-                               attn_ms[i][h] * 1e-3))
-    tot_f = sum(f for f, _, _ in per_launch)
-    tot_b = sum(b for _, b, _ in per_launch)
-    tot_t = sum(t for _, _, t in per_launch)
-    n_launch = len(per_launch)
-    t_tc = tot_f / (peaks["tc_sustained"] * 1e12)
-    t_hbm = tot_b / (peaks["hbm"] * 1e9)
-    if t_tc >= t_hbm:
-        roof = dict(bound="tensor", achieved=tot_f / tot_t / 1e12, peak=peaks["tc_sustained"], unit="TFLOP/s")
-    else:
-        roof = dict(bound="hbm", achieved=tot_b / tot_t / 1e9, peak=peaks["hbm"], unit="GB/s")
-    roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = attn_traffic(args, nsub) if args.scale == 1.0 else args.traffic_bytes
-    roof["peak_source"] = peaks["source"] + (" sustained bf16" if roof["bound"] == "tensor" else " hbm copy")
-    roof["kernel"] = "k_tree_attn"
-    roof["mean_launch_us"] = 1e6 * tot_t / n_launch
-    roof["algorithmic_flops_per_launch"] = tot_f / n_launch
-    roof["algorithmic_bytes_per_launch"] = tot_b / n_launch
-    roof["launches_per_step"] = nsub
-    roof["other_bound_frac"] = (t_hbm if roof["bound"] == "tensor" else t_tc) / tot_t
+    # the attention kernel's own roofline: the same trajectory on one stream
+    # (32 sequences a launch), where each launch shares the GPU with nothing,
+    # so its event time is the kernel's own duration
+    ss = single_stream_attn(sources, inp, p, cfg, cap, kv0, dev, weights, kc, vc, q_pool, kt_pool, vt_pool, hits_d,
+                            plen_d, rtok_d, P, W, min(K, 64), flops_seq, bytes_seq)
+    roof = attn_roofline(ss["flops"], ss["bytes"], ss["seconds"], ss["launches"], peaks)
+    roof["traffic"] = (attn_traffic(args, roof["algorithmic_bytes_per_launch"]) if args.scale == 1.0
+                       else args.traffic_bytes)
+    roof["traffic_ratio_to_algorithmic"] = ATTN_TRAFFIC["ratio"] if roof["traffic"] is not None else None
+    roof["algorithmic_bytes_first_launches"] = ss["bytes_by_launch"][:3]
+    roof["launch"] = (f"k_tree_attn over all {B} sequences on one stream (the step loop's trajectory, "
+                      f"first {ss['launches']} timed steps), CUDA events on its stream")
+    # the pipelined step's own launches (16 sequences each): their event times
+    # include the other sub-batch's kernels running beside them
+    piped_f = sum(float(flops_seq[i].sum()) for i in range(K))
+    piped_t = sum(attn_ms[i][h] for i in range(K) for h in range(nsub)) * 1e-3
+    piped = {"launches": K * nsub, "mean_launch_us": 1e6 * piped_t / (K * nsub),
+             "tflops_per_launch_time": piped_f / piped_t / 1e12,
+             "note": "per sub-batch launch; the two sub-batches' kernels overlap, so a launch's event time "
+                     "includes time shared with the other sub-batch" if nsub > 1 else "the timed loop itself"}
 
     out = {
         "metric": METRIC, "value": weak_value(K, ws, t_max), "unit": UNIT, "n_gpus": ws, "steps": K, "warmup": W,
@@ -424,7 +424,8 @@ def run_ours(args, rank, ws, local):
                                "argmax_accept_append": mean2(stage_ms["tail"]), "all": t_ms / K},
         "queries_per_s": ws * B * K / (t_max * 1e-3),
         "retrievals_per_s": ws * (2 * (B * K - hits_used)) / (t_max * 1e-3),
-        "tree_attn_tflops": tot_f / tot_t / 1e12,
+        "tree_attn_tflops": roof["achieved_tflops"],
+        "attn_in_timed_step": piped,
         "avg_acceptance_length": float(np.mean([a.mean() + 1 for a in acc_hist])),
         "avg_tree_nodes": float(np.mean([n.mean() for n in nodes_hist])),
         # trees by node count in 32-node bins (1-32, 33-64, 65-96, 97-128): with four
@@ -432,13 +433,6 @@ def run_ours(args, rank, ws, local):
         "tree_nodes_bins": np.bincount((np.concatenate(nodes_hist) - 1) // 32, minlength=n_pad // 32).tolist(),
         "datastore_build": {"tokens": build_tokens, "seconds": build_s, "tokens_per_s": build_tokens / build_s},
     }
-    if nsub > 1:
-        # the attention kernel alone on the step loop's launches: the same
-        # trajectory on one stream (its launches share the GPU with nothing), for
-        # the kernel's own roofline beside the pipelined step's
-        out["attn_single_stream"] = single_stream_attn(
-            sources, inp, p, cfg, cap, kv0, dev, weights, kc, vc, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P,
-            W, min(K, 64), flops_seq, bytes_seq, peaks, roof["bound"])
     if not args.no_e2e:
         loop.reset()
         out["e2e"] = run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws)
@@ -448,24 +442,33 @@ def run_ours(args, rank, ws, local):
 
 
 def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W, K):
-    """The same trajectory again, from the start: the W warm-up steps eager,
-    then the K timed steps replayed from CUDA graphs of G steps each (G = 8, 4
-    or 2, the largest that divides K and the pool size), one graph per pool
-    offset (they read the pooled activations directly); a step's small draws
-    are copied into the graph's input buffers before each replay.  With
+    """The same trajectory again, from the start: the W warm-up steps eager
+    (one more when W is odd, since a graph starts at an even step: its
+    lengths ping-pong between two buffers), then the timed steps replayed
+    from CUDA graphs of G steps each (G = 8, 4 or 2, the largest that divides
+    the pool size and the number of timed steps), one graph per pool offset
+    (they read the pooled activations directly); a step's small draws are
+    copied into the graph's input buffers before each replay.  The timed
+    steps are the K steps after the warm-up, or K - 1 when the odd warm-up
+    took one of them (K - 1 is then rounded down to a multiple of 2).  With
     sub-batches a graph forks to their streams and joins them once, at its
     end."""
     import torch
-    G = next((g for g in (8, 4, 2) if K % g == 0 and P % g == 0), None)
-    if G is None or W % 2 or W < 2:
-        return {"skipped": "needs an even warm-up of at least 2 and an even pool size and step count"}
+    W2 = W + (W % 2)
+    K2 = K - (W2 - W)
+    G = next((g for g in (8, 4, 2) if K2 % g == 0 and P % g == 0), None)
+    if G is None:
+        K2 -= K2 % 2
+        G = 2 if P % 2 == 0 and K2 >= 2 else None
+    if G is None:
+        return {"skipped": "needs an even pool size and at least 2 steps after the warm-up"}
     loop.reset()
-    for s in range(W):  # eager warm-up; it also makes workspaces and kernel attributes
+    for s in range(W2):  # eager warm-up; it also makes workspaces and kernel attributes
         loop.step(q_pool[s % P], kt_pool[s % P], vt_pool[s % P], hits_d[s], plen_d[s], rtok_d[s])
     small = [(torch.empty_like(hits_d[0]), torch.empty_like(plen_d[0]), torch.empty_like(rtok_d[0])) for _ in range(G)]
     graphs = {}
     for i in range(P // G):
-        s0 = W + i * G
+        s0 = W2 + i * G
         graphs[s0 % P] = loop.capture([(q_pool[(s0 + t) % P], kt_pool[(s0 + t) % P], vt_pool[(s0 + t) % P]) + small[t]
                                        for t in range(G)])
 
@@ -479,20 +482,23 @@ def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W,
     torch.cuda.synchronize()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     start.record()
-    for i in range(0, K, G):
-        block(W + i)
+    for i in range(0, K2, G):
+        block(W2 + i)
     end.record()
     torch.cuda.synchronize()
-    ms = start.elapsed_time(end) / K
-    return {"ms_per_step": ms, "steps_per_s": 1e3 / ms, "graphs": len(graphs), "steps_per_graph": G,
+    ms = start.elapsed_time(end) / K2
+    return {"ms_per_step": ms, "steps_per_s": 1e3 / ms, "steps": K2, "eager_warmup_steps": W2, "graphs": len(graphs),
+            "steps_per_graph": G,
             "note": f"the timed steps from graphs of {G} steps (first replays include the graphs' upload); "
                     "the step's small draws copied in before each replay"}
 
 
 def single_stream_attn(sources, inp, p, cfg, cap, kv0, dev, weights, kc, vc, q_pool, kt_pool, vt_pool, hits_d, plen_d,
-                       rtok_d, P, W, K2, flops_seq, bytes_seq, peaks, bound):
-    """Per-launch attention roofline of the first K2 timed steps run on one
-    stream (the step loop over the whole batch), from the same starting state."""
+                       rtok_d, P, W, K2, flops_seq, bytes_seq):
+    """The attention launches of the first K2 timed steps, run on one stream
+    (the step loop over the whole batch, from the same starting state, the
+    same trajectory), each timed with CUDA events on its stream.  Returns the
+    launches' total algorithmic FLOPs and bytes and their total time."""
     import torch
 
     import paper_2502_17139_gb300.synth as synth
@@ -516,12 +522,30 @@ def single_stream_attn(sources, inp, p, cfg, cap, kv0, dev, weights, kc, vc, q_p
     t = sum(a.elapsed_time(b) for a, b in evs) * 1e-3
     f = sum(float(flops_seq[i].sum()) for i in range(K2))
     by = sum(float(bytes_seq[i].sum()) for i in range(K2))
-    if bound == "tensor":
-        ach, peak, unit = f / t / 1e12, peaks["tc_sustained"], "TFLOP/s"
-    else:
-        ach, peak, unit = by / t / 1e9, peaks["hbm"], "GB/s"
-    return {"steps": K2, "mean_launch_us": 1e6 * t / K2, "achieved": ach, "peak": peak, "unit": unit,
-            "frac": ach / peak}
+    return {"launches": K2, "seconds": t, "flops": f, "bytes": by,
+            "bytes_by_launch": [float(bytes_seq[i].sum()) for i in range(K2)]}
+
+
+def attn_roofline(flops, nbytes, seconds, launches, peaks):
+    """The roofline object of the attention kernel from its launches' total
+    algorithmic FLOPs and bytes and their total event time.  The kernel is
+    timed in a region of milliseconds, so the tensor peak is the burst one.
+    The bound is whichever floor (tensor time or HBM time) is larger; the
+    other side's fraction is reported beside it."""
+    ach_tf = flops / seconds / 1e12
+    ach_gb = nbytes / seconds / 1e9
+    tensor_frac = ach_tf / peaks["tc_burst"]
+    hbm_frac = ach_gb / peaks["hbm"]
+    tensor_bound = flops / (peaks["tc_burst"] * 1e12) >= nbytes / (peaks["hbm"] * 1e9)
+    roof = dict(bound="tensor" if tensor_bound else "hbm", achieved=ach_tf if tensor_bound else ach_gb,
+                peak=peaks["tc_burst"] if tensor_bound else peaks["hbm"], unit="TFLOP/s" if tensor_bound else "GB/s")
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["peak_source"] = peaks["source"] + (" burst bf16 (bf16_tflops)" if tensor_bound else " hbm copy (hbm_gbs)")
+    roof.update(kernel="k_tree_attn", launches=launches, mean_launch_us=1e6 * seconds / launches,
+                algorithmic_flops_per_launch=flops / launches, algorithmic_bytes_per_launch=nbytes / launches,
+                achieved_tflops=ach_tf, tensor_frac=tensor_frac, achieved_gbs=ach_gb, hbm_frac=hbm_frac,
+                tensor_frac_of_sustained=ach_tf / peaks["tc_sustained"])
+    return roof
 
 
 def mean2(rows):
@@ -699,9 +723,17 @@ def cpu_baseline(inp, cfg, kv0, avg_nodes, B, budget_s=20.0):
 
 
 def run_reference(args, rank, ws):
-    """CPU oracle arm: each step runs one sequence of the batch through the
-    whole oracle pipeline (its retrievals, tree, acceptance, append and the
-    attention of one kv-head group) and is scaled to a full step."""
+    """CPU oracle arm: the step loop through the oracle on the host cores.
+
+    Every timed step is a full, unsampled step of all B sequences: the
+    replay-cache lookup and the retrievals it does not serve (both sources,
+    linear corpus scans), the trees, the tree attention of every (sequence,
+    node, query head) row in fp64 against the whole KV cache, the synthetic
+    target model, acceptance and the cache append.  As in the GPU arm, a
+    recording pass first fills the replay cache along the trajectory (no
+    hits, no attention), and the W warm-up steps advance the trajectory
+    before the timed ones; they skip the attention, which does not steer the
+    trajectory."""
     if rank != 0:
         return None
     import paper_2502_17139_gb300.synth as synth
@@ -710,57 +742,66 @@ def run_reference(args, rank, ws):
     inp = make_inputs(args.scale, args.batch, 0, K + W + 1)
     cfg, B, kv0 = inp["cfg"], inp["B"], inp["kv0"]
     H, Hkv, D, n_pad, d = cfg["H"], cfg["Hkv"], cfg["D"], cfg["n_pad"], cfg["draft_len"]
-    G = H // Hkv
+    cap = kv0 + (K + W + 1) * (d + 1) + 8
     rng = synth.rng_for(5, 999)
-    bits = lambda a: (a.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
-    kc = bits(rng.standard_normal((1, 1, kv0 + (K + W + 1) * (d + 1), D), dtype=np.float32))
-    kt = bits(rng.standard_normal((1, 1, n_pad, D), dtype=np.float32))
-    q = bits(rng.standard_normal((1, n_pad, G, D), dtype=np.float32))
-    ctx = inp["ctx"].copy()
-    cl = inp["cl"].copy()
-    times, attn_times = [], []
-    for s in range(K + W):
-        b = s % B
-        # the GPU arm replays a recorded trajectory, so every step that asks
-        # for a cache hit gets one: such a step's retrieval is not counted
-        tr0 = time.perf_counter()
-        res = [orc.retrieve(T, ctx[b:b + 1], cl[b:b + 1], cfg["n_max"], cfg["n_min"], cfg["top_k"], d, 4096)
-               for T in inp["corpora"]]
-        t_ret = 0.0 if inp["hits"][s, b] else time.perf_counter() - tr0
-        t0 = time.perf_counter()
-        root = ctx[b:b + 1, cl[b] - 1]
-        tr = orc.build_tree(res, src_weights(args), root, np.array([kv0], np.int32), cfg["node_budget"], n_pad)
-        n = int(tr["n_nodes"][0])
-        rows = np.array([(0, i, h) for i in range(n) for h in range(G)], np.int32)
-        ta = time.perf_counter()
-        orc.tree_attn(q, kc, kc, np.array([kv0], np.int32), kt, kt, tr["mask"], tr["n_nodes"], rows=rows)
-        ta = time.perf_counter() - ta
-        am = orc.synth_argmax(tr["tok"], tr["parent"], tr["n_nodes"], inp["plen"][s][b:b + 1], inp["rtok"][s][b:b + 1],
-                              synth.VOCAB)
-        ac = orc.accept(tr["tok"], tr["parent"], tr["n_nodes"], am, d + 2)
-        a = int(ac["acc_len"][0])
-        for t in range(a):
-            ctx[b, cl[b] + t] = tr["tok"][0, ac["path"][0, t + 1]]
-        ctx[b, cl[b] + a] = ac["bonus"][0]
-        cl[b] += a + 1
-        dt = time.perf_counter() - t0
-        if s >= W:
-            times.append(dt - ta + t_ret)
-            attn_times.append(ta)
-    # one sampled step = one sequence with one of its Hkv attention groups;
-    # a full step is B sequences with all Hkv groups each
-    step_s = B * (statistics.mean(times) + Hkv * statistics.mean(attn_times))
+    block = (rng.standard_normal(1 << 22, dtype=np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    tile = lambda shape, off: np.resize(np.roll(block, off), shape)  # bf16 N(0,1) bit patterns
+    kc, vc = tile((B, Hkv, cap, D), 0), tile((B, Hkv, cap, D), 12345)
+    q, kt, vt = tile((B, n_pad, H, D), 777), tile((B, Hkv, n_pad, D), 999), tile((B, Hkv, n_pad, D), 4242)
+    po = dict(n_max=cfg["n_max"], n_min=cfg["n_min"], top_k=cfg["top_k"], max_occ=4096)
+    weights = src_weights(args)
+    cache = {}
+
+    def run(hits, timed_from, attention):
+        ctx, cl = inp["ctx"].copy(), inp["cl"].copy()
+        kvl = np.full(B, kv0, np.int32)
+        times = []
+        for s in range(W + K):
+            t0 = time.perf_counter()
+            keys = [orc.cache_key(ctx[b], cl[b], po["n_max"]) for b in range(B)]
+            served = [bool(hits[s, b]) and keys[b] in cache for b in range(B)]
+            todo = np.array([b for b in range(B) if not served[b]], np.int64)
+            res = [dict(drafts=np.full((B, po["top_k"], d), PAD_TOKEN, np.uint32),
+                        draft_len=np.zeros((B, po["top_k"]), np.int32), count=np.zeros((B, po["top_k"]), np.uint32),
+                        n_drafts=np.zeros(B, np.int32), match_len=np.zeros(B, np.int32)) for _ in inp["corpora"]]
+            for b in range(B):
+                if served[b]:
+                    for si, r in enumerate(res):
+                        for name in r:
+                            r[name][b] = cache[keys[b]][si][name]
+            if len(todo):
+                for si, T in enumerate(inp["corpora"]):
+                    r = orc.retrieve(T, ctx[todo], cl[todo], po["n_max"], po["n_min"], po["top_k"], d, po["max_occ"])
+                    for name in r:
+                        res[si][name][todo] = r[name]
+                for b in todo:
+                    cache[keys[b]] = [{name: r[name][b].copy() for name in r} for r in res]
+            root = ctx[np.arange(B), cl - 1]
+            tr = orc.build_tree(res, weights, root, kvl, cfg["node_budget"], n_pad)
+            if attention and s >= timed_from:
+                orc.tree_attn(q, kc, vc, kvl, kt, vt, tr["mask"], tr["n_nodes"])
+            am = orc.synth_argmax(tr["tok"], tr["parent"], tr["n_nodes"], inp["plen"][s], inp["rtok"][s], synth.VOCAB)
+            ac = orc.accept(tr["tok"], tr["parent"], tr["n_nodes"], am, d + 2)
+            kvl, cl, _ = orc.kv_append(ac["path"], ac["acc_len"], ac["bonus"], tr["tok"], kt, vt, kc, vc, kvl, ctx, cl)
+            if s >= timed_from:
+                times.append(time.perf_counter() - t0)
+        return times
+
+    run(np.zeros_like(inp["hits"]), W + K, False)   # recording pass
+    times = run(inp["hits"], W, True)
+    step_s = statistics.mean(times)
     cores = orc.hardware_threads()
     value = 1.0 / step_s
+    sample = (f"every timed step is a full step of all {B} sequences (replay-cache lookup, retrieval on both sources "
+              f"for the queries it does not serve, trees, fp64 tree attention of every row, acceptance, append); "
+              f"{K} timed steps after {W} warm-up steps and a recording pass")
     return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": K, "warmup": W,
             "ms_per_step": 1e3 * step_s, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f64 attention + u32 retrieval", "data": "synthetic", "impl": "reference",
-            "config": {"workload": WORKLOAD, "batch_per_gpu": B, "kv_len0": kv0, "parallelism": "cpu oracle"},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                             "sample": (f"each step: 1 of {B} sequences through the oracle pipeline (retrieval on "
-                                        f"both sources, not counted when the replayed cache serves it, tree, 1 of {Hkv} kv-head "
-                                        f"attention groups, acceptance, append); attention scaled x{Hkv}, the "
-                                        f"sequence scaled x{B}")},
+            "config": {"workload": WORKLOAD if args.scale == 1.0 else WORKLOAD + f" (scaled x{args.scale})",
+                       "batch_per_gpu": B, "kv_len0": kv0, "parallelism": "cpu oracle"},
+            "step_seconds": {"min": min(times), "max": max(times)},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
@@ -1387,6 +1428,54 @@ def run_decoder(args, rank, ws, local):
             "clocks": clock_rec}
 
 
+def run_gemm(args, rank, ws, local):
+    """fc_gemm_bf16 (the library's tcgen05 GEMM) on the decoder's shapes over
+    2048 tree rows (32 sequences x 64 nodes, DeepSeek-Coder 1.3B's width),
+    timed beside torch.matmul (cuBLAS) on the same operands in the same run.
+    Each shape runs back to back on operands that stay resident; the weights
+    of the larger shapes exceed L2."""
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    peaks = load_peaks()
+    M = 2048
+    shapes = [("q", 2048, 2048), ("kv", 2048, 4096), ("o", 2048, 2048), ("gate_up", 2048, 11008),
+              ("down", 5504, 2048), ("lm_head", 2048, 32256)]
+    per_layer = {"q", "kv", "o", "gate_up", "down"}
+    g = torch.Generator(device=dev)
+    g.manual_seed(7)
+    rows, ours_t, lib_t, flops_t = [], 0.0, 0.0, 0.0
+    for name, K, N in shapes:
+        a = torch.randn((M, K), generator=g, device=dev).to(torch.bfloat16)
+        b = (torch.randn((K, N), generator=g, device=dev) * K ** -0.5).to(torch.bfloat16)
+        c = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+        c_ref = torch.empty_like(c)
+        t_ours = _cuda_ms(lambda: fc.fc_gemm_bf16(a, b, out=c), reps=max(args.steps, 5), warm=max(args.warmup, 3))
+        t_lib = _cuda_ms(lambda: torch.matmul(a, b, out=c_ref), reps=max(args.steps, 5), warm=max(args.warmup, 3))
+        torch.cuda.synchronize()
+        assert fc.fc_get_error() == "FC_OK"
+        diff = float((c.float() - c_ref.float()).abs().max())
+        fl = 2.0 * M * N * K
+        w = 24 if name in per_layer else 1  # occurrences in one 24-layer forward
+        ours_t += w * t_ours
+        lib_t += w * t_lib
+        flops_t += w * fl
+        rows.append({"gemm": name, "M": M, "N": N, "K": K, "ours_us": 1e3 * t_ours, "cublas_us": 1e3 * t_lib,
+                     "ours_tflops": fl / t_ours / 1e9, "cublas_tflops": fl / t_lib / 1e9,
+                     "ours_frac_of_burst": fl / t_ours / 1e9 / peaks["tc_burst"], "max_abs_diff_vs_cublas": diff})
+    ach = flops_t / ours_t / 1e9
+    return {"metric": "decoder GEMM TFLOP/s", "value": ach, "unit": "TFLOP/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "dtype": "bf16 (fp32 accumulate)",
+            "data": "synthetic", "config": {"workload": "decoder GEMMs of a 24-layer DeepSeek-Coder-1.3B-shaped "
+                                                        "forward over 2048 tree rows, weighted by occurrences"},
+            "cublas_tflops": flops_t / lib_t / 1e9, "ratio_to_cublas": lib_t / ours_t,
+            "roofline": {"bound": "tensor", "achieved": ach, "peak": peaks["tc_burst"], "unit": "TFLOP/s",
+                         "frac": ach / peaks["tc_burst"], "peak_source": peaks["source"] + " burst bf16"},
+            "shapes": rows}
+
+
 def main(argv=None):
     args = parse_args(argv)
     rank, ws, local = dist_setup(args.gpus)
@@ -1406,6 +1495,8 @@ def main(argv=None):
         out = run_cache(args, rank, ws, local)
     elif args.mode == "decoder":
         out = run_decoder(args, rank, ws, local)
+    elif args.mode == "gemm":
+        out = run_gemm(args, rank, ws, local)
     else:
         out = run_ours(args, rank, ws, local)
     if rank == 0 and out is not None:
