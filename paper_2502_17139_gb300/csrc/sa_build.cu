@@ -11,7 +11,6 @@
 // re-ranks by scanning "key differs from its predecessor" flags.  The loop
 // stops when every rank is distinct.  All passes stream the arrays once
 // (HBM-bound); only the rank gather rank[i + h] is random.
-#include <mutex>
 
 #include "fc_common.cuh"
 
@@ -404,34 +403,32 @@ extern "C" fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n, ui
 // application that owns every device allocation.  They can still build a
 // small datastore (a repository's own project store) here.
 //
-// The array is a file-scope __device__ variable, so every GPU that loads the
-// library holds it until the process exits.  Host code cannot pass the
-// variable's name to a kernel (on the host it is only a stand-in, not a device
-// address): the device address is looked up once per device, with that
-// device current, by cudaGetSymbolAddress on the first call made on it.  That
-// first call should come before any stream capture starts.  Every call shares
-// the one array and leaves its contents behind; the build clears what must
-// start at zero itself.  Calls whose work overlaps on the GPU (two streams,
-// two host threads) race on the array and must not be made.
+// The array is a file-scope __device__ variable.  A GPU holds it from the
+// moment this file's device code is loaded there until the process exits.
+// Under CUDA's default lazy module loading that moment is the first datastore
+// build (this entry point or fc_datastore_build) made on the device, not the
+// library's load: the first call itself places the 30 MiB.  A caller that
+// reserves all free device memory must therefore make one call (a small
+// corpus is enough) before reserving it.
+//
+// Host code cannot pass the variable's name to a kernel (on the host it is
+// only a stand-in, not a device address): every call looks up the device
+// address on the current device with cudaGetSymbolAddress.  The lookup is
+// not cached, so the address stays right after a device reset reloads the
+// module elsewhere.  The first call on a device loads the module, so it
+// should come before any stream capture.  Every call shares the one array
+// and leaves its contents behind; the build clears what must start at zero
+// itself.  Calls whose work overlaps on the GPU (two streams, two host
+// threads) race on the array and must not be made.
 // ---------------------------------------------------------------------------
 namespace {
 constexpr size_t kNoAllocScratchBytes = (size_t)30 << 20;  // 30 MiB
 static __device__ __align__(256) unsigned char g_sa_scratch[kNoAllocScratchBytes];
 
-constexpr int kMaxDevices = 64;
-void* g_scratch_ptr[kMaxDevices] = {nullptr};
-std::mutex g_scratch_mu;
-
 fc_status scratch_for_current_device(void** out) {
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FC_ERR_CUDA;
-  std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_ptr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_sa_scratch) != cudaSuccess || !p) return FC_ERR_CUDA;
-    g_scratch_ptr[dev] = p;
-  }
-  *out = g_scratch_ptr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_sa_scratch) != cudaSuccess || !p) return FC_ERR_CUDA;
+  *out = p;
   return FC_OK;
 }
 }  // namespace

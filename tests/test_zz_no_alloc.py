@@ -7,9 +7,17 @@ scratch space compiled into the library.  This test calls it through the C ABI
 twice in a row (the second corpus is smaller, so leftovers of the first call
 stay in the shared scratch array) and compares each suffix array and bucket
 table with fc_datastore_build's, which must agree exactly (integer outputs).
-It lives in its own file so that pytest collects it after every other test.
+It also checks the property the entry point exists for: once a first call
+has placed the library's scratch array on the device, a call changes the
+device's free memory by nothing.  A fresh process measures what that first
+call places.  The file is named so that pytest collects it after every other
+test.
 """
 import ctypes as C
+import json
+import os
+import subprocess
+import sys
 
 import numpy as np
 import pytest
@@ -68,3 +76,56 @@ def test_noalloc_rejects_oversized_corpus(fc):
     rc = fc.LIB.fc_datastore_build_noalloc(C.c_void_p(tokens.data_ptr()), n, 4, C.c_void_p(tokens.data_ptr()),
                                            C.c_void_p(tokens.data_ptr()), C.c_void_p(tokens.data_ptr()), None, None)
     assert fc.STATUS[rc] == "FC_ERR_CAPACITY"
+
+
+def test_noalloc_call_allocates_nothing(fc):
+    tokens = _corpus(3, 200_000, 1000)
+    _noalloc_call(fc, tokens, 1000)  # the first call on this device places the scratch array
+    torch.cuda.synchronize()
+    sa = torch.empty(tokens.numel(), dtype=torch.int32, device="cuda")
+    bucket = torch.empty(1001, dtype=torch.int32, device="cuda")
+    lcp = torch.empty(tokens.numel(), dtype=torch.uint8, device="cuda")
+    torch.cuda.synchronize()
+    for _ in range(2):
+        free0 = torch.cuda.mem_get_info()[0]
+        rc = fc.LIB.fc_datastore_build_noalloc(C.c_void_p(tokens.data_ptr()), tokens.numel(), 1000,
+                                               C.c_void_p(sa.data_ptr()), C.c_void_p(bucket.data_ptr()),
+                                               C.c_void_p(lcp.data_ptr()),
+                                               C.c_void_p(torch.cuda.current_stream().cuda_stream), None)
+        torch.cuda.synchronize()
+        assert rc == 0
+        assert torch.cuda.mem_get_info()[0] == free0
+
+
+_FIRST_CALL = r"""
+import ctypes as C, json, sys
+import torch
+sys.path.insert(0, sys.argv[1])
+import paper_2502_17139_gb300.fastcoder as fc
+n = 100_000
+tokens = torch.randint(0, 50, (n,), dtype=torch.int32, device="cuda")
+sa = torch.empty(n, dtype=torch.int32, device="cuda")
+bucket = torch.empty(51, dtype=torch.int32, device="cuda")
+lcp = torch.empty(n, dtype=torch.uint8, device="cuda")
+torch.cuda.synchronize()
+free = [torch.cuda.mem_get_info()[0]]
+for _ in range(2):
+    rc = fc.LIB.fc_datastore_build_noalloc(C.c_void_p(tokens.data_ptr()), n, 50, C.c_void_p(sa.data_ptr()),
+                                           C.c_void_p(bucket.data_ptr()), C.c_void_p(lcp.data_ptr()), None, None)
+    torch.cuda.synchronize()
+    assert rc == 0, rc
+    free.append(torch.cuda.mem_get_info()[0])
+print(json.dumps({"first_call_bytes": free[0] - free[1], "second_call_bytes": free[1] - free[2]}))
+"""
+
+
+def test_noalloc_first_call_in_fresh_process(fc):
+    """In a fresh process the first call loads the library's datastore-build
+    module on the device, which places the 30 MiB scratch array (and the
+    module's code); the second call places nothing."""
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, "-c", _FIRST_CALL, root], capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    got = json.loads(r.stdout.strip().splitlines()[-1])
+    assert got["second_call_bytes"] == 0
+    assert 30 << 20 <= got["first_call_bytes"] <= 64 << 20, got
