@@ -39,7 +39,8 @@ typedef enum {
   FC_ERR_CAPACITY = 4,     /* a cache, context or path would overflow its capacity */
   FC_ERR_TIMEOUT = 5,      /* a bounded device-side wait ran out; the kernel returned */
   FC_ERR_CUDA = 6,         /* a CUDA runtime/driver call failed */
-  FC_ERR_INTERNAL = 7      /* an internal consistency check failed */
+  FC_ERR_INTERNAL = 7,     /* an internal consistency check failed */
+  FC_ERR_IO = 8            /* a datastore file could not be written or read, or failed its checks */
 } fc_status;
 
 typedef void* fc_stream; /* cudaStream_t */
@@ -130,15 +131,51 @@ fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n_tokens, uint32
  * d_bucket and d_lcp.
  *   n_tokens must be <= FC_NOALLOC_MAX_TOKENS; larger corpora return
  *   FC_ERR_CAPACITY (use fc_datastore_build with a workspace instead).
- * The first call on a device looks up the array's device address on that
- * device; make it before any stream capture.  All calls share the array:
- * calls whose work overlaps on the GPU (other streams, other host threads)
- * race on it and must not be made.  Synchronous, like fc_datastore_build.
+ * Under CUDA's default lazy module loading the array is placed on a device
+ * by the first datastore build made there (this call or
+ * fc_datastore_build), so that first call needs 30 MiB of free device
+ * memory: a caller that reserves all free memory makes one call (any small
+ * corpus) before reserving it.  Later calls allocate nothing.  Every call
+ * looks up the array's device address on the current device; the first
+ * call on a device loads the library's module there, so make it before any
+ * stream capture.  All calls share the array and find the last call's
+ * contents in it: calls whose work overlaps on the GPU (other streams,
+ * other host threads) race on it and must not be made.  Synchronous, like
+ * fc_datastore_build.
  */
 #define FC_NOALLOC_MAX_TOKENS 1048576ull
 fc_status fc_datastore_build_noalloc(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t vocab,
                                      uint32_t* d_sa, uint32_t* d_bucket, uint8_t* d_lcp,
                                      fc_stream s, fc_datastore* out);
+
+/*
+ * A built datastore on disk (the paper builds its datastores offline, once:
+ * Section IV-A, Section V-C).  One file holds the corpus, the suffix array,
+ * the bucket table and the LCP array, little endian, after a 64-byte header
+ * (magic "FCDSTORE", version 1, vocab, n_tokens, payload bytes, and an FNV-1a
+ * checksum over the payload's 64-bit words); the layout is spelled out in
+ * datastore_io.cu.  on_host != 0: the arrays are host memory (no CUDA call is
+ * made); otherwise device memory, moved through a 64 MiB pinned staging
+ * buffer that the call allocates and frees (these two calls are the only ones
+ * in the library that allocate, host memory only).  Synchronous.
+ *
+ * fc_datastore_save: writes ds to path (replacing the file).  FC_ERR_IO when
+ *   the file cannot be written.
+ * fc_datastore_file_info: n_tokens and vocab from a file's header, so the
+ *   caller can size the buffers.  FC_ERR_IO for a missing or foreign file.
+ * fc_datastore_load: reads a file into the caller's buffers: tokens and sa
+ *   [n_tokens] uint32 (tokens 16-byte aligned), bucket [vocab + 1] uint32,
+ *   lcp [n_tokens] uint8; n_capacity and vocab_capacity bound what the
+ *   buffers hold (FC_ERR_CAPACITY beyond them).  FC_ERR_IO for a missing,
+ *   foreign, truncated or overlong file or a checksum mismatch; the buffers
+ *   may then hold part of the file.  On success `out` (may be NULL) views
+ *   the loaded store.
+ */
+fc_status fc_datastore_save(const char* path, const fc_datastore* ds, int on_host, fc_stream s);
+fc_status fc_datastore_file_info(const char* path, uint64_t* n_tokens, uint32_t* vocab);
+fc_status fc_datastore_load(const char* path, uint32_t* tokens, uint32_t* sa, uint32_t* bucket, uint8_t* lcp,
+                            uint64_t n_capacity, uint32_t vocab_capacity, int on_host, fc_stream s,
+                            fc_datastore* out);
 
 /*
  * The reversed corpus out[i] = tokens[n_tokens - 1 - i] (device buffers of
@@ -511,12 +548,16 @@ fc_status fc_tree_attn_rope(const void* d_q, const void* d_k_cache, const void* 
  * (rotated) and values, and plain GEMMs.  bf16 tensors, row-major, 16-byte
  * aligned; fp32 arithmetic inside.
  * ------------------------------------------------------------------------ */
-/* Workspace bytes fc_gemm_bf16 can use (a caller-owned buffer; NULL works,
- * possibly slower). */
+/* Workspace bytes fc_gemm_bf16 uses: 0 (the arguments stay for callers that
+ * pass a buffer; it is not read). */
 size_t fc_gemm_workspace(void);
 
-/* C[M][N] = A[M][K] B[K][N] (cuBLASLt, fp32 accumulate).  N and K multiples
- * of 8.  Not part of the paper's method: plain library GEMMs. */
+/* C[M][N] = A[M][K] B[K][N], row-major bf16 (A the activations, B the weights
+ * as stored, [K][N]), fp32 accumulation, C rounded to bf16.  The library's
+ * own tcgen05 kernel: tiles of 128 x 256, TMA-fed, accumulators in tensor
+ * memory, persistent over the GPU's SMs.  N and K multiples of 8 (else
+ * FC_ERR_UNSUPPORTED); pointers 16-byte aligned.  Asynchronous; a bounded
+ * wait that runs out sets FC_ERR_TIMEOUT in the device error word. */
 fc_status fc_gemm_bf16(const void* d_a, const void* d_b, void* d_c, int M, int N, int K, void* d_ws,
                        size_t ws_bytes, fc_stream s);
 

@@ -1,27 +1,18 @@
 // The pieces of a decoder forward around the tree attention (Section IV-D:
 // the target model verifies every draft in one forward), for a LLaMA-family
 // model like the paper's: token embedding, residual add + RMSNorm, the
-// SiLU-gated MLP's activation, the head-major layout of the tree's keys
-// (rotated) and values, and plain GEMMs through cuBLASLt.
+// SiLU-gated MLP's activation and the head-major layout of the tree's keys
+// (rotated) and values.  The GEMMs are gemm.cu's tcgen05 kernel.
 //
-//   * fc_gemm_bf16: C[M][N] = A[M][K] B[K][N], row-major bf16, fp32
-//     accumulate.  Row-major C = A B is column-major C^T = B^T A^T, so B's
-//     memory is cuBLASLt's first operand.  The heuristic's algorithm is cached
-//     per shape.
 //   * k_embed: one row per warp; ids >= vocab (tree padding) embed as zeros.
 //   * k_add_rmsnorm: one row per warp; x += r is rounded to bf16 (the
 //     residual stream), then out = x / sqrt(mean(x^2) + eps) * w in fp32.
 //   * k_silu_mul: out = silu(gate) * up, fp32 math.
 //   * k_rope_heads: node-major projection rows -> head-major [B][heads][n][D],
 //     rotated by position (the rotation of tree_attn.cu) or copied.
-#include <cublasLt.h>
-
 #include <algorithm>
 #include <cmath>
 
-#include <map>
-#include <mutex>
-#include <tuple>
 
 #include "fc_common.cuh"
 
@@ -181,79 +172,9 @@ __global__ void k_rope_heads(const __nv_bfloat16* __restrict__ in, int stride, _
   }
 }
 
-// ---- cuBLASLt
-struct Lt {
-  std::mutex mu;
-  cublasLtHandle_t h = nullptr;
-  std::map<std::tuple<int, int, int, size_t>, cublasLtMatmulAlgo_t> algos;
-};
-Lt& lt() {
-  static Lt s;
-  return s;
-}
-
 bool aligned16(const void* p) { return reinterpret_cast<uintptr_t>(p) % 16 == 0; }
 
 }  // namespace
-
-extern "C" size_t fc_gemm_workspace(void) { return (size_t)32 << 20; }
-
-extern "C" fc_status fc_gemm_bf16(const void* d_a, const void* d_b, void* d_c, int M, int N, int K, void* d_ws,
-                                  size_t ws_bytes, fc_stream stream) {
-  if (M < 0 || N < 1 || K < 1) return FC_ERR_INVALID_ARG;
-  if (M == 0) return FC_OK;
-  if (!d_a || !d_b || !d_c) return FC_ERR_INVALID_ARG;
-  if (!aligned16(d_a) || !aligned16(d_b) || !aligned16(d_c) || (d_ws && !aligned16(d_ws))) return FC_ERR_INVALID_ARG;
-  if (N % 8 || K % 8) return FC_ERR_UNSUPPORTED;
-  Lt& s = lt();
-  std::lock_guard<std::mutex> g(s.mu);
-  if (!s.h && cublasLtCreate(&s.h) != CUBLAS_STATUS_SUCCESS) return FC_ERR_CUDA;
-  const size_t ws = d_ws ? ws_bytes : 0;
-  cublasLtMatmulDesc_t op = nullptr;
-  cublasLtMatrixLayout_t lb = nullptr, la = nullptr, lc = nullptr;
-  fc_status st = FC_OK;
-  // column-major: C^T (N x M, ld N) = B^T (N x K, ld N) * A^T (K x M, ld K)
-  if (cublasLtMatmulDescCreate(&op, CUBLAS_COMPUTE_32F, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS ||
-      cublasLtMatrixLayoutCreate(&lb, CUDA_R_16BF, N, K, N) != CUBLAS_STATUS_SUCCESS ||
-      cublasLtMatrixLayoutCreate(&la, CUDA_R_16BF, K, M, K) != CUBLAS_STATUS_SUCCESS ||
-      cublasLtMatrixLayoutCreate(&lc, CUDA_R_16BF, N, M, N) != CUBLAS_STATUS_SUCCESS) {
-    st = FC_ERR_CUDA;
-  }
-  cublasLtMatmulAlgo_t algo;
-  if (st == FC_OK) {
-    auto key = std::make_tuple(M, N, K, ws);
-    auto it = s.algos.find(key);
-    if (it != s.algos.end()) {
-      algo = it->second;
-    } else {
-      cublasLtMatmulPreference_t pref = nullptr;
-      cublasLtMatmulHeuristicResult_t res;
-      int n_res = 0;
-      if (cublasLtMatmulPreferenceCreate(&pref) != CUBLAS_STATUS_SUCCESS ||
-          cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES, &ws, sizeof ws) !=
-              CUBLAS_STATUS_SUCCESS ||
-          cublasLtMatmulAlgoGetHeuristic(s.h, op, lb, la, lc, lc, pref, 1, &res, &n_res) != CUBLAS_STATUS_SUCCESS ||
-          n_res < 1) {
-        st = FC_ERR_UNSUPPORTED;
-      } else {
-        algo = res.algo;
-        s.algos[key] = algo;
-      }
-      if (pref) cublasLtMatmulPreferenceDestroy(pref);
-    }
-  }
-  if (st == FC_OK) {
-    const float one = 1.f, zero = 0.f;
-    if (cublasLtMatmul(s.h, op, &one, d_b, lb, d_a, la, &zero, d_c, lc, d_c, lc, &algo, d_ws, ws,
-                       static_cast<cudaStream_t>(stream)) != CUBLAS_STATUS_SUCCESS)
-      st = FC_ERR_CUDA;
-  }
-  if (lc) cublasLtMatrixLayoutDestroy(lc);
-  if (la) cublasLtMatrixLayoutDestroy(la);
-  if (lb) cublasLtMatrixLayoutDestroy(lb);
-  if (op) cublasLtMatmulDescDestroy(op);
-  return st;
-}
 
 extern "C" fc_status fc_embed(const uint32_t* d_tok, int n, const void* d_table, int vocab, int hidden, void* d_out,
                               fc_stream stream) {

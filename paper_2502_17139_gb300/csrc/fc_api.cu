@@ -8,6 +8,7 @@ extern "C" unsigned int fc_take_error_step(cudaStream_t s);
 extern "C" unsigned int fc_take_error_attn(cudaStream_t s);
 extern "C" unsigned int fc_take_error_cache(cudaStream_t s);
 extern "C" unsigned int fc_take_error_dec(cudaStream_t s);
+extern "C" unsigned int fc_take_error_gemm(cudaStream_t s);
 
 extern "C" const char* fc_status_string(fc_status s) {
   switch (s) {
@@ -19,6 +20,7 @@ extern "C" const char* fc_status_string(fc_status s) {
     case FC_ERR_TIMEOUT: return "FC_ERR_TIMEOUT";
     case FC_ERR_CUDA: return "FC_ERR_CUDA";
     case FC_ERR_INTERNAL: return "FC_ERR_INTERNAL";
+    case FC_ERR_IO: return "FC_ERR_IO";
   }
   return "FC_ERR_UNKNOWN";
 }
@@ -30,7 +32,7 @@ extern "C" fc_status fc_get_error(fc_stream stream) {
   if (cudaStreamSynchronize(s) != cudaSuccess) return FC_ERR_CUDA;
   unsigned int e = fc_take_error_sa(s) | fc_take_error_ret(s) | fc_take_error_tree(s) | fc_take_error_step(s) |
                    fc_take_error_attn(s) | fc_take_error_cache(s) |
-                   fc_take_error_dec(s);
+                   fc_take_error_dec(s) | fc_take_error_gemm(s);
   if (e & FC_EBIT_INTERNAL) return FC_ERR_INTERNAL;
   if (e & FC_EBIT_TIMEOUT) return FC_ERR_TIMEOUT;
   if (e & FC_EBIT_CAPACITY) return FC_ERR_CAPACITY;

@@ -14,6 +14,7 @@ from __future__ import annotations
 import ctypes as C
 import os
 
+import numpy as np
 import torch
 
 from . import build as _build
@@ -24,7 +25,7 @@ MAX_OCC = 4096
 MAX_NODES = 128
 
 STATUS = {0: "FC_OK", 1: "FC_ERR_INVALID_ARG", 2: "FC_ERR_UNSUPPORTED", 3: "FC_ERR_WORKSPACE",
-          4: "FC_ERR_CAPACITY", 5: "FC_ERR_TIMEOUT", 6: "FC_ERR_CUDA", 7: "FC_ERR_INTERNAL"}
+          4: "FC_ERR_CAPACITY", 5: "FC_ERR_TIMEOUT", 6: "FC_ERR_CUDA", 7: "FC_ERR_INTERNAL", 8: "FC_ERR_IO"}
 
 
 class FastCoderError(RuntimeError):
@@ -50,7 +51,7 @@ class fc_cache(C.Structure):
 
 
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
-           "fc_datastore_build_noalloc",
+           "fc_datastore_build_noalloc", "fc_datastore_save", "fc_datastore_file_info", "fc_datastore_load",
            "fc_retrieve", "fc_retrieve_all", "fc_retrieve_rev", "fc_reverse_tokens", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
            "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_embed",
@@ -70,6 +71,9 @@ def _load():
         "fc_datastore_build_workspace": (sz, [u64, u32]),
         "fc_datastore_build": (C.c_int, [vp, u64, u32, vp, vp, vp, vp, sz, vp, C.POINTER(fc_datastore)]),
         "fc_datastore_build_noalloc": (C.c_int, [vp, u64, u32, vp, vp, vp, vp, C.POINTER(fc_datastore)]),
+        "fc_datastore_save": (C.c_int, [C.c_char_p, C.POINTER(fc_datastore), i32, vp]),
+        "fc_datastore_file_info": (C.c_int, [C.c_char_p, C.POINTER(C.c_uint64), C.POINTER(C.c_uint32)]),
+        "fc_datastore_load": (C.c_int, [C.c_char_p, vp, vp, vp, vp, u64, u32, i32, vp, C.POINTER(fc_datastore)]),
         "fc_retrieve": (C.c_int, [C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp, fc_retrieve_params,
                                   vp, vp, vp, vp, vp, vp]),
         "fc_retrieve_all": (C.c_int, [C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp, fc_retrieve_params,
@@ -201,6 +205,55 @@ def fc_datastore_build(tokens: torch.Tensor, vocab: int, workspace: torch.Tensor
     _check("fc_datastore_build", LIB.fc_datastore_build(_ptr(tokens), n, vocab, _ptr(sa), _ptr(bucket), _ptr(lcp),
                                                         _ptr(ws), ws.numel(), _stream(), None))
     return Datastore(tokens, sa, bucket, lcp, vocab)
+
+
+def _np_ptr(a):
+    return C.c_void_p(a.ctypes.data)
+
+
+def fc_datastore_save(ds: Datastore, path: str) -> None:
+    """Writes a device datastore to ``path`` (synchronous)."""
+    _check("fc_datastore_save", LIB.fc_datastore_save(os.fsencode(path), C.byref(ds.view), 0, _stream()))
+
+
+def fc_datastore_file_info(path: str):
+    """(n_tokens, vocab) from a datastore file's header."""
+    n, v = C.c_uint64(0), C.c_uint32(0)
+    _check("fc_datastore_file_info", LIB.fc_datastore_file_info(os.fsencode(path), C.byref(n), C.byref(v)))
+    return int(n.value), int(v.value)
+
+
+def fc_datastore_load(path: str, device="cuda") -> Datastore:
+    """Reads a datastore file into new device tensors (synchronous)."""
+    n, vocab = fc_datastore_file_info(path)
+    tokens = torch.empty(n, dtype=torch.int32, device=device)
+    sa = torch.empty(n, dtype=torch.int32, device=device)
+    bucket = torch.empty(vocab + 1, dtype=torch.int32, device=device)
+    lcp = torch.empty(n, dtype=torch.uint8, device=device)
+    _check("fc_datastore_load", LIB.fc_datastore_load(os.fsencode(path), _ptr(tokens), _ptr(sa), _ptr(bucket),
+                                                      _ptr(lcp), n, vocab, 0, _stream(), None))
+    return Datastore(tokens, sa, bucket, lcp, vocab)
+
+
+def datastore_save_host(path: str, tokens, sa, bucket, lcp) -> None:
+    """The same file from host arrays (numpy uint32 tokens / sa / bucket,
+    uint8 lcp); no CUDA call is made."""
+    arrs = [np.ascontiguousarray(tokens, np.uint32), np.ascontiguousarray(sa, np.uint32),
+            np.ascontiguousarray(bucket, np.uint32), np.ascontiguousarray(lcp, np.uint8)]
+    view = fc_datastore(arrs[0].ctypes.data, arrs[1].ctypes.data, arrs[2].ctypes.data, arrs[3].ctypes.data,
+                        len(arrs[0]), len(arrs[2]) - 1)
+    _check("fc_datastore_save", LIB.fc_datastore_save(os.fsencode(path), C.byref(view), 1, None))
+
+
+def datastore_load_host(path: str):
+    """A datastore file into host arrays: dict(tokens, sa, bucket, lcp)."""
+    n, vocab = fc_datastore_file_info(path)
+    out = dict(tokens=np.empty(n, np.uint32), sa=np.empty(n, np.uint32), bucket=np.empty(vocab + 1, np.uint32),
+               lcp=np.empty(n, np.uint8))
+    _check("fc_datastore_load", LIB.fc_datastore_load(os.fsencode(path), _np_ptr(out["tokens"]), _np_ptr(out["sa"]),
+                                                      _np_ptr(out["bucket"]), _np_ptr(out["lcp"]), n, vocab, 1, None,
+                                                      None))
+    return out
 
 
 NOALLOC_MAX_TOKENS = 1 << 20
@@ -552,21 +605,9 @@ def fc_tree_attn_rope(q, k_cache, v_cache, kv_len, k_tree_rot, v_tree, mask, n_n
 
 
 # ------------------------------------------------------- decoder blocks
-_GEMM_WS = {}
-
-
-def gemm_workspace(device):
-    """The cuBLASLt workspace fc_gemm_bf16 uses, one per device and shared by every
-    call: GEMMs that may overlap on different streams need their own."""
-    key = str(device)
-    if key not in _GEMM_WS:
-        _GEMM_WS[key] = torch.empty(int(LIB.fc_gemm_workspace()), dtype=torch.uint8, device=device)
-    return _GEMM_WS[key]
-
-
-def fc_gemm_bf16(a, b, out=None, workspace=None):
-    """a [M, K] @ b [K, N] (bf16, row-major) -> [M, N] bf16.  ``workspace``:
-    None (the shared per-device one) or a uint8 device tensor."""
+def fc_gemm_bf16(a, b, out=None):
+    """a [M, K] @ b [K, N] (bf16, row-major) -> [M, N] bf16 (the library's
+    tcgen05 GEMM; it needs no workspace)."""
     _need(a, torch.bfloat16, "a")
     _need(b, torch.bfloat16, "b")
     M, K = a.shape
@@ -574,8 +615,10 @@ def fc_gemm_bf16(a, b, out=None, workspace=None):
     if K != K2:
         raise ValueError("inner dimensions differ")
     o = out if out is not None else torch.empty((M, N), dtype=torch.bfloat16, device=a.device)
-    ws = workspace if workspace is not None else gemm_workspace(a.device)
-    _check("fc_gemm_bf16", LIB.fc_gemm_bf16(_ptr(a), _ptr(b), _ptr(o), M, N, K, _ptr(ws), ws.numel(), _stream()))
+    _need(o, torch.bfloat16, "out")
+    if tuple(o.shape) != (M, N):
+        raise ValueError("out must be [M, N]")
+    _check("fc_gemm_bf16", LIB.fc_gemm_bf16(_ptr(a), _ptr(b), _ptr(o), M, N, K, None, 0, _stream()))
     return o
 
 
