@@ -81,7 +81,7 @@ def parse_args(argv=None):
     ap.add_argument("--batch", type=int, default=32)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--mode", choices=["step", "attn", "argmax", "configs", "retrieve", "algorithm1", "cache", "gemm",
+    ap.add_argument("--mode", choices=["step", "attn", "argmax", "configs", "retrieve", "algorithm1", "cache", "gemm", "build",
                                        "decoder"],
                     default="step",
                     help="step: the full step loop (the benchmark); attn: tree attention alone on the step loop's "
@@ -106,6 +106,7 @@ def parse_args(argv=None):
     ap.add_argument("--fill", type=int, default=None,
                     help="algorithm1 / cache modes: steps that fill the CACHE first (default 100 / 450)")
     ap.add_argument("--skip-1b", action="store_true", help="configs mode: leave out the 1B-token configuration")
+    ap.add_argument("--tokens", type=int, default=100_000_000, help="build mode: corpus tokens (Zipf 1.1)")
     ap.add_argument("--traffic-bytes", type=float, default=None,
                     help="ncu dram read+write bytes of one single-stream tree-attention launch of this workload")
     return ap.parse_args(argv)
@@ -1117,6 +1118,14 @@ def run_retrieve(args, rank, ws, local):
            "config": {"workload": f"two-source retrieval (5M + 100M tokens), {args.batch} contexts of 128, "
                                   f"n 16->2, top-64 x 10"},
            "us_per_query_source": ms * 1e3 / (2 * args.batch)}
+    # the same search without the suffix keys (probes read the suffix array,
+    # then the corpus), on the same queries
+    plain = [s.without_keys() for s in sources]
+    rp = fc.fc_retrieve(plain, ctx_d, cl_d, p)
+    assert all(torch.equal(res[k], rp[k]) for k in res) and fc.fc_get_error() == "FC_OK"
+    ms_p = _gpu_ms(lambda: fc.fc_retrieve(plain, ctx_d, cl_d, p, out=rp), reps=args.steps, warm=args.warmup)
+    out["without_keys"] = {"ms_per_step": ms_p, "us_per_query_source": ms_p * 1e3 / (2 * args.batch),
+                           "query_sources_per_s": 2 * args.batch / (ms_p * 1e-3)}
     if args.rev:
         # the reversed-corpus variant on the same queries: n* by one narrowing
         # search in the reversed suffix arrays, then the forward search for n*
@@ -1476,6 +1485,39 @@ def run_gemm(args, rank, ws, local):
             "shapes": rows}
 
 
+def run_build(args, rank, ws, local):
+    """fc_datastore_build alone: a Zipf(1.1) corpus of --tokens tokens over
+    vocab 32256 (the general store's law), built --steps times after
+    --warmup builds; CUDA events around each synchronous build."""
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    import paper_2502_17139_gb300.synth as synth
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    rng = synth.rng_for(2, 77)
+    T = synth.zipf_tokens(rng, args.tokens, 1.1, synth.VOCAB, device=dev)
+    tok = torch.from_numpy(T.view(np.int32)).to(dev)
+    n = tok.numel()
+    ws_t = torch.empty(fc.fc_datastore_build_workspace(n, synth.VOCAB), dtype=torch.uint8, device=dev)
+    times = []
+    for i in range(args.warmup + args.steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        ds = fc.fc_datastore_build(tok, synth.VOCAB, workspace=ws_t)
+        e1.record()
+        torch.cuda.synchronize()
+        if i >= args.warmup:
+            times.append(e0.elapsed_time(e1))
+        del ds
+    assert fc.fc_get_error() == "FC_OK"
+    ms = statistics.mean(times)
+    return {"metric": "datastore build tokens/s", "value": n / (ms * 1e-3), "unit": "tokens/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_build": ms, "higher_is_better": True,
+            "dtype": "u32", "data": "synthetic",
+            "config": {"workload": f"suffix array + bucket table + LCP of {n} Zipf(1.1) tokens, vocab 32256"}}
+
+
 def main(argv=None):
     args = parse_args(argv)
     rank, ws, local = dist_setup(args.gpus)
@@ -1497,6 +1539,8 @@ def main(argv=None):
         out = run_decoder(args, rank, ws, local)
     elif args.mode == "gemm":
         out = run_gemm(args, rank, ws, local)
+    elif args.mode == "build":
+        out = run_build(args, rank, ws, local)
     else:
         out = run_ours(args, rank, ws, local)
     if rank == 0 and out is not None:

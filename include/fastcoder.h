@@ -95,7 +95,23 @@ typedef struct {
                               FC_LCP_CAP; lcp[0] = 0 */
   uint64_t n_tokens;       /* 1 <= n_tokens < 2^32 - 1 */
   uint32_t vocab;          /* 1 <= vocab < 2^31 */
+  const uint32_t* keys;    /* device, optional (NULL: not used): [n_tokens][8] suffix
+                              keys from fc_datastore_keys, 32-byte aligned */
 } fc_datastore;
+
+/*
+ * Suffix keys: an index over the suffix array, not a step of the paper.
+ * Entry j (8 uint32, 32 bytes) holds sa[j] and the suffix's tokens 1..7
+ * (FC_PAD_TOKEN past the corpus end).  With keys set in the datastore view,
+ * fc_retrieve's binary-search probes read one 32-byte entry (one DRAM
+ * sector) where they would read the suffix array and then the corpus: a
+ * probe touches the corpus only when the pattern's first eight tokens tie
+ * with the suffix's.  Results are identical with and without keys.
+ *   ds      a built datastore (tokens and sa are read)
+ *   d_keys  [n_tokens][8] uint32 out, 32-byte aligned (32 bytes per token)
+ * Asynchronous.  The caller then sets ds.keys = d_keys in its view.
+ */
+fc_status fc_datastore_keys(const fc_datastore* ds, uint32_t* d_keys, fc_stream s);
 
 /* Workspace bytes fc_datastore_build needs for n_tokens tokens. */
 size_t fc_datastore_build_workspace(uint64_t n_tokens, uint32_t vocab);

@@ -144,6 +144,7 @@ fc_status read_header(std::FILE* f, uint64_t* n, uint32_t* vocab, uint64_t* sum)
 }  // namespace
 
 extern "C" fc_status fc_datastore_save(const char* path, const fc_datastore* ds, int on_host, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (!path || !ds || !ds->tokens || !ds->sa || !ds->bucket || !ds->lcp || ds->n_tokens == 0 ||
       ds->n_tokens >= 0xFFFFFFFFull || ds->vocab == 0)
     return FC_ERR_INVALID_ARG;
@@ -183,6 +184,7 @@ extern "C" fc_status fc_datastore_save(const char* path, const fc_datastore* ds,
 }
 
 extern "C" fc_status fc_datastore_file_info(const char* path, uint64_t* n_tokens, uint32_t* vocab) {
+  FC_NVTX_RANGE();
   if (!path || !n_tokens || !vocab) return FC_ERR_INVALID_ARG;
   if (!little_endian()) return FC_ERR_UNSUPPORTED;
   std::FILE* f = std::fopen(path, "rb");
@@ -196,6 +198,7 @@ extern "C" fc_status fc_datastore_file_info(const char* path, uint64_t* n_tokens
 extern "C" fc_status fc_datastore_load(const char* path, uint32_t* tokens, uint32_t* sa, uint32_t* bucket,
                                        uint8_t* lcp, uint64_t n_capacity, uint32_t vocab_capacity, int on_host,
                                        fc_stream stream, fc_datastore* out) {
+  FC_NVTX_RANGE();
   if (!path || !tokens || !sa || !bucket || !lcp) return FC_ERR_INVALID_ARG;
   if (!little_endian()) return FC_ERR_UNSUPPORTED;
   std::FILE* f = std::fopen(path, "rb");
@@ -233,6 +236,7 @@ extern "C" fc_status fc_datastore_load(const char* path, uint32_t* tokens, uint3
     out->lcp = lcp;
     out->n_tokens = n;
     out->vocab = vocab;
+    out->keys = nullptr;
   }
   return st;
 }

@@ -54,6 +54,7 @@ struct DsView {
   const uint8_t* lcp;
   uint64_t n;
   uint32_t vocab;
+  const uint4* keys;  // suffix keys (two uint4 per SA entry) or nullptr
 };
 struct DsArgs {
   DsView ds[FC_MAX_SOURCES];
@@ -107,6 +108,31 @@ __device__ __forceinline__ int cmp_suffix_vec(const uint32_t* __restrict__ T, ui
     }
   }
   return res;
+}
+
+// The same sign for the suffix at SA index piv, from its key entry: the
+// suffix start and tokens 1..7 in one 32-byte read (FC_PAD_TOKEN past the
+// corpus end, where the suffix ended and sorts first).  Tokens from 8 on
+// come from the corpus, and only when the first eight tie.
+__device__ __forceinline__ int cmp_suffix_key(const uint4* __restrict__ keys, const uint32_t* __restrict__ T,
+                                              uint64_t N, uint32_t piv, const uint32_t* pat, int n, uint32_t* at) {
+  const uint4 a = __ldg(keys + 2 * (size_t)piv), c = __ldg(keys + 2 * (size_t)piv + 1);
+  *at = a.x;
+  const uint32_t t[8] = {a.x, a.y, a.z, a.w, c.x, c.y, c.z, c.w};
+  int res = 0;
+#pragma unroll
+  for (int k = 1; k < 8; ++k) {
+    if (k < n && res == 0) {
+      const uint32_t v = t[k], q = pat[k];
+      if (v == FC_PAD_TOKEN)
+        res = -1;
+      else if (v != q)
+        res = v < q ? -1 : 1;
+    }
+  }
+  if (res != 0 || n <= 8) return res;
+  // token 7 is known equal: compare tokens 8 .. n-1
+  return cmp_suffix_vec(T, N, (uint64_t)a.x + 7, pat + 7, n - 7);
 }
 
 struct RetSmem {
@@ -237,7 +263,10 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev
         const uint32_t piv = lo + (uint32_t)(((uint64_t)(hl + 1) * (hi - lo)) / 17u);
         bool pred = true;  // suffix at piv is past the bound's side
         if (active) {
-          const int c = cmp_suffix_vec(T, N, __ldg(ds.sa + piv), pat, n);
+          uint32_t at = 0;
+          const int c = ds.keys ? cmp_suffix_key(ds.keys, T, N, piv, pat, n, &at)
+                                : cmp_suffix_vec(T, N, (at = __ldg(ds.sa + piv)), pat, n);
+          FC_DEBUG_CHECK(at < N);
           pred = upper ? (c > 0) : (c >= 0);
         }
         const unsigned bal = __ballot_sync(0xFFFFFFFFu, !pred) & half_mask;
@@ -318,17 +347,19 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev
     int t = e / d, x = e - t * d;
     uint32_t v = FC_PAD_TOKEN;
     if (t < nd) {
-      const uint32_t pp = __ldg(ds.sa + first + sm.runs[run_at(t)]) + (uint32_t)ns;
-      uint64_t len = min((uint64_t)d, N - pp);
-      if ((uint64_t)x < len) v = __ldg(T + pp + x);
+      const uint64_t pp = (uint64_t)__ldg(ds.sa + first + sm.runs[run_at(t)]) + (uint64_t)ns;
+      if (FC_DEBUG_CHECK(pp < N)) {
+        const uint64_t len = min((uint64_t)d, N - pp);
+        if ((uint64_t)x < len) v = __ldg(T + pp + x);
+      }
     }
     dr[e] = v;
   }
   for (int t = tid; t < k; t += RT_THREADS) {
     if (t < nd) {
       const uint32_t r = run_at(t);
-      const uint32_t pp = __ldg(ds.sa + first + sm.runs[r]) + (uint32_t)ns;
-      dl[t] = (int32_t)min((uint64_t)d, N - pp);
+      const uint64_t pp = (uint64_t)__ldg(ds.sa + first + sm.runs[r]) + (uint64_t)ns;
+      dl[t] = pp < N ? (int32_t)min((uint64_t)d, N - pp) : 0;
       ct[t] = run_count(r);
     } else {
       dl[t] = 0;
@@ -510,7 +541,9 @@ static fc_status launch_retrieve(bool all, const fc_datastore* sources, const fc
         ds.vocab == 0)
       return FC_ERR_INVALID_ARG;
     if (reinterpret_cast<uintptr_t>(ds.tokens) % 16) return FC_ERR_INVALID_ARG;  // read as 16-byte vectors
-    a.ds[s] = DsView{ds.tokens, ds.sa, ds.bucket, ds.lcp, ds.n_tokens, ds.vocab};
+    if (reinterpret_cast<uintptr_t>(ds.keys) % 32) return FC_ERR_INVALID_ARG;
+    a.ds[s] = DsView{ds.tokens, ds.sa, ds.bucket, ds.lcp, ds.n_tokens, ds.vocab,
+                     reinterpret_cast<const uint4*>(ds.keys)};
   }
   DsArgs r{};
   if (rev_sources) {
@@ -518,7 +551,7 @@ static fc_status launch_retrieve(bool all, const fc_datastore* sources, const fc
       const fc_datastore& rv = rev_sources[s];
       if (!rv.tokens || !rv.sa || !rv.bucket || rv.n_tokens != sources[s].n_tokens || rv.vocab != sources[s].vocab)
         return FC_ERR_INVALID_ARG;
-      r.ds[s] = DsView{rv.tokens, rv.sa, rv.bucket, rv.lcp, rv.n_tokens, rv.vocab};
+      r.ds[s] = DsView{rv.tokens, rv.sa, rv.bucket, rv.lcp, rv.n_tokens, rv.vocab, nullptr};
     }
   }
   const int variant = all ? 2 : (rev_sources ? 1 : 0);
@@ -540,6 +573,7 @@ extern "C" fc_status fc_retrieve(const fc_datastore* sources, int n_sources, con
                                  const int32_t* d_ctx_len, int batch, const int32_t* d_skip, fc_retrieve_params p,
                                  uint32_t* d_drafts, int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
                                  int32_t* d_match_len, fc_stream stream) {
+  FC_NVTX_RANGE();
   return launch_retrieve(false, sources, nullptr, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, d_drafts,
                          d_draft_len, d_count, d_n_drafts, d_match_len, stream);
 }
@@ -548,6 +582,7 @@ extern "C" fc_status fc_retrieve_all(const fc_datastore* sources, int n_sources,
                                      int ctx_stride, const int32_t* d_ctx_len, int batch, const int32_t* d_skip,
                                      fc_retrieve_params p, uint32_t* d_drafts, int32_t* d_draft_len,
                                      uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len, fc_stream stream) {
+  FC_NVTX_RANGE();
   return launch_retrieve(true, sources, nullptr, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, d_drafts,
                          d_draft_len, d_count, d_n_drafts, d_match_len, stream);
 }
@@ -557,6 +592,7 @@ extern "C" fc_status fc_retrieve_rev(const fc_datastore* sources, const fc_datas
                                      const int32_t* d_skip, fc_retrieve_params p, uint32_t* d_drafts,
                                      int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
                                      int32_t* d_match_len, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (!rev_sources) return FC_ERR_INVALID_ARG;
   return launch_retrieve(false, sources, rev_sources, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, d_skip, p, d_drafts,
                          d_draft_len, d_count, d_n_drafts, d_match_len, stream);
@@ -574,6 +610,7 @@ static bool rc_args_ok(int capacity, int n_sources, const fc_retrieve_params& p)
 
 extern "C" fc_status fc_rcache_init(void* d_table, size_t bytes, int capacity, int n_sources, fc_retrieve_params p,
                                     fc_stream stream) {
+  FC_NVTX_RANGE();
   if (!d_table || !rc_args_ok(capacity, n_sources, p)) return FC_ERR_INVALID_ARG;
   if (bytes < fc_rcache_bytes(capacity, n_sources, p)) return FC_ERR_WORKSPACE;
   unsigned g = (unsigned)std::min<size_t>((capacity + 255) / 256, 4096);
@@ -587,6 +624,7 @@ extern "C" fc_status fc_rcache_lookup(const void* d_table, int capacity, int n_s
                                       const int32_t* d_want_hit, int32_t* d_skip, uint32_t* d_drafts,
                                       int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts,
                                       int32_t* d_match_len, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (!d_table || !rc_args_ok(capacity, n_sources, p) || batch < 0 || ctx_stride < 1) return FC_ERR_INVALID_ARG;
   if (batch == 0) return FC_OK;
   if (!d_ctx || !d_ctx_len || !d_skip || !d_drafts || !d_draft_len || !d_count || !d_n_drafts || !d_match_len)
@@ -603,6 +641,7 @@ extern "C" fc_status fc_rcache_insert(void* d_table, int capacity, int n_sources
                                       const int32_t* d_skip, const uint32_t* d_drafts, const int32_t* d_draft_len,
                                       const uint32_t* d_count, const int32_t* d_n_drafts, const int32_t* d_match_len,
                                       fc_stream stream) {
+  FC_NVTX_RANGE();
   if (!d_table || !rc_args_ok(capacity, n_sources, p) || batch < 0 || ctx_stride < 1) return FC_ERR_INVALID_ARG;
   if (batch == 0) return FC_OK;
   if (!d_ctx || !d_ctx_len || !d_drafts || !d_draft_len || !d_count || !d_n_drafts || !d_match_len)

@@ -316,6 +316,7 @@ extern "C" size_t fc_datastore_build_workspace(uint64_t n_tokens, uint32_t vocab
 extern "C" fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n, uint32_t vocab, uint32_t* d_sa,
                                         uint32_t* d_bucket, uint8_t* d_lcp, void* d_ws, size_t ws_bytes,
                                         fc_stream stream, fc_datastore* out) {
+  FC_NVTX_RANGE();
   if (!d_tokens || !d_sa || !d_bucket || !d_lcp || n == 0 || n >= 0xFFFFFFFFull || vocab == 0 ||
       vocab >= 0x80000000u)
     return FC_ERR_INVALID_ARG;
@@ -389,6 +390,7 @@ extern "C" fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n, ui
     out->lcp = d_lcp;
     out->n_tokens = n;
     out->vocab = vocab;
+    out->keys = nullptr;
   }
   return FC_OK;
 }
@@ -436,12 +438,44 @@ fc_status scratch_for_current_device(void** out) {
 extern "C" fc_status fc_datastore_build_noalloc(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t vocab,
                                                 uint32_t* d_sa, uint32_t* d_bucket, uint8_t* d_lcp,
                                                 fc_stream stream, fc_datastore* out) {
+  FC_NVTX_RANGE();
   if (n_tokens > FC_NOALLOC_MAX_TOKENS) return FC_ERR_CAPACITY;
   if (n_tokens > 0 && fc_datastore_build_workspace(n_tokens, vocab) > kNoAllocScratchBytes) return FC_ERR_CAPACITY;
   void* ws = nullptr;
   fc_status st = scratch_for_current_device(&ws);
   if (st != FC_OK) return st;
   return fc_datastore_build(d_tokens, n_tokens, vocab, d_sa, d_bucket, d_lcp, ws, kNoAllocScratchBytes, stream, out);
+}
+
+// ---------------------------------------------------------------------------
+// Suffix keys: entry j = (sa[j], T[sa[j] + 1 .. sa[j] + 7]), FC_PAD_TOKEN past
+// the corpus end; 32 bytes, written as two 16-byte stores.
+// ---------------------------------------------------------------------------
+namespace {
+__global__ void k_suffix_keys(const uint32_t* __restrict__ T, const uint32_t* __restrict__ sa, uint64_t n,
+                              uint4* __restrict__ keys) {
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  for (uint64_t j = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; j < n; j += stride) {
+    const uint64_t i = __ldg(sa + j);
+    uint32_t t[8];
+    t[0] = (uint32_t)i;
+#pragma unroll
+    for (int k = 1; k < 8; ++k) t[k] = (i + k < n) ? __ldg(T + i + k) : FC_PAD_TOKEN;
+    keys[2 * j] = make_uint4(t[0], t[1], t[2], t[3]);
+    keys[2 * j + 1] = make_uint4(t[4], t[5], t[6], t[7]);
+  }
+}
+}  // namespace
+
+extern "C" fc_status fc_datastore_keys(const fc_datastore* ds, uint32_t* d_keys, fc_stream stream) {
+  FC_NVTX_RANGE();
+  if (!ds || !ds->tokens || !ds->sa || !d_keys || ds->n_tokens == 0 || ds->n_tokens >= 0xFFFFFFFFull)
+    return FC_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(d_keys) % 32) return FC_ERR_INVALID_ARG;
+  const uint64_t n = ds->n_tokens;
+  k_suffix_keys<<<grid_for(n, 256), 256, 0, static_cast<cudaStream_t>(stream)>>>(ds->tokens, ds->sa, n,
+                                                                                 reinterpret_cast<uint4*>(d_keys));
+  return FC_CHECK_LAUNCH();
 }
 
 // ---------------------------------------------------------------------------
@@ -470,6 +504,7 @@ __global__ void k_reverse(const uint32_t* __restrict__ in, uint64_t n, uint32_t*
 
 extern "C" fc_status fc_reverse_tokens(const uint32_t* d_tokens, uint64_t n_tokens, uint32_t* d_out,
                                        fc_stream stream) {
+  FC_NVTX_RANGE();
   if (n_tokens == 0) return FC_OK;
   if (!d_tokens || !d_out || d_tokens == d_out || n_tokens >= 0xFFFFFFFFull) return FC_ERR_INVALID_ARG;
   const uint64_t a = reinterpret_cast<uintptr_t>(d_tokens), b = reinterpret_cast<uintptr_t>(d_out);

@@ -37,7 +37,7 @@ class FastCoderError(RuntimeError):
 
 class fc_datastore(C.Structure):
     _fields_ = [("tokens", C.c_void_p), ("sa", C.c_void_p), ("bucket", C.c_void_p), ("lcp", C.c_void_p),
-                ("n_tokens", C.c_uint64), ("vocab", C.c_uint32)]
+                ("n_tokens", C.c_uint64), ("vocab", C.c_uint32), ("keys", C.c_void_p)]
 
 
 class fc_retrieve_params(C.Structure):
@@ -51,7 +51,7 @@ class fc_cache(C.Structure):
 
 
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
-           "fc_datastore_build_noalloc", "fc_datastore_save", "fc_datastore_file_info", "fc_datastore_load",
+           "fc_datastore_build_noalloc", "fc_datastore_keys", "fc_datastore_save", "fc_datastore_file_info", "fc_datastore_load",
            "fc_retrieve", "fc_retrieve_all", "fc_retrieve_rev", "fc_reverse_tokens", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
            "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_embed",
@@ -59,7 +59,8 @@ EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build
 
 
 def _load():
-    path = _build.LIB
+    # FC_DEBUG=1 loads the bounds-checking debug build (build(debug=True))
+    path = _build.LIB_DEBUG if os.environ.get("FC_DEBUG", "0") not in ("", "0") else _build.LIB
     if not os.path.exists(path):
         raise ImportError(f"libfastcoder.so is not built ({path}); run __graft_entry__.build()")
     lib = C.CDLL(path)
@@ -71,6 +72,7 @@ def _load():
         "fc_datastore_build_workspace": (sz, [u64, u32]),
         "fc_datastore_build": (C.c_int, [vp, u64, u32, vp, vp, vp, vp, sz, vp, C.POINTER(fc_datastore)]),
         "fc_datastore_build_noalloc": (C.c_int, [vp, u64, u32, vp, vp, vp, vp, C.POINTER(fc_datastore)]),
+        "fc_datastore_keys": (C.c_int, [C.POINTER(fc_datastore), vp, vp]),
         "fc_datastore_save": (C.c_int, [C.c_char_p, C.POINTER(fc_datastore), i32, vp]),
         "fc_datastore_file_info": (C.c_int, [C.c_char_p, C.POINTER(C.c_uint64), C.POINTER(C.c_uint32)]),
         "fc_datastore_load": (C.c_int, [C.c_char_p, vp, vp, vp, vp, u64, u32, i32, vp, C.POINTER(fc_datastore)]),
@@ -175,24 +177,41 @@ def fc_get_error(stream=None) -> str:
 # --------------------------------------------------------------- datastore
 class Datastore:
     """A built datastore: the token corpus, its suffix array, bucket table and
-    LCP array (device tensors owned here), plus the C view struct."""
+    LCP array (device tensors owned here), optionally its suffix keys
+    (fc_datastore_keys), plus the C view struct."""
 
-    def __init__(self, tokens, sa, bucket, lcp, vocab):
+    def __init__(self, tokens, sa, bucket, lcp, vocab, keys=None):
         self.tokens, self.sa, self.bucket, self.lcp, self.vocab = tokens, sa, bucket, lcp, int(vocab)
+        self.keys = keys
         self.view = fc_datastore(tokens.data_ptr(), sa.data_ptr(), bucket.data_ptr(), lcp.data_ptr(),
-                                 tokens.numel(), int(vocab))
+                                 tokens.numel(), int(vocab), None if keys is None else keys.data_ptr())
 
     @property
     def n_tokens(self):
         return self.tokens.numel()
+
+    def without_keys(self):
+        """The same store viewed without its suffix keys (the search then reads
+        the suffix array and the corpus)."""
+        return Datastore(self.tokens, self.sa, self.bucket, self.lcp, self.vocab)
+
+
+def fc_datastore_keys(ds: Datastore) -> Datastore:
+    """Builds the suffix keys of a datastore (32 bytes per token) and returns
+    the store with them in its view."""
+    keys = torch.empty((ds.n_tokens, 8), dtype=torch.int32, device=ds.tokens.device)
+    _check("fc_datastore_keys", LIB.fc_datastore_keys(C.byref(ds.view), _ptr(keys), _stream()))
+    return Datastore(ds.tokens, ds.sa, ds.bucket, ds.lcp, ds.vocab, keys)
 
 
 def fc_datastore_build_workspace(n_tokens: int, vocab: int) -> int:
     return int(LIB.fc_datastore_build_workspace(n_tokens, vocab))
 
 
-def fc_datastore_build(tokens: torch.Tensor, vocab: int, workspace: torch.Tensor | None = None) -> Datastore:
-    """tokens: int32 [N] on the GPU (uint32 ids < vocab).  Synchronous."""
+def fc_datastore_build(tokens: torch.Tensor, vocab: int, workspace: torch.Tensor | None = None,
+                       keys: bool = True) -> Datastore:
+    """tokens: int32 [N] on the GPU (uint32 ids < vocab).  Synchronous.  With
+    ``keys`` the suffix keys are built too (fc_datastore_keys)."""
     _need(tokens, torch.int32, "tokens")
     n = tokens.numel()
     sa = torch.empty(n, dtype=torch.int32, device=tokens.device)
@@ -204,7 +223,8 @@ def fc_datastore_build(tokens: torch.Tensor, vocab: int, workspace: torch.Tensor
         raise ValueError("workspace too small")
     _check("fc_datastore_build", LIB.fc_datastore_build(_ptr(tokens), n, vocab, _ptr(sa), _ptr(bucket), _ptr(lcp),
                                                         _ptr(ws), ws.numel(), _stream(), None))
-    return Datastore(tokens, sa, bucket, lcp, vocab)
+    ds = Datastore(tokens, sa, bucket, lcp, vocab)
+    return fc_datastore_keys(ds) if keys else ds
 
 
 def _np_ptr(a):
@@ -232,7 +252,7 @@ def fc_datastore_load(path: str, device="cuda") -> Datastore:
     lcp = torch.empty(n, dtype=torch.uint8, device=device)
     _check("fc_datastore_load", LIB.fc_datastore_load(os.fsencode(path), _ptr(tokens), _ptr(sa), _ptr(bucket),
                                                       _ptr(lcp), n, vocab, 0, _stream(), None))
-    return Datastore(tokens, sa, bucket, lcp, vocab)
+    return fc_datastore_keys(Datastore(tokens, sa, bucket, lcp, vocab))
 
 
 def datastore_save_host(path: str, tokens, sa, bucket, lcp) -> None:
@@ -341,8 +361,9 @@ def fc_reverse_tokens(tokens: torch.Tensor, out: torch.Tensor | None = None) -> 
 
 
 def fc_datastore_build_reversed(tokens: torch.Tensor, vocab: int) -> Datastore:
-    """The datastore of the reversed corpus, for fc_retrieve_rev."""
-    return fc_datastore_build(fc_reverse_tokens(tokens), vocab)
+    """The datastore of the reversed corpus, for fc_retrieve_rev (its narrowing
+    search reads the reversed suffix array directly; no suffix keys)."""
+    return fc_datastore_build(fc_reverse_tokens(tokens), vocab, keys=False)
 
 
 def fc_retrieve_rev(sources, rev_sources, ctx, ctx_len, p: fc_retrieve_params, skip=None, out=None):

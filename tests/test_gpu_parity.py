@@ -114,8 +114,13 @@ def test_retrieve_c1(fc, orc, c1):
     check_no_error(fc)
 
 
+@pytest.mark.parametrize("keys", [True, False])
 @pytest.mark.parametrize("seed", range(8))
-def test_retrieve_tiny_sweep(fc, orc, seed):
+def test_retrieve_tiny_sweep(fc, orc, seed, keys):
+    """Tiny alphabets (2-6 tokens), so probes tie on their first eight tokens
+    and the search reads the corpus; contexts copied from anywhere in the
+    corpus, the end included; n_max up to 32.  With the suffix keys (one
+    32-byte read per probe) and without them (suffix array, then corpus)."""
     rng = np.random.default_rng(500 + seed)
     N = int(rng.integers(2, 3000))
     vocab = int(rng.integers(2, 7))
@@ -133,10 +138,24 @@ def test_retrieve_tiny_sweep(fc, orc, seed):
     k, d = int(rng.integers(1, 257)), int(rng.integers(1, 17))
     max_occ = [1, 3, 4096, 17][seed % 4]
     ds = fc.fc_datastore_build(dev(T), vocab)
-    g = fc.fc_retrieve([ds], dev(ctx), dev(cl), fc.params(n_max, n_min, k, d, max_occ))
+    assert ds.keys is not None
+    g = fc.fc_retrieve([ds if keys else ds.without_keys()], dev(ctx), dev(cl), fc.params(n_max, n_min, k, d, max_occ))
     r = orc.retrieve(T, ctx, cl, n_max, n_min, k, d, max_occ)
     compare_retrieval(g, r)
     check_no_error(fc)
+
+
+def test_suffix_keys_layout(fc):
+    """Entry j of the suffix keys: sa[j], then the suffix's tokens 1..7
+    (FC_PAD_TOKEN past the corpus end)."""
+    rng = np.random.default_rng(31)
+    T = rng.integers(0, 5, 3001).astype(np.uint32)
+    ds = fc.fc_datastore_build(dev(T), 5)
+    sa = host_u32(ds.sa)
+    keys = host_u32(ds.keys).reshape(-1, 8)
+    Tp = np.concatenate([T, np.full(8, PAD, np.uint32)])
+    want = np.stack([sa] + [Tp[sa.astype(np.int64) + k] for k in range(1, 8)], 1)
+    assert np.array_equal(keys, want)
 
 
 def test_retrieve_two_sources_and_skip(fc, orc):
