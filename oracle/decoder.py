@@ -50,6 +50,16 @@ def widen(b16):
     return (b16.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
 
 
+def round_bf16(x):
+    """Nearest bf16 value (ties to even) of each element, as float64.  Used
+    only by forward(..., store_bf16=True)."""
+    f = np.ascontiguousarray(x, np.float64).astype(np.float32)
+    u = f.view(np.uint32).astype(np.uint64)
+    lsb = (u >> 16) & 1
+    r = ((u + 0x7FFF + lsb) >> 16) << 16
+    return r.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
 def rmsnorm(x, w, eps):
     return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps) * w
 
@@ -92,12 +102,20 @@ def ancestors_of(parent, n):
     return res
 
 
-def forward(cfg, W, tokens, parent, n_nodes, kv_len, k_caches, v_caches, pos):
+def forward(cfg, W, tokens, parent, n_nodes, kv_len, k_caches, v_caches, pos, store_bf16=False):
     """The tree forward for a batch.  W: dict of float64 weights (widened),
     with W["layers"][l] a dict per layer.  tokens/parent/pos [B][n_pad];
     k_caches/v_caches [L][B][Hkv][cap][D] (float64, keys rotated).  Returns
     (logits [B][n_pad][vocab] with padding rows zero, k_new [L][B][n_pad][Hkv][D]
-    rotated tree keys, v_new [L][B][n_pad][Hkv][D])."""
+    rotated tree keys, v_new [L][B][n_pad][Hkv][D]).
+
+    store_bf16: round every intermediate to bf16 where a bf16 forward stores
+    it (the residual stream after each add, each norm's output, the
+    projections, the rotated keys, the attention output, the MLP activation
+    and the logits), fp64 otherwise.  The paper states no precision; this
+    variant measures how far bf16 storage alone moves the result, which sizes
+    the tolerance of a bf16 forward against the fp64 one."""
+    rb = round_bf16 if store_bf16 else (lambda a: a)
     B, n_pad = tokens.shape
     logits = np.zeros((B, n_pad, cfg.vocab))
     k_new = np.zeros((cfg.layers, B, n_pad, cfg.Hkv, cfg.D))
@@ -110,18 +128,18 @@ def forward(cfg, W, tokens, parent, n_nodes, kv_len, k_caches, v_caches, pos):
         ok = ids < cfg.vocab
         x[ok] = W["embed"][ids[ok]]
         for l, Lw in enumerate(W["layers"]):
-            h = rmsnorm(x, Lw["attn_norm"], cfg.eps)
-            q = (h @ Lw["wq"]).reshape(n, cfg.H, cfg.D)
-            kv = (h @ Lw["wkv"]).reshape(n, 2, cfg.Hkv, cfg.D)
+            h = rb(rmsnorm(x, Lw["attn_norm"], cfg.eps))
+            q = rb(h @ Lw["wq"]).reshape(n, cfg.H, cfg.D)
+            kv = rb(h @ Lw["wkv"]).reshape(n, 2, cfg.Hkv, cfg.D)
             k, v = kv[:, 0], kv[:, 1]
-            k_new[l, b, :n] = O.rope(k, np.repeat(pos[b, :n, None], cfg.Hkv, 1), cfg.rope_base)
+            k_new[l, b, :n] = rb(O.rope(k, np.repeat(pos[b, :n, None], cfg.Hkv, 1), cfg.rope_base))
             v_new[l, b, :n] = v
-            a = tree_attention(q, k_caches[l][b], v_caches[l][b], int(kv_len[b]), k, v, anc, n, pos[b], cfg)
-            x = x + a.reshape(n, cfg.H * cfg.D) @ Lw["wo"]
-            h = rmsnorm(x, Lw["mlp_norm"], cfg.eps)
-            gu = h @ Lw["wgu"]
-            x = x + (silu(gu[:, :cfg.inter]) * gu[:, cfg.inter:]) @ Lw["wd"]
-        logits[b, :n] = rmsnorm(x, W["final_norm"], cfg.eps) @ W["lm_head"]
+            a = rb(tree_attention(q, k_caches[l][b], v_caches[l][b], int(kv_len[b]), k, v, anc, n, pos[b], cfg))
+            x = rb(x + rb(a.reshape(n, cfg.H * cfg.D) @ Lw["wo"]))
+            h = rb(rmsnorm(x, Lw["mlp_norm"], cfg.eps))
+            gu = rb(h @ Lw["wgu"])
+            x = rb(x + rb(rb(silu(gu[:, :cfg.inter]) * gu[:, cfg.inter:]) @ Lw["wd"]))
+        logits[b, :n] = rb(rb(rmsnorm(x, W["final_norm"], cfg.eps)) @ W["lm_head"])
     return logits, k_new, v_new
 
 

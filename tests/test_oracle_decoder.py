@@ -159,3 +159,41 @@ def test_numpy_attention_matches_the_c_oracle(dec, orc):
         got = dec.tree_attention(w(q[b]), w(kc[b]), w(vc[b]), int(kvl[b]), w(kt[b]).transpose(1, 0, 2),
                                  w(vt[b]).transpose(1, 0, 2), dec.ancestors_of(par[b], n), n, m["pos"][b], cfg)
         assert np.allclose(got, ref[b, :n], atol=1e-10)
+
+
+def test_round_bf16_matches_the_format(dec):
+    """round_bf16 (used only for the bf16-storage variant of the forward) is
+    round-to-nearest-even onto the bf16 grid: checked against torch's own
+    conversion, and on hand values at and between grid points."""
+    import torch
+    rng = np.random.default_rng(3)
+    x = np.concatenate([rng.standard_normal(20000) * 10.0 ** rng.integers(-30, 30, 20000),
+                        [0.0, -0.0, 1.0, 1 + 2.0 ** -8, 1 + 3 * 2.0 ** -9, 1 + 2.0 ** -9, 3.0e38]])
+    x = x.astype(np.float32).astype(np.float64)  # fp32 inputs: one rounding, as the GPU stores
+    want = torch.from_numpy(x).float().to(torch.bfloat16).double().numpy()
+    assert np.array_equal(dec.round_bf16(x), want)
+    assert dec.round_bf16(np.array([1 + 2.0 ** -8]))[0] == 1.0          # a tie goes to the even neighbour
+    assert dec.round_bf16(np.array([1 + 3 * 2.0 ** -8]))[0] == 1 + 2.0 ** -6
+
+
+def test_store_bf16_forward_stays_near_the_exact_one(dec, orc):
+    """The bf16-storage variant differs from the exact forward by rounding
+    only: a few bf16 ulps of the logits' scale, never zero, never more."""
+    cfg, W, kc, vc, kvl = setup(dec, 21, B=2)
+    B, n_pad = 2, 64
+    rng = synth.rng_for(91)
+    tok = np.full((B, n_pad), 0xFFFFFFFF, np.uint32)
+    par = np.full((B, n_pad), -1, np.int32)
+    nn = np.array([20, 7], np.int32)
+    pos = np.full((B, n_pad), -1, np.int32)
+    for b in range(B):
+        t, p = synth.random_tree(rng, int(nn[b]), 5, 3, cfg.vocab)
+        tok[b, :nn[b]], par[b, :nn[b]] = t, p
+        depth = np.zeros(nn[b], np.int32)
+        for i in range(1, nn[b]):
+            depth[i] = depth[p[i]] + 1
+        pos[b, :nn[b]] = kvl[b] + depth
+    ref = dec.forward(cfg, W, tok, par, nn, kvl, kc, vc, pos)[0]
+    mir = dec.forward(cfg, W, tok, par, nn, kvl, kc, vc, pos, store_bf16=True)[0]
+    d = np.abs(mir - ref).max()
+    assert 0 < d <= 0.05 * np.abs(ref).max()
