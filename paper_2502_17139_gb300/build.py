@@ -3,6 +3,11 @@
 Each .cu under csrc/ compiles in parallel to an object file; the objects link
 into one shared library against the shared CUDA runtime (the same runtime
 PyTorch uses).  Nothing is installed outside the package directory.
+
+build(debug=True) makes libfastcoder_debug.so in _build_debug/: the same
+sources with -DFC_DEBUG, whose kernels bounds-check the indexes their
+gathers take from data and report a bad one as FC_ERR_INTERNAL.  The binding
+loads it instead of the release library when FC_DEBUG=1 is set.
 """
 from __future__ import annotations
 
@@ -16,6 +21,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libfastcoder.so")
+BUILD_DEBUG = os.path.join(HERE, "_build_debug")
+LIB_DEBUG = os.path.join(BUILD_DEBUG, "libfastcoder_debug.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -43,10 +50,13 @@ def _stale(obj, src):
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    os.makedirs(BUILD, exist_ok=True)
+def build(force: bool = False, verbose: bool = False, extra_flags=(), debug: bool = False) -> str:
+    out_dir, lib = (BUILD_DEBUG, LIB_DEBUG) if debug else (BUILD, LIB)
+    if debug:
+        extra_flags = list(extra_flags) + ["-DFC_DEBUG"]
+    os.makedirs(out_dir, exist_ok=True)
     srcs = sources()
-    objs = [os.path.join(BUILD, os.path.basename(s)[:-3] + ".o") for s in srcs]
+    objs = [os.path.join(out_dir, os.path.basename(s)[:-3] + ".o") for s in srcs]
     todo = [(s, o) for s, o in zip(srcs, objs) if force or _stale(o, s)]
     cc = nvcc()
 
@@ -63,16 +73,16 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
             for msg in ex.map(compile_one, todo):
                 if verbose and msg:
                     print(msg)
-    if todo or not os.path.exists(LIB):
-        tmp = LIB + f".tmp{os.getpid()}"
+    if todo or not os.path.exists(lib):
+        tmp = lib + f".tmp{os.getpid()}"
         cmd = [cc] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + objs
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stderr}")
-        os.replace(tmp, LIB)
-    return LIB
+        os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":
     import sys
-    print(build(force="--force" in sys.argv, verbose=True))
+    print(build(force="--force" in sys.argv, verbose=True, debug="--debug" in sys.argv))

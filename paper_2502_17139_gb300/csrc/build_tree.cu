@@ -784,6 +784,7 @@ extern "C" fc_status fc_build_tree(int n_sources, const uint32_t* d_drafts, cons
                                    int batch, int node_budget, int n_pad, uint32_t* d_tok, int32_t* d_parent,
                                    int32_t* d_depth, int32_t* d_pos, uint64_t* d_mask, int32_t* d_n_nodes,
                                    fc_stream stream) {
+  FC_NVTX_RANGE();
   if (n_sources < 1 || n_sources > FC_MAX_SOURCES || top_k < 1 || draft_len < 1 || batch < 0 || !src_weight)
     return FC_ERR_INVALID_ARG;
   if (n_pad != 64 && n_pad != 128) return FC_ERR_UNSUPPORTED;
@@ -810,6 +811,7 @@ extern "C" fc_status fc_build_tree(int n_sources, const uint32_t* d_drafts, cons
 extern "C" fc_status fc_tree_mask(const int32_t* d_parent, const int32_t* d_n_nodes, const int32_t* d_kv_len,
                                   int batch, int n_pad, int32_t* d_depth, int32_t* d_pos, uint64_t* d_mask,
                                   fc_stream stream) {
+  FC_NVTX_RANGE();
   if (batch < 0) return FC_ERR_INVALID_ARG;
   if (n_pad != 64 && n_pad != 128) return FC_ERR_UNSUPPORTED;
   if (batch == 0) return FC_OK;
@@ -839,6 +841,7 @@ extern "C" fc_status fc_build_tree_all(int n_sources, const uint32_t* d_drafts, 
                                        int node_budget, int n_pad, void* d_ws, size_t ws_bytes, uint32_t* d_tok,
                                        int32_t* d_parent, int32_t* d_depth, int32_t* d_pos, uint64_t* d_mask,
                                        int32_t* d_n_nodes, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (n_sources < 1 || n_sources > FC_MAX_SOURCES || slots < 1 || draft_len < 1 || batch < 0 || !src_weight)
     return FC_ERR_INVALID_ARG;
   if (n_pad != 64 && n_pad != 128) return FC_ERR_UNSUPPORTED;

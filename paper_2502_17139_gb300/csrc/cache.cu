@@ -743,6 +743,7 @@ CacheView view_of(const fc_cache* c) {
 }  // namespace
 
 extern "C" fc_status fc_cache_init(const fc_cache* cache, int batch, const int32_t* d_prompt_len, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (!cache_ok(cache) || batch < 0) return FC_ERR_INVALID_ARG;
   if (batch == 0) return FC_OK;
   if (!d_prompt_len) return FC_ERR_INVALID_ARG;
@@ -757,6 +758,7 @@ extern "C" size_t fc_missing_bytes(int capacity, int key_len) {
 }
 
 extern "C" fc_status fc_missing_init(void* d_table, size_t bytes, int capacity, int key_len, fc_stream stream) {
+  FC_NVTX_RANGE();
   const size_t need = fc_missing_bytes(capacity, key_len);
   if (!d_table || need == 0) return FC_ERR_INVALID_ARG;
   if (bytes < need) return FC_ERR_WORKSPACE;
@@ -768,6 +770,7 @@ extern "C" fc_status fc_cache_search(const fc_cache* cache, const void* d_missin
                                      fc_retrieve_params p, int n_sources, uint32_t* d_drafts, int32_t* d_draft_len,
                                      uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len, int32_t* d_state,
                                      fc_stream stream) {
+  FC_NVTX_RANGE();
   if (!cache_ok(cache) || batch < 0 || ctx_stride < 1 || n_sources < 0 || n_sources >= FC_MAX_SOURCES ||
       batch > 65535 * 16)
     return FC_ERR_INVALID_ARG;
@@ -802,6 +805,7 @@ extern "C" fc_status fc_cache_search(const fc_cache* cache, const void* d_missin
 extern "C" fc_status fc_missing_insert(void* d_missing, int missing_capacity, int key_len, const uint32_t* d_ctx,
                                        int ctx_stride, const int32_t* d_ctx_len, int batch, const int32_t* d_state,
                                        const int32_t* d_n_drafts, int n_sources, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (!d_missing || !missing_cap_ok(missing_capacity) || key_len < 1 || key_len > FC_MAX_NMAX || batch < 0 ||
       ctx_stride < 1 || n_sources < 0 || n_sources > FC_MAX_SOURCES)
     return FC_ERR_INVALID_ARG;
@@ -816,6 +820,7 @@ extern "C" fc_status fc_missing_insert(void* d_missing, int missing_capacity, in
 extern "C" fc_status fc_cache_update(const fc_cache* cache, const uint32_t* d_ctx, int ctx_stride,
                                      const int32_t* d_ctx_len_old, const int32_t* d_ctx_len_new,
                                      const int32_t* d_acc_len, int batch, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (!cache_ok(cache) || batch < 0 || ctx_stride < 1) return FC_ERR_INVALID_ARG;
   if (batch == 0) return FC_OK;
   if (!d_ctx || !d_ctx_len_old || !d_ctx_len_new || !d_acc_len) return FC_ERR_INVALID_ARG;

@@ -178,6 +178,7 @@ bool aligned16(const void* p) { return reinterpret_cast<uintptr_t>(p) % 16 == 0;
 
 extern "C" fc_status fc_embed(const uint32_t* d_tok, int n, const void* d_table, int vocab, int hidden, void* d_out,
                               fc_stream stream) {
+  FC_NVTX_RANGE();
   if (n < 0 || vocab < 1 || hidden < 8 || hidden % 8) return FC_ERR_INVALID_ARG;
   if (n == 0) return FC_OK;
   if (!d_tok || !d_table || !d_out || !aligned16(d_table) || !aligned16(d_out)) return FC_ERR_INVALID_ARG;
@@ -188,6 +189,7 @@ extern "C" fc_status fc_embed(const uint32_t* d_tok, int n, const void* d_table,
 
 extern "C" fc_status fc_add_rmsnorm(void* d_x, const void* d_r, const void* d_w, void* d_out, int rows, int dim,
                                     float eps, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (rows < 0 || dim < 8 || dim % 8 || !(eps >= 0.f)) return FC_ERR_INVALID_ARG;
   if (rows == 0) return FC_OK;
   if (!d_x || !d_w || !d_out || !aligned16(d_x) || !aligned16(d_w) || !aligned16(d_out) || (d_r && !aligned16(d_r)))
@@ -200,6 +202,7 @@ extern "C" fc_status fc_add_rmsnorm(void* d_x, const void* d_r, const void* d_w,
 }
 
 extern "C" fc_status fc_silu_mul(const void* d_gu, void* d_out, int rows, int inter, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (rows < 0 || inter < 8 || inter % 8) return FC_ERR_INVALID_ARG;
   if (rows == 0) return FC_OK;
   if (!d_gu || !d_out || !aligned16(d_gu) || !aligned16(d_out)) return FC_ERR_INVALID_ARG;
@@ -212,6 +215,7 @@ extern "C" fc_status fc_silu_mul(const void* d_gu, void* d_out, int rows, int in
 
 extern "C" fc_status fc_rope_heads(const void* d_in, int in_stride, void* d_out, int batch, int n_pad, int heads, int D,
                                    const int32_t* d_pos, float base, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (batch < 0 || n_pad < 1 || heads < 1 || D < 16 || D > 1024 || D % 16 || in_stride < heads * D ||
       in_stride % 8)
     return FC_ERR_INVALID_ARG;

@@ -28,6 +28,7 @@ extern "C" const char* fc_status_string(fc_status s) {
 extern "C" const char* fc_version(void) { return "0.1.0"; }
 
 extern "C" fc_status fc_get_error(fc_stream stream) {
+  FC_NVTX_RANGE();
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (cudaStreamSynchronize(s) != cudaSuccess) return FC_ERR_CUDA;
   unsigned int e = fc_take_error_sa(s) | fc_take_error_ret(s) | fc_take_error_tree(s) | fc_take_error_step(s) |

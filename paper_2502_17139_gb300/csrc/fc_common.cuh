@@ -7,7 +7,20 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/fastcoder.h"
+
+// One NVTX range per C-ABI call, named after the call: a profiler's timeline
+// then shows which entry point enqueued which kernels.  With no tool
+// attached the push and pop are calls into empty functions.
+struct FcNvtxRange {
+  explicit FcNvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~FcNvtxRange() { nvtxRangePop(); }
+  FcNvtxRange(const FcNvtxRange&) = delete;
+  FcNvtxRange& operator=(const FcNvtxRange&) = delete;
+};
+#define FC_NVTX_RANGE() FcNvtxRange fc_nvtx_range_(__func__)
 
 // ---------------------------------------------------------------------------
 // Device error word.  Kernels OR one of these bits in; fc_get_error() reads
@@ -32,6 +45,21 @@
   }
 
 __device__ __forceinline__ void fc_flag(unsigned int* word, unsigned int bit) { atomicOr(word, bit); }
+
+// Debug builds (compiled with -DFC_DEBUG into libfastcoder_debug.so) check
+// the indexes that gathers take from data, such as suffix-array entries,
+// before using them: an index out of range sets FC_ERR_INTERNAL in the
+// translation unit's error word and the access is skipped.  Release builds
+// trust the datastores and trees they are given (this library builds both).
+__device__ __forceinline__ bool fc_debug_ok(bool ok, unsigned int* word) {
+  if (!ok) fc_flag(word, FC_EBIT_INTERNAL);
+  return ok;
+}
+#ifdef FC_DEBUG
+#define FC_DEBUG_CHECK(ok) fc_debug_ok((ok), &g_fc_err)
+#else
+#define FC_DEBUG_CHECK(ok) true
+#endif
 
 // Host: map a CUDA launch result to a status.
 static inline fc_status fc_cuda_status(cudaError_t e) { return e == cudaSuccess ? FC_OK : FC_ERR_CUDA; }

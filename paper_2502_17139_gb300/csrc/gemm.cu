@@ -240,6 +240,7 @@ extern "C" size_t fc_gemm_workspace(void) { return 0; }
 
 extern "C" fc_status fc_gemm_bf16(const void* d_a, const void* d_b, void* d_c, int M, int N, int K, void* d_ws,
                                   size_t ws_bytes, fc_stream stream) {
+  FC_NVTX_RANGE();
   (void)d_ws;
   (void)ws_bytes;
   if (M < 0 || N < 1 || K < 1) return FC_ERR_INVALID_ARG;

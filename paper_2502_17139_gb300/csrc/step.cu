@@ -291,6 +291,7 @@ __global__ void k_synth_argmax(const uint32_t* __restrict__ tok, const int32_t* 
 extern "C" fc_status fc_accept(const uint32_t* d_tok, const int32_t* d_parent, const int32_t* d_n_nodes,
                                const uint32_t* d_argmax, int batch, int n_pad, int32_t* d_acc_len, int32_t* d_path,
                                int path_cap, uint32_t* d_bonus, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (batch < 0 || n_pad < 1 || n_pad > 1024 || path_cap < 1) return FC_ERR_INVALID_ARG;
   if (batch == 0) return FC_OK;
   if (!d_tok || !d_parent || !d_n_nodes || !d_argmax || !d_acc_len || !d_path || !d_bonus) return FC_ERR_INVALID_ARG;
@@ -305,6 +306,7 @@ extern "C" fc_status fc_argmax_accept(const void* d_logits, int vocab, const uin
                                       const int32_t* d_parent, const int32_t* d_n_nodes, int batch, int n_pad,
                                       uint32_t* d_argmax, int32_t* d_acc_len, int32_t* d_path, int path_cap,
                                       uint32_t* d_bonus, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (batch < 0 || n_pad < 1 || n_pad > 1024 || path_cap < 1 || vocab < 1) return FC_ERR_INVALID_ARG;
   if (batch > 65535) return FC_ERR_UNSUPPORTED;
   if (batch == 0) return FC_OK;
@@ -340,6 +342,7 @@ extern "C" fc_status fc_kv_append(const int32_t* d_path, const int32_t* d_acc_le
                                   const int32_t* d_kv_len_in, int32_t* d_kv_len_out, uint32_t* d_ctx, int ctx_stride,
                                   const int32_t* d_ctx_len_in, int32_t* d_ctx_len_out, uint32_t* d_root_out,
                                   fc_stream stream) {
+  FC_NVTX_RANGE();
   if (batch < 0 || n_pad < 1 || Hkv < 1 || D < 8 || D % 8 || path_cap < 1 || kv_cap < 1 || ctx_stride < 1)
     return FC_ERR_INVALID_ARG;
   if (batch == 0) return FC_OK;
@@ -360,6 +363,7 @@ extern "C" fc_status fc_kv_append(const int32_t* d_path, const int32_t* d_acc_le
 extern "C" fc_status fc_synth_argmax(const uint32_t* d_tok, const int32_t* d_parent, const int32_t* d_n_nodes,
                                      int batch, int n_pad, const int32_t* d_plen, const uint32_t* d_rtok,
                                      uint32_t vocab, uint32_t* d_argmax, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (batch < 0 || n_pad < 1 || n_pad > FC_MAX_NODES || vocab < 2) return FC_ERR_INVALID_ARG;
   if (batch == 0) return FC_OK;
   if (!d_tok || !d_parent || !d_n_nodes || !d_plen || !d_rtok || !d_argmax) return FC_ERR_INVALID_ARG;
@@ -395,6 +399,7 @@ __global__ void k_selftest_wait(int arrive, unsigned long long limit_cycles) {
 }  // namespace
 
 extern "C" fc_status fc_selftest_wait(int arrive, unsigned long long limit_cycles, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (limit_cycles == 0 || limit_cycles > 4000000000ull) return FC_ERR_INVALID_ARG;
   k_selftest_wait<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(arrive, limit_cycles);
   return FC_CHECK_LAUNCH();

@@ -920,6 +920,7 @@ extern "C" fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const 
                                   const int32_t* d_kv_len, const void* d_k_tree, const void* d_v_tree,
                                   const uint64_t* d_mask, const int32_t* d_n_nodes, int batch, int n_pad, int H, int Hkv,
                                   int D, float scale, void* d_out, void* d_ws, size_t ws_bytes, fc_stream stream) {
+  FC_NVTX_RANGE();
   return launch_tree_attn(d_q, d_k_cache, d_v_cache, kv_cap, d_kv_len, d_k_tree, d_v_tree, d_mask, d_n_nodes, batch,
                           n_pad, H, Hkv, D, scale, d_out, d_ws, ws_bytes, nullptr, 0.f, stream);
 }
@@ -929,6 +930,7 @@ extern "C" fc_status fc_tree_attn_rope(const void* d_q, const void* d_k_cache, c
                                        const uint64_t* d_mask, const int32_t* d_n_nodes, int batch, int n_pad, int H,
                                        int Hkv, int D, float scale, const int32_t* d_pos, float rope_base,
                                        void* d_out, void* d_ws, size_t ws_bytes, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (!(rope_base > 0.f) || !std::isfinite(rope_base)) return FC_ERR_INVALID_ARG;
   if (batch > 0 && !d_pos) return FC_ERR_INVALID_ARG;
   return launch_tree_attn(d_q, d_k_cache, d_v_cache, kv_cap, d_kv_len, d_k_tree, d_v_tree, d_mask, d_n_nodes, batch,
@@ -937,6 +939,7 @@ extern "C" fc_status fc_tree_attn_rope(const void* d_q, const void* d_k_cache, c
 
 extern "C" fc_status fc_rope(const void* d_in, void* d_out, int batch, int n_pad, int heads, int D, int layout,
                              const int32_t* d_pos, float base, fc_stream stream) {
+  FC_NVTX_RANGE();
   if (batch < 0 || n_pad < 1 || heads < 1 || D < 16 || D > 1024 || D % 16 || (layout != 0 && layout != 1))
     return FC_ERR_INVALID_ARG;
   if (!(base > 0.f) || !std::isfinite(base)) return FC_ERR_INVALID_ARG;

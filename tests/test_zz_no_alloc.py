@@ -127,5 +127,6 @@ def test_noalloc_first_call_in_fresh_process(fc):
     r = subprocess.run([sys.executable, "-c", _FIRST_CALL, root], capture_output=True, text=True, timeout=300)
     assert r.returncode == 0, r.stderr[-2000:]
     got = json.loads(r.stdout.strip().splitlines()[-1])
+    print("fc_datastore_build_noalloc in a fresh process:", got)
     assert got["second_call_bytes"] == 0
     assert 30 << 20 <= got["first_call_bytes"] <= 64 << 20, got
