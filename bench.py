@@ -1420,6 +1420,27 @@ def run_decoder(args, rank, ws, local):
     torch.cuda.synchronize()
     fwd_ms = f0.elapsed_time(f1)
     attn_ms = sum(a.elapsed_time(b) for a, b in aev["attn"])
+    # the same forward without per-layer events: host enqueue time, device time
+    # eager, and device time replayed from a CUDA graph (no launch gaps)
+    torch.cuda.synchronize()
+    h0 = time.perf_counter()
+    f0.record()
+    td.forward(t["tok"], t["n_nodes"], t["mask"], t["pos"], loop.kv_len_now)
+    f1.record()
+    host_ms = 1e3 * (time.perf_counter() - h0)
+    torch.cuda.synchronize()
+    eager_ms = f0.elapsed_time(f1)
+    g_fwd = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_fwd):
+        td.forward(t["tok"], t["n_nodes"], t["mask"], t["pos"], loop.kv_len_now)
+    g_fwd.replay()
+    torch.cuda.synchronize()
+    f0.record()
+    for _ in range(3):
+        g_fwd.replay()
+    f1.record()
+    torch.cuda.synchronize()
+    graph_ms = f0.elapsed_time(f1) / 3
     peaks = load_peaks()
     gemm_tflops = gemm_flops / ((fwd_ms - attn_ms) * 1e-3) / 1e12
     return {"metric": METRIC, "value": weak_value(K, ws, t_max), "unit": UNIT, "n_gpus": ws, "steps": K, "warmup": W,
@@ -1432,7 +1453,8 @@ def run_decoder(args, rank, ws, local):
             "stages_ms_per_step": stage,
             "tokens_per_s": float((acc + 1).sum() / (t_max * 1e-3) * ws),
             "mean_accepted": float(acc.mean()),
-            "forward": {"ms": fwd_ms, "attention_ms": attn_ms, "gemm_and_rest_ms": fwd_ms - attn_ms,
+            "forward": {"ms": fwd_ms, "eager_ms_no_events": eager_ms, "host_enqueue_ms": host_ms,
+                        "graph_replay_ms": graph_ms, "attention_ms": attn_ms, "gemm_and_rest_ms": fwd_ms - attn_ms,
                         "gemm_tflops": gemm_tflops, "gemm_frac_of_sustained_bf16": gemm_tflops / peaks["tc_sustained"]},
             "clocks": clock_rec}
 
@@ -1455,14 +1477,23 @@ def run_gemm(args, rank, ws, local):
     per_layer = {"q", "kv", "o", "gate_up", "down"}
     g = torch.Generator(device=dev)
     g.manual_seed(7)
-    rows, ours_t, lib_t, flops_t = [], 0.0, 0.0, 0.0
+    rows, ours_t, lib_t, flops_t, lt_t, lt_ok = [], 0.0, 0.0, 0.0, 0.0, True
     for name, K, N in shapes:
         a = torch.randn((M, K), generator=g, device=dev).to(torch.bfloat16)
         b = (torch.randn((K, N), generator=g, device=dev) * K ** -0.5).to(torch.bfloat16)
         c = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
         c_ref = torch.empty_like(c)
-        t_ours = _cuda_ms(lambda: fc.fc_gemm_bf16(a, b, out=c), reps=max(args.steps, 5), warm=max(args.warmup, 3))
-        t_lib = _cuda_ms(lambda: torch.matmul(a, b, out=c_ref), reps=max(args.steps, 5), warm=max(args.warmup, 3))
+        reps, warm = max(args.steps, 5), max(args.warmup, 3)
+        t_ours = _cuda_ms(lambda: fc.fc_gemm_bf16(a, b, out=c), reps=reps, warm=warm)
+        t_lib = _cuda_ms(lambda: torch.matmul(a, b, out=c_ref), reps=reps, warm=warm)
+        t_lt = None
+        try:  # the same product through cuBLASLt (torch's other BLAS back end)
+            prev = torch.backends.cuda.preferred_blas_library()
+            torch.backends.cuda.preferred_blas_library("cublaslt")
+            t_lt = _cuda_ms(lambda: torch.matmul(a, b, out=c_ref), reps=reps, warm=warm)
+            torch.backends.cuda.preferred_blas_library(prev)
+        except (AttributeError, RuntimeError, TypeError):
+            pass
         torch.cuda.synchronize()
         assert fc.fc_get_error() == "FC_OK"
         diff = float((c.float() - c_ref.float()).abs().max())
@@ -1470,16 +1501,52 @@ def run_gemm(args, rank, ws, local):
         w = 24 if name in per_layer else 1  # occurrences in one 24-layer forward
         ours_t += w * t_ours
         lib_t += w * t_lib
+        if t_lt is None:
+            lt_ok = False
+        else:
+            lt_t += w * t_lt
         flops_t += w * fl
         rows.append({"gemm": name, "M": M, "N": N, "K": K, "ours_us": 1e3 * t_ours, "cublas_us": 1e3 * t_lib,
+                     "cublaslt_us": None if t_lt is None else 1e3 * t_lt,
                      "ours_tflops": fl / t_ours / 1e9, "cublas_tflops": fl / t_lib / 1e9,
+                     "cublaslt_tflops": None if t_lt is None else fl / t_lt / 1e9,
                      "ours_frac_of_burst": fl / t_ours / 1e9 / peaks["tc_burst"], "max_abs_diff_vs_cublas": diff})
+    # the decoder's two fused epilogues against the unfused pair of calls
+    B, n_pad, Hkv, inter = 32, 64, 16, 5504
+    h = torch.randn((M, 2048), generator=g, device=dev).to(torch.bfloat16)
+    wkv = (torch.randn((2048, 2 * Hkv * 128), generator=g, device=dev) * 2048 ** -0.5).to(torch.bfloat16)
+    wgu = (torch.randn((2048, 2 * inter), generator=g, device=dev) * 2048 ** -0.5).to(torch.bfloat16)
+    wgu_il = fc.fc_interleave_gate_up(wgu)
+    pos = torch.arange(n_pad, device=dev, dtype=torch.int32).repeat(B, 1) + 2048
+    k_rot = torch.empty((B, Hkv, n_pad, 128), dtype=torch.bfloat16, device=dev)
+    v_h = torch.empty_like(k_rot)
+    kv = torch.empty((M, 2 * Hkv * 128), dtype=torch.bfloat16, device=dev)
+    gu = torch.empty((M, 2 * inter), dtype=torch.bfloat16, device=dev)
+    act = torch.empty((M, inter), dtype=torch.bfloat16, device=dev)
+
+    def unfused_kv():
+        fc.fc_gemm_bf16(h, wkv, out=kv)
+        fc.fc_rope_heads(kv, 0, 2 * Hkv * 128, k_rot, B, n_pad, Hkv, 128, pos, 10000.0)
+        fc.fc_rope_heads(kv, Hkv * 128, 2 * Hkv * 128, v_h, B, n_pad, Hkv, 128, pos, 0.0)
+
+    def unfused_gu():
+        fc.fc_gemm_bf16(h, wgu, out=gu)
+        fc.fc_silu_mul(gu, act)
+
+    fused = {"kv_heads_us": 1e3 * _cuda_ms(lambda: fc.fc_gemm_kv_heads(h, wkv, B, n_pad, Hkv, pos, 10000.0, k_rot, v_h)),
+             "kv_gemm_then_rope_heads_us": 1e3 * _cuda_ms(unfused_kv),
+             "silu_mul_us": 1e3 * _cuda_ms(lambda: fc.fc_gemm_silu_mul(h, wgu_il, act)),
+             "gu_gemm_then_silu_mul_us": 1e3 * _cuda_ms(unfused_gu)}
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_OK"
     ach = flops_t / ours_t / 1e9
     return {"metric": "decoder GEMM TFLOP/s", "value": ach, "unit": "TFLOP/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "dtype": "bf16 (fp32 accumulate)",
             "data": "synthetic", "config": {"workload": "decoder GEMMs of a 24-layer DeepSeek-Coder-1.3B-shaped "
                                                         "forward over 2048 tree rows, weighted by occurrences"},
             "cublas_tflops": flops_t / lib_t / 1e9, "ratio_to_cublas": lib_t / ours_t,
+            "cublaslt_tflops": flops_t / lt_t / 1e9 if lt_ok else None,
+            "ratio_to_cublaslt": lt_t / ours_t if lt_ok else None, "fused_epilogues": fused,
             "roofline": {"bound": "tensor", "achieved": ach, "peak": peaks["tc_burst"], "unit": "TFLOP/s",
                          "frac": ach / peaks["tc_burst"], "peak_source": peaks["source"] + " burst bf16"},
             "shapes": rows}

@@ -577,6 +577,30 @@ size_t fc_gemm_workspace(void);
 fc_status fc_gemm_bf16(const void* d_a, const void* d_b, void* d_c, int M, int N, int K, void* d_ws,
                        size_t ws_bytes, fc_stream s);
 
+/* The decoder's K/V projection with its next step folded into the GEMM's
+ * epilogue: kv = A[M][K] Wkv[K][2 Hkv D] (Hkv key heads, then Hkv value heads
+ * of D = 128 columns), rows (sequence b, node i) = b * n_pad + i, M = batch *
+ * n_pad.  From the fp32 accumulators the key heads are rotated by d_pos[b][i]
+ * (RoPE, rotate-half pairing, as fc_rope; a negative position leaves the row
+ * unrotated), and both are written head-major and rounded once to bf16:
+ * d_k_rot and d_v_heads [batch][Hkv][n_pad][D], the layout fc_tree_attn and
+ * fc_kv_append read.  D != 128 or K % 8 gives FC_ERR_UNSUPPORTED. */
+fc_status fc_gemm_kv_heads(const void* d_a, const void* d_wkv, int M, int K, int Hkv, int D, int batch, int n_pad,
+                           const int32_t* d_pos, float rope_base, void* d_k_rot, void* d_v_heads, fc_stream s);
+
+/* The gate/up projection with the SiLU-gated product folded into the GEMM's
+ * epilogue: act[M][inter] = silu(A Wg) * (A Wu), fp32 inside, rounded once
+ * to bf16.  d_wgu holds Wg and Wu interleaved in 128-column blocks, as
+ * fc_interleave_gate_up writes them.  inter % 128 or K % 8 gives
+ * FC_ERR_UNSUPPORTED. */
+fc_status fc_gemm_silu_mul(const void* d_a, const void* d_wgu, int M, int K, int inter, void* d_act, fc_stream s);
+
+/* Weight preparation for fc_gemm_silu_mul (once, at load): d_wgu [K][2 inter]
+ * (the gate columns, then the up columns) -> d_out [K][2 inter] with block t
+ * of 256 columns = gate columns 128t .. 128t+127, then up columns 128t ..
+ * 128t+127.  Buffers must not overlap. */
+fc_status fc_interleave_gate_up(const void* d_wgu, void* d_out, int K, int inter, fc_stream s);
+
 /* out[t][:] = table[tok[t]][:]; an id >= vocab (tree padding) gives zeros.
  * hidden a multiple of 8. */
 fc_status fc_embed(const uint32_t* d_tok, int n, const void* d_table, int vocab, int hidden, void* d_out,

@@ -110,9 +110,11 @@ def forward(cfg, W, tokens, parent, n_nodes, kv_len, k_caches, v_caches, pos, st
     rotated tree keys, v_new [L][B][n_pad][Hkv][D]).
 
     store_bf16: round every intermediate to bf16 where a bf16 forward stores
-    it (the residual stream after each add, each norm's output, the
-    projections, the rotated keys, the attention output, the MLP activation
-    and the logits), fp64 otherwise.  The paper states no precision; this
+    it (the residual stream after each add, each norm's output, the query,
+    output and down projections, the rotated keys and the values, the
+    attention output, the MLP activation and the logits), fp64 otherwise;
+    the key/value and gate/up projections are consumed unrounded by the
+    rotation and by SiLU * up.  The paper states no precision; this
     variant measures how far bf16 storage alone moves the result, which sizes
     the tolerance of a bf16 forward against the fp64 one."""
     rb = round_bf16 if store_bf16 else (lambda a: a)
@@ -130,14 +132,14 @@ def forward(cfg, W, tokens, parent, n_nodes, kv_len, k_caches, v_caches, pos, st
         for l, Lw in enumerate(W["layers"]):
             h = rb(rmsnorm(x, Lw["attn_norm"], cfg.eps))
             q = rb(h @ Lw["wq"]).reshape(n, cfg.H, cfg.D)
-            kv = rb(h @ Lw["wkv"]).reshape(n, 2, cfg.Hkv, cfg.D)
-            k, v = kv[:, 0], kv[:, 1]
+            kv = (h @ Lw["wkv"]).reshape(n, 2, cfg.Hkv, cfg.D)
+            k, v = kv[:, 0], rb(kv[:, 1])
             k_new[l, b, :n] = rb(O.rope(k, np.repeat(pos[b, :n, None], cfg.Hkv, 1), cfg.rope_base))
             v_new[l, b, :n] = v
             a = rb(tree_attention(q, k_caches[l][b], v_caches[l][b], int(kv_len[b]), k, v, anc, n, pos[b], cfg))
             x = rb(x + rb(a.reshape(n, cfg.H * cfg.D) @ Lw["wo"]))
             h = rb(rmsnorm(x, Lw["mlp_norm"], cfg.eps))
-            gu = rb(h @ Lw["wgu"])
+            gu = h @ Lw["wgu"]
             x = rb(x + rb(rb(silu(gu[:, :cfg.inter]) * gu[:, cfg.inter:]) @ Lw["wd"]))
         logits[b, :n] = rb(rb(rmsnorm(x, W["final_norm"], cfg.eps)) @ W["lm_head"])
     return logits, k_new, v_new

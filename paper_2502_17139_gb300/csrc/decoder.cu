@@ -5,7 +5,7 @@
 // (rotated) and values.  The GEMMs are gemm.cu's tcgen05 kernel.
 //
 //   * k_embed: one row per warp; ids >= vocab (tree padding) embed as zeros.
-//   * k_add_rmsnorm: one row per warp; x += r is rounded to bf16 (the
+//   * k_add_rmsnorm: one CTA per row; x += r is rounded to bf16 (the
 //     residual stream), then out = x / sqrt(mean(x^2) + eps) * w in fp32.
 //   * k_silu_mul: out = silu(gate) * up, fp32 math.
 //   * k_rope_heads: node-major projection rows -> head-major [B][heads][n][D],
@@ -45,15 +45,25 @@ __device__ __forceinline__ uint32_t f2bf(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&r);
 }
 
-__global__ void k_add_rmsnorm(uint4* __restrict__ x, const uint4* __restrict__ r, const uint4* __restrict__ w,
-                              uint4* __restrict__ out, int rows, int dim, float eps) {
-  const int row = blockIdx.x * ROWS_PER_BLOCK + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+// One CTA of NORM_THREADS per row; a thread holds up to NORM_CHUNKS 16-byte
+// chunks of the row in registers between the sum of squares and the scaling,
+// so the row is read once.  Rows wider than NORM_THREADS * NORM_CHUNKS chunks
+// reread the rest.
+constexpr int NORM_THREADS = 256, NORM_CHUNKS = 2;
+
+__global__ void __launch_bounds__(NORM_THREADS) k_add_rmsnorm(uint4* __restrict__ x, const uint4* __restrict__ r,
+                                                              const uint4* __restrict__ w, uint4* __restrict__ out,
+                                                              int rows, int dim, float eps) {
+  __shared__ float s_part[NORM_THREADS / 32];
+  const int row = blockIdx.x, tid = threadIdx.x, lane = tid & 31, wp = tid >> 5;
   if (row >= rows) return;
   const int cw = dim / 8;
   uint4* xr = x + (size_t)row * cw;
   const uint4* rr = r ? r + (size_t)row * cw : nullptr;
+  uint4 keep[NORM_CHUNKS];
   float ss = 0.f;
-  for (int c = lane; c < cw; c += 32) {
+  // x (+ r): rounded to bf16 and written back when r is given; sum of squares
+  auto load = [&](int c) {
     uint4 v = xr[c];
     if (rr) {  // the residual stream in bf16: x + r, rounded
       const uint4 a = rr[c];
@@ -72,13 +82,25 @@ __global__ void k_add_rmsnorm(uint4* __restrict__ x, const uint4* __restrict__ r
       const float2 f = bf2f(vv[q]);
       ss = fmaf(f.x, f.x, fmaf(f.y, f.y, ss));
     }
+    return v;
+  };
+#pragma unroll
+  for (int k = 0; k < NORM_CHUNKS; ++k) {
+    const int c = tid + k * NORM_THREADS;
+    if (c < cw) keep[k] = load(c);
   }
+  for (int c = tid + NORM_CHUNKS * NORM_THREADS; c < cw; c += NORM_THREADS) load(c);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
-  const float inv = rsqrtf(ss / (float)dim + eps);
+  if (lane == 0) s_part[wp] = ss;
+  __syncthreads();
+  float tot = 0.f;
+#pragma unroll
+  for (int i = 0; i < NORM_THREADS / 32; ++i) tot += s_part[i];
+  const float inv = rsqrtf(tot / (float)dim + eps);
   uint4* orow = out + (size_t)row * cw;
-  for (int c = lane; c < cw; c += 32) {
-    const uint4 v = xr[c], g = w[c];
+  auto store = [&](int c, const uint4& v) {
+    const uint4 g = w[c];
     const uint32_t* vv = &v.x;
     const uint32_t* gg = &g.x;
     uint4 res;
@@ -89,7 +111,13 @@ __global__ void k_add_rmsnorm(uint4* __restrict__ x, const uint4* __restrict__ r
       rv[q] = f2bf(f.x * inv * gw.x, f.y * inv * gw.y);
     }
     orow[c] = res;
+  };
+#pragma unroll
+  for (int k = 0; k < NORM_CHUNKS; ++k) {
+    const int c = tid + k * NORM_THREADS;
+    if (c < cw) store(c, keep[k]);
   }
+  for (int c = tid + NORM_CHUNKS * NORM_THREADS; c < cw; c += NORM_THREADS) store(c, xr[c]);
 }
 
 __global__ void k_silu_mul(const uint4* __restrict__ gu, uint4* __restrict__ out, int rows, int inter) {
@@ -112,19 +140,6 @@ __global__ void k_silu_mul(const uint4* __restrict__ gu, uint4* __restrict__ out
   }
 }
 
-// ---- the rotation of tree_attn.cu (rotate-half pairing, f_i as a float
-// pair from fp64, Cody-Waite reduction of the angle, MUFU sine/cosine)
-constexpr int ROPE_MAX_HALF = 512;
-
-__device__ __forceinline__ void rope_sincos(float pos, float2 f, float& sn, float& cs) {
-  const float a_hi = pos * f.x;
-  const float a_lo = fmaf(pos, f.y, fmaf(pos, f.x, -a_hi));
-  const float k = rintf(a_hi * 0.15915493667125702f);
-  float r = fmaf(-k, 6.2831854820251465f, a_hi);
-  r = fmaf(-k, -1.7484555314695172e-07f, r) + a_lo;
-  __sincosf(r, &sn, &cs);
-}
-
 // node-major rows in[(b * n_pad + i) * stride + h * D + d] -> head-major
 // out[((b * heads + h) * n_pad + i) * D + d], rotated by pos[b][i] when
 // rotate != 0 (a negative position is copied unrotated).  One thread per pair
@@ -132,7 +147,7 @@ __device__ __forceinline__ void rope_sincos(float pos, float2 f, float& sn, floa
 __global__ void k_rope_heads(const __nv_bfloat16* __restrict__ in, int stride, __nv_bfloat16* __restrict__ out,
                              int B, int n_pad, int heads, int D, const int32_t* __restrict__ pos, int rotate,
                              double nl2f) {
-  __shared__ float2 tab[ROPE_MAX_HALF];
+  __shared__ float2 tab[FC_ROPE_MAX_HALF];
   if (rotate) {
     for (int i = threadIdx.x; i < D / 2; i += blockDim.x) {
       const double f = exp2((double)i * nl2f);
@@ -160,8 +175,8 @@ __global__ void k_rope_heads(const __nv_bfloat16* __restrict__ in, int stride, _
       for (int q = 0; q < 4; ++q) {
         const float2 xl = bf2f(l[q]), xh = bf2f(hh[q]);
         float s0, c0, s1, c1;
-        rope_sincos((float)p, tab[8 * c + 2 * q], s0, c0);
-        rope_sincos((float)p, tab[8 * c + 2 * q + 1], s1, c1);
+        fc_rope_sincos((float)p, tab[8 * c + 2 * q], s0, c0);
+        fc_rope_sincos((float)p, tab[8 * c + 2 * q + 1], s1, c1);
         l[q] = f2bf(xl.x * c0 - xh.x * s0, xl.y * c1 - xh.y * s1);
         hh[q] = f2bf(xh.x * c0 + xl.x * s0, xh.y * c1 + xl.y * s1);
       }
@@ -194,10 +209,9 @@ extern "C" fc_status fc_add_rmsnorm(void* d_x, const void* d_r, const void* d_w,
   if (rows == 0) return FC_OK;
   if (!d_x || !d_w || !d_out || !aligned16(d_x) || !aligned16(d_w) || !aligned16(d_out) || (d_r && !aligned16(d_r)))
     return FC_ERR_INVALID_ARG;
-  k_add_rmsnorm<<<(rows + ROWS_PER_BLOCK - 1) / ROWS_PER_BLOCK, ROWS_PER_BLOCK * 32, 0,
-                  static_cast<cudaStream_t>(stream)>>>(static_cast<uint4*>(d_x), static_cast<const uint4*>(d_r),
-                                                       static_cast<const uint4*>(d_w), static_cast<uint4*>(d_out),
-                                                       rows, dim, eps);
+  k_add_rmsnorm<<<rows, NORM_THREADS, 0, static_cast<cudaStream_t>(stream)>>>(
+      static_cast<uint4*>(d_x), static_cast<const uint4*>(d_r), static_cast<const uint4*>(d_w),
+      static_cast<uint4*>(d_out), rows, dim, eps);
   return FC_CHECK_LAUNCH();
 }
 

@@ -278,6 +278,35 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N, ui
   return (1u << 4) | (1u << 7) | (1u << 10) | (b_mn_major << 16) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
 
+// ---- rotary position embedding (Su et al., RoFormer), rotate-half pairing:
+// dimension i pairs with i + D/2 and turns by pos * f_i, f_i = base^(-2i/D).
+// f_i is held as two floats (hi + lo, from fp64), so that pos * f_i comes out
+// as hi * pos, its exact rounding error (an fma) and lo * pos: the angle is
+// good to ~1e-7 rad at any position below 2^24, where a plain fp32 product
+// would be off by pos * f_i * 2^-24.  The angle is reduced modulo 2 pi with a
+// two-constant Cody-Waite split (2 pi rounded to fp32, then the rest) before
+// the MUFU sine and cosine, which are accurate on [-pi, pi].
+constexpr int FC_ROPE_MAX_HALF = 512;  // D / 2 for D up to 1024
+
+// tab[i] = (hi, lo) of f_i for i < half, filled by the calling block's
+// threads; the caller synchronises before use.
+__device__ __forceinline__ void fc_rope_table(float2* tab, int half, double nl2f) {
+  for (int i = threadIdx.x; i < half; i += blockDim.x) {
+    const double f = exp2((double)i * nl2f);
+    const float hi = (float)f;
+    tab[i] = make_float2(hi, (float)(f - (double)hi));
+  }
+}
+
+__device__ __forceinline__ void fc_rope_sincos(float pos, float2 f, float& sn, float& cs) {
+  const float a_hi = pos * f.x;
+  const float a_lo = fmaf(pos, f.y, fmaf(pos, f.x, -a_hi));
+  const float k = rintf(a_hi * 0.15915493667125702f);  // a / (2 pi), rounded
+  float r = fmaf(-k, 6.2831854820251465f, a_hi);        // 2 pi rounded to fp32
+  r = fmaf(-k, -1.7484555314695172e-07f, r) + a_lo;     // 2 pi minus that
+  __sincosf(r, &sn, &cs);
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);

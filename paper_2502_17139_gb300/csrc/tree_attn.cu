@@ -95,43 +95,14 @@ struct AttnArgs {
   double rope_nl2f;    // -2 log2(base) / D: pair i turns by pos * 2^(i * rope_nl2f)
 };
 
-// ---- rotary position embedding (Su et al., RoFormer), rotate-half pairing:
-// dimension i pairs with i + D/2 and turns by pos * f_i, f_i = base^(-2i/D).
-// f_i is held as two floats (hi + lo, from fp64), so that pos * f_i comes out
-// as hi * pos, its exact rounding error (an fma) and lo * pos: the angle is
-// good to ~1e-7 rad at any position below 2^24, where a plain fp32 product
-// would be off by pos * f_i * 2^-24.  The angle is reduced modulo 2 pi with a
-// two-constant Cody-Waite split (2 pi rounded to fp32, then the rest) before
-// the MUFU sine and cosine, which are accurate on [-pi, pi].
-constexpr int ROPE_MAX_HALF = 512;  // D / 2 for D up to 1024
-
-// tab[i] = (hi, lo) of f_i for i < half, filled by the calling block's
-// threads; the caller synchronises before use.
-__device__ __forceinline__ void rope_table(float2* tab, int half, double nl2f) {
-  for (int i = threadIdx.x; i < half; i += blockDim.x) {
-    const double f = exp2((double)i * nl2f);
-    const float hi = (float)f;
-    tab[i] = make_float2(hi, (float)(f - (double)hi));
-  }
-}
-
-__device__ __forceinline__ void rope_sincos(float pos, float2 f, float& sn, float& cs) {
-  const float a_hi = pos * f.x;
-  const float a_lo = fmaf(pos, f.y, fmaf(pos, f.x, -a_hi));
-  const float k = rintf(a_hi * 0.15915493667125702f);  // a / (2 pi), rounded
-  float r = fmaf(-k, 6.2831854820251465f, a_hi);        // 2 pi rounded to fp32
-  r = fmaf(-k, -1.7484555314695172e-07f, r) + a_lo;     // 2 pi minus that
-  __sincosf(r, &sn, &cs);
-}
-
 // Rotates the two pairs held by one 32-bit word of each half: l holds
 // dimensions i, i + 1 and h the same dimensions + D/2.
 __device__ __forceinline__ void rope_word(uint32_t& l, uint32_t& h, float pos, const float2* tab, int i) {
   __nv_bfloat162 lb = *reinterpret_cast<__nv_bfloat162*>(&l), hb = *reinterpret_cast<__nv_bfloat162*>(&h);
   const float2 xl = __bfloat1622float2(lb), xh = __bfloat1622float2(hb);
   float s0, c0, s1, c1;
-  rope_sincos(pos, tab[i], s0, c0);
-  rope_sincos(pos, tab[i + 1], s1, c1);
+  fc_rope_sincos(pos, tab[i], s0, c0);
+  fc_rope_sincos(pos, tab[i + 1], s1, c1);
   lb = __float22bfloat162_rn(make_float2(xl.x * c0 - xh.x * s0, xl.y * c1 - xh.y * s1));
   hb = __float22bfloat162_rn(make_float2(xh.x * c0 + xl.x * s0, xh.y * c1 + xl.y * s1));
   l = *reinterpret_cast<uint32_t*>(&lb);
@@ -334,7 +305,7 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   // Q tiles: rows (head in group, node) packed densely, 128-byte swizzled, K-major.
   if constexpr (ROPE) {
     __shared__ float2 s_rope[HD / 2];
-    rope_table(s_rope, HD / 2, a.rope_nl2f);
+    fc_rope_table(s_rope, HD / 2, a.rope_nl2f);
     __syncthreads();
     stage_q_rope(smem + OFF_Q, a.q, a.pos, s_rope, b, g, a.G, a.H, a.n_pad, nn, row0, rows_total, tid);
   } else
@@ -804,8 +775,8 @@ uint64_t attn_units(int batch, int n_pad, int H, int Hkv) {
 // [B][heads][n_pad][D] (tree keys).  One thread per pair of partner chunks.
 __global__ void k_rope(const uint4* __restrict__ in, uint4* __restrict__ out, int B, int n_pad, int heads, int D,
                        int layout, const int32_t* __restrict__ pos, double nl2f) {
-  __shared__ float2 tab[ROPE_MAX_HALF];
-  rope_table(tab, D / 2, nl2f);
+  __shared__ float2 tab[FC_ROPE_MAX_HALF];
+  fc_rope_table(tab, D / 2, nl2f);
   __syncthreads();
   const int ch = D / 16;  // 16-byte chunks per half row
   const size_t items = (size_t)B * n_pad * heads * ch;

@@ -2,16 +2,18 @@
 verifies every draft, each token attending to the cached context and to its
 tree ancestors at position kv_len + depth), for a LLaMA-family decoder like
 the paper's models, composed from the C-ABI calls (argument marshalling
-only; every step runs in the library's kernels or cuBLASLt).
+only; every step runs in the library's kernels).
 
-Per layer: add + RMSNorm -> Q projection -> the fused K/V projection, its
-keys rotated and both laid out head-major (fc_rope_heads) -> tree attention
-with the queries rotated inside the kernel (fc_tree_attn_rope) over the
-layer's rotated cache -> output projection -> add + RMSNorm -> gate/up
-projection -> SiLU * up -> down projection.  The residual adds are fused into
-the next norm; after the last layer the final norm feeds the LM head.  The
-tree's rotated keys and values of every layer stay in buffers until the
-accepted path is appended to the caches.
+Per layer: add + RMSNorm -> Q projection -> the K/V projection, whose GEMM
+epilogue rotates the key heads and writes both head-major (fc_gemm_kv_heads)
+-> tree attention with the queries rotated inside the kernel
+(fc_tree_attn_rope) over the layer's rotated cache -> output projection ->
+add + RMSNorm -> the gate/up projection, whose GEMM epilogue applies SiLU *
+up (fc_gemm_silu_mul, weights interleaved once at construction) -> down
+projection.  The residual adds are fused into the next norm; after the last
+layer the final norm feeds the LM head.  The tree's rotated keys and values
+of every layer stay in buffers until the accepted path is appended to the
+caches.
 """
 from __future__ import annotations
 
@@ -56,12 +58,12 @@ class TreeDecoder:
         self.x = torch.empty((T, s.hidden), **bf)
         self.h = torch.empty((T, s.hidden), **bf)
         self.q = torch.empty((T, s.H * s.D), **bf)
-        self.kv = torch.empty((T, 2 * s.Hkv * s.D), **bf)
+        # the gate/up weights in the 128-column interleave fc_gemm_silu_mul reads
+        self.wgu = [fc.fc_interleave_gate_up(Lw["wgu"]) for Lw in W["layers"]]
         self.k_rot = [torch.empty((B, s.Hkv, n_pad, s.D), **bf) for _ in range(s.layers)]
         self.v_heads = [torch.empty((B, s.Hkv, n_pad, s.D), **bf) for _ in range(s.layers)]
         self.attn = torch.empty((T, s.H * s.D), **bf)
         self.o = torch.empty((T, s.hidden), **bf)
-        self.gu = torch.empty((T, 2 * s.inter), **bf)
         self.act = torch.empty((T, s.inter), **bf)
         self.logits = torch.empty((T, s.vocab), **bf)
 
@@ -77,9 +79,7 @@ class TreeDecoder:
         for l, Lw in enumerate(W["layers"]):
             fc.fc_add_rmsnorm(self.x, r, Lw["attn_norm"], self.h, s.eps)
             fc.fc_gemm_bf16(self.h, Lw["wq"], out=self.q)
-            fc.fc_gemm_bf16(self.h, Lw["wkv"], out=self.kv)
-            fc.fc_rope_heads(self.kv, 0, 2 * s.Hkv * s.D, self.k_rot[l], B, n_pad, s.Hkv, s.D, pos, s.rope_base)
-            fc.fc_rope_heads(self.kv, s.Hkv * s.D, 2 * s.Hkv * s.D, self.v_heads[l], B, n_pad, s.Hkv, s.D, pos, 0.0)
+            fc.fc_gemm_kv_heads(self.h, Lw["wkv"], B, n_pad, s.Hkv, pos, s.rope_base, self.k_rot[l], self.v_heads[l])
             ev = None
             if events is not None and "attn" in events:
                 ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -92,8 +92,7 @@ class TreeDecoder:
                 ev[1].record()
             fc.fc_gemm_bf16(self.attn, Lw["wo"], out=self.o)
             fc.fc_add_rmsnorm(self.x, self.o, Lw["mlp_norm"], self.h, s.eps)
-            fc.fc_gemm_bf16(self.h, Lw["wgu"], out=self.gu)
-            fc.fc_silu_mul(self.gu, self.act)
+            fc.fc_gemm_silu_mul(self.h, self.wgu[l], self.act)
             fc.fc_gemm_bf16(self.act, Lw["wd"], out=self.o)
             r = self.o
         fc.fc_add_rmsnorm(self.x, r, W["final_norm"], self.h, s.eps)

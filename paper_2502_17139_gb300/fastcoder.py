@@ -54,7 +54,7 @@ EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build
            "fc_datastore_build_noalloc", "fc_datastore_keys", "fc_datastore_save", "fc_datastore_file_info", "fc_datastore_load",
            "fc_retrieve", "fc_retrieve_all", "fc_retrieve_rev", "fc_reverse_tokens", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
-           "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_embed",
+           "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_gemm_kv_heads", "fc_gemm_silu_mul", "fc_interleave_gate_up", "fc_embed",
            "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
 
 
@@ -109,6 +109,9 @@ def _load():
         "fc_gemm_workspace": (sz, []),
         "fc_selftest_wait": (C.c_int, [i32, C.c_ulonglong, vp]),
         "fc_gemm_bf16": (C.c_int, [vp, vp, vp, i32, i32, i32, vp, sz, vp]),
+        "fc_gemm_kv_heads": (C.c_int, [vp, vp, i32, i32, i32, i32, i32, i32, vp, C.c_float, vp, vp, vp]),
+        "fc_gemm_silu_mul": (C.c_int, [vp, vp, i32, i32, i32, vp, vp]),
+        "fc_interleave_gate_up": (C.c_int, [vp, vp, i32, i32, vp]),
         "fc_embed": (C.c_int, [vp, i32, vp, i32, i32, vp, vp]),
         "fc_add_rmsnorm": (C.c_int, [vp, vp, vp, vp, i32, i32, C.c_float, vp]),
         "fc_silu_mul": (C.c_int, [vp, vp, i32, i32, vp]),
@@ -641,6 +644,46 @@ def fc_gemm_bf16(a, b, out=None):
         raise ValueError("out must be [M, N]")
     _check("fc_gemm_bf16", LIB.fc_gemm_bf16(_ptr(a), _ptr(b), _ptr(o), M, N, K, None, 0, _stream()))
     return o
+
+
+def fc_gemm_kv_heads(a, wkv, batch, n_pad, Hkv, pos, rope_base, k_rot, v_heads):
+    """kv = a [batch * n_pad, K] @ wkv [K, 2 * Hkv * 128]; key heads rotated by
+    pos [batch, n_pad] into k_rot, value heads into v_heads (both
+    [batch, Hkv, n_pad, 128], bf16)."""
+    _need(a, torch.bfloat16, "a")
+    _need(wkv, torch.bfloat16, "wkv")
+    _need(pos, torch.int32, "pos", (batch, n_pad))
+    M, K = a.shape
+    D = 128
+    if tuple(wkv.shape) != (K, 2 * Hkv * D):
+        raise ValueError("wkv must be [K, 2 * Hkv * 128]")
+    for t, name in ((k_rot, "k_rot"), (v_heads, "v_heads")):
+        _need(t, torch.bfloat16, name, (batch, Hkv, n_pad, D))
+    _check("fc_gemm_kv_heads", LIB.fc_gemm_kv_heads(_ptr(a), _ptr(wkv), M, K, Hkv, D, batch, n_pad, _ptr(pos),
+                                                    C.c_float(rope_base), _ptr(k_rot), _ptr(v_heads), _stream()))
+
+
+def fc_interleave_gate_up(wgu, out=None):
+    """[K, 2 * inter] gate|up weights -> 128-column blocks interleaved, for
+    fc_gemm_silu_mul."""
+    _need(wgu, torch.bfloat16, "wgu")
+    K, n2 = wgu.shape
+    o = out if out is not None else torch.empty_like(wgu)
+    _check("fc_interleave_gate_up", LIB.fc_interleave_gate_up(_ptr(wgu), _ptr(o), K, n2 // 2, _stream()))
+    return o
+
+
+def fc_gemm_silu_mul(a, wgu_interleaved, out):
+    """out [M, inter] = silu(a @ Wg) * (a @ Wu), with the weights interleaved by
+    fc_interleave_gate_up."""
+    _need(a, torch.bfloat16, "a")
+    _need(wgu_interleaved, torch.bfloat16, "wgu_interleaved")
+    M, K = a.shape
+    inter = wgu_interleaved.shape[1] // 2
+    _need(out, torch.bfloat16, "out", (M, inter))
+    _check("fc_gemm_silu_mul", LIB.fc_gemm_silu_mul(_ptr(a), _ptr(wgu_interleaved), M, K, inter, _ptr(out),
+                                                    _stream()))
+    return out
 
 
 def fc_embed(tok, table, out):

@@ -150,17 +150,29 @@ def chained_layer_checks(fc, dec, td, s, tok, nn, mask, pos, kvl):
         assert (np.abs(f64(td.h) - ref)[rows] <= (BF * (1 + d) + d) * np.abs(ref)[rows] + 1e-30).all()
         h = f64(td.h)
         fc.fc_gemm_bf16(td.h, Lw["wq"], out=td.q)
-        fc.fc_gemm_bf16(td.h, Lw["wkv"], out=td.kv)
         assert gemm_bound_ok(h[rows], f64(Lw["wq"]), f64(td.q)[rows])
-        assert gemm_bound_ok(h[rows], f64(Lw["wkv"]), f64(td.kv)[rows])
-        fc.fc_rope_heads(td.kv, 0, 2 * s.Hkv * s.D, td.k_rot[l], B, n_pad, s.Hkv, s.D, pos, s.rope_base)
-        fc.fc_rope_heads(td.kv, s.Hkv * s.D, 2 * s.Hkv * s.D, td.v_heads[l], B, n_pad, s.Hkv, s.D, pos, 0.0)
+        # the K/V projection, rotated and laid out head-major in the GEMM's epilogue
+        fc.fc_gemm_kv_heads(td.h, Lw["wkv"], B, n_pad, s.Hkv, pos, s.rope_base, td.k_rot[l], td.v_heads[l])
+        wkv = f64(Lw["wkv"])
+        K = wkv.shape[0]
+        G = K * U32 / (1 - K * U32) * (np.abs(h) @ np.abs(wkv))
+        kv = (h @ wkv).reshape(B, n_pad, 2, s.Hkv, s.D)
+        Gk = G.reshape(B, n_pad, 2, s.Hkv, s.D)
+        pp = np.repeat(pos.cpu().numpy()[:, :, None], s.Hkv, 2)
+        from oracle import oracle as orc
+        want_k = orc.rope(kv[:, :, 0], np.maximum(pp, 0), s.rope_base)
+        want_k[pp < 0] = kv[:, :, 0][pp < 0]
+        pair = lambda x: x + np.concatenate([x[..., 64:], x[..., :64]], -1)
+        lim = BF * np.abs(want_k) + (1 + BF) * pair(Gk[:, :, 0]) + 2.0 ** -20 * pair(np.abs(kv[:, :, 0]))
+        got_k = f64(td.k_rot[l]).transpose(0, 2, 1, 3)
+        assert (np.abs(got_k - want_k) <= lim).all()
+        got_v = f64(td.v_heads[l]).transpose(0, 2, 1, 3)
+        assert (np.abs(got_v - kv[:, :, 1]) <= BF * np.abs(kv[:, :, 1]) + (1 + BF) * Gk[:, :, 1]).all()
         fc.fc_tree_attn_rope(td.q.view(B, n_pad, s.H, s.D), td.k_cache[l], td.v_cache[l], kvl, td.k_rot[l],
                              td.v_heads[l], mask, dev(nn), pos, s.rope_base, out=td.attn.view(B, n_pad, s.H, s.D))
         torch.cuda.synchronize()
         # the attention on the GPU's own bf16 inputs, every row, in fp64
         bits = lambda t: t.cpu().view(torch.int16).numpy().view(np.uint16)
-        from oracle import oracle as orc
         # fc_tree_attn_rope rotates Q while staging it (the tree keys arrive rotated):
         # rotate Q here and round it to bf16 as the kernel stores it
         qh = orc.rope(f64(td.q.view(B, n_pad, s.H, s.D)), np.repeat(pos.cpu().numpy()[:, :, None], s.H, 2))
@@ -178,12 +190,18 @@ def chained_layer_checks(fc, dec, td, s, tok, nn, mask, pos, kvl):
         fc.fc_add_rmsnorm(td.x, td.o, Lw["mlp_norm"], td.h, s.eps)
         assert (np.abs(f64(td.x) - (x0 + o)) <= (BF + U32) * np.abs(x0 + o)).all()
         h = f64(td.h)
-        fc.fc_gemm_bf16(td.h, Lw["wgu"], out=td.gu)
-        assert gemm_bound_ok(h[rows], f64(Lw["wgu"]), f64(td.gu)[rows])
-        fc.fc_silu_mul(td.gu, td.act)
-        gu = f64(td.gu)
-        ref = dec.silu(gu[:, :s.inter]) * gu[:, s.inter:]
-        assert (np.abs(f64(td.act) - ref)[rows] <= 2 * BF * np.abs(ref)[rows] + 1e-30).all()
+        # the gate/up projection with SiLU * up in the GEMM's epilogue
+        fc.fc_gemm_silu_mul(td.h, td.wgu[l], td.act)
+        wgu = f64(Lw["wgu"])
+        K = wgu.shape[0]
+        G = K * U32 / (1 - K * U32) * (np.abs(h) @ np.abs(wgu))
+        gu = h @ wgu
+        g, u = gu[:, :s.inter], gu[:, s.inter:]
+        silu = dec.silu(g)
+        ref = silu * u
+        lim = (BF + 2.0 ** -10) * np.abs(ref) + 1.1 * np.abs(u) * G[:, :s.inter] + np.abs(silu) * G[:, s.inter:] \
+            + G[:, :s.inter] * G[:, s.inter:] + 1e-30
+        assert (np.abs(f64(td.act) - ref)[rows] <= lim[rows]).all()
         act = f64(td.act)
         fc.fc_gemm_bf16(td.act, Lw["wd"], out=td.o)
         assert gemm_bound_ok(act[rows], f64(Lw["wd"]), f64(td.o)[rows])

@@ -12,7 +12,8 @@
   replay hits) in lockstep with the oracle's step loop, and its tree
   attention on every row of one step against the fp64 oracle.
 * The decoder forward at DeepSeek-Coder 1.3B's layer width against the fp64
-  oracle on every node of two sequences.
+  oracle on every node of two sequences, within three times the distance
+  that bf16 storage alone puts between the oracle and the exact forward.
 * Algorithm 1 on the default two-source store through properties that hold
   at any size (served drafts and their counts recounted in the stores, no
   longer match, missing-table keys absent from both corpora).
@@ -285,16 +286,22 @@ def test_decoder_full_width(fc, orc):
     torch.cuda.synchronize()
     assert fc.fc_get_error() == "FC_OK"
     ref, k_new, v_new = dec.forward(cfg, W, tok, par, nn, kvl, kc, vc, m["pos"])
+    mir, k_mir, v_mir = dec.forward(cfg, W, tok, par, nn, kvl, kc, vc, m["pos"], store_bf16=True)
     got = f64(logits)
+    # tolerance: three times the distance that bf16 storage alone puts between the
+    # oracle's forward and the exact one (the derivation is in tests/test_gpu_decoder.py)
     for b in range(B):
         n = int(nn[b])
-        assert np.abs(got[b, :n] - ref[b, :n]).max() <= 0.06
+        tol = 3 * np.abs(mir[b, :n] - ref[b, :n]).max()
+        assert 0 < tol and np.abs(got[b, :n] - ref[b, :n]).max() <= tol
         top2 = np.sort(ref[b, :n], axis=1)[:, -2:]
-        clear = top2[:, 1] - top2[:, 0] > 0.25
+        clear = top2[:, 1] - top2[:, 0] > tol
         assert (np.argmax(got[b, :n], 1)[clear] == np.argmax(ref[b, :n], 1)[clear]).all()
         for l in range(s.layers):
-            assert np.abs(f64(td.k_rot[l])[b, :, :n].transpose(1, 0, 2) - k_new[l, b, :n]).max() <= 0.06
-            assert np.abs(f64(td.v_heads[l])[b, :, :n].transpose(1, 0, 2) - v_new[l, b, :n]).max() <= 0.06
+            tk = 3 * np.abs(k_mir[l, b, :n] - k_new[l, b, :n]).max()
+            tv = max(3 * np.abs(v_mir[l, b, :n] - v_new[l, b, :n]).max(), 2.0 ** -8 * np.abs(v_new[l, b, :n]).max())
+            assert np.abs(f64(td.k_rot[l])[b, :, :n].transpose(1, 0, 2) - k_new[l, b, :n]).max() <= tk
+            assert np.abs(f64(td.v_heads[l])[b, :, :n].transpose(1, 0, 2) - v_new[l, b, :n]).max() <= tv
 
 
 def test_algorithm1_full_size_properties(fc):

@@ -95,3 +95,77 @@ def test_gemm_back_to_back_and_empty(fc):
         fc.fc_gemm_bf16(bad, torch.empty((12, 16), dtype=torch.bfloat16, device="cuda"))
     assert e.value.status == "FC_ERR_UNSUPPORTED"
     assert fc.fc_get_error() == "FC_OK"
+
+
+def gemm_magnitude(a, b):
+    """Exact product and the fp32-accumulation error bound per element."""
+    A = a.double().cpu().numpy()
+    Bm = b.double().cpu().numpy()
+    K = A.shape[1]
+    u = 2.0 ** -23
+    return A @ Bm, K * u / (1 - K * u) * (np.abs(A) @ np.abs(Bm))
+
+
+@pytest.mark.parametrize("batch,n_pad,Hkv,K", [(3, 64, 2, 256), (2, 128, 1, 520), (5, 64, 3, 2048)])
+def test_gemm_kv_heads(fc, orc, batch, n_pad, Hkv, K):
+    """The K/V projection with RoPE and the head-major layout in its epilogue,
+    against the exact product rotated by the oracle's RoPE (O12).  Bound per
+    element: one bf16 rounding of the result, plus the accumulation bound of
+    both members of the rotated pair, plus 2^-20 of their magnitudes for the
+    fp32 rotation (angle to ~1e-7 rad)."""
+    M, D = batch * n_pad, 128
+    a, w = operands(M, 2 * Hkv * D, K, 11 * K + Hkv)
+    rng = np.random.default_rng(K)
+    pos = rng.integers(0, 70000, (batch, n_pad)).astype(np.int32)
+    pos[:, -5:] = -1  # padding rows stay unrotated
+    k_rot = torch.full((batch, Hkv, n_pad, D), float("nan"), dtype=torch.bfloat16, device="cuda")
+    v_heads = torch.full_like(k_rot, float("nan"))
+    fc.fc_gemm_kv_heads(a, w, batch, n_pad, Hkv, torch.from_numpy(pos).cuda(), 10000.0, k_rot, v_heads)
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_OK"
+    exact, G = gemm_magnitude(a, w)
+    kv = exact.reshape(batch, n_pad, 2, Hkv, D)
+    Gk = G.reshape(batch, n_pad, 2, Hkv, D)
+    kk = kv[:, :, 0]
+    p = np.repeat(pos[:, :, None], Hkv, 2)
+    want_k = orc.rope(kk, np.maximum(p, 0))
+    want_k[p < 0] = kk[p < 0]
+    pair = lambda x: x + np.concatenate([x[..., 64:], x[..., :64]], -1)  # |x_d| + |x_(d +- 64)|
+    lim_k = 2.0 ** -8 * np.abs(want_k) + (1 + 2.0 ** -8) * pair(Gk[:, :, 0]) + 2.0 ** -20 * pair(np.abs(kk))
+    got_k = k_rot.double().cpu().numpy().transpose(0, 2, 1, 3)
+    assert (np.abs(got_k - want_k) <= lim_k).all()
+    want_v = kv[:, :, 1]
+    lim_v = 2.0 ** -8 * np.abs(want_v) + (1 + 2.0 ** -8) * Gk[:, :, 1]
+    got_v = v_heads.double().cpu().numpy().transpose(0, 2, 1, 3)
+    assert (np.abs(got_v - want_v) <= lim_v).all()
+
+
+def test_interleave_gate_up(fc):
+    K, inter = 72, 384
+    w = torch.randn((K, 2 * inter)).to(torch.bfloat16).cuda()
+    out = fc.fc_interleave_gate_up(w)
+    torch.cuda.synchronize()
+    g, u = w[:, :inter].cpu(), w[:, inter:].cpu()
+    o = out.cpu().view(K, inter // 128, 2, 128)
+    assert torch.equal(o[:, :, 0].reshape(K, inter), g) and torch.equal(o[:, :, 1].reshape(K, inter), u)
+
+
+@pytest.mark.parametrize("M,K,inter", [(777, 512, 384), (2048, 2048, 5504)])
+def test_gemm_silu_mul(fc, M, K, inter):
+    """silu(A Wg) * (A Wu) from the fp32 accumulators, rounded once: within one
+    bf16 rounding of the exact value, plus the accumulation bounds carried
+    through (|d silu / dg| <= 1.1), plus 2^-10 of the value for the fp32
+    evaluation with the hardware exponential."""
+    a, w = operands(M, 2 * inter, K, M + inter)
+    act = torch.empty((M, inter), dtype=torch.bfloat16, device="cuda")
+    fc.fc_gemm_silu_mul(a, fc.fc_interleave_gate_up(w), act)
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_OK"
+    exact, G = gemm_magnitude(a, w)
+    g, u = exact[:, :inter], exact[:, inter:]
+    silu = g / (1 + np.exp(-g))
+    ref = silu * u
+    lim = (2.0 ** -8 + 2.0 ** -10) * np.abs(ref) + 1.1 * np.abs(u) * G[:, :inter] + np.abs(silu) * G[:, inter:] \
+        + G[:, :inter] * G[:, inter:] + 1e-30
+    got = act.double().cpu().numpy()
+    assert (np.abs(got - ref) <= lim).all()
