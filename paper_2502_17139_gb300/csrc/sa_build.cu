@@ -115,18 +115,32 @@ __global__ void __launch_bounds__(RS_THREADS) k_radix_hist(const uint64_t* __res
 
 // Stable scatter of one 8-bit digit.  offs[d * nb + block] is the exclusive
 // scan of the digit-major histogram: where this block's digit-d keys start.
+// The block first ranks its keys (per warp with __match_any_sync, then across
+// warps and digits), places them in shared memory in digit order, and then
+// writes them out in that order: consecutive threads write consecutive
+// addresses of a digit's run, so the stores coalesce instead of spraying
+// 8- and 4-byte writes over 256 runs.
+constexpr uint32_t RS_SMEM = RS_TILE * (8 + 4);  // keys and values of one tile
+
 __global__ void __launch_bounds__(RS_THREADS) k_radix_scatter(const uint64_t* __restrict__ kin,
                                                               const uint32_t* __restrict__ vin,
                                                               uint64_t* __restrict__ kout,
                                                               uint32_t* __restrict__ vout, uint64_t n, int shift,
                                                               const uint32_t* __restrict__ offs, uint64_t nb) {
+  extern __shared__ __align__(16) unsigned char rs_smem[];
+  uint64_t* skey = reinterpret_cast<uint64_t*>(rs_smem);
+  uint32_t* sval = reinterpret_cast<uint32_t*>(rs_smem + RS_TILE * 8);
   __shared__ uint32_t wbin[RS_WARPS][256];
   __shared__ uint32_t base_s[256];
+  __shared__ uint32_t doff[256];   // where digit d starts in the block's digit order
+  __shared__ uint32_t wsum[RS_THREADS / 32];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   for (int d = tid; d < RS_WARPS * 256; d += RS_THREADS) (&wbin[0][0])[d] = 0;
   base_s[tid] = offs[(uint64_t)tid * nb + blockIdx.x];
   __syncthreads();
-  const uint64_t w0 = blockIdx.x * (uint64_t)RS_TILE + (uint64_t)warp * RS_WARP_CHUNK;
+  const uint64_t b0 = blockIdx.x * (uint64_t)RS_TILE;
+  const uint32_t count = (uint32_t)min((uint64_t)RS_TILE, n - b0);
+  const uint64_t w0 = b0 + (uint64_t)warp * RS_WARP_CHUNK;
   const uint32_t lt = (1u << lane) - 1u;
   uint64_t key[RS_ITEMS];
   uint32_t val[RS_ITEMS];
@@ -146,25 +160,44 @@ __global__ void __launch_bounds__(RS_THREADS) k_radix_scatter(const uint64_t* __
     __syncwarp();
   }
   __syncthreads();
-  {
-    uint32_t run = 0;
+  // per digit (thread tid = digit): warp prefix, then the digit's block total
+  uint32_t run = 0;
 #pragma unroll
-    for (int w = 0; w < RS_WARPS; ++w) {
-      uint32_t c = wbin[w][tid];
-      wbin[w][tid] = run;
-      run += c;
-    }
+  for (int w = 0; w < RS_WARPS; ++w) {
+    uint32_t c = wbin[w][tid];
+    wbin[w][tid] = run;
+    run += c;
   }
+  // exclusive scan of the digit totals over the 256 digits
+  uint32_t inc = run;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+    if (lane >= o) inc += y;
+  }
+  if (lane == 31) wsum[warp] = inc;
+  __syncthreads();
+  uint32_t before = 0;
+  for (int w = 0; w < warp; ++w) before += wsum[w];
+  doff[tid] = before + inc - run;
   __syncthreads();
 #pragma unroll
   for (int it = 0; it < RS_ITEMS; ++it) {
     uint64_t idx = w0 + (uint64_t)it * 32 + lane;
     if (idx < n) {
-      uint32_t d = (uint32_t)(key[it] >> shift) & 255u;
-      uint64_t pos = (uint64_t)base_s[d] + wbin[warp][d] + lr[it];
-      kout[pos] = key[it];
-      vout[pos] = val[it];
+      const uint32_t d = (uint32_t)(key[it] >> shift) & 255u;
+      const uint32_t at = doff[d] + wbin[warp][d] + lr[it];
+      skey[at] = key[it];
+      sval[at] = val[it];
     }
+  }
+  __syncthreads();
+  for (uint32_t j = tid; j < count; j += RS_THREADS) {
+    const uint64_t k = skey[j];
+    const uint32_t d = (uint32_t)(k >> shift) & 255u;
+    const uint64_t pos = (uint64_t)base_s[d] + (j - doff[d]);
+    kout[pos] = k;
+    vout[pos] = sval[j];
   }
 }
 
@@ -336,6 +369,8 @@ extern "C" fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n, ui
   const unsigned g = grid_for(n, 256);
   uint32_t hctl[2] = {0, 0};
 
+  if (cudaFuncSetAttribute(k_radix_scatter, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)RS_SMEM) != cudaSuccess)
+    return FC_ERR_CUDA;
   if (cudaMemsetAsync(ctl, 0, 64, s) != cudaSuccess) return FC_ERR_CUDA;
   k_check_tokens<<<g, 256, 0, s>>>(d_tokens, n, vocab, ctl);
   if (cudaMemcpyAsync(hctl, ctl, 8, cudaMemcpyDeviceToHost, s) != cudaSuccess) return FC_ERR_CUDA;
@@ -359,7 +394,7 @@ extern "C" fc_status fc_datastore_build(const uint32_t* d_tokens, uint64_t n, ui
     for (int p = 0; p < np; ++p) {
       k_radix_hist<<<(unsigned)L.nb, RS_THREADS, 0, s>>>(kin, n, shifts[p], hist, L.nb);
       if (exclusive_scan(hist, 256 * L.nb, stmp, s) != cudaSuccess) return FC_ERR_CUDA;
-      k_radix_scatter<<<(unsigned)L.nb, RS_THREADS, 0, s>>>(kin, vin, kout, vout, n, shifts[p], hist, L.nb);
+      k_radix_scatter<<<(unsigned)L.nb, RS_THREADS, RS_SMEM, s>>>(kin, vin, kout, vout, n, shifts[p], hist, L.nb);
       std::swap(kin, kout);
       std::swap(vin, vout);
     }
