@@ -134,7 +134,7 @@ __global__ void k_silu_mul(const uint4* __restrict__ gu, uint4* __restrict__ out
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const float2 a = bf2f(gg[q]), b = bf2f(uu[q]);
-      rv[q] = f2bf(a.x / (1.f + __expf(-a.x)) * b.x, a.y / (1.f + __expf(-a.y)) * b.y);
+      rv[q] = f2bf(__fdividef(a.x, 1.f + __expf(-a.x)) * b.x, __fdividef(a.y, 1.f + __expf(-a.y)) * b.y);
     }
     out[e] = res;
   }

@@ -237,7 +237,9 @@ __global__ void __launch_bounds__(GM_THREADS, 1)
 #pragma unroll
             for (int u = 0; u < 32; ++u) {
               const float x = __uint_as_float(gv[u]);
-              a[u] = x / (1.f + __expf(-x)) * __uint_as_float(uv[u]);
+              // the fast divide: an IEEE division takes a slow path for a zero dividend,
+              // which doubled this epilogue's time on padding rows (all zeros)
+              a[u] = __fdividef(x, 1.f + __expf(-x)) * __uint_as_float(uv[u]);
             }
 #pragma unroll
             for (int u = 0; u < 4; ++u)
