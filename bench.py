@@ -1465,9 +1465,6 @@ def run_gemm(args, rank, ws, local):
     timed beside torch.matmul (cuBLAS) on the same operands in the same run.
     Each shape runs back to back on operands that stay resident; the weights
     of the larger shapes exceed L2."""
-    # the library GEMMs get the 32 MiB workspace a direct cuBLASLt caller would give them
-    os.environ.setdefault("CUBLASLT_WORKSPACE_SIZE", "32768")
-    os.environ.setdefault("CUBLAS_WORKSPACE_CONFIG", ":32768:2")
     import torch
 
     import paper_2502_17139_gb300.fastcoder as fc
