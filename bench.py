@@ -15,8 +15,8 @@ before timing; their build time is reported separately.
 
 Arms:
   default           the CUDA path (libfastcoder.so through its C ABI)
-  --impl reference  the CPU oracle, timed on the host cores on a bounded
-                    sample of the same workload per step, scaled to a step
+  --impl reference  the CPU oracle, timed on the host cores, each timed step
+                    one full, unsampled step of all 32 sequences
 
 Under torchrun every rank runs an independent batch of 32 sequences on its
 own GPU against replicated datastores (no data-path collective); the timed
@@ -25,6 +25,8 @@ region is bracketed by barriers and the slowest rank's time is used.
 from __future__ import annotations
 
 import argparse
+import contextlib
+import gc
 import json
 import os
 import statistics
@@ -93,8 +95,9 @@ def parse_args(argv=None):
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
     ap.add_argument("--no-graph", action="store_true",
                     help="step mode: skip timing the same steps replayed from CUDA graphs (two steps per graph)")
-    ap.add_argument("--split", type=int, default=2,
-                    help="step mode: sub-batches of the sequences, each on its own CUDA stream (1: one stream)")
+    ap.add_argument("--split", type=int, default=4,
+                    help="step mode: sub-batches of the sequences, each on CUDA streams of its own, issued by the "
+                         "native step executor (1: the single-stream StepLoop)")
     ap.add_argument("--all-occ", action="store_true",
                     help="retrieve mode: also time the all-occurrence trie (fc_retrieve_all + fc_build_tree_all)")
     ap.add_argument("--rev", action="store_true",
@@ -129,6 +132,19 @@ def attn_traffic(args, algorithmic_bytes_per_launch):
     if h.hexdigest() != ATTN_TRAFFIC["sha256"]:
         return None
     return ATTN_TRAFFIC["ratio"] * algorithmic_bytes_per_launch
+
+
+@contextlib.contextmanager
+def no_gc():
+    """The Python garbage collector off inside a timed region: a collection
+    pause on the host would land in a wall-clock (e2e) number."""
+    was = gc.isenabled()
+    gc.disable()
+    try:
+        yield
+    finally:
+        if was:
+            gc.enable()
 
 
 def load_peaks():
@@ -339,6 +355,11 @@ def run_ours(args, rank, ws, local):
     mk = lambda: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
     # stage events per timed step and sub-batch (recorded on the sub-batch's stream)
     stage_ev = [[dict(attn=mk(), retrieve=mk(), tree=mk(), tail=mk()) for _ in range(nsub)] for _ in range(K)]
+    for per_step in stage_ev:  # torch creates an event at its first record: do that before the timed region
+        for d in per_step:
+            for a, b in d.values():
+                a.record()
+                b.record()
 
     def do_step(s, timed_idx=None):
         j = s % P
@@ -354,12 +375,13 @@ def run_ours(args, rank, ws, local):
     clocks = ClockSampler(local)
     clocks.wait_first()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    start.record(stream)
-    for i in range(K):
-        do_step(W + i, i)
-    join(loop)
-    end.record(stream)
-    torch.cuda.synchronize()
+    with no_gc():
+        start.record(stream)
+        for i in range(K):
+            do_step(W + i, i)
+        join(loop)
+        end.record(stream)
+        torch.cuda.synchronize()
     clock_rec = clocks.stop()
     barrier(ws)
     t_ms = start.elapsed_time(end)
@@ -413,7 +435,9 @@ def run_ours(args, rank, ws, local):
                    "batch_per_gpu": B, "global_batch": B * ws, "kv_len0": kv0, "n_pad": n_pad,
                    "l2": "inputs larger than L2 (KV cache %.1f GB per GPU)" % (2 * kc.numel() * 2 / 1e9),
                    "parallelism": f"replicas x{ws}",
-                   "streams": f"{nsub} sub-batches of {B // nsub}-{-(-B // nsub)} sequences, one CUDA stream each"},
+                   "streams": (f"{nsub} sub-batches of {B // nsub}-{-(-B // nsub)} sequences issued by the native "
+                               "step executor, each on a chain stream and an attention stream" if nsub > 1
+                               else "one stream")},
         "roofline": roof,
         "gpu_launches": 8 * K * nsub,
         "clocks": clock_rec,
@@ -664,10 +688,12 @@ def run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws):
     run(0, W)
     torch.cuda.synchronize()
     barrier(ws)
-    t0 = time.perf_counter()
-    run(W, K)
-    torch.cuda.synchronize()
-    t = max_over_ranks(time.perf_counter() - t0, ws)
+    with no_gc():
+        t0 = time.perf_counter()
+        run(W, K)
+        torch.cuda.synchronize()
+        t1 = time.perf_counter()
+    t = max_over_ranks(t1 - t0, ws)
     d = sets[0]
     h2d = d["q"].numel() * 2 + d["k"].numel() * 2 + d["v"].numel() * 2 + 4 * (2 * B + d["r"].numel())
     return {"value": weak_value(K, ws, t * 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),

@@ -687,6 +687,107 @@ fc_status fc_synth_argmax(const uint32_t* d_tok, const int32_t* d_parent, const 
                           int batch, int n_pad, const int32_t* d_plen, const uint32_t* d_rtok,
                           uint32_t vocab, uint32_t* d_argmax, fc_stream s);
 
+/* ------------------------------------------------------------------------
+ * Native step executor (the decoding step of Section IV-C and IV-D over
+ * sub-batches: replay-cache lookup -> fc_retrieve -> insert ->
+ * fc_build_tree -> [fc_rope] -> fc_tree_attn[_rope] -> fc_synth_argmax ->
+ * fc_accept -> fc_kv_append).  One call enqueues the whole step of every
+ * sub-batch; each sub-batch runs on two streams the executor owns, a
+ * high-priority one for its latency-bound chain and a low-priority one for
+ * its attention, so sub-batches overlap.  The executor owns no device
+ * memory: all buffers below belong to the caller and must outlive it.
+ * ------------------------------------------------------------------------ */
+typedef struct {
+  int32_t batch;            /* sequences in this sub-batch (>= 1) */
+  int32_t first;            /* index of its first sequence in the batch-wide step inputs */
+  uint32_t* ctx;            /* [batch][ctx_stride] contexts, appended to in place */
+  int32_t ctx_stride;
+  int32_t* ctx_len[2];      /* [batch] each; a step of phase c reads [c] and writes [1 - c] */
+  int32_t* kv_len[2];       /* [batch] each; as ctx_len */
+  uint32_t* root;           /* [batch] the next tree's root token, rewritten by each step */
+  void* rcache;             /* fc_rcache_init'ed table, or NULL (no replay cache) */
+  int32_t rcache_capacity;
+  int32_t* skip;            /* [batch] scratch: queries the replay cache served */
+  /* retrieval outputs, fc_retrieve's layout with top_k slots */
+  uint32_t* drafts;
+  int32_t* draft_len;
+  uint32_t* count;
+  int32_t* n_drafts;
+  int32_t* match_len;
+  /* tree outputs, fc_build_tree's layout */
+  uint32_t* tok;
+  int32_t* parent;
+  int32_t* depth;
+  int32_t* pos;
+  uint64_t* mask;
+  int32_t* n_nodes;
+  void* k_cache;            /* bf16 [batch][Hkv][kv_cap][D]: this sub-batch's rows */
+  void* v_cache;
+  void* k_tree_rot;         /* bf16 [batch][Hkv][n_pad][D] rotated tree keys (RoPE only, else NULL) */
+  void* attn_out;           /* bf16 [batch][n_pad][H][D] */
+  void* attn_ws;            /* fc_tree_attn workspace of this sub-batch (NULL: no key split) */
+  size_t attn_ws_bytes;
+  uint32_t* argmax;         /* [batch][n_pad] */
+  int32_t* acc_len;         /* [batch] */
+  int32_t* path;            /* [batch][path_cap] */
+  uint32_t* bonus;          /* [batch] */
+} fc_pipeline_part;
+
+typedef struct {
+  const fc_datastore* sources;  /* host [n_sources], copied at creation */
+  int32_t n_sources;
+  fc_retrieve_params p;
+  const uint32_t* src_weight;   /* host [n_sources] tree weights (Eq. 3), copied */
+  int32_t node_budget, n_pad, H, Hkv, D, kv_cap, path_cap;
+  uint32_t vocab;               /* the synthetic target model's vocabulary */
+  float scale;                  /* attention scale (> 0) */
+  float rope_base;              /* 0: q and tree keys arrive rotated; > 0: RoPE base */
+  int32_t n_parts;
+  const fc_pipeline_part* parts;  /* host [n_parts], copied */
+} fc_pipeline_desc;
+
+typedef struct fc_pipeline fc_pipeline;
+
+/* Checks the description (FC_ERR_INVALID_ARG: a missing buffer, a
+ * non-positive size, equal ping-pong buffers), creates the streams and
+ * events and returns the executor in *out.  FC_ERR_CUDA if a stream or
+ * event cannot be created (nothing is left allocated). */
+fc_status fc_pipeline_create(const fc_pipeline_desc* desc, fc_pipeline** out);
+
+/*
+ * Enqueues one step of every sub-batch.  Per-step inputs are batch-wide
+ * device arrays; sub-batch h reads its rows from `first`:
+ *   d_q [B][n_pad][H][D] bf16, d_k_tree and d_v_tree [B][Hkv][n_pad][D]
+ *   bf16 (unrotated when rope_base > 0), d_want_hit [B] (NULL: every query
+ *   may hit the replay cache), d_plen [B], d_rtok [B][n_pad] (the synthetic
+ *   model's draws).
+ * phase (0 or 1) selects the ping-pong lengths read; alternate it.  flags:
+ * 0, or FC_PIPELINE_NO_ATTENTION to leave out the attention launch (the
+ * synthetic predictions do not read its output; d_q may then be NULL).  Every
+ * sub-batch first waits for the work enqueued on `caller`; `caller` does not
+ * wait for the sub-batches (fc_pipeline_join does).  stage_events: NULL, or
+ * [n_parts][4][2] cudaEvent_t (NULL entries skipped) recorded at the start
+ * and end of the retrieval, tree, attention and verification stages.  A
+ * non-OK status from an entry point is returned at once, and the
+ * sub-batches' later launches of this step are not enqueued.
+ */
+#define FC_PIPELINE_NO_ATTENTION 1
+fc_status fc_pipeline_step(fc_pipeline* pl, int phase, int flags, const void* d_q, const void* d_k_tree,
+                           const void* d_v_tree, const int32_t* d_want_hit, const int32_t* d_plen,
+                           const uint32_t* d_rtok, fc_stream caller, void* const* stage_events);
+
+/* The stream that runs sub-batch `part`'s chain (lookup .. append; the
+ * attention runs on a second stream and rejoins it before the predictions),
+ * or NULL for a bad argument.  Work the caller enqueues there runs after
+ * the sub-batch's steps enqueued so far, e.g. reading its results back. */
+fc_stream fc_pipeline_stream(const fc_pipeline* pl, int part);
+
+/* `caller` waits for everything enqueued on the sub-batches' streams. */
+fc_status fc_pipeline_join(fc_pipeline* pl, fc_stream caller);
+
+/* Waits for the executor's streams, then frees its streams and events. */
+void fc_pipeline_destroy(fc_pipeline* pl);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1,0 +1,215 @@
+// Native step executor: one call enqueues a whole decoding step (Section
+// IV-C and IV-D: retrieval -> draft tree -> tree attention -> verification
+// -> cache append) for every sub-batch of a batch, each sub-batch on CUDA
+// streams of its own.
+//
+// The sequences of a batch are independent, so sub-batch h may run step
+// s + 1 while sub-batch h' is still in step s.  Per sub-batch the executor
+// owns two streams: a high-priority one for the latency-bound chain
+// (replay-cache lookup, retrieval, insert, tree build, predictions,
+// acceptance, append) and a low-priority one for the attention launch,
+// ordered by an event pair.  When SMs free up, the block scheduler then
+// starts another sub-batch's chain ahead of this sub-batch's remaining
+// attention CTAs.  The executor holds no device memory: every buffer
+// belongs to the caller, and every launch goes through this library's own
+// entry points.  Issuing a step costs the host one call instead of one call
+// per kernel, so several sub-batches can be kept in flight.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <new>
+#include <vector>
+
+#include "../../include/fastcoder.h"
+#include "fc_common.cuh"
+
+struct fc_pipeline {
+  fc_pipeline_desc d;
+  std::vector<fc_pipeline_part> parts;
+  std::vector<fc_datastore> sources;
+  std::vector<uint32_t> weight;
+  std::vector<cudaStream_t> chain, attn;
+  std::vector<cudaEvent_t> ev_pre, ev_post, ev_done;
+  cudaEvent_t ev_start = nullptr;
+};
+
+namespace {
+
+void destroy_handles(fc_pipeline* pl) {
+  for (cudaStream_t s : pl->chain)
+    if (s) cudaStreamDestroy(s);
+  for (cudaStream_t s : pl->attn)
+    if (s) cudaStreamDestroy(s);
+  for (auto* v : {&pl->ev_pre, &pl->ev_post, &pl->ev_done})
+    for (cudaEvent_t e : *v)
+      if (e) cudaEventDestroy(e);
+  if (pl->ev_start) cudaEventDestroy(pl->ev_start);
+}
+
+bool part_ok(const fc_pipeline_desc& d, const fc_pipeline_part& p) {
+  if (p.batch < 1 || p.first < 0 || p.ctx_stride < 1) return false;
+  const void* need[] = {p.ctx, p.ctx_len[0], p.ctx_len[1], p.kv_len[0], p.kv_len[1], p.root, p.skip, p.drafts,
+                        p.draft_len, p.count, p.n_drafts, p.match_len, p.tok, p.parent, p.depth, p.pos, p.mask,
+                        p.n_nodes, p.k_cache, p.v_cache, p.attn_out, p.argmax, p.acc_len, p.path, p.bonus};
+  for (const void* q : need)
+    if (!q) return false;
+  if (p.ctx_len[0] == p.ctx_len[1] || p.kv_len[0] == p.kv_len[1]) return false;
+  if (p.rcache && p.rcache_capacity < 1) return false;
+  if (d.rope_base > 0.f && !p.k_tree_rot) return false;
+  return true;
+}
+
+// Stage events of part h: [4 stages][start, end]; null entries are skipped.
+void stage_event(void* const* ev, int h, int stage, int end, cudaStream_t s) {
+  if (!ev) return;
+  cudaEvent_t e = static_cast<cudaEvent_t>(ev[h * 8 + stage * 2 + end]);
+  if (e) cudaEventRecord(e, s);
+}
+
+#define FC_TRY(call)                  \
+  do {                                \
+    const fc_status st_ = (call);     \
+    if (st_ != FC_OK) return st_;     \
+  } while (0)
+
+}  // namespace
+
+extern "C" fc_status fc_pipeline_create(const fc_pipeline_desc* d, fc_pipeline** out) {
+  FC_NVTX_RANGE();
+  if (!d || !out) return FC_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (d->n_parts < 1 || !d->parts || d->n_sources < 1 || !d->sources || !d->src_weight) return FC_ERR_INVALID_ARG;
+  if (d->node_budget < 1 || d->n_pad < 1 || d->H < 1 || d->Hkv < 1 || d->D < 1 || d->kv_cap < 1 ||
+      d->path_cap < 1 || d->vocab < 1 || !(d->scale > 0.f) || d->rope_base < 0.f)
+    return FC_ERR_INVALID_ARG;
+  for (int h = 0; h < d->n_parts; ++h)
+    if (!part_ok(*d, d->parts[h])) return FC_ERR_INVALID_ARG;
+  fc_pipeline* pl = new (std::nothrow) fc_pipeline();
+  if (!pl) return FC_ERR_CAPACITY;
+  pl->d = *d;
+  pl->parts.assign(d->parts, d->parts + d->n_parts);
+  pl->sources.assign(d->sources, d->sources + d->n_sources);
+  pl->weight.assign(d->src_weight, d->src_weight + d->n_sources);
+  pl->d.parts = nullptr;  // the copies above are the ones used
+  pl->d.sources = nullptr;
+  pl->d.src_weight = nullptr;
+  int lo = 0, hi = 0;  // least and greatest priority (greatest is the most negative)
+  bool ok = cudaDeviceGetStreamPriorityRange(&lo, &hi) == cudaSuccess;
+  const int p_chain = std::max(hi, -1), p_attn = lo;
+  const int n = d->n_parts;
+  pl->chain.assign(n, nullptr);
+  pl->attn.assign(n, nullptr);
+  pl->ev_pre.assign(n, nullptr);
+  pl->ev_post.assign(n, nullptr);
+  pl->ev_done.assign(n, nullptr);
+  ok = ok && cudaEventCreateWithFlags(&pl->ev_start, cudaEventDisableTiming) == cudaSuccess;
+  for (int h = 0; ok && h < n; ++h) {
+    ok = cudaStreamCreateWithPriority(&pl->chain[h], cudaStreamNonBlocking, p_chain) == cudaSuccess &&
+         cudaStreamCreateWithPriority(&pl->attn[h], cudaStreamNonBlocking, p_attn) == cudaSuccess &&
+         cudaEventCreateWithFlags(&pl->ev_pre[h], cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&pl->ev_post[h], cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&pl->ev_done[h], cudaEventDisableTiming) == cudaSuccess;
+  }
+  if (!ok) {
+    destroy_handles(pl);
+    delete pl;
+    return FC_ERR_CUDA;
+  }
+  *out = pl;
+  return FC_OK;
+}
+
+extern "C" void fc_pipeline_destroy(fc_pipeline* pl) {
+  if (!pl) return;
+  for (cudaStream_t s : pl->chain)
+    if (s) cudaStreamSynchronize(s);
+  for (cudaStream_t s : pl->attn)
+    if (s) cudaStreamSynchronize(s);
+  destroy_handles(pl);
+  delete pl;
+}
+
+extern "C" fc_status fc_pipeline_step(fc_pipeline* pl, int phase, int flags, const void* d_q, const void* d_k_tree,
+                                      const void* d_v_tree, const int32_t* d_want_hit, const int32_t* d_plen,
+                                      const uint32_t* d_rtok, fc_stream caller, void* const* stage_events) {
+  FC_NVTX_RANGE();
+  const bool attention = !(flags & FC_PIPELINE_NO_ATTENTION);
+  if (!pl || (phase != 0 && phase != 1) || (flags & ~FC_PIPELINE_NO_ATTENTION) || (attention && !d_q) || !d_k_tree ||
+      !d_v_tree || !d_plen || !d_rtok)
+    return FC_ERR_INVALID_ARG;
+  const fc_pipeline_desc& d = pl->d;
+  const int c = phase, nx = 1 - phase, S = d.n_sources, Np = d.n_pad;
+  const bool rope = d.rope_base > 0.f;
+  const size_t q_row = (size_t)Np * d.H * d.D * 2, kt_row = (size_t)d.Hkv * Np * d.D * 2;  // bytes per sequence
+  if (cudaEventRecord(pl->ev_start, static_cast<cudaStream_t>(caller)) != cudaSuccess) return FC_ERR_CUDA;
+  for (int h = 0; h < d.n_parts; ++h) {
+    const fc_pipeline_part& P = pl->parts[h];
+    cudaStream_t s = pl->chain[h], sa = pl->attn[h];
+    const int B = P.batch;
+    if (cudaStreamWaitEvent(s, pl->ev_start, 0) != cudaSuccess) return FC_ERR_CUDA;
+    const void* q = attention ? static_cast<const char*>(d_q) + (size_t)P.first * q_row : nullptr;
+    const void* kt = static_cast<const char*>(d_k_tree) + (size_t)P.first * kt_row;
+    const void* vt = static_cast<const char*>(d_v_tree) + (size_t)P.first * kt_row;
+    const int32_t* want = d_want_hit ? d_want_hit + P.first : nullptr;
+
+    stage_event(stage_events, h, 0, 0, s);
+    if (P.rcache)
+      FC_TRY(fc_rcache_lookup(P.rcache, P.rcache_capacity, S, d.p, P.ctx, P.ctx_stride, P.ctx_len[c], B, want,
+                              P.skip, P.drafts, P.draft_len, P.count, P.n_drafts, P.match_len, s));
+    FC_TRY(fc_retrieve(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.rcache ? P.skip : nullptr,
+                       d.p, P.drafts, P.draft_len, P.count, P.n_drafts, P.match_len, s));
+    if (P.rcache)
+      FC_TRY(fc_rcache_insert(P.rcache, P.rcache_capacity, S, d.p, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.skip,
+                              P.drafts, P.draft_len, P.count, P.n_drafts, P.match_len, s));
+    stage_event(stage_events, h, 0, 1, s);
+    stage_event(stage_events, h, 1, 0, s);
+    FC_TRY(fc_build_tree(S, P.drafts, P.draft_len, P.count, P.n_drafts, pl->weight.data(), d.p.top_k,
+                         d.p.draft_len, P.root, P.kv_len[c], B, d.node_budget, Np, P.tok, P.parent, P.depth, P.pos,
+                         P.mask, P.n_nodes, s));
+    stage_event(stage_events, h, 1, 1, s);
+    if (rope) {
+      FC_TRY(fc_rope(kt, P.k_tree_rot, B, Np, d.Hkv, d.D, 1, P.pos, d.rope_base, s));
+      kt = P.k_tree_rot;
+    }
+    if (attention) {  // on its own stream, ordered by an event pair
+      if (cudaEventRecord(pl->ev_pre[h], s) != cudaSuccess || cudaStreamWaitEvent(sa, pl->ev_pre[h], 0) != cudaSuccess)
+        return FC_ERR_CUDA;
+      stage_event(stage_events, h, 2, 0, sa);
+      if (rope)
+        FC_TRY(fc_tree_attn_rope(q, P.k_cache, P.v_cache, d.kv_cap, P.kv_len[c], kt, vt, P.mask, P.n_nodes, B, Np,
+                                 d.H, d.Hkv, d.D, d.scale, P.pos, d.rope_base, P.attn_out, P.attn_ws,
+                                 P.attn_ws_bytes, sa));
+      else
+        FC_TRY(fc_tree_attn(q, P.k_cache, P.v_cache, d.kv_cap, P.kv_len[c], kt, vt, P.mask, P.n_nodes, B, Np, d.H,
+                            d.Hkv, d.D, d.scale, P.attn_out, P.attn_ws, P.attn_ws_bytes, sa));
+      stage_event(stage_events, h, 2, 1, sa);
+      if (cudaEventRecord(pl->ev_post[h], sa) != cudaSuccess ||
+          cudaStreamWaitEvent(s, pl->ev_post[h], 0) != cudaSuccess)
+        return FC_ERR_CUDA;
+    }
+    stage_event(stage_events, h, 3, 0, s);
+    FC_TRY(fc_synth_argmax(P.tok, P.parent, P.n_nodes, B, Np, d_plen + P.first, d_rtok + (size_t)P.first * Np,
+                           d.vocab, P.argmax, s));
+    FC_TRY(fc_accept(P.tok, P.parent, P.n_nodes, P.argmax, B, Np, P.acc_len, P.path, d.path_cap, P.bonus, s));
+    FC_TRY(fc_kv_append(P.path, P.acc_len, P.bonus, P.tok, kt, vt, B, Np, d.Hkv, d.D, d.path_cap, P.k_cache,
+                        P.v_cache, d.kv_cap, P.kv_len[c], P.kv_len[nx], P.ctx, P.ctx_stride, P.ctx_len[c],
+                        P.ctx_len[nx], P.root, s));
+    stage_event(stage_events, h, 3, 1, s);
+  }
+  return FC_OK;
+}
+
+extern "C" fc_stream fc_pipeline_stream(const fc_pipeline* pl, int part) {
+  if (!pl || part < 0 || part >= (int)pl->chain.size()) return nullptr;
+  return pl->chain[part];
+}
+
+extern "C" fc_status fc_pipeline_join(fc_pipeline* pl, fc_stream caller) {
+  if (!pl) return FC_ERR_INVALID_ARG;
+  cudaStream_t cs = static_cast<cudaStream_t>(caller);
+  for (size_t h = 0; h < pl->chain.size(); ++h)
+    if (cudaEventRecord(pl->ev_done[h], pl->chain[h]) != cudaSuccess ||
+        cudaStreamWaitEvent(cs, pl->ev_done[h], 0) != cudaSuccess)
+      return FC_ERR_CUDA;
+  return FC_OK;
+}

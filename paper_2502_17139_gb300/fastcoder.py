@@ -11,8 +11,10 @@ uint64 mask words in int64 tensors, bf16 tensors as torch.bfloat16.
 """
 from __future__ import annotations
 
+import atexit
 import ctypes as C
 import os
+import weakref
 
 import numpy as np
 import torch
@@ -50,12 +52,33 @@ class fc_cache(C.Structure):
                 ("chunk", C.c_int32), ("ctx_keep", C.c_int32)]
 
 
+class fc_pipeline_part(C.Structure):
+    _fields_ = [("batch", C.c_int32), ("first", C.c_int32), ("ctx", C.c_void_p), ("ctx_stride", C.c_int32),
+                ("ctx_len", C.c_void_p * 2), ("kv_len", C.c_void_p * 2), ("root", C.c_void_p),
+                ("rcache", C.c_void_p), ("rcache_capacity", C.c_int32), ("skip", C.c_void_p),
+                ("drafts", C.c_void_p), ("draft_len", C.c_void_p), ("count", C.c_void_p), ("n_drafts", C.c_void_p),
+                ("match_len", C.c_void_p), ("tok", C.c_void_p), ("parent", C.c_void_p), ("depth", C.c_void_p),
+                ("pos", C.c_void_p), ("mask", C.c_void_p), ("n_nodes", C.c_void_p), ("k_cache", C.c_void_p),
+                ("v_cache", C.c_void_p), ("k_tree_rot", C.c_void_p), ("attn_out", C.c_void_p),
+                ("attn_ws", C.c_void_p), ("attn_ws_bytes", C.c_size_t), ("argmax", C.c_void_p),
+                ("acc_len", C.c_void_p), ("path", C.c_void_p), ("bonus", C.c_void_p)]
+
+
+class fc_pipeline_desc(C.Structure):
+    _fields_ = [("sources", C.POINTER(fc_datastore)), ("n_sources", C.c_int32), ("p", fc_retrieve_params),
+                ("src_weight", C.POINTER(C.c_uint32)), ("node_budget", C.c_int32), ("n_pad", C.c_int32),
+                ("H", C.c_int32), ("Hkv", C.c_int32), ("D", C.c_int32), ("kv_cap", C.c_int32),
+                ("path_cap", C.c_int32), ("vocab", C.c_uint32), ("scale", C.c_float), ("rope_base", C.c_float),
+                ("n_parts", C.c_int32), ("parts", C.POINTER(fc_pipeline_part))]
+
+
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
            "fc_datastore_build_noalloc", "fc_datastore_keys", "fc_datastore_save", "fc_datastore_file_info", "fc_datastore_load",
            "fc_retrieve", "fc_retrieve_all", "fc_retrieve_rev", "fc_reverse_tokens", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
            "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_gemm_kv_heads", "fc_gemm_silu_mul", "fc_interleave_gate_up", "fc_embed",
-           "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax"]
+           "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax",
+           "fc_pipeline_create", "fc_pipeline_step", "fc_pipeline_stream", "fc_pipeline_join", "fc_pipeline_destroy"]
 
 
 def _load():
@@ -124,6 +147,11 @@ def _load():
         "fc_kv_append": (C.c_int, [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, i32,
                                    vp, vp, vp, vp]),
         "fc_synth_argmax": (C.c_int, [vp, vp, vp, i32, i32, vp, vp, u32, vp, vp]),
+        "fc_pipeline_create": (C.c_int, [C.POINTER(fc_pipeline_desc), C.POINTER(vp)]),
+        "fc_pipeline_step": (C.c_int, [vp, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]),
+        "fc_pipeline_join": (C.c_int, [vp, vp]),
+        "fc_pipeline_stream": (vp, [vp, i32]),
+        "fc_pipeline_destroy": (None, [vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -767,3 +795,107 @@ def fc_synth_argmax(tok, parent, n_nodes, plen, rtok, vocab, out=None):
     _check("fc_synth_argmax", LIB.fc_synth_argmax(_ptr(tok), _ptr(parent), _ptr(n_nodes), B, Np, _ptr(plen),
                                                   _ptr(rtok), vocab, _ptr(o), _stream()))
     return o
+
+
+# ------------------------------------------------------ native step executor
+PIPELINE_NO_ATTENTION = 1
+_PIPELINES = weakref.WeakSet()
+
+
+@atexit.register
+def _close_pipelines():
+    # before the CUDA runtime shuts down: destroying streams later is unsafe
+    for pl in list(_PIPELINES):
+        pl.close()
+
+
+def pipeline_part(batch, first, ctx, ctx_len, kv_len, root, rcache, skip, res, tree, k_cache, v_cache, k_tree_rot,
+                  attn_out, attn_ws, argmax, acc) -> fc_pipeline_part:
+    """One sub-batch's buffers (device tensors the caller keeps alive):
+    ctx_len and kv_len are pairs (the ping-pong lengths), rcache a
+    RetrievalCache or None, res/tree/acc the dicts of retrieve_outputs,
+    tree_outputs and fc_accept's outputs."""
+    _need(ctx, torch.int32, "ctx", (batch, ctx.shape[1]))
+    for t in (*ctx_len, *kv_len, root, skip):
+        _need(t, torch.int32, "length", (batch,))
+    _need(k_cache, torch.bfloat16, "k_cache")
+    _need(v_cache, torch.bfloat16, "v_cache", tuple(k_cache.shape))
+    return fc_pipeline_part(
+        batch, first, _ptr(ctx), ctx.shape[1], (C.c_void_p * 2)(*[t.data_ptr() for t in ctx_len]),
+        (C.c_void_p * 2)(*[t.data_ptr() for t in kv_len]), _ptr(root), _ptr(rcache.table) if rcache else None,
+        rcache.capacity if rcache else 0, _ptr(skip), _ptr(res["drafts"]), _ptr(res["draft_len"]), _ptr(res["count"]),
+        _ptr(res["n_drafts"]), _ptr(res["match_len"]), _ptr(tree["tok"]), _ptr(tree["parent"]), _ptr(tree["depth"]),
+        _ptr(tree["pos"]), _ptr(tree["mask"]), _ptr(tree["n_nodes"]), _ptr(k_cache), _ptr(v_cache), _ptr(k_tree_rot),
+        _ptr(attn_out), _ptr(attn_ws), 0 if attn_ws is None else attn_ws.numel() * attn_ws.element_size(),
+        _ptr(argmax), _ptr(acc["acc_len"]), _ptr(acc["path"]), _ptr(acc["bonus"]))
+
+
+class Pipeline:
+    """fc_pipeline: the native step executor over sub-batches.  ``parts`` are
+    pipeline_part() descriptions; their tensors must outlive this object."""
+
+    def __init__(self, sources, p: fc_retrieve_params, src_weight, node_budget, n_pad, H, Hkv, D, kv_cap, path_cap,
+                 vocab, parts, scale=None, rope_base=None):
+        S = len(sources)
+        if len(src_weight) != S:
+            raise ValueError("one tree weight per source")
+        self.B = sum(pt.batch for pt in parts)
+        self.shapes = ((self.B, n_pad, H, D), (self.B, Hkv, n_pad, D), (self.B,), (self.B, n_pad))
+        views = (fc_datastore * S)(*[s.view for s in sources])
+        w = (C.c_uint32 * S)(*[int(x) for x in src_weight])
+        arr = (fc_pipeline_part * len(parts))(*parts)
+        desc = fc_pipeline_desc(views, S, p, w, node_budget, n_pad, H, Hkv, D, kv_cap, path_cap, vocab,
+                                float(scale) if scale is not None else D ** -0.5,
+                                0.0 if rope_base is None else float(rope_base), len(parts), arr)
+        h = C.c_void_p()
+        _check("fc_pipeline_create", LIB.fc_pipeline_create(C.byref(desc), C.byref(h)))
+        self.handle = h
+        self.n_parts = len(parts)
+        self._destroy = LIB.fc_pipeline_destroy
+        # each sub-batch's chain stream, for work that must follow its steps
+        self.streams = [torch.cuda.ExternalStream(LIB.fc_pipeline_stream(h, i)) for i in range(len(parts))]
+        _PIPELINES.add(self)
+
+    def step(self, phase, q, k_tree, v_tree, want_hit, plen, rtok, attention=True, events=None):
+        """Enqueue one step of every sub-batch after the work on the current
+        stream (inputs batch-wide, as fc_pipeline_step); ``events``: None or,
+        per sub-batch, a dict mapping "retrieve" / "tree" / "attn" / "tail" to
+        a (start, end) pair of torch.cuda.Event."""
+        qs, ks, bs, rs = self.shapes
+        if attention:
+            _need(q, torch.bfloat16, "q", qs)
+        _need(k_tree, torch.bfloat16, "k_tree", ks)
+        _need(v_tree, torch.bfloat16, "v_tree", ks)
+        _need(plen, torch.int32, "plen", bs)
+        _need(rtok, torch.int32, "rtok", rs)
+        if want_hit is not None:
+            _need(want_hit, torch.int32, "want_hit", bs)
+        ev = None
+        if events is not None:
+            ev = (C.c_void_p * (8 * self.n_parts))()
+            for h, e in enumerate(events):
+                for j, nm in enumerate(("retrieve", "tree", "attn", "tail")):
+                    for k in range(2):
+                        if e and nm in e:
+                            t = e[nm][k]
+                            if not t.cuda_event:  # torch creates its events at the first record
+                                t.record()
+                            ev[8 * h + 2 * j + k] = t.cuda_event
+        _check("fc_pipeline_step", LIB.fc_pipeline_step(
+            self.handle, phase, 0 if attention else PIPELINE_NO_ATTENTION, _ptr(q) if attention else None,
+            _ptr(k_tree), _ptr(v_tree), _ptr(want_hit), _ptr(plen), _ptr(rtok), _stream(), ev))
+
+    def join(self):
+        """The current stream waits for everything enqueued on the sub-batches."""
+        _check("fc_pipeline_join", LIB.fc_pipeline_join(self.handle, _stream()))
+
+    def close(self):
+        if getattr(self, "handle", None):
+            self._destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

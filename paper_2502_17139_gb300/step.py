@@ -19,7 +19,8 @@ Every call is asynchronous on the current stream and allocates nothing, so
 steps can be captured once into a CUDA graph and replayed (lengths ping-pong
 between two buffers, so a graph holds an even number of consecutive steps).
 PipelinedStepLoop runs the step over sub-batches of the sequences on streams
-of their own.
+of their own, through the native step executor (fc_pipeline_step): one C call
+enqueues every sub-batch's kernels.
 """
 from __future__ import annotations
 
@@ -248,24 +249,26 @@ def sub_batch_slices(B, n_split):
 
 
 class PipelinedStepLoop:
-    """The step loop over sub-batches of the sequences, each on its own CUDA
-    stream.
+    """The step loop over sub-batches of the sequences, each on CUDA streams
+    of its own, issued by the native step executor (fc_pipeline).
 
     The sequences of a batch are independent, so sub-batch h can run step
     s + 1 while sub-batch h' is still in step s. Then one sub-batch's small,
     latency-bound kernels (retrieval, tree build, acceptance, append) run on
     the SMs that the other's attention launch leaves idle in its last wave;
     an SM that holds an attention CTA has no room for any other CTA.  Each
-    sub-batch is a StepLoop over a slice of the sequences.  They share the
-    datastores and slices of one pair of KV caches, and every per-sequence
-    result is the single loop's.  The replay cache is per sub-batch; it
-    replays deterministic retrieval results, so that changes no output.
+    sub-batch owns the buffers of a StepLoop over a slice of the sequences.
+    They share the datastores and slices of one pair of KV caches, and every
+    per-sequence result is the single loop's.  The replay cache is per
+    sub-batch; it replays deterministic retrieval results, so that changes no
+    output.  One fc_pipeline_step call enqueues a step of every sub-batch:
+    the host cost of a step no longer grows by a Python call per kernel.
 
-    step() makes every sub-batch stream wait for the work already enqueued
-    on the caller's stream, so inputs written there are visible.  It does not
-    make the caller's stream wait for the sub-batches, or they could not
-    overlap; join() does that, and must precede any read of the results on
-    the caller's stream.  Only the replay-cache configuration (with optional
+    step() makes every sub-batch wait for the work already enqueued on the
+    caller's stream, so inputs written there are visible.  It does not make
+    the caller's stream wait for the sub-batches, or they could not overlap;
+    join() does that, and must precede any read of the results on the
+    caller's stream.  Only the replay-cache configuration (with optional
     RoPE) is pipelined; Algorithm 1's missing table is shared by the whole
     batch, so it stays with StepLoop."""
 
@@ -278,38 +281,32 @@ class PipelinedStepLoop:
         self.k_cache = k_cache if k_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         self.v_cache = v_cache if v_cache is not None else torch.zeros(shape, dtype=torch.bfloat16, device=device)
         kv0 = np.broadcast_to(np.asarray(kv_len0, np.int32), (B,))
+        # the StepLoops hold each sub-batch's buffers and initial state
         self.loops = [StepLoop(sources, ctx[sl], ctx_len[sl], p, node_budget, n_pad, src_weight, H, Hkv, D, kv_cap,
                                kv0[sl], vocab, cache_capacity=cache_capacity, device=device,
                                k_cache=self.k_cache[sl], v_cache=self.v_cache[sl], rope_base=rope_base)
                       for sl in self.slices]
-        # Each sub-batch's small kernels run on a high-priority stream and its
-        # attention on a low-priority one: when SMs free up, the block scheduler
-        # then starts the other sub-batch's latency-bound chain (retrieval, tree,
-        # acceptance) ahead of this sub-batch's remaining attention CTAs.
-        self.streams = [torch.cuda.Stream(device=device, priority=-1) for _ in self.slices]
-        for lp in self.loops:
-            lp.attn_stream = torch.cuda.Stream(device=device, priority=0)
-        self._start = torch.cuda.Event()
-        self._done = [torch.cuda.Event() for _ in self.slices]
+        parts = [fc.pipeline_part(sl.stop - sl.start, sl.start, lp.ctx, lp.ctx_len, lp.kv_len, lp.root, lp.cache,
+                                  lp.skip, lp.res, lp.tree, lp.k_cache, lp.v_cache, lp.k_tree_rot, lp.attn_out,
+                                  lp.attn_ws, lp.argmax, lp.acc)
+                 for lp, sl in zip(self.loops, self.slices)]
+        lp0 = self.loops[0]
+        self.pipe = fc.Pipeline(sources, p, lp0.tree_weight, node_budget, n_pad, H, Hkv, D, kv_cap, lp0.path_cap,
+                                vocab, parts, rope_base=rope_base)
+        self.streams = self.pipe.streams  # each sub-batch's chain stream (lookup .. append)
 
     def step(self, q, k_tree, v_tree, want_hit, plen, rtok, attention=True, events=None):
         """Enqueue one step of every sub-batch (arguments as StepLoop.step,
         for the whole batch); ``events``: None or one StepLoop events dict per
-        sub-batch, recorded on its stream."""
-        self._start.record()
-        cut = lambda t, sl: None if t is None else t[sl]
-        for h, (lp, sl, st) in enumerate(zip(self.loops, self.slices, self.streams)):
-            st.wait_event(self._start)
-            with torch.cuda.stream(st):
-                lp.step(cut(q, sl), cut(k_tree, sl), cut(v_tree, sl), want_hit[sl], plen[sl], rtok[sl],
-                        attention=attention, events=None if events is None else events[h])
+        sub-batch, recorded on its streams."""
+        self.pipe.step(self.loops[0].cur, q, k_tree, v_tree, want_hit, plen, rtok, attention=attention,
+                       events=events)
+        for lp in self.loops:
+            lp.cur = 1 - lp.cur
 
     def join(self):
         """The caller's current stream waits for everything enqueued so far."""
-        cur = torch.cuda.current_stream()
-        for ev, st in zip(self._done, self.streams):
-            ev.record(st)
-            cur.wait_event(ev)
+        self.pipe.join()
 
     def capture(self, inputs, attention=True):
         """An even number of steps of every sub-batch in one CUDA graph (fork

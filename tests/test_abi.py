@@ -183,3 +183,44 @@ def test_trie_all_validation_without_gpu(lib):
     assert L.fc_build_tree_all(3, *args, 256, 1 << 40, *outs) == 2       # too many drafts: FC_ERR_UNSUPPORTED
     assert L.fc_build_tree_all(2, *args[:10], 128, 96, 256, 1 << 40, *outs) == 2  # n_pad 96
     assert L.fc_build_tree_all(2, *args[:10], 0, 128, 256, 1 << 40, *outs) == 1   # budget 0
+
+
+def test_pipeline_host_validation(lib):
+    """The native step executor rejects bad descriptions before it creates
+    any stream (nothing here touches a GPU)."""
+    import paper_2502_17139_gb300.fastcoder as fc
+    L = fc.LIB
+    h = C.c_void_p()
+    assert L.fc_pipeline_create(None, C.byref(h)) == 1 and not h.value
+    views = (fc.fc_datastore * 1)(fc.fc_datastore(16, 16, 16, 16, 10, 5))
+    w = (C.c_uint32 * 1)(1)
+    buf = [16 * (i + 1) for i in range(40)]
+    part = fc.fc_pipeline_part(4, 0, buf[0], 64, (C.c_void_p * 2)(buf[1], buf[2]), (C.c_void_p * 2)(buf[3], buf[4]),
+                               buf[5], None, 0, buf[6], buf[7], buf[8], buf[9], buf[10], buf[11], buf[12], buf[13],
+                               buf[14], buf[15], buf[16], buf[17], buf[18], buf[19], None, buf[20], None, 0, buf[21],
+                               buf[22], buf[23], buf[24])
+
+    def desc(parts, n_parts=None, **kw):
+        d = dict(node_budget=64, n_pad=128, H=32, Hkv=8, D=128, kv_cap=1024, path_cap=10, vocab=1000, scale=0.1,
+                 rope_base=0.0)
+        d.update(kw)
+        arr = (fc.fc_pipeline_part * max(1, len(parts)))(*parts)
+        return fc.fc_pipeline_desc(views, 1, fc.params(16, 2, 16, 8), w, d["node_budget"], d["n_pad"], d["H"],
+                                   d["Hkv"], d["D"], d["kv_cap"], d["path_cap"], d["vocab"], d["scale"],
+                                   d["rope_base"], len(parts) if n_parts is None else n_parts, arr)
+
+    assert L.fc_pipeline_create(C.byref(desc([part], n_parts=0)), C.byref(h)) == 1
+    assert L.fc_pipeline_create(C.byref(desc([part], scale=0.0)), C.byref(h)) == 1
+    assert L.fc_pipeline_create(C.byref(desc([part], rope_base=1e4)), C.byref(h)) == 1  # RoPE needs k_tree_rot
+    same = fc.fc_pipeline_part.from_buffer_copy(part)
+    same.kv_len[1] = same.kv_len[0]  # the ping-pong buffers must differ
+    assert L.fc_pipeline_create(C.byref(desc([same])), C.byref(h)) == 1
+    missing = fc.fc_pipeline_part.from_buffer_copy(part)
+    missing.mask = None
+    assert L.fc_pipeline_create(C.byref(desc([missing])), C.byref(h)) == 1
+    assert not h.value
+    nul = None
+    assert L.fc_pipeline_step(nul, 0, 0, 16, 16, 16, nul, 16, 16, nul, nul) == 1
+    assert L.fc_pipeline_join(nul, nul) == 1
+    assert L.fc_pipeline_stream(nul, 0) is None
+    L.fc_pipeline_destroy(nul)

@@ -170,3 +170,62 @@ def test_pipelined_kv_split_workspaces(fc):
         piped.join()
         same(state(single), state(piped))
     assert fc.fc_get_error() == "FC_OK"
+
+
+def test_pipelined_rope_matches_single_loop(fc, setup):
+    """The executor's RoPE path (tree keys rotated by fc_rope, queries inside
+    the attention kernel) against the single loop's."""
+    from paper_2502_17139_gb300.step import PipelinedStepLoop, StepLoop
+    single = StepLoop(*setup["args"], **setup["kw"], rope_base=10000.0)
+    piped = PipelinedStepLoop(2, *setup["args"], **setup["kw"], rope_base=10000.0)
+    for s in range(4):
+        single.step(*setup["ins"][s])
+        piped.step(*setup["ins"][s])
+        piped.join()
+        same(state(single), state(piped))
+    assert fc.fc_get_error() == "FC_OK"
+
+
+def test_pipelined_without_attention(fc, setup):
+    """A step without the attention launch follows the same trajectory (the
+    synthetic predictions do not read the attention output) and leaves the
+    output untouched."""
+    from paper_2502_17139_gb300.step import PipelinedStepLoop
+    full = PipelinedStepLoop(3, *setup["args"], **setup["kw"])
+    bare = PipelinedStepLoop(3, *setup["args"], **setup["kw"])
+    for lp in bare.loops:
+        lp.attn_out.fill_(float("nan"))
+    for s in range(4):
+        full.step(*setup["ins"][s])
+        q, kt, vt, h, p, r = setup["ins"][s]
+        bare.step(None, kt, vt, h, p, r, attention=False)
+    full.join()
+    bare.join()
+    a, b = state(full), state(bare)
+    assert torch.isnan(b.pop("attn")).all()
+    a.pop("attn")
+    same(a, b)
+
+
+def test_pipelined_stage_events_and_streams(fc, setup):
+    """Stage events land in order on each sub-batch's streams, and work the
+    caller enqueues on a sub-batch's exposed stream follows its step."""
+    from paper_2502_17139_gb300.step import PipelinedStepLoop
+    piped = PipelinedStepLoop(2, *setup["args"], **setup["kw"])
+    mk = lambda: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    evs = [dict(retrieve=mk(), tree=mk(), attn=mk(), tail=mk()) for _ in piped.loops]
+    piped.step(*setup["ins"][0], events=evs)
+    outs = []
+    for lp, st in zip(piped.loops, piped.streams):
+        with torch.cuda.stream(st):
+            outs.append(lp.acc["acc_len"].clone())
+    piped.join()
+    torch.cuda.synchronize()
+    for e in evs:
+        t = {k: a.elapsed_time(b) for k, (a, b) in e.items()}
+        assert all(v >= 0 for v in t.values()), t
+        assert e["retrieve"][1].elapsed_time(e["tree"][0]) >= 0
+        assert e["tree"][1].elapsed_time(e["attn"][0]) >= 0
+        assert e["attn"][1].elapsed_time(e["tail"][0]) >= 0
+    for lp, o in zip(piped.loops, outs):
+        assert torch.equal(o, lp.acc["acc_len"])
