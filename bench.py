@@ -134,6 +134,14 @@ def attn_traffic(args, algorithmic_bytes_per_launch):
     return ATTN_TRAFFIC["ratio"] * algorithmic_bytes_per_launch
 
 
+def step_status(fc, loop):
+    """The device errors of a step loop: fc_get_error() and, for the pipelined
+    loop, every sub-batch's own error word (the most severe first found)."""
+    sts = [fc.fc_get_error()] + (loop.errors() if hasattr(loop, "errors") else [])
+    bad = [x for x in sts if x != "FC_OK"]
+    return bad[0] if bad else "FC_OK"
+
+
 @contextlib.contextmanager
 def no_gc():
     """The Python garbage collector off inside a timed region: a collection
@@ -369,7 +377,7 @@ def run_ours(args, rank, ws, local):
     for s in range(W):
         do_step(s)
     join(loop)
-    assert fc.fc_get_error() == "FC_OK"
+    assert step_status(fc, loop) == "FC_OK"
     barrier(ws)
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
@@ -385,14 +393,14 @@ def run_ours(args, rank, ws, local):
     clock_rec = clocks.stop()
     barrier(ws)
     t_ms = start.elapsed_time(end)
-    status = fc.fc_get_error()
+    status = step_status(fc, loop)
     assert status == "FC_OK", status
     t_max = max_over_ranks(t_ms, ws)
     graph_rec = None
     if not args.no_graph:
         try:
             graph_rec = run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W, K)
-            assert fc.fc_get_error() == "FC_OK"
+            assert step_status(fc, loop) == "FC_OK"
         except Exception as e:  # reported, not fatal: the eager line stands
             graph_rec = {"error": f"{type(e).__name__}: {e}"[:200]}
     stage_ms = {k: [[a.elapsed_time(b) for a, b in (stage_ev[i][h][k] for h in range(nsub))] for i in range(K)]
@@ -693,6 +701,9 @@ def run_e2e(loop, inp, dev, W, K, P, q_pool, kt_pool, vt_pool, ws):
         run(W, K)
         torch.cuda.synchronize()
         t1 = time.perf_counter()
+    import paper_2502_17139_gb300.fastcoder as fc
+    status = step_status(fc, loop)
+    assert status == "FC_OK", status
     t = max_over_ranks(t1 - t0, ws)
     d = sets[0]
     h2d = d["q"].numel() * 2 + d["k"].numel() * 2 + d["v"].numel() * 2 + 4 * (2 * B + d["r"].numel())

@@ -74,7 +74,9 @@ const char* fc_version(void);
  * Synchronous.  The word is shared by every stream of the process: with
  * work on several streams, have s wait for them first (or synchronize the
  * device), or an error recorded later on another stream is missed by this
- * call and reported by the next.
+ * call and reported by the next.  The native step executor can give each
+ * sub-batch a word of its own instead (fc_pipeline_part.err, read by
+ * fc_pipeline_error), so that its errors are attributed to it exactly.
  */
 fc_status fc_get_error(fc_stream s);
 
@@ -731,6 +733,9 @@ typedef struct {
   int32_t* acc_len;         /* [batch] */
   int32_t* path;            /* [batch][path_cap] */
   uint32_t* bonus;          /* [batch] */
+  uint32_t* err;            /* this sub-batch's device error word (4 bytes, zeroed by the
+                               caller; fc_pipeline_error reads it), or NULL: its kernels
+                               then record errors in the library-wide words of fc_get_error */
 } fc_pipeline_part;
 
 typedef struct {
@@ -775,6 +780,14 @@ fc_status fc_pipeline_create(const fc_pipeline_desc* desc, fc_pipeline** out);
 fc_status fc_pipeline_step(fc_pipeline* pl, int phase, int flags, const void* d_q, const void* d_k_tree,
                            const void* d_v_tree, const int32_t* d_want_hit, const int32_t* d_plen,
                            const uint32_t* d_rtok, fc_stream caller, void* const* stage_events);
+
+/* Waits for sub-batch `part`'s work enqueued so far, then returns and clears
+ * its error word: the most severe device-detected error its kernels recorded
+ * (FC_OK if none).  With a word per sub-batch an error is reported for the
+ * sub-batch that raised it, whatever the other sub-batches' streams do.
+ * FC_ERR_INVALID_ARG if the sub-batch was created without a word.
+ * Synchronous. */
+fc_status fc_pipeline_error(fc_pipeline* pl, int part);
 
 /* The stream that runs sub-batch `part`'s chain (lookup .. append; the
  * attention runs on a second stream and rejoins it before the predictions),

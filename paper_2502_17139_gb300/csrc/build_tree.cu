@@ -45,6 +45,7 @@ struct TreeOut {
   int32_t* pos;
   uint64_t* mask;
   int32_t* n_nodes;
+  unsigned int* err;  // the launch's error word (NULL: this file's own)
 };
 
 struct BtLayout {
@@ -275,7 +276,7 @@ __global__ void __launch_bounds__(BT_THREADS) k_build_tree(TreeIn in, int S, int
     len[j] = l;
     uint32_t cnt = in.count[sb * k + t];
     if (cnt > (1u << 20)) {  // weights are packed into 46-bit sort keys
-      fc_flag(&g_fc_err, FC_EBIT_INVALID);
+      fc_flag(FC_ERR_WORD(out.err), FC_EBIT_INVALID);
       cnt = 1u << 20;
     }
     w[j] = (uint64_t)in.w[s] * cnt;
@@ -393,7 +394,7 @@ __global__ void __launch_bounds__(BT_THREADS) k_build_tree(TreeIn in, int S, int
   }
   __syncthreads();
   const uint32_t nkept = block_scan_array(tab, (int)(U * (uint32_t)d), wsum);
-  if (nkept != (uint32_t)nsel && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INTERNAL);
+  if (nkept != (uint32_t)nsel && tid == 0) fc_flag(FC_ERR_WORD(out.err), FC_EBIT_INTERNAL);
   for (uint32_t c = tid; c < C; c += BT_THREADS) {
     const uint64_t key = ckey[c];
     if (nsel > 0 && key >= thr) {
@@ -563,7 +564,7 @@ __global__ void __launch_bounds__(BT_THREADS, 1) k_build_tree_all(TreeIn in, int
     len[j] = l;
     uint32_t cnt = in.count[sb * k + t];
     if (cnt > (1u << 17)) {  // weights are packed into 46-bit selection keys
-      fc_flag(&g_fc_err, FC_EBIT_INVALID);
+      fc_flag(FC_ERR_WORD(out.err), FC_EBIT_INVALID);
       cnt = 1u << 17;
     }
     w[j] = (uint64_t)in.w[s] * cnt;
@@ -592,7 +593,7 @@ __global__ void __launch_bounds__(BT_THREADS, 1) k_build_tree_all(TreeIn in, int
   const int nw = n_pad / 64;
   const size_t obase = (size_t)b * n_pad;
   if (s_bad) {  // reject the query: a root-only tree
-    if (tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+    if (tid == 0) fc_flag(FC_ERR_WORD(out.err), FC_EBIT_INVALID);
     for (int i = tid; i < n_pad; i += BT_THREADS) {
       out.tok[obase + i] = (i == 0) ? root_tok[b] : FC_PAD_TOKEN;
       out.parent[obase + i] = -1;
@@ -702,7 +703,7 @@ __global__ void __launch_bounds__(BT_THREADS, 1) k_build_tree_all(TreeIn in, int
   }
   __syncthreads();
   const uint32_t nkept = block_scan_array(tab, (int)(U * (uint32_t)d), wsum);
-  if (nkept != (uint32_t)nsel && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INTERNAL);
+  if (nkept != (uint32_t)nsel && tid == 0) fc_flag(FC_ERR_WORD(out.err), FC_EBIT_INTERNAL);
   for (uint32_t c = tid; c < C; c += BT_THREADS) {
     const uint64_t key = ckey[c];
     if (nsel > 0 && key >= thr) {
@@ -746,7 +747,7 @@ __global__ void __launch_bounds__(BT_THREADS, 1) k_build_tree_all(TreeIn in, int
 // Mask, depth, position ids from parent pointers: one warp per tree.
 __global__ void k_tree_mask(const int32_t* __restrict__ parent, const int32_t* __restrict__ n_nodes,
                             const int32_t* __restrict__ kv_len, int B, int n_pad, int32_t* __restrict__ depth,
-                            int32_t* __restrict__ pos, uint64_t* __restrict__ mask) {
+                            int32_t* __restrict__ pos, uint64_t* __restrict__ mask, unsigned int* err) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (warp >= B) return;
   const int b = warp, nw = n_pad / 64;
@@ -756,7 +757,7 @@ __global__ void k_tree_mask(const int32_t* __restrict__ parent, const int32_t* _
   for (int i = lane; i < n_pad && !bad; i += 32)
     if (i < n && i > 0 && (parent[base + i] < 0 || parent[base + i] >= i)) bad = true;
   bad = __any_sync(0xFFFFFFFFu, bad);
-  if (bad && lane == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+  if (bad && lane == 0) fc_flag(FC_ERR_WORD(err), FC_EBIT_INVALID);
   for (int i = lane; i < n_pad; i += 32) {
     uint64_t m0 = 0, m1 = 0;
     int de = -1, po = -1;
@@ -799,7 +800,7 @@ extern "C" fc_status fc_build_tree(int n_sources, const uint32_t* d_drafts, cons
     return FC_ERR_INVALID_ARG;
   TreeIn in{d_drafts, d_draft_len, d_count, d_n_drafts, {0, 0, 0, 0}};
   for (int s = 0; s < n_sources; ++s) in.w[s] = src_weight[s];
-  TreeOut out{d_tok, d_parent, d_depth, d_pos, d_mask, d_n_nodes};
+  TreeOut out{d_tok, d_parent, d_depth, d_pos, d_mask, d_n_nodes, fc_error_slot()};
   const size_t smem = bt_layout(n_sources * top_k, draft_len).total;
   if (cudaFuncSetAttribute(k_build_tree, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return FC_ERR_CUDA;
@@ -819,7 +820,7 @@ extern "C" fc_status fc_tree_mask(const int32_t* d_parent, const int32_t* d_n_no
   const int threads = 128;
   const unsigned blocks = (unsigned)((batch * 32 + threads - 1) / threads);
   k_tree_mask<<<blocks, threads, 0, static_cast<cudaStream_t>(stream)>>>(d_parent, d_n_nodes, d_kv_len, batch, n_pad,
-                                                                         d_depth, d_pos, d_mask);
+                                                                         d_depth, d_pos, d_mask, fc_error_slot());
   return FC_CHECK_LAUNCH();
 }
 
@@ -858,7 +859,7 @@ extern "C" fc_status fc_build_tree_all(int n_sources, const uint32_t* d_drafts, 
   if (reinterpret_cast<uintptr_t>(d_ws) % 256) return FC_ERR_INVALID_ARG;
   TreeIn in{d_drafts, d_draft_len, d_count, d_n_drafts, {0, 0, 0, 0}};
   for (int s = 0; s < n_sources; ++s) in.w[s] = src_weight[s];
-  TreeOut out{d_tok, d_parent, d_depth, d_pos, d_mask, d_n_nodes};
+  TreeOut out{d_tok, d_parent, d_depth, d_pos, d_mask, d_n_nodes, fc_error_slot()};
   k_build_tree_all<<<batch, BT_THREADS, 0, static_cast<cudaStream_t>(stream)>>>(
       in, n_sources, batch, slots, draft_len, d_root_tok, d_kv_len, node_budget, n_pad,
       static_cast<unsigned char*>(d_ws), per, out);

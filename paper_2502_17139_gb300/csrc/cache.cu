@@ -57,6 +57,7 @@ struct CacheView {
   uint32_t* words;
   int32_t* meta;
   int capacity, min_size, chunk, ctx_keep;
+  unsigned int* err;  // the launch's error word (NULL: this file's own)
 };
 
 struct ResOut {
@@ -235,7 +236,7 @@ __global__ void __launch_bounds__(CS_THREADS, 1) k_cache_search(CacheView c, con
     sm.bad = 0;
     sm.best = 0;
     sm.nocc = 0;
-    if (nt_raw < 0 || nt_raw > c.capacity) fc_flag(&g_fc_err, FC_EBIT_INTERNAL);
+    if (nt_raw < 0 || nt_raw > c.capacity) fc_flag(FC_ERR_WORD(c.err), FC_EBIT_INTERNAL);
   }
   __syncthreads();
   if (tid < cap) {
@@ -250,7 +251,7 @@ __global__ void __launch_bounds__(CS_THREADS, 1) k_cache_search(CacheView c, con
   }
   __syncthreads();
   const bool bad = sm.bad != 0;
-  if (bad && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+  if (bad && tid == 0) fc_flag(FC_ERR_WORD(c.err), FC_EBIT_INVALID);
   const bool active = searched && !bad;
 
   // ---- pass 1: at every position with a continuation, the length of the
@@ -679,7 +680,7 @@ __global__ void __launch_bounds__(CU_WARPS * 32) k_cache_update(CacheView c, con
   int32_t* meta = c.meta + 4 * (size_t)b;
   int w = meta[0], ns = meta[1], mark = meta[2], dropped = meta[3];
   if (o < 0 || n < o || n > stride || mark < 0 || w < 0 || w > c.capacity) {
-    if (lane == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+    if (lane == 0) fc_flag(FC_ERR_WORD(c.err), FC_EBIT_INVALID);
     return;
   }
   const uint32_t* row = ctx + (size_t)b * stride;
@@ -688,7 +689,7 @@ __global__ void __launch_bounds__(CU_WARPS * 32) k_cache_update(CacheView c, con
     bool bad = false;
     for (int i = lane; i < L; i += 32) bad |= row[s0 + i] >= FC_SEP_TOKEN;
     if (__any_sync(0xFFFFFFFFu, bad)) {
-      if (lane == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+      if (lane == 0) fc_flag(FC_ERR_WORD(c.err), FC_EBIT_INVALID);
       return;
     }
     if (w + L + 1 <= c.capacity) {
@@ -737,7 +738,7 @@ bool missing_cap_ok(int capacity) {
 }
 
 CacheView view_of(const fc_cache* c) {
-  return CacheView{c->d_words, c->d_meta, c->capacity, c->min_size, c->chunk, c->ctx_keep};
+  return CacheView{c->d_words, c->d_meta, c->capacity, c->min_size, c->chunk, c->ctx_keep, fc_error_slot()};
 }
 
 }  // namespace

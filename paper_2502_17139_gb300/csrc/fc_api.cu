@@ -10,6 +10,16 @@ extern "C" unsigned int fc_take_error_cache(cudaStream_t s);
 extern "C" unsigned int fc_take_error_dec(cudaStream_t s);
 extern "C" unsigned int fc_take_error_gemm(cudaStream_t s);
 
+namespace {
+thread_local unsigned int* t_error_slot = nullptr;
+}
+
+unsigned int* fc_error_slot() { return t_error_slot; }
+
+FcErrorScope::FcErrorScope(unsigned int* word) : prev(t_error_slot) { t_error_slot = word; }
+
+FcErrorScope::~FcErrorScope() { t_error_slot = prev; }
+
 extern "C" const char* fc_status_string(fc_status s) {
   switch (s) {
     case FC_OK: return "FC_OK";
@@ -34,9 +44,5 @@ extern "C" fc_status fc_get_error(fc_stream stream) {
   unsigned int e = fc_take_error_sa(s) | fc_take_error_ret(s) | fc_take_error_tree(s) | fc_take_error_step(s) |
                    fc_take_error_attn(s) | fc_take_error_cache(s) |
                    fc_take_error_dec(s) | fc_take_error_gemm(s);
-  if (e & FC_EBIT_INTERNAL) return FC_ERR_INTERNAL;
-  if (e & FC_EBIT_TIMEOUT) return FC_ERR_TIMEOUT;
-  if (e & FC_EBIT_CAPACITY) return FC_ERR_CAPACITY;
-  if (e & FC_EBIT_INVALID) return FC_ERR_INVALID_ARG;
-  return FC_OK;
+  return fc_status_of_bits(e);
 }

@@ -46,6 +46,24 @@ struct FcNvtxRange {
 
 __device__ __forceinline__ void fc_flag(unsigned int* word, unsigned int bit) { atomicOr(word, bit); }
 
+// Kernels take the error word of their launch as an argument: NULL means
+// their translation unit's own word (collected by fc_get_error), a device
+// pointer a word of the caller's (fc_pipeline gives every sub-batch its own,
+// so an error is reported for the sub-batch that raised it).
+#define FC_ERR_WORD(err) ((err) ? (err) : &g_fc_err)
+
+// Host: the error word that launches made by the calling thread pass to their
+// kernels (NULL unless an FcErrorScope is active on this thread).
+unsigned int* fc_error_slot();
+// Host: routes the calling thread's launches to `word` while in scope.
+struct FcErrorScope {
+  unsigned int* prev;
+  explicit FcErrorScope(unsigned int* word);
+  ~FcErrorScope();
+  FcErrorScope(const FcErrorScope&) = delete;
+  FcErrorScope& operator=(const FcErrorScope&) = delete;
+};
+
 // Debug builds (compiled with -DFC_DEBUG into libfastcoder_debug.so) check
 // the indexes that gathers take from data, such as suffix-array entries,
 // before using them: an index out of range sets FC_ERR_INTERNAL in the
@@ -60,6 +78,15 @@ __device__ __forceinline__ bool fc_debug_ok(bool ok, unsigned int* word) {
 #else
 #define FC_DEBUG_CHECK(ok) true
 #endif
+
+// Host: the status of a set of error bits, the most severe first.
+static inline fc_status fc_status_of_bits(unsigned int e) {
+  if (e & FC_EBIT_INTERNAL) return FC_ERR_INTERNAL;
+  if (e & FC_EBIT_TIMEOUT) return FC_ERR_TIMEOUT;
+  if (e & FC_EBIT_CAPACITY) return FC_ERR_CAPACITY;
+  if (e & FC_EBIT_INVALID) return FC_ERR_INVALID_ARG;
+  return FC_OK;
+}
 
 // Host: map a CUDA launch result to a status.
 static inline fc_status fc_cuda_status(cudaError_t e) { return e == cudaSuccess ? FC_OK : FC_ERR_CUDA; }

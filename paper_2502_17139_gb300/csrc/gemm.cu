@@ -70,6 +70,7 @@ struct GemmArgs {
   const int32_t* pos;    // [B][n_pad]; a negative position leaves its row unrotated
   int n_pad, hkv;
   double rope_nl2f;      // -2 log2(base) / 128
+  unsigned int* err;     // the launch's error word (NULL: this file's own)
 };
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
@@ -295,7 +296,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
-  if (tid == 0 && s_abort) fc_flag(&g_fc_err, FC_EBIT_TIMEOUT);
+  if (tid == 0 && s_abort) fc_flag(FC_ERR_WORD(g.err), FC_EBIT_TIMEOUT);
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
@@ -347,6 +348,7 @@ fc_status launch_gemm(const void* d_a, const void* d_b, int M, int N, int K, Gem
   g.N = N;
   g.K = K;
   g.tiles_m = (M + BM - 1) / BM;
+  g.err = fc_error_slot();
   const int64_t tiles = (int64_t)g.tiles_m * ((N + BN - 1) / BN);
   if (tiles > 0x7FFFFFFF) return FC_ERR_UNSUPPORTED;
   g.tiles = (int)tiles;

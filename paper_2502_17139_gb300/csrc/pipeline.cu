@@ -151,6 +151,7 @@ extern "C" fc_status fc_pipeline_step(fc_pipeline* pl, int phase, int flags, con
     const void* kt = static_cast<const char*>(d_k_tree) + (size_t)P.first * kt_row;
     const void* vt = static_cast<const char*>(d_v_tree) + (size_t)P.first * kt_row;
     const int32_t* want = d_want_hit ? d_want_hit + P.first : nullptr;
+    FcErrorScope scope(P.err);  // the sub-batch's kernels record errors in its own word
 
     stage_event(stage_events, h, 0, 0, s);
     if (P.rcache)
@@ -197,6 +198,19 @@ extern "C" fc_status fc_pipeline_step(fc_pipeline* pl, int phase, int flags, con
     stage_event(stage_events, h, 3, 1, s);
   }
   return FC_OK;
+}
+
+extern "C" fc_status fc_pipeline_error(fc_pipeline* pl, int part) {
+  FC_NVTX_RANGE();
+  if (!pl || part < 0 || part >= (int)pl->parts.size() || !pl->parts[part].err) return FC_ERR_INVALID_ARG;
+  cudaStream_t s = pl->chain[part];
+  unsigned int* w = pl->parts[part].err;
+  unsigned int h = 0;
+  // the chain stream already follows the attention stream of every step
+  if (cudaMemcpyAsync(&h, w, sizeof h, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaMemsetAsync(w, 0, sizeof h, s) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess)
+    return FC_ERR_CUDA;
+  return fc_status_of_bits(h);
 }
 
 extern "C" fc_stream fc_pipeline_stream(const fc_pipeline* pl, int part) {

@@ -66,6 +66,7 @@ struct RetOut {
   uint32_t* count;
   int32_t* n_drafts;
   int32_t* match_len;
+  unsigned int* err;  // the launch's error word (NULL: this file's own)
 };
 
 // Sign of the suffix T[i..N) cut to n tokens against pat[0..n), knowing
@@ -232,7 +233,7 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev
     if (t >= ds.vocab) sm.bad = 1;
   }
   __syncthreads();
-  if (sm.bad && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+  if (sm.bad && tid == 0) fc_flag(FC_ERR_WORD(o.err), FC_EBIT_INVALID);
 
   // ---- search: one warp per n, one half-warp per bound, 16 pivots a round
   // (lengths n_top down to n_top - n_count + 1; with the reversed corpus only n*)
@@ -493,7 +494,7 @@ __global__ void k_rc_insert(uint32_t* table, int capacity, int S, fc_retrieve_pa
         present = true;  // an equal key holds the same (deterministic) result
       }
     }
-    if (slot < 0 && !present) fc_flag(&g_fc_err, FC_EBIT_CAPACITY);
+    if (slot < 0 && !present) fc_flag(FC_ERR_WORD(o.err), FC_EBIT_CAPACITY);
     sm.slot = slot;
   }
   __syncthreads();
@@ -562,7 +563,7 @@ static fc_status launch_retrieve(bool all, const fc_datastore* sources, const fc
       return FC_ERR_CUDA;
     attr_done[variant] = true;
   }
-  RetOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len};
+  RetOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len, fc_error_slot()};
   dim3 grid((unsigned)batch, (unsigned)n_sources);
   kern<<<grid, RT_THREADS, sizeof(RetSmem), static_cast<cudaStream_t>(stream)>>>(a, r, d_ctx, ctx_stride, d_ctx_len,
                                                                                  batch, d_skip, p, o);
@@ -629,7 +630,7 @@ extern "C" fc_status fc_rcache_lookup(const void* d_table, int capacity, int n_s
   if (batch == 0) return FC_OK;
   if (!d_ctx || !d_ctx_len || !d_skip || !d_drafts || !d_draft_len || !d_count || !d_n_drafts || !d_match_len)
     return FC_ERR_INVALID_ARG;
-  RetOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len};
+  RetOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len, fc_error_slot()};
   k_rc_lookup<<<batch, 128, 0, static_cast<cudaStream_t>(stream)>>>(static_cast<const uint32_t*>(d_table), capacity,
                                                                      n_sources, p, d_ctx, ctx_stride, d_ctx_len, batch,
                                                                      d_want_hit, d_skip, o);
@@ -647,7 +648,7 @@ extern "C" fc_status fc_rcache_insert(void* d_table, int capacity, int n_sources
   if (!d_ctx || !d_ctx_len || !d_drafts || !d_draft_len || !d_count || !d_n_drafts || !d_match_len)
     return FC_ERR_INVALID_ARG;
   RetOut o{const_cast<uint32_t*>(d_drafts), const_cast<int32_t*>(d_draft_len), const_cast<uint32_t*>(d_count),
-           const_cast<int32_t*>(d_n_drafts), const_cast<int32_t*>(d_match_len)};
+           const_cast<int32_t*>(d_n_drafts), const_cast<int32_t*>(d_match_len), fc_error_slot()};
   k_rc_insert<<<batch, 128, 0, static_cast<cudaStream_t>(stream)>>>(static_cast<uint32_t*>(d_table), capacity,
                                                                      n_sources, p, d_ctx, ctx_stride, d_ctx_len, batch,
                                                                      d_skip, o);

@@ -22,7 +22,8 @@ __global__ void __launch_bounds__(ACC_WARPS * 32) k_accept(const uint32_t* __res
                                                            const int32_t* __restrict__ n_nodes,
                                                            const uint32_t* __restrict__ argmax, int B, int n_pad,
                                                            int32_t* __restrict__ acc_len, int32_t* __restrict__ path,
-                                                           int path_cap, uint32_t* __restrict__ bonus) {
+                                                           int path_cap, uint32_t* __restrict__ bonus,
+                                                           unsigned int* err) {
   extern __shared__ uint32_t acc_smem[];  // [ACC_WARPS][3][n_pad]
   // Launched as a programmatic dependent of the row argmax (fc_argmax_accept):
   // wait here until that grid's results are visible.  A no-op otherwise.
@@ -67,7 +68,7 @@ __global__ void __launch_bounds__(ACC_WARPS * 32) k_accept(const uint32_t* __res
     pth[0] = 0;
     acc_len[b] = len;
     bonus[b] = s_am[cur];
-    if (overflow) fc_flag(&g_fc_err, FC_EBIT_CAPACITY);
+    if (overflow) fc_flag(FC_ERR_WORD(err), FC_EBIT_CAPACITY);
   }
 }
 
@@ -79,7 +80,8 @@ __global__ void k_kv_append(const int32_t* __restrict__ path, const int32_t* __r
                             int D, int path_cap, uint4* __restrict__ k_cache, uint4* __restrict__ v_cache, int kv_cap,
                             const int32_t* __restrict__ kv_len_in, int32_t* __restrict__ kv_len_out,
                             uint32_t* __restrict__ ctx, int ctx_stride, const int32_t* __restrict__ ctx_len_in,
-                            int32_t* __restrict__ ctx_len_out, uint32_t* __restrict__ root_out) {
+                            int32_t* __restrict__ ctx_len_out, uint32_t* __restrict__ root_out,
+                            unsigned int* err) {
   const int b = blockIdx.x;
   const int a = acc_len[b];
   const int kvl = kv_len_in[b], cl = ctx_len_in[b];
@@ -87,7 +89,7 @@ __global__ void k_kv_append(const int32_t* __restrict__ path, const int32_t* __r
                   cl + a + 1 <= ctx_stride;
   if (!ok) {
     if (threadIdx.x == 0) {
-      fc_flag(&g_fc_err, FC_EBIT_CAPACITY);
+      fc_flag(FC_ERR_WORD(err), FC_EBIT_CAPACITY);
       kv_len_out[b] = kvl;
       ctx_len_out[b] = cl;
       root_out[b] = (cl > 0 && cl <= ctx_stride) ? ctx[(size_t)b * ctx_stride + cl - 1] : 0u;
@@ -102,7 +104,7 @@ __global__ void k_kv_append(const int32_t* __restrict__ path, const int32_t* __r
     int t = r / Hkv, g = r - t * Hkv;
     int node = pth[t];
     if (node < 0 || node >= n_pad) {
-      fc_flag(&g_fc_err, FC_EBIT_INVALID);
+      fc_flag(FC_ERR_WORD(err), FC_EBIT_INVALID);
       continue;
     }
     size_t src = (((size_t)b * Hkv + g) * n_pad + node) * vec + x;
@@ -298,7 +300,7 @@ extern "C" fc_status fc_accept(const uint32_t* d_tok, const int32_t* d_parent, c
   const unsigned blocks = (unsigned)((batch + ACC_WARPS - 1) / ACC_WARPS);
   const size_t smem = (size_t)ACC_WARPS * 3 * n_pad * sizeof(uint32_t);  // <= 48 KB for n_pad <= 1024
   k_accept<<<blocks, ACC_WARPS * 32, smem, static_cast<cudaStream_t>(stream)>>>(
-      d_tok, d_parent, d_n_nodes, d_argmax, batch, n_pad, d_acc_len, d_path, path_cap, d_bonus);
+      d_tok, d_parent, d_n_nodes, d_argmax, batch, n_pad, d_acc_len, d_path, path_cap, d_bonus, fc_error_slot());
   return FC_CHECK_LAUNCH();
 }
 
@@ -331,7 +333,7 @@ extern "C" fc_status fc_argmax_accept(const void* d_logits, int vocab, const uin
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
   if (cudaLaunchKernelEx(&cfg, k_accept, d_tok, d_parent, d_n_nodes, (const uint32_t*)d_argmax, batch, n_pad,
-                         d_acc_len, d_path, path_cap, d_bonus) != cudaSuccess)
+                         d_acc_len, d_path, path_cap, d_bonus, fc_error_slot()) != cudaSuccess)
     return FC_ERR_CUDA;
   return FC_CHECK_LAUNCH();
 }
@@ -356,7 +358,7 @@ extern "C" fc_status fc_kv_append(const int32_t* d_path, const int32_t* d_acc_le
   k_kv_append<<<batch, 256, 0, static_cast<cudaStream_t>(stream)>>>(
       d_path, d_acc_len, d_bonus, d_tok, static_cast<const uint4*>(d_k_tree), static_cast<const uint4*>(d_v_tree), n_pad,
       Hkv, D, path_cap, static_cast<uint4*>(d_k_cache), static_cast<uint4*>(d_v_cache), kv_cap, d_kv_len_in,
-      d_kv_len_out, d_ctx, ctx_stride, d_ctx_len_in, d_ctx_len_out, d_root_out);
+      d_kv_len_out, d_ctx, ctx_stride, d_ctx_len_in, d_ctx_len_out, d_root_out, fc_error_slot());
   return FC_CHECK_LAUNCH();
 }
 
@@ -381,7 +383,7 @@ extern "C" fc_status fc_synth_argmax(const uint32_t* d_tok, const int32_t* d_par
 // without faulting or hanging anything.
 // ---------------------------------------------------------------------------
 namespace {
-__global__ void k_selftest_wait(int arrive, unsigned long long limit_cycles) {
+__global__ void k_selftest_wait(int arrive, unsigned long long limit_cycles, unsigned int* err) {
   __shared__ __align__(8) uint64_t bar_word;
   __shared__ int abort_flag;
   const uint32_t bar = smem_u32(&bar_word);
@@ -393,7 +395,7 @@ __global__ void k_selftest_wait(int arrive, unsigned long long limit_cycles) {
   __syncthreads();
   if (threadIdx.x == 0) {
     if (arrive) mbar_arrive(bar);
-    if (!mbar_wait_bounded(bar, 0, &abort_flag, limit_cycles)) fc_flag(&g_fc_err, FC_EBIT_TIMEOUT);
+    if (!mbar_wait_bounded(bar, 0, &abort_flag, limit_cycles)) fc_flag(FC_ERR_WORD(err), FC_EBIT_TIMEOUT);
   }
 }
 }  // namespace
@@ -401,6 +403,6 @@ __global__ void k_selftest_wait(int arrive, unsigned long long limit_cycles) {
 extern "C" fc_status fc_selftest_wait(int arrive, unsigned long long limit_cycles, fc_stream stream) {
   FC_NVTX_RANGE();
   if (limit_cycles == 0 || limit_cycles > 4000000000ull) return FC_ERR_INVALID_ARG;
-  k_selftest_wait<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(arrive, limit_cycles);
+  k_selftest_wait<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(arrive, limit_cycles, fc_error_slot());
   return FC_CHECK_LAUNCH();
 }

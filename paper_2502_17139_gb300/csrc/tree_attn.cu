@@ -90,6 +90,7 @@ struct AttnArgs {
   int* ws_cnt;     // [split units][2]: arrival tickets, finished partials (zeroed before the launch)
   float2* ws_ml;   // [split units][parts - 1][256 rows]: (m, l) of a partial
   float* ws_o;     // [split units][parts - 1][256 rows][128]: unnormalised O of a partial
+  unsigned int* err;  // the launch's error word (NULL: this file's own)
   float scale_log2;
   const int32_t* pos;  // [B][n_pad] node positions: rotate Q by them (RoPE), or nullptr
   double rope_nl2f;    // -2 log2(base) / D: pair i turns by pos * 2^(i * rope_nl2f)
@@ -228,7 +229,7 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   const int nn_raw = a.n_nodes[b], kvl = a.kv_len[b];
   const bool bad = nn_raw < 1 || nn_raw > a.n_pad || kvl < 0 || kvl > a.kv_cap;
   const int nn = bad ? 0 : nn_raw;
-  if (bad && c == 0 && part == 0 && tid == 0) fc_flag(&g_fc_err, FC_EBIT_INVALID);
+  if (bad && c == 0 && part == 0 && tid == 0) fc_flag(FC_ERR_WORD(a.err), FC_EBIT_INVALID);
 
   // Zero the padding rows (nodes >= n_nodes) of this group: the group's part-0
   // CTAs share them (row r of the G x pad padding rows goes to CTA r mod ctas),
@@ -686,7 +687,7 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
-  if (tid == 0 && s_abort) fc_flag(&g_fc_err, FC_EBIT_TIMEOUT);
+  if (tid == 0 && s_abort) fc_flag(FC_ERR_WORD(a.err), FC_EBIT_TIMEOUT);
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
@@ -872,6 +873,7 @@ static fc_status launch_tree_attn(const void* d_q, const void* d_k_cache, const 
   a.ws_cnt = nullptr;
   a.ws_ml = nullptr;
   a.ws_o = nullptr;
+  a.err = fc_error_slot();
   a.pos = d_pos;
   a.rope_nl2f = d_pos ? -2.0 * std::log2((double)rope_base) / HD : 0.0;
   if (sp.parts > 1) {

@@ -61,7 +61,7 @@ class fc_pipeline_part(C.Structure):
                 ("pos", C.c_void_p), ("mask", C.c_void_p), ("n_nodes", C.c_void_p), ("k_cache", C.c_void_p),
                 ("v_cache", C.c_void_p), ("k_tree_rot", C.c_void_p), ("attn_out", C.c_void_p),
                 ("attn_ws", C.c_void_p), ("attn_ws_bytes", C.c_size_t), ("argmax", C.c_void_p),
-                ("acc_len", C.c_void_p), ("path", C.c_void_p), ("bonus", C.c_void_p)]
+                ("acc_len", C.c_void_p), ("path", C.c_void_p), ("bonus", C.c_void_p), ("err", C.c_void_p)]
 
 
 class fc_pipeline_desc(C.Structure):
@@ -78,7 +78,8 @@ EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
            "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_gemm_kv_heads", "fc_gemm_silu_mul", "fc_interleave_gate_up", "fc_embed",
            "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax",
-           "fc_pipeline_create", "fc_pipeline_step", "fc_pipeline_stream", "fc_pipeline_join", "fc_pipeline_destroy"]
+           "fc_pipeline_create", "fc_pipeline_step", "fc_pipeline_stream", "fc_pipeline_error", "fc_pipeline_join",
+           "fc_pipeline_destroy"]
 
 
 def _load():
@@ -151,6 +152,7 @@ def _load():
         "fc_pipeline_step": (C.c_int, [vp, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]),
         "fc_pipeline_join": (C.c_int, [vp, vp]),
         "fc_pipeline_stream": (vp, [vp, i32]),
+        "fc_pipeline_error": (C.c_int, [vp, i32]),
         "fc_pipeline_destroy": (None, [vp]),
     }
     for name, (res, args) in sig.items():
@@ -810,11 +812,14 @@ def _close_pipelines():
 
 
 def pipeline_part(batch, first, ctx, ctx_len, kv_len, root, rcache, skip, res, tree, k_cache, v_cache, k_tree_rot,
-                  attn_out, attn_ws, argmax, acc) -> fc_pipeline_part:
+                  attn_out, attn_ws, argmax, acc, err=None) -> fc_pipeline_part:
     """One sub-batch's buffers (device tensors the caller keeps alive):
     ctx_len and kv_len are pairs (the ping-pong lengths), rcache a
     RetrievalCache or None, res/tree/acc the dicts of retrieve_outputs,
-    tree_outputs and fc_accept's outputs."""
+    tree_outputs and fc_accept's outputs, err None or a zeroed one-element
+    int32 tensor: the sub-batch's own error word."""
+    if err is not None:
+        _need(err, torch.int32, "err", (1,))
     _need(ctx, torch.int32, "ctx", (batch, ctx.shape[1]))
     for t in (*ctx_len, *kv_len, root, skip):
         _need(t, torch.int32, "length", (batch,))
@@ -827,7 +832,7 @@ def pipeline_part(batch, first, ctx, ctx_len, kv_len, root, rcache, skip, res, t
         _ptr(res["n_drafts"]), _ptr(res["match_len"]), _ptr(tree["tok"]), _ptr(tree["parent"]), _ptr(tree["depth"]),
         _ptr(tree["pos"]), _ptr(tree["mask"]), _ptr(tree["n_nodes"]), _ptr(k_cache), _ptr(v_cache), _ptr(k_tree_rot),
         _ptr(attn_out), _ptr(attn_ws), 0 if attn_ws is None else attn_ws.numel() * attn_ws.element_size(),
-        _ptr(argmax), _ptr(acc["acc_len"]), _ptr(acc["path"]), _ptr(acc["bonus"]))
+        _ptr(argmax), _ptr(acc["acc_len"]), _ptr(acc["path"]), _ptr(acc["bonus"]), _ptr(err))
 
 
 class Pipeline:
@@ -888,6 +893,12 @@ class Pipeline:
     def join(self):
         """The current stream waits for everything enqueued on the sub-batches."""
         _check("fc_pipeline_join", LIB.fc_pipeline_join(self.handle, _stream()))
+
+    def error(self, part):
+        """Sub-batch ``part``'s device errors since the last call (a status
+        name; waits for its work, clears its word)."""
+        code = LIB.fc_pipeline_error(self.handle, part)
+        return STATUS.get(code, str(code))
 
     def close(self):
         if getattr(self, "handle", None):

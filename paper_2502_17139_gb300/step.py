@@ -286,10 +286,12 @@ class PipelinedStepLoop:
                                kv0[sl], vocab, cache_capacity=cache_capacity, device=device,
                                k_cache=self.k_cache[sl], v_cache=self.v_cache[sl], rope_base=rope_base)
                       for sl in self.slices]
+        # every sub-batch records its device errors in a word of its own
+        self.err_words = torch.zeros((len(self.slices), 1), dtype=torch.int32, device=device)
         parts = [fc.pipeline_part(sl.stop - sl.start, sl.start, lp.ctx, lp.ctx_len, lp.kv_len, lp.root, lp.cache,
                                   lp.skip, lp.res, lp.tree, lp.k_cache, lp.v_cache, lp.k_tree_rot, lp.attn_out,
-                                  lp.attn_ws, lp.argmax, lp.acc)
-                 for lp, sl in zip(self.loops, self.slices)]
+                                  lp.attn_ws, lp.argmax, lp.acc, err=self.err_words[h])
+                 for h, (lp, sl) in enumerate(zip(self.loops, self.slices))]
         lp0 = self.loops[0]
         self.pipe = fc.Pipeline(sources, p, lp0.tree_weight, node_budget, n_pad, H, Hkv, D, kv_cap, lp0.path_cap,
                                 vocab, parts, rope_base=rope_base)
@@ -307,6 +309,12 @@ class PipelinedStepLoop:
     def join(self):
         """The caller's current stream waits for everything enqueued so far."""
         self.pipe.join()
+
+    def errors(self):
+        """Each sub-batch's device errors since the last call (status names;
+        waits for the sub-batches and clears their words).  The sub-batches'
+        kernels report here, not through fc_get_error."""
+        return [self.pipe.error(h) for h in range(len(self.loops))]
 
     def capture(self, inputs, attention=True):
         """An even number of steps of every sub-batch in one CUDA graph (fork

@@ -208,7 +208,7 @@ def test_step_loop_full_store_lockstep(fc, orc):
         got["bonus"].append(host_u32(loop.acc["bonus"]))
         got["n_nodes"].append(loop.tree["n_nodes"].cpu().numpy())
     torch.cuda.synchronize()
-    assert fc.fc_get_error() == "FC_OK"
+    assert fc.fc_get_error() == "FC_OK" and loop.errors() == ["FC_OK", "FC_OK"]
     # the oracle, one sub-batch at a time with a replay cache of its own
     po = dict(n_max=cfg["n_max"], n_min=cfg["n_min"], top_k=cfg["top_k"], draft_len=d, max_occ=4096,
               node_budget=cfg["node_budget"], n_pad=n_pad)

@@ -77,7 +77,7 @@ def test_pipelined_matches_single_loop(fc, setup, n_split):
         piped.step(*setup["ins"][s])
         piped.join()
         same(state(single), state(piped))
-    assert fc.fc_get_error() == "FC_OK"
+    assert fc.fc_get_error() == "FC_OK" and piped.errors() == ["FC_OK"] * n_split
     # reset replays the same trajectory
     piped.reset()
     for s in range(2):
@@ -229,3 +229,21 @@ def test_pipelined_stage_events_and_streams(fc, setup):
         assert e["attn"][1].elapsed_time(e["tail"][0]) >= 0
     for lp, o in zip(piped.loops, outs):
         assert torch.equal(o, lp.acc["acc_len"])
+
+
+def test_pipelined_errors_attributed_to_their_sub_batch(fc, setup):
+    """A context token outside the vocabulary in one sequence of sub-batch 1:
+    its retrieval records FC_ERR_INVALID_ARG in sub-batch 1's own error word;
+    sub-batch 0's word and the library-wide words stay clean, and the word
+    reads clean again after it was taken."""
+    from paper_2502_17139_gb300.step import PipelinedStepLoop
+    srcs, ctx, cl = setup["args"][:3]
+    bad = np.array(ctx, copy=True)
+    b = 6  # in the second sub-batch (sequences 4..8)
+    bad[b, int(cl[b]) - 3] = synth.VOCAB + 5
+    piped = PipelinedStepLoop(2, srcs, bad, cl, *setup["args"][3:], **setup["kw"])
+    piped.step(*setup["ins"][0])
+    piped.join()
+    assert piped.errors() == ["FC_OK", "FC_ERR_INVALID_ARG"]
+    assert fc.fc_get_error() == "FC_OK"
+    assert piped.errors() == ["FC_OK", "FC_OK"]
