@@ -421,11 +421,54 @@ __device__ void rc_load_key(RcSmem& sm, const uint32_t* ctx, int stride, const i
   __syncthreads();
 }
 
-__device__ bool rc_key_equal(const uint32_t* entry, const RcSmem& sm) {
-  if (entry[0] != (uint32_t)sm.klen) return false;
-  for (int i = 0; i < sm.klen; ++i)
-    if (entry[1 + i] != sm.key[i]) return false;
-  return true;
+// Warp 0 compares the entry's key with sm.key: lane i reads key word i, so
+// the words arrive in one round trip (n_max <= 32).  `head` is the entry's
+// first word, already read.  Warp-uniform result.
+__device__ bool rc_key_equal_warp(const uint32_t* entry, uint32_t head, const RcSmem& sm, int lane) {
+  const bool len_ok = head == (uint32_t)sm.klen;
+  const uint32_t w = (len_ok && lane < sm.klen) ? entry[1 + lane] : 0u;
+  return __all_sync(0xFFFFFFFFu, len_ok && (lane >= sm.klen || w == sm.key[lane]));
+}
+
+// A query's outputs and a cache entry's result area, word by word: flat
+// index i over S * rc_src_words(p) words (source s, then drafts, draft
+// lengths, counts, n_drafts, match_len) names one word of the entry
+// (entry[i]) and one output word (*rc_out_word(...)).
+__device__ __forceinline__ uint32_t* rc_out_word(const RetOut& o, int i, int per, int k, int d, int B, int b) {
+  const int s = i / per, r = i - s * per;
+  const size_t sb = (size_t)s * B + b;
+  if (r < k * d) return o.drafts + sb * k * d + r;
+  if (r < k * d + k) return reinterpret_cast<uint32_t*>(o.draft_len) + sb * k + (r - k * d);
+  if (r < k * d + 2 * k) return o.count + sb * k + (r - k * d - k);
+  return r == k * d + 2 * k ? reinterpret_cast<uint32_t*>(o.n_drafts) + sb : reinterpret_cast<uint32_t*>(o.match_len) + sb;
+}
+
+// Copies a query's whole result between a cache entry and the outputs with
+// the CTA's threads, sixteen loads in flight per thread before their stores
+// (a lookup or an insert is a few such round trips, not one per array).
+template <bool TO_OUT>
+__device__ __forceinline__ void rc_copy(uint32_t* entry, const RetOut& o, int S, const fc_retrieve_params& p, int B,
+                                        int b) {
+  constexpr int U = 16;
+  const int k = p.top_k, d = p.draft_len, per = (int)rc_src_words(p), n = S * per;
+  for (int i0 = threadIdx.x; i0 < n; i0 += U * blockDim.x) {
+    uint32_t v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + u * blockDim.x;
+      v[u] = i < n ? (TO_OUT ? entry[i] : *rc_out_word(o, i, per, k, d, B, b)) : 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i < n) {
+        if (TO_OUT)
+          *rc_out_word(o, i, per, k, d, B, b) = v[u];
+        else
+          entry[i] = v[u];
+      }
+    }
+  }
 }
 
 __global__ void k_rc_lookup(const uint32_t* __restrict__ table, int capacity, int S, fc_retrieve_params p,
@@ -435,41 +478,30 @@ __global__ void k_rc_lookup(const uint32_t* __restrict__ table, int capacity, in
   const int b = blockIdx.x;
   rc_load_key(sm, ctx, stride, ctx_len, b, p.n_max);
   const size_t ew = rc_entry_words(S, p);
-  if (threadIdx.x == 0) {
+  if (threadIdx.x < 32) {  // warp 0 probes; every lane takes the same path
+    const int lane = threadIdx.x;
     int slot = -1;
     if (!want || want[b]) {
-      uint64_t h = rc_hash(sm.key, sm.klen);
+      const uint64_t h = rc_hash(sm.key, sm.klen);
       for (int probe = 0; probe < capacity; ++probe) {
-        size_t e = (h + probe) & (uint64_t)(capacity - 1);
+        const size_t e = (h + probe) & (uint64_t)(capacity - 1);
         const uint32_t* ent = table + e * ew;
-        uint32_t st = ent[0];
+        const uint32_t st = ent[0];
         if (st == RC_EMPTY) break;
-        if (st != RC_CLAIMED && rc_key_equal(ent, sm)) {
+        if (st != RC_CLAIMED && rc_key_equal_warp(ent, st, sm, lane)) {
           slot = (int)e;
           break;
         }
       }
     }
-    sm.slot = slot;
-    skip[b] = slot >= 0 ? 1 : 0;
+    if (lane == 0) {
+      sm.slot = slot;
+      skip[b] = slot >= 0 ? 1 : 0;
+    }
   }
   __syncthreads();
   if (sm.slot < 0) return;
-  const uint32_t* src = table + (size_t)sm.slot * ew + 1 + p.n_max;
-  const int k = p.top_k, d = p.draft_len;
-  for (int s = 0; s < S; ++s) {
-    const uint32_t* e = src + s * rc_src_words(p);
-    size_t sb = (size_t)s * B + b;
-    for (int i = threadIdx.x; i < k * d; i += blockDim.x) o.drafts[sb * k * d + i] = e[i];
-    for (int i = threadIdx.x; i < k; i += blockDim.x) {
-      o.draft_len[sb * k + i] = (int32_t)e[k * d + i];
-      o.count[sb * k + i] = e[k * d + k + i];
-    }
-    if (threadIdx.x == 0) {
-      o.n_drafts[sb] = (int32_t)e[k * d + 2 * k];
-      o.match_len[sb] = (int32_t)e[k * d + 2 * k + 1];
-    }
-  }
+  rc_copy<true>(const_cast<uint32_t*>(table) + (size_t)sm.slot * ew + 1 + p.n_max, o, S, p, B, b);
 }
 
 __global__ void k_rc_insert(uint32_t* table, int capacity, int S, fc_retrieve_params p,
@@ -480,42 +512,33 @@ __global__ void k_rc_insert(uint32_t* table, int capacity, int S, fc_retrieve_pa
   if (skip && skip[b]) return;
   rc_load_key(sm, ctx, stride, ctx_len, b, p.n_max);
   const size_t ew = rc_entry_words(S, p);
-  if (threadIdx.x == 0) {
+  if (threadIdx.x < 32) {  // warp 0 probes: lane 0 claims, the warp compares keys
+    const int lane = threadIdx.x;
     int slot = -1;
     bool present = false;
-    uint64_t h = rc_hash(sm.key, sm.klen);
+    const uint64_t h = rc_hash(sm.key, sm.klen);
     for (int probe = 0; probe < capacity && slot < 0 && !present; ++probe) {
-      size_t e = (h + probe) & (uint64_t)(capacity - 1);
+      const size_t e = (h + probe) & (uint64_t)(capacity - 1);
       uint32_t* ent = table + e * ew;
-      uint32_t st = atomicCAS(ent, RC_EMPTY, RC_CLAIMED);
+      uint32_t st = 0;
+      if (lane == 0) st = atomicCAS(ent, RC_EMPTY, RC_CLAIMED);
+      st = __shfl_sync(0xFFFFFFFFu, st, 0);
       if (st == RC_EMPTY) {
         slot = (int)e;
-      } else if (st != RC_CLAIMED && rc_key_equal(ent, sm)) {
+      } else if (st != RC_CLAIMED && rc_key_equal_warp(ent, st, sm, lane)) {
         present = true;  // an equal key holds the same (deterministic) result
       }
     }
-    if (slot < 0 && !present) fc_flag(FC_ERR_WORD(o.err), FC_EBIT_CAPACITY);
-    sm.slot = slot;
+    if (lane == 0) {
+      if (slot < 0 && !present) fc_flag(FC_ERR_WORD(o.err), FC_EBIT_CAPACITY);
+      sm.slot = slot;
+    }
   }
   __syncthreads();
   if (sm.slot < 0) return;
   uint32_t* ent = table + (size_t)sm.slot * ew;
   for (int i = threadIdx.x; i < sm.klen; i += blockDim.x) ent[1 + i] = sm.key[i];
-  uint32_t* dst = ent + 1 + p.n_max;
-  const int k = p.top_k, d = p.draft_len;
-  for (int s = 0; s < S; ++s) {
-    uint32_t* e = dst + s * rc_src_words(p);
-    size_t sb = (size_t)s * B + b;
-    for (int i = threadIdx.x; i < k * d; i += blockDim.x) e[i] = o.drafts[sb * k * d + i];
-    for (int i = threadIdx.x; i < k; i += blockDim.x) {
-      e[k * d + i] = (uint32_t)o.draft_len[sb * k + i];
-      e[k * d + k + i] = o.count[sb * k + i];
-    }
-    if (threadIdx.x == 0) {
-      e[k * d + 2 * k] = (uint32_t)o.n_drafts[sb];
-      e[k * d + 2 * k + 1] = (uint32_t)o.match_len[sb];
-    }
-  }
+  rc_copy<false>(ent + 1 + p.n_max, o, S, p, B, b);
   __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) atomicExch(ent, (uint32_t)sm.klen);
