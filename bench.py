@@ -84,13 +84,17 @@ def parse_args(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--mode", choices=["step", "attn", "argmax", "configs", "retrieve", "algorithm1", "cache", "gemm", "build",
+                                       "small",
                                        "decoder"],
                     default="step",
                     help="step: the full step loop (the benchmark); attn: tree attention alone on the step loop's "
                          "attention shape with seeded trees (a small profiling / sweep target); argmax: greedy "
                          "verification from bf16 logits (fc_argmax_accept) on the step loop's tree shape; configs: "
                          "every stage of the five benchmark configurations timed once each (a report, not the "
-                         "benchmark line); retrieve: two-source retrieval alone for --batch queries (batch sweeps)")
+                         "benchmark line); retrieve: two-source retrieval alone for --batch queries (batch sweeps); "
+                         "small: the step's small kernels (tree build, predictions, acceptance, KV append, "
+                         "replay-cache lookup) over the batches of --batches")
+    ap.add_argument("--batches", default="32,256,2048,16384", help="small mode: comma-separated batch sizes")
     ap.add_argument("--nodes", type=int, default=128, help="attn mode: tree nodes per sequence")
     ap.add_argument("--kv", type=int, default=16384, help="attn mode: KV cache length")
     ap.add_argument("--no-graph", action="store_true",
@@ -1203,6 +1207,90 @@ def run_retrieve(args, rank, ws, local):
     return out
 
 
+def run_small(args, rank, ws, local):
+    """Batch sweep of the step's small kernels on the step loop's own inputs
+    (two-source retrieval on the 5M + 100M stores, the step mix of contexts):
+    tree build, synthetic predictions, acceptance, KV append and a replay-cache
+    lookup that hits.  At the step loop's batch these are latency chains; the
+    sweep shows where each one reaches its bandwidth.  Times are means of
+    back-to-back calls (`_gpu_ms`); bytes are the algorithmic bytes of each
+    call, and the HBM fraction is of the measured copy peak."""
+    import torch
+
+    import paper_2502_17139_gb300.fastcoder as fc
+    import paper_2502_17139_gb300.synth as synth
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    cfg, c5 = synth.WORKLOADS[2], synth.WORKLOADS[5]
+    rng = synth.rng_for(2)
+    corpora = [synth.build_corpus(rng, spec, device="cuda")[0] for spec in cfg["corpus"]]
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32) if a.dtype == np.uint32
+                                        else np.ascontiguousarray(a)).to(dev)
+    sources = [fc.fc_datastore_build(to_dev(T), synth.VOCAB) for T in corpora]
+    p = fc.params(c5["n_max"], c5["n_min"], c5["top_k"], c5["draft_len"], 4096)
+    S, k, d, n_pad, Hkv, D = 2, c5["top_k"], c5["draft_len"], c5["n_pad"], c5["Hkv"], c5["D"]
+    path_cap, cap = d + 2, 2 * (d + 2)
+    peak = load_peaks()["hbm"]
+    batches = [int(x) for x in args.batches.split(",")]
+    rows = []
+    for B in batches:
+        ctx, cl, _ = synth.make_contexts(rng, B, c5["ctx_len"], c5["n_copy"], corpora + [None], c5["probs"], 1.1,
+                                         ctx_stride=c5["ctx_len"] + 2 * path_cap)
+        ctx_d, cl_d = to_dev(ctx), to_dev(cl)
+        res = fc.fc_retrieve(sources, ctx_d, cl_d, p)
+        root = to_dev(ctx[np.arange(B), cl - 1])
+        kvl = torch.zeros(B, dtype=torch.int32, device=dev)
+        tree = fc.fc_build_tree(res, [1, 1], root, kvl, c5["node_budget"], n_pad)
+        plen_h, rtok_h = synth.argmax_draws(rng, B, n_pad)
+        plen, rtok = to_dev(plen_h), to_dev(rtok_h)
+        am = fc.fc_synth_argmax(tree["tok"], tree["parent"], tree["n_nodes"], plen, rtok, synth.VOCAB)
+        acc = fc.fc_accept(tree["tok"], tree["parent"], tree["n_nodes"], am, path_cap)
+        kt = torch.randn((B, Hkv, n_pad, D), device=dev).to(torch.bfloat16)
+        kc = torch.zeros((B, Hkv, cap, D), dtype=torch.bfloat16, device=dev)
+        vc = torch.zeros_like(kc)
+        kv_out = torch.empty_like(kvl)
+        ctx_w = ctx_d.clone()
+        cl_out = torch.empty_like(cl_d)
+        root_out = torch.empty_like(root)
+        rc = fc.RetrievalCache(1 << max(10, int(2 * B - 1).bit_length()), S, p)
+        skip = torch.zeros(B, dtype=torch.int32, device=dev)
+        fc.fc_rcache_insert(rc, ctx_d, cl_d, skip, res)
+        got = fc.retrieve_outputs(S, B, p, dev)
+        assert fc.fc_get_error() == "FC_OK"
+        calls = {
+            "build_tree": lambda: fc.fc_build_tree(res, [1, 1], root, kvl, c5["node_budget"], n_pad, out=tree),
+            "synth_argmax": lambda: fc.fc_synth_argmax(tree["tok"], tree["parent"], tree["n_nodes"], plen, rtok,
+                                                       synth.VOCAB, out=am),
+            "accept": lambda: fc.fc_accept(tree["tok"], tree["parent"], tree["n_nodes"], am, path_cap, out=acc),
+            "kv_append": lambda: fc.fc_kv_append(acc, tree["tok"], kt, kt, kc, vc, kvl, kv_out, ctx_w, cl_d, cl_out,
+                                                 root_out),
+            "rcache_lookup_hit": lambda: fc.fc_rcache_lookup(rc, ctx_d, cl_d, None, skip, got),
+        }
+        a_len = acc["acc_len"].double()
+        nn = tree["n_nodes"].double()
+        alg = {  # algorithmic bytes of one call over the batch
+            "build_tree": B * (S * k * (d + 2) * 4 + S * 4 + 8) + B * (n_pad * (16 + n_pad // 8) + 4),
+            "synth_argmax": B * (n_pad * 16 + 8),
+            "accept": float((nn * 12).sum().item()) + B * (4 + 4 * (path_cap + 2)),
+            "kv_append": float(((a_len + 1) * Hkv * D * 2 * 2 * 2).sum().item()) + B * 4 * (4 + path_cap + 2),
+            "rcache_lookup_hit": B * (2 * S * (k * d + 2 * k + 2) * 4 + 4 * c5["n_max"] + 8),
+        }
+        rec = {"batch": B, "mean_tree_nodes": float(nn.mean().item()),
+               "mean_acc_len": float(a_len.mean().item())}
+        for nm, fn in calls.items():
+            ms = _gpu_ms(fn, reps=args.steps, warm=args.warmup)
+            rec[nm] = {"us": ms * 1e3, "us_per_sequence": ms * 1e3 / B, "alg_bytes": alg[nm],
+                       "gbs": alg[nm] / (ms * 1e-3) / 1e9, "hbm_frac": alg[nm] / (ms * 1e-3) / 1e9 / peak}
+        assert fc.fc_get_error() == "FC_OK" and int(skip.sum().item()) == B
+        rows.append(rec)
+        del kt, kc, vc
+        torch.cuda.empty_cache()
+    return {"metric": "small-kernel batch sweep", "value": None, "unit": "us", "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "config": {"workload": "the step's small kernels on two-source retrieval "
+                                                          "(5M + 100M), trees <= 128 nodes, GQA 8 KV heads"},
+            "hbm_peak_gbs": peak, "sweep": rows}
+
+
 def run_algorithm1(args, rank, ws, local):
     """The step loop of the default workload with Algorithm 1 in place of the
     replay cache: per sequence a CACHE (l = 50, 20-token output pieces,
@@ -1645,6 +1733,8 @@ def main(argv=None):
         out = run_gemm(args, rank, ws, local)
     elif args.mode == "build":
         out = run_build(args, rank, ws, local)
+    elif args.mode == "small":
+        out = run_small(args, rank, ws, local)
     else:
         out = run_ours(args, rank, ws, local)
     if rank == 0 and out is not None:
