@@ -56,9 +56,9 @@ UNIT = "steps/s"
 # ratio x the algorithmic bytes per launch of its own launches.  The ratio is valid
 # only for the kernel sources it was taken on (their SHA-256 below); otherwise the
 # bench reports traffic as null until it is measured again.
-ATTN_TRAFFIC = {"ratio": 1.0631,
+ATTN_TRAFFIC = {"ratio": 1.0632,
                 "sources": ["paper_2502_17139_gb300/csrc/tree_attn.cu", "paper_2502_17139_gb300/csrc/fc_common.cuh"],
-                "sha256": "387990e68e95a9a0f3410acd6298df6b55bfdf50d2440818de3c09d528bcecf2"}
+                "sha256": "e09792ea970a9ba2a02c4bb0e8df1e8d8784ca4f89f936405d073c9037f7d4dd"}
 
 WORKLOAD = ("full step loop: two-source datastore 100M (Zipf 1.1) + 5M (Zipf 1.3, 20k planted repeats) tokens, "
             "vocab 32256, batch 32, ctx 128, n 16->2, top-64 x 10 tokens per source, tree <=128 nodes, "

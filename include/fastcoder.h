@@ -522,6 +522,15 @@ fc_status fc_tree_attn(const void* d_q, const void* d_k_cache, const void* d_v_c
  * scheduling aid for filling the GPU. */
 size_t fc_tree_attn_workspace(int batch, int n_pad, int H, int Hkv);
 
+/* 1 if fc_tree_attn serves this shape with its streaming kernel on the
+ * current device, else 0 (also for an unsupported shape).  The streaming
+ * kernel takes launches whose groups fit one 128-row tile (H / Hkv * n_pad
+ * <= 128) and whose caches are short, with several groups per SM: each CTA
+ * serves groups in turn and overlaps one group's epilogue with the next one's
+ * query staging and first blocks.  Results equal the per-group kernel's.
+ * Host-only, launches nothing. */
+int fc_tree_attn_streamed(int batch, int n_pad, int H, int Hkv, int kv_cap);
+
 /* How many parts fc_tree_attn splits each row chunk's keys into for this
  * shape and workspace size on the current device (1 = no split; 0 for an
  * unsupported shape).  Host-only, launches nothing. */

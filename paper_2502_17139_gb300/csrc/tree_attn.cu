@@ -273,15 +273,15 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     return;
   }
 
-  // K and V of block j into stage j & 1 (the tree's own K/V form the last block)
+  // K and V of block j into stage j & 1 (the tree's own K/V form the last
+  // block; the tree maps' box is 128 rows, so rows >= n_pad arrive as zeros)
   auto load_kv = [&](int j, bool k_part) {
     const int st = j & 1;
     const bool tree = kb + j >= nblk_c;
-    const uint32_t bytes = tree ? (uint32_t)a.n_pad * 64 * 2 * 2 : TILE_BYTES;
     const CUtensorMap* m = k_part ? (tree ? &tm_kt : &tm_kc) : (tree ? &tm_vt : &tm_vc);
     const int y = tree ? 0 : (kb + j) * BN;
     const uint32_t dst = (k_part ? sK : sV) + st * TILE_BYTES, fb = bar((k_part ? B_KFULL : B_VFULL) + st);
-    mbar_expect_tx(fb, bytes);
+    mbar_expect_tx(fb, TILE_BYTES);
     tma_load_3d(dst, m, 0, y, bg, fb);
     tma_load_3d(dst + HALF_BYTES, m, 64, y, bg, fb);
   };
@@ -378,12 +378,16 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
           tc_mma_f16_tmem_a(tmem + 256 + x * 128, tmem + sb * 128 + kk * 8,
                             smem_desc_sw128(vb + kk * 2048, HALF_BYTES, 1024), IDESC_PV, (jj > 0 || kk > 0));
       };
-      auto zero_ragged_v = [&](int jj) {  // never let garbage (possibly NaN) rows meet a zero probability
+      // Never let garbage (possibly NaN) V rows meet a zero probability: the
+      // cache's rows past kv_len and the tree's rows past n_nodes (the tree
+      // tile's rows >= n_pad arrived as zeros).
+      auto zero_ragged_v = [&](int jj) {
         const int gj = kb + jj;
-        const int nv = (gj < nblk_c) ? min(BN, kvl - gj * BN) : nn;
-        if (nv < BN) {
+        const bool tree = gj >= nblk_c;
+        const int nv = tree ? nn : min(BN, kvl - gj * BN), top = tree ? a.n_pad : BN;
+        if (nv < top) {
           unsigned char* vt = smem + OFF_V + (jj & 1) * TILE_BYTES;
-          for (int e = lane; e < (BN - nv) * 16; e += 32) {
+          for (int e = lane; e < (top - nv) * 16; e += 32) {
             const int r = nv + (e >> 4), ch = e & 15;
             *reinterpret_cast<uint4*>(vt + (ch >> 3) * HALF_BYTES + r * 128 + (ch & 7) * 16) = make_uint4(0, 0, 0, 0);
           }
@@ -695,6 +699,454 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Streaming variant for short one-tile units: every group's rows fit one
+// 128-row tile (G * n_pad <= 128) and the caches are short, so a unit is a
+// handful of K/V blocks and a CTA per unit would pay its set-up (barriers,
+// tensor memory, Q staging, pipeline fill) and its epilogue for each few
+// blocks.  Here a CTA serves units blockIdx.x, blockIdx.x + gridDim.x, ... in
+// turn and keeps the pipeline full across them: one K/V stage ring runs over
+// the concatenated blocks of all its units, and Q and O alternate between two
+// buffers per unit (Q_A / Q_B in shared memory, O_A / O_B in tensor memory),
+// so warps 2-3 stage unit t + 1's queries and the MMA warp multiplies its
+// first blocks while the softmax warps still write unit t's output.  The
+// arithmetic per block is k_tree_attn's one-tile path, block for block, so the
+// results are the same.
+struct StreamUnit {
+  int b, g, nn, kvl, nblk_c, nblk;  // nblk = 0: no work (a length out of range, recorded)
+  bool bad;
+};
+
+__device__ __forceinline__ StreamUnit stream_unit(const AttnArgs& a, int u) {
+  StreamUnit su;
+  su.b = u / a.Hkv;
+  su.g = u - su.b * a.Hkv;
+  const int nn = a.n_nodes[su.b], kvl = a.kv_len[su.b];
+  su.bad = nn < 1 || nn > a.n_pad || kvl < 0 || kvl > a.kv_cap;
+  su.nn = su.bad ? 0 : nn;
+  su.kvl = su.bad ? 0 : kvl;
+  su.nblk_c = (su.kvl + BN - 1) / BN;
+  su.nblk = su.bad ? 0 : su.nblk_c + 1;  // + the tree block, the unit's last
+  return su;
+}
+
+// Walks a CTA's blocks in order: unit t (the t-th of this CTA), its block j,
+// and `live` = how many units with work came before (it picks the Q and O
+// buffers and their barrier phases).
+struct StreamCursor {
+  int t, j, live, n_units;
+  StreamUnit su;
+  __device__ __forceinline__ bool valid() const { return t < n_units; }
+  __device__ __forceinline__ void skip_empty(const AttnArgs& a) {
+    while (t < n_units && su.nblk == 0) {
+      ++t;
+      if (t < n_units) su = stream_unit(a, (int)blockIdx.x + t * (int)gridDim.x);
+    }
+  }
+  __device__ __forceinline__ void start(const AttnArgs& a, int n) {
+    t = 0, j = 0, live = 0, n_units = n;
+    if (n > 0) su = stream_unit(a, (int)blockIdx.x);
+    skip_empty(a);
+  }
+  __device__ __forceinline__ void next(const AttnArgs& a) {
+    if (++j < su.nblk) return;
+    j = 0;
+    ++live;
+    ++t;
+    if (t < n_units) su = stream_unit(a, (int)blockIdx.x + t * (int)gridDim.x);
+    skip_empty(a);
+  }
+};
+
+// Shared-memory layout and barrier slots of the streaming kernel with NST K/V
+// stages.  With three stages the Q buffers hold 64 rows (the launch's groups
+// have G * n_pad <= 64 rows): the 128-row MMA then reads 64 rows past each
+// buffer, rows whose scores no output row uses.
+template <int NST>
+struct StreamLayout {
+  static constexpr int QROWS = NST == 3 ? 64 : 128;
+  static constexpr uint32_t QHALF = QROWS * 128, QTILE = 2 * QHALF;
+  static constexpr uint32_t OFF_Q = 0;                           // Q buffers 0, 1
+  static constexpr uint32_t OFF_K = OFF_Q + 2 * QTILE;           // NST stages
+  static constexpr uint32_t OFF_V = OFF_K + NST * TILE_BYTES;    // NST stages
+  static constexpr uint32_t OFF_BAR = OFF_V + NST * TILE_BYTES;
+  static constexpr uint32_t SMEM = OFF_BAR + 256 + 1024;         // + alignment slack
+  // barrier slots (8 bytes each)
+  static constexpr int KFULL = 0, VFULL = NST, KEMPTY = 2 * NST, VEMPTY = 3 * NST;  // [NST] each
+  static constexpr int SFULL = 4 * NST;       // [2] S buffer ready
+  static constexpr int PFULL = SFULL + 2;     // [2] P written into S buffer (128 arrivals)
+  static constexpr int ODONE = PFULL + 2;     // a PV into O done (one completion per block)
+  static constexpr int DRAIN = ODONE + 1;     // MMA drain on abort
+  static constexpr int OFIN = DRAIN + 1;      // [2] the last PV of a unit into O buffer done
+  static constexpr int OFREE = OFIN + 2;      // [2] the softmax warps have read O buffer out (128 arrivals)
+  static constexpr int QFULL = OFREE + 2;     // [2] Q buffer staged (64 arrivals, warps 2-3)
+  static constexpr int QFREE = QFULL + 2;     // [2] the last QK reading Q buffer done
+  static constexpr int NBARS = QFREE + 2;
+  static_assert(NBARS * 8 <= 256, "barrier area");
+  static_assert(SMEM + 1024 <= 232448, "shared memory per CTA (the kernel's static part is 1024 bytes)");
+};
+// Register split of the streaming kernel: the softmax warpgroup rises to
+// REGS_SOFTMAX, warps 8-11 (idle) keep the launch's count, and the producer
+// warpgroup (two block cursors in the MMA warp) drops to what is left.
+constexpr int REGS_PRODUCER_STREAM = 96;
+static_assert(128 * REGS_PRODUCER_STREAM + 128 * REGS_SOFTMAX + 128 * REGS_LAUNCH <= TA_THREADS * REGS_LAUNCH,
+              "register split");
+
+template <int NST>
+__global__ void __launch_bounds__(TA_THREADS, 1)
+    k_tree_attn_stream(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
+                       const __grid_constant__ CUtensorMap tm_kt, const __grid_constant__ CUtensorMap tm_vt,
+                       AttnArgs a) {
+  using L = StreamLayout<NST>;
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int U = a.B * a.Hkv;
+  const int n_units = max(0, (U - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x);
+  unsigned char* smem =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t sQ = sbase + L::OFF_Q, sK = sbase + L::OFF_K, sV = sbase + L::OFF_V;
+  const uint32_t bar0 = sbase + L::OFF_BAR;
+  auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
+
+  // K or V of global block J (block j of unit su) into stage J % NST.  The tree
+  // maps' box is 128 rows: rows >= n_pad arrive as zeros.
+  auto load_kv = [&](int J, const StreamUnit& su, int j, bool k_part) {
+    const int st = J % NST;
+    const bool tree = j >= su.nblk_c;
+    const CUtensorMap* m = k_part ? (tree ? &tm_kt : &tm_kc) : (tree ? &tm_vt : &tm_vc);
+    const int y = tree ? 0 : j * BN, z = su.b * a.Hkv + su.g;
+    const uint32_t dst = (k_part ? sK : sV) + st * TILE_BYTES, fb = bar((k_part ? L::KFULL : L::VFULL) + st);
+    mbar_expect_tx(fb, TILE_BYTES);
+    tma_load_3d(dst, m, 0, y, z, fb);
+    tma_load_3d(dst + HALF_BYTES, m, 64, y, z, fb);
+  };
+  if (tid == 0) {
+    s_abort = 0;
+    for (int i = 0; i < L::NBARS; ++i) {
+      const bool p128 = i == L::PFULL || i == L::PFULL + 1 || i == L::OFREE || i == L::OFREE + 1;
+      const bool q64 = i == L::QFULL || i == L::QFULL + 1;
+      mbar_init(bar(i), p128 ? 128u : (q64 ? 64u : 1u));
+    }
+    fence_mbar_init();
+    prefetch_tmap(&tm_kc);
+    prefetch_tmap(&tm_vc);
+    prefetch_tmap(&tm_kt);
+    prefetch_tmap(&tm_vt);
+    StreamCursor c;
+    c.start(a, n_units);
+    for (int J = 0; J < NST && c.valid(); ++J, c.next(a)) {  // the stages are free: start the first copies now
+      load_kv(J, c.su, c.j, true);
+      load_kv(J, c.su, c.j, false);
+    }
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&s_tmem), TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+  if (warp < 4) {
+    regs_dec<REGS_PRODUCER_STREAM>();
+    if (warp == 0) {
+      // ---------------- TMA producer: the CTA's blocks in order ----------------
+      if (lane == 0) {
+        StreamCursor c;
+        c.start(a, n_units);
+        int J = 0, issued = 0;
+        for (; c.valid(); ++J, c.next(a)) {
+          if (J < NST) {
+            issued = J + 1;
+            continue;
+          }
+          const int st = J % NST;
+          const uint32_t par = ((J / NST) - 1) & 1;
+          if (!mbar_wait_bounded(bar(L::KEMPTY + st), par, &s_abort, WAIT_CYCLES)) break;
+          load_kv(J, c.su, c.j, true);
+          if (!mbar_wait_bounded(bar(L::VEMPTY + st), par, &s_abort, WAIT_CYCLES)) {
+            issued = J + 1;  // the K copy of this block is in flight
+            break;
+          }
+          load_kv(J, c.su, c.j, false);
+          issued = J + 1;
+        }
+        if (s_abort) {  // let the copies already issued land before the CTA exits
+          volatile int dummy = 0;
+          for (int j = max(0, issued - NST); j < issued; ++j) {
+            mbar_wait_bounded(bar(L::KFULL + j % NST), (j / NST) & 1, &dummy, DRAIN_CYCLES);
+            mbar_wait_bounded(bar(L::VFULL + j % NST), (j / NST) & 1, &dummy, DRAIN_CYCLES);
+          }
+        }
+      }
+      __syncwarp();
+    } else if (warp >= 2) {
+      // ---------------- warps 2-3: each unit's queries into its Q buffer, and
+      // the zero rows of nodes >= n_nodes ----------------
+      const int t0 = tid - 64;  // 0..63
+      int live = 0;
+      bool ok = true;
+      for (int t = 0; t < n_units && ok; ++t) {
+        const StreamUnit su = stream_unit(a, (int)blockIdx.x + t * (int)gridDim.x);
+        if (su.bad && t0 == 0) fc_flag(FC_ERR_WORD(a.err), FC_EBIT_INVALID);
+        const int pad = a.n_pad - su.nn;
+        for (int e = t0; e < a.G * pad * (HD / 8); e += 64) {  // padding rows (all rows of a bad unit)
+          const int r = e / (HD / 8), ch = e % (HD / 8);
+          const int hh = r / pad, i = su.nn + (r - hh * pad);
+          reinterpret_cast<uint4*>(a.out + (((size_t)su.b * a.n_pad + i) * a.H + su.g * a.G + hh) * HD)[ch] =
+              make_uint4(0, 0, 0, 0);
+        }
+        if (su.nblk == 0) continue;
+        const int q = live & 1;
+        if (live >= 2 && !(ok = warp_wait(bar(L::QFREE + q), ((live >> 1) - 1) & 1, &s_abort))) break;
+        const int rows_total = a.G * su.nn;
+        unsigned char* qt = smem + L::OFF_Q + q * L::QTILE;
+        for (int e = t0; e < L::QROWS * 16; e += 64) {
+          const int r = e >> 4, ch = e & 15, half = ch >> 3, gran = ch & 7;
+          uint4 v = make_uint4(0, 0, 0, 0);
+          if (r < rows_total) {
+            const int hh = r / su.nn, i = r - hh * su.nn;
+            v = reinterpret_cast<const uint4*>(a.q + (((size_t)su.b * a.n_pad + i) * a.H + su.g * a.G + hh) * HD)[ch];
+          }
+          *reinterpret_cast<uint4*>(qt + half * L::QHALF + r * 128 + ((gran ^ (r & 7)) << 4)) = v;
+        }
+        fence_proxy_async_smem();
+        mbar_arrive(bar(L::QFULL + q));
+        ++live;
+      }
+    } else {
+      // ---------------- MMA issuer (+ padding V rows of tree blocks zeroed) -------
+      constexpr uint32_t IDESC_QK = idesc_bf16_f32(BM, BN, 0);
+      constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, HD, 1);
+      bool ok = true;
+      // S buffer J & 1 <- Q buffer q . K(stage J % NST)^T
+      auto issue_qk = [&](int J, int q) {
+        const uint32_t kb = sK + (J % NST) * TILE_BYTES, qb = sQ + q * L::QTILE;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          tc_mma_f16(tmem + (J & 1) * 128, smem_desc_sw128(qb + (kk >> 2) * L::QHALF + (kk & 3) * 32, 16, 1024),
+                     smem_desc_sw128(kb + (kk >> 2) * HALF_BYTES + (kk & 3) * 32, 16, 1024), IDESC_QK, kk > 0);
+        }
+        tc_commit(bar(L::SFULL + (J & 1)));
+      };
+      // the QK of the block under cursor c (global index J), once its Q and K are there
+      auto qk_step = [&](const StreamCursor& c, int J) -> bool {
+        const int q = c.live & 1;
+        if (c.j == 0 && !warp_wait(bar(L::QFULL + q), (c.live >> 1) & 1, &s_abort)) return false;
+        if (!warp_wait(bar(L::KFULL + J % NST), (J / NST) & 1, &s_abort)) return false;
+        tc_fence_after();
+        issue_qk(J, q);
+        tc_commit(bar(L::KEMPTY + J % NST));
+        if (c.j == c.su.nblk - 1) tc_commit(bar(L::QFREE + q));  // the unit's last QK: its Q buffer frees
+        return true;
+      };
+      StreamCursor cq, cp;
+      cq.start(a, n_units);
+      cp = cq;
+      int Jq = 0;
+      for (; ok && Jq < 2 && cq.valid(); ++Jq, cq.next(a)) ok = qk_step(cq, Jq);
+      for (int J = 0; ok && cp.valid(); ++J, cp.next(a)) {
+        const int st = J % NST, o = cp.live & 1;
+        if (!(ok = warp_wait(bar(L::VFULL + st), (J / NST) & 1, &s_abort))) break;
+        {  // never let garbage (possibly NaN) V rows meet a zero probability: the
+           // cache's rows past kv_len and the tree's rows past n_nodes (the tree
+           // tile's rows >= n_pad arrived as zeros)
+          const bool tree = cp.j >= cp.su.nblk_c;
+          const int nv = tree ? cp.su.nn : min(BN, cp.su.kvl - cp.j * BN);
+          const int top = tree ? a.n_pad : BN;
+          if (nv < top) {
+            unsigned char* vt = smem + L::OFF_V + st * TILE_BYTES;
+            for (int e = lane; e < (top - nv) * 16; e += 32) {
+              const int r = nv + (e >> 4), ch = e & 15;
+              *reinterpret_cast<uint4*>(vt + (ch >> 3) * HALF_BYTES + r * 128 + (ch & 7) * 16) =
+                  make_uint4(0, 0, 0, 0);
+            }
+            fence_proxy_async_smem();
+          }
+          __syncwarp();
+        }
+        if (!(ok = warp_wait(bar(L::PFULL + (J & 1)), (J >> 1) & 1, &s_abort))) break;
+        // a unit's first PV overwrites its O buffer: the unit two back must be read out
+        if (cp.j == 0 && cp.live >= 2 && !(ok = warp_wait(bar(L::OFREE + o), ((cp.live >> 1) - 1) & 1, &s_abort)))
+          break;
+        tc_fence_after();
+        {
+          const uint32_t vb = sV + st * TILE_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < BN / 16; ++kk)  // 8 packed columns per 16 keys
+            tc_mma_f16_tmem_a(tmem + 256 + o * 128, tmem + (J & 1) * 128 + kk * 8,
+                              smem_desc_sw128(vb + kk * 2048, HALF_BYTES, 1024), IDESC_PV, (cp.j > 0 || kk > 0));
+        }
+        tc_commit(bar(L::ODONE));
+        tc_commit(bar(L::VEMPTY + st));
+        if (cp.j == cp.su.nblk - 1) tc_commit(bar(L::OFIN + o));
+        if (cq.valid()) {  // QK two blocks ahead, into the S buffer PV(J) has just read
+          ok = qk_step(cq, Jq);
+          ++Jq;
+          cq.next(a);
+        }
+      }
+      if (__any_sync(0xFFFFFFFFu, s_abort)) {  // let issued MMAs retire before the tensor memory is freed
+        tc_commit(bar(L::DRAIN));
+        volatile int dummy = 0;
+        mbar_wait_bounded(bar(L::DRAIN), 0, &dummy, DRAIN_CYCLES);
+      }
+    }
+  } else {
+    if (warp < 8) {
+      regs_inc<REGS_SOFTMAX>();
+      // ---------------- softmax warpgroup: thread = row of the unit's tile ----------------
+      const int q4 = warp & 3;
+      const int r = q4 * 32 + lane;
+      const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+      StreamCursor c;
+      c.start(a, n_units);
+      bool ok = true;
+      const int nw = a.n_pad / 64;
+      bool row_ok = false;
+      __nv_bfloat16* dst = nullptr;
+      uint64_t m0 = 0, m1 = 0;
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int J = 0; ok && c.valid(); ++J, c.next(a)) {
+        const int o = c.live & 1;
+        const uint32_t tO = tmem + 256 + o * 128 + lane_off;
+        if (c.j == 0) {  // a new unit: its row, mask row (first read in its last block) and running state
+          row_ok = r < a.G * c.su.nn;
+          const int hh = row_ok ? r / c.su.nn : 0, i = row_ok ? r - hh * c.su.nn : 0;
+          dst = a.out + (((size_t)c.su.b * a.n_pad + i) * a.H + c.su.g * a.G + hh) * HD;
+          const uint64_t* mrow = a.mask + ((size_t)c.su.b * a.n_pad + i) * nw;
+          m0 = mrow[0];
+          m1 = (nw > 1) ? mrow[1] : 0ull;
+          m_run = -INFINITY;
+          l_run = 0.f;
+        }
+        const int sb = J & 1;
+        const uint32_t tS = tmem + sb * 128 + lane_off;
+        if (!(ok = warp_wait(bar(L::SFULL + sb), (J >> 1) & 1, &s_abort))) break;
+        tc_fence_after();
+        const bool tree = c.j == c.su.nblk - 1;
+        if (q4 * 32 >= L::QROWS) {  // lanes past the Q buffer's rows: no output row, keep the phases only
+          tc_fence_before();
+          mbar_arrive(bar(L::PFULL + sb));
+          if (tree) {
+            if (!(ok = warp_wait(bar(L::OFIN + o), (c.live >> 1) & 1, &s_abort))) break;
+            tc_fence_after();
+            tc_fence_before();
+            mbar_arrive(bar(L::OFREE + o));
+          }
+          continue;
+        }
+        const int nv = tree ? BN : min(BN, c.su.kvl - c.j * BN);
+        const bool masked = tree || nv < BN;  // block-uniform
+        auto keep_bits = [&](int q) -> uint32_t {
+          if (tree) return (uint32_t)((q < 2 ? m0 : m1) >> (32 * (q & 1)));
+          const int lo = nv - 32 * q;
+          return lo >= 32 ? 0xFFFFFFFFu : (lo <= 0 ? 0u : ((1u << lo) - 1u));
+        };
+        uint32_t sv[128];
+#pragma unroll
+        for (int c4 = 0; c4 < 4; ++c4) tmem_ld32(tS + c4 * 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[c4 * 32]));
+        tc_wait_ld();
+        if (masked) {
+#pragma unroll
+          for (int c4 = 0; c4 < 4; ++c4) {
+            const uint32_t kbits = keep_bits(c4);
+#pragma unroll
+            for (int cc = 0; cc < 32; ++cc)
+              if (!(kbits & (1u << cc))) sv[c4 * 32 + cc] = __float_as_uint(-INFINITY);
+          }
+        }
+        float pm[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
+#pragma unroll
+        for (int cc = 0; cc < 128; cc += 2)
+          pm[(cc >> 1) & 7] = fmax3(pm[(cc >> 1) & 7], __uint_as_float(sv[cc]), __uint_as_float(sv[cc + 1]));
+        const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * a.scale_log2;
+        const float m_new = (mx > m_run + RESCALE_THRESHOLD) ? mx : m_run;
+        const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
+        const float alpha = fast_exp2(m_run - m_use);
+        // PV of the unit's previous block may still run: wait for it
+        if (c.j > 0 && __any_sync(0xFFFFFFFFu, alpha != 1.f)) {
+          if (!(ok = warp_wait(bar(L::ODONE), (J - 1) & 1, &s_abort))) break;
+          tc_fence_after();
+#pragma unroll
+          for (int cc = 0; cc < HD / 32; ++cc) {
+            uint32_t ov[32];
+            tmem_ld32(tO + cc * 32, ov);
+            tc_wait_ld();
+#pragma unroll
+            for (int u = 0; u < 32; ++u) ov[u] = __float_as_uint(__uint_as_float(ov[u]) * alpha);
+            tmem_st32(tO + cc * 32, ov);
+          }
+        }
+        uint64_t ps2[4] = {0ull, 0ull, 0ull, 0ull};
+        const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2), nm2 = f2_pack(-m_use, -m_use);
+#pragma unroll
+        for (int c4 = 0; c4 < 4; ++c4) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int qq = 0; qq < 16; ++qq) {
+            const int cc = c4 * 32 + 2 * qq;
+            float x0, x1;
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sv[cc]), __uint_as_float(sv[cc + 1])), sc2, nm2), x0, x1);
+            const float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
+            ps2[qq & 3] = f2_add(ps2[qq & 3], f2_pack(p0, p1));
+            pk[qq] = pack_bf16x2(p0, p1);
+          }
+          tmem_st16(tS + c4 * 16, pk);
+        }
+        tc_wait_st();
+        float ps[8];
+        f2_unpack(ps2[0], ps[0], ps[1]);
+        f2_unpack(ps2[1], ps[2], ps[3]);
+        f2_unpack(ps2[2], ps[4], ps[5]);
+        f2_unpack(ps2[3], ps[6], ps[7]);
+        const float sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+        l_run = l_run * alpha + sum;
+        m_run = m_new;
+        tc_fence_before();
+        mbar_arrive(bar(L::PFULL + sb));
+        if (tree) {  // the unit's last block: read its O out, then free the buffer
+          if (!(ok = warp_wait(bar(L::OFIN + o), (c.live >> 1) & 1, &s_abort))) break;
+          tc_fence_after();
+          const float inv = 1.f / l_run;
+#pragma unroll
+          for (int cc = 0; cc < HD / 32; ++cc) {
+            uint32_t ov[32];
+            tmem_ld32(tO + cc * 32, ov);
+            tc_wait_ld();
+            if (row_ok) {
+#pragma unroll
+              for (int u = 0; u < 32; u += 8) {
+                uint4 v;
+                v.x = pack_bf16x2(__uint_as_float(ov[u + 0]) * inv, __uint_as_float(ov[u + 1]) * inv);
+                v.y = pack_bf16x2(__uint_as_float(ov[u + 2]) * inv, __uint_as_float(ov[u + 3]) * inv);
+                v.z = pack_bf16x2(__uint_as_float(ov[u + 4]) * inv, __uint_as_float(ov[u + 5]) * inv);
+                v.w = pack_bf16x2(__uint_as_float(ov[u + 6]) * inv, __uint_as_float(ov[u + 7]) * inv);
+                *reinterpret_cast<uint4*>(dst + cc * 32 + u) = v;
+              }
+            }
+          }
+          tc_fence_before();
+          mbar_arrive(bar(L::OFREE + o));
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (tid == 0 && s_abort) fc_flag(FC_ERR_WORD(a.err), FC_EBIT_TIMEOUT);
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------------------
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   static std::once_flag once;
@@ -767,6 +1219,24 @@ SplitPlan choose_split(uint64_t units, int kv_cap, size_t ws_bytes) {
   return sp;
 }
 
+// Which kernel serves a launch of one-tile units (G * n_pad <= 128, caches
+// of at most STREAM_MAX_KV keys; RoPE launches keep the per-unit kernel).
+// Per-unit CTAs pay a unit's set-up and epilogue, about
+// STREAM_OVERHEAD_BLOCKS blocks' time, on top of its nb blocks; streaming
+// CTAs pay them once but each serves ceil(units / SMs) whole units, where
+// per-unit CTAs spread units / SMs (and split the last wave's keys).  The
+// streaming kernel is chosen when its estimate is no longer.
+constexpr int STREAM_MAX_KV = 4096;
+constexpr int STREAM_OVERHEAD_BLOCKS = 3;
+bool use_stream(uint64_t units, int G, int n_pad, int kv_cap, bool rope) {
+  if (rope || G * n_pad > BM || kv_cap > STREAM_MAX_KV) return false;
+  const int sms = sm_count();
+  if (sms <= 0 || units <= (uint64_t)sms) return false;
+  const uint64_t nb = (uint64_t)(kv_cap + BN - 1) / BN + 1;
+  const uint64_t waves = (units + sms - 1) / sms;
+  return waves * nb * (uint64_t)sms <= units * (nb + STREAM_OVERHEAD_BLOCKS);
+}
+
 uint64_t attn_units(int batch, int n_pad, int H, int Hkv) {
   return (uint64_t)batch * Hkv * (((uint64_t)(H / Hkv) * n_pad + TILES * BM - 1) / (TILES * BM));
 }
@@ -812,9 +1282,16 @@ extern "C" size_t fc_tree_attn_workspace(int batch, int n_pad, int H, int Hkv) {
   return ws_layout(std::min<uint64_t>(units, (uint64_t)std::max(sms, 1)), MAX_PARTS).total;
 }
 
+extern "C" int fc_tree_attn_streamed(int batch, int n_pad, int H, int Hkv, int kv_cap) {
+  if (batch < 1 || H < 1 || Hkv < 1 || kv_cap < 1 || H % Hkv != 0 || (n_pad != 64 && n_pad != 128)) return 0;
+  return use_stream(attn_units(batch, n_pad, H, Hkv), H / Hkv, n_pad, kv_cap, false) ? 1 : 0;
+}
+
 extern "C" int fc_tree_attn_parts(int batch, int n_pad, int H, int Hkv, int kv_cap, size_t ws_bytes) {
   if (batch < 1 || H < 1 || Hkv < 1 || kv_cap < 1 || H % Hkv != 0 || (n_pad != 64 && n_pad != 128)) return 0;
-  return choose_split(attn_units(batch, n_pad, H, Hkv), kv_cap, ws_bytes).parts;
+  const uint64_t units = attn_units(batch, n_pad, H, Hkv);
+  if (use_stream(units, H / Hkv, n_pad, kv_cap, false)) return 1;  // no key split there
+  return choose_split(units, kv_cap, ws_bytes).parts;
 }
 
 static fc_status launch_tree_attn(const void* d_q, const void* d_k_cache, const void* d_v_cache, int kv_cap,
@@ -837,17 +1314,21 @@ static fc_status launch_tree_attn(const void* d_q, const void* d_k_cache, const 
   const int G = H / Hkv;
   const int ctas = (G * n_pad + TILES * BM - 1) / (TILES * BM);
   const uint64_t units = attn_units(batch, n_pad, H, Hkv);
-  const SplitPlan sp = choose_split(units, kv_cap, d_ws ? ws_bytes : 0);
+  const bool streamed = use_stream(units, G, n_pad, kv_cap, d_pos != nullptr);
+  const SplitPlan sp = streamed ? SplitPlan{units, 1} : choose_split(units, kv_cap, d_ws ? ws_bytes : 0);
   const uint64_t n_split = units - sp.u_split;
-  const uint64_t grid = sp.u_split + n_split * sp.parts;
+  const uint64_t grid = streamed ? (uint64_t)sm_count() : sp.u_split + n_split * sp.parts;
   if (grid > 0x7FFFFFFFull) return FC_ERR_UNSUPPORTED;
   CUtensorMap mkc, mvc, mkt, mvt;
   if (!make_map(&mkc, d_k_cache, (uint64_t)kv_cap, groups, BN) || !make_map(&mvc, d_v_cache, (uint64_t)kv_cap, groups, BN) ||
-      !make_map(&mkt, d_k_tree, (uint64_t)n_pad, groups, (uint32_t)n_pad) ||
-      !make_map(&mvt, d_v_tree, (uint64_t)n_pad, groups, (uint32_t)n_pad))
+      !make_map(&mkt, d_k_tree, (uint64_t)n_pad, groups, BN) || !make_map(&mvt, d_v_tree, (uint64_t)n_pad, groups, BN))
     return FC_ERR_CUDA;
-  auto kern = d_pos ? k_tree_attn<true> : k_tree_attn<false>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES) != cudaSuccess)
+  // the streaming kernel keeps three K/V stages when a group's rows fit 64
+  const bool three = streamed && G * n_pad <= 64;
+  auto kern = streamed ? (three ? k_tree_attn_stream<3> : k_tree_attn_stream<2>)
+                       : (d_pos ? k_tree_attn<true> : k_tree_attn<false>);
+  const uint32_t smem_bytes = streamed ? (three ? StreamLayout<3>::SMEM : StreamLayout<2>::SMEM) : SMEM_BYTES;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes) != cudaSuccess)
     return FC_ERR_CUDA;
   {  // the register split needs the whole launch allocation (see REGS_LAUNCH)
     cudaFuncAttributes fa;
@@ -885,7 +1366,7 @@ static fc_status launch_tree_attn(const void* d_q, const void* d_k_cache, const 
     if (cudaMemsetAsync(a.ws_cnt, 0, n_split * 2 * sizeof(int), static_cast<cudaStream_t>(stream)) != cudaSuccess)
       return FC_ERR_CUDA;
   }
-  kern<<<(unsigned)grid, TA_THREADS, SMEM_BYTES, static_cast<cudaStream_t>(stream)>>>(mkc, mvc, mkt, mvt, a);
+  kern<<<(unsigned)grid, TA_THREADS, smem_bytes, static_cast<cudaStream_t>(stream)>>>(mkc, mvc, mkt, mvt, a);
   return FC_CHECK_LAUNCH();
 }
 

@@ -76,7 +76,7 @@ EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build
            "fc_datastore_build_noalloc", "fc_datastore_keys", "fc_datastore_save", "fc_datastore_file_info", "fc_datastore_load",
            "fc_retrieve", "fc_retrieve_all", "fc_retrieve_rev", "fc_reverse_tokens", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
-           "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_gemm_kv_heads", "fc_gemm_silu_mul", "fc_interleave_gate_up", "fc_embed",
+           "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_tree_attn_streamed", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_gemm_kv_heads", "fc_gemm_silu_mul", "fc_interleave_gate_up", "fc_embed",
            "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax",
            "fc_pipeline_create", "fc_pipeline_step", "fc_pipeline_stream", "fc_pipeline_error", "fc_pipeline_join",
            "fc_pipeline_destroy"]
@@ -143,6 +143,7 @@ def _load():
         "fc_tree_attn_rope": (C.c_int, [vp, vp, vp, i32, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, C.c_float, vp,
                                         C.c_float, vp, vp, sz, vp]),
         "fc_tree_attn_parts": (C.c_int, [i32, i32, i32, i32, i32, sz]),
+        "fc_tree_attn_streamed": (C.c_int, [i32, i32, i32, i32, i32]),
         "fc_accept": (C.c_int, [vp, vp, vp, vp, i32, i32, vp, vp, i32, vp, vp]),
         "fc_argmax_accept": (C.c_int, [vp, i32, vp, vp, vp, i32, i32, vp, vp, vp, i32, vp, vp]),
         "fc_kv_append": (C.c_int, [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, i32,

@@ -488,6 +488,89 @@ def test_attn_kv_split_two_tiles(fc, orc):
     _attn_case(fc, orc, 7, B, 128, 32, 8, kvl, 2048, nn=nn, full_rows=False, want_parts=2)
 
 
+def test_attn_stream_c1_shape(fc, orc):
+    """The c1 launch (1024 one-tile groups, 512-key caches) runs on the
+    streaming kernel: several groups per CTA."""
+    assert fc.LIB.fc_tree_attn_streamed(32, 64, 32, 32, 512) == 1
+    assert fc.LIB.fc_tree_attn_streamed(16, 64, 32, 32, 4096) == 0  # c3: long caches, per-group CTAs
+    assert fc.LIB.fc_tree_attn_streamed(32, 128, 32, 8, 16384) == 0  # two-tile groups
+
+
+def test_attn_stream_ragged(fc, orc):
+    """Streaming kernel, one head per group: ragged caches (empty, one key,
+    block edges) and trees (one node to full), every row against the oracle."""
+    B, H = 40, 16
+    assert fc.LIB.fc_tree_attn_streamed(B, 64, H, H, 512) == 1
+    base_k, base_n = [0, 1, 127, 128, 129, 300, 511, 512], [1, 2, 63, 64, 64, 5, 1, 33]
+    kvl = [base_k[b % 8] for b in range(B)]
+    nn = [base_n[(b * 3) % 8] for b in range(B)]
+    _attn_case(fc, orc, 21, B, 64, H, H, kvl, 512, nn=nn)
+
+
+def test_attn_stream_gqa2(fc, orc):
+    """Streaming kernel with two query heads per group (128 rows of 64-node
+    trees) and caches up to 1000 keys."""
+    B, H, Hkv = 80, 16, 8
+    assert fc.LIB.fc_tree_attn_streamed(B, 64, H, Hkv, 1024) == 1
+    rng = synth.rng_for(53)
+    kvl = [int(rng.integers(0, 1001)) if b % 5 else [0, 1000][b % 2] for b in range(B)]
+    _attn_case(fc, orc, 22, B, 64, H, Hkv, kvl, 1024, full_rows=False, sample=3000)
+
+
+def test_attn_stream_matches_per_group_kernel(fc, orc):
+    """The same sequences through the streaming kernel (40 sequences, 320
+    groups) and through the per-group kernel (the first 19: 152 groups, one
+    wave, no key split): bit-identical outputs."""
+    B, H, n_pad, cap = 40, 8, 64, 512
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    Bs = sms // H
+    assert fc.LIB.fc_tree_attn_streamed(B, n_pad, H, H, cap) == 1
+    assert fc.LIB.fc_tree_attn_streamed(Bs, n_pad, H, H, cap) == 0
+    rng = synth.rng_for(54)
+    tok, par, nn = _random_trees(rng, B, n_pad)
+    kvl = rng.integers(0, cap + 1, B).astype(np.int32)
+    q = synth.randn_bf16((B, n_pad, H, 128), 61, "cuda")
+    kc = synth.randn_bf16((B, H, cap, 128), 62, "cuda")
+    vc = synth.randn_bf16((B, H, cap, 128), 63, "cuda")
+    kt = synth.randn_bf16((B, H, n_pad, 128), 64, "cuda")
+    vt = synth.randn_bf16((B, H, n_pad, 128), 65, "cuda")
+    gm = fc.fc_tree_mask(dev(par), dev(nn), dev(kvl))
+    out = fc.fc_tree_attn(q, kc, vc, dev(kvl), kt, vt, gm["mask"], dev(nn))
+    part = fc.fc_tree_attn(q[:Bs].contiguous(), kc[:Bs].contiguous(), vc[:Bs].contiguous(), dev(kvl[:Bs]),
+                           kt[:Bs].contiguous(), vt[:Bs].contiguous(), gm["mask"][:Bs].contiguous(), dev(nn[:Bs]))
+    torch.cuda.synchronize()
+    check_no_error(fc)
+    assert torch.equal(out[:Bs], part)
+
+
+def test_attn_stream_bad_length(fc, orc):
+    """A node count out of range in one sequence: FC_ERR_INVALID_ARG, that
+    sequence's rows all zero, every other sequence still right."""
+    B, H, n_pad, cap = 40, 8, 64, 512
+    assert fc.LIB.fc_tree_attn_streamed(B, n_pad, H, H, cap) == 1
+    rng = synth.rng_for(55)
+    tok, par, nn = _random_trees(rng, B, n_pad)
+    kvl = rng.integers(0, cap + 1, B).astype(np.int32)
+    q = synth.randn_bf16((B, n_pad, H, 128), 71, "cuda")
+    kc = synth.randn_bf16((B, H, cap, 128), 72, "cuda")
+    vc = synth.randn_bf16((B, H, cap, 128), 73, "cuda")
+    kt = synth.randn_bf16((B, H, n_pad, 128), 74, "cuda")
+    vt = synth.randn_bf16((B, H, n_pad, 128), 75, "cuda")
+    gm = fc.fc_tree_mask(dev(par), dev(nn), dev(kvl))
+    good = fc.fc_tree_attn(q, kc, vc, dev(kvl), kt, vt, gm["mask"], dev(nn))
+    torch.cuda.synchronize()
+    check_no_error(fc)
+    bad_nn = nn.copy()
+    bad_nn[17] = n_pad + 1
+    out = torch.full_like(q, float("nan"))
+    fc.fc_tree_attn(q, kc, vc, dev(kvl), kt, vt, gm["mask"], dev(bad_nn), out=out)
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_ERR_INVALID_ARG"
+    assert (out[17] == 0).all()
+    keep = [b for b in range(B) if b != 17]
+    assert torch.equal(out[keep], good[keep])
+
+
 def test_attn_c3_shape_full(fc, orc):
     # c3: B=16, H=Hkv=32, KV 4096, 64-node trees; every row against the fp64 oracle
     _attn_case(fc, orc, 5, 16, 64, 32, 32, [4096] * 16, 4096, nn=[64] * 16)
