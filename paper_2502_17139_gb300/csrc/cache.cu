@@ -781,18 +781,26 @@ extern "C" fc_status fc_cache_search(const fc_cache* cache, const void* d_missin
   if (batch == 0) return FC_OK;
   if (!d_ctx || !d_ctx_len || !d_drafts || !d_draft_len || !d_count || !d_n_drafts || !d_match_len || !d_state)
     return FC_ERR_INVALID_ARG;
-  static size_t smem_limit = 0;
-  if (!smem_limit) {
-    int dev = 0, optin = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
-      return FC_ERR_CUDA;
+  // the device's opt-in shared memory per block, set as the kernel's limit once per device
+  static std::atomic<unsigned long long> attr_done;
+  static std::atomic<size_t> dev_limit[64];
+  size_t smem_limit = 0;
+  const fc_status st = fc_once_per_device(attr_done, [&](int dev) {
+    int optin = 0;
+    if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return FC_ERR_CUDA;
     const size_t limit = (size_t)optin;
-    const size_t most = cs_smem_bytes(FC_CACHE_MAX_WORDS, cs_rows_cap(FC_CACHE_MAX_WORDS, limit));
-    if (most > limit) return FC_ERR_INTERNAL;
+    if (cs_smem_bytes(FC_CACHE_MAX_WORDS, cs_rows_cap(FC_CACHE_MAX_WORDS, limit)) > limit) return FC_ERR_INTERNAL;
     if (cudaFuncSetAttribute(k_cache_search, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)limit) != cudaSuccess)
       return FC_ERR_CUDA;
+    if (dev < 64) dev_limit[dev].store(limit);
     smem_limit = limit;
+    return FC_OK;
+  });
+  if (st != FC_OK) return st;
+  if (!smem_limit) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev >= 64) return FC_ERR_CUDA;
+    smem_limit = dev_limit[dev].load();
   }
   const uint32_t rows_cap = cs_rows_cap(cache->capacity, smem_limit);
   ResOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len};

@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include <nvtx3/nvToolsExt.h>
 
 #include "../../include/fastcoder.h"
@@ -86,6 +88,20 @@ static inline fc_status fc_status_of_bits(unsigned int e) {
   if (e & FC_EBIT_CAPACITY) return FC_ERR_CAPACITY;
   if (e & FC_EBIT_INVALID) return FC_ERR_INVALID_ARG;
   return FC_OK;
+}
+
+// Host: runs set_up(device) once per device (kernel attributes are per
+// device); `done` holds a bit per device already set up (devices past 63 are
+// set up on every call).
+template <typename F>
+fc_status fc_once_per_device(std::atomic<unsigned long long>& done, F&& set_up) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return FC_ERR_CUDA;
+  const unsigned long long bit = dev < 64 ? 1ull << dev : 0ull;
+  if (bit && (done.load(std::memory_order_acquire) & bit)) return FC_OK;
+  const fc_status st = set_up(dev);
+  if (st == FC_OK && bit) done.fetch_or(bit, std::memory_order_acq_rel);
+  return st;
 }
 
 // Host: map a CUDA launch result to a status.

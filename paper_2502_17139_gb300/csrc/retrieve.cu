@@ -580,12 +580,11 @@ static fc_status launch_retrieve(bool all, const fc_datastore* sources, const fc
   }
   const int variant = all ? 2 : (rev_sources ? 1 : 0);
   auto kern = all ? k_retrieve<false, true> : (rev_sources ? k_retrieve<true, false> : k_retrieve<false, false>);
-  static bool attr_done[3] = {false, false, false};
-  if (!attr_done[variant]) {
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(RetSmem)) != cudaSuccess)
-      return FC_ERR_CUDA;
-    attr_done[variant] = true;
-  }
+  static std::atomic<unsigned long long> attr_done[3];
+  const fc_status st = fc_once_per_device(attr_done[variant], [&](int) {
+    return fc_cuda_status(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(RetSmem)));
+  });
+  if (st != FC_OK) return st;
   RetOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len, fc_error_slot()};
   dim3 grid((unsigned)batch, (unsigned)n_sources);
   kern<<<grid, RT_THREADS, sizeof(RetSmem), static_cast<cudaStream_t>(stream)>>>(a, r, d_ctx, ctx_stride, d_ctx_len,
