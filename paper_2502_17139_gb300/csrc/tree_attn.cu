@@ -1009,6 +1009,42 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
       __nv_bfloat16* dst = nullptr;
       uint64_t m0 = 0, m1 = 0;
       float m_run = -INFINITY, l_run = 0.f;
+      // A unit's output is written once the next unit's first P is handed
+      // over: its last PV then runs while this warpgroup already works on the
+      // next unit's scores, instead of being waited for.
+      bool pend = false, pend_row_ok = false;
+      int pend_o = 0;
+      uint32_t pend_par = 0;
+      float pend_l = 1.f;
+      __nv_bfloat16* pend_dst = nullptr;
+      auto flush = [&]() -> bool {  // the pending unit's O: normalise, store, free the buffer
+        if (!pend) return true;
+        pend = false;
+        if (!warp_wait(bar(L::OFIN + pend_o), pend_par, &s_abort)) return false;
+        tc_fence_after();
+        const uint32_t tP = tmem + 256 + pend_o * 128 + lane_off;
+        const float inv = 1.f / pend_l;
+#pragma unroll
+        for (int cc = 0; cc < HD / 32; ++cc) {
+          uint32_t ov[32];
+          tmem_ld32(tP + cc * 32, ov);
+          tc_wait_ld();
+          if (pend_row_ok) {
+#pragma unroll
+            for (int u = 0; u < 32; u += 8) {
+              uint4 v;
+              v.x = pack_bf16x2(__uint_as_float(ov[u + 0]) * inv, __uint_as_float(ov[u + 1]) * inv);
+              v.y = pack_bf16x2(__uint_as_float(ov[u + 2]) * inv, __uint_as_float(ov[u + 3]) * inv);
+              v.z = pack_bf16x2(__uint_as_float(ov[u + 4]) * inv, __uint_as_float(ov[u + 5]) * inv);
+              v.w = pack_bf16x2(__uint_as_float(ov[u + 6]) * inv, __uint_as_float(ov[u + 7]) * inv);
+              *reinterpret_cast<uint4*>(pend_dst + cc * 32 + u) = v;
+            }
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(bar(L::OFREE + pend_o));
+        return true;
+      };
       for (int J = 0; ok && c.valid(); ++J, c.next(a)) {
         const int o = c.live & 1;
         const uint32_t tO = tmem + 256 + o * 128 + lane_off;
@@ -1110,31 +1146,17 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         m_run = m_new;
         tc_fence_before();
         mbar_arrive(bar(L::PFULL + sb));
-        if (tree) {  // the unit's last block: read its O out, then free the buffer
-          if (!(ok = warp_wait(bar(L::OFIN + o), (c.live >> 1) & 1, &s_abort))) break;
-          tc_fence_after();
-          const float inv = 1.f / l_run;
-#pragma unroll
-          for (int cc = 0; cc < HD / 32; ++cc) {
-            uint32_t ov[32];
-            tmem_ld32(tO + cc * 32, ov);
-            tc_wait_ld();
-            if (row_ok) {
-#pragma unroll
-              for (int u = 0; u < 32; u += 8) {
-                uint4 v;
-                v.x = pack_bf16x2(__uint_as_float(ov[u + 0]) * inv, __uint_as_float(ov[u + 1]) * inv);
-                v.y = pack_bf16x2(__uint_as_float(ov[u + 2]) * inv, __uint_as_float(ov[u + 3]) * inv);
-                v.z = pack_bf16x2(__uint_as_float(ov[u + 4]) * inv, __uint_as_float(ov[u + 5]) * inv);
-                v.w = pack_bf16x2(__uint_as_float(ov[u + 6]) * inv, __uint_as_float(ov[u + 7]) * inv);
-                *reinterpret_cast<uint4*>(dst + cc * 32 + u) = v;
-              }
-            }
-          }
-          tc_fence_before();
-          mbar_arrive(bar(L::OFREE + o));
+        if (c.j == 0 && !(ok = flush())) break;  // the previous unit's output
+        if (tree) {  // the unit's last block: its output follows the next unit's first P
+          pend = true;
+          pend_o = o;
+          pend_par = (c.live >> 1) & 1;
+          pend_l = l_run;
+          pend_row_ok = row_ok;
+          pend_dst = dst;
         }
       }
+      if (ok) ok = flush();  // the last unit's output
     }
   }
   tc_fence_before();
