@@ -451,7 +451,8 @@ def run_ours(args, rank, ws, local):
                                "step executor, each on a chain stream and an attention stream" if nsub > 1
                                else "one stream")},
         "roofline": roof,
-        "gpu_launches": 8 * K * nsub,
+        # per sub-batch step: cached retrieval, insert, tree, attention, predictions, accept, append
+        "gpu_launches": 7 * K * nsub,
         "clocks": clock_rec,
         # each stage's mean time per sub-batch launch; with sub-batches on separate
         # streams the stages of different sub-batches overlap, so they do not add up to "all"

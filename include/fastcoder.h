@@ -305,6 +305,20 @@ fc_status fc_rcache_lookup(const void* d_table, int capacity, int n_sources, fc_
                            int32_t* d_n_drafts, int32_t* d_match_len, fc_stream s);
 
 /*
+ * fc_rcache_lookup and then fc_retrieve on the queries it did not serve, in
+ * one launch: each (query, source) CTA first looks the query's key up and,
+ * when served, copies its source's stored result; the others retrieve.  The
+ * outputs and d_skip are exactly those of the two calls (a served query
+ * records no token error, as there).  Arguments as the two calls; d_skip
+ * [batch] is written (1 = served).
+ */
+fc_status fc_retrieve_cached(const fc_datastore* sources, int n_sources, const uint32_t* d_ctx,
+                             int ctx_stride, const int32_t* d_ctx_len, int batch, const void* d_table,
+                             int capacity, const int32_t* d_want_hit, int32_t* d_skip,
+                             fc_retrieve_params p, uint32_t* d_drafts, int32_t* d_draft_len,
+                             uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len, fc_stream s);
+
+/*
  * Stores the retrieval outputs of every query with d_skip[b] == 0 under its
  * key (replacing an equal key).  A full table records FC_ERR_CAPACITY.
  */

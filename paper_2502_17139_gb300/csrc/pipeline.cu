@@ -6,7 +6,7 @@
 // The sequences of a batch are independent, so sub-batch h may run step
 // s + 1 while sub-batch h' is still in step s.  Per sub-batch the executor
 // owns two streams: a high-priority one for the latency-bound chain
-// (replay-cache lookup, retrieval, insert, tree build, predictions,
+// (replay-cache lookup with retrieval, insert, tree build, predictions,
 // acceptance, append) and a low-priority one for the attention launch,
 // ordered by an event pair.  When SMs free up, the block scheduler then
 // starts another sub-batch's chain ahead of this sub-batch's remaining
@@ -154,11 +154,13 @@ extern "C" fc_status fc_pipeline_step(fc_pipeline* pl, int phase, int flags, con
     FcErrorScope scope(P.err);  // the sub-batch's kernels record errors in its own word
 
     stage_event(stage_events, h, 0, 0, s);
-    if (P.rcache)
-      FC_TRY(fc_rcache_lookup(P.rcache, P.rcache_capacity, S, d.p, P.ctx, P.ctx_stride, P.ctx_len[c], B, want,
-                              P.skip, P.drafts, P.draft_len, P.count, P.n_drafts, P.match_len, s));
-    FC_TRY(fc_retrieve(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.rcache ? P.skip : nullptr,
-                       d.p, P.drafts, P.draft_len, P.count, P.n_drafts, P.match_len, s));
+    if (P.rcache)  // replay-cache lookup and retrieval of the queries it did not serve, one launch
+      FC_TRY(fc_retrieve_cached(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.rcache,
+                                P.rcache_capacity, want, P.skip, d.p, P.drafts, P.draft_len, P.count, P.n_drafts,
+                                P.match_len, s));
+    else
+      FC_TRY(fc_retrieve(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, nullptr, d.p, P.drafts,
+                         P.draft_len, P.count, P.n_drafts, P.match_len, s));
     if (P.rcache)
       FC_TRY(fc_rcache_insert(P.rcache, P.rcache_capacity, S, d.p, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.skip,
                               P.drafts, P.draft_len, P.count, P.n_drafts, P.match_len, s));

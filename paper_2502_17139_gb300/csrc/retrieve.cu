@@ -148,6 +148,16 @@ struct RetSmem {
   uint32_t wsum[RT_THREADS / 32];
   RunsScratch rs;
   uint32_t n_star, first, cnt, bad, n_rev;
+  int32_t rc_slot;
+};
+
+// The replay-cache lookup folded into retrieval (fc_retrieve_cached): table
+// NULL means none.
+struct RcFused {
+  const uint32_t* table;
+  int capacity;
+  const int32_t* want;  // NULL: every query may be served
+  int32_t* skip;        // out: 1 = served from the cache
 };
 
 // n* through the reversed corpus R (R[i] = T[N-1-i]), by one warp.  The
@@ -207,11 +217,116 @@ __device__ int rev_match_len(const DsView& rv, const uint32_t* __restrict__ T, u
   return best;
 }
 
+// ---------------------------------------------------------------------------
+// Replay cache.  Entry layout (32-bit words): [0] key length or EMPTY /
+// CLAIMED, [1 .. 1+n_max) key tokens, then per source: drafts[k*d],
+// draft_len[k], count[k], n_drafts, match_len.
+// ---------------------------------------------------------------------------
+constexpr uint32_t RC_EMPTY = 0xFFFFFFFFu;
+constexpr uint32_t RC_CLAIMED = 0xFFFFFFFEu;
+
+__host__ __device__ inline size_t rc_src_words(const fc_retrieve_params& p) {
+  return (size_t)p.top_k * p.draft_len + 2 * (size_t)p.top_k + 2;
+}
+__host__ __device__ inline size_t rc_entry_words(int S, const fc_retrieve_params& p) {
+  size_t w = 1 + (size_t)p.n_max + (size_t)S * rc_src_words(p);
+  return (w + 3) & ~(size_t)3;
+}
+
+__device__ uint64_t rc_hash(const uint32_t* key, int len) {
+  uint64_t h = 1469598103934665603ull ^ (uint64_t)len;
+  for (int i = 0; i < len; ++i) {
+    h ^= key[i];
+    h *= 1099511628211ull;
+  }
+  h ^= h >> 29;
+  return h;
+}
+
+struct RcSmem {
+  uint32_t key[FC_MAX_NMAX];
+  int klen;
+  int slot;
+};
+
+__device__ void rc_load_key(RcSmem& sm, const uint32_t* ctx, int stride, const int32_t* ctx_len, int b, int n_max) {
+  int m = max(0, min((int)ctx_len[b], stride));
+  int kl = min(n_max, m);
+  if (threadIdx.x < kl) sm.key[threadIdx.x] = ctx[(size_t)b * stride + (m - kl) + threadIdx.x];
+  if (threadIdx.x == 0) sm.klen = kl;
+  __syncthreads();
+}
+
+// Warp 0 compares the entry's key with sm.key: lane i reads key word i, so
+// the words arrive in one round trip (n_max <= 32).  `head` is the entry's
+// first word, already read.  Warp-uniform result.
+__device__ bool rc_key_equal_warp(const uint32_t* entry, uint32_t head, const uint32_t* key, int klen, int lane) {
+  const bool len_ok = head == (uint32_t)klen;
+  const uint32_t w = (len_ok && lane < klen) ? entry[1 + lane] : 0u;
+  return __all_sync(0xFFFFFFFFu, len_ok && (lane >= klen || w == key[lane]));
+}
+
+// Warp 0's probe for `key`: the slot of an entry holding it, or -1 (an empty
+// slot ends the chain).  Every lane returns the same slot.
+__device__ int rc_find_warp(const uint32_t* table, int capacity, size_t ew, const uint32_t* key, int klen, int lane) {
+  const uint64_t h = rc_hash(key, klen);
+  for (int probe = 0; probe < capacity; ++probe) {
+    const size_t e = (h + probe) & (uint64_t)(capacity - 1);
+    const uint32_t* ent = table + e * ew;
+    const uint32_t st = ent[0];
+    if (st == RC_EMPTY) break;
+    if (st != RC_CLAIMED && rc_key_equal_warp(ent, st, key, klen, lane)) return (int)e;
+  }
+  return -1;
+}
+
+// A query's outputs and a cache entry's result area, word by word: flat
+// index i over S * rc_src_words(p) words (source s, then drafts, draft
+// lengths, counts, n_drafts, match_len) names one word of the entry
+// (entry[i]) and one output word (*rc_out_word(...)).
+__device__ __forceinline__ uint32_t* rc_out_word(const RetOut& o, int i, int per, int k, int d, int B, int b) {
+  const int s = i / per, r = i - s * per;
+  const size_t sb = (size_t)s * B + b;
+  if (r < k * d) return o.drafts + sb * k * d + r;
+  if (r < k * d + k) return reinterpret_cast<uint32_t*>(o.draft_len) + sb * k + (r - k * d);
+  if (r < k * d + 2 * k) return o.count + sb * k + (r - k * d - k);
+  return r == k * d + 2 * k ? reinterpret_cast<uint32_t*>(o.n_drafts) + sb : reinterpret_cast<uint32_t*>(o.match_len) + sb;
+}
+
+// Copies a query's whole result between a cache entry and the outputs with
+// the CTA's threads, sixteen loads in flight per thread before their stores
+// (a lookup or an insert is a few such round trips, not one per array).
+template <bool TO_OUT>
+__device__ __forceinline__ void rc_copy(uint32_t* entry, const RetOut& o, int S, const fc_retrieve_params& p, int B,
+                                        int b, int s_first = 0, int s_count = -1) {
+  constexpr int U = 16;
+  const int k = p.top_k, d = p.draft_len, per = (int)rc_src_words(p);
+  const int n = (s_first + (s_count < 0 ? S - s_first : s_count)) * per;  // sources [s_first, s_first + count)
+  for (int i0 = s_first * per + threadIdx.x; i0 < n; i0 += U * blockDim.x) {
+    uint32_t v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + u * blockDim.x;
+      v[u] = i < n ? (TO_OUT ? entry[i] : *rc_out_word(o, i, per, k, d, B, b)) : 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i < n) {
+        if (TO_OUT)
+          *rc_out_word(o, i, per, k, d, B, b) = v[u];
+        else
+          entry[i] = v[u];
+      }
+    }
+  }
+}
+
 template <bool REV, bool ALL>
 __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev, const uint32_t* __restrict__ ctx,
                                                          int stride, const int32_t* __restrict__ ctx_len, int B,
                                                          const int32_t* __restrict__ skip, fc_retrieve_params p,
-                                                         RetOut o) {
+                                                         RetOut o, RcFused rc) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   RetSmem& sm = *reinterpret_cast<RetSmem*>(smem_raw);
   const int b = blockIdx.x, s = blockIdx.y, tid = threadIdx.x;
@@ -233,6 +348,28 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev
     if (t >= ds.vocab) sm.bad = 1;
   }
   __syncthreads();
+  if constexpr (!REV && !ALL) {
+    // Replay cache first: the key is the context's last min(n_max, ctx_len)
+    // tokens, the ones just loaded.  A served query copies this source's
+    // stored result and is done (as fc_rcache_lookup, then a skipped
+    // retrieval: a served query records no token error).
+    if (rc.table) {
+      if (tid < 32) {
+        const size_t ew = rc_entry_words((int)gridDim.y, p);
+        const int slot = (!rc.want || rc.want[b]) ? rc_find_warp(rc.table, rc.capacity, ew, sm.ctx, cap, tid) : -1;
+        if (tid == 0) sm.rc_slot = slot;
+      }
+      __syncthreads();
+      const int slot = sm.rc_slot;
+      if (s == 0 && tid == 0) rc.skip[b] = slot >= 0 ? 1 : 0;
+      if (slot >= 0) {
+        const size_t ew = rc_entry_words((int)gridDim.y, p);
+        rc_copy<true>(const_cast<uint32_t*>(rc.table) + (size_t)slot * ew + 1 + p.n_max, o, (int)gridDim.y, p, B, b,
+                      s, 1);
+        return;
+      }
+    }
+  }
   if (sm.bad && tid == 0) fc_flag(FC_ERR_WORD(o.err), FC_EBIT_INVALID);
 
   // ---- search: one warp per n, one half-warp per bound, 16 pivots a round
@@ -375,100 +512,10 @@ __global__ void __launch_bounds__(RT_THREADS) k_retrieve(DsArgs args, DsArgs rev
 
 bool params_ok(const fc_retrieve_params& p) { return fc_retrieve_params_ok(p); }
 
-// ---------------------------------------------------------------------------
-// Replay cache.  Entry layout (32-bit words): [0] key length or EMPTY /
-// CLAIMED, [1 .. 1+n_max) key tokens, then per source: drafts[k*d],
-// draft_len[k], count[k], n_drafts, match_len.
-// ---------------------------------------------------------------------------
-constexpr uint32_t RC_EMPTY = 0xFFFFFFFFu;
-constexpr uint32_t RC_CLAIMED = 0xFFFFFFFEu;
-
-__host__ __device__ inline size_t rc_src_words(const fc_retrieve_params& p) {
-  return (size_t)p.top_k * p.draft_len + 2 * (size_t)p.top_k + 2;
-}
-__host__ __device__ inline size_t rc_entry_words(int S, const fc_retrieve_params& p) {
-  size_t w = 1 + (size_t)p.n_max + (size_t)S * rc_src_words(p);
-  return (w + 3) & ~(size_t)3;
-}
-
-__device__ uint64_t rc_hash(const uint32_t* key, int len) {
-  uint64_t h = 1469598103934665603ull ^ (uint64_t)len;
-  for (int i = 0; i < len; ++i) {
-    h ^= key[i];
-    h *= 1099511628211ull;
-  }
-  h ^= h >> 29;
-  return h;
-}
-
 __global__ void k_rc_init(uint32_t* table, int capacity, size_t entry_words) {
   for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < (size_t)capacity;
        e += (size_t)gridDim.x * blockDim.x)
     table[e * entry_words] = RC_EMPTY;
-}
-
-struct RcSmem {
-  uint32_t key[FC_MAX_NMAX];
-  int klen;
-  int slot;
-};
-
-__device__ void rc_load_key(RcSmem& sm, const uint32_t* ctx, int stride, const int32_t* ctx_len, int b, int n_max) {
-  int m = max(0, min((int)ctx_len[b], stride));
-  int kl = min(n_max, m);
-  if (threadIdx.x < kl) sm.key[threadIdx.x] = ctx[(size_t)b * stride + (m - kl) + threadIdx.x];
-  if (threadIdx.x == 0) sm.klen = kl;
-  __syncthreads();
-}
-
-// Warp 0 compares the entry's key with sm.key: lane i reads key word i, so
-// the words arrive in one round trip (n_max <= 32).  `head` is the entry's
-// first word, already read.  Warp-uniform result.
-__device__ bool rc_key_equal_warp(const uint32_t* entry, uint32_t head, const RcSmem& sm, int lane) {
-  const bool len_ok = head == (uint32_t)sm.klen;
-  const uint32_t w = (len_ok && lane < sm.klen) ? entry[1 + lane] : 0u;
-  return __all_sync(0xFFFFFFFFu, len_ok && (lane >= sm.klen || w == sm.key[lane]));
-}
-
-// A query's outputs and a cache entry's result area, word by word: flat
-// index i over S * rc_src_words(p) words (source s, then drafts, draft
-// lengths, counts, n_drafts, match_len) names one word of the entry
-// (entry[i]) and one output word (*rc_out_word(...)).
-__device__ __forceinline__ uint32_t* rc_out_word(const RetOut& o, int i, int per, int k, int d, int B, int b) {
-  const int s = i / per, r = i - s * per;
-  const size_t sb = (size_t)s * B + b;
-  if (r < k * d) return o.drafts + sb * k * d + r;
-  if (r < k * d + k) return reinterpret_cast<uint32_t*>(o.draft_len) + sb * k + (r - k * d);
-  if (r < k * d + 2 * k) return o.count + sb * k + (r - k * d - k);
-  return r == k * d + 2 * k ? reinterpret_cast<uint32_t*>(o.n_drafts) + sb : reinterpret_cast<uint32_t*>(o.match_len) + sb;
-}
-
-// Copies a query's whole result between a cache entry and the outputs with
-// the CTA's threads, sixteen loads in flight per thread before their stores
-// (a lookup or an insert is a few such round trips, not one per array).
-template <bool TO_OUT>
-__device__ __forceinline__ void rc_copy(uint32_t* entry, const RetOut& o, int S, const fc_retrieve_params& p, int B,
-                                        int b) {
-  constexpr int U = 16;
-  const int k = p.top_k, d = p.draft_len, per = (int)rc_src_words(p), n = S * per;
-  for (int i0 = threadIdx.x; i0 < n; i0 += U * blockDim.x) {
-    uint32_t v[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = i0 + u * blockDim.x;
-      v[u] = i < n ? (TO_OUT ? entry[i] : *rc_out_word(o, i, per, k, d, B, b)) : 0u;
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = i0 + u * blockDim.x;
-      if (i < n) {
-        if (TO_OUT)
-          *rc_out_word(o, i, per, k, d, B, b) = v[u];
-        else
-          entry[i] = v[u];
-      }
-    }
-  }
 }
 
 __global__ void k_rc_lookup(const uint32_t* __restrict__ table, int capacity, int S, fc_retrieve_params p,
@@ -480,20 +527,7 @@ __global__ void k_rc_lookup(const uint32_t* __restrict__ table, int capacity, in
   const size_t ew = rc_entry_words(S, p);
   if (threadIdx.x < 32) {  // warp 0 probes; every lane takes the same path
     const int lane = threadIdx.x;
-    int slot = -1;
-    if (!want || want[b]) {
-      const uint64_t h = rc_hash(sm.key, sm.klen);
-      for (int probe = 0; probe < capacity; ++probe) {
-        const size_t e = (h + probe) & (uint64_t)(capacity - 1);
-        const uint32_t* ent = table + e * ew;
-        const uint32_t st = ent[0];
-        if (st == RC_EMPTY) break;
-        if (st != RC_CLAIMED && rc_key_equal_warp(ent, st, sm, lane)) {
-          slot = (int)e;
-          break;
-        }
-      }
-    }
+    const int slot = (!want || want[b]) ? rc_find_warp(table, capacity, ew, sm.key, sm.klen, lane) : -1;
     if (lane == 0) {
       sm.slot = slot;
       skip[b] = slot >= 0 ? 1 : 0;
@@ -525,7 +559,7 @@ __global__ void k_rc_insert(uint32_t* table, int capacity, int S, fc_retrieve_pa
       st = __shfl_sync(0xFFFFFFFFu, st, 0);
       if (st == RC_EMPTY) {
         slot = (int)e;
-      } else if (st != RC_CLAIMED && rc_key_equal_warp(ent, st, sm, lane)) {
+      } else if (st != RC_CLAIMED && rc_key_equal_warp(ent, st, sm.key, sm.klen, lane)) {
         present = true;  // an equal key holds the same (deterministic) result
       }
     }
@@ -550,7 +584,7 @@ static fc_status launch_retrieve(bool all, const fc_datastore* sources, const fc
                                  const uint32_t* d_ctx, int ctx_stride, const int32_t* d_ctx_len, int batch,
                                  const int32_t* d_skip, fc_retrieve_params p, uint32_t* d_drafts,
                                  int32_t* d_draft_len, uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len,
-                                 fc_stream stream) {
+                                 fc_stream stream, RcFused rc = RcFused{nullptr, 0, nullptr, nullptr}) {
   if (!sources || n_sources < 1 || n_sources > FC_MAX_SOURCES || batch < 0 || ctx_stride < 1 ||
       batch > 65535 * 16)
     return FC_ERR_INVALID_ARG;
@@ -588,7 +622,7 @@ static fc_status launch_retrieve(bool all, const fc_datastore* sources, const fc
   RetOut o{d_drafts, d_draft_len, d_count, d_n_drafts, d_match_len, fc_error_slot()};
   dim3 grid((unsigned)batch, (unsigned)n_sources);
   kern<<<grid, RT_THREADS, sizeof(RetSmem), static_cast<cudaStream_t>(stream)>>>(a, r, d_ctx, ctx_stride, d_ctx_len,
-                                                                                 batch, d_skip, p, o);
+                                                                                 batch, d_skip, p, o, rc);
   return FC_CHECK_LAUNCH();
 }
 
@@ -657,6 +691,19 @@ extern "C" fc_status fc_rcache_lookup(const void* d_table, int capacity, int n_s
                                                                      n_sources, p, d_ctx, ctx_stride, d_ctx_len, batch,
                                                                      d_want_hit, d_skip, o);
   return FC_CHECK_LAUNCH();
+}
+
+extern "C" fc_status fc_retrieve_cached(const fc_datastore* sources, int n_sources, const uint32_t* d_ctx,
+                                        int ctx_stride, const int32_t* d_ctx_len, int batch, const void* d_table,
+                                        int capacity, const int32_t* d_want_hit, int32_t* d_skip,
+                                        fc_retrieve_params p, uint32_t* d_drafts, int32_t* d_draft_len,
+                                        uint32_t* d_count, int32_t* d_n_drafts, int32_t* d_match_len,
+                                        fc_stream stream) {
+  FC_NVTX_RANGE();
+  if (!d_table || !rc_args_ok(capacity, n_sources, p) || (batch > 0 && !d_skip)) return FC_ERR_INVALID_ARG;
+  return launch_retrieve(false, sources, nullptr, n_sources, d_ctx, ctx_stride, d_ctx_len, batch, nullptr, p, d_drafts,
+                         d_draft_len, d_count, d_n_drafts, d_match_len, stream,
+                         RcFused{static_cast<const uint32_t*>(d_table), capacity, d_want_hit, d_skip});
 }
 
 extern "C" fc_status fc_rcache_insert(void* d_table, int capacity, int n_sources, fc_retrieve_params p,

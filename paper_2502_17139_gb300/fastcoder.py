@@ -74,7 +74,7 @@ class fc_pipeline_desc(C.Structure):
 
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
            "fc_datastore_build_noalloc", "fc_datastore_keys", "fc_datastore_save", "fc_datastore_file_info", "fc_datastore_load",
-           "fc_retrieve", "fc_retrieve_all", "fc_retrieve_rev", "fc_reverse_tokens", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert",
+           "fc_retrieve", "fc_retrieve_all", "fc_retrieve_rev", "fc_reverse_tokens", "fc_rcache_bytes", "fc_rcache_init", "fc_rcache_lookup", "fc_rcache_insert", "fc_retrieve_cached",
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
            "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_tree_attn_streamed", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_gemm_kv_heads", "fc_gemm_silu_mul", "fc_interleave_gate_up", "fc_embed",
            "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax",
@@ -113,6 +113,8 @@ def _load():
                                        vp, vp, vp, vp, vp, vp]),
         "fc_rcache_insert": (C.c_int, [vp, i32, i32, fc_retrieve_params, vp, i32, vp, i32, vp,
                                        vp, vp, vp, vp, vp, vp]),
+        "fc_retrieve_cached": (C.c_int, [C.POINTER(fc_datastore), i32, vp, i32, vp, i32, vp, i32, vp, vp,
+                                         fc_retrieve_params, vp, vp, vp, vp, vp, vp]),
         "fc_cache_init": (C.c_int, [C.POINTER(fc_cache), i32, vp, vp]),
         "fc_cache_search": (C.c_int, [C.POINTER(fc_cache), vp, i32, vp, i32, vp, i32, fc_retrieve_params, i32,
                                       vp, vp, vp, vp, vp, vp, vp]),
@@ -437,6 +439,24 @@ def fc_rcache_lookup(cache: RetrievalCache, ctx, ctx_len, want_hit, skip, out):
         _ptr(cache.table), cache.capacity, cache.n_sources, cache.p, _ptr(ctx), stride, _ptr(ctx_len), B,
         _ptr(want_hit), _ptr(skip), _ptr(out["drafts"]), _ptr(out["draft_len"]), _ptr(out["count"]),
         _ptr(out["n_drafts"]), _ptr(out["match_len"]), _stream()))
+
+
+def fc_retrieve_cached(sources, cache: RetrievalCache, ctx, ctx_len, want_hit, skip, p: fc_retrieve_params, out):
+    """fc_rcache_lookup + fc_retrieve of the queries it did not serve, in one
+    launch (skip [B] written: 1 = served)."""
+    S = len(sources)
+    _need(ctx, torch.int32, "ctx")
+    B, stride = ctx.shape
+    _need(ctx_len, torch.int32, "ctx_len", (B,))
+    _need(skip, torch.int32, "skip", (B,))
+    if want_hit is not None:
+        _need(want_hit, torch.int32, "want_hit", (B,))
+    views = (fc_datastore * S)(*[s.view for s in sources])
+    _check("fc_retrieve_cached", LIB.fc_retrieve_cached(
+        views, S, _ptr(ctx), stride, _ptr(ctx_len), B, _ptr(cache.table), cache.capacity, _ptr(want_hit), _ptr(skip),
+        p, _ptr(out["drafts"]), _ptr(out["draft_len"]), _ptr(out["count"]), _ptr(out["n_drafts"]),
+        _ptr(out["match_len"]), _stream()))
+    return out
 
 
 def fc_rcache_insert(cache: RetrievalCache, ctx, ctx_len, skip, res):

@@ -12,8 +12,8 @@ Retrieval takes one of two forms:
     fc_missing_insert; after the append, fc_cache_update stores the verified
     retrieval and the completed output pieces.  The tree merges S + 1 result
     slots, the CACHE's last.
-  * otherwise the context-keyed replay cache: lookup -> fc_retrieve on the
-    queries it did not serve -> insert.
+  * otherwise the context-keyed replay cache: lookup and fc_retrieve on the
+    queries it did not serve (one launch, fc_retrieve_cached) -> insert.
 
 Every call is asynchronous on the current stream and allocates nothing, so
 steps can be captured once into a CUDA graph and replayed (lengths ping-pong
@@ -120,8 +120,8 @@ class StepLoop:
             fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, skip=self.skip, out=self.res)
             fc.fc_missing_insert(self.missing, self.ctx, self.ctx_len[c], self.skip, self.res["n_drafts"], S)
         elif self.cache is not None:
-            fc.fc_rcache_lookup(self.cache, self.ctx, self.ctx_len[c], want_hit, self.skip, self.res)
-            fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, skip=self.skip, out=self.res)
+            fc.fc_retrieve_cached(self.sources, self.cache, self.ctx, self.ctx_len[c], want_hit, self.skip, self.p,
+                                  self.res)
             fc.fc_rcache_insert(self.cache, self.ctx, self.ctx_len[c], self.skip, self.res)
         else:
             fc.fc_retrieve(self.sources, self.ctx, self.ctx_len[c], self.p, out=self.res)

@@ -122,3 +122,44 @@ def test_rcache_present_key_not_duplicated_and_full_table(fc):
         for b in np.flatnonzero(hits):
             assert torch.equal(g[:, b], host[k][:, b]), (k, b)
     assert fc.fc_get_error() == "FC_OK"
+
+
+def test_retrieve_cached_equals_lookup_then_retrieve(fc):
+    """fc_retrieve_cached against fc_rcache_lookup followed by fc_retrieve on
+    the queries it did not serve: the same outputs and skip flags, for a
+    half-filled cache, a want mask, a short context and a context with a token
+    outside the vocabulary (recorded only when that query is not served)."""
+    import paper_2502_17139_gb300.synth as synth
+    rng = synth.rng_for(81)
+    vocab = 300
+    Ts = [synth.make_corpus(rng, n, 1.1, vocab)[0] for n in (20_000, 5_000)]
+    srcs = [fc.fc_datastore_build(torch.from_numpy(T.view(np.int32)).cuda(), vocab) for T in Ts]
+    B, stride = 24, 40
+    ctx, cl, _ = synth.make_contexts(rng, B, 32, 8, Ts + [None], [0.4, 0.4, 0.2], 1.1, vocab=vocab, ctx_stride=stride)
+    cl = cl.copy()
+    cl[3] = 2  # shorter than n_max
+    ctx[5, cl[5] - 2] = vocab + 7  # a token outside the vocabulary
+    ctx_d, cl_d = torch.from_numpy(ctx.view(np.int32)).cuda(), torch.from_numpy(cl).cuda()
+    p = fc.params(12, 2, 16, 6, 512)
+    cache = fc.RetrievalCache(64, 2, p)
+    # fill the cache with the even queries' results
+    fill = fc.fc_retrieve(srcs, ctx_d, cl_d, p)
+    skip_fill = torch.tensor([b % 2 for b in range(B)], dtype=torch.int32, device="cuda")
+    fc.fc_rcache_insert(cache, ctx_d, cl_d, skip_fill, fill)
+    fc.fc_get_error()  # the out-of-vocabulary query recorded its error while filling
+    for want_h in (None, np.array([1 if b % 3 else 0 for b in range(B)], np.int32)):
+        want = None if want_h is None else torch.from_numpy(want_h).cuda()
+        ref = fc.retrieve_outputs(2, B, p, "cuda")
+        skip_ref = torch.full((B,), 9, dtype=torch.int32, device="cuda")
+        fc.fc_rcache_lookup(cache, ctx_d, cl_d, want, skip_ref, ref)
+        fc.fc_retrieve(srcs, ctx_d, cl_d, p, skip=skip_ref, out=ref)
+        err_ref = fc.fc_get_error()
+        got = fc.retrieve_outputs(2, B, p, "cuda")
+        skip = torch.full((B,), 9, dtype=torch.int32, device="cuda")
+        fc.fc_retrieve_cached(srcs, cache, ctx_d, cl_d, want, skip, p, got)
+        err = fc.fc_get_error()
+        assert err == err_ref
+        assert torch.equal(skip, skip_ref)
+        assert int(skip.sum().item()) > 0 and int(skip.sum().item()) < B
+        for k in ref:
+            assert torch.equal(got[k], ref[k]), k
