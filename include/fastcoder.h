@@ -804,6 +804,19 @@ fc_status fc_pipeline_step(fc_pipeline* pl, int phase, int flags, const void* d_
                            const void* d_v_tree, const int32_t* d_want_hit, const int32_t* d_plen,
                            const uint32_t* d_rtok, fc_stream caller, void* const* stage_events);
 
+/* fc_pipeline_step for sub-batch `part` alone: its work waits for the work
+ * enqueued on `caller` and then runs on its own streams; the other
+ * sub-batches are untouched.  With it each sub-batch can be captured into a
+ * CUDA graph of its own, so that replays never join the sub-batches.
+ * stage_events as fc_pipeline_step's (entries of other sub-batches unused). */
+fc_status fc_pipeline_step_part(fc_pipeline* pl, int part, int phase, int flags, const void* d_q,
+                                const void* d_k_tree, const void* d_v_tree, const int32_t* d_want_hit,
+                                const int32_t* d_plen, const uint32_t* d_rtok, fc_stream caller,
+                                void* const* stage_events);
+
+/* `caller` waits for everything enqueued on sub-batch `part`'s streams. */
+fc_status fc_pipeline_join_part(fc_pipeline* pl, int part, fc_stream caller);
+
 /* Waits for sub-batch `part`'s work enqueued so far, then returns and clears
  * its error word: the most severe device-detected error its kernels recorded
  * (FC_OK if none).  With a word per sub-batch an error is reported for the

@@ -29,7 +29,7 @@ struct fc_pipeline {
   std::vector<fc_datastore> sources;
   std::vector<uint32_t> weight;
   std::vector<cudaStream_t> chain, attn;
-  std::vector<cudaEvent_t> ev_pre, ev_post, ev_done;
+  std::vector<cudaEvent_t> ev_pre, ev_post, ev_done, ev_fork;
   cudaEvent_t ev_start = nullptr;
 };
 
@@ -40,7 +40,7 @@ void destroy_handles(fc_pipeline* pl) {
     if (s) cudaStreamDestroy(s);
   for (cudaStream_t s : pl->attn)
     if (s) cudaStreamDestroy(s);
-  for (auto* v : {&pl->ev_pre, &pl->ev_post, &pl->ev_done})
+  for (auto* v : {&pl->ev_pre, &pl->ev_post, &pl->ev_done, &pl->ev_fork})
     for (cudaEvent_t e : *v)
       if (e) cudaEventDestroy(e);
   if (pl->ev_start) cudaEventDestroy(pl->ev_start);
@@ -102,13 +102,15 @@ extern "C" fc_status fc_pipeline_create(const fc_pipeline_desc* d, fc_pipeline**
   pl->ev_pre.assign(n, nullptr);
   pl->ev_post.assign(n, nullptr);
   pl->ev_done.assign(n, nullptr);
+  pl->ev_fork.assign(n, nullptr);
   ok = ok && cudaEventCreateWithFlags(&pl->ev_start, cudaEventDisableTiming) == cudaSuccess;
   for (int h = 0; ok && h < n; ++h) {
     ok = cudaStreamCreateWithPriority(&pl->chain[h], cudaStreamNonBlocking, p_chain) == cudaSuccess &&
          cudaStreamCreateWithPriority(&pl->attn[h], cudaStreamNonBlocking, p_attn) == cudaSuccess &&
          cudaEventCreateWithFlags(&pl->ev_pre[h], cudaEventDisableTiming) == cudaSuccess &&
          cudaEventCreateWithFlags(&pl->ev_post[h], cudaEventDisableTiming) == cudaSuccess &&
-         cudaEventCreateWithFlags(&pl->ev_done[h], cudaEventDisableTiming) == cudaSuccess;
+         cudaEventCreateWithFlags(&pl->ev_done[h], cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&pl->ev_fork[h], cudaEventDisableTiming) == cudaSuccess;
   }
   if (!ok) {
     destroy_handles(pl);
@@ -129,77 +131,110 @@ extern "C" void fc_pipeline_destroy(fc_pipeline* pl) {
   delete pl;
 }
 
+namespace {
+
+// One sub-batch's step on its streams (the chain stream already waits for
+// whatever the step must follow).
+fc_status enqueue_part(fc_pipeline* pl, int h, int c, bool attention, const void* d_q, const void* d_k_tree,
+                       const void* d_v_tree, const int32_t* d_want_hit, const int32_t* d_plen,
+                       const uint32_t* d_rtok, void* const* stage_events) {
+  const fc_pipeline_desc& d = pl->d;
+  const int nx = 1 - c, S = d.n_sources, Np = d.n_pad;
+  const bool rope = d.rope_base > 0.f;
+  const size_t q_row = (size_t)Np * d.H * d.D * 2, kt_row = (size_t)d.Hkv * Np * d.D * 2;  // bytes per sequence
+  const fc_pipeline_part& P = pl->parts[h];
+  cudaStream_t s = pl->chain[h], sa = pl->attn[h];
+  const int B = P.batch;
+  const void* q = attention ? static_cast<const char*>(d_q) + (size_t)P.first * q_row : nullptr;
+  const void* kt = static_cast<const char*>(d_k_tree) + (size_t)P.first * kt_row;
+  const void* vt = static_cast<const char*>(d_v_tree) + (size_t)P.first * kt_row;
+  const int32_t* want = d_want_hit ? d_want_hit + P.first : nullptr;
+  FcErrorScope scope(P.err);  // the sub-batch's kernels record errors in its own word
+
+  stage_event(stage_events, h, 0, 0, s);
+  if (P.rcache)  // replay-cache lookup and retrieval of the queries it did not serve, one launch
+    FC_TRY(fc_retrieve_cached(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.rcache,
+                              P.rcache_capacity, want, P.skip, d.p, P.drafts, P.draft_len, P.count, P.n_drafts,
+                              P.match_len, s));
+  else
+    FC_TRY(fc_retrieve(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, nullptr, d.p, P.drafts,
+                       P.draft_len, P.count, P.n_drafts, P.match_len, s));
+  if (P.rcache)
+    FC_TRY(fc_rcache_insert(P.rcache, P.rcache_capacity, S, d.p, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.skip,
+                            P.drafts, P.draft_len, P.count, P.n_drafts, P.match_len, s));
+  stage_event(stage_events, h, 0, 1, s);
+  stage_event(stage_events, h, 1, 0, s);
+  FC_TRY(fc_build_tree(S, P.drafts, P.draft_len, P.count, P.n_drafts, pl->weight.data(), d.p.top_k,
+                       d.p.draft_len, P.root, P.kv_len[c], B, d.node_budget, Np, P.tok, P.parent, P.depth, P.pos,
+                       P.mask, P.n_nodes, s));
+  stage_event(stage_events, h, 1, 1, s);
+  if (rope) {
+    FC_TRY(fc_rope(kt, P.k_tree_rot, B, Np, d.Hkv, d.D, 1, P.pos, d.rope_base, s));
+    kt = P.k_tree_rot;
+  }
+  if (attention) {  // on its own stream, ordered by an event pair
+    if (cudaEventRecord(pl->ev_pre[h], s) != cudaSuccess || cudaStreamWaitEvent(sa, pl->ev_pre[h], 0) != cudaSuccess)
+      return FC_ERR_CUDA;
+    stage_event(stage_events, h, 2, 0, sa);
+    if (rope)
+      FC_TRY(fc_tree_attn_rope(q, P.k_cache, P.v_cache, d.kv_cap, P.kv_len[c], kt, vt, P.mask, P.n_nodes, B, Np,
+                               d.H, d.Hkv, d.D, d.scale, P.pos, d.rope_base, P.attn_out, P.attn_ws,
+                               P.attn_ws_bytes, sa));
+    else
+      FC_TRY(fc_tree_attn(q, P.k_cache, P.v_cache, d.kv_cap, P.kv_len[c], kt, vt, P.mask, P.n_nodes, B, Np, d.H,
+                          d.Hkv, d.D, d.scale, P.attn_out, P.attn_ws, P.attn_ws_bytes, sa));
+    stage_event(stage_events, h, 2, 1, sa);
+    if (cudaEventRecord(pl->ev_post[h], sa) != cudaSuccess ||
+        cudaStreamWaitEvent(s, pl->ev_post[h], 0) != cudaSuccess)
+      return FC_ERR_CUDA;
+  }
+  stage_event(stage_events, h, 3, 0, s);
+  FC_TRY(fc_synth_argmax(P.tok, P.parent, P.n_nodes, B, Np, d_plen + P.first, d_rtok + (size_t)P.first * Np,
+                         d.vocab, P.argmax, s));
+  FC_TRY(fc_accept(P.tok, P.parent, P.n_nodes, P.argmax, B, Np, P.acc_len, P.path, d.path_cap, P.bonus, s));
+  FC_TRY(fc_kv_append(P.path, P.acc_len, P.bonus, P.tok, kt, vt, B, Np, d.Hkv, d.D, d.path_cap, P.k_cache,
+                      P.v_cache, d.kv_cap, P.kv_len[c], P.kv_len[nx], P.ctx, P.ctx_stride, P.ctx_len[c],
+                      P.ctx_len[nx], P.root, s));
+  stage_event(stage_events, h, 3, 1, s);
+  return FC_OK;
+}
+
+bool step_args_ok(const fc_pipeline* pl, int phase, int flags, const void* d_q, const void* d_k_tree,
+                  const void* d_v_tree, const int32_t* d_plen, const uint32_t* d_rtok) {
+  const bool attention = !(flags & FC_PIPELINE_NO_ATTENTION);
+  return pl && (phase == 0 || phase == 1) && !(flags & ~FC_PIPELINE_NO_ATTENTION) && (!attention || d_q) &&
+         d_k_tree && d_v_tree && d_plen && d_rtok;
+}
+
+}  // namespace
+
 extern "C" fc_status fc_pipeline_step(fc_pipeline* pl, int phase, int flags, const void* d_q, const void* d_k_tree,
                                       const void* d_v_tree, const int32_t* d_want_hit, const int32_t* d_plen,
                                       const uint32_t* d_rtok, fc_stream caller, void* const* stage_events) {
   FC_NVTX_RANGE();
+  if (!step_args_ok(pl, phase, flags, d_q, d_k_tree, d_v_tree, d_plen, d_rtok)) return FC_ERR_INVALID_ARG;
   const bool attention = !(flags & FC_PIPELINE_NO_ATTENTION);
-  if (!pl || (phase != 0 && phase != 1) || (flags & ~FC_PIPELINE_NO_ATTENTION) || (attention && !d_q) || !d_k_tree ||
-      !d_v_tree || !d_plen || !d_rtok)
-    return FC_ERR_INVALID_ARG;
-  const fc_pipeline_desc& d = pl->d;
-  const int c = phase, nx = 1 - phase, S = d.n_sources, Np = d.n_pad;
-  const bool rope = d.rope_base > 0.f;
-  const size_t q_row = (size_t)Np * d.H * d.D * 2, kt_row = (size_t)d.Hkv * Np * d.D * 2;  // bytes per sequence
   if (cudaEventRecord(pl->ev_start, static_cast<cudaStream_t>(caller)) != cudaSuccess) return FC_ERR_CUDA;
-  for (int h = 0; h < d.n_parts; ++h) {
-    const fc_pipeline_part& P = pl->parts[h];
-    cudaStream_t s = pl->chain[h], sa = pl->attn[h];
-    const int B = P.batch;
-    if (cudaStreamWaitEvent(s, pl->ev_start, 0) != cudaSuccess) return FC_ERR_CUDA;
-    const void* q = attention ? static_cast<const char*>(d_q) + (size_t)P.first * q_row : nullptr;
-    const void* kt = static_cast<const char*>(d_k_tree) + (size_t)P.first * kt_row;
-    const void* vt = static_cast<const char*>(d_v_tree) + (size_t)P.first * kt_row;
-    const int32_t* want = d_want_hit ? d_want_hit + P.first : nullptr;
-    FcErrorScope scope(P.err);  // the sub-batch's kernels record errors in its own word
-
-    stage_event(stage_events, h, 0, 0, s);
-    if (P.rcache)  // replay-cache lookup and retrieval of the queries it did not serve, one launch
-      FC_TRY(fc_retrieve_cached(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.rcache,
-                                P.rcache_capacity, want, P.skip, d.p, P.drafts, P.draft_len, P.count, P.n_drafts,
-                                P.match_len, s));
-    else
-      FC_TRY(fc_retrieve(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, nullptr, d.p, P.drafts,
-                         P.draft_len, P.count, P.n_drafts, P.match_len, s));
-    if (P.rcache)
-      FC_TRY(fc_rcache_insert(P.rcache, P.rcache_capacity, S, d.p, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.skip,
-                              P.drafts, P.draft_len, P.count, P.n_drafts, P.match_len, s));
-    stage_event(stage_events, h, 0, 1, s);
-    stage_event(stage_events, h, 1, 0, s);
-    FC_TRY(fc_build_tree(S, P.drafts, P.draft_len, P.count, P.n_drafts, pl->weight.data(), d.p.top_k,
-                         d.p.draft_len, P.root, P.kv_len[c], B, d.node_budget, Np, P.tok, P.parent, P.depth, P.pos,
-                         P.mask, P.n_nodes, s));
-    stage_event(stage_events, h, 1, 1, s);
-    if (rope) {
-      FC_TRY(fc_rope(kt, P.k_tree_rot, B, Np, d.Hkv, d.D, 1, P.pos, d.rope_base, s));
-      kt = P.k_tree_rot;
-    }
-    if (attention) {  // on its own stream, ordered by an event pair
-      if (cudaEventRecord(pl->ev_pre[h], s) != cudaSuccess || cudaStreamWaitEvent(sa, pl->ev_pre[h], 0) != cudaSuccess)
-        return FC_ERR_CUDA;
-      stage_event(stage_events, h, 2, 0, sa);
-      if (rope)
-        FC_TRY(fc_tree_attn_rope(q, P.k_cache, P.v_cache, d.kv_cap, P.kv_len[c], kt, vt, P.mask, P.n_nodes, B, Np,
-                                 d.H, d.Hkv, d.D, d.scale, P.pos, d.rope_base, P.attn_out, P.attn_ws,
-                                 P.attn_ws_bytes, sa));
-      else
-        FC_TRY(fc_tree_attn(q, P.k_cache, P.v_cache, d.kv_cap, P.kv_len[c], kt, vt, P.mask, P.n_nodes, B, Np, d.H,
-                            d.Hkv, d.D, d.scale, P.attn_out, P.attn_ws, P.attn_ws_bytes, sa));
-      stage_event(stage_events, h, 2, 1, sa);
-      if (cudaEventRecord(pl->ev_post[h], sa) != cudaSuccess ||
-          cudaStreamWaitEvent(s, pl->ev_post[h], 0) != cudaSuccess)
-        return FC_ERR_CUDA;
-    }
-    stage_event(stage_events, h, 3, 0, s);
-    FC_TRY(fc_synth_argmax(P.tok, P.parent, P.n_nodes, B, Np, d_plen + P.first, d_rtok + (size_t)P.first * Np,
-                           d.vocab, P.argmax, s));
-    FC_TRY(fc_accept(P.tok, P.parent, P.n_nodes, P.argmax, B, Np, P.acc_len, P.path, d.path_cap, P.bonus, s));
-    FC_TRY(fc_kv_append(P.path, P.acc_len, P.bonus, P.tok, kt, vt, B, Np, d.Hkv, d.D, d.path_cap, P.k_cache,
-                        P.v_cache, d.kv_cap, P.kv_len[c], P.kv_len[nx], P.ctx, P.ctx_stride, P.ctx_len[c],
-                        P.ctx_len[nx], P.root, s));
-    stage_event(stage_events, h, 3, 1, s);
+  for (int h = 0; h < pl->d.n_parts; ++h) {
+    if (cudaStreamWaitEvent(pl->chain[h], pl->ev_start, 0) != cudaSuccess) return FC_ERR_CUDA;
+    FC_TRY(enqueue_part(pl, h, phase, attention, d_q, d_k_tree, d_v_tree, d_want_hit, d_plen, d_rtok, stage_events));
   }
   return FC_OK;
+}
+
+extern "C" fc_status fc_pipeline_step_part(fc_pipeline* pl, int part, int phase, int flags, const void* d_q,
+                                           const void* d_k_tree, const void* d_v_tree, const int32_t* d_want_hit,
+                                           const int32_t* d_plen, const uint32_t* d_rtok, fc_stream caller,
+                                           void* const* stage_events) {
+  FC_NVTX_RANGE();
+  if (!step_args_ok(pl, phase, flags, d_q, d_k_tree, d_v_tree, d_plen, d_rtok) || part < 0 ||
+      part >= pl->d.n_parts)
+    return FC_ERR_INVALID_ARG;
+  if (cudaEventRecord(pl->ev_fork[part], static_cast<cudaStream_t>(caller)) != cudaSuccess ||
+      cudaStreamWaitEvent(pl->chain[part], pl->ev_fork[part], 0) != cudaSuccess)
+    return FC_ERR_CUDA;
+  return enqueue_part(pl, part, phase, !(flags & FC_PIPELINE_NO_ATTENTION), d_q, d_k_tree, d_v_tree, d_want_hit,
+                      d_plen, d_rtok, stage_events);
 }
 
 extern "C" fc_status fc_pipeline_error(fc_pipeline* pl, int part) {
@@ -218,6 +253,14 @@ extern "C" fc_status fc_pipeline_error(fc_pipeline* pl, int part) {
 extern "C" fc_stream fc_pipeline_stream(const fc_pipeline* pl, int part) {
   if (!pl || part < 0 || part >= (int)pl->chain.size()) return nullptr;
   return pl->chain[part];
+}
+
+extern "C" fc_status fc_pipeline_join_part(fc_pipeline* pl, int part, fc_stream caller) {
+  if (!pl || part < 0 || part >= (int)pl->chain.size()) return FC_ERR_INVALID_ARG;
+  if (cudaEventRecord(pl->ev_done[part], pl->chain[part]) != cudaSuccess ||
+      cudaStreamWaitEvent(static_cast<cudaStream_t>(caller), pl->ev_done[part], 0) != cudaSuccess)
+    return FC_ERR_CUDA;
+  return FC_OK;
 }
 
 extern "C" fc_status fc_pipeline_join(fc_pipeline* pl, fc_stream caller) {

@@ -78,7 +78,7 @@ EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build
            "fc_cache_init", "fc_cache_search", "fc_cache_update", "fc_missing_bytes", "fc_missing_init",
            "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_tree_attn_streamed", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_gemm_kv_heads", "fc_gemm_silu_mul", "fc_interleave_gate_up", "fc_embed",
            "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax",
-           "fc_pipeline_create", "fc_pipeline_step", "fc_pipeline_stream", "fc_pipeline_error", "fc_pipeline_join",
+           "fc_pipeline_create", "fc_pipeline_step", "fc_pipeline_step_part", "fc_pipeline_join_part", "fc_pipeline_stream", "fc_pipeline_error", "fc_pipeline_join",
            "fc_pipeline_destroy"]
 
 
@@ -154,6 +154,8 @@ def _load():
         "fc_pipeline_create": (C.c_int, [C.POINTER(fc_pipeline_desc), C.POINTER(vp)]),
         "fc_pipeline_step": (C.c_int, [vp, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]),
         "fc_pipeline_join": (C.c_int, [vp, vp]),
+        "fc_pipeline_step_part": (C.c_int, [vp, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]),
+        "fc_pipeline_join_part": (C.c_int, [vp, i32, vp]),
         "fc_pipeline_stream": (vp, [vp, i32]),
         "fc_pipeline_error": (C.c_int, [vp, i32]),
         "fc_pipeline_destroy": (None, [vp]),
@@ -882,11 +884,12 @@ class Pipeline:
         self.streams = [torch.cuda.ExternalStream(LIB.fc_pipeline_stream(h, i)) for i in range(len(parts))]
         _PIPELINES.add(self)
 
-    def step(self, phase, q, k_tree, v_tree, want_hit, plen, rtok, attention=True, events=None):
-        """Enqueue one step of every sub-batch after the work on the current
-        stream (inputs batch-wide, as fc_pipeline_step); ``events``: None or,
-        per sub-batch, a dict mapping "retrieve" / "tree" / "attn" / "tail" to
-        a (start, end) pair of torch.cuda.Event."""
+    def step(self, phase, q, k_tree, v_tree, want_hit, plen, rtok, attention=True, events=None, part=None):
+        """Enqueue one step of every sub-batch (or of sub-batch ``part``
+        alone) after the work on the current stream (inputs batch-wide, as
+        fc_pipeline_step); ``events``: None or, per sub-batch, a dict mapping
+        "retrieve" / "tree" / "attn" / "tail" to a (start, end) pair of
+        torch.cuda.Event."""
         qs, ks, bs, rs = self.shapes
         if attention:
             _need(q, torch.bfloat16, "q", qs)
@@ -907,13 +910,20 @@ class Pipeline:
                             if not t.cuda_event:  # torch creates its events at the first record
                                 t.record()
                             ev[8 * h + 2 * j + k] = t.cuda_event
-        _check("fc_pipeline_step", LIB.fc_pipeline_step(
-            self.handle, phase, 0 if attention else PIPELINE_NO_ATTENTION, _ptr(q) if attention else None,
-            _ptr(k_tree), _ptr(v_tree), _ptr(want_hit), _ptr(plen), _ptr(rtok), _stream(), ev))
+        args = (phase, 0 if attention else PIPELINE_NO_ATTENTION, _ptr(q) if attention else None, _ptr(k_tree),
+                _ptr(v_tree), _ptr(want_hit), _ptr(plen), _ptr(rtok), _stream(), ev)
+        if part is None:
+            _check("fc_pipeline_step", LIB.fc_pipeline_step(self.handle, *args))
+        else:
+            _check("fc_pipeline_step_part", LIB.fc_pipeline_step_part(self.handle, part, *args))
 
-    def join(self):
-        """The current stream waits for everything enqueued on the sub-batches."""
-        _check("fc_pipeline_join", LIB.fc_pipeline_join(self.handle, _stream()))
+    def join(self, part=None):
+        """The current stream waits for everything enqueued on the sub-batches
+        (or on sub-batch ``part``)."""
+        if part is None:
+            _check("fc_pipeline_join", LIB.fc_pipeline_join(self.handle, _stream()))
+        else:
+            _check("fc_pipeline_join_part", LIB.fc_pipeline_join_part(self.handle, part, _stream()))
 
     def error(self, part):
         """Sub-batch ``part``'s device errors since the last call (a status

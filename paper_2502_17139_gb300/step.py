@@ -333,6 +333,28 @@ class PipelinedStepLoop:
             self.join()
         return g
 
+    def capture_parts(self, inputs, attention=True):
+        """One CUDA graph per sub-batch, each holding an even number of steps
+        of that sub-batch alone (inputs as capture).  Replay them on streams of
+        their own: the sub-batches then never join, as in the eager loop.  A
+        sub-batch reads only its slice of the inputs, so each may copy its
+        slice of the next inputs on its own stream before its replay."""
+        if any(lp.cur != 0 for lp in self.loops):
+            raise RuntimeError("capture at an even step")
+        if len(inputs) < 2 or len(inputs) % 2:
+            raise ValueError("capture an even number of steps (the lengths alternate between two buffers)")
+        self.join()
+        torch.cuda.current_stream().synchronize()
+        graphs = []
+        for h in range(len(self.loops)):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, capture_error_mode="thread_local"):
+                for t, ins in enumerate(inputs):
+                    self.pipe.step(t & 1, *ins, attention=attention, part=h)
+                self.pipe.join(part=h)
+            graphs.append(g)
+        return graphs
+
     def reset(self):
         self.join()
         for lp in self.loops:

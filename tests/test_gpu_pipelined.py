@@ -247,3 +247,44 @@ def test_pipelined_errors_attributed_to_their_sub_batch(fc, setup):
     assert piped.errors() == ["FC_OK", "FC_ERR_INVALID_ARG"]
     assert fc.fc_get_error() == "FC_OK"
     assert piped.errors() == ["FC_OK", "FC_OK"]
+
+
+def test_pipelined_part_graphs(fc, setup):
+    """One CUDA graph per sub-batch (fc_pipeline_step_part), each replayed on a
+    stream of its own, follows the eager pipelined trajectory."""
+    from paper_2502_17139_gb300.step import PipelinedStepLoop
+    ins, steps = setup["ins"], setup["steps"]
+    eager = PipelinedStepLoop(3, *setup["args"], **setup["kw"])
+    want = []
+    for s in range(steps):
+        eager.step(*ins[s])
+        if s % 2 == 1:
+            eager.join()
+            want.append(state(eager))
+    graphed = PipelinedStepLoop(3, *setup["args"], **setup["kw"])
+    graphed.step(*ins[0])
+    graphed.step(*ins[1])
+    graphed.join()
+    static = [tuple(t.clone() for t in ins[2]), tuple(t.clone() for t in ins[3])]
+    graphs = graphed.capture_parts(static)
+    assert len(graphs) == 3
+    streams = [torch.cuda.Stream() for _ in graphs]
+    got = []
+    main = torch.cuda.current_stream()
+    for s in range(2, steps, 2):
+        for j in range(2):
+            for dst, src in zip(static[j], ins[s + j]):
+                dst.copy_(src)
+        ready = torch.cuda.Event()
+        ready.record(main)
+        for g, st in zip(graphs, streams):
+            st.wait_event(ready)
+            with torch.cuda.stream(st):
+                g.replay()
+        for st in streams:
+            main.wait_stream(st)
+        got.append(state(graphed))
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_OK" and graphed.errors() == ["FC_OK"] * 3
+    for w, gt in zip(want[1:], got):
+        same(w, gt)
