@@ -56,6 +56,10 @@ def test_host_validation_without_gpu(lib):
     assert L.fc_retrieve(views, 1, 1, 64, 1, 4, nul, fc.params(16, 2, 16, 8, 0), 1, 1, 1, 1, 1, nul) == 2
     # empty batch is a no-op
     assert L.fc_retrieve(views, 1, nul, 64, nul, 0, nul, p, nul, nul, nul, nul, nul, nul) == 0
+    # cached retrieval: no table, a capacity that is not a power of two, no skip output
+    assert L.fc_retrieve_cached(views, 1, 16, 64, 16, 4, nul, 64, nul, 16, p, 16, 16, 16, 16, 16, nul) == 1
+    assert L.fc_retrieve_cached(views, 1, 16, 64, 16, 4, 16, 60, nul, 16, p, 16, 16, 16, 16, 16, nul) == 1
+    assert L.fc_retrieve_cached(views, 1, 16, 64, 16, 4, 16, 64, nul, nul, p, 16, 16, 16, 16, 16, nul) == 1
     # attention: head dim / tree padding / GQA ratio outside the supported set
     args = [1, 1, 1, 128, 1, 1, 1, 8, 1, 2]
     assert L.fc_tree_attn(*args, 64, 32, 8, 64, C.c_float(0.1), 1, nul, 0, nul) == 2
@@ -221,6 +225,9 @@ def test_pipeline_host_validation(lib):
     assert not h.value
     nul = None
     assert L.fc_pipeline_step(nul, 0, 0, 16, 16, 16, nul, 16, 16, nul, nul) == 1
+    assert L.fc_pipeline_step_part(nul, 0, 0, 0, 16, 16, 16, nul, 16, 16, nul, nul) == 1
     assert L.fc_pipeline_join(nul, nul) == 1
+    assert L.fc_pipeline_join_part(nul, 0, nul) == 1
+    assert L.fc_pipeline_error(nul, 0) == 1
     assert L.fc_pipeline_stream(nul, 0) is None
     L.fc_pipeline_destroy(nul)
