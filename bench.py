@@ -100,7 +100,7 @@ def parse_args(argv=None):
     ap.add_argument("--no-graph", action="store_true",
                     help="step mode: skip timing the same steps replayed from CUDA graphs (two steps per graph)")
     ap.add_argument("--split", type=int, default=4,
-                    help="step mode: sub-batches of the sequences, each on CUDA streams of its own, issued by the "
+                    help="step and algorithm1 modes: sub-batches of the sequences, each on CUDA streams of its own, issued by the "
                          "native step executor (1: the single-stream StepLoop)")
     ap.add_argument("--all-occ", action="store_true",
                     help="retrieve mode: also time the all-occurrence trie (fc_retrieve_all + fc_build_tree_all)")
@@ -1309,15 +1309,19 @@ def run_small(args, rank, ws, local):
 def run_algorithm1(args, rank, ws, local):
     """The step loop of the default workload with Algorithm 1 in place of the
     replay cache: per sequence a CACHE (l = 50, 20-token output pieces,
-    8192 words), one missing table for the batch.  --fill untimed steps fill
-    the CACHE first, so the timed steps search active stores; the stage
-    events time the CACHE search, the whole retrieval stage (CACHE search,
-    datastore fallback, missing-table insert) and the CACHE update."""
+    8192 words), a missing table per sub-batch (one for the batch with
+    --split 1).  --fill untimed steps fill the CACHE first, so the timed
+    steps search active stores.  With --split N > 1 the native step executor
+    runs N sub-batches on streams of their own, as in the default mode; the
+    stage events then time each sub-batch's retrieval stage (CACHE search,
+    datastore fallback, missing-table insert), tree, attention and tail
+    (predictions, acceptance, append, CACHE update).  With --split 1 they
+    also time the CACHE search and the CACHE update alone."""
     import torch
 
     import paper_2502_17139_gb300.fastcoder as fc
     import paper_2502_17139_gb300.synth as synth
-    from paper_2502_17139_gb300.step import StepLoop
+    from paper_2502_17139_gb300.step import PipelinedStepLoop, StepLoop
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
@@ -1344,10 +1348,15 @@ def run_algorithm1(args, rank, ws, local):
     vt_pool = torch.randn((P, B, Hkv, n_pad, D), generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
     plen_d, rtok_d = to_dev(inp["plen"]), to_dev(inp["rtok"])
     zeros = torch.zeros(B, dtype=torch.int32, device=dev)
+    nsub = max(1, min(args.split, B))
 
     def make():
-        return StepLoop(sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, [1, 1], H, Hkv, D, cap, kv0,
-                        synth.VOCAB, device=dev, k_cache=kc, v_cache=vc, seq_cache=seq)
+        largs = (sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, [1, 1], H, Hkv, D, cap, kv0,
+                 synth.VOCAB)
+        lkw = dict(device=dev, k_cache=kc, v_cache=vc, seq_cache=seq)
+        return PipelinedStepLoop(nsub, *largs, **lkw) if nsub > 1 else StepLoop(*largs, **lkw)
+
+    loops_of = lambda lp: lp.loops if nsub > 1 else [lp]
 
     # untimed pass over the whole trajectory: what each step's retrieval did
     loop = make()
@@ -1355,6 +1364,8 @@ def run_algorithm1(args, rank, ws, local):
     for s in range(F + W + K):
         j = s % P
         loop.step(q_pool[j], kt_pool[j], vt_pool[j], zeros, plen_d[s], rtok_d[s], attention=False)
+        if nsub > 1:
+            loop.join()
         codes.append(loop.skip.clone())
         accs.append(loop.acc["acc_len"].clone())
     codes = torch.stack(codes).cpu().numpy()[F + W:]
@@ -1363,44 +1374,59 @@ def run_algorithm1(args, rank, ws, local):
     vc[:, :, kv0:].zero_()
 
     loop = make()
-    names = ("retrieve", "cache_search", "cache_update", "tree", "attn", "tail")
-    ev = {nm: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-          for nm in names}
+    mk = lambda: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    names = ("retrieve", "tree", "attn", "tail") + (() if nsub > 1 else ("cache_search", "cache_update"))
+    ev = [[{nm: mk() for nm in names} for _ in range(nsub)] for _ in range(K)]
+    for per_step in ev:  # torch creates an event at its first record: do that before the timed region
+        for e in per_step:
+            for a, b in e.values():
+                a.record()
+                b.record()
 
     def do_step(s, i=None):
         j = s % P
-        loop.step(q_pool[j], kt_pool[j], vt_pool[j], zeros, plen_d[s], rtok_d[s],
-                  events=None if i is None else {nm: ev[nm][i] for nm in names})
+        evs = None if i is None else (ev[i] if nsub > 1 else ev[i][0])
+        loop.step(q_pool[j], kt_pool[j], vt_pool[j], zeros, plen_d[s], rtok_d[s], events=evs)
 
     for s in range(F + W):
         do_step(s)
-    assert fc.fc_get_error() == "FC_OK"
+    if nsub > 1:
+        loop.join()
+    assert step_status(fc, loop) == "FC_OK"
     barrier(ws)
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
     clocks.wait_first()
     stream = torch.cuda.current_stream()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    start.record(stream)
-    for i in range(K):
-        do_step(F + W + i, i)
-    end.record(stream)
-    torch.cuda.synchronize()
+    with no_gc():
+        start.record(stream)
+        for i in range(K):
+            do_step(F + W + i, i)
+        if nsub > 1:
+            loop.join()
+        end.record(stream)
+        torch.cuda.synchronize()
     clock_rec = clocks.stop()
     barrier(ws)
-    assert fc.fc_get_error() == "FC_OK"
+    status = step_status(fc, loop)
+    assert status == "FC_OK", status
     t_max = max_over_ranks(start.elapsed_time(end), ws)
-    stage = {nm: statistics.mean(a.elapsed_time(b) for a, b in ev[nm]) for nm in names}
-    meta = loop.seq_cache.meta.cpu().numpy()
-    m_stored = int(loop.missing.table[0].item())
+    # each stage's mean time per sub-batch launch (sub-batches overlap: they do not add up)
+    stage = {nm: statistics.mean(a.elapsed_time(b) for per_step in ev for e in per_step for a, b in [e[nm]])
+             for nm in names}
+    subs = loops_of(loop)
+    meta = torch.cat([lp.seq_cache.meta for lp in subs]).cpu().numpy()
+    m_stored = sum(int(lp.missing.table[0].item()) for lp in subs)
     # the same contexts, retrieved from the datastore alone, and the CACHE
-    # search alone on the final stores (both repeatable: they write only
-    # their outputs)
+    # search alone on the final stores of one sub-batch (both repeatable:
+    # they write only their outputs)
     res_all = fc.fc_retrieve(sources, loop.ctx, loop.ctx_len_now, p)
     ds_ms = _gpu_ms(lambda: fc.fc_retrieve(sources, loop.ctx, loop.ctx_len_now, p, out=res_all), reps=20, warm=3)
-    st = torch.empty(B, dtype=torch.int32, device=dev)
-    res_c = fc.retrieve_outputs(len(sources) + 1, B, p, dev)
-    cs_ms = _gpu_ms(lambda: fc.fc_cache_search(loop.seq_cache, loop.missing, loop.ctx, loop.ctx_len_now, p,
+    lp0 = subs[0]
+    st = torch.empty(lp0.B, dtype=torch.int32, device=dev)
+    res_c = fc.retrieve_outputs(len(sources) + 1, lp0.B, p, dev)
+    cs_ms = _gpu_ms(lambda: fc.fc_cache_search(lp0.seq_cache, lp0.missing, lp0.ctx, lp0.ctx_len_now, p,
                                                len(sources), res_c, st), reps=20, warm=3)
     n_q = codes.size
     return {"metric": METRIC, "value": weak_value(K, ws, t_max), "unit": UNIT, "n_gpus": ws, "steps": K,
@@ -1409,7 +1435,14 @@ def run_algorithm1(args, rank, ws, local):
             "config": {"workload": WORKLOAD.replace("50% replay-cache hits", "Algorithm 1: per-sequence CACHE "
                                                     "(l=50, 20-token pieces, 8192 words) + missing table"),
                        "fill_steps": F, "batch_per_gpu": B, "kv_len0": kv0,
-                       "l2": "inputs larger than L2 (KV cache 2.2 GB per GPU)"},
+                       "l2": "inputs larger than L2 (KV cache 2.2 GB per GPU)",
+                       "streams": (f"{nsub} sub-batches of {B // nsub}-{-(-B // nsub)} sequences issued by the "
+                                   "native step executor, each with its own missing table" if nsub > 1
+                                   else "one stream, one missing table")},
+            # per sub-batch step: CACHE search, retrieval, missing insert, tree, attention,
+            # predictions, accept, append, CACHE update
+            "gpu_launches": 9 * K * nsub,
+            "sub_batches": nsub,
             "stages_ms_per_step": stage,
             "cache": {"served_frac": float((codes == 1).sum() / n_q), "skipped_frac": float((codes == 2).sum() / n_q),
                       "datastore_frac": float((codes == 0).sum() / n_q),
@@ -1417,6 +1450,7 @@ def run_algorithm1(args, rank, ws, local):
                       "acc_len_datastore": float(accs[codes == 0].mean()) if (codes == 0).any() else None,
                       "mean_sequences": float(meta[:, 1].mean()), "mean_words": float(meta[:, 0].mean()),
                       "missing_keys": m_stored, "cache_search_alone_us": cs_ms * 1e3,
+                      "cache_search_alone_batch": lp0.B,
                       "datastore_retrieval_all_queries_us": ds_ms * 1e3},
             "clocks": clock_rec}
 

@@ -714,9 +714,10 @@ fc_status fc_synth_argmax(const uint32_t* d_tok, const int32_t* d_parent, const 
 
 /* ------------------------------------------------------------------------
  * Native step executor (the decoding step of Section IV-C and IV-D over
- * sub-batches: replay-cache lookup -> fc_retrieve -> insert ->
+ * sub-batches: replay-cache lookup -> fc_retrieve -> insert (or Algorithm
+ * 1's CACHE search -> fc_retrieve -> missing-table insert) ->
  * fc_build_tree -> [fc_rope] -> fc_tree_attn[_rope] -> fc_synth_argmax ->
- * fc_accept -> fc_kv_append).  One call enqueues the whole step of every
+ * fc_accept -> fc_kv_append [-> fc_cache_update]).  One call enqueues the whole step of every
  * sub-batch; each sub-batch runs on two streams the executor owns, a
  * high-priority one for its latency-bound chain and a low-priority one for
  * its attention, so sub-batches overlap.  The executor owns no device
@@ -759,6 +760,15 @@ typedef struct {
   uint32_t* err;            /* this sub-batch's device error word (4 bytes, zeroed by the
                                caller; fc_pipeline_error reads it), or NULL: its kernels
                                then record errors in the library-wide words of fc_get_error */
+  /* Algorithm 1 (Section IV-B/C) in place of the replay cache (rcache must then be NULL):
+   * fc_cache_search -> fc_retrieve of the queries it leaves to the datastore ->
+   * fc_missing_insert, and fc_cache_update after the append.  The retrieval outputs
+   * above then hold n_sources + 1 slots, the CACHE's last, and `skip` holds the
+   * search's per-query state. */
+  fc_cache seq_cache;       /* this sub-batch's CACHE (fc_cache_init'ed); d_words NULL: none */
+  void* missing;            /* this sub-batch's missing table M (fc_missing_init'ed with key
+                               length n_min), or NULL: no M */
+  int32_t missing_capacity;
 } fc_pipeline_part;
 
 typedef struct {
@@ -772,12 +782,15 @@ typedef struct {
   float rope_base;              /* 0: q and tree keys arrive rotated; > 0: RoPE base */
   int32_t n_parts;
   const fc_pipeline_part* parts;  /* host [n_parts], copied */
+  uint32_t cache_weight;        /* tree weight of the CACHE slot (parts with a CACHE) */
 } fc_pipeline_desc;
 
 typedef struct fc_pipeline fc_pipeline;
 
 /* Checks the description (FC_ERR_INVALID_ARG: a missing buffer, a
- * non-positive size, equal ping-pong buffers), creates the streams and
+ * non-positive size, equal ping-pong buffers, a sub-batch with both a
+ * replay cache and a CACHE, a missing table without a CACHE, a CACHE view
+ * fc_cache_search would reject), creates the streams and
  * events and returns the executor in *out.  FC_ERR_CUDA if a stream or
  * event cannot be created (nothing is left allocated). */
 fc_status fc_pipeline_create(const fc_pipeline_desc* desc, fc_pipeline** out);

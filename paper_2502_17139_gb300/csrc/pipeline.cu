@@ -6,8 +6,9 @@
 // The sequences of a batch are independent, so sub-batch h may run step
 // s + 1 while sub-batch h' is still in step s.  Per sub-batch the executor
 // owns two streams: a high-priority one for the latency-bound chain
-// (replay-cache lookup with retrieval, insert, tree build, predictions,
-// acceptance, append) and a low-priority one for the attention launch,
+// (replay-cache lookup with retrieval and insert, or Algorithm 1's CACHE
+// search, retrieval and missing-table insert; tree build, predictions,
+// acceptance, append and, with the CACHE, its update) and a low-priority one for the attention launch,
 // ordered by an event pair.  When SMs free up, the block scheduler then
 // starts another sub-batch's chain ahead of this sub-batch's remaining
 // attention CTAs.  The executor holds no device memory: every buffer
@@ -17,6 +18,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cstdint>
 #include <new>
 #include <vector>
 
@@ -56,6 +58,19 @@ bool part_ok(const fc_pipeline_desc& d, const fc_pipeline_part& p) {
   if (p.ctx_len[0] == p.ctx_len[1] || p.kv_len[0] == p.kv_len[1]) return false;
   if (p.rcache && p.rcache_capacity < 1) return false;
   if (d.rope_base > 0.f && !p.k_tree_rot) return false;
+  const fc_cache& q = p.seq_cache;
+  if (q.d_words) {  // Algorithm 1: the CACHE replaces the replay cache
+    if (p.rcache || !q.d_meta || q.capacity < 16 || q.capacity % 4 || q.capacity > FC_CACHE_MAX_WORDS ||
+        q.min_size < 0 || q.chunk < 1 || q.ctx_keep < 0 || q.ctx_keep > FC_MAX_NMAX ||
+        reinterpret_cast<uintptr_t>(q.d_words) % 16)
+      return false;
+    // M: a power-of-two capacity from 2 to 2^24 slots
+    if (p.missing && (p.missing_capacity < 2 || p.missing_capacity > (1 << 24) ||
+                      (p.missing_capacity & (p.missing_capacity - 1))))
+      return false;
+  } else if (p.missing) {
+    return false;
+  }
   return true;
 }
 
@@ -90,6 +105,7 @@ extern "C" fc_status fc_pipeline_create(const fc_pipeline_desc* d, fc_pipeline**
   pl->parts.assign(d->parts, d->parts + d->n_parts);
   pl->sources.assign(d->sources, d->sources + d->n_sources);
   pl->weight.assign(d->src_weight, d->src_weight + d->n_sources);
+  pl->weight.push_back(d->cache_weight);  // slot n_sources: the CACHE's result (Algorithm 1 parts)
   pl->d.parts = nullptr;  // the copies above are the ones used
   pl->d.sources = nullptr;
   pl->d.src_weight = nullptr;
@@ -151,20 +167,29 @@ fc_status enqueue_part(fc_pipeline* pl, int h, int c, bool attention, const void
   const int32_t* want = d_want_hit ? d_want_hit + P.first : nullptr;
   FcErrorScope scope(P.err);  // the sub-batch's kernels record errors in its own word
 
+  const bool seq = P.seq_cache.d_words != nullptr;
   stage_event(stage_events, h, 0, 0, s);
-  if (P.rcache)  // replay-cache lookup and retrieval of the queries it did not serve, one launch
+  if (seq) {  // Algorithm 1: the CACHE and M first, the datastores for the queries they leave
+    FC_TRY(fc_cache_search(&P.seq_cache, P.missing, P.missing_capacity, P.ctx, P.ctx_stride, P.ctx_len[c], B, d.p,
+                           S, P.drafts, P.draft_len, P.count, P.n_drafts, P.match_len, P.skip, s));
+    FC_TRY(fc_retrieve(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.skip, d.p, P.drafts,
+                       P.draft_len, P.count, P.n_drafts, P.match_len, s));
+    if (P.missing)
+      FC_TRY(fc_missing_insert(P.missing, P.missing_capacity, d.p.n_min, P.ctx, P.ctx_stride, P.ctx_len[c], B,
+                               P.skip, P.n_drafts, S, s));
+  } else if (P.rcache) {  // replay-cache lookup and retrieval of the queries it did not serve, one launch
     FC_TRY(fc_retrieve_cached(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.rcache,
                               P.rcache_capacity, want, P.skip, d.p, P.drafts, P.draft_len, P.count, P.n_drafts,
                               P.match_len, s));
-  else
-    FC_TRY(fc_retrieve(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, nullptr, d.p, P.drafts,
-                       P.draft_len, P.count, P.n_drafts, P.match_len, s));
-  if (P.rcache)
     FC_TRY(fc_rcache_insert(P.rcache, P.rcache_capacity, S, d.p, P.ctx, P.ctx_stride, P.ctx_len[c], B, P.skip,
                             P.drafts, P.draft_len, P.count, P.n_drafts, P.match_len, s));
+  } else {
+    FC_TRY(fc_retrieve(pl->sources.data(), S, P.ctx, P.ctx_stride, P.ctx_len[c], B, nullptr, d.p, P.drafts,
+                       P.draft_len, P.count, P.n_drafts, P.match_len, s));
+  }
   stage_event(stage_events, h, 0, 1, s);
   stage_event(stage_events, h, 1, 0, s);
-  FC_TRY(fc_build_tree(S, P.drafts, P.draft_len, P.count, P.n_drafts, pl->weight.data(), d.p.top_k,
+  FC_TRY(fc_build_tree(seq ? S + 1 : S, P.drafts, P.draft_len, P.count, P.n_drafts, pl->weight.data(), d.p.top_k,
                        d.p.draft_len, P.root, P.kv_len[c], B, d.node_budget, Np, P.tok, P.parent, P.depth, P.pos,
                        P.mask, P.n_nodes, s));
   stage_event(stage_events, h, 1, 1, s);
@@ -195,6 +220,8 @@ fc_status enqueue_part(fc_pipeline* pl, int h, int c, bool attention, const void
   FC_TRY(fc_kv_append(P.path, P.acc_len, P.bonus, P.tok, kt, vt, B, Np, d.Hkv, d.D, d.path_cap, P.k_cache,
                       P.v_cache, d.kv_cap, P.kv_len[c], P.kv_len[nx], P.ctx, P.ctx_stride, P.ctx_len[c],
                       P.ctx_len[nx], P.root, s));
+  if (seq)  // the verified retrieval and the completed output pieces go to the CACHE
+    FC_TRY(fc_cache_update(&P.seq_cache, P.ctx, P.ctx_stride, P.ctx_len[c], P.ctx_len[nx], P.acc_len, B, s));
   stage_event(stage_events, h, 3, 1, s);
   return FC_OK;
 }

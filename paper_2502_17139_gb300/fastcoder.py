@@ -61,7 +61,8 @@ class fc_pipeline_part(C.Structure):
                 ("pos", C.c_void_p), ("mask", C.c_void_p), ("n_nodes", C.c_void_p), ("k_cache", C.c_void_p),
                 ("v_cache", C.c_void_p), ("k_tree_rot", C.c_void_p), ("attn_out", C.c_void_p),
                 ("attn_ws", C.c_void_p), ("attn_ws_bytes", C.c_size_t), ("argmax", C.c_void_p),
-                ("acc_len", C.c_void_p), ("path", C.c_void_p), ("bonus", C.c_void_p), ("err", C.c_void_p)]
+                ("acc_len", C.c_void_p), ("path", C.c_void_p), ("bonus", C.c_void_p), ("err", C.c_void_p),
+                ("seq_cache", fc_cache), ("missing", C.c_void_p), ("missing_capacity", C.c_int32)]
 
 
 class fc_pipeline_desc(C.Structure):
@@ -69,7 +70,7 @@ class fc_pipeline_desc(C.Structure):
                 ("src_weight", C.POINTER(C.c_uint32)), ("node_budget", C.c_int32), ("n_pad", C.c_int32),
                 ("H", C.c_int32), ("Hkv", C.c_int32), ("D", C.c_int32), ("kv_cap", C.c_int32),
                 ("path_cap", C.c_int32), ("vocab", C.c_uint32), ("scale", C.c_float), ("rope_base", C.c_float),
-                ("n_parts", C.c_int32), ("parts", C.POINTER(fc_pipeline_part))]
+                ("n_parts", C.c_int32), ("parts", C.POINTER(fc_pipeline_part)), ("cache_weight", C.c_uint32)]
 
 
 EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build_workspace", "fc_datastore_build",
@@ -835,14 +836,18 @@ def _close_pipelines():
 
 
 def pipeline_part(batch, first, ctx, ctx_len, kv_len, root, rcache, skip, res, tree, k_cache, v_cache, k_tree_rot,
-                  attn_out, attn_ws, argmax, acc, err=None) -> fc_pipeline_part:
+                  attn_out, attn_ws, argmax, acc, err=None, seq_cache=None, missing=None) -> fc_pipeline_part:
     """One sub-batch's buffers (device tensors the caller keeps alive):
     ctx_len and kv_len are pairs (the ping-pong lengths), rcache a
     RetrievalCache or None, res/tree/acc the dicts of retrieve_outputs,
     tree_outputs and fc_accept's outputs, err None or a zeroed one-element
-    int32 tensor: the sub-batch's own error word."""
+    int32 tensor: the sub-batch's own error word.  seq_cache / missing: a
+    SequenceCache and MissingTable (Algorithm 1, in place of rcache); res
+    then holds one more slot, the CACHE's."""
     if err is not None:
         _need(err, torch.int32, "err", (1,))
+    if seq_cache is not None and seq_cache.batch != batch:
+        raise ValueError("the CACHE must cover the sub-batch")
     _need(ctx, torch.int32, "ctx", (batch, ctx.shape[1]))
     for t in (*ctx_len, *kv_len, root, skip):
         _need(t, torch.int32, "length", (batch,))
@@ -855,7 +860,9 @@ def pipeline_part(batch, first, ctx, ctx_len, kv_len, root, rcache, skip, res, t
         _ptr(res["n_drafts"]), _ptr(res["match_len"]), _ptr(tree["tok"]), _ptr(tree["parent"]), _ptr(tree["depth"]),
         _ptr(tree["pos"]), _ptr(tree["mask"]), _ptr(tree["n_nodes"]), _ptr(k_cache), _ptr(v_cache), _ptr(k_tree_rot),
         _ptr(attn_out), _ptr(attn_ws), 0 if attn_ws is None else attn_ws.numel() * attn_ws.element_size(),
-        _ptr(argmax), _ptr(acc["acc_len"]), _ptr(acc["path"]), _ptr(acc["bonus"]), _ptr(err))
+        _ptr(argmax), _ptr(acc["acc_len"]), _ptr(acc["path"]), _ptr(acc["bonus"]), _ptr(err),
+        seq_cache.view if seq_cache is not None else fc_cache(), _ptr(missing.table) if missing else None,
+        missing.capacity if missing else 0)
 
 
 class Pipeline:
@@ -865,16 +872,17 @@ class Pipeline:
     def __init__(self, sources, p: fc_retrieve_params, src_weight, node_budget, n_pad, H, Hkv, D, kv_cap, path_cap,
                  vocab, parts, scale=None, rope_base=None):
         S = len(sources)
-        if len(src_weight) != S:
-            raise ValueError("one tree weight per source")
+        if len(src_weight) not in (S, S + 1):
+            raise ValueError("one tree weight per source, and optionally the CACHE slot's")
         self.B = sum(pt.batch for pt in parts)
         self.shapes = ((self.B, n_pad, H, D), (self.B, Hkv, n_pad, D), (self.B,), (self.B, n_pad))
         views = (fc_datastore * S)(*[s.view for s in sources])
-        w = (C.c_uint32 * S)(*[int(x) for x in src_weight])
+        w = (C.c_uint32 * S)(*[int(x) for x in src_weight[:S]])
         arr = (fc_pipeline_part * len(parts))(*parts)
         desc = fc_pipeline_desc(views, S, p, w, node_budget, n_pad, H, Hkv, D, kv_cap, path_cap, vocab,
                                 float(scale) if scale is not None else D ** -0.5,
-                                0.0 if rope_base is None else float(rope_base), len(parts), arr)
+                                0.0 if rope_base is None else float(rope_base), len(parts), arr,
+                                int(src_weight[S]) if len(src_weight) > S else 1)
         h = C.c_void_p()
         _check("fc_pipeline_create", LIB.fc_pipeline_create(C.byref(desc), C.byref(h)))
         self.handle = h

@@ -268,12 +268,18 @@ class PipelinedStepLoop:
     caller's stream, so inputs written there are visible.  It does not make
     the caller's stream wait for the sub-batches, or they could not overlap;
     join() does that, and must precede any read of the results on the
-    caller's stream.  Only the replay-cache configuration (with optional
-    RoPE) is pipelined; Algorithm 1's missing table is shared by the whole
-    batch, so it stays with StepLoop."""
+    caller's stream.
+
+    With ``seq_cache`` (Algorithm 1, as StepLoop's) every sub-batch keeps a
+    CACHE and a missing table M of its own.  The CACHE is per sequence in
+    any case.  M only lets a query skip a datastore search that would find
+    nothing (its keys are contexts whose search found no continuation in any
+    source), so a per-sub-batch M changes no draft: each sub-batch is
+    exactly the single loop over its slice of the sequences."""
 
     def __init__(self, n_split, sources, ctx, ctx_len, p, node_budget, n_pad, src_weight, H, Hkv, D, kv_cap,
-                 kv_len0, vocab, cache_capacity=1 << 14, device="cuda", k_cache=None, v_cache=None, rope_base=None):
+                 kv_len0, vocab, cache_capacity=1 << 14, device="cuda", k_cache=None, v_cache=None, rope_base=None,
+                 seq_cache=None):
         B = ctx.shape[0]
         self.slices = sub_batch_slices(B, n_split)
         self.B = B
@@ -284,13 +290,15 @@ class PipelinedStepLoop:
         # the StepLoops hold each sub-batch's buffers and initial state
         self.loops = [StepLoop(sources, ctx[sl], ctx_len[sl], p, node_budget, n_pad, src_weight, H, Hkv, D, kv_cap,
                                kv0[sl], vocab, cache_capacity=cache_capacity, device=device,
-                               k_cache=self.k_cache[sl], v_cache=self.v_cache[sl], rope_base=rope_base)
+                               k_cache=self.k_cache[sl], v_cache=self.v_cache[sl], rope_base=rope_base,
+                               seq_cache=seq_cache)
                       for sl in self.slices]
         # every sub-batch records its device errors in a word of its own
         self.err_words = torch.zeros((len(self.slices), 1), dtype=torch.int32, device=device)
         parts = [fc.pipeline_part(sl.stop - sl.start, sl.start, lp.ctx, lp.ctx_len, lp.kv_len, lp.root, lp.cache,
                                   lp.skip, lp.res, lp.tree, lp.k_cache, lp.v_cache, lp.k_tree_rot, lp.attn_out,
-                                  lp.attn_ws, lp.argmax, lp.acc, err=self.err_words[h])
+                                  lp.attn_ws, lp.argmax, lp.acc, err=self.err_words[h],
+                                  seq_cache=lp.seq_cache if lp.seq else None, missing=lp.missing if lp.seq else None)
                  for h, (lp, sl) in enumerate(zip(self.loops, self.slices))]
         lp0 = self.loops[0]
         self.pipe = fc.Pipeline(sources, p, lp0.tree_weight, node_budget, n_pad, H, Hkv, D, kv_cap, lp0.path_cap,

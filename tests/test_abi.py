@@ -222,6 +222,20 @@ def test_pipeline_host_validation(lib):
     missing = fc.fc_pipeline_part.from_buffer_copy(part)
     missing.mask = None
     assert L.fc_pipeline_create(C.byref(desc([missing])), C.byref(h)) == 1
+    # Algorithm 1 parts: a CACHE view fc_cache_search would reject, a CACHE
+    # beside a replay cache, a missing table without a CACHE or of a bad size
+    def seq(cache=(buf[30], buf[31], 8192, 50, 20, 16), rcache=None, missing=buf[32], cap=1 << 10):
+        q = fc.fc_pipeline_part.from_buffer_copy(part)
+        q.seq_cache = fc.fc_cache(*cache) if cache else fc.fc_cache()
+        q.rcache, q.rcache_capacity = rcache, 16 if rcache else 0
+        q.missing, q.missing_capacity = missing, cap
+        return q
+    for bad in (seq(rcache=buf[33]), seq(cache=None), seq(cap=3), seq(cap=1 << 25), seq(cap=1),
+                seq(cache=(buf[30], buf[31], 8190, 50, 20, 16)), seq(cache=(buf[30], buf[31], 8, 50, 20, 16)),
+                seq(cache=(buf[30] + 8, buf[31], 8192, 50, 20, 16)), seq(cache=(buf[30], None, 8192, 50, 20, 16)),
+                seq(cache=(buf[30], buf[31], 8192, -1, 20, 16)), seq(cache=(buf[30], buf[31], 8192, 50, 0, 16)),
+                seq(cache=(buf[30], buf[31], 8192, 50, 20, 33))):
+        assert L.fc_pipeline_create(C.byref(desc([part, bad])), C.byref(h)) == 1
     assert not h.value
     nul = None
     assert L.fc_pipeline_step(nul, 0, 0, 16, 16, 16, nul, 16, 16, nul, nul) == 1

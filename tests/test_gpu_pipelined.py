@@ -288,3 +288,67 @@ def test_pipelined_part_graphs(fc, setup):
     assert fc.fc_get_error() == "FC_OK" and graphed.errors() == ["FC_OK"] * 3
     for w, gt in zip(want[1:], got):
         same(w, gt)
+
+
+SEQ = dict(capacity=2048, min_size=3, chunk=8, ctx_keep=16, missing_capacity=1 << 10, weight=2)
+
+
+def seq_state(lp):
+    """A StepLoop's CACHE words and meta, missing table and search states."""
+    return dict(words=lp.seq_cache.words.cpu().clone(), meta=lp.seq_cache.meta.cpu().clone(),
+                missing=lp.missing.table.cpu().clone(), skip=lp.skip.cpu().clone())
+
+
+def test_pipelined_algorithm1_matches_slice_loops(fc, setup):
+    """Algorithm 1 through the executor (CACHE search -> retrieval -> missing
+    insert ... append -> CACHE update per sub-batch), against a StepLoop over
+    each sub-batch's slice of the sequences: every result bit-exact, the
+    attention within 2e-2, and the CACHE stores, missing tables and search
+    states byte for byte; against the single loop over the whole batch (one
+    missing table): the same trees, acceptance, contexts and CACHE stores.
+    The CACHE slot's tree weight is 2, so a wrong slot weight shows in the
+    trees."""
+    from paper_2502_17139_gb300.step import PipelinedStepLoop, StepLoop
+    srcs, ctx, cl = setup["args"][:3]
+    rest, kw, ins = setup["args"][3:], setup["kw"], setup["ins"]
+    piped = PipelinedStepLoop(2, *setup["args"], **kw, seq_cache=SEQ)
+    slices = piped.slices
+    per = [StepLoop(srcs, ctx[sl], cl[sl], *rest, **kw, seq_cache=SEQ) for sl in slices]
+    whole = StepLoop(*setup["args"], **kw, seq_cache=SEQ)
+    codes = []
+    for s in range(setup["steps"]):
+        piped.step(*ins[s])
+        for lp, sl in zip(per, slices):
+            lp.step(*[t[sl] for t in ins[s]])
+        whole.step(*ins[s])
+        piped.join()
+        torch.cuda.synchronize()
+        for h, (lp, sl) in enumerate(zip(per, slices)):
+            a, b = state(lp), state(piped.loops[h])
+            same(a, b)
+            sa, sb = seq_state(lp), seq_state(piped.loops[h])
+            for k in sa:
+                assert torch.equal(sa[k], sb[k]), (s, h, k)
+        a, b = state(whole), state(piped)
+        same(a, b)
+        assert torch.equal(whole.seq_cache.words.cpu(), torch.cat([lp.seq_cache.words for lp in piped.loops]).cpu())
+        assert torch.equal(whole.seq_cache.meta.cpu(), torch.cat([lp.seq_cache.meta for lp in piped.loops]).cpu())
+        codes.append(piped.skip.cpu().numpy())
+    codes = np.stack(codes)
+    assert (codes == 1).any() and (codes == 0).any()  # the CACHE served some queries, the datastores others
+    assert sum(int(lp.missing.table[0].item()) for lp in piped.loops) > 0  # M took keys
+    assert fc.fc_get_error() == "FC_OK" and piped.errors() == ["FC_OK", "FC_OK"]
+    # reset empties the CACHE and M and replays the same trajectory
+    piped.reset()
+    for lp in per:
+        lp.reset()
+    for s in range(2):
+        piped.step(*ins[s])
+        for lp, sl in zip(per, slices):
+            lp.step(*[t[sl] for t in ins[s]])
+    piped.join()
+    for h, lp in enumerate(per):
+        same(state(lp), state(piped.loops[h]))
+        sa, sb = seq_state(lp), seq_state(piped.loops[h])
+        for k in sa:
+            assert torch.equal(sa[k], sb[k]), (h, k)
