@@ -698,6 +698,13 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   }
 }
 
+// 16-byte asynchronous global -> shared copies (cp.async, no mbarrier): a
+// thread issues all of its copies before it waits once for them.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
+
 // ---------------------------------------------------------------------------
 // Streaming variant for short one-tile units: every group's rows fit one
 // 128-row tile (G * n_pad <= 128) and the caches are short, so a unit is a
@@ -810,6 +817,34 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
   const uint32_t bar0 = sbase + L::OFF_BAR;
   auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
 
+  // warps 2-3: a unit's queries into Q buffer q (rows past the unit's G * nn
+  // are zeros), every row's copy in flight at once; the caller waits
+  // (cp_async_wait_all) before it signals the buffer staged
+  auto stage_q = [&](const StreamUnit& su, int q) {
+    const int t0 = tid - 64, rows_total = a.G * su.nn;
+    const uint32_t qt = sQ + q * L::QTILE;
+    for (int e = t0; e < L::QROWS * 16; e += 64) {
+      const int r = e >> 4, ch = e & 15, half = ch >> 3, gran = ch & 7;
+      const uint32_t d = qt + half * L::QHALF + r * 128 + ((gran ^ (r & 7)) << 4);
+      if (r < rows_total) {
+        const int hh = r / su.nn, i = r - hh * su.nn;
+        cp_async16(d, a.q + (((size_t)su.b * a.n_pad + i) * a.H + su.g * a.G + hh) * HD + ch * 8);
+      } else {
+        *reinterpret_cast<uint4*>(smem + (d - sbase)) = make_uint4(0, 0, 0, 0);
+      }
+    }
+  };
+  // The first unit's queries are requested before anything else, so that they
+  // do not queue behind every CTA's first K/V stages.
+  bool q_pre = false;
+  if ((warp == 2 || warp == 3) && n_units > 0) {
+    const StreamUnit su0 = stream_unit(a, (int)blockIdx.x);
+    if (su0.nblk > 0) {
+      stage_q(su0, 0);
+      q_pre = true;
+    }
+  }
+
   // K or V of global block J (block j of unit su) into stage J % NST.  The tree
   // maps' box is 128 rows: rows >= n_pad arrive as zeros.
   auto load_kv = [&](int J, const StreamUnit& su, int j, bool k_part) {
@@ -901,17 +936,8 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         if (su.nblk == 0) continue;
         const int q = live & 1;
         if (live >= 2 && !(ok = warp_wait(bar(L::QFREE + q), ((live >> 1) - 1) & 1, &s_abort))) break;
-        const int rows_total = a.G * su.nn;
-        unsigned char* qt = smem + L::OFF_Q + q * L::QTILE;
-        for (int e = t0; e < L::QROWS * 16; e += 64) {
-          const int r = e >> 4, ch = e & 15, half = ch >> 3, gran = ch & 7;
-          uint4 v = make_uint4(0, 0, 0, 0);
-          if (r < rows_total) {
-            const int hh = r / su.nn, i = r - hh * su.nn;
-            v = reinterpret_cast<const uint4*>(a.q + (((size_t)su.b * a.n_pad + i) * a.H + su.g * a.G + hh) * HD)[ch];
-          }
-          *reinterpret_cast<uint4*>(qt + half * L::QHALF + r * 128 + ((gran ^ (r & 7)) << 4)) = v;
-        }
+        if (!(t == 0 && q_pre)) stage_q(su, q);
+        cp_async_wait_all();
         fence_proxy_async_smem();
         mbar_arrive(bar(L::QFULL + q));
         ++live;
