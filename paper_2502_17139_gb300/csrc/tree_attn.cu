@@ -197,6 +197,13 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
   return __all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar, parity, abort, WAIT_CYCLES));
 }
 
+// 16-byte asynchronous global -> shared copies (cp.async, no mbarrier): a
+// thread issues all of its copies before it waits once for them.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
+
 // ROPE: the queries arrive unrotated and are rotated by a.pos while staged
 // (a separate instance, so the plain kernel's code is unchanged).
 template <bool ROPE>
@@ -309,18 +316,21 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     fc_rope_table(s_rope, HD / 2, a.rope_nl2f);
     __syncthreads();
     stage_q_rope(smem + OFF_Q, a.q, a.pos, s_rope, b, g, a.G, a.H, a.n_pad, nn, row0, rows_total, tid);
-  } else
-  for (int e = tid; e < TILES * BM * 16; e += TA_THREADS) {
-    const int r = e >> 4, ch = e & 15, half = ch >> 3, gran = ch & 7;
-    const int tile = r / BM, rt = r - tile * BM;
-    const int rg = row0 + r;
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (rg < rows_total) {
-      const int hh = rg / nn, i = rg - hh * nn;
-      v = reinterpret_cast<const uint4*>(a.q + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD)[ch];
+  } else {
+    // asynchronous 16-byte copies: all of a thread's rows in flight at once
+    for (int e = tid; e < TILES * BM * 16; e += TA_THREADS) {
+      const int r = e >> 4, ch = e & 15, half = ch >> 3, gran = ch & 7;
+      const int tile = r / BM, rt = r - tile * BM;
+      const int rg = row0 + r;
+      const uint32_t off = OFF_Q + tile * TILE_BYTES + half * HALF_BYTES + rt * 128 + ((gran ^ (rt & 7)) << 4);
+      if (rg < rows_total) {
+        const int hh = rg / nn, i = rg - hh * nn;
+        cp_async16(sbase + off, a.q + (((size_t)b * a.n_pad + i) * a.H + g * a.G + hh) * HD + ch * 8);
+      } else {
+        *reinterpret_cast<uint4*>(smem + off) = make_uint4(0, 0, 0, 0);
+      }
     }
-    *reinterpret_cast<uint4*>(smem + OFF_Q + tile * TILE_BYTES + half * HALF_BYTES + rt * 128 +
-                              ((gran ^ (rt & 7)) << 4)) = v;
+    cp_async_wait_all();
   }
   fence_proxy_async_smem();
   tc_fence_before();
@@ -697,13 +707,6 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
     tmem_dealloc(tmem, TMEM_COLS);
   }
 }
-
-// 16-byte asynchronous global -> shared copies (cp.async, no mbarrier): a
-// thread issues all of its copies before it waits once for them.
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
 
 // ---------------------------------------------------------------------------
 // Streaming variant for short one-tile units: every group's rows fit one
