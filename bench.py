@@ -489,8 +489,8 @@ def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W,
     copied into the graph's input buffers before each replay.  The timed
     steps are the K steps after the warm-up, or K - 1 when the odd warm-up
     took one of them (K - 1 is then rounded down to a multiple of 2).  With
-    sub-batches a graph forks to their streams and joins them once, at its
-    end."""
+    sub-batches each sub-batch has graphs of its own, captured by the step
+    executor so that their kernels keep the eager streams' priorities."""
     import torch
     W2 = W + (W % 2)
     K2 = K - (W2 - W)
@@ -510,7 +510,7 @@ def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W,
     for i in range(P // G):
         s0 = W2 + i * G
         ins = [(q_pool[(s0 + t) % P], kt_pool[(s0 + t) % P], vt_pool[(s0 + t) % P]) + small[t] for t in range(G)]
-        graphs[s0 % P] = loop.capture_parts(ins) if parts else [loop.capture(ins)]
+        graphs[s0 % P] = loop.capture_native(ins) if parts else [loop.capture(ins)]
     main = torch.cuda.current_stream()
     streams = [torch.cuda.Stream() for _ in slices] if parts else [main]
 
@@ -523,7 +523,8 @@ def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W,
                     small[t][0][sl].copy_(hits_d[s + t][sl])
                     small[t][1][sl].copy_(plen_d[s + t][sl])
                     small[t][2][sl].copy_(rtok_d[s + t][sl])
-                graphs[s % P][h].replay()
+                g = graphs[s % P][h]
+                g.launch() if parts else g.replay()
 
     torch.cuda.synchronize()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -540,7 +541,8 @@ def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W,
     return {"ms_per_step": ms, "steps_per_s": 1e3 / ms, "steps": K2, "eager_warmup_steps": W2,
             "graphs": sum(len(g) for g in graphs.values()), "steps_per_graph": G,
             "note": f"the timed steps from graphs of {G} steps"
-                    + (", one graph per sub-batch replayed on its own stream (the sub-batches never join)"
+                    + (", one graph per sub-batch captured by the step executor (kernel nodes at their "
+                       "streams' priorities) and launched into a stream of its own (the sub-batches never join)"
                        if parts else "") + " (first replays include the graphs' upload); the step's small draws "
                     "copied in before each replay"}
 

@@ -847,6 +847,40 @@ fc_stream fc_pipeline_stream(const fc_pipeline* pl, int part);
 /* `caller` waits for everything enqueued on the sub-batches' streams. */
 fc_status fc_pipeline_join(fc_pipeline* pl, fc_stream caller);
 
+/*
+ * A CUDA graph of n_steps consecutive steps of sub-batch `part`, captured
+ * from its streams: step t reads phase (phase0 + t) & 1 and the inputs
+ * d_q[t], d_k_tree[t], d_v_tree[t], d_want_hit[t] (d_want_hit itself may be
+ * NULL), d_plen[t], d_rtok[t] (host arrays of n_steps device pointers, each
+ * as fc_pipeline_step's; d_q may be NULL with FC_PIPELINE_NO_ATTENTION).
+ * Every kernel node keeps the priority of the stream it runs on in the eager
+ * step (the chain above the attention), and the graph is instantiated to run
+ * by those node priorities, whatever stream it is launched into.  Capturing
+ * enqueues nothing: the sub-batch's state advances by n_steps at each launch,
+ * so launch graphs whose phases continue the sub-batch's.  The graph holds
+ * the pointers it was captured with; it must not outlive them or the
+ * executor.  FC_ERR_INVALID_ARG for a bad argument, FC_ERR_CUDA if the
+ * capture or instantiation fails (nothing is left allocated).
+ */
+typedef struct fc_pipeline_graph fc_pipeline_graph;
+fc_status fc_pipeline_capture_part(fc_pipeline* pl, int part, int n_steps, int phase0, int flags,
+                                   const void* const* d_q, const void* const* d_k_tree,
+                                   const void* const* d_v_tree, const int32_t* const* d_want_hit,
+                                   const int32_t* const* d_plen, const uint32_t* const* d_rtok,
+                                   fc_pipeline_graph** out);
+
+/* Launches the graph into `s`: it runs after the work already enqueued on s,
+ * and s's later work runs after it. */
+fc_status fc_pipeline_graph_launch(fc_pipeline_graph* g, fc_stream s);
+
+/* Counts the graph's kernel nodes by priority: *n_chain at the chain
+ * stream's, *n_attn at the attention stream's (FC_ERR_INTERNAL if a node
+ * has another). */
+fc_status fc_pipeline_graph_kernels(const fc_pipeline_graph* g, int* n_chain, int* n_attn);
+
+/* Frees the graph (NULL is ignored); launches already made still run. */
+void fc_pipeline_graph_destroy(fc_pipeline_graph* g);
+
 /* Waits for the executor's streams, then frees its streams and events. */
 void fc_pipeline_destroy(fc_pipeline* pl);
 

@@ -33,6 +33,16 @@ struct fc_pipeline {
   std::vector<cudaStream_t> chain, attn;
   std::vector<cudaEvent_t> ev_pre, ev_post, ev_done, ev_fork;
   cudaEvent_t ev_start = nullptr;
+  int p_chain = 0, p_attn = 0;                    // the two streams' priorities
+  std::vector<cudaGraphNode_t>* capture_attn = nullptr;  // while capturing: the attention nodes
+};
+
+// A sub-batch's steps captured into a CUDA graph whose kernel nodes keep the
+// priorities of the streams they were captured on.
+struct fc_pipeline_graph {
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+  int p_chain = 0, p_attn = 0;
 };
 
 namespace {
@@ -112,6 +122,8 @@ extern "C" fc_status fc_pipeline_create(const fc_pipeline_desc* d, fc_pipeline**
   int lo = 0, hi = 0;  // least and greatest priority (greatest is the most negative)
   bool ok = cudaDeviceGetStreamPriorityRange(&lo, &hi) == cudaSuccess;
   const int p_chain = std::max(hi, -1), p_attn = lo;
+  pl->p_chain = p_chain;
+  pl->p_attn = p_attn;
   const int n = d->n_parts;
   pl->chain.assign(n, nullptr);
   pl->attn.assign(n, nullptr);
@@ -209,6 +221,15 @@ fc_status enqueue_part(fc_pipeline* pl, int h, int c, bool attention, const void
       FC_TRY(fc_tree_attn(q, P.k_cache, P.v_cache, d.kv_cap, P.kv_len[c], kt, vt, P.mask, P.n_nodes, B, Np, d.H,
                           d.Hkv, d.D, d.scale, P.attn_out, P.attn_ws, P.attn_ws_bytes, sa));
     stage_event(stage_events, h, 2, 1, sa);
+    if (pl->capture_attn) {  // capturing: the attention launch is the node the attention stream ends on
+      cudaStreamCaptureStatus cs;
+      const cudaGraphNode_t* deps = nullptr;
+      size_t nd = 0;
+      if (cudaStreamGetCaptureInfo(sa, &cs, nullptr, nullptr, &deps, nullptr, &nd) != cudaSuccess ||
+          cs != cudaStreamCaptureStatusActive)
+        return FC_ERR_CUDA;
+      pl->capture_attn->insert(pl->capture_attn->end(), deps, deps + nd);
+    }
     if (cudaEventRecord(pl->ev_post[h], sa) != cudaSuccess ||
         cudaStreamWaitEvent(s, pl->ev_post[h], 0) != cudaSuccess)
       return FC_ERR_CUDA;
@@ -299,3 +320,108 @@ extern "C" fc_status fc_pipeline_join(fc_pipeline* pl, fc_stream caller) {
       return FC_ERR_CUDA;
   return FC_OK;
 }
+
+namespace {
+
+void graph_free(fc_pipeline_graph* g) {
+  if (!g) return;
+  if (g->exec) cudaGraphExecDestroy(g->exec);
+  if (g->graph) cudaGraphDestroy(g->graph);
+  delete g;
+}
+
+// The graph's kernel nodes, with their type checked.
+fc_status kernel_nodes(cudaGraph_t graph, std::vector<cudaGraphNode_t>* out) {
+  size_t n = 0;
+  if (cudaGraphGetNodes(graph, nullptr, &n) != cudaSuccess) return FC_ERR_CUDA;
+  std::vector<cudaGraphNode_t> nodes(n);
+  if (n && cudaGraphGetNodes(graph, nodes.data(), &n) != cudaSuccess) return FC_ERR_CUDA;
+  out->clear();
+  for (cudaGraphNode_t v : nodes) {
+    cudaGraphNodeType t;
+    if (cudaGraphNodeGetType(v, &t) != cudaSuccess) return FC_ERR_CUDA;
+    if (t == cudaGraphNodeTypeKernel) out->push_back(v);
+  }
+  return FC_OK;
+}
+
+}  // namespace
+
+extern "C" fc_status fc_pipeline_capture_part(fc_pipeline* pl, int part, int n_steps, int phase0, int flags,
+                                              const void* const* d_q, const void* const* d_k_tree,
+                                              const void* const* d_v_tree, const int32_t* const* d_want_hit,
+                                              const int32_t* const* d_plen, const uint32_t* const* d_rtok,
+                                              fc_pipeline_graph** out) {
+  FC_NVTX_RANGE();
+  if (!out) return FC_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!pl || part < 0 || part >= pl->d.n_parts || n_steps < 1 || (phase0 != 0 && phase0 != 1) || !d_k_tree ||
+      !d_v_tree || !d_plen || !d_rtok || (!(flags & FC_PIPELINE_NO_ATTENTION) && !d_q))
+    return FC_ERR_INVALID_ARG;
+  for (int t = 0; t < n_steps; ++t)
+    if (!step_args_ok(pl, (phase0 + t) & 1, flags, d_q ? d_q[t] : nullptr, d_k_tree[t], d_v_tree[t], d_plen[t],
+                      d_rtok[t]))
+      return FC_ERR_INVALID_ARG;
+  const bool attention = !(flags & FC_PIPELINE_NO_ATTENTION);
+  fc_pipeline_graph* g = new (std::nothrow) fc_pipeline_graph();
+  if (!g) return FC_ERR_CAPACITY;
+  g->p_chain = pl->p_chain;
+  g->p_attn = pl->p_attn;
+  std::vector<cudaGraphNode_t> attn_nodes;
+  cudaStream_t s = pl->chain[part];
+  if (cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+    graph_free(g);
+    return FC_ERR_CUDA;
+  }
+  pl->capture_attn = &attn_nodes;
+  fc_status st = FC_OK;
+  for (int t = 0; t < n_steps && st == FC_OK; ++t)
+    st = enqueue_part(pl, part, (phase0 + t) & 1, attention, d_q ? d_q[t] : nullptr, d_k_tree[t], d_v_tree[t],
+                      d_want_hit ? d_want_hit[t] : nullptr, d_plen[t], d_rtok[t], nullptr);
+  pl->capture_attn = nullptr;
+  const cudaError_t ce = cudaStreamEndCapture(s, &g->graph);  // ends the capture on every path
+  if (st == FC_OK && ce != cudaSuccess) st = FC_ERR_CUDA;
+  // every kernel at its stream's priority: the chain's above the attention's
+  std::vector<cudaGraphNode_t> kn;
+  if (st == FC_OK) st = kernel_nodes(g->graph, &kn);
+  for (size_t i = 0; st == FC_OK && i < kn.size(); ++i) {
+    cudaLaunchAttributeValue v{};
+    v.priority = std::find(attn_nodes.begin(), attn_nodes.end(), kn[i]) != attn_nodes.end() ? g->p_attn : g->p_chain;
+    if (cudaGraphKernelNodeSetAttribute(kn[i], cudaLaunchAttributePriority, &v) != cudaSuccess) st = FC_ERR_CUDA;
+  }
+  if (st == FC_OK &&
+      cudaGraphInstantiateWithFlags(&g->exec, g->graph, cudaGraphInstantiateFlagUseNodePriority) != cudaSuccess)
+    st = FC_ERR_CUDA;
+  if (st != FC_OK) {
+    graph_free(g);
+    return st;
+  }
+  *out = g;
+  return FC_OK;
+}
+
+extern "C" fc_status fc_pipeline_graph_launch(fc_pipeline_graph* g, fc_stream s) {
+  if (!g || !g->exec) return FC_ERR_INVALID_ARG;
+  return cudaGraphLaunch(g->exec, static_cast<cudaStream_t>(s)) == cudaSuccess ? FC_OK : FC_ERR_CUDA;
+}
+
+extern "C" fc_status fc_pipeline_graph_kernels(const fc_pipeline_graph* g, int* n_chain, int* n_attn) {
+  if (!g || !g->graph || !n_chain || !n_attn) return FC_ERR_INVALID_ARG;
+  std::vector<cudaGraphNode_t> kn;
+  const fc_status st = kernel_nodes(g->graph, &kn);
+  if (st != FC_OK) return st;
+  *n_chain = *n_attn = 0;
+  for (cudaGraphNode_t v : kn) {
+    cudaLaunchAttributeValue a{};
+    if (cudaGraphKernelNodeGetAttribute(v, cudaLaunchAttributePriority, &a) != cudaSuccess) return FC_ERR_CUDA;
+    if (a.priority == g->p_attn && g->p_attn != g->p_chain)
+      ++*n_attn;
+    else if (a.priority == g->p_chain)
+      ++*n_chain;
+    else
+      return FC_ERR_INTERNAL;
+  }
+  return FC_OK;
+}
+
+extern "C" void fc_pipeline_graph_destroy(fc_pipeline_graph* g) { graph_free(g); }

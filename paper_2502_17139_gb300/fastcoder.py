@@ -80,6 +80,7 @@ EXPORTS = ["fc_status_string", "fc_version", "fc_get_error", "fc_datastore_build
            "fc_missing_insert", "fc_build_tree", "fc_build_tree_all_workspace", "fc_build_tree_all", "fc_tree_mask", "fc_tree_attn", "fc_tree_attn_workspace", "fc_tree_attn_parts", "fc_tree_attn_streamed", "fc_rope", "fc_tree_attn_rope", "fc_gemm_workspace", "fc_gemm_bf16", "fc_gemm_kv_heads", "fc_gemm_silu_mul", "fc_interleave_gate_up", "fc_embed",
            "fc_add_rmsnorm", "fc_silu_mul", "fc_rope_heads", "fc_selftest_wait", "fc_accept", "fc_argmax_accept", "fc_kv_append", "fc_synth_argmax",
            "fc_pipeline_create", "fc_pipeline_step", "fc_pipeline_step_part", "fc_pipeline_join_part", "fc_pipeline_stream", "fc_pipeline_error", "fc_pipeline_join",
+           "fc_pipeline_capture_part", "fc_pipeline_graph_launch", "fc_pipeline_graph_kernels", "fc_pipeline_graph_destroy",
            "fc_pipeline_destroy"]
 
 
@@ -160,6 +161,10 @@ def _load():
         "fc_pipeline_stream": (vp, [vp, i32]),
         "fc_pipeline_error": (C.c_int, [vp, i32]),
         "fc_pipeline_destroy": (None, [vp]),
+        "fc_pipeline_capture_part": (C.c_int, [vp, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp]),
+        "fc_pipeline_graph_launch": (C.c_int, [vp, vp]),
+        "fc_pipeline_graph_kernels": (C.c_int, [vp, C.POINTER(C.c_int), C.POINTER(C.c_int)]),
+        "fc_pipeline_graph_destroy": (None, [vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -826,11 +831,14 @@ def fc_synth_argmax(tok, parent, n_nodes, plen, rtok, vocab, out=None):
 # ------------------------------------------------------ native step executor
 PIPELINE_NO_ATTENTION = 1
 _PIPELINES = weakref.WeakSet()
+_GRAPHS = weakref.WeakSet()
 
 
 @atexit.register
 def _close_pipelines():
-    # before the CUDA runtime shuts down: destroying streams later is unsafe
+    # before the CUDA runtime shuts down: destroying graphs and streams later is unsafe
+    for g in list(_GRAPHS):
+        g.close()
     for pl in list(_PIPELINES):
         pl.close()
 
@@ -863,6 +871,37 @@ def pipeline_part(batch, first, ctx, ctx_len, kv_len, root, rcache, skip, res, t
         _ptr(argmax), _ptr(acc["acc_len"]), _ptr(acc["path"]), _ptr(acc["bonus"]), _ptr(err),
         seq_cache.view if seq_cache is not None else fc_cache(), _ptr(missing.table) if missing else None,
         missing.capacity if missing else 0)
+
+
+class PipelineGraph:
+    """fc_pipeline_graph: captured steps of one sub-batch (Pipeline.capture).
+    It keeps its executor and input tensors alive."""
+
+    def __init__(self, handle, pipe, inputs):
+        self.handle, self._pipe, self._inputs = handle, pipe, inputs
+        self._destroy = LIB.fc_pipeline_graph_destroy
+        _GRAPHS.add(self)
+
+    def launch(self):
+        """Launch into the current stream."""
+        _check("fc_pipeline_graph_launch", LIB.fc_pipeline_graph_launch(self.handle, _stream()))
+
+    def kernels(self):
+        """(kernel nodes at the chain stream's priority, at the attention stream's)."""
+        a, b = C.c_int(), C.c_int()
+        _check("fc_pipeline_graph_kernels", LIB.fc_pipeline_graph_kernels(self.handle, C.byref(a), C.byref(b)))
+        return a.value, b.value
+
+    def close(self):
+        if getattr(self, "handle", None):
+            self._destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 class Pipeline:
@@ -932,6 +971,33 @@ class Pipeline:
             _check("fc_pipeline_join", LIB.fc_pipeline_join(self.handle, _stream()))
         else:
             _check("fc_pipeline_join_part", LIB.fc_pipeline_join_part(self.handle, part, _stream()))
+
+    def capture(self, part, inputs, phase0=0, attention=True):
+        """A CUDA graph of len(inputs) steps of sub-batch ``part`` (inputs:
+        tuples (q, k_tree, v_tree, want_hit, plen, rtok) of batch-wide device
+        tensors, read at every launch; q may be None without attention),
+        whose kernels keep their streams' priorities (fc_pipeline_capture_part).
+        Returns a PipelineGraph; launching it advances the sub-batch."""
+        qs, ks, bs, rs = self.shapes
+        n = len(inputs)
+        arrs = [(C.c_void_p * n)() for _ in range(6)]
+        for t, (q, kt, vt, wh, pl, rt) in enumerate(inputs):
+            if attention:
+                _need(q, torch.bfloat16, "q", qs)
+            _need(kt, torch.bfloat16, "k_tree", ks)
+            _need(vt, torch.bfloat16, "v_tree", ks)
+            _need(pl, torch.int32, "plen", bs)
+            _need(rt, torch.int32, "rtok", rs)
+            if wh is not None:
+                _need(wh, torch.int32, "want_hit", bs)
+            for a, x in zip(arrs, (q if attention else None, kt, vt, wh, pl, rt)):
+                a[t] = _ptr(x)
+        g = C.c_void_p()
+        want = None if all(w is None for _, _, _, w, _, _ in inputs) else arrs[3]
+        _check("fc_pipeline_capture_part", LIB.fc_pipeline_capture_part(
+            self.handle, part, n, phase0, 0 if attention else PIPELINE_NO_ATTENTION, arrs[0] if attention else None,
+            arrs[1], arrs[2], want, arrs[4], arrs[5], C.byref(g)))
+        return PipelineGraph(g, self, inputs)
 
     def error(self, part):
         """Sub-batch ``part``'s device errors since the last call (a status

@@ -363,6 +363,19 @@ class PipelinedStepLoop:
             graphs.append(g)
         return graphs
 
+    def capture_native(self, inputs, attention=True):
+        """As capture_parts, through the executor's own capture
+        (fc_pipeline_capture_part): one graph per sub-batch whose kernels keep
+        the priorities of the eager step's streams (the chain's above the
+        attention's), which a graph captured through torch loses.  Returns one
+        fc.PipelineGraph per sub-batch; launch each into a stream of its own
+        (graph.launch() on the current stream)."""
+        if any(lp.cur != 0 for lp in self.loops):
+            raise RuntimeError("capture at an even step")
+        if len(inputs) < 2 or len(inputs) % 2:
+            raise ValueError("capture an even number of steps (the lengths alternate between two buffers)")
+        return [self.pipe.capture(h, inputs, 0, attention) for h in range(len(self.loops))]
+
     def reset(self):
         self.join()
         for lp in self.loops:

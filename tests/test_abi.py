@@ -244,4 +244,13 @@ def test_pipeline_host_validation(lib):
     assert L.fc_pipeline_join_part(nul, 0, nul) == 1
     assert L.fc_pipeline_error(nul, 0) == 1
     assert L.fc_pipeline_stream(nul, 0) is None
+    g = C.c_void_p(7)
+    arr = (C.c_void_p * 2)(16, 16)
+    assert L.fc_pipeline_capture_part(nul, 0, 2, 0, 0, arr, arr, arr, None, arr, arr, C.byref(g)) == 1
+    assert not g.value  # cleared on failure
+    assert L.fc_pipeline_capture_part(nul, 0, 2, 0, 0, arr, arr, arr, None, arr, arr, None) == 1
+    assert L.fc_pipeline_graph_launch(nul, nul) == 1
+    a, b = C.c_int(), C.c_int()
+    assert L.fc_pipeline_graph_kernels(nul, C.byref(a), C.byref(b)) == 1
+    L.fc_pipeline_graph_destroy(nul)
     L.fc_pipeline_destroy(nul)

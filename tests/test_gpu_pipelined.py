@@ -352,3 +352,54 @@ def test_pipelined_algorithm1_matches_slice_loops(fc, setup):
         sa, sb = seq_state(lp), seq_state(piped.loops[h])
         for k in sa:
             assert torch.equal(sa[k], sb[k]), (h, k)
+
+
+@pytest.mark.parametrize("algorithm1", [False, True], ids=["replay_cache", "algorithm1"])
+def test_pipelined_native_graphs(fc, setup, algorithm1):
+    """The executor's own capture (fc_pipeline_capture_part): one graph of two
+    steps per sub-batch, launched into a stream of its own, follows the eager
+    pipelined trajectory (with the replay cache, and with Algorithm 1's CACHE
+    and missing table), and its kernel nodes carry the eager streams'
+    priorities: per step one attention node and the chain's six (eight with
+    the CACHE) above it."""
+    from paper_2502_17139_gb300.step import PipelinedStepLoop
+    ins, steps = setup["ins"], setup["steps"]
+    kw = dict(setup["kw"], seq_cache=SEQ) if algorithm1 else setup["kw"]
+    eager = PipelinedStepLoop(3, *setup["args"], **kw)
+    want = []
+    for s in range(steps):
+        eager.step(*ins[s])
+        if s % 2 == 1:
+            eager.join()
+            want.append(state(eager))
+    graphed = PipelinedStepLoop(3, *setup["args"], **kw)
+    graphed.step(*ins[0])
+    graphed.step(*ins[1])
+    graphed.join()
+    static = [tuple(t.clone() for t in ins[2]), tuple(t.clone() for t in ins[3])]
+    graphs = graphed.capture_native(static)
+    assert len(graphs) == 3
+    for g in graphs:
+        assert g.kernels() == ((8 if algorithm1 else 6) * 2, 2)
+    streams = [torch.cuda.Stream() for _ in graphs]
+    got = []
+    main = torch.cuda.current_stream()
+    for s in range(2, steps, 2):
+        for j in range(2):
+            for dst, src in zip(static[j], ins[s + j]):
+                dst.copy_(src)
+        ready = torch.cuda.Event()
+        ready.record(main)
+        for g, st in zip(graphs, streams):
+            st.wait_event(ready)
+            with torch.cuda.stream(st):
+                g.launch()
+        for st in streams:
+            main.wait_stream(st)
+        got.append(state(graphed))
+    torch.cuda.synchronize()
+    assert fc.fc_get_error() == "FC_OK" and graphed.errors() == ["FC_OK"] * 3
+    for w, gt in zip(want[1:], got):
+        same(w, gt)
+    for g in graphs:
+        g.close()
