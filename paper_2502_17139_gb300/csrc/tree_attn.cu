@@ -88,8 +88,8 @@ struct AttnArgs {
   int u_split;     // units [0, u_split) run whole, one CTA each; the rest ...
   int parts;       // ... have their KV blocks split over this many CTAs (1..MAX_PARTS)
   int* ws_cnt;     // [split units][2]: arrival tickets, finished partials (zeroed before the launch)
-  float2* ws_ml;   // [split units][parts - 1][256 rows]: (m, l) of a partial
-  float* ws_o;     // [split units][parts - 1][256 rows][128]: unnormalised O of a partial
+  float2* ws_ml;   // [split units][parts][256 rows]: (m, l) of a partial, by part
+  float* ws_o;     // [split units][parts][256 rows][128]: unnormalised O of a partial, by part
   unsigned int* err;  // the launch's error word (NULL: this file's own)
   float scale_log2;
   const int32_t* pos;  // [B][n_pad] node positions: rotate Q by them (RoPE), or nullptr
@@ -603,18 +603,20 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
       // attention over a key set is a ratio of two sums over its keys, so the
       // parts' (m, l, O) over disjoint key ranges merge exactly:
       //   m* = max m_t,  l* = sum l_t 2^(m_t - m*),  O = sum O_t 2^(m_t - m*) / l*.
-      // Each CTA takes a ticket when done; all but the last store their rows,
-      // the last waits (bounded) until they have, then merges and writes out.
-      // The CTAs it waits for are resident: they took their tickets before it.
+      // Each CTA takes a ticket when done; all but the last store their rows
+      // in their part's slot, the last waits (bounded) until they have, then
+      // merges and writes out.  The CTAs it waits for are resident: they took
+      // their tickets before it.  The merge sums the parts in part order,
+      // whichever CTA merges, so the result does not depend on timing.
       named_sync(1, 256);
       if (tid == 128) s_ticket = atomicAdd(a.ws_cnt + 2 * su, 1);
       named_sync(1, 256);
       const int t = s_ticket;
-      const size_t slot0 = (size_t)su * (a.parts - 1) * (TILES * BM);  // the unit's first slot row
+      const size_t slot0 = (size_t)su * a.parts * (TILES * BM);  // the unit's first slot row
       const int lr = x * BM + r;                                          // row within the unit
       if (t < n_contrib - 1) {
         if (fin) {
-          float* od = a.ws_o + (slot0 + (size_t)t * (TILES * BM) + lr) * HD;
+          float* od = a.ws_o + (slot0 + (size_t)part * (TILES * BM) + lr) * HD;
 #pragma unroll
           for (int cc = 0; cc < HD / 32; ++cc) {
             uint32_t o[32];
@@ -628,7 +630,7 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
                                    __uint_as_float(o[u + 3])));
             }
           }
-          if (row_ok) __stcg(a.ws_ml + slot0 + (size_t)t * (TILES * BM) + lr, make_float2(m_run, l_run));
+          if (row_ok) __stcg(a.ws_ml + slot0 + (size_t)part * (TILES * BM) + lr, make_float2(m_run, l_run));
         }
         named_sync(1, 256);
         if (tid == 128) {
@@ -648,20 +650,29 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
         }
         named_sync(1, 256);
         if (fin && s_ready) {
-          float mt[MAX_PARTS - 1], wt[MAX_PARTS - 1];
-          float mstar = m_run;
-          for (int u = 0; u < n_contrib - 1; ++u) {
-            const float2 ml = row_ok ? __ldcg(a.ws_ml + slot0 + (size_t)u * (TILES * BM) + lr) : make_float2(m_run, 0.f);
-            mt[u] = ml.x;
-            wt[u] = ml.y;  // l for now
+          // the parts with keys, in part order; this CTA's own partial at its index
+          auto contributes = [&](int h) { return (h + 1) * nblk_all / nparts > h * nblk_all / nparts; };
+          float mt[MAX_PARTS], wt[MAX_PARTS];
+          float mstar = -INFINITY;
+#pragma unroll
+          for (int h = 0; h < MAX_PARTS; ++h) {
+            mt[h] = -INFINITY;
+            wt[h] = 0.f;
+            if (h >= nparts || !contributes(h)) continue;
+            const float2 ml = h == part ? make_float2(m_run, l_run)
+                                        : (row_ok ? __ldcg(a.ws_ml + slot0 + (size_t)h * (TILES * BM) + lr)
+                                                  : make_float2(m_run, 0.f));
+            mt[h] = ml.x;
+            wt[h] = ml.y;  // l for now
             mstar = fmaxf(mstar, ml.x);
           }
-          const float w_own = exp2f(m_run - mstar);
-          float lstar = l_run * w_own;
-          for (int u = 0; u < n_contrib - 1; ++u) {
-            const float w = exp2f(mt[u] - mstar);
-            lstar += wt[u] * w;
-            wt[u] = w;
+          float lstar = 0.f;
+#pragma unroll
+          for (int h = 0; h < MAX_PARTS; ++h) {
+            if (h >= nparts || !contributes(h)) continue;
+            const float w = exp2f(mt[h] - mstar);
+            lstar += wt[h] * w;
+            wt[h] = w;
           }
           const float inv = 1.f / lstar;
 #pragma unroll
@@ -672,16 +683,23 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
             if (row_ok) {
               float acc[32];
 #pragma unroll
-              for (int u = 0; u < 32; ++u) acc[u] = __uint_as_float(o[u]) * w_own;
-              for (int t2 = 0; t2 < n_contrib - 1; ++t2) {
-                const float* os = a.ws_o + (slot0 + (size_t)t2 * (TILES * BM) + lr) * HD + cc * 32;
+              for (int u = 0; u < 32; ++u) acc[u] = 0.f;
 #pragma unroll
-                for (int u = 0; u < 32; u += 4) {
-                  const float4 v = __ldcg(reinterpret_cast<const float4*>(os + u));
-                  acc[u] += v.x * wt[t2];
-                  acc[u + 1] += v.y * wt[t2];
-                  acc[u + 2] += v.z * wt[t2];
-                  acc[u + 3] += v.w * wt[t2];
+              for (int h = 0; h < MAX_PARTS; ++h) {
+                if (h >= nparts || !contributes(h)) continue;
+                if (h == part) {
+#pragma unroll
+                  for (int u = 0; u < 32; ++u) acc[u] += __uint_as_float(o[u]) * wt[h];
+                } else {
+                  const float* os = a.ws_o + (slot0 + (size_t)h * (TILES * BM) + lr) * HD + cc * 32;
+#pragma unroll
+                  for (int u = 0; u < 32; u += 4) {
+                    const float4 v = __ldcg(reinterpret_cast<const float4*>(os + u));
+                    acc[u] += v.x * wt[h];
+                    acc[u + 1] += v.y * wt[h];
+                    acc[u + 2] += v.z * wt[h];
+                    acc[u + 3] += v.w * wt[h];
+                  }
                 }
               }
 #pragma unroll
@@ -1230,7 +1248,7 @@ struct WsLayout {
 };
 WsLayout ws_layout(uint64_t units, int parts) {
   WsLayout w;
-  const uint64_t slots = units * (uint64_t)(parts - 1) * (TILES * BM);
+  const uint64_t slots = units * (uint64_t)parts * (TILES * BM);
   w.cnt = 0;
   w.ml = (units * 2 * sizeof(int) + 255) / 256 * 256;
   w.o = w.ml + (slots * sizeof(float2) + 255) / 256 * 256;

@@ -488,6 +488,43 @@ def test_attn_kv_split_two_tiles(fc, orc):
     _attn_case(fc, orc, 7, B, 128, 32, 8, kvl, 2048, nn=nn, full_rows=False, want_parts=2)
 
 
+def test_attn_kv_split_deterministic(fc):
+    """With the last wave's keys split over several CTAs, whichever CTA of a
+    unit finishes last merges the parts; it sums them in part order, so
+    repeated launches on the same inputs give the same bits.  The step loop's
+    shape (32 sequences, GQA 32/8, 128-node padding, 16384-key caches, trees
+    of 1 to 128 nodes), 12 launches."""
+    B, n_pad, H, Hkv, cap = 32, 128, 32, 8, 16384
+    rng = synth.rng_for(53)
+    nn = rng.integers(1, n_pad + 1, B).astype(np.int32)
+    kvl = rng.integers(cap - 200, cap + 1, B).astype(np.int32)
+    par = np.full((B, n_pad), -1, np.int32)
+    for b in range(B):
+        _, p = synth.random_tree(rng, int(nn[b]), 10, 4, 1000)
+        par[b, :nn[b]] = p
+    D = 128
+    q = synth.randn_bf16((B, n_pad, H, D), 61, "cuda")
+    kc = synth.randn_bf16((B, Hkv, cap, D), 62, "cuda")
+    vc = synth.randn_bf16((B, Hkv, cap, D), 63, "cuda")
+    kt = synth.randn_bf16((B, Hkv, n_pad, D), 64, "cuda")
+    vt = synth.randn_bf16((B, Hkv, n_pad, D), 65, "cuda")
+    gm = fc.fc_tree_mask(dev(par), dev(nn), dev(kvl))
+    ws = fc.attn_workspace(B, n_pad, H, Hkv, "cuda")
+    assert fc.LIB.fc_tree_attn_parts(B, n_pad, H, Hkv, cap, ws.numel()) > 1
+    out = torch.empty_like(q)
+    first = None
+    for _ in range(12):
+        out.fill_(float("nan"))
+        fc.fc_tree_attn(q, kc, vc, dev(kvl), kt, vt, gm["mask"], dev(nn), out=out, workspace=ws)
+        torch.cuda.synchronize()
+        if first is None:
+            first = out.clone()
+            assert not torch.isnan(first).any()
+        else:
+            assert torch.equal(out, first)
+    check_no_error(fc)
+
+
 def test_attn_stream_c1_shape(fc, orc):
     """The c1 launch (1024 one-tile groups, 512-key caches) runs on the
     streaming kernel: several groups per CTA."""
