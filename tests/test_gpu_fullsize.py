@@ -385,3 +385,45 @@ def test_algorithm1_full_size_properties(fc):
         for T in inp["corpora"]:
             hit = (T[:-2] == k0) & (T[1:-1] == k1)
             assert not hit.any()
+
+
+def test_algorithm1_full_size_pipelined_equals_single(fc):
+    """Algorithm 1 through the step executor (4 sub-batches, a missing table
+    each) against the single loop over the whole batch (one missing table) on
+    the default step loop's store (100M + 5M tokens, 32 sequences, l = 50):
+    after every step the same trees and acceptance, and after 100 steps the
+    same contexts, lengths and CACHE stores.  A missing table only skips
+    searches that would find nothing, so splitting it changes no draft."""
+    import bench
+    from paper_2502_17139_gb300.step import PipelinedStepLoop, StepLoop
+    steps = 100
+    inp = bench.make_inputs(1.0, 32, 0, steps + 1)
+    cfg, B = inp["cfg"], inp["B"]
+    d = cfg["draft_len"]
+    sources = [fc.fc_datastore_build(dev(T), synth.VOCAB) for T in inp["corpora"]]
+    p = fc.params(cfg["n_max"], cfg["n_min"], cfg["top_k"], d, 4096)
+    seq = dict(capacity=8192, min_size=50, chunk=20, ctx_keep=16, missing_capacity=1 << 16, weight=1)
+    kv0 = 64
+    args = (sources, inp["ctx"], inp["cl"], p, 128, 128, [1, 1], 32, 8, 128, kv0 + (steps + 1) * (d + 1) + 8, kv0,
+            synth.VOCAB)
+    single = StepLoop(*args, seq_cache=seq)
+    piped = PipelinedStepLoop(4, *args, seq_cache=seq)
+    kt = torch.zeros((B, 8, 128, 128), dtype=torch.bfloat16, device="cuda")
+    zeros = torch.zeros(B, dtype=torch.int32, device="cuda")
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).cuda()
+    served = 0
+    for s in range(steps):
+        ins = (None, kt, kt, zeros, to_dev(inp["plen"][s]), to_dev(inp["rtok"][s]))
+        single.step(*ins, attention=False)
+        piped.step(*ins, attention=False)
+        piped.join()
+        for k in ("n_nodes", "tok", "parent"):
+            assert torch.equal(single.tree[k], piped.tree[k]), (s, k)
+        assert torch.equal(single.acc["acc_len"], piped.acc["acc_len"]), s
+        served += int((piped.skip == 1).sum())
+    assert served > 0  # the CACHE served queries
+    assert torch.equal(single.ctx, piped.ctx)
+    assert torch.equal(single.ctx_len_now, piped.ctx_len_now)
+    assert torch.equal(single.seq_cache.words, torch.cat([lp.seq_cache.words for lp in piped.loops]))
+    assert torch.equal(single.seq_cache.meta, torch.cat([lp.seq_cache.meta for lp in piped.loops]))
+    assert fc.fc_get_error() == "FC_OK" and piped.errors() == ["FC_OK"] * 4
