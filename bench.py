@@ -484,13 +484,16 @@ def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W,
     (one more when W is odd, since a graph starts at an even step: its
     lengths ping-pong between two buffers), then the timed steps replayed
     from CUDA graphs of G steps each (G = 8, 4 or 2, the largest that divides
-    the pool size and the number of timed steps), one graph per pool offset
-    (they read the pooled activations directly); a step's small draws are
-    copied into the graph's input buffers before each replay.  The timed
-    steps are the K steps after the warm-up, or K - 1 when the odd warm-up
-    took one of them (K - 1 is then rounded down to a multiple of 2).  With
-    sub-batches each sub-batch has graphs of its own, captured by the step
-    executor so that their kernels keep the eager streams' priorities."""
+    the pool size and the number of timed steps).  The timed steps are the K
+    steps after the warm-up, or K - 1 when the odd warm-up took one of them
+    (K - 1 is then rounded down to a multiple of 2).
+    A pipelined loop: every window of G timed steps has, per sub-batch, a
+    graph of its own captured by the step executor (kernels at the eager
+    streams' priorities, uploaded at capture), reading that window's inputs
+    where the eager loop reads them; each sub-batch launches its graphs into
+    a stream of its own, so the sub-batches never join.  One stream: one graph
+    per pool offset, reading the pooled activations directly, with a step's
+    small draws copied into the graph's input buffers before each replay."""
     import torch
     W2 = W + (W % 2)
     K2 = K - (W2 - W)
@@ -503,28 +506,34 @@ def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W,
     loop.reset()
     for s in range(W2):  # eager warm-up; it also makes workspaces and kernel attributes
         loop.step(q_pool[s % P], kt_pool[s % P], vt_pool[s % P], hits_d[s], plen_d[s], rtok_d[s])
-    small = [(torch.empty_like(hits_d[0]), torch.empty_like(plen_d[0]), torch.empty_like(rtok_d[0])) for _ in range(G)]
-    parts = hasattr(loop, "capture_parts")  # a pipelined loop: one graph per sub-batch, never joined
+    parts = hasattr(loop, "capture_native")  # a pipelined loop: graphs per sub-batch, never joined
     slices = loop.slices if parts else [slice(None)]
+    small = [(torch.empty_like(hits_d[0]), torch.empty_like(plen_d[0]), torch.empty_like(rtok_d[0])) for _ in range(G)]
     graphs = {}
-    for i in range(P // G):
-        s0 = W2 + i * G
-        ins = [(q_pool[(s0 + t) % P], kt_pool[(s0 + t) % P], vt_pool[(s0 + t) % P]) + small[t] for t in range(G)]
-        graphs[s0 % P] = loop.capture_native(ins) if parts else [loop.capture(ins)]
+    if parts:
+        for s0 in range(W2, W2 + K2, G):
+            ins = [(q_pool[(s0 + t) % P], kt_pool[(s0 + t) % P], vt_pool[(s0 + t) % P], hits_d[s0 + t], plen_d[s0 + t],
+                    rtok_d[s0 + t]) for t in range(G)]
+            graphs[s0] = loop.capture_native(ins)
+    else:
+        for i in range(P // G):
+            s0 = W2 + i * G
+            ins = [(q_pool[(s0 + t) % P], kt_pool[(s0 + t) % P], vt_pool[(s0 + t) % P]) + small[t] for t in range(G)]
+            graphs[s0 % P] = [loop.capture(ins)]
     main = torch.cuda.current_stream()
     streams = [torch.cuda.Stream() for _ in slices] if parts else [main]
 
     def block(s):
-        # each sub-batch copies its slice of the step's small draws on its own
-        # stream, then replays its graph there
-        for h, (sl, st) in enumerate(zip(slices, streams)):
-            with torch.cuda.stream(st):
-                for t in range(G):
-                    small[t][0][sl].copy_(hits_d[s + t][sl])
-                    small[t][1][sl].copy_(plen_d[s + t][sl])
-                    small[t][2][sl].copy_(rtok_d[s + t][sl])
-                g = graphs[s % P][h]
-                g.launch() if parts else g.replay()
+        if parts:  # each sub-batch launches its graph of this window on its own stream
+            for h, st in enumerate(streams):
+                with torch.cuda.stream(st):
+                    graphs[s][h].launch()
+            return
+        for t in range(G):  # one stream: the step's small draws into the graph's buffers, then the replay
+            small[t][0].copy_(hits_d[s + t])
+            small[t][1].copy_(plen_d[s + t])
+            small[t][2].copy_(rtok_d[s + t])
+        graphs[s % P][0].replay()
 
     torch.cuda.synchronize()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -541,10 +550,12 @@ def run_graph_pass(loop, q_pool, kt_pool, vt_pool, hits_d, plen_d, rtok_d, P, W,
     return {"ms_per_step": ms, "steps_per_s": 1e3 / ms, "steps": K2, "eager_warmup_steps": W2,
             "graphs": sum(len(g) for g in graphs.values()), "steps_per_graph": G,
             "note": f"the timed steps from graphs of {G} steps"
-                    + (", one graph per sub-batch captured by the step executor (kernel nodes at their "
-                       "streams' priorities) and launched into a stream of its own (the sub-batches never join)"
-                       if parts else "") + " (first replays include the graphs' upload); the step's small draws "
-                    "copied in before each replay"}
+                    + (", per window of steps and sub-batch, captured by the step executor (kernel nodes at their "
+                       "streams' priorities, uploaded at capture) and reading the window's inputs where the eager "
+                       "loop reads them; each sub-batch launches its graphs into a stream of its own (the "
+                       "sub-batches never join)" if parts else
+                       " (first replays include the graphs' upload); the step's small draws copied in before "
+                       "each replay")}
 
 
 def single_stream_attn(sources, inp, p, cfg, cap, kv0, dev, weights, kc, vc, q_pool, kt_pool, vt_pool, hits_d, plen_d,

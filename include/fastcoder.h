@@ -855,8 +855,10 @@ fc_status fc_pipeline_join(fc_pipeline* pl, fc_stream caller);
  * as fc_pipeline_step's; d_q may be NULL with FC_PIPELINE_NO_ATTENTION).
  * Every kernel node keeps the priority of the stream it runs on in the eager
  * step (the chain above the attention), and the graph is instantiated to run
- * by those node priorities, whatever stream it is launched into.  Capturing
- * enqueues nothing: the sub-batch's state advances by n_steps at each launch,
+ * by those node priorities, whatever stream it is launched into.  The graph
+ * is uploaded to the device on the sub-batch's chain stream, so that its
+ * first launch does not pay for it.  Capturing enqueues no kernel: the
+ * sub-batch's state advances by n_steps at each launch,
  * so launch graphs whose phases continue the sub-batch's.  The graph holds
  * the pointers it was captured with; it must not outlive them or the
  * executor.  FC_ERR_INVALID_ARG for a bad argument, FC_ERR_CUDA if the

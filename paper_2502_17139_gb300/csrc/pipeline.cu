@@ -392,6 +392,8 @@ extern "C" fc_status fc_pipeline_capture_part(fc_pipeline* pl, int part, int n_s
   if (st == FC_OK &&
       cudaGraphInstantiateWithFlags(&g->exec, g->graph, cudaGraphInstantiateFlagUseNodePriority) != cudaSuccess)
     st = FC_ERR_CUDA;
+  // the executable graph's device-side setup now, not at its first launch
+  if (st == FC_OK && cudaGraphUpload(g->exec, s) != cudaSuccess) st = FC_ERR_CUDA;
   if (st != FC_OK) {
     graph_free(g);
     return st;
