@@ -291,3 +291,48 @@ def test_trajectory_invariants(orc, a1):
         for i in range(pieces):
             s0 = 40 + i * cp.chunk
             assert tuple(ctx2[b, s0:s0 + cp.chunk].tolist()) in stored
+
+
+def test_missing_table_split_changes_no_draft(orc, a1):
+    """A missing table per slice of the sequences (the step executor keeps one
+    per sub-batch) instead of one for the batch changes no draft: M only
+    skips datastore searches that would find nothing.  The oracle's Algorithm
+    1 over the whole batch and over each slice on its own give the same
+    trees, acceptance, contexts and CACHE stores; the search states differ
+    only where the whole batch's M skipped a query that its slice searched,
+    and that search found nothing."""
+    import paper_2502_17139_gb300.synth as syn
+    rng = np.random.default_rng(4321)
+    vocab = 64
+    corpora = [syn.zipf_tokens(rng, 400, 1.1, vocab=vocab).astype(np.uint32),
+               syn.zipf_tokens(rng, 200, 1.1, vocab=vocab).astype(np.uint32)]
+    B, H, steps, stride = 16, 8, 40, 256
+    ctx = np.zeros((B, stride), np.uint32)
+    ctx[:, :40] = rng.integers(0, vocab, (B, 40))
+    cl = np.full(B, 40, np.int32)
+    p = dict(n_max=8, n_min=2, top_k=4, draft_len=4, max_occ=64, node_budget=16, n_pad=16)
+    plen = rng.integers(0, 3, (steps, B)).astype(np.int32)
+    rtok = rng.integers(0, vocab, (steps, B, 16)).astype(np.uint32)
+    cp = a1.CacheParams(min_size=50, chunk=5, ctx_keep=8, capacity=4096)  # M at work, the CACHE inactive
+
+    def run(sl):
+        return a1.step_loop(corpora, ctx[sl], cl[sl], steps, p, cp, plen[:, sl], rtok[:, sl], [1, 1], 1, vocab, 1024)
+
+    whole = run(slice(0, B))
+    parts = [run(slice(0, H)), run(slice(H, B))]
+    for k in ("acc_len", "bonus", "n_nodes"):
+        got = np.concatenate([np.stack(pt[0][k]) for pt in parts], axis=1)
+        assert np.array_equal(np.stack(whole[0][k]), got), k
+    assert np.array_equal(whole[1], np.concatenate([pt[1] for pt in parts]))
+    assert np.array_equal(whole[2], np.concatenate([pt[2] for pt in parts]))
+    st_w = whole[4]
+    for h, pt in enumerate(parts):
+        for i, e in enumerate(pt[4].entries):
+            assert [x.tolist() for x in e] == [x.tolist() for x in st_w.entries[H * h + i]]
+    code_w = np.stack(whole[0]["code"])
+    code_p = np.concatenate([np.stack(pt[0]["code"]) for pt in parts], axis=1)
+    nd_p = np.concatenate([np.stack(pt[0]["n_drafts"]) for pt in parts], axis=2)  # [steps, S + 1, B]
+    diff = code_w != code_p
+    assert diff.any(), "the whole batch's M never skipped a query its slice searched: scenario too weak"
+    assert (code_w[diff] == a1.SKIP_MISSING).all() and (code_p[diff] == a1.SERVE_DATASTORE).all()
+    assert (nd_p[:, :2][np.broadcast_to(diff[:, None, :], nd_p[:, :2].shape)] == 0).all()
