@@ -56,9 +56,9 @@ UNIT = "steps/s"
 # ratio x the algorithmic bytes per launch of its own launches.  The ratio is valid
 # only for the kernel sources it was taken on (their SHA-256 below); otherwise the
 # bench reports traffic as null until it is measured again.
-ATTN_TRAFFIC = {"ratio": 1.0572,
+ATTN_TRAFFIC = {"ratio": 1.0624,
                 "sources": ["paper_2502_17139_gb300/csrc/tree_attn.cu", "paper_2502_17139_gb300/csrc/fc_common.cuh"],
-                "sha256": "38fc7f5c7235628b6b88af3035e516570577a92633bc84280c44ecd4c4dcb990"}
+                "sha256": "43b044e94f2cc97452818a22d11aa8bcea7db9717ac19c720f55fd3e5c941192"}
 
 WORKLOAD = ("full step loop: two-source datastore 100M (Zipf 1.1) + 5M (Zipf 1.3, 20k planted repeats) tokens, "
             "vocab 32256, batch 32, ctx 128, n 16->2, top-64 x 10 tokens per source, tree <=128 nodes, "

@@ -197,6 +197,17 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
   return __all_sync(0xFFFFFFFFu, mbar_wait_bounded(bar, parity, abort, WAIT_CYCLES));
 }
 
+// An L2 prefetch of a tensor-map tile (no shared memory, no barrier).
+__device__ __forceinline__ void tma_prefetch_l2_3d(const CUtensorMap* map, int x, int y, int z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+// One-tile CTAs are bound by their K/V delivery: they prefetch the cache
+// blocks this far ahead of their loads into L2.
+constexpr int PF_ONE_TILE = 2;
+
 // 16-byte asynchronous global -> shared copies (cp.async, no mbarrier): a
 // thread issues all of its copies before it waits once for them.
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
@@ -353,6 +364,13 @@ __global__ void __launch_bounds__(TA_THREADS, 1)
           }
           load_kv(j, false);
           issued = j + 1;
+          const int jp = kb + j + PF_ONE_TILE;
+          if (!has_b && j + PF_ONE_TILE < nblk && jp < nblk_c) {  // a cache block of this CTA's share
+            tma_prefetch_l2_3d(&tm_kc, 0, jp * BN, bg);
+            tma_prefetch_l2_3d(&tm_kc, 64, jp * BN, bg);
+            tma_prefetch_l2_3d(&tm_vc, 0, jp * BN, bg);
+            tma_prefetch_l2_3d(&tm_vc, 64, jp * BN, bg);
+          }
         }
         if (s_abort) {  // let the copies already issued land before the CTA exits
           volatile int dummy = 0;
