@@ -403,3 +403,50 @@ def test_pipelined_native_graphs(fc, setup, algorithm1):
         same(w, gt)
     for g in graphs:
         g.close()
+
+
+def test_pipelined_native_graphs_rope_and_no_attention(fc, setup):
+    """The executor's own graphs with RoPE (the tree keys rotated by fc_rope on
+    the chain: seven chain nodes a step, the attention rotating the queries)
+    follow the eager pipelined trajectory; graphs captured without the
+    attention launch hold only the chain's six nodes a step and follow the
+    eager trajectory without attention."""
+    from paper_2502_17139_gb300.step import PipelinedStepLoop
+    ins, steps = setup["ins"], 6
+    for rope, attention in ((10000.0, True), (None, False)):
+        kw = dict(setup["kw"], rope_base=rope)
+        eager = PipelinedStepLoop(2, *setup["args"], **kw)
+        want = []
+        for s in range(steps):
+            eager.step(*ins[s], attention=attention)
+            if s % 2 == 1:
+                eager.join()
+                want.append(state(eager))
+        graphed = PipelinedStepLoop(2, *setup["args"], **kw)
+        graphed.step(*ins[0], attention=attention)
+        graphed.step(*ins[1], attention=attention)
+        graphed.join()
+        windows = {s: graphed.capture_native([ins[s], ins[s + 1]], attention=attention) for s in range(2, steps, 2)}
+        for gs in windows.values():
+            for g in gs:
+                assert g.kernels() == ((7 if rope else 6) * 2, 2 if attention else 0)
+        streams = [torch.cuda.Stream() for _ in graphed.loops]
+        main = torch.cuda.current_stream()
+        got = []
+        for s in range(2, steps, 2):
+            ready = torch.cuda.Event()
+            ready.record(main)
+            for g, st in zip(windows[s], streams):
+                st.wait_event(ready)
+                with torch.cuda.stream(st):
+                    g.launch()
+            for st in streams:
+                main.wait_stream(st)
+            got.append(state(graphed))
+        torch.cuda.synchronize()
+        assert fc.fc_get_error() == "FC_OK" and graphed.errors() == ["FC_OK"] * 2
+        for w, gt in zip(want[1:], got):
+            if not attention:
+                w.pop("attn")
+                gt.pop("attn")
+            same(w, gt)
