@@ -161,9 +161,9 @@ def test_step_loop_full_store_lockstep(fc, orc):
     """The benchmarked configuration at full size: the 100M + 5M two-source
     store, 32 sequences with 128-token contexts, n 16 -> 2, top-64 x 10 per
     source, 128-node trees, GQA 32/8, head dim 128, KV 16384, a seeded 50%
-    replay-cache hit pattern, and the bench's launch configuration (two
-    sub-batches of 16 sequences on streams of their own, each with its own
-    replay cache).  A recording pass fills the caches; the replayed pass is
+    replay-cache hit pattern, and the bench's launch configuration (four
+    sub-batches of 8 sequences issued by the step executor, each on streams of
+    its own with its own replay cache).  A recording pass fills the caches; the replayed pass is
     compared with the oracle's step loop step by step: which queries the
     cache served, tree sizes, accepted lengths, bonus tokens, and at the end
     every context, context length and KV length.  The last step's tree
@@ -183,7 +183,7 @@ def test_step_loop_full_store_lockstep(fc, orc):
     vc = synth.randn_bf16((B, Hkv, cap, D), 502, "cuda")
     acts = [(synth.randn_bf16((B, n_pad, H, D), 510 + i, "cuda"), synth.randn_bf16((B, Hkv, n_pad, D), 520 + i, "cuda"),
              synth.randn_bf16((B, Hkv, n_pad, D), 530 + i, "cuda")) for i in range(2)]
-    loop = PipelinedStepLoop(2, sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, [1, 1], H, Hkv, D, cap,
+    loop = PipelinedStepLoop(4, sources, inp["ctx"], inp["cl"], p, cfg["node_budget"], n_pad, [1, 1], H, Hkv, D, cap,
                              kv0, synth.VOCAB, cache_capacity=1 << 14, k_cache=kc, v_cache=vc)
     # the per-step inputs stay resident: the sub-batch streams read them after
     # step() returns, so they must not be temporaries
@@ -208,7 +208,7 @@ def test_step_loop_full_store_lockstep(fc, orc):
         got["bonus"].append(host_u32(loop.acc["bonus"]))
         got["n_nodes"].append(loop.tree["n_nodes"].cpu().numpy())
     torch.cuda.synchronize()
-    assert fc.fc_get_error() == "FC_OK" and loop.errors() == ["FC_OK", "FC_OK"]
+    assert fc.fc_get_error() == "FC_OK" and loop.errors() == ["FC_OK"] * 4
     # the oracle, one sub-batch at a time with a replay cache of its own
     po = dict(n_max=cfg["n_max"], n_min=cfg["n_min"], top_k=cfg["top_k"], draft_len=d, max_occ=4096,
               node_budget=cfg["node_budget"], n_pad=n_pad)
